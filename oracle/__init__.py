@@ -1,0 +1,202 @@
+"""CPU oracle for the MOBO candidate-scoring step (test infrastructure only).
+
+A plain fp64 C implementation (``boute_oracle.c``) of what the scoring step
+computes, written from the paper (Sec. 4.3 problem, Sec. 5.2 MOBO workflow and
+constrained qNEHVI, Sec. 6 kernels and outcome transforms), plus this ctypes
+wrapper. Only the test suite, ``__graft_entry__.smoke()`` and ``bench.py``'s
+CPU-baseline leg may import it; the CUDA library never does, and the two share
+no code.
+
+Parity pins live in ``tests/test_oracle_pins.py``. Functions without an
+independent pin: none.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "boute_oracle.c")
+_LIB = os.path.join(_HERE, "_build", "liboracle.so")
+_lib = None
+
+_dp = ctypes.POINTER(ctypes.c_double)
+_fp = ctypes.POINTER(ctypes.c_float)
+_ip = ctypes.POINTER(ctypes.c_int)
+_lp = ctypes.POINTER(ctypes.c_longlong)
+_bp = ctypes.POINTER(ctypes.c_ubyte)
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (plain C11, OpenMP over candidates)."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < max(
+            os.path.getmtime(_SRC), os.path.getmtime(os.path.join(_HERE, "boute_oracle.h"))):
+        os.makedirs(os.path.dirname(_LIB), exist_ok=True)
+        tmp = _LIB + f".{os.getpid()}.tmp"
+        subprocess.check_call(["gcc", "-std=c11", "-O2", "-fopenmp", "-fPIC", "-shared",
+                               "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        L = ctypes.CDLL(build())
+        L.bo_standardize.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp]
+        L.bo_matern52.argtypes = [_dp, _dp, ctypes.c_int, _dp, ctypes.c_double]
+        L.bo_matern52.restype = ctypes.c_double
+        L.bo_gp_fit.argtypes = [_dp, _dp, ctypes.c_int, ctypes.c_int, _dp, ctypes.c_double,
+                                ctypes.c_double, _dp, _dp]
+        L.bo_gp_posterior.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp, ctypes.c_double,
+                                      _dp, _dp, _fp, ctypes.c_longlong, _dp, _dp, ctypes.c_int]
+        L.bo_gp_posterior.restype = None
+        L.bo_pareto_front.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp, _bp, _ip]
+        L.bo_hv.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp, _dp]
+        L.bo_hv.restype = ctypes.c_double
+        L.bo_hvi.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp, _dp]
+        L.bo_hvi.restype = ctypes.c_double
+        L.bo_ehvi2d.argtypes = [_dp, _dp, ctypes.c_longlong, _dp, ctypes.c_int, _dp, _dp,
+                                ctypes.c_int]
+        L.bo_ehvi2d.restype = None
+        L.bo_mc_hvi.argtypes = [_dp, _dp, ctypes.c_longlong, ctypes.c_int, _fp, ctypes.c_int,
+                                ctypes.c_longlong, _dp, ctypes.c_int, _dp, _dp, ctypes.c_int]
+        L.bo_mc_hvi.restype = None
+        L.bo_topk.argtypes = [_dp, ctypes.c_longlong, ctypes.c_int, _lp, _dp]
+        L.bo_topk.restype = None
+        L.bo_default_threads.restype = ctypes.c_int
+        _lib = L
+    return _lib
+
+
+def _d(a):
+    a = np.ascontiguousarray(a, dtype=np.float64)
+    return a, a.ctypes.data_as(_dp)
+
+
+def _f(a):
+    a = np.ascontiguousarray(a, dtype=np.float32)
+    return a, a.ctypes.data_as(_fp)
+
+
+class NotPositiveDefinite(ArithmeticError):
+    pass
+
+
+def default_threads() -> int:
+    return int(lib().bo_default_threads())
+
+
+def standardize(Y):
+    Y, pY = _d(Y)
+    n, m = Y.shape
+    out = np.empty_like(Y)
+    rc = lib().bo_standardize(pY, n, m, out.ctypes.data_as(_dp))
+    if rc:
+        raise ValueError(rc)
+    return out
+
+
+def matern52(a, b, ls, s2=1.0) -> float:
+    a, pa = _d(a)
+    b, pb = _d(b)
+    ls, pl = _d(ls)
+    return float(lib().bo_matern52(pa, pb, a.size, pl, s2))
+
+
+def gp_fit(X, y, ls, s2, noise):
+    """Returns (L, alpha); raises NotPositiveDefinite on a failed pivot."""
+    X, pX = _d(X)
+    y, py = _d(y)
+    ls, pl = _d(ls)
+    n, d = X.shape
+    L = np.empty((n, n))
+    alpha = np.empty(n)
+    rc = lib().bo_gp_fit(pX, py, n, d, pl, float(s2), float(noise), L.ctypes.data_as(_dp),
+                         alpha.ctypes.data_as(_dp))
+    if rc == 2:
+        raise NotPositiveDefinite("kernel matrix not positive definite")
+    if rc:
+        raise ValueError(rc)
+    return L, alpha
+
+
+def gp_posterior(X, ls, s2, L, alpha, Xc, threads: int = 0):
+    """Posterior mean and variance (fp64) at fp32 candidates Xc (N x d)."""
+    X, pX = _d(X)
+    ls, pl = _d(ls)
+    L, pL = _d(L)
+    alpha, pa = _d(alpha)
+    Xc, pc = _f(Xc)
+    n, d = X.shape
+    N = Xc.shape[0]
+    mean = np.empty(N)
+    var = np.empty(N)
+    lib().bo_gp_posterior(pX, n, d, pl, float(s2), pL, pa, pc, N, mean.ctypes.data_as(_dp),
+                          var.ctypes.data_as(_dp), threads)
+    return mean, var
+
+
+def pareto_front(Y, ref):
+    """Returns (mask (n,) bool, order (P,) int: kept indices sorted lexicographically)."""
+    Y, pY = _d(Y)
+    ref, pr = _d(ref)
+    n, m = Y.shape
+    mask = np.zeros(n, np.uint8)
+    order = np.zeros(max(n, 1), np.int32)
+    P = lib().bo_pareto_front(pY, n, m, pr, mask.ctypes.data_as(_bp), order.ctypes.data_as(_ip))
+    return mask.astype(bool), order[:P].astype(np.int64)
+
+
+def hv(F, ref) -> float:
+    F, pF = _d(np.asarray(F, dtype=np.float64).reshape(-1, len(ref)))
+    ref, pr = _d(ref)
+    return float(lib().bo_hv(pF, F.shape[0], F.shape[1], pr, None))
+
+
+def hvi(F, ref, y) -> float:
+    F, pF = _d(np.asarray(F, dtype=np.float64).reshape(-1, len(ref)))
+    ref, pr = _d(ref)
+    y, py = _d(y)
+    return float(lib().bo_hvi(pF, F.shape[0], F.shape[1], pr, py))
+
+
+def ehvi2d(mean, var, F, ref, threads: int = 0):
+    """mean, var: N x 2; F: P x 2 sorted by f1 ascending."""
+    mean, pm = _d(mean)
+    var, pv = _d(var)
+    F, pF = _d(np.asarray(F, dtype=np.float64).reshape(-1, 2))
+    ref, pr = _d(ref)
+    N = mean.shape[0]
+    acq = np.empty(N)
+    lib().bo_ehvi2d(pm, pv, N, pF, F.shape[0], pr, acq.ctypes.data_as(_dp), threads)
+    return acq
+
+
+def mc_hvi(mean, var, eps, F, ref, eps_stride: int | None = None, threads: int = 0):
+    """mean, var: N x m; eps: float32 (N, m, S) (or (1, m, S) with eps_stride=0)."""
+    mean, pm = _d(mean)
+    var, pv = _d(var)
+    eps, pe = _f(eps)
+    m = mean.shape[1]
+    S = eps.shape[-1]
+    stride = m * S if eps_stride is None else eps_stride
+    F, pF = _d(np.asarray(F, dtype=np.float64).reshape(-1, m))
+    ref, pr = _d(ref)
+    N = mean.shape[0]
+    acq = np.empty(N)
+    lib().bo_mc_hvi(pm, pv, N, m, pe, S, stride, pF, F.shape[0], pr, acq.ctypes.data_as(_dp),
+                    threads)
+    return acq
+
+
+def topk(acq, k: int):
+    acq, pa = _d(acq)
+    k = min(k, acq.size)
+    idx = np.empty(k, np.int64)
+    val = np.empty(k)
+    lib().bo_topk(pa, acq.size, k, idx.ctypes.data_as(_lp), val.ctypes.data_as(_dp))
+    return idx, val

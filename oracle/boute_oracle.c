@@ -1,0 +1,337 @@
+/*
+ * CPU oracle for the MOBO candidate-scoring step of BOute (arXiv 2602.10729).
+ * TEST INFRASTRUCTURE ONLY: see boute_oracle.h. Plain fp64 C, no BLAS, no
+ * blocking or reordering beyond the textbook definitions cited per function.
+ */
+#include "boute_oracle.h"
+
+#define _GNU_SOURCE
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+int bo_default_threads(void) {
+#ifdef _OPENMP
+  return omp_get_max_threads();
+#else
+  return 1;
+#endif
+}
+
+static int nthreads_or_default(int nthreads) {
+  return nthreads > 0 ? nthreads : bo_default_threads();
+}
+
+/* ---- Sec. 6: Standardize outcome transform ------------------------------ */
+int bo_standardize(const double *Y, int n, int m, double *Ys) {
+  if (n < 0 || m < 1 || (n > 0 && (!Y || !Ys))) return 1;
+  for (int t = 0; t < m; ++t) {
+    double mean = 0.0;
+    for (int i = 0; i < n; ++i) mean += Y[(long)i * m + t];
+    mean = n > 0 ? mean / n : 0.0;
+    double ss = 0.0;
+    for (int i = 0; i < n; ++i) {
+      double z = Y[(long)i * m + t] - mean;
+      ss += z * z;
+    }
+    double sd = n > 1 ? sqrt(ss / (n - 1)) : 1.0;
+    if (!(sd >= 1e-8)) sd = 1.0;
+    for (int i = 0; i < n; ++i) Ys[(long)i * m + t] = (Y[(long)i * m + t] - mean) / sd;
+  }
+  return 0;
+}
+
+/* ---- Sec. 6 (i): ARD Matern-5/2 with ScaleKernel ------------------------ */
+double bo_matern52(const double *a, const double *b, int d, const double *ls, double s2) {
+  double r2 = 0.0;
+  for (int t = 0; t < d; ++t) {
+    double z = (a[t] - b[t]) / ls[t];
+    r2 += z * z;
+  }
+  double r = sqrt(r2);
+  double sr = sqrt(5.0) * r;
+  return s2 * (1.0 + sr + 5.0 * r2 / 3.0) * exp(-sr);
+}
+
+/* ---- Sec. 5.2 (i) / Sec. 6: exact GP fit --------------------------------- */
+int bo_gp_fit(const double *X, const double *y, int n, int d, const double *ls,
+              double s2, double noise, double *L, double *alpha) {
+  if (n < 1 || d < 1 || !X || !y || !ls || !L || !alpha) return 1;
+  /* K = s2 M52(X, X) + noise I, lower triangle written straight into L */
+  for (int i = 0; i < n; ++i)
+    for (int j = 0; j < n; ++j)
+      L[(long)i * n + j] = j <= i ? bo_matern52(X + (long)i * d, X + (long)j * d, d, ls, s2) +
+                                        (i == j ? noise : 0.0)
+                                  : 0.0;
+  /* Cholesky-Banachiewicz, row by row, in place */
+  for (int i = 0; i < n; ++i) {
+    for (int j = 0; j <= i; ++j) {
+      double s = L[(long)i * n + j];
+      for (int k = 0; k < j; ++k) s -= L[(long)i * n + k] * L[(long)j * n + k];
+      if (i == j) {
+        if (!(s > 0.0)) return 2;
+        L[(long)i * n + i] = sqrt(s);
+      } else {
+        L[(long)i * n + j] = s / L[(long)j * n + j];
+      }
+    }
+  }
+  /* alpha = L^-T (L^-1 y) */
+  for (int i = 0; i < n; ++i) {
+    double s = y[i];
+    for (int k = 0; k < i; ++k) s -= L[(long)i * n + k] * alpha[k];
+    alpha[i] = s / L[(long)i * n + i];
+  }
+  for (int i = n - 1; i >= 0; --i) {
+    double s = alpha[i];
+    for (int k = i + 1; k < n; ++k) s -= L[(long)k * n + i] * alpha[k];
+    alpha[i] = s / L[(long)i * n + i];
+  }
+  return 0;
+}
+
+void bo_gp_posterior(const double *X, int n, int d, const double *ls, double s2,
+                     const double *L, const double *alpha, const float *Xc,
+                     long long N, double *mean, double *var, int nthreads) {
+  int nt = nthreads_or_default(nthreads);
+#pragma omp parallel num_threads(nt)
+  {
+    double *kv = (double *)malloc(sizeof(double) * (size_t)(2 * n + d));
+    double *v = kv + n, *xc = kv + 2 * n;
+#pragma omp for schedule(static)
+    for (long long c = 0; c < N; ++c) {
+      for (int t = 0; t < d; ++t) xc[t] = (double)Xc[c * d + t];
+      double mu = 0.0;
+      for (int j = 0; j < n; ++j) {
+        kv[j] = bo_matern52(xc, X + (long)j * d, d, ls, s2);
+        mu += kv[j] * alpha[j];
+      }
+      double vv = 0.0;
+      for (int i = 0; i < n; ++i) { /* v = L^-1 k* */
+        double s = kv[i];
+        for (int j = 0; j < i; ++j) s -= L[(long)i * n + j] * v[j];
+        v[i] = s / L[(long)i * n + i];
+        vv += v[i] * v[i];
+      }
+      double s2v = s2 - vv;
+      mean[c] = mu;
+      var[c] = s2v > 0.0 ? s2v : 0.0;
+    }
+    free(kv);
+  }
+}
+
+/* ---- Sec. 5.2: Pareto-optimal set (minimisation) ------------------------- */
+static _Thread_local const double *g_sortY;
+static _Thread_local int g_sortM;
+static int cmp_lex(const void *pa, const void *pb) {
+  int a = *(const int *)pa, b = *(const int *)pb;
+  for (int t = 0; t < g_sortM; ++t) {
+    double ya = g_sortY[(long)a * g_sortM + t], yb = g_sortY[(long)b * g_sortM + t];
+    if (ya < yb) return -1;
+    if (ya > yb) return 1;
+  }
+  return (a > b) - (a < b);
+}
+
+int bo_pareto_front(const double *Y, int n, int m, const double *ref,
+                    unsigned char *mask, int *order) {
+  if (n < 0 || m < 1) return -1;
+  int P = 0;
+  for (int i = 0; i < n; ++i) {
+    const double *yi = Y + (long)i * m;
+    int keep = 1;
+    for (int t = 0; t < m; ++t)
+      if (!(yi[t] < ref[t])) keep = 0;
+    for (int j = 0; j < n && keep; ++j) {
+      if (j == i) continue;
+      const double *yj = Y + (long)j * m;
+      int all_le = 1, any_lt = 0, all_eq = 1;
+      for (int t = 0; t < m; ++t) {
+        if (yj[t] > yi[t]) all_le = 0;
+        if (yj[t] < yi[t]) any_lt = 1;
+        if (yj[t] != yi[t]) all_eq = 0;
+      }
+      if (all_le && any_lt) keep = 0;      /* j dominates i */
+      if (all_eq && j < i) keep = 0;       /* duplicate: lowest index survives */
+    }
+    mask[i] = (unsigned char)keep;
+    if (keep) order[P++] = i;
+  }
+  g_sortY = Y;
+  g_sortM = m;
+  qsort(order, (size_t)P, sizeof(int), cmp_lex);
+  return P;
+}
+
+/* ---- Hypervolume by slicing ---------------------------------------------- */
+long long bo_hv_scratch_size(int P, int m) {
+  /* each recursion level copies at most P points of its dimension */
+  return (long long)(P + 1) * m * (m + 1) + 16;
+}
+
+static int cmp_dbl2(const void *pa, const void *pb) { /* (f1, f2) lexicographic */
+  const double *a = (const double *)pa, *b = (const double *)pb;
+  if (a[0] != b[0]) return a[0] < b[0] ? -1 : 1;
+  if (a[1] != b[1]) return a[1] < b[1] ? -1 : 1;
+  return 0;
+}
+
+static _Thread_local int g_lastdim;
+static int cmp_last(const void *pa, const void *pb) {
+  const double *a = (const double *)pa, *b = (const double *)pb;
+  double x = a[g_lastdim], y = b[g_lastdim];
+  return (x > y) - (x < y);
+}
+
+/* pts: Q x m points, all strictly better than ref; may be reordered. */
+static double hv_rec(double *pts, int Q, int m, const double *ref, double *scratch) {
+  if (Q == 0) return 0.0;
+  if (m == 1) {
+    double lo = ref[0];
+    for (int i = 0; i < Q; ++i)
+      if (pts[i] < lo) lo = pts[i];
+    return ref[0] - lo;
+  }
+  if (m == 2) { /* staircase sweep along f1 */
+    qsort(pts, (size_t)Q, 2 * sizeof(double), cmp_dbl2);
+    double hv = 0.0, cur = ref[1];
+    for (int i = 0; i < Q; ++i) {
+      if (pts[2 * i + 1] < cur) {
+        hv += (ref[0] - pts[2 * i]) * (cur - pts[2 * i + 1]);
+        cur = pts[2 * i + 1];
+      }
+    }
+    return hv;
+  }
+  /* slice along the last objective: between consecutive levels the
+   * cross-section is the (m-1)-D hypervolume of the points below the level */
+  g_lastdim = m - 1;
+  qsort(pts, (size_t)Q, (size_t)m * sizeof(double), cmp_last);
+  double *sub = scratch, *rest = scratch + (long)Q * (m - 1);
+  double hv = 0.0;
+  for (int j = 0; j < Q; ++j) {
+    double z0 = pts[(long)j * m + m - 1];
+    double z1 = j + 1 < Q ? pts[(long)(j + 1) * m + m - 1] : ref[m - 1];
+    if (z1 <= z0) continue;
+    for (int i = 0; i <= j; ++i)
+      memcpy(sub + (long)i * (m - 1), pts + (long)i * m, sizeof(double) * (m - 1));
+    double a = hv_rec(sub, j + 1, m - 1, ref, rest);
+    g_lastdim = m - 1; /* restore after recursion (the comparator is not reentrant) */
+    hv += (z1 - z0) * a;
+  }
+  return hv;
+}
+
+double bo_hv(const double *F, int P, int m, const double *ref, double *scratch) {
+  double *own = NULL;
+  if (!scratch) {
+    own = (double *)malloc(sizeof(double) * (size_t)bo_hv_scratch_size(P, m));
+    scratch = own;
+  }
+  double *pts = scratch;
+  int Q = 0;
+  for (int i = 0; i < P; ++i) {
+    int in = 1;
+    for (int t = 0; t < m; ++t)
+      if (!(F[(long)i * m + t] < ref[t])) in = 0;
+    if (in) memcpy(pts + (long)(Q++) * m, F + (long)i * m, sizeof(double) * m);
+  }
+  double hv = hv_rec(pts, Q, m, ref, pts + (long)(P + 1) * m);
+  free(own);
+  return hv;
+}
+
+double bo_hvi(const double *F, int P, int m, const double *ref, const double *y) {
+  double *all = (double *)malloc(sizeof(double) * (size_t)(P + 1) * m);
+  memcpy(all, F, sizeof(double) * (size_t)P * m);
+  memcpy(all + (long)P * m, y, sizeof(double) * m);
+  double v = bo_hv(all, P + 1, m, ref, NULL) - bo_hv(F, P, m, ref, NULL);
+  free(all);
+  return v;
+}
+
+/* ---- closed-form 2-D EHVI ------------------------------------------------ */
+static double std_cdf(double z) { return 0.5 * erfc(-z / sqrt(2.0)); }
+static double std_pdf(double z) { return exp(-0.5 * z * z) / sqrt(2.0 * 3.14159265358979323846); }
+
+/* psi(c) = E[(c - Y)_+], Y ~ N(mu, sigma^2); psi(-inf) = 0 */
+static double psi(double c, double mu, double sigma) {
+  if (isinf(c) && c < 0) return 0.0;
+  if (!(sigma > 0.0)) return c > mu ? c - mu : 0.0;
+  double z = (c - mu) / sigma;
+  return (c - mu) * std_cdf(z) + sigma * std_pdf(z);
+}
+
+void bo_ehvi2d(const double *mean, const double *var, long long N, const double *F,
+               int P, const double *ref, double *acq, int nthreads) {
+  int nt = nthreads_or_default(nthreads);
+#pragma omp parallel for schedule(static) num_threads(nt)
+  for (long long c = 0; c < N; ++c) {
+    double mu1 = mean[2 * c], mu2 = mean[2 * c + 1];
+    double sg1 = sqrt(var[2 * c]), sg2 = sqrt(var[2 * c + 1]);
+    double e = 0.0;
+    for (int i = 0; i <= P; ++i) {
+      /* cell i: f1 in [a_i, b_i), f2 below u_i */
+      double a = i == 0 ? -INFINITY : F[2 * (i - 1)];
+      double b = i == P ? ref[0] : F[2 * i];
+      double u = i == 0 ? ref[1] : F[2 * (i - 1) + 1];
+      e += (psi(b, mu1, sg1) - psi(a, mu1, sg1)) * psi(u, mu2, sg2);
+    }
+    acq[c] = e;
+  }
+}
+
+/* ---- Monte-Carlo HVI ------------------------------------------------------ */
+void bo_mc_hvi(const double *mean, const double *var, long long N, int m,
+               const float *eps, int S, long long eps_stride, const double *F,
+               int P, const double *ref, double *acq, int nthreads) {
+  int nt = nthreads_or_default(nthreads);
+  double hvF = bo_hv(F, P, m, ref, NULL);
+  long long scr = bo_hv_scratch_size(P + 1, m);
+#pragma omp parallel num_threads(nt)
+  {
+    double *all = (double *)malloc(sizeof(double) * (size_t)((P + 1) * m + m + scr));
+    double *sg = all + (long)(P + 1) * m, *scratch = sg + m;
+    memcpy(all, F, sizeof(double) * (size_t)P * m);
+#pragma omp for schedule(dynamic, 64)
+    for (long long c = 0; c < N; ++c) {
+      for (int t = 0; t < m; ++t) sg[t] = sqrt(var[c * m + t]);
+      double sum = 0.0;
+      for (int s = 0; s < S; ++s) {
+        for (int t = 0; t < m; ++t)
+          all[(long)P * m + t] =
+              mean[c * m + t] + sg[t] * (double)eps[c * eps_stride + (long long)t * S + s];
+        sum += bo_hv(all, P + 1, m, ref, scratch) - hvF;
+      }
+      acq[c] = sum / S;
+    }
+    free(all);
+  }
+}
+
+/* ---- top-k ----------------------------------------------------------------- */
+static _Thread_local const double *g_topv;
+static int cmp_top(const void *pa, const void *pb) {
+  long long a = *(const long long *)pa, b = *(const long long *)pb;
+  double va = g_topv[a], vb = g_topv[b];
+  if (isnan(va)) va = -INFINITY;
+  if (isnan(vb)) vb = -INFINITY;
+  if (va != vb) return va > vb ? -1 : 1;
+  return (a > b) - (a < b);
+}
+
+void bo_topk(const double *acq, long long N, int k, long long *idx, double *val) {
+  long long *ord = (long long *)malloc(sizeof(long long) * (size_t)(N > 0 ? N : 1));
+  for (long long i = 0; i < N; ++i) ord[i] = i;
+  g_topv = acq;
+  qsort(ord, (size_t)N, sizeof(long long), cmp_top);
+  for (int i = 0; i < k && i < N; ++i) {
+    idx[i] = ord[i];
+    val[i] = acq[ord[i]];
+  }
+  free(ord);
+}

@@ -1,0 +1,93 @@
+/*
+ * CPU oracle for the MOBO candidate-scoring step of BOute (arXiv 2602.10729).
+ *
+ * TEST INFRASTRUCTURE ONLY. This is a plain, slow, obviously correct fp64
+ * restatement of what the scoring step computes, written from the paper, used
+ * to check the CUDA library. Only the test suite, the package smoke check and
+ * the benchmark's CPU-baseline leg may load it; the product path never does.
+ * It shares no code, header, table or helper with the CUDA library.
+ *
+ * Conventions: all matrices are row-major, contiguous; doubles unless noted.
+ * Every objective is minimised (Sec. 4.3, problem formulation).
+ * Return codes: 0 ok, 1 invalid argument, 2 matrix not positive definite.
+ */
+#ifndef BOUTE_ORACLE_H
+#define BOUTE_ORACLE_H
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Outcome standardisation (Sec. 6, "Standardize" outcome transform):
+ * Ys[:,t] = (Y[:,t] - mean_t) / std_t, std with the n-1 denominator; a column
+ * with n < 2 or std < 1e-8 is divided by 1. Y, Ys: n x m. */
+int bo_standardize(const double *Y, int n, int m, double *Ys);
+
+/* ARD Matern-5/2 kernel with outputscale (Sec. 6 (i): MaternKernel nu=2.5
+ * wrapped in ScaleKernel): s2 (1 + sqrt5 r + 5 r^2/3) exp(-sqrt5 r),
+ * r^2 = sum_t ((a_t - b_t) / ls_t)^2. */
+double bo_matern52(const double *a, const double *b, int d, const double *ls, double s2);
+
+/* Exact GP fit with fixed hyperparameters (Sec. 5.2 step (i); Sec. 6
+ * SingleTaskGP, zero prior mean on standardised outcomes):
+ * K = s2 M52(X, X) + noise I, L = chol(K) (Cholesky-Banachiewicz, no jitter),
+ * alpha = K^-1 y by forward then back substitution.
+ * X: n x d; y: n; ls: d; L: n x n (upper triangle set to 0); alpha: n.
+ * Returns 2 when a pivot is not positive. */
+int bo_gp_fit(const double *X, const double *y, int n, int d, const double *ls,
+              double s2, double noise, double *L, double *alpha);
+
+/* Latent-function posterior at fp32 candidates (cast to double):
+ * mean = k*^T alpha, var = max(0, s2 - v^T v) with v = L^-1 k* by forward
+ * substitution. Xc: N x d float; mean, var: N. nthreads <= 0: library default. */
+void bo_gp_posterior(const double *X, int n, int d, const double *ls, double s2,
+                     const double *L, const double *alpha, const float *Xc,
+                     long long N, double *mean, double *var, int nthreads);
+
+/* Pareto front of observed outcomes (Sec. 5.2, Pareto-optimal set; all
+ * objectives minimised): point i is kept iff no j dominates it (Y_j <= Y_i in
+ * every objective, < in one), no exact duplicate j < i exists, and
+ * Y_i,t < ref_t for every t. mask: n bytes (1 = kept). order: the kept indices
+ * sorted by f1, then f2, ..., then index. Returns P = number kept. */
+int bo_pareto_front(const double *Y, int n, int m, const double *ref,
+                    unsigned char *mask, int *order);
+
+/* Hypervolume dominated by the points F (P x m) and bounded by ref, by
+ * recursive slicing along the last objective with a 2-D staircase sweep at
+ * the bottom. Points not strictly better than ref in every objective add
+ * nothing. scratch: at least bo_hv_scratch_size(P, m) doubles, or NULL. */
+double bo_hv(const double *F, int P, int m, const double *ref, double *scratch);
+long long bo_hv_scratch_size(int P, int m);
+
+/* Hypervolume improvement of y over F: HV(F u {y}) - HV(F). */
+double bo_hvi(const double *F, int P, int m, const double *ref, const double *y);
+
+/* Closed-form expected hypervolume improvement for two independent Gaussian
+ * objectives (the expectation of HVI in Sec. 5.2 "Constrained qNEHVI", taken
+ * in closed form over the P+1 cells of the sorted 2-D front):
+ * EHVI = sum_i [psi1(b_i) - psi1(a_i)] psi2(u_i),
+ * psi(c) = E[(c - Y)_+] = (c - mu) Phi(z) + sigma phi(z), z = (c - mu)/sigma.
+ * mean, var: N x 2; F: P x 2 sorted by f1 ascending; acq: N. */
+void bo_ehvi2d(const double *mean, const double *var, long long N, const double *F,
+               int P, const double *ref, double *acq, int nthreads);
+
+/* Monte-Carlo hypervolume improvement (Sec. 5.2: expectation of HVI over
+ * posterior samples, by Monte-Carlo integration): sample s of candidate c is
+ * y_t = mean_t + sqrt(var_t) eps[c*eps_stride + t*S + s]; acq = mean over the
+ * S samples of HV(F u {y}) - HV(F). mean, var: N x m; eps: float. */
+void bo_mc_hvi(const double *mean, const double *var, long long N, int m,
+               const float *eps, int S, long long eps_stride, const double *F,
+               int P, const double *ref, double *acq, int nthreads);
+
+/* Top-k selection (Sec. 5.2 step (ii): the next configuration is the best
+ * scored candidate): the first k entries of the order (value descending, NaN
+ * as -infinity, equal values by ascending index). idx, val: k. */
+void bo_topk(const double *acq, long long N, int k, long long *idx, double *val);
+
+/* Number of OpenMP threads a call with nthreads <= 0 uses. */
+int bo_default_threads(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -1,0 +1,69 @@
+"""The scoring step composed from oracle functions (test infrastructure only).
+
+Follows the order of one MOBO iteration (Sec. 5.2, "Overall MOBO workflow"):
+standardise the observed outcomes, fit one exact GP per objective
+(independent GPs combined as a model list, Sec. 6), take the Pareto front of
+the observed outcomes, evaluate the posterior and the acquisition at every
+candidate, and select the best k.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import numpy as np
+
+from . import (ehvi2d, gp_fit, gp_posterior, mc_hvi, pareto_front, standardize, topk)
+
+
+@dataclass
+class FittedProblem:
+    X: np.ndarray  # n x d observed points
+    Ys: np.ndarray  # n x m standardised outcomes
+    ls: np.ndarray  # m x d
+    s2: np.ndarray  # m
+    noise: np.ndarray  # m
+    L: list  # per objective, n x n
+    alpha: list  # per objective, n
+    ref: np.ndarray
+    mask: np.ndarray  # front membership (n,)
+    front: np.ndarray  # P x m, sorted
+
+
+def fit_problem(X, Y, ls, s2, noise, ref) -> FittedProblem:
+    Ys = standardize(Y)
+    Ls, alphas = [], []
+    for t in range(Ys.shape[1]):
+        L, a = gp_fit(X, Ys[:, t], ls[t], s2[t], noise[t])
+        Ls.append(L)
+        alphas.append(a)
+    mask, order = pareto_front(Ys, ref)
+    return FittedProblem(np.asarray(X, np.float64), Ys, np.asarray(ls, np.float64),
+                         np.asarray(s2, np.float64), np.asarray(noise, np.float64), Ls, alphas,
+                         np.asarray(ref, np.float64), mask, Ys[order])
+
+
+def posterior(fp: FittedProblem, Xc, threads: int = 0):
+    """mean, var: N x m (fp64)."""
+    Xc = np.ascontiguousarray(Xc, np.float32)
+    m = fp.Ys.shape[1]
+    mean = np.empty((Xc.shape[0], m))
+    var = np.empty((Xc.shape[0], m))
+    for t in range(m):
+        mean[:, t], var[:, t] = gp_posterior(fp.X, fp.ls[t], fp.s2[t], fp.L[t], fp.alpha[t], Xc,
+                                             threads)
+    return mean, var
+
+
+def acquisition(fp: FittedProblem, mean, var, mode: str, eps=None, threads: int = 0):
+    if mode == "ehvi":
+        return ehvi2d(mean, var, fp.front, fp.ref, threads)
+    if mode == "mc":
+        return mc_hvi(mean, var, eps, fp.front, fp.ref, threads=threads)
+    raise ValueError(mode)
+
+
+def score(fp: FittedProblem, Xc, mode: str, k: int, eps=None, threads: int = 0):
+    mean, var = posterior(fp, Xc, threads)
+    acq = acquisition(fp, mean, var, mode, eps, threads)
+    idx, val = topk(acq, k)
+    return mean, var, acq, idx, val

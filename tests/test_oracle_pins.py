@@ -1,0 +1,418 @@
+"""Pins of the CPU oracle against facts that do not come from the oracle itself:
+closed forms, a different special-function route to the same kernel, library
+linear algebra on the same definitions, brute-force enumeration, quadrature,
+invariants and hand-derived worked examples (tests/golden/). A plausible
+mistake anywhere in the oracle (dropped term, wrong sign or index, transposed
+operand) fails at least one of these."""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import scipy.integrate
+import scipy.linalg
+import scipy.special
+
+import oracle
+from oracle import pipeline
+from paper_2602_10729_gb300 import workloads as wl
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden", "hypervolume_cases.json")
+
+
+# --------------------------------------------------------------- Matern 5/2
+def _matern_bessel(r, nu, s2):
+    """General Matern covariance through the modified Bessel function K_nu."""
+    if r == 0:
+        return s2
+    z = math.sqrt(2 * nu) * r
+    return s2 * 2 ** (1 - nu) / scipy.special.gamma(nu) * z ** nu * scipy.special.kv(nu, z)
+
+
+@pytest.mark.parametrize("r", [0.0, 1e-3, 0.1, 0.5, 1.0, 2.0, 3.7, 8.0])
+def test_matern52_equals_general_matern_at_nu_2p5(r):
+    ls = np.array([0.3, 1.7, 0.9])
+    u = np.array([0.2, -0.5, 0.4])
+    u = u / np.linalg.norm(u / ls) * r if r > 0 else np.zeros(3)  # scaled distance r
+    a = np.array([0.1, 0.2, 0.3])
+    got = oracle.matern52(a, a + u, ls, 1.7)
+    assert got == pytest.approx(_matern_bessel(r, 2.5, 1.7), rel=1e-12, abs=1e-300)
+
+
+def test_matern52_symmetry_and_ard():
+    rng = np.random.default_rng(3)
+    a, b = rng.random(5), rng.random(5)
+    ls = rng.random(5) + 0.2
+    assert oracle.matern52(a, b, ls) == oracle.matern52(b, a, ls)
+    # a lengthscale of infinity removes that dimension from the distance
+    ls2 = ls.copy(); ls2[2] = np.inf
+    b2 = b.copy(); b2[2] = a[2]
+    assert oracle.matern52(a, b, ls2) == pytest.approx(oracle.matern52(a, b2, ls), rel=1e-15)
+
+
+# ------------------------------------------------------------ standardise
+def test_standardize_moments_and_affine_invariance():
+    rng = np.random.default_rng(0)
+    Y = rng.normal(3.0, 2.0, (50, 3))
+    Ys = oracle.standardize(Y)
+    np.testing.assert_allclose(Ys.mean(0), 0, atol=1e-14)
+    np.testing.assert_allclose(Ys.std(0, ddof=1), 1, rtol=1e-13)
+    np.testing.assert_allclose(oracle.standardize(4.0 * Y - 7.0), Ys, atol=1e-13)
+    # constant column / single row: divided by one
+    Yc = np.ones((4, 1)) * 5.0
+    np.testing.assert_allclose(oracle.standardize(Yc), 0.0)
+    np.testing.assert_allclose(oracle.standardize(np.array([[2.0, 3.0]])), 0.0)
+
+
+# --------------------------------------------------------------- GP fit
+def _kernel_matrix(X, ls, s2, noise):
+    n = len(X)
+    K = np.array([[oracle.matern52(X[i], X[j], ls, s2) for j in range(n)] for i in range(n)])
+    return K + noise * np.eye(n)
+
+
+@pytest.mark.parametrize("wi", [0, 1, 4])
+def test_cholesky_residual_and_library_factor(wi):
+    w = wl.WORKLOADS[wi]
+    X, Y = wl.training_set(w, 0)
+    ls, s2, noise = wl.hyperparameters(w, 0)
+    y = oracle.standardize(Y)[:, 0]
+    L, alpha = oracle.gp_fit(X, y, ls[0], s2[0], noise[0])
+    K = _kernel_matrix(X, ls[0], s2[0], noise[0])
+    assert np.linalg.norm(L @ L.T - K) / np.linalg.norm(K) < 1e-12
+    assert np.all(np.triu(L, 1) == 0) and np.all(np.diag(L) > 0)
+    np.testing.assert_allclose(L, scipy.linalg.cholesky(K, lower=True), atol=1e-12)
+    np.testing.assert_allclose(alpha, np.linalg.solve(K, y), rtol=1e-9, atol=1e-10)
+
+
+def test_cholesky_tiny_matches_gauss_jordan_solve():
+    X = np.array([[0.0, 0.0], [0.3, 0.1], [0.9, 0.5]])
+    ls = np.array([0.5, 0.7])
+    y = np.array([1.0, -2.0, 0.5])
+    L, alpha = oracle.gp_fit(X, y, ls, 2.0, 0.01)
+    K = _kernel_matrix(X, ls, 2.0, 0.01)
+    # Gauss-Jordan elimination on [K | y], written out
+    A = np.hstack([K, y[:, None]])
+    for c in range(3):
+        A[c] /= A[c, c]
+        for r in range(3):
+            if r != c:
+                A[r] -= A[r, c] * A[c]
+    np.testing.assert_allclose(alpha, A[:, 3], rtol=1e-12)
+
+
+def test_not_positive_definite_is_reported():
+    X = np.array([[0.1, 0.2], [0.1, 0.2], [0.5, 0.5]])  # duplicate rows, no noise
+    with pytest.raises(oracle.NotPositiveDefinite):
+        oracle.gp_fit(X, np.zeros(3), np.ones(2), 1.0, 0.0)
+
+
+# ------------------------------------------------------------ posterior
+def _fit(X, y, ls, s2, noise):
+    L, a = oracle.gp_fit(X, y, ls, s2, noise)
+    return L, a
+
+
+def test_posterior_matches_schur_complement_by_library_solve():
+    w = wl.WORKLOADS[0]
+    X, Y = wl.training_set(w, 0)
+    ls, s2, noise = wl.hyperparameters(w, 0)
+    y = oracle.standardize(Y)[:, 1]
+    L, a = _fit(X, y, ls[1], s2[1], noise[1])
+    Xc = wl.candidates(w, 0, 0, 64)
+    mean, var = oracle.gp_posterior(X, ls[1], s2[1], L, a, Xc)
+    K = _kernel_matrix(X, ls[1], s2[1], noise[1])
+    Ks = np.array([[oracle.matern52(c.astype(np.float64), x, ls[1], s2[1]) for x in X] for c in Xc])
+    np.testing.assert_allclose(mean, Ks @ np.linalg.solve(K, y), rtol=1e-9, atol=1e-11)
+    sol = np.linalg.solve(K, Ks.T)
+    np.testing.assert_allclose(var, s2[1] - np.einsum("ij,ji->i", Ks, sol), rtol=1e-8, atol=1e-11)
+
+
+def test_posterior_interpolates_as_noise_vanishes():
+    rng = np.random.default_rng(5)
+    X = rng.random((20, 3)).astype(np.float32).astype(np.float64)  # exactly representable
+    y = rng.normal(size=20)
+    ls = np.full(3, 0.15)
+    L, a = _fit(X, y, ls, 1.0, 1e-10)
+    mean, var = oracle.gp_posterior(X, ls, 1.0, L, a, X.astype(np.float32))
+    np.testing.assert_allclose(mean, y, atol=1e-6)
+    assert np.all(var >= 0) and np.all(var < 1e-7)
+
+
+def test_posterior_bounds_and_far_field():
+    w = wl.WORKLOADS[1]
+    X, Y = wl.training_set(w, 0)
+    ls, s2, noise = wl.hyperparameters(w, 0)
+    y = oracle.standardize(Y)[:, 0]
+    L, a = _fit(X, y, ls[0], s2[0], noise[0])
+    Xc = wl.candidates(w, 0, 0, 500)
+    mean, var = oracle.gp_posterior(X, ls[0], s2[0], L, a, Xc)
+    assert np.all(var >= 0) and np.all(var <= s2[0])
+    far = (Xc[:5] + 1000.0).astype(np.float32)
+    mf, vf = oracle.gp_posterior(X, ls[0], s2[0], L, a, far)
+    np.testing.assert_allclose(mf, 0.0, atol=1e-300)
+    np.testing.assert_allclose(vf, s2[0], rtol=1e-15)
+
+
+def test_posterior_single_point_closed_form():
+    X = np.array([[0.25, 0.5]])
+    ls = np.array([0.4, 0.9])
+    s2, noise, y = 1.3, 0.2, np.array([0.7])
+    L, a = _fit(X, y, ls, s2, noise)
+    c = np.array([[0.5, 0.125]], np.float32)
+    k = _matern_bessel(np.linalg.norm((c[0].astype(np.float64) - X[0]) / ls), 2.5, s2)
+    mean, var = oracle.gp_posterior(X, ls, s2, L, a, c)
+    assert mean[0] == pytest.approx(k * y[0] / (s2 + noise), rel=1e-12)
+    assert var[0] == pytest.approx(s2 - k * k / (s2 + noise), rel=1e-12)
+
+
+# ------------------------------------------------------------ Pareto front
+def _front_bruteforce(Y, ref):
+    n = len(Y)
+    keep = np.all(Y < ref, 1)
+    for i in range(n):
+        le = np.all(Y <= Y[i], 1)
+        lt = np.any(Y < Y[i], 1)
+        eq = np.all(Y == Y[i], 1)
+        if np.any(le & lt) or np.any(eq[:i]):
+            keep[i] = False
+    return keep
+
+
+def test_pareto_hand_case():
+    Y = np.array([[1, 3], [2, 2], [3, 1], [2, 3], [1, 3], [0, 5], [5, 0]], float)
+    mask, order = oracle.pareto_front(Y, np.array([4.0, 4.0]))
+    # (2,3) is dominated by (2,2); index 4 duplicates index 0; (0,5), (5,0) lie beyond ref
+    assert mask.tolist() == [True, True, True, False, False, False, False]
+    assert order.tolist() == [0, 1, 2]
+
+
+@pytest.mark.parametrize("m", [2, 3])
+def test_pareto_invariants_and_bruteforce(m):
+    rng = np.random.default_rng(m)
+    Y = np.round(rng.normal(size=(300, m)), 1)  # rounding creates ties and duplicates
+    ref = np.full(m, 1.1)
+    mask, order = oracle.pareto_front(Y, ref)
+    assert mask.tolist() == _front_bruteforce(Y, ref).tolist()
+    F = Y[order]
+    assert sorted(order.tolist()) == np.flatnonzero(mask).tolist()
+    assert all(tuple(F[i]) < tuple(F[i + 1]) for i in range(len(F) - 1))  # strictly sorted
+    for i in np.flatnonzero(~mask):  # dropped: dominated/duplicated by a kept point, or beyond ref
+        if np.all(Y[i] < ref):
+            assert np.any(np.all(F <= Y[i], 1))
+
+
+# ------------------------------------------------------------ hypervolume
+def _hv_grid(F, ref):
+    """Count unit cells [z, z+1) inside the dominated region (integer data)."""
+    F = np.asarray(F, int).reshape(-1, len(ref))
+    lo = F.min(0) if len(F) else np.asarray(ref)
+    axes = [np.arange(lo[t], ref[t]) for t in range(len(ref))]
+    if any(len(a) == 0 for a in axes):
+        return 0
+    Z = np.stack(np.meshgrid(*axes, indexing="ij"), -1).reshape(-1, len(ref))
+    return int(np.any(np.all(F[None, :, :] <= Z[:, None, :], -1), 1).sum())
+
+
+def test_hv_golden_cases():
+    gold = json.load(open(GOLD))
+    for case in gold["hv"]:
+        assert oracle.hv(case["F"], np.array(case["ref"], float)) == pytest.approx(case["hv"], abs=1e-12)
+    for case in gold["hvi"]:
+        got = oracle.hvi(case["F"], np.array(case["ref"], float), np.array(case["y"], float))
+        assert got == pytest.approx(case["hvi"], abs=1e-12)
+
+
+@pytest.mark.parametrize("m,seed", [(2, 0), (2, 1), (3, 2), (3, 3), (4, 4)])
+def test_hv_matches_grid_enumeration(m, seed):
+    rng = np.random.default_rng(seed)
+    ref = np.full(m, 8 if m < 4 else 5)
+    for _ in range(20):
+        F = rng.integers(0, ref[0] + 2, size=(rng.integers(0, 9), m))
+        assert oracle.hv(F.astype(float), ref.astype(float)) == _hv_grid(F, ref)
+        y = rng.integers(0, ref[0], size=m)
+        want = _hv_grid(np.vstack([F, y]), ref) - _hv_grid(F, ref)
+        assert oracle.hvi(F.astype(float), ref.astype(float), y.astype(float)) == want
+
+
+# ------------------------------------------------------------ EHVI (closed form)
+def _hvi_staircase_integral(F, ref, y):
+    """2-D HVI by integrating, over z1 in [y1, r1), the exposed height
+    min(r2, h(z1)) - y2 where h(z1) = min{p2 : p in F, p1 <= z1}."""
+    F = np.asarray(F, float).reshape(-1, 2)
+    cuts = sorted({y[0], ref[0], *[p[0] for p in F if y[0] < p[0] < ref[0]]})
+    tot = 0.0
+    for a, b in zip(cuts[:-1], cuts[1:]):
+        h = min([ref[1]] + [p[1] for p in F if p[0] <= a])
+        tot += (b - a) * max(0.0, h - y[1])
+    return tot if y[0] < ref[0] else 0.0
+
+
+def _front2d(seed, P):
+    rng = np.random.default_rng(seed)
+    x = np.sort(rng.uniform(-1.5, 0.8, P))
+    ys = np.sort(rng.uniform(-1.5, 0.8, P))[::-1]
+    return np.stack([x, ys], 1)
+
+
+def test_ehvi_golden_cases():
+    gold = json.load(open(GOLD))
+    for case in gold["ehvi2d"]:
+        got = oracle.ehvi2d(np.array([case["mean"]]), np.array([case["var"]]),
+                            np.array(case["F"], float).reshape(-1, 2), np.array(case["ref"]))
+        assert got[0] == pytest.approx(case["ehvi"], rel=1e-14)
+
+
+def test_ehvi_empty_front_by_quadrature():
+    ref = np.array([1.1, 1.1])
+    mean = np.array([[0.3, 1.5], [-2.0, 0.9]])
+    var = np.array([[0.49, 0.25], [1.7, 0.01]])
+
+    def e_pos(r, mu, s):
+        f = lambda y: (r - y) * math.exp(-0.5 * ((y - mu) / s) ** 2) / (s * math.sqrt(2 * math.pi))
+        return scipy.integrate.quad(f, mu - 40 * s, r, epsabs=1e-14, epsrel=1e-12, limit=200)[0]
+
+    got = oracle.ehvi2d(mean, var, np.zeros((0, 2)), ref)
+    for c in range(2):
+        want = e_pos(ref[0], mean[c, 0], math.sqrt(var[c, 0])) * e_pos(ref[1], mean[c, 1],
+                                                                        math.sqrt(var[c, 1]))
+        assert got[c] == pytest.approx(want, rel=1e-9)
+
+
+def test_hvi_cell_sum_and_staircase_integral_agree():
+    F = _front2d(7, 6)
+    ref = np.array([1.1, 1.1])
+    rng = np.random.default_rng(8)
+    for y in rng.uniform(-2, 1.5, (200, 2)):
+        assert oracle.hvi(F, ref, y) == pytest.approx(_hvi_staircase_integral(F, ref, y),
+                                                      abs=1e-12)
+
+
+@pytest.mark.parametrize("case", range(4))
+def test_ehvi_matches_brute_force_monte_carlo(case):
+    """1e6 samples per candidate; candidates whose EHVI is not a tail event."""
+    F = _front2d(11 + case, 6)
+    ref = np.array([1.1, 1.1])
+    rng = np.random.default_rng(100 + case)
+    mu = F.min(0) + rng.uniform(-0.6, 0.3, 2)  # improving on most samples
+    sd = rng.uniform(0.08, 0.2, 2)
+    got = oracle.ehvi2d(mu[None], (sd ** 2)[None], F, ref)[0]
+    n = 1_000_000  # antithetic pairs: z and -z
+    Z = rng.standard_normal((n // 2, 2))
+    Ysmp = mu + sd * np.concatenate([Z, -Z])
+    # vectorised staircase integral of the HVI of every sample
+    cuts = np.concatenate([F[:, 0], [ref[0]]])
+    lefts = np.concatenate([[-np.inf], F[:, 0]])
+    heights = np.concatenate([[ref[1]], F[:, 1]])
+    w = np.clip(cuts[None, :] - np.maximum(lefts[None, :], Ysmp[:, :1]), 0, None)
+    h = np.clip(heights[None, :] - Ysmp[:, 1:], 0, None)
+    mc = (w * h).sum(1)
+    se = (0.5 * (mc[:n // 2] + mc[n // 2:])).std() / math.sqrt(n // 2)
+    assert se < 3e-4 * got  # the 1e-3 bar is at least 3 standard errors wide
+    assert abs(got - mc.mean()) < 1e-3 * got
+
+
+def test_ehvi_by_2d_quadrature_against_exact_hvi():
+    F = _front2d(21, 4)
+    ref = np.array([1.1, 1.1])
+    mu, sd = np.array([0.0, -0.2]), np.array([0.4, 0.3])
+    got = oracle.ehvi2d(mu[None], (sd ** 2)[None], F, ref)[0]
+    pdf = lambda y, m, s: math.exp(-0.5 * ((y - m) / s) ** 2) / (s * math.sqrt(2 * math.pi))
+    breaks = sorted(set(F[:, 0].tolist() + [ref[0]]))
+    tot = 0.0
+    lo = mu[0] - 9 * sd[0]
+    for a, b in zip([lo] + breaks[:-1], breaks):
+        if b <= lo:
+            continue
+        tot += scipy.integrate.dblquad(
+            lambda y2, y1: oracle.hvi(F, ref, np.array([y1, y2])) * pdf(y1, mu[0], sd[0]) *
+            pdf(y2, mu[1], sd[1]), max(a, lo), b, mu[1] - 9 * sd[1], ref[1],
+            epsabs=1e-10, epsrel=1e-8)[0]
+    assert got == pytest.approx(tot, rel=1e-5)
+
+
+def test_ehvi_limits_and_sign():
+    F = _front2d(31, 5)
+    ref = np.array([1.1, 1.1])
+    rng = np.random.default_rng(32)
+    mu = rng.uniform(-2, 2, (300, 2))
+    var = rng.uniform(0, 1, (300, 2))
+    e = oracle.ehvi2d(mu, var, F, ref)
+    assert np.all(e >= 0)
+    # sigma -> 0: EHVI -> HVI(mu)
+    e0 = oracle.ehvi2d(mu, np.zeros_like(var), F, ref)
+    for c in range(300):
+        assert e0[c] == pytest.approx(oracle.hvi(F, ref, mu[c]), abs=1e-13)
+    e1 = oracle.ehvi2d(mu[:20], np.full((20, 2), 1e-16), F, ref)
+    np.testing.assert_allclose(e1, e0[:20], atol=1e-7)
+    # a candidate well inside the dominated region with tiny sigma: ~0
+    dom = F.max(0) + 0.5
+    assert oracle.ehvi2d(dom[None], np.full((1, 2), 1e-4), F, ref)[0] < 1e-12
+
+
+# ------------------------------------------------------------ MC HVI
+@pytest.mark.parametrize("m", [2, 3])
+def test_mc_hvi_is_the_sample_mean_of_exact_hvi(m):
+    rng = np.random.default_rng(40 + m)
+    ref = np.full(m, 1.1)
+    Yobs = rng.normal(size=(60, m))
+    mask, order = oracle.pareto_front(Yobs, ref)
+    F = Yobs[order]
+    N, S = 7, 16
+    mean = rng.normal(size=(N, m))
+    var = rng.uniform(0, 0.5, (N, m))
+    eps = rng.standard_normal((N, m, S)).astype(np.float32)
+    got = oracle.mc_hvi(mean, var, eps, F, ref)
+    for c in range(N):
+        ys = mean[c][:, None] + np.sqrt(var[c])[:, None] * eps[c].astype(np.float64)
+        want = np.mean([oracle.hvi(F, ref, ys[:, s]) for s in range(S)])
+        assert got[c] == pytest.approx(want, rel=1e-12, abs=1e-15)
+    # shared normals (candidate stride 0) equal per-candidate copies of the same block
+    shared = oracle.mc_hvi(mean, var, eps[:1], F, ref, eps_stride=0)
+    rep = oracle.mc_hvi(mean, var, np.repeat(eps[:1], N, 0), F, ref)
+    np.testing.assert_allclose(shared, rep, rtol=0, atol=0)
+
+
+def test_mc_hvi_zero_variance_and_convergence_to_closed_form():
+    F = _front2d(51, 5)
+    ref = np.array([1.1, 1.1])
+    mu = np.array([[-0.3, 0.1], [0.2, -0.6]])
+    eps = np.random.default_rng(52).standard_normal((2, 2, 8)).astype(np.float32)
+    z = oracle.mc_hvi(mu, np.zeros((2, 2)), eps, F, ref)
+    for c in range(2):
+        assert z[c] == pytest.approx(oracle.hvi(F, ref, mu[c]), abs=1e-14)
+    var = np.array([[0.2, 0.1], [0.05, 0.3]])
+    S = 200_000
+    eps = np.random.default_rng(53).standard_normal((1, 2, S)).astype(np.float32)
+    mc = oracle.mc_hvi(mu, var, eps, F, ref, eps_stride=0)
+    cf = oracle.ehvi2d(mu, var, F, ref)
+    np.testing.assert_allclose(mc, cf, rtol=1e-2)
+
+
+# ------------------------------------------------------------ top-k
+def test_topk_order_ties_and_nan():
+    rng = np.random.default_rng(60)
+    acq = np.round(rng.random(5000), 3)  # many ties
+    acq[[5, 17, 400]] = np.nan
+    acq[[9, 10]] = np.inf
+    idx, val = oracle.topk(acq, 64)
+    key = np.where(np.isnan(acq), -np.inf, acq)
+    ref_order = np.lexsort((np.arange(acq.size), -key))
+    assert idx.tolist() == ref_order[:64].tolist()
+    assert np.array_equal(val, acq[ref_order[:64]])
+    idx_all, _ = oracle.topk(acq, 10**6)  # k > N returns N entries, NaN last
+    assert idx_all.tolist() == ref_order.tolist()
+
+
+# ------------------------------------------------------------ composed step
+def test_pipeline_config0_end_to_end_shapes_and_topk_consistency():
+    w = wl.WORKLOADS[0]
+    X, Y = wl.training_set(w, 0)
+    ls, s2, noise = wl.hyperparameters(w, 0)
+    fp = pipeline.fit_problem(X, Y, ls, s2, noise, wl.ref_point(w))
+    Xc = wl.candidates(w, 0)
+    mean, var, acq, idx, val = pipeline.score(fp, Xc, w.mode, w.k)
+    assert mean.shape == (w.N, 2) and acq.shape == (w.N,) and idx.shape == (w.k,)
+    assert np.all(acq >= 0) and np.all(np.diff(val) <= 0)
+    assert fp.front.shape[0] == int(fp.mask.sum())
