@@ -1,0 +1,200 @@
+/*
+ * libboute: GB300-native candidate scoring for the multi-objective Bayesian
+ * optimisation (MOBO) loop of BOute (arXiv 2602.10729).
+ *
+ * One MOBO iteration (Sec. 5.2, "Overall MOBO workflow") fits one Gaussian
+ * process per objective, then optimises the hypervolume-improvement
+ * acquisition (Sec. 5.2, "Constrained qNEHVI") over the decision space and
+ * selects the next configuration theta*. This library implements that step
+ * over a discrete candidate set: standardise -> fit -> Pareto front ->
+ * posterior -> acquisition -> top-k. All objectives are minimised (Sec. 4.3).
+ *
+ * Conventions (every entry point):
+ *  - Arrays are DEVICE pointers, owned by the caller, row-major and
+ *    contiguous, unless the argument says "host". Only boute_gp and
+ *    boute_engine objects own device memory, freed by their *_free call.
+ *  - Every call is asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *    default stream) unless it says it synchronises.
+ *  - Argument errors are returned synchronously and launch nothing. Errors
+ *    raised on the device (a non-positive Cholesky pivot, a wait that timed
+ *    out) are recorded in a device status word and returned by the next call
+ *    that synchronises (boute_gp_status, boute_engine_step*).
+ *  - B independent problems share one call; problem b's data follow
+ *    problem b-1's in every array.
+ *  - Limits: d <= 32, m <= 4 (m <= 3 for Monte-Carlo HVI, m == 2 for the
+ *    closed-form EHVI), 1 <= n <= 2048, B*N < 2^31, k <= 1024.
+ *
+ * Status codes are the boute_status values; every function returns one.
+ */
+#ifndef BOUTE_H
+#define BOUTE_H
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  BOUTE_OK = 0,
+  BOUTE_ERR_INVALID_ARG = 1, /* bad size, null pointer, unsupported shape */
+  BOUTE_ERR_NOT_PD = 2,      /* kernel matrix not positive definite */
+  BOUTE_ERR_CUDA = 3,        /* a CUDA runtime call failed */
+  BOUTE_ERR_OOM = 4,         /* device allocation failed */
+  BOUTE_ERR_UNSUPPORTED = 5, /* no sm_103a device, or shape beyond the limits */
+  BOUTE_ERR_TIMEOUT = 6      /* a device-side wait gave up (nothing hung) */
+} boute_status;
+
+typedef enum { BOUTE_ACQ_EHVI2D = 0, BOUTE_ACQ_MC_HVI = 1 } boute_acq_mode;
+
+/* Human-readable name of a status code (static string). */
+const char *boute_status_string(int status);
+
+/* Number of kernels this library has launched in this process (all streams).
+ * A monotone counter; differences bracket a region of work. */
+unsigned long long boute_launch_count(void);
+
+/* ---- a0: outcome standardisation -----------------------------------------
+ * Sec. 6 (outcome transform "Standardize", applied after Sec. 5.2 S4's
+ * Log/Logit, which stay with the caller): Ys[b,:,t] = (Y[b,:,t] - mean) / std,
+ * std with the n-1 denominator; a column with n < 2 or std < 1e-8 is divided
+ * by 1. Y, Ys: B x n x m fp64 (may alias). */
+int boute_standardize(const double *Y, int B, int n, int m, double *Ys, void *stream);
+
+/* ---- a1: GP fit ------------------------------------------------------------
+ * Sec. 5.2 step (i) and Sec. 6: one exact GP per objective (SingleTaskGP
+ * models combined as a ModelListGP), ARD Matern-5/2 covariance with an
+ * outputscale (MaternKernel nu=2.5 in a ScaleKernel), zero prior mean on
+ * standardised outcomes, fixed hyperparameters:
+ *   K = s2 * M52(X, X) + noise * I,  L = chol(K) (fp64, no jitter),
+ *   the library keeps L^-1 and alpha = K^-1 y as the tensor-core operand of
+ *   the posterior contraction.
+ * boute_gp_create allocates a handle for B problems x m objectives of n
+ * points in d dimensions (the only allocating call of the fit path);
+ * boute_gp_fit recomputes it asynchronously from
+ *   X: B x n x d fp64; Ys: B x n x m fp64 (standardised outcomes);
+ *   lengthscale: B x m x d fp64; outputscale, noise: B x m fp64.
+ * boute_gp_status synchronises `stream` and returns BOUTE_ERR_NOT_PD if a
+ * pivot of any problem/objective was not positive (its posterior is then
+ * undefined), else the first recorded device error, else BOUTE_OK; it clears
+ * the recorded status. */
+typedef struct boute_gp boute_gp;
+int boute_gp_create(int B, int n, int d, int m, boute_gp **out);
+int boute_gp_fit(boute_gp *gp, const double *X, const double *Ys, const double *lengthscale,
+                 const double *outputscale, const double *noise, void *stream);
+int boute_gp_status(boute_gp *gp, void *stream);
+void boute_gp_free(boute_gp *gp);
+
+/* ---- a2 + a3: posterior -----------------------------------------------------
+ * Latent-function posterior of every objective at N candidates per problem
+ * (Sec. 5.2: the acquisition is taken over the GP posterior):
+ *   mean = K* alpha,  var = max(0, s2 - rowsum((K* L^-T)^2)),
+ * with the Matern-5/2 cross-covariance K* built tile by tile in shared memory
+ * and contracted on the tensor cores in 3xTF32 (fp32-accurate) without ever
+ * being written to HBM.
+ *   Xc: B x N x d fp32 candidates (points of [0,1]^d or any real values);
+ *   mean, var: B x m x N fp32 (objective-major per problem). */
+int boute_gp_posterior(const boute_gp *gp, const float *Xc, long long N, float *mean,
+                       float *var, void *stream);
+
+/* ---- a4: Pareto front and box decomposition ---------------------------------
+ * Sec. 5.2 (Pareto-optimal set; Sec. 4.3, minimisation): point i of problem b
+ * is on the front iff no point dominates it (<= in every objective, < in
+ * one), no exact duplicate with a smaller index exists, and it is strictly
+ * better than ref in every objective.
+ *   Ys: B x n x m fp64; ref: B x m fp64;
+ *   mask: B x n bytes (1 = on the front);
+ *   front: B x n x m fp64, rows [0, P[b]) = the front sorted by f1, then f2,
+ *          ..., then index (rows beyond P[b] are left unspecified);
+ *   P: B ints. */
+int boute_pareto_front(const double *Ys, int B, int n, int m, const double *ref,
+                       unsigned char *mask, double *front, int *P, void *stream);
+
+/* Disjoint boxes covering the region that improves on the front and is below
+ * ref ({z <= ref : no front point p <= z}), the region whose volume inside
+ * [y, ref] is the hypervolume improvement of y (Sec. 5.2). m = 2: the P+1
+ * strips of the staircase; m = 3: a sweep along f3 (at most 2P+1 boxes).
+ * Lower bounds may be -infinity.
+ *   front, P: as written by boute_pareto_front (capacity n rows per problem);
+ *   lower, upper: B x (2n+2) x m fp32; K: B ints (boxes per problem). */
+int boute_box_decompose(const double *front, const int *P, int B, int n, int m,
+                        const double *ref, float *lower, float *upper, int *K, void *stream);
+
+/* ---- a5: acquisition ----------------------------------------------------------
+ * Expected hypervolume improvement (Sec. 5.2, "Constrained qNEHVI": the
+ * expectation of HVI over the posterior), for m = 2 independent objectives in
+ * closed form over the P+1 staircase cells:
+ *   EHVI = sum_i [psi1(b_i) - psi1(a_i)] psi2(u_i),  psi(c) = E[(c - Y)_+].
+ *   mean, var: B x 2 x N fp32 (boute_gp_posterior's layout);
+ *   front, P: boute_pareto_front's output, n = its row capacity; ref: B x 2;
+ *   acq: B x N fp32. */
+int boute_acq_ehvi(const float *mean, const float *var, int B, long long N, const double *front,
+                   const int *P, int n, const double *ref, float *acq, void *stream);
+
+/* Monte-Carlo hypervolume improvement (Sec. 5.2: the expectation estimated by Monte-Carlo
+ * integration over posterior samples): sample s of candidate c is
+ * y_t = mean_t + sqrt(var_t) * eps[c][t][s]; acq = mean over S samples of the
+ * exact HVI of y, the volume of [y, ref] inside the boxes.
+ *   lower, upper, K, box_cap: boute_box_decompose's output (box_cap = 2n+2);
+ *   eps: fp32 base normals, candidate c of problem b at
+ *        eps + (b*N + c) * eps_cand_stride, laid out m x S; eps_cand_stride =
+ *        m*S for per-candidate normals, 0 for normals shared by all candidates
+ *        of a problem (then problem b's block is at eps + b*m*S);
+ *   acq: B x N fp32. 2 <= m <= 3, 1 <= S. */
+int boute_acq_mc_hvi(const float *mean, const float *var, int B, long long N, int m,
+                     const float *lower, const float *upper, const int *K, int box_cap,
+                     const float *eps, int S, long long eps_cand_stride, float *acq,
+                     void *stream);
+
+/* ---- a6: selection ------------------------------------------------------------
+ * Sec. 5.2 step (ii): the next configuration(s) to evaluate are the best
+ * scored candidates. Per problem, the k largest acq values in the order
+ * (value descending, NaN as -infinity, -0 as +0, equal values by ascending
+ * index); idx: B x k int64 (candidate index within its problem), val: B x k
+ * fp32 (the acq value at idx). k <= min(N, 1024). Uses stream-ordered
+ * scratch from the CUDA memory pool. */
+int boute_select_topk(const float *acq, int B, long long N, int k, long long *idx, float *val,
+                      void *stream);
+
+/* ---- the whole scoring step ---------------------------------------------------
+ * An engine owns every intermediate buffer of one workload shape and runs
+ * a0..a6 as one launch sequence on one stream.
+ * boute_engine_step: device inputs; boute_engine_step_host: HOST inputs and
+ * outputs (copied in and out on `stream` inside the call); both synchronise
+ * and return the fit status or the first device error.
+ *   X: B x n x d fp64; Y: B x n x m fp64 raw outcomes (standardised inside);
+ *   lengthscale: B x m x d; outputscale, noise: B x m; ref: B x m (fp64);
+ *   Xc: B x N x d fp32; eps: B x N x m x S fp32 (mode MC_HVI; NULL otherwise);
+ *   idx: B x k int64, val: B x k fp32.
+ * boute_engine_step_async: as boute_engine_step without the final
+ * synchronisation (device errors surface at the next synchronising call). */
+typedef struct boute_engine boute_engine;
+int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S, int k,
+                        boute_engine **out);
+int boute_engine_step(boute_engine *e, const double *X, const double *Y,
+                      const double *lengthscale, const double *outputscale,
+                      const double *noise, const double *ref, const float *Xc, const float *eps,
+                      long long *idx, float *val, void *stream);
+int boute_engine_step_async(boute_engine *e, const double *X, const double *Y,
+                            const double *lengthscale, const double *outputscale,
+                            const double *noise, const double *ref, const float *Xc,
+                            const float *eps, long long *idx, float *val, void *stream);
+int boute_engine_step_host(boute_engine *e, const double *X, const double *Y,
+                           const double *lengthscale, const double *outputscale,
+                           const double *noise, const double *ref, const float *Xc,
+                           const float *eps, long long *idx, float *val, void *stream);
+/* Copies the last step's per-candidate results into caller buffers (device
+ * pointers; any may be NULL): acq B x N, mean and var B x m x N (fp32). */
+int boute_engine_scores(const boute_engine *e, float *acq, float *mean, float *var, void *stream);
+/* Stage timing on the engine's stream: once enabled, every step records a
+ * CUDA event at each stage boundary (standardise, fit, front, boxes,
+ * posterior, acquisition, top-k); boute_engine_stage_times waits for the
+ * last step and writes its 7 stage durations in milliseconds (count >= 7). */
+int boute_engine_set_timing(boute_engine *e, int on);
+int boute_engine_stage_times(boute_engine *e, float *ms, int count);
+/* Kernels one boute_engine_step launches. */
+int boute_engine_launches_per_step(const boute_engine *e);
+void boute_engine_free(boute_engine *e);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

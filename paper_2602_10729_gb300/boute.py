@@ -1,0 +1,285 @@
+"""Thin ctypes binding of libboute (include/boute.h): argument marshalling only.
+
+Every function carries the C entry point's name and forwards torch tensors'
+device pointers and the current CUDA stream; all arithmetic runs in the
+library's kernels. There is no fallback: if ``libboute.so`` has not been built,
+or the device is not sm_103a, calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from . import build as _build
+
+BOUTE_OK, BOUTE_ERR_INVALID_ARG, BOUTE_ERR_NOT_PD, BOUTE_ERR_CUDA = 0, 1, 2, 3
+BOUTE_ERR_OOM, BOUTE_ERR_UNSUPPORTED, BOUTE_ERR_TIMEOUT = 4, 5, 6
+BOUTE_ACQ_EHVI2D, BOUTE_ACQ_MC_HVI = 0, 1
+
+#: exported symbols declared in include/boute.h
+SYMBOLS = (
+    "boute_status_string", "boute_launch_count", "boute_standardize", "boute_gp_create",
+    "boute_gp_fit", "boute_gp_status", "boute_gp_free", "boute_gp_posterior",
+    "boute_pareto_front", "boute_box_decompose", "boute_acq_ehvi", "boute_acq_mc_hvi",
+    "boute_select_topk", "boute_engine_create", "boute_engine_step", "boute_engine_step_async",
+    "boute_engine_step_host", "boute_engine_scores", "boute_engine_set_timing",
+    "boute_engine_stage_times", "boute_engine_launches_per_step", "boute_engine_free",
+)
+#: stage names of boute_engine_stage_times, in order
+STAGES = ("standardize", "fit", "front", "boxes", "posterior", "acquisition", "topk")
+
+_lib = None
+_vp = ctypes.c_void_p
+_i = ctypes.c_int
+_ll = ctypes.c_longlong
+
+
+class BouteError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        super().__init__(f"{where}: {status_string(code)} ({code})")
+        self.code = code
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(path: str | None = None):
+    """Load libboute.so; raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = path or _build.LIB
+    if not os.path.exists(path):
+        raise RuntimeError(f"libboute.so not built ({path}); run __graft_entry__.build()")
+    L = ctypes.CDLL(path)
+    sig = {
+        "boute_status_string": ([_i], ctypes.c_char_p),
+        "boute_launch_count": ([], ctypes.c_ulonglong),
+        "boute_standardize": ([_vp, _i, _i, _i, _vp, _vp], _i),
+        "boute_gp_create": ([_i, _i, _i, _i, ctypes.POINTER(_vp)], _i),
+        "boute_gp_fit": ([_vp, _vp, _vp, _vp, _vp, _vp, _vp], _i),
+        "boute_gp_status": ([_vp, _vp], _i),
+        "boute_gp_free": ([_vp], None),
+        "boute_gp_posterior": ([_vp, _vp, _ll, _vp, _vp, _vp], _i),
+        "boute_pareto_front": ([_vp, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
+        "boute_box_decompose": ([_vp, _vp, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
+        "boute_acq_ehvi": ([_vp, _vp, _i, _ll, _vp, _vp, _i, _vp, _vp, _vp], _i),
+        "boute_acq_mc_hvi": ([_vp, _vp, _i, _ll, _i, _vp, _vp, _vp, _i, _vp, _i, _ll, _vp, _vp],
+                             _i),
+        "boute_select_topk": ([_vp, _i, _ll, _i, _vp, _vp, _vp], _i),
+        "boute_engine_create": ([_i, _i, _i, _i, _ll, _i, _i, _i, ctypes.POINTER(_vp)], _i),
+        "boute_engine_step": ([_vp] * 11 + [_vp], _i),
+        "boute_engine_step_async": ([_vp] * 11 + [_vp], _i),
+        "boute_engine_step_host": ([_vp] * 11 + [_vp], _i),
+        "boute_engine_scores": ([_vp, _vp, _vp, _vp, _vp], _i),
+        "boute_engine_set_timing": ([_vp, _i], _i),
+        "boute_engine_stage_times": ([_vp, ctypes.POINTER(ctypes.c_float), _i], _i),
+        "boute_engine_launches_per_step": ([_vp], _i),
+        "boute_engine_free": ([_vp], None),
+    }
+    for name, (args, res) in sig.items():
+        f = getattr(L, name)
+        f.argtypes = args
+        f.restype = res
+    _lib = L
+    return L
+
+
+def status_string(code: int) -> str:
+    try:
+        return load().boute_status_string(code).decode()
+    except Exception:
+        return f"status {code}"
+
+
+def _check(rc: int, where: str):
+    if rc != BOUTE_OK:
+        raise BouteError(rc, where)
+
+
+def _p(t, dtype=None, device=True):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"expected {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError("tensors must be contiguous")
+    if device and not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    return t.data_ptr()
+
+
+def _s(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else stream
+
+
+def boute_launch_count() -> int:
+    return int(load().boute_launch_count())
+
+
+def boute_standardize(Y, Ys, stream=None):
+    B, n, m = Y.shape
+    _check(load().boute_standardize(_p(Y, torch.float64), B, n, m, _p(Ys, torch.float64),
+                                    _s(stream)), "boute_standardize")
+
+
+class Gp:
+    """Owner of a boute_gp handle (device factors of B problems x m objectives)."""
+
+    def __init__(self, B: int, n: int, d: int, m: int):
+        self.B, self.n, self.d, self.m = B, n, d, m
+        h = _vp()
+        _check(load().boute_gp_create(B, n, d, m, ctypes.byref(h)), "boute_gp_create")
+        self.handle = h
+
+    def free(self):
+        if self.handle:
+            load().boute_gp_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def boute_gp_create(B, n, d, m) -> Gp:
+    return Gp(B, n, d, m)
+
+
+def boute_gp_fit(gp: Gp, X, Ys, lengthscale, outputscale, noise, stream=None):
+    f64 = torch.float64
+    _check(load().boute_gp_fit(gp.handle, _p(X, f64), _p(Ys, f64), _p(lengthscale, f64),
+                               _p(outputscale, f64), _p(noise, f64), _s(stream)), "boute_gp_fit")
+
+
+def boute_gp_status(gp: Gp, stream=None) -> int:
+    return int(load().boute_gp_status(gp.handle, _s(stream)))
+
+
+def boute_gp_free(gp: Gp):
+    gp.free()
+
+
+def boute_gp_posterior(gp: Gp, Xc, N: int, mean, var, stream=None):
+    f32 = torch.float32
+    _check(load().boute_gp_posterior(gp.handle, _p(Xc, f32), N, _p(mean, f32), _p(var, f32),
+                                     _s(stream)), "boute_gp_posterior")
+
+
+def boute_pareto_front(Ys, B, n, m, ref, mask, front, P, stream=None):
+    f64 = torch.float64
+    _check(load().boute_pareto_front(_p(Ys, f64), B, n, m, _p(ref, f64), _p(mask, torch.uint8),
+                                     _p(front, f64), _p(P, torch.int32), _s(stream)),
+           "boute_pareto_front")
+
+
+def boute_box_decompose(front, P, B, n, m, ref, lower, upper, K, stream=None):
+    _check(load().boute_box_decompose(_p(front, torch.float64), _p(P, torch.int32), B, n, m,
+                                      _p(ref, torch.float64), _p(lower, torch.float32),
+                                      _p(upper, torch.float32), _p(K, torch.int32), _s(stream)),
+           "boute_box_decompose")
+
+
+def boute_acq_ehvi(mean, var, B, N, front, P, n, ref, acq, stream=None):
+    f32 = torch.float32
+    _check(load().boute_acq_ehvi(_p(mean, f32), _p(var, f32), B, N, _p(front, torch.float64),
+                                 _p(P, torch.int32), n, _p(ref, torch.float64), _p(acq, f32),
+                                 _s(stream)), "boute_acq_ehvi")
+
+
+def boute_acq_mc_hvi(mean, var, B, N, m, lower, upper, K, box_cap, eps, S, eps_cand_stride, acq,
+                     stream=None):
+    f32 = torch.float32
+    _check(load().boute_acq_mc_hvi(_p(mean, f32), _p(var, f32), B, N, m, _p(lower, f32),
+                                   _p(upper, f32), _p(K, torch.int32), box_cap, _p(eps, f32), S,
+                                   eps_cand_stride, _p(acq, f32), _s(stream)), "boute_acq_mc_hvi")
+
+
+def boute_select_topk(acq, B, N, k, idx, val, stream=None):
+    _check(load().boute_select_topk(_p(acq, torch.float32), B, N, k, _p(idx, torch.int64),
+                                    _p(val, torch.float32), _s(stream)), "boute_select_topk")
+
+
+class Engine:
+    """Owner of a boute_engine (all buffers of one scoring-step shape)."""
+
+    def __init__(self, B, n, d, m, N, mode, S, k):
+        self.B, self.n, self.d, self.m, self.N, self.mode, self.S, self.k = (
+            B, n, d, m, N, mode, S, k)
+        h = _vp()
+        _check(load().boute_engine_create(B, n, d, m, N, mode, S, k, ctypes.byref(h)),
+               "boute_engine_create")
+        self.handle = h
+
+    def free(self):
+        if self.handle:
+            load().boute_engine_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def boute_engine_create(B, n, d, m, N, mode, S, k) -> Engine:
+    return Engine(B, n, d, m, N, mode, S, k)
+
+
+def _engine_args(X, Y, ls, s2, noise, ref, Xc, eps, idx, val, device):
+    f64, f32 = torch.float64, torch.float32
+    return (_p(X, f64, device), _p(Y, f64, device), _p(ls, f64, device), _p(s2, f64, device),
+            _p(noise, f64, device), _p(ref, f64, device), _p(Xc, f32, device),
+            _p(eps, f32, device), _p(idx, torch.int64, device), _p(val, f32, device))
+
+
+def boute_engine_step(e: Engine, X, Y, ls, s2, noise, ref, Xc, eps, idx, val, stream=None):
+    """Device tensors in and out; synchronises; raises on a fit or device error."""
+    _check(load().boute_engine_step(e.handle, *_engine_args(X, Y, ls, s2, noise, ref, Xc, eps,
+                                                            idx, val, True), _s(stream)),
+           "boute_engine_step")
+
+
+def boute_engine_step_async(e: Engine, X, Y, ls, s2, noise, ref, Xc, eps, idx, val, stream=None):
+    _check(load().boute_engine_step_async(e.handle, *_engine_args(
+        X, Y, ls, s2, noise, ref, Xc, eps, idx, val, True), _s(stream)), "boute_engine_step_async")
+
+
+def boute_engine_step_host(e: Engine, X, Y, ls, s2, noise, ref, Xc, eps, idx, val, stream=None):
+    """HOST (CPU, ideally pinned) tensors in and out; copies inside the call."""
+    _check(load().boute_engine_step_host(e.handle, *_engine_args(
+        X, Y, ls, s2, noise, ref, Xc, eps, idx, val, False), _s(stream)), "boute_engine_step_host")
+
+
+def boute_engine_scores(e: Engine, acq=None, mean=None, var=None, stream=None):
+    f32 = torch.float32
+    _check(load().boute_engine_scores(e.handle, _p(acq, f32), _p(mean, f32), _p(var, f32),
+                                      _s(stream)), "boute_engine_scores")
+
+
+def boute_engine_set_timing(e: Engine, on: bool = True):
+    _check(load().boute_engine_set_timing(e.handle, int(on)), "boute_engine_set_timing")
+
+
+def boute_engine_stage_times(e: Engine) -> dict:
+    ms = (ctypes.c_float * len(STAGES))()
+    _check(load().boute_engine_stage_times(e.handle, ms, len(STAGES)), "boute_engine_stage_times")
+    return dict(zip(STAGES, (float(x) for x in ms)))
+
+
+def boute_engine_launches_per_step(e: Engine) -> int:
+    return int(load().boute_engine_launches_per_step(e.handle))
+
+
+def boute_engine_free(e: Engine):
+    e.free()

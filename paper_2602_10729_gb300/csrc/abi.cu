@@ -1,0 +1,407 @@
+// The C ABI of libboute (declared in include/boute.h): argument validation,
+// handle and engine ownership, and the launch sequence of one scoring step.
+#include <atomic>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+
+#include "internal.h"
+
+namespace boute {
+
+static std::atomic<unsigned long long> g_launches{0};
+void count_launch(int k) { g_launches.fetch_add((unsigned long long)k); }
+unsigned long long launch_count() { return g_launches.load(); }
+
+int last_launch_status() {
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) return BOUTE_OK;
+  if (e == cudaErrorMemoryAllocation) return BOUTE_ERR_OOM;
+  std::fprintf(stderr, "libboute: %s\n", cudaGetErrorString(e));
+  return BOUTE_ERR_CUDA;
+}
+
+// The kernels are built for sm_103a only: refuse other devices up front.
+static int device_ok() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return BOUTE_ERR_UNSUPPORTED;
+  int major = 0, minor = 0;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+  cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+  return (major == 10 && minor == 3) ? BOUTE_OK : BOUTE_ERR_UNSUPPORTED;
+}
+
+template <class T>
+static int dalloc(T **p, size_t count) {
+  *p = nullptr;
+  if (count == 0) return BOUTE_OK;
+  cudaError_t e = cudaMalloc((void **)p, count * sizeof(T));
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    *p = nullptr;
+    return BOUTE_ERR_OOM;
+  }
+  return BOUTE_OK;
+}
+
+static int pad_dims(int d) { return d <= 8 ? 8 : d <= 12 ? 12 : d <= 16 ? 16 : d <= 24 ? 24 : 32; }
+
+static int shape_ok(int B, int n, int d, int m) {
+  return B >= 1 && n >= 1 && n <= BOUTE_MAX_N && d >= 1 && d <= BOUTE_MAX_D && m >= 1 &&
+         m <= BOUTE_MAX_M;
+}
+
+}  // namespace boute
+
+using namespace boute;
+
+struct boute_gp {
+  Gp g;
+};
+
+struct boute_engine {
+  int B, n, d, m, mode, S, k;
+  long long N;
+  boute_gp *gp;
+  double *X, *Y, *Ys, *ls, *s2, *noise, *ref, *front;
+  unsigned char *mask;
+  int *P, *K;
+  float *lower, *upper, *Xc, *eps, *mean, *var, *acq, *val;
+  long long *idx;
+  void *scratch;
+  int launches;
+  int timing;                  // record one CUDA event per stage boundary
+  cudaEvent_t ev[8];           // boundaries of the stages of the last step
+  int nstage;
+};
+
+// Stage order of one step; boxes run only in Monte-Carlo mode (zero-length
+// stage otherwise).
+enum { ST_STANDARDIZE, ST_FIT, ST_FRONT, ST_BOXES, ST_POSTERIOR, ST_ACQ, ST_TOPK, ST_COUNT };
+
+extern "C" {
+
+const char *boute_status_string(int s) {
+  switch (s) {
+    case BOUTE_OK: return "ok";
+    case BOUTE_ERR_INVALID_ARG: return "invalid argument";
+    case BOUTE_ERR_NOT_PD: return "kernel matrix not positive definite";
+    case BOUTE_ERR_CUDA: return "CUDA error";
+    case BOUTE_ERR_OOM: return "out of device memory";
+    case BOUTE_ERR_UNSUPPORTED: return "unsupported device or shape";
+    case BOUTE_ERR_TIMEOUT: return "device-side wait timed out";
+  }
+  return "unknown status";
+}
+
+unsigned long long boute_launch_count(void) { return launch_count(); }
+
+int boute_standardize(const double *Y, int B, int n, int m, double *Ys, void *stream) {
+  if (!Y || !Ys || B < 1 || n < 1 || m < 1) return BOUTE_ERR_INVALID_ARG;
+  if (int r = device_ok()) return r;
+  return launch_standardize(Y, B, n, m, Ys, (cudaStream_t)stream);
+}
+
+int boute_gp_create(int B, int n, int d, int m, boute_gp **out) {
+  if (!out) return BOUTE_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!shape_ok(B, n, d, m)) return BOUTE_ERR_INVALID_ARG;
+  if (int r = device_ok()) return r;
+  boute_gp *h = new (std::nothrow) boute_gp();
+  if (!h) return BOUTE_ERR_OOM;
+  Gp &g = h->g;
+  g.B = B; g.n = n; g.d = d; g.m = m; g.DP = pad_dims(d);
+  g.plan = make_post_plan(n);
+  const size_t BM = (size_t)B * m;
+  int r = BOUTE_OK;
+  r |= dalloc(&g.K, BM * n * n);
+  r |= dalloc(&g.W, BM * n * n);
+  r |= dalloc(&g.alpha, BM * n);
+  r |= dalloc(&g.bop, BM * (size_t)g.plan.image_floats);
+  r |= dalloc(&g.xt, BM * (size_t)g.plan.npad * 2 * g.DP);
+  r |= dalloc(&g.invls, BM * 2 * g.DP);
+  r |= dalloc(&g.s2f, BM);
+  r |= dalloc(&g.status, 1);
+  if (r != BOUTE_OK) {
+    boute_gp_free(h);
+    return BOUTE_ERR_OOM;
+  }
+  cudaMemset(g.status, 0, sizeof(int));
+  // operand images are fully rewritten by every fit; zero them once so that
+  // padding never holds stale bits
+  cudaMemset(g.bop, 0, BM * (size_t)g.plan.image_floats * sizeof(float));
+  *out = h;
+  return BOUTE_OK;
+}
+
+int boute_gp_fit(boute_gp *gp, const double *X, const double *Ys, const double *lengthscale,
+                 const double *outputscale, const double *noise, void *stream) {
+  if (!gp || !X || !Ys || !lengthscale || !outputscale || !noise) return BOUTE_ERR_INVALID_ARG;
+  return launch_fit(&gp->g, X, Ys, lengthscale, outputscale, noise, (cudaStream_t)stream);
+}
+
+int boute_gp_status(boute_gp *gp, void *stream) {
+  if (!gp) return BOUTE_ERR_INVALID_ARG;
+  if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return last_launch_status();
+  int st = 0;
+  if (cudaMemcpy(&st, gp->g.status, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return last_launch_status();
+  cudaMemset(gp->g.status, 0, sizeof(int));
+  return st;
+}
+
+void boute_gp_free(boute_gp *gp) {
+  if (!gp) return;
+  Gp &g = gp->g;
+  cudaFree(g.K); cudaFree(g.W); cudaFree(g.alpha); cudaFree(g.bop); cudaFree(g.xt);
+  cudaFree(g.invls); cudaFree(g.s2f); cudaFree(g.status);
+  delete gp;
+}
+
+int boute_gp_posterior(const boute_gp *gp, const float *Xc, long long N, float *mean, float *var,
+                       void *stream) {
+  if (!gp || N < 0 || (N > 0 && (!Xc || !mean || !var))) return BOUTE_ERR_INVALID_ARG;
+  if ((long long)gp->g.B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;
+  return launch_posterior(&gp->g, Xc, N, mean, var, (cudaStream_t)stream);
+}
+
+int boute_pareto_front(const double *Ys, int B, int n, int m, const double *ref,
+                       unsigned char *mask, double *front, int *P, void *stream) {
+  if (!Ys || !ref || !mask || !front || !P || !shape_ok(B, n, 1, m)) return BOUTE_ERR_INVALID_ARG;
+  if (int r = device_ok()) return r;
+  return launch_pareto(Ys, B, n, m, ref, mask, front, P, (cudaStream_t)stream);
+}
+
+int boute_box_decompose(const double *front, const int *P, int B, int n, int m, const double *ref,
+                        float *lower, float *upper, int *K, void *stream) {
+  if (!front || !P || !ref || !lower || !upper || !K || !shape_ok(B, n, 1, m))
+    return BOUTE_ERR_INVALID_ARG;
+  if (m < 2 || m > 3) return BOUTE_ERR_UNSUPPORTED;
+  if (int r = device_ok()) return r;
+  return launch_boxes(front, P, B, n, m, ref, lower, upper, K, (cudaStream_t)stream);
+}
+
+int boute_acq_ehvi(const float *mean, const float *var, int B, long long N, const double *front,
+                   const int *P, int n, const double *ref, float *acq, void *stream) {
+  if (B < 1 || N < 0 || n < 1 || n > BOUTE_MAX_N || !front || !P || !ref ||
+      (N > 0 && (!mean || !var || !acq)))
+    return BOUTE_ERR_INVALID_ARG;
+  if ((long long)B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;
+  if (int r = device_ok()) return r;
+  return launch_ehvi(mean, var, B, N, front, P, n, ref, acq, (cudaStream_t)stream);
+}
+
+int boute_acq_mc_hvi(const float *mean, const float *var, int B, long long N, int m,
+                     const float *lower, const float *upper, const int *K, int box_cap,
+                     const float *eps, int S, long long eps_cand_stride, float *acq,
+                     void *stream) {
+  if (B < 1 || N < 0 || S < 1 || box_cap < 1 || eps_cand_stride < 0 || !lower || !upper || !K ||
+      (N > 0 && (!mean || !var || !acq || !eps)))
+    return BOUTE_ERR_INVALID_ARG;
+  if (m < 2 || m > 3) return BOUTE_ERR_UNSUPPORTED;
+  if ((long long)B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;
+  if ((size_t)box_cap * m * 2 * sizeof(float) > 200 * 1024) return BOUTE_ERR_UNSUPPORTED;
+  if (int r = device_ok()) return r;
+  return launch_mchvi(mean, var, B, N, m, lower, upper, K, box_cap, eps, S, eps_cand_stride, acq,
+                      (cudaStream_t)stream);
+}
+
+int boute_select_topk(const float *acq, int B, long long N, int k, long long *idx, float *val,
+                      void *stream) {
+  if (!acq || !idx || !val || B < 1 || N < 1 || k < 1 || k > 1024 || k > N)
+    return BOUTE_ERR_INVALID_ARG;
+  if ((long long)B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;
+  if (int r = device_ok()) return r;
+  cudaStream_t s = (cudaStream_t)stream;
+  void *scratch = nullptr;
+  if (cudaMallocAsync(&scratch, topk_scratch_bytes(B, N, k), s) != cudaSuccess) {
+    cudaGetLastError();
+    return BOUTE_ERR_OOM;
+  }
+  int r = launch_topk(acq, B, N, k, idx, val, scratch, s);
+  cudaFreeAsync(scratch, s);
+  return r;
+}
+
+// ---- engine -------------------------------------------------------------------
+void boute_engine_free(boute_engine *e) {
+  if (!e) return;
+  boute_gp_free(e->gp);
+  if (e->timing)
+    for (int i = 0; i <= ST_COUNT; ++i) cudaEventDestroy(e->ev[i]);
+  void *ptrs[] = {e->X, e->Y, e->Ys, e->ls, e->s2, e->noise, e->ref, e->front, e->mask, e->P,
+                  e->K, e->lower, e->upper, e->Xc, e->eps, e->mean, e->var, e->acq, e->val,
+                  e->idx, e->scratch};
+  for (void *p : ptrs) cudaFree(p);
+  delete e;
+}
+
+int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S, int k,
+                        boute_engine **out) {
+  if (!out) return BOUTE_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!shape_ok(B, n, d, m) || N < 1 || k < 1 || k > 1024 || k > N) return BOUTE_ERR_INVALID_ARG;
+  if ((long long)B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;
+  if (mode == BOUTE_ACQ_EHVI2D && m != 2) return BOUTE_ERR_INVALID_ARG;
+  if (mode == BOUTE_ACQ_MC_HVI && (m < 2 || m > 3 || S < 1)) return BOUTE_ERR_INVALID_ARG;
+  if (mode != BOUTE_ACQ_EHVI2D && mode != BOUTE_ACQ_MC_HVI) return BOUTE_ERR_INVALID_ARG;
+  if (int r = device_ok()) return r;
+  boute_engine *e = new (std::nothrow) boute_engine();
+  if (!e) return BOUTE_ERR_OOM;
+  std::memset(e, 0, sizeof(*e));
+  e->B = B; e->n = n; e->d = d; e->m = m; e->N = N; e->mode = mode; e->S = S; e->k = k;
+  int r = boute_gp_create(B, n, d, m, &e->gp);
+  const size_t Bn = (size_t)B * n, BN = (size_t)B * N, cap = 2 * (size_t)n + 2;
+  r |= dalloc(&e->X, Bn * d);
+  r |= dalloc(&e->Y, Bn * m);
+  r |= dalloc(&e->Ys, Bn * m);
+  r |= dalloc(&e->ls, (size_t)B * m * d);
+  r |= dalloc(&e->s2, (size_t)B * m);
+  r |= dalloc(&e->noise, (size_t)B * m);
+  r |= dalloc(&e->ref, (size_t)B * m);
+  r |= dalloc(&e->front, Bn * m);
+  r |= dalloc(&e->mask, Bn);
+  r |= dalloc(&e->P, (size_t)B);
+  r |= dalloc(&e->K, (size_t)B);
+  r |= dalloc(&e->lower, (size_t)B * cap * m);
+  r |= dalloc(&e->upper, (size_t)B * cap * m);
+  r |= dalloc(&e->Xc, BN * d);
+  if (mode == BOUTE_ACQ_MC_HVI) r |= dalloc(&e->eps, BN * m * S);
+  r |= dalloc(&e->mean, BN * m);
+  r |= dalloc(&e->var, BN * m);
+  r |= dalloc(&e->acq, BN);
+  r |= dalloc(&e->idx, (size_t)B * k);
+  r |= dalloc(&e->val, (size_t)B * k);
+  r |= dalloc((unsigned char **)&e->scratch, topk_scratch_bytes(B, N, k));
+  if (r != BOUTE_OK) {
+    boute_engine_free(e);
+    return BOUTE_ERR_OOM;
+  }
+  *out = e;
+  return BOUTE_OK;
+}
+
+static int engine_run(boute_engine *e, const double *X, const double *Y, const double *ls,
+                      const double *s2, const double *noise, const double *ref, const float *Xc,
+                      const float *eps, long long *idx, float *val, cudaStream_t s) {
+  const unsigned long long l0 = launch_count();
+  int r;
+  const int B = e->B, n = e->n, m = e->m;
+  auto mark = [&](int stage) {
+    if (e->timing) cudaEventRecord(e->ev[stage], s);
+  };
+  mark(ST_STANDARDIZE);
+  if ((r = launch_standardize(Y, B, n, m, e->Ys, s))) return r;
+  mark(ST_FIT);
+  if ((r = launch_fit(&e->gp->g, X, e->Ys, ls, s2, noise, s))) return r;
+  mark(ST_FRONT);
+  if ((r = launch_pareto(e->Ys, B, n, m, ref, e->mask, e->front, e->P, s))) return r;
+  mark(ST_BOXES);
+  if (e->mode == BOUTE_ACQ_MC_HVI)
+    if ((r = launch_boxes(e->front, e->P, B, n, m, ref, e->lower, e->upper, e->K, s))) return r;
+  mark(ST_POSTERIOR);
+  if ((r = launch_posterior(&e->gp->g, Xc, e->N, e->mean, e->var, s))) return r;
+  mark(ST_ACQ);
+  if (e->mode == BOUTE_ACQ_EHVI2D) {
+    if ((r = launch_ehvi(e->mean, e->var, B, e->N, e->front, e->P, n, ref, e->acq, s))) return r;
+  } else {
+    if ((r = launch_mchvi(e->mean, e->var, B, e->N, m, e->lower, e->upper, e->K, 2 * n + 2, eps,
+                          e->S, (long long)m * e->S, e->acq, s)))
+      return r;
+  }
+  mark(ST_TOPK);
+  if ((r = launch_topk(e->acq, B, e->N, e->k, idx, val, e->scratch, s))) return r;
+  mark(ST_COUNT);
+  e->launches = (int)(launch_count() - l0);
+  return BOUTE_OK;
+}
+
+static int engine_args_ok(const boute_engine *e, const void *X, const void *Y, const void *ls,
+                          const void *s2, const void *noise, const void *ref, const void *Xc,
+                          const void *eps, const void *idx, const void *val) {
+  if (!e || !X || !Y || !ls || !s2 || !noise || !ref || !Xc || !idx || !val) return 0;
+  if (e->mode == BOUTE_ACQ_MC_HVI && !eps) return 0;
+  return 1;
+}
+
+int boute_engine_step_async(boute_engine *e, const double *X, const double *Y,
+                            const double *lengthscale, const double *outputscale,
+                            const double *noise, const double *ref, const float *Xc,
+                            const float *eps, long long *idx, float *val, void *stream) {
+  if (!engine_args_ok(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val))
+    return BOUTE_ERR_INVALID_ARG;
+  return engine_run(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val,
+                    (cudaStream_t)stream);
+}
+
+int boute_engine_step(boute_engine *e, const double *X, const double *Y,
+                      const double *lengthscale, const double *outputscale, const double *noise,
+                      const double *ref, const float *Xc, const float *eps, long long *idx,
+                      float *val, void *stream) {
+  int r = boute_engine_step_async(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx,
+                                  val, stream);
+  if (r) return r;
+  return boute_gp_status(e->gp, stream);
+}
+
+int boute_engine_step_host(boute_engine *e, const double *X, const double *Y,
+                           const double *lengthscale, const double *outputscale,
+                           const double *noise, const double *ref, const float *Xc,
+                           const float *eps, long long *idx, float *val, void *stream) {
+  if (!engine_args_ok(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val))
+    return BOUTE_ERR_INVALID_ARG;
+  cudaStream_t s = (cudaStream_t)stream;
+  const size_t B = e->B, n = e->n, d = e->d, m = e->m, N = e->N, S = e->S, k = e->k;
+  cudaMemcpyAsync(e->X, X, B * n * d * sizeof(double), cudaMemcpyHostToDevice, s);
+  cudaMemcpyAsync(e->Y, Y, B * n * m * sizeof(double), cudaMemcpyHostToDevice, s);
+  cudaMemcpyAsync(e->ls, lengthscale, B * m * d * sizeof(double), cudaMemcpyHostToDevice, s);
+  cudaMemcpyAsync(e->s2, outputscale, B * m * sizeof(double), cudaMemcpyHostToDevice, s);
+  cudaMemcpyAsync(e->noise, noise, B * m * sizeof(double), cudaMemcpyHostToDevice, s);
+  cudaMemcpyAsync(e->ref, ref, B * m * sizeof(double), cudaMemcpyHostToDevice, s);
+  cudaMemcpyAsync(e->Xc, Xc, B * N * d * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (e->mode == BOUTE_ACQ_MC_HVI)
+    cudaMemcpyAsync(e->eps, eps, B * N * m * S * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (int r = last_launch_status()) return r;
+  int r = engine_run(e, e->X, e->Y, e->ls, e->s2, e->noise, e->ref, e->Xc, e->eps, e->idx,
+                     e->val, s);
+  if (r) return r;
+  cudaMemcpyAsync(idx, e->idx, B * k * sizeof(long long), cudaMemcpyDeviceToHost, s);
+  cudaMemcpyAsync(val, e->val, B * k * sizeof(float), cudaMemcpyDeviceToHost, s);
+  if (int r2 = last_launch_status()) return r2;
+  return boute_gp_status(e->gp, stream);
+}
+
+int boute_engine_scores(const boute_engine *e, float *acq, float *mean, float *var,
+                        void *stream) {
+  if (!e) return BOUTE_ERR_INVALID_ARG;
+  cudaStream_t s = (cudaStream_t)stream;
+  const size_t BN = (size_t)e->B * e->N;
+  if (acq) cudaMemcpyAsync(acq, e->acq, BN * sizeof(float), cudaMemcpyDeviceToDevice, s);
+  if (mean) cudaMemcpyAsync(mean, e->mean, BN * e->m * sizeof(float), cudaMemcpyDeviceToDevice, s);
+  if (var) cudaMemcpyAsync(var, e->var, BN * e->m * sizeof(float), cudaMemcpyDeviceToDevice, s);
+  return last_launch_status();
+}
+
+int boute_engine_set_timing(boute_engine *e, int on) {
+  if (!e) return BOUTE_ERR_INVALID_ARG;
+  if (on && !e->timing) {
+    for (int i = 0; i <= ST_COUNT; ++i)
+      if (cudaEventCreate(&e->ev[i]) != cudaSuccess) return last_launch_status();
+    e->timing = 1;
+  }
+  return BOUTE_OK;
+}
+
+int boute_engine_stage_times(boute_engine *e, float *ms, int count) {
+  if (!e || !ms || count < ST_COUNT || !e->timing) return BOUTE_ERR_INVALID_ARG;
+  if (cudaEventSynchronize(e->ev[ST_COUNT]) != cudaSuccess) return last_launch_status();
+  for (int i = 0; i < ST_COUNT; ++i)
+    if (cudaEventElapsedTime(&ms[i], e->ev[i], e->ev[i + 1]) != cudaSuccess)
+      return last_launch_status();
+  return BOUTE_OK;
+}
+
+int boute_engine_launches_per_step(const boute_engine *e) { return e ? e->launches : 0; }
+
+}  // extern "C"

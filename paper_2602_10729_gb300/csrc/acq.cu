@@ -1,0 +1,188 @@
+// Acquisition kernels: closed-form 2-objective EHVI and Monte-Carlo
+// hypervolume improvement over the box decomposition of the front.
+#include <math.h>
+
+#include <algorithm>
+
+#include "internal.h"
+
+namespace boute {
+
+namespace {
+
+constexpr float kInvSqrt2Pi = 0.3989422804014327f;
+constexpr float kInvSqrt2 = 0.7071067811865476f;
+
+// Small part of psi: with z = (x - mu)/sigma, E[(x - Y)_+] = max(x - mu, 0) +
+// sigma * gm(z), gm(z) = phi(|z|) - |z| Phi(-|z|) >= 0 (the identity
+// G(z) = z + G(-z) for G(z) = z Phi(z) + phi(z)). Keeping the linear part
+// apart avoids cancellation for points far to either side of x.
+__device__ __forceinline__ float gm(float z) {
+  const float t = fabsf(z);
+  return expf(-0.5f * t * t) * kInvSqrt2Pi - t * (0.5f * erfcf(t * kInvSqrt2));
+}
+
+// ---- closed-form EHVI, m = 2 ---------------------------------------------------
+// Cells i = 0..P of the front sorted by f1: f1 in [a_i, b_i), f2 below u_i,
+// a_0 = -inf, b_P = r1, u_0 = r2. EHVI = sum_i [psi1(b_i) - psi1(a_i)] psi2(u_i).
+__global__ void __launch_bounds__(256) ehvi2d_kernel(const float *mean, const float *var,
+                                                     long long N, const double *front,
+                                                     const int *P, int n, const double *ref,
+                                                     float *acq) {
+  extern __shared__ float cells[];  // bnd[n+1] (b_i), up[n+1] (u_i)
+  const int b = blockIdx.y;
+  const int Pb = P[b];
+  float *bnd = cells, *up = cells + (n + 1);
+  const double *F = front + (size_t)b * n * 2;
+  const float r1 = (float)ref[2 * b], r2 = (float)ref[2 * b + 1];
+  for (int i = threadIdx.x; i <= Pb; i += blockDim.x) {
+    bnd[i] = i == Pb ? r1 : (float)F[2 * i];
+    up[i] = i == 0 ? r2 : (float)F[2 * (i - 1) + 1];
+  }
+  __syncthreads();
+  const float *m1 = mean + (size_t)b * 2 * N, *m2 = m1 + N;
+  const float *v1 = var + (size_t)b * 2 * N, *v2 = v1 + N;
+  for (long long c = (long long)blockIdx.x * blockDim.x + threadIdx.x; c < N;
+       c += (long long)gridDim.x * blockDim.x) {
+    const float mu1 = m1[c], mu2 = m2[c];
+    const float sg1 = sqrtf(fmaxf(v1[c], 0.f)), sg2 = sqrtf(fmaxf(v2[c], 0.f));
+    const float is1 = sg1 > 0.f ? 1.f / sg1 : 0.f, is2 = sg2 > 0.f ? 1.f / sg2 : 0.f;
+    float e = 0.f, ga = 0.f, a = -INFINITY;
+    for (int i = 0; i <= Pb; ++i) {
+      const float bb = bnd[i], u = up[i];
+      const float gb = sg1 > 0.f ? gm((bb - mu1) * is1) : 0.f;
+      const float lin = mu1 <= a ? bb - a : (mu1 <= bb ? bb - mu1 : 0.f);
+      const float D = fmaxf(fmaf(sg1, gb - ga, lin), 0.f);
+      const float g2 = sg2 > 0.f ? gm((u - mu2) * is2) : 0.f;
+      const float psi2 = fmaf(sg2, g2, fmaxf(u - mu2, 0.f));
+      e = fmaf(D, psi2, e);
+      ga = gb;
+      a = bb;
+    }
+    acq[(size_t)b * N + c] = e;
+  }
+}
+
+// ---- Monte-Carlo HVI: one warp per candidate, lanes over samples ---------------
+// Each sample's HVI is the volume of [y, ref] inside the disjoint boxes:
+// sum_k prod_t (u_kt - max(l_kt, y_t))_+.
+template <int M>
+__global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const float *var, int B,
+                                                    long long N, const float *lower,
+                                                    const float *upper, const int *Kc,
+                                                    int box_cap, const float *eps, int S,
+                                                    long long eps_stride, float *acq) {
+  extern __shared__ float boxes[];  // per problem in this block: lo[K][M], hi[K][M]
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
+  const int b = blockIdx.y;
+  const int K = Kc[b];
+  float *lo = boxes, *hi = boxes + (size_t)box_cap * M;
+  for (int i = threadIdx.x; i < K * M; i += blockDim.x) {
+    lo[i] = lower[(size_t)b * box_cap * M + i];
+    hi[i] = upper[(size_t)b * box_cap * M + i];
+  }
+  __syncthreads();
+  const float *mb = mean + (size_t)b * M * N, *vb = var + (size_t)b * M * N;
+  const bool vec = (S % 128) == 0 && ((uintptr_t)eps & 15) == 0 && (eps_stride % 4) == 0;
+  for (long long c = (long long)blockIdx.x * wpb + warp; c < N; c += (long long)gridDim.x * wpb) {
+    float mu[M], sg[M];
+#pragma unroll
+    for (int t = 0; t < M; ++t) {
+      mu[t] = mb[(size_t)t * N + c];
+      sg[t] = sqrtf(fmaxf(vb[(size_t)t * N + c], 0.f));
+    }
+    const float *e = eps + ((size_t)b * N + c) * eps_stride +
+                     (eps_stride == 0 ? (size_t)b * M * S : 0);
+    float sum = 0.f;
+    if (vec) {
+      for (int s0 = 4 * lane; s0 < S; s0 += 128) {
+        float4 z[M];
+#pragma unroll
+        for (int t = 0; t < M; ++t) z[t] = __ldcs((const float4 *)(e + (size_t)t * S + s0));
+        float y[4][M];
+#pragma unroll
+        for (int t = 0; t < M; ++t) {
+          y[0][t] = fmaf(sg[t], z[t].x, mu[t]);
+          y[1][t] = fmaf(sg[t], z[t].y, mu[t]);
+          y[2][t] = fmaf(sg[t], z[t].z, mu[t]);
+          y[3][t] = fmaf(sg[t], z[t].w, mu[t]);
+        }
+        for (int k = 0; k < K; ++k) {
+          float l[M], h[M];
+#pragma unroll
+          for (int t = 0; t < M; ++t) {
+            l[t] = lo[k * M + t];
+            h[t] = hi[k * M + t];
+          }
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            float v = fmaxf(h[0] - fmaxf(l[0], y[j][0]), 0.f);
+#pragma unroll
+            for (int t = 1; t < M; ++t) v *= fmaxf(h[t] - fmaxf(l[t], y[j][t]), 0.f);
+            sum += v;
+          }
+        }
+      }
+    } else {
+      for (int s = lane; s < S; s += 32) {
+        float y[M];
+#pragma unroll
+        for (int t = 0; t < M; ++t) y[t] = fmaf(sg[t], e[(size_t)t * S + s], mu[t]);
+        for (int k = 0; k < K; ++k) {
+          float v = fmaxf(hi[k * M] - fmaxf(lo[k * M], y[0]), 0.f);
+#pragma unroll
+          for (int t = 1; t < M; ++t) v *= fmaxf(hi[k * M + t] - fmaxf(lo[k * M + t], y[t]), 0.f);
+          sum += v;
+        }
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    if (lane == 0) acq[(size_t)b * N + c] = sum / (float)S;
+  }
+}
+
+}  // namespace
+
+int launch_ehvi(const float *mean, const float *var, int B, long long N, const double *front,
+                const int *P, int n, const double *ref, float *acq, cudaStream_t s) {
+  if (N <= 0) return BOUTE_OK;
+  int sms = 152;
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
+  const long long want = (N + 255) / 256;
+  const unsigned gx = (unsigned)std::max<long long>(1, std::min<long long>(want, (long long)sms * 8 / std::max(1, B) + 1));
+  ehvi2d_kernel<<<dim3(gx, B), 256, 2 * (n + 1) * sizeof(float), s>>>(mean, var, N, front, P, n,
+                                                                     ref, acq);
+  count_launch();
+  return last_launch_status();
+}
+
+int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
+                 const float *lower, const float *upper, const int *K, int box_cap,
+                 const float *eps, int S, long long eps_stride, float *acq, cudaStream_t s) {
+  if (N <= 0) return BOUTE_OK;
+  int sms = 152;
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
+  const int wpb = 16;
+  const long long want = (N + wpb - 1) / wpb;
+  const unsigned gx =
+      (unsigned)std::max<long long>(1, std::min<long long>(want, (long long)sms * 4 / std::max(1, B) + 1));
+  const size_t smem = 2 * (size_t)box_cap * m * sizeof(float);
+  if (smem > 48 * 1024) {
+    cudaFuncSetAttribute(mchvi_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaFuncSetAttribute(mchvi_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  }
+  if (m == 2) {
+    mchvi_kernel<2><<<dim3(gx, B), wpb * 32, smem, s>>>(mean, var, B, N, lower, upper, K, box_cap,
+                                                        eps, S, eps_stride, acq);
+  } else if (m == 3) {
+    mchvi_kernel<3><<<dim3(gx, B), wpb * 32, smem, s>>>(mean, var, B, N, lower, upper, K, box_cap,
+                                                        eps, S, eps_stride, acq);
+  } else {
+    return BOUTE_ERR_UNSUPPORTED;
+  }
+  count_launch();
+  return last_launch_status();
+}
+
+}  // namespace boute

@@ -1,0 +1,46 @@
+// Host-side declarations shared by the translation units of libboute.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+
+namespace boute {
+
+// The boute_gp handle: fp64 factors plus the prepacked tensor-core operands.
+struct Gp {
+  int B, n, d, m, DP;  // DP = d rounded up to a multiple of 4 (register tile)
+  PostPlan plan;
+  double *K;      // B*m x n x n: kernel matrix, overwritten by L (lower)
+  double *W;      // B*m x n x n: L^-1 (lower)
+  double *alpha;  // B*m x n
+  float *bop;     // B*m x plan.image_floats: [L^-1 ; alpha^T] as tf32 hi/lo images
+  float *xt;      // B*m x nchunk x 2 x 32 x DP: X / lengthscale as fp32 hi/lo
+  float *invls;   // B*m x 2 x DP: 1 / lengthscale as fp32 hi/lo
+  float *s2f;     // B*m: outputscale
+  int *status;    // device status word (first error wins)
+};
+
+void count_launch(int k = 1);
+unsigned long long launch_count();
+int last_launch_status();  // BOUTE_OK or BOUTE_ERR_CUDA after a launch
+
+int launch_standardize(const double *Y, int B, int n, int m, double *Ys, cudaStream_t s);
+int launch_fit(Gp *gp, const double *X, const double *Ys, const double *ls, const double *s2,
+               const double *noise, cudaStream_t s);
+int launch_posterior(const Gp *gp, const float *Xc, long long N, float *mean, float *var,
+                     cudaStream_t s);
+int launch_pareto(const double *Ys, int B, int n, int m, const double *ref, unsigned char *mask,
+                  double *front, int *P, cudaStream_t s);
+int launch_boxes(const double *front, const int *P, int B, int n, int m, const double *ref,
+                 float *lower, float *upper, int *K, cudaStream_t s);
+int launch_ehvi(const float *mean, const float *var, int B, long long N, const double *front,
+                const int *P, int n, const double *ref, float *acq, cudaStream_t s);
+int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
+                 const float *lower, const float *upper, const int *K, int box_cap,
+                 const float *eps, int S, long long eps_stride, float *acq, cudaStream_t s);
+size_t topk_scratch_bytes(int B, long long N, int k);
+int launch_topk(const float *acq, int B, long long N, int k, long long *idx, float *val,
+                void *scratch, cudaStream_t s);
+
+}  // namespace boute

@@ -1,0 +1,163 @@
+"""Test helpers: run the scoring step through the C-ABI one entry point at a
+time (so every intermediate can be compared), and the oracle on the same
+seeded inputs. The tolerances live here, with their derivation."""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import numpy as np
+
+import oracle
+from oracle import pipeline as opl
+from paper_2602_10729_gb300 import workloads as wl
+
+# ---- tolerances ----------------------------------------------------------------
+# Posterior (3xTF32 contraction, fp32 accumulate): relative 1e-5 against the
+# quantity's natural scale: |g - o| <= 1e-5 * max(|o|, s) for the mean (s is
+# the prior standard deviation), |g - o| <= 1e-5 * s2 for the variance, whose
+# fp32 value s2 - ||v||^2 carries an absolute rounding error of order eps32 * s2
+# whatever its size.
+POST_REL = 1e-5
+# Acquisition: relative 1e-4 against max(|o|, 1e-3 * max_j |o_j|), the largest
+# value of the problem setting the scale below which fp32 rounding of the
+# O(1) terms dominates.
+ACQ_REL = 1e-4
+ACQ_FLOOR = 1e-3
+
+
+def check_mean(g, o, s2, rel=POST_REL):
+    g, o = np.asarray(g, np.float64), np.asarray(o, np.float64)
+    s = np.sqrt(np.asarray(s2, np.float64))
+    err = np.abs(g - o) / np.maximum(np.abs(o), s)
+    assert np.all(np.isfinite(g)), "non-finite posterior mean"
+    assert err.max() <= rel, f"mean rel err {err.max():.3g} at {np.argmax(err)}"
+    return float(err.max())
+
+
+def check_var(g, o, s2, rel=POST_REL):
+    g, o = np.asarray(g, np.float64), np.asarray(o, np.float64)
+    err = np.abs(g - o) / np.asarray(s2, np.float64)
+    assert np.all(np.isfinite(g)) and np.all(g >= 0), "bad posterior variance"
+    assert err.max() <= rel, f"var rel err {err.max():.3g} at {np.argmax(err)}"
+    return float(err.max())
+
+
+def acq_err(g, o, scale=None):
+    g, o = np.asarray(g, np.float64), np.asarray(o, np.float64)
+    scale = np.abs(o).max() if scale is None else scale
+    return np.abs(g - o) / np.maximum(np.abs(o), ACQ_FLOOR * max(scale, 1e-300))
+
+
+def check_acq(g, o, rel=ACQ_REL, scale=None):
+    e = acq_err(g, o, scale)
+    assert np.all(np.isfinite(g)), "non-finite acquisition"
+    assert e.max() <= rel, f"acq rel err {e.max():.3g} at {np.argmax(e)} (g={g[np.argmax(e)]}, o={o[np.argmax(e)]})"
+    return float(e.max())
+
+
+def check_topk_consistent(idx_g, acq_o, k, tol_abs):
+    """End-to-end top-k: the GPU may differ from the oracle only among
+    candidates whose oracle values are within tol_abs of the k-th value."""
+    order = np.lexsort((np.arange(acq_o.size), -acq_o))
+    kth = acq_o[order[k - 1]]
+    sel = set(int(i) for i in idx_g)
+    must = {int(i) for i in order[:k] if acq_o[i] > kth + tol_abs}
+    assert must <= sel, f"missing clear winners {sorted(must - sel)[:5]}"
+    for i in sel:
+        assert acq_o[i] >= kth - tol_abs, f"selected {i} with oracle {acq_o[i]} < kth {kth}"
+
+
+# ---- workload on the host -------------------------------------------------------
+@dataclass
+class HostProblem:
+    w: wl.Workload
+    X: np.ndarray  # B x n x d
+    Y: np.ndarray  # B x n x m (raw)
+    ls: np.ndarray  # B x m x d
+    s2: np.ndarray  # B x m
+    noise: np.ndarray  # B x m
+    ref: np.ndarray  # B x m
+    Xc: np.ndarray  # B x N x d float32
+    eps: np.ndarray | None  # B x N x m x S float32
+
+
+def host_problem(w: wl.Workload, N: int | None = None, threads: int = 8) -> HostProblem:
+    N = w.N if N is None else N
+    Xs, Ys, L, S2, NZ = [], [], [], [], []
+    for b in range(w.B):
+        X, Y = wl.training_set(w, b)
+        ls, s2, nz = wl.hyperparameters(w, b)
+        Xs.append(X); Ys.append(Y); L.append(ls); S2.append(s2); NZ.append(nz)
+    Xc = np.stack([wl.candidates(w, b, 0, N, threads) for b in range(w.B)])
+    eps = None
+    if w.mode == "mc":
+        eps = np.stack([wl.base_normals(w, b, 0, N, threads) for b in range(w.B)])
+    ref = np.tile(wl.ref_point(w), (w.B, 1))
+    return HostProblem(w, np.stack(Xs), np.stack(Ys), np.stack(L), np.stack(S2), np.stack(NZ),
+                       ref, Xc, eps)
+
+
+def oracle_fit(hp: HostProblem, b: int) -> opl.FittedProblem:
+    return opl.fit_problem(hp.X[b], hp.Y[b], hp.ls[b], hp.s2[b], hp.noise[b], hp.ref[b])
+
+
+# ---- GPU: one ABI call at a time ------------------------------------------------
+def gpu_pipeline(hp: HostProblem, N: int | None = None, mean_var_in=None):
+    """Runs standardise -> fit -> front -> boxes -> posterior -> acq -> top-k
+    through the C-ABI and returns every intermediate on the host.
+    mean_var_in: optional (mean, var) B x m x N float32 fed to the
+    acquisition instead of the GPU posterior (isolated acquisition test)."""
+    import torch
+
+    from paper_2602_10729_gb300 import boute as bt
+    w = hp.w
+    B, n, d, m = w.B, w.n, w.d, w.m
+    N = hp.Xc.shape[1] if N is None else N
+    dev = torch.device("cuda")
+    t = lambda a, dt=None: torch.as_tensor(np.ascontiguousarray(a), device=dev, dtype=dt)
+    X, Y = t(hp.X, torch.float64), t(hp.Y, torch.float64)
+    ls, s2, nz, ref = (t(hp.ls, torch.float64), t(hp.s2, torch.float64),
+                       t(hp.noise, torch.float64), t(hp.ref, torch.float64))
+    Xc = t(hp.Xc[:, :N], torch.float32)
+    Ys = torch.empty_like(Y)
+    bt.boute_standardize(Y, Ys)
+    gp = bt.boute_gp_create(B, n, d, m)
+    bt.boute_gp_fit(gp, X, Ys, ls, s2, nz)
+    st = bt.boute_gp_status(gp)
+    mask = torch.empty((B, n), dtype=torch.uint8, device=dev)
+    front = torch.zeros((B, n, m), dtype=torch.float64, device=dev)
+    P = torch.empty(B, dtype=torch.int32, device=dev)
+    bt.boute_pareto_front(Ys, B, n, m, ref, mask, front, P)
+    mean = torch.empty((B, m, N), dtype=torch.float32, device=dev)
+    var = torch.empty_like(mean)
+    out = dict(status=st, Ys=Ys.cpu().numpy(), mask=mask.cpu().numpy().astype(bool),
+               front=front.cpu().numpy(), P=P.cpu().numpy())
+    if st != 0:
+        gp.free()
+        return out
+    bt.boute_gp_posterior(gp, Xc, N, mean, var)
+    if mean_var_in is not None:
+        mi, vi = (t(a, torch.float32) for a in mean_var_in)
+    else:
+        mi, vi = mean, var
+    acq = torch.empty((B, N), dtype=torch.float32, device=dev)
+    cap = 2 * n + 2
+    if w.mode == "ehvi":
+        bt.boute_acq_ehvi(mi, vi, B, N, front, P, n, ref, acq)
+    else:
+        lower = torch.empty((B, cap, m), dtype=torch.float32, device=dev)
+        upper = torch.empty_like(lower)
+        K = torch.empty(B, dtype=torch.int32, device=dev)
+        bt.boute_box_decompose(front, P, B, n, m, ref, lower, upper, K)
+        eps = t(hp.eps[:, :N], torch.float32)
+        bt.boute_acq_mc_hvi(mi, vi, B, N, m, lower, upper, K, cap, eps, w.S, m * w.S, acq)
+        out.update(lower=lower.cpu().numpy(), upper=upper.cpu().numpy(), K=K.cpu().numpy())
+    k = min(w.k, N)
+    idx = torch.empty((B, k), dtype=torch.int64, device=dev)
+    val = torch.empty((B, k), dtype=torch.float32, device=dev)
+    bt.boute_select_topk(acq, B, N, k, idx, val)
+    torch.cuda.synchronize()
+    out.update(mean=mean.cpu().numpy(), var=var.cpu().numpy(), acq=acq.cpu().numpy(),
+               idx=idx.cpu().numpy(), val=val.cpu().numpy(), status=bt.boute_gp_status(gp))
+    gp.free()
+    return out

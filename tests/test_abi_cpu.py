@@ -1,0 +1,72 @@
+"""Host-side checks of the C-ABI library (no GPU needed): it builds for
+sm_103a, loads, exports every entry point that include/boute.h declares,
+and rejects bad arguments before touching a device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2602_10729_gb300 import boute as bt
+from paper_2602_10729_gb300 import build as bld
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    bld.build()
+    return bt.load()
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "boute.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(boute_\w+)\s*\(", src)))
+
+
+def test_header_declares_the_binding_surface():
+    assert declared_functions() == sorted(bt.SYMBOLS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_library_targets_sm103a_only():
+    out = os.popen(f"/usr/local/cuda/bin/cuobjdump --list-elf {bld.LIB} 2>/dev/null").read()
+    archs = set(re.findall(r"sm_\d+a?", out))
+    assert archs == {"sm_103a"}, archs
+
+
+def test_status_strings(lib):
+    assert bt.status_string(0) == "ok"
+    assert "positive definite" in bt.status_string(2)
+    assert bt.status_string(99) == "unknown status"
+
+
+def test_invalid_arguments_are_rejected_before_any_device_call(lib):
+    h = ctypes.c_void_p()
+    assert lib.boute_gp_create(0, 4, 2, 1, ctypes.byref(h)) == bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_gp_create(1, 4, 33, 1, ctypes.byref(h)) == bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_gp_create(1, 4096, 2, 1, ctypes.byref(h)) == bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_gp_create(1, 4, 2, 1, None) == bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_select_topk(None, 1, 10, 3, None, None, None) == bt.BOUTE_ERR_INVALID_ARG
+    p = ctypes.c_void_p(16)
+    assert lib.boute_select_topk(p, 1, 10, 11, p, p, None) == bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_select_topk(p, 1, 10, 0, p, p, None) == bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_engine_create(1, 8, 2, 3, 100, bt.BOUTE_ACQ_EHVI2D, 0, 4,
+                                   ctypes.byref(h)) == bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_acq_mc_hvi(p, p, 1, 10, 4, p, p, p, 4, p, 8, 32, p, None) in (
+        bt.BOUTE_ERR_UNSUPPORTED, bt.BOUTE_ERR_INVALID_ARG)
+    assert lib.boute_gp_status(None, None) == bt.BOUTE_ERR_INVALID_ARG
+
+
+def test_valid_calls_without_a_device_report_unsupported(lib):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a device is present")
+    h = ctypes.c_void_p()
+    assert lib.boute_gp_create(1, 4, 2, 1, ctypes.byref(h)) == bt.BOUTE_ERR_UNSUPPORTED
+    assert not h.value

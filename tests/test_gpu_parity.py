@@ -1,0 +1,117 @@
+"""Parity of the CUDA path (through the C-ABI) with the CPU oracle, step by
+step and end to end, on the five workloads at sizes the oracle finishes in
+seconds (several 128-candidate tiles plus a ragged tail)."""
+import numpy as np
+import pytest
+
+import oracle
+from _pipeline import (ACQ_REL, check_acq, check_mean, check_topk_consistent, check_var,
+                       gpu_pipeline, host_problem, oracle_fit)
+from oracle import pipeline as opl
+from paper_2602_10729_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+# (workload index, N, B): N not a multiple of 128 to leave a ragged last tile
+SCALED = [(0, 4096 + 77, 1), (1, 3000 + 5, 1), (2, 2000 + 3, 1), (3, 700 + 11, 1), (4, 1500 + 1, 3)]
+
+
+@pytest.fixture(scope="module", params=SCALED, ids=lambda p: wl.WORKLOADS[p[0]].name)
+def case(request):
+    wi, N, B = request.param
+    w = wl.scaled(wl.WORKLOADS[wi], N=N, B=B)
+    hp = host_problem(w)
+    g = gpu_pipeline(hp)
+    fits = [oracle_fit(hp, b) for b in range(B)]
+    return w, hp, g, fits
+
+
+def test_fit_status_ok(case):
+    w, hp, g, fits = case
+    assert g["status"] == 0
+
+
+def test_standardize(case):
+    w, hp, g, fits = case
+    for b, fp in enumerate(fits):
+        np.testing.assert_allclose(g["Ys"][b], fp.Ys, rtol=1e-13, atol=1e-13)
+
+
+def test_pareto_front(case):
+    w, hp, g, fits = case
+    for b, fp in enumerate(fits):
+        assert g["mask"][b].tolist() == fp.mask.tolist()
+        P = int(g["P"][b])
+        assert P == fp.front.shape[0]
+        np.testing.assert_allclose(g["front"][b][:P], fp.front, rtol=0, atol=1e-13)
+
+
+def test_posterior(case):
+    w, hp, g, fits = case
+    for b, fp in enumerate(fits):
+        mean, var = opl.posterior(fp, hp.Xc[b])
+        for t in range(w.m):
+            check_mean(g["mean"][b, t], mean[:, t], fp.s2[t])
+            check_var(g["var"][b, t], var[:, t], fp.s2[t])
+
+
+def test_acquisition_end_to_end(case):
+    w, hp, g, fits = case
+    for b, fp in enumerate(fits):
+        mean, var = opl.posterior(fp, hp.Xc[b])
+        acq = opl.acquisition(fp, mean, var, w.mode, None if hp.eps is None else hp.eps[b])
+        check_acq(g["acq"][b], acq)
+
+
+def test_topk_end_to_end(case):
+    w, hp, g, fits = case
+    for b, fp in enumerate(fits):
+        mean, var = opl.posterior(fp, hp.Xc[b])
+        acq = opl.acquisition(fp, mean, var, w.mode, None if hp.eps is None else hp.eps[b])
+        k = min(w.k, acq.size)
+        tol = ACQ_REL * np.maximum(np.abs(acq), 1e-3 * np.abs(acq).max())
+        check_topk_consistent(g["idx"][b], acq, k, float(2 * tol.max()))
+        # values are the GPU's own acquisition at the returned indices, in order
+        assert np.array_equal(g["val"][b], g["acq"][b][g["idx"][b]])
+        assert np.all(np.diff(g["val"][b]) <= 0)
+
+
+def test_acquisition_isolated_on_oracle_posterior(case):
+    """The acquisition kernel alone: fed the oracle's posterior rounded to
+    fp32, against the oracle's acquisition of the same rounded values."""
+    w, hp, g, fits = case
+    N = hp.Xc.shape[1]
+    mi = np.empty((w.B, w.m, N), np.float32)
+    vi = np.empty_like(mi)
+    posts = []
+    for b, fp in enumerate(fits):
+        mean, var = opl.posterior(fp, hp.Xc[b])
+        mi[b], vi[b] = mean.T, var.T
+        posts.append((mi[b].T.astype(np.float64), vi[b].T.astype(np.float64)))
+    g2 = gpu_pipeline(hp, mean_var_in=(mi, vi))
+    for b, fp in enumerate(fits):
+        acq = opl.acquisition(fp, *posts[b], w.mode, None if hp.eps is None else hp.eps[b])
+        check_acq(g2["acq"][b], acq)
+
+
+def test_topk_bit_exact_on_oracle_values(case):
+    """Selection alone: the GPU top-k of the oracle's acquisition (as fp32)
+    equals the oracle's top-k of the same values, index for index."""
+    import torch
+
+    from paper_2602_10729_gb300 import boute as bt
+    w, hp, g, fits = case
+    N = hp.Xc.shape[1]
+    vals = np.empty((w.B, N), np.float32)
+    for b, fp in enumerate(fits):
+        mean, var = opl.posterior(fp, hp.Xc[b])
+        vals[b] = opl.acquisition(fp, mean, var, w.mode, None if hp.eps is None else hp.eps[b])
+    k = min(w.k, N)
+    a = torch.as_tensor(vals, device="cuda")
+    idx = torch.empty((w.B, k), dtype=torch.int64, device="cuda")
+    val = torch.empty((w.B, k), dtype=torch.float32, device="cuda")
+    bt.boute_select_topk(a, w.B, N, k, idx, val)
+    for b in range(w.B):
+        oi, ov = oracle.topk(vals[b].astype(np.float64), k)
+        assert idx[b].cpu().numpy().tolist() == oi.tolist()
+        assert np.array_equal(val[b].cpu().numpy(), ov.astype(np.float32))
