@@ -115,11 +115,13 @@ int boute_gp_create(int B, int n, int d, int m, boute_gp **out) {
   g.plan = make_post_plan(n);
   const size_t BM = (size_t)B * m;
   int r = BOUTE_OK;
-  r |= dalloc(&g.K, BM * n * n);
-  r |= dalloc(&g.W, BM * n * n);
-  r |= dalloc(&g.alpha, BM * n);
+  r |= dalloc(&g.Kh, BM * n * n);
+  r |= dalloc(&g.Kl, BM * n * n);
+  const size_t np = g.plan.npad;
+  r |= dalloc(&g.Aws, BM * np * (np + 1));
+  r |= dalloc(&g.Wws, BM * np * (np + 1));
   r |= dalloc(&g.bop, BM * (size_t)g.plan.image_floats);
-  r |= dalloc(&g.xt, BM * (size_t)g.plan.npad * 2 * g.DP);
+  r |= dalloc(&g.xt, BM * (size_t)g.plan.nchunk * xt_chunk_floats(g.DP));
   r |= dalloc(&g.invls, BM * 2 * g.DP);
   r |= dalloc(&g.s2f, BM);
   r |= dalloc(&g.status, 1);
@@ -154,7 +156,7 @@ int boute_gp_status(boute_gp *gp, void *stream) {
 void boute_gp_free(boute_gp *gp) {
   if (!gp) return;
   Gp &g = gp->g;
-  cudaFree(g.K); cudaFree(g.W); cudaFree(g.alpha); cudaFree(g.bop); cudaFree(g.xt);
+  cudaFree(g.Kh); cudaFree(g.Kl); cudaFree(g.Aws); cudaFree(g.Wws); cudaFree(g.bop); cudaFree(g.xt);
   cudaFree(g.invls); cudaFree(g.s2f); cudaFree(g.status);
   delete gp;
 }

@@ -7,7 +7,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include "../../include/boute.h"
+#include "boute.h"
 
 #define BOUTE_MAX_D 32       // candidate dimension limit (registers per thread)
 #define BOUTE_MAX_M 4        // objectives per problem
@@ -21,10 +21,11 @@ namespace boute {
 
 // ---------------------------------------------------------------- host/device
 // Operand-image plan of the posterior contraction for one (problem, objective):
-// output columns [0, n) are the rows of L^-1, column n is alpha, the rest pad
-// to a multiple of 16. Columns are processed in passes of at most 256 (one
+// output columns [0, n) are the rows of L^-1, padded with zero rows to a
+// multiple of 16. Columns are processed in passes of at most 256 (one
 // tcgen05.mma N); pass p needs the reduction chunks [0, kc[p]) only, because
-// row j of L^-1 is zero beyond column j.
+// row j of L^-1 is zero beyond column j. (The mean K* alpha is reduced on the
+// CUDA cores while K* is built, in compensated fp32.)
 struct PostPlan {
   int n, npad, ncols, npass, nchunk;
   int col0[BOUTE_MAX_PASS], ncol[BOUTE_MAX_PASS], kc[BOUTE_MAX_PASS];
@@ -34,21 +35,24 @@ struct PostPlan {
 
 inline __host__ __device__ int round_up(int x, int r) { return (x + r - 1) / r * r; }
 
+// Floats of one training-point chunk of the posterior's side input: X/ls as
+// fp32 hi [32][DP], lo [32][DP], then alpha [32].
+inline __host__ __device__ int xt_chunk_floats(int DP) { return 2 * BOUTE_KCHUNK * DP + BOUTE_KCHUNK; }
+
 inline PostPlan make_post_plan(int n) {
   PostPlan p{};
   p.n = n;
   p.npad = round_up(n, BOUTE_KCHUNK);
   p.nchunk = p.npad / BOUTE_KCHUNK;
-  p.ncols = round_up(n + 1, 16);
+  p.ncols = round_up(n, 16);
   p.npass = (p.ncols + 255) / 256;
   long long off = 0;
   for (int q = 0; q < p.npass; ++q) {
     p.col0[q] = 256 * q;
     p.ncol[q] = (p.ncols - p.col0[q]) < 256 ? (p.ncols - p.col0[q]) : 256;
-    int last_col = p.col0[q] + p.ncol[q] - 1;
-    // the pass holding alpha (column n) needs every chunk
-    int need = (last_col >= n) ? p.npad : round_up(last_col + 1, BOUTE_KCHUNK);
-    p.kc[q] = need / BOUTE_KCHUNK;
+    const int last_col = p.col0[q] + p.ncol[q] - 1;
+    const int need = round_up(last_col + 1, BOUTE_KCHUNK);
+    p.kc[q] = (need < p.npad ? need : p.npad) / BOUTE_KCHUNK;
     p.off[q] = off;
     off += (long long)p.kc[q] * 2 * p.ncol[q] * BOUTE_KCHUNK;
   }

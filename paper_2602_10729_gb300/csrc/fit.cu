@@ -50,23 +50,32 @@ __global__ void standardize_kernel(const double *Y, int n, int m, double *Ys) {
   for (int i = threadIdx.x; i < n; i += blockDim.x) ys[(size_t)i * m] = (y[(size_t)i * m] - mean) / sd;
 }
 
-// ---- K = s2 M52(X, X) + noise I, per (problem, objective) --------------------
+// ---- K = s2 M52(X, X) + noise I (full, symmetric), per (problem, objective) ----
+// fp64 arithmetic, stored as an fp32 pair (hi = K rounded, lo = K - hi): the
+// factorisation works on hi, the refinement of alpha on hi + lo.
 __global__ void kernel_matrix_kernel(const double *X, int n, int d, int m, const double *ls,
-                                     const double *s2, const double *noise, double *Kall) {
+                                     const double *s2, const double *noise, float *Kh_all,
+                                     float *Kl_all) {
+  __shared__ double il[BOUTE_MAX_D];
   const int bt = blockIdx.z, b = bt / m;
-  const int i = blockIdx.y * 16 + threadIdx.y, j = blockIdx.x * 16 + threadIdx.x;
+  for (int t = threadIdx.y * blockDim.x + threadIdx.x; t < d; t += blockDim.x * blockDim.y)
+    il[t] = 1.0 / ls[(size_t)bt * d + t];
+  __syncthreads();
+  const int i = blockIdx.y * blockDim.y + threadIdx.y, j = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n || j >= n) return;
   const double *xi = X + ((size_t)b * n + i) * d, *xj = X + ((size_t)b * n + j) * d;
-  const double *l = ls + (size_t)bt * d;
   double r2 = 0.0;
   for (int t = 0; t < d; ++t) {
-    double z = (xi[t] - xj[t]) / l[t];
-    r2 += z * z;
+    const double z = (xi[t] - xj[t]) * il[t];
+    r2 = fma(z, z, r2);
   }
   const double r = sqrt(r2), sr = sqrt(5.0) * r;
   double k = s2[bt] * (1.0 + sr + 5.0 * r2 / 3.0) * exp(-sr);
   if (i == j) k += noise[bt];
-  Kall[(size_t)bt * n * n + (size_t)i * n + j] = k;
+  const float kh = (float)k;
+  const size_t o = (size_t)bt * n * n + (size_t)i * n + j;
+  Kh_all[o] = kh;
+  Kl_all[o] = (float)(k - (double)kh);
 }
 
 // ---- scaled training inputs, 1/lengthscale and outputscale in fp32 -----------
@@ -75,14 +84,15 @@ __global__ void prep_kernel(const double *X, int n, int d, int m, int DP, int np
                             float *s2f) {
   const int bt = blockIdx.y, b = bt / m;
   const double *l = ls + (size_t)bt * d;
-  float *x = xt + (size_t)bt * npad * 2 * DP;
+  const int cf = xt_chunk_floats(DP);
+  float *x = xt + (size_t)bt * (npad / BOUTE_KCHUNK) * cf;
   const int total = npad * DP;
   for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < total; e += gridDim.x * blockDim.x) {
     const int j = e / DP, t = e % DP;
     double v = (j < n && t < d) ? X[((size_t)b * n + j) * d + t] / l[t] : 0.0;
     float hi = (float)v, lo = (float)(v - (double)hi);
     const int c = j / BOUTE_KCHUNK, jj = j % BOUTE_KCHUNK;
-    float *blk = x + (size_t)c * 2 * BOUTE_KCHUNK * DP;
+    float *blk = x + (size_t)c * cf;
     blk[jj * DP + t] = hi;
     blk[BOUTE_KCHUNK * DP + jj * DP + t] = lo;
   }
@@ -97,47 +107,155 @@ __global__ void prep_kernel(const double *X, int n, int d, int m, int DP, int np
   }
 }
 
-// ---- right-looking Cholesky, one block per (problem, objective) --------------
-// Column j: pivot sqrt, scale the column below it, rank-1 update of the
-// trailing lower triangle (warp per row, lanes along the row). The matrix
-// lives in shared memory when it fits, else in global memory (L2-resident).
+// Error-free product and sum on fp32 pairs (Dekker / Knuth).
+__device__ __forceinline__ void two_prod(float a, float b, float &p, float &e) {
+  p = a * b;
+  e = fmaf(a, b, -p);
+}
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
+  s = a + b;
+  const float bb = s - a;
+  e = (a - (s - bb)) + (b - bb);
+}
+
+// ---- factorisation: one block per (problem, objective) -------------------------
+// Blocked right-looking Cholesky of K (its fp32 rounding) in 32-column panels:
+// one warp factors each diagonal block in registers, then the block forms the
+// panel below it (row-parallel forward substitution) and the trailing update
+// (4 x 4 register tiles). The diagonal blocks of W = L^-1 are inverted
+// afterwards, one warp each, concurrently, and W is completed block
+// row by block row, W_IJ = -W_II sum_{K=J}^{I-1} L_IK W_KJ. fp32 arithmetic on
+// the FP32 pipes: the fp32 factor is as accurate as the posterior needs, while
+// alpha, which carries the condition number, gets one step of iterative
+// refinement against the fp64-accurate K = hi + lo with double-float
+// residuals. A pivot at or below 16 * eps32 times its original diagonal entry
+// counts as not positive. Matrix and inverse live in shared memory (row stride
+// NP+1, NP = n rounded up to 32, padded with the identity) when they fit, else
+// in the handle's global workspace.
 template <bool SMEM>
-__global__ void __launch_bounds__(512) chol_kernel(double *Kall, int n, int *status) {
-  extern __shared__ double sm[];
+__global__ void __launch_bounds__(256, 1) fit32_kernel(const float *Kh_all, const float *Kl_all,
+                                                    const double *Ys, int n, int m, float *Aws,
+                                                    float *Wws, float *xt, int DP, int npad,
+                                                    int *status) {
+  extern __shared__ float sm[];
   __shared__ int bad;
-  __shared__ double piv;
-  double *G = Kall + (size_t)blockIdx.x * n * n;
-  double *A = SMEM ? sm : G;
-  double *col = SMEM ? sm + (size_t)n * n : sm;
+  const int bt = blockIdx.x, b = bt / m, t = bt % m;
   const int tid = threadIdx.x, nthr = blockDim.x, lane = tid & 31, warp = tid >> 5,
             nw = nthr >> 5;
-  if (SMEM)
-    for (int e = tid; e < n * n; e += nthr) A[e] = G[e];
+  const int NP = npad, ld = NP + 1;
+  const float *Kh = Kh_all + (size_t)bt * n * n, *Kl = Kl_all + (size_t)bt * n * n;
+  float *A = SMEM ? sm : Aws + (size_t)bt * NP * ld;
+  float *W = SMEM ? sm + (size_t)NP * ld : Wws + (size_t)bt * NP * ld;
+  float *vec = SMEM ? sm + 2 * (size_t)NP * ld : sm;  // col, dg, y, tv, al, r: 6 x NP
+  float *dg = vec + NP, *yv = vec + 2 * NP, *tv = vec + 3 * NP, *al = vec + 4 * NP,
+        *rv = vec + 5 * NP;
+  const double *y = Ys + (size_t)b * n * m + t;
+
+  for (int e = tid; e < NP * ld; e += nthr) {
+    const int i = e / ld, k = e % ld;
+    float v = 0.f;
+    if (k <= i && k < NP) v = (i < n) ? Kh[(size_t)i * n + k] : (i == k ? 1.f : 0.f);
+    A[e] = v;
+    W[e] = 0.f;
+  }
+  for (int i = tid; i < NP; i += nthr) {
+    yv[i] = i < n ? (float)y[(size_t)i * m] : 0.f;
+    dg[i] = i < n ? Kh[(size_t)i * n + i] : 1.f;
+  }
   if (tid == 0) bad = 0;
   __syncthreads();
-  for (int j = 0; j < n; ++j) {
-    if (tid == 0) {
-      double p = A[(size_t)j * n + j];
-      if (!(p > 0.0)) {
-        bad = 1;
-      } else {
-        p = sqrt(p);
-        A[(size_t)j * n + j] = p;
-        piv = p;
+  // ---- blocked Cholesky, 32-column panels --------------------------------------
+  const int nb = NP / 32;
+  const unsigned FULL = 0xffffffffu;
+  for (int p = 0; p < nb; ++p) {
+    const int p0 = 32 * p;
+    // (a) one warp factors the diagonal block, register-resident (lane = row):
+    //     at step c, column c of L is formed and broadcast by shuffles to
+    //     update the trailing rows of the block.
+    if (warp == 0) {
+      float a[32];
+      float *Ar = A + (size_t)(p0 + lane) * ld + p0;
+#pragma unroll
+      for (int c = 0; c < 32; ++c) a[c] = (c <= lane) ? Ar[c] : 0.f;
+      const float dgl = dg[p0 + lane];
+      bool ok = true;
+#pragma unroll
+      for (int c = 0; c < 32; ++c) {
+        const float piv = __shfl_sync(FULL, a[c], c);
+        if (!(piv > 16.f * 1.1920929e-7f * __shfl_sync(FULL, dgl, c))) ok = false;
+        float inv = rsqrtf(piv);
+        inv = inv * fmaf(-0.5f * piv * inv, inv, 1.5f);  // one Newton step
+        const float l = lane > c ? a[c] * inv : (lane == c ? piv * inv : 0.f);
+        a[c] = l;
+#pragma unroll
+        for (int c2 = 0; c2 < 32; ++c2) {
+          if (c2 > c) {
+            const float lc2 = __shfl_sync(FULL, l, c2);
+            if (lane >= c2) a[c2] = fmaf(-l, lc2, a[c2]);
+          }
+        }
       }
+      if (!ok && lane == 0) bad = 1;
+#pragma unroll
+      for (int c = 0; c < 32; ++c)
+        if (c <= lane) Ar[c] = a[c];
     }
     __syncthreads();
     if (bad) break;
-    for (int i = j + 1 + tid; i < n; i += nthr) {
-      double v = A[(size_t)i * n + j] / piv;
-      A[(size_t)i * n + j] = v;
-      col[i] = v;
+    const int r0 = p0 + 32, rows = NP - r0;
+    const float *Lp = A + (size_t)p0 * ld + p0;  // L_pp, lower
+    {
+      // (b) panel below the diagonal block: row r solves x L_pp^T = A_r,p
+      //     by forward substitution (x in registers), one row per thread
+      for (int r = r0 + tid; r < NP; r += nthr) {
+        float *ar = A + (size_t)r * ld + p0;
+        float x[32];
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          float s0 = ar[c], s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+          for (int q = 0; q < 32; q += 4) {
+            if (q < c) s0 = fmaf(-x[q], Lp[(size_t)c * ld + q], s0);
+            if (q + 1 < c) s1 = fmaf(-x[q + 1], Lp[(size_t)c * ld + q + 1], s1);
+            if (q + 2 < c) s2 = fmaf(-x[q + 2], Lp[(size_t)c * ld + q + 2], s2);
+            if (q + 3 < c) s3 = fmaf(-x[q + 3], Lp[(size_t)c * ld + q + 3], s3);
+          }
+          x[c] = ((s0 + s1) + (s2 + s3)) / Lp[(size_t)c * ld + c];
+        }
+#pragma unroll
+        for (int c = 0; c < 32; ++c) ar[c] = x[c];
+      }
     }
     __syncthreads();
-    for (int i = j + 1 + warp; i < n; i += nw) {
-      const double li = col[i];
-      double *row = A + (size_t)i * n;
-      for (int k = j + 1 + lane; k <= i; k += 32) row[k] -= li * col[k];
+    // (c) trailing update of the lower triangle, 4 x 4 register tiles:
+    //     A_ij -= sum_q L_i,p0+q L_j,p0+q for r0 <= j <= i < NP
+    const int th = rows / 4;
+    const int ntile = th * (th + 1) / 2;
+    for (int tix = tid; tix < ntile; tix += nthr) {
+      int ti = (int)((sqrtf(8.f * tix + 1.f) - 1.f) * 0.5f);
+      while (ti * (ti + 1) / 2 > tix) --ti;
+      while ((ti + 1) * (ti + 2) / 2 <= tix) ++ti;
+      const int tj = tix - ti * (ti + 1) / 2;
+      const int i0 = r0 + 4 * ti, j0 = r0 + 4 * tj;
+      float acc[4][4] = {};
+#pragma unroll 4
+      for (int q = 0; q < 32; ++q) {
+        float x[4], y4[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          x[u] = A[(size_t)(i0 + u) * ld + p0 + q];
+          y4[u] = A[(size_t)(j0 + u) * ld + p0 + q];
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v)
+          if (ti != tj || v <= u) A[(size_t)(i0 + u) * ld + j0 + v] -= acc[u][v];
     }
     __syncthreads();
   }
@@ -145,67 +263,173 @@ __global__ void __launch_bounds__(512) chol_kernel(double *Kall, int n, int *sta
     if (tid == 0) set_status(status, BOUTE_ERR_NOT_PD);
     return;
   }
-  for (int e = tid; e < n * n; e += nthr) {
-    const int i = e / n, k = e % n;
-    G[e] = k <= i ? A[e] : 0.0;
-  }
-}
-
-// ---- W = L^-1: one warp per column, forward substitution on e_j --------------
-__global__ void trinv_kernel(const double *Lall, double *Wall, int n, const int *status) {
-  extern __shared__ double wsm[];
-  if (*status == BOUTE_ERR_NOT_PD) return;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
-  const int j = blockIdx.x * wpb + warp;
-  const size_t bt = blockIdx.y;
-  if (j >= n) return;
-  const double *L = Lall + bt * n * n;
-  double *W = Wall + bt * n * n;
-  double *w = wsm + (size_t)warp * n;
-  if (lane == 0) w[j] = 1.0 / L[(size_t)j * n + j];
-  __syncwarp();
-  for (int i = j + 1; i < n; ++i) {
-    const double *Li = L + (size_t)i * n;
-    double s = 0.0;
-    for (int k = j + lane; k < i; k += 32) s += Li[k] * w[k];
-    s = warp_sum(s);
-    if (lane == 0) w[i] = -s / Li[i];
-    __syncwarp();
-  }
-  for (int i = lane; i < n; i += 32) W[(size_t)i * n + j] = i >= j ? w[i] : 0.0;
-}
-
-// ---- alpha = W^T (W y) ------------------------------------------------------------
-__global__ void alpha_kernel(const double *Wall, const double *Ys, int n, int m,
-                             double *alpha_all, const int *status) {
-  extern __shared__ double tv[];
-  if (*status == BOUTE_ERR_NOT_PD) return;
-  const int bt = blockIdx.x, b = bt / m, t = bt % m;
-  const double *W = Wall + (size_t)bt * n * n;
-  const double *y = Ys + (size_t)b * n * m + t;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  for (int i = warp; i < n; i += nw) {
-    double s = 0.0;
-    for (int k = lane; k <= i; k += 32) s += W[(size_t)i * n + k] * y[(size_t)k * m];
-    s = warp_sum(s);
-    if (lane == 0) tv[i] = s;
+  // ---- diagonal blocks of W = L^-1: warp I inverts L_II (lane = column) --------
+  for (int I = warp; I < nb; I += nw) {
+    const float *Lb = A + (size_t)(32 * I) * ld + 32 * I;
+    float w[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      float s0 = (i == lane) ? 1.f : 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+      for (int l = 0; l < 32; l += 4) {
+        if (l < i) s0 = fmaf(-Lb[(size_t)i * ld + l], w[l], s0);
+        if (l + 1 < i) s1 = fmaf(-Lb[(size_t)i * ld + l + 1], w[l + 1], s1);
+        if (l + 2 < i) s2 = fmaf(-Lb[(size_t)i * ld + l + 2], w[l + 2], s2);
+        if (l + 3 < i) s3 = fmaf(-Lb[(size_t)i * ld + l + 3], w[l + 3], s3);
+      }
+      w[i] = ((s0 + s1) + (s2 + s3)) / Lb[(size_t)i * ld + i];
+    }
+    float *Wb = W + (size_t)(32 * I) * ld + 32 * I;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) Wb[(size_t)i * ld + lane] = w[i];
   }
   __syncthreads();
-  for (int k = threadIdx.x; k < n; k += blockDim.x) {
-    double s = 0.0;
-    for (int i = k; i < n; ++i) s += W[(size_t)i * n + k] * tv[i];
-    alpha_all[(size_t)bt * n + k] = s;
+  // ---- off-diagonal blocks of W = L^-1, block row by block row ------------------
+  // W_IJ = -W_II T_IJ, T_IJ = sum_{K=J}^{I-1} L_IK W_KJ; T is parked, transposed,
+  // in the (unused) upper triangle of W. 4 x 4 register tiles.
+  for (int I = 1; I < nb; ++I) {
+    const int nt = I * 64;  // J < I, 8 x 8 tiles per block
+    for (int tix = tid; tix < nt; tix += nthr) {
+      const int J = tix / 64, rb = 4 * ((tix / 8) % 8), cb = 4 * (tix % 8);
+      float acc[4][4] = {};
+#pragma unroll 4
+      for (int q = 32 * J; q < 32 * I; ++q) {
+        float x[4], y4[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          x[u] = A[(size_t)(32 * I + rb + u) * ld + q];
+          y4[u] = W[(size_t)q * ld + 32 * J + cb + u];
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v)
+          W[(size_t)(32 * J + cb + v) * ld + 32 * I + rb + u] = acc[u][v];
+    }
+    __syncthreads();
+    for (int tix = tid; tix < nt; tix += nthr) {
+      const int J = tix / 64, rb = 4 * ((tix / 8) % 8), cb = 4 * (tix % 8);
+      float acc[4][4] = {};
+#pragma unroll 4
+      for (int q = 0; q < 32; ++q) {  // W_II is lower triangular: zeros above
+        float x[4], y4[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          x[u] = W[(size_t)(32 * I + rb + u) * ld + 32 * I + q];
+          y4[u] = W[(size_t)(32 * J + cb + u) * ld + 32 * I + q];
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) W[(size_t)(32 * I + rb + u) * ld + 32 * J + cb + v] = -acc[u][v];
+    }
+    __syncthreads();
   }
+  // ---- alpha0 = W^T (W y), refined once against K = hi + lo ----------------------
+  // out = W^T (W rhs): thread per row, then thread per column (4 accumulators)
+  auto solve = [&](const float *rhs, float *out) {
+    for (int i = tid; i < NP; i += nthr) {
+      const float *wr = W + (size_t)i * ld;
+      float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+      int k = 0;
+      for (; k + 3 <= i; k += 4) {
+        s0 = fmaf(wr[k], rhs[k], s0);
+        s1 = fmaf(wr[k + 1], rhs[k + 1], s1);
+        s2 = fmaf(wr[k + 2], rhs[k + 2], s2);
+        s3 = fmaf(wr[k + 3], rhs[k + 3], s3);
+      }
+      for (; k <= i; ++k) s0 = fmaf(wr[k], rhs[k], s0);
+      tv[i] = (s0 + s1) + (s2 + s3);
+    }
+    __syncthreads();
+    for (int k = tid; k < NP; k += nthr) {
+      float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+      int i = k;
+      for (; i + 3 < NP; i += 4) {
+        s0 = fmaf(W[(size_t)i * ld + k], tv[i], s0);
+        s1 = fmaf(W[(size_t)(i + 1) * ld + k], tv[i + 1], s1);
+        s2 = fmaf(W[(size_t)(i + 2) * ld + k], tv[i + 2], s2);
+        s3 = fmaf(W[(size_t)(i + 3) * ld + k], tv[i + 3], s3);
+      }
+      for (; i < NP; ++i) s0 = fmaf(W[(size_t)i * ld + k], tv[i], s0);
+      out[k] = (s0 + s1) + (s2 + s3);
+    }
+    __syncthreads();
+  };
+  solve(yv, al);
+  // residual r = y - K alpha0 in double-float: half a warp per row, all the
+  // row's loads issued before the arithmetic
+  {
+    const int half = lane >> 4, hl = lane & 15;
+    for (int i = 2 * warp + half; i < NP; i += 2 * nw) {
+      float sh = 0.f, sl = 0.f;
+      if (i < n) {
+        const float *kh = Kh + (size_t)i * n, *kl = Kl + (size_t)i * n;
+        for (int k0 = 0; k0 < n; k0 += 128) {
+          float h8[8], l8[8], a8[8];
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int k = k0 + hl + 16 * u;
+            h8[u] = k < n ? kh[k] : 0.f;
+            l8[u] = k < n ? kl[k] : 0.f;
+            a8[u] = k < n ? al[k] : 0.f;
+          }
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            float pr, e, s_, e2;
+            two_prod(h8[u], a8[u], pr, e);
+            two_sum(sh, pr, s_, e2);
+            sh = s_;
+            sl += e2 + fmaf(l8[u], a8[u], e);
+          }
+        }
+      }
+#pragma unroll
+      for (int o = 8; o > 0; o >>= 1) {  // within the half warp
+        const float oh = __shfl_xor_sync(FULL, sh, o);
+        const float ol = __shfl_xor_sync(FULL, sl, o);
+        float s_, e;
+        two_sum(sh, oh, s_, e);
+        sh = s_;
+        sl += ol + e;
+      }
+      if (hl == 0 && i < n) {
+        const double yi = y[(size_t)i * m];
+        const float yh = (float)yi, yl = (float)(yi - (double)yh);
+        rv[i] = (yh - sh) + (yl - sl);
+      }
+    }
+  }
+  for (int i = n + tid; i < NP; i += nthr) rv[i] = 0.f;
+  __syncthreads();
+  solve(rv, rv);
+  for (int k = tid; k < NP; k += nthr) al[k] += rv[k];
+  __syncthreads();
+  // outputs: W (row stride ld) for the operand packing, alpha into the side input
+  if (SMEM)
+    for (int e = tid; e < NP * ld; e += nthr) Wws[(size_t)bt * NP * ld + e] = W[e];
+  const int cf = xt_chunk_floats(DP);
+  float *xa = xt + (size_t)bt * (npad / BOUTE_KCHUNK) * cf + 2 * BOUTE_KCHUNK * DP;
+  for (int k = tid; k < npad; k += nthr)
+    xa[(size_t)(k / BOUTE_KCHUNK) * cf + k % BOUTE_KCHUNK] = k < n ? al[k] : 0.f;
 }
 
-// ---- operand images [L^-1 ; alpha^T] as tf32 hi/lo, swizzled -----------------
-__global__ void pack_kernel(const double *Wall, const double *alpha_all, PostPlan plan,
-                            float *bop, const int *status) {
+// ---- operand images of L^-1 as tf32 hi/lo, swizzled ---------------------------
+__global__ void pack_kernel(const float *Wws, PostPlan plan, float *bop, const int *status) {
   if (*status == BOUTE_ERR_NOT_PD) return;
   const size_t bt = blockIdx.y;
-  const int n = plan.n;
-  const double *W = Wall + bt * n * n;
-  const double *al = alpha_all + bt * n;
+  const int n = plan.n, ld = plan.npad + 1;
+  const float *W = Wws + bt * plan.npad * ld;
   float *img = bop + bt * plan.image_floats;
   const long long total = (long long)plan.ncols * plan.npad;
   for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < total;
@@ -213,13 +437,9 @@ __global__ void pack_kernel(const double *Wall, const double *alpha_all, PostPla
     const int g = (int)(e / plan.npad), k = (int)(e % plan.npad);
     const int p = g >> 8, c = k / BOUTE_KCHUNK;
     if (c >= plan.kc[p]) continue;
-    double v = 0.0;
-    if (k < n) {
-      if (g < n) v = k <= g ? W[(size_t)g * n + k] : 0.0;
-      else if (g == n) v = al[k];
-    }
-    const float hi = tf32_rna((float)v);
-    const float lo = tf32_rna((float)(v - (double)hi));
+    const float v = (k < n && g < n && k <= g) ? W[(size_t)g * ld + k] : 0.f;
+    const float hi = tf32_rna(v);
+    const float lo = tf32_rna(v - hi);
     const int ncol = plan.ncol[p];
     float *blk = img + plan.off[p] + (long long)c * 2 * ncol * BOUTE_KCHUNK;
     const int o = sw128_off(g - plan.col0[p], k % BOUTE_KCHUNK);
@@ -236,32 +456,30 @@ int launch_standardize(const double *Y, int B, int n, int m, double *Ys, cudaStr
   return last_launch_status();
 }
 
+size_t fit_smem_bytes(int np) { return (2 * (size_t)np * (np + 1) + 6 * (size_t)np) * sizeof(float); }
+
 int launch_fit(Gp *gp, const double *X, const double *Ys, const double *ls, const double *s2,
                const double *noise, cudaStream_t s) {
   const int n = gp->n, d = gp->d, m = gp->m, BM = gp->B * gp->m;
   cudaMemsetAsync(gp->status, 0, sizeof(int), s);  // a new fit starts with a clean status
-  dim3 g1((n + 15) / 16, (n + 15) / 16, BM);
-  kernel_matrix_kernel<<<g1, dim3(16, 16), 0, s>>>(X, n, d, m, ls, s2, noise, gp->K);
+  dim3 g1((n + 7) / 8, (n + 7) / 8, BM);
+  kernel_matrix_kernel<<<g1, dim3(8, 8), 0, s>>>(X, n, d, m, ls, s2, noise, gp->Kh, gp->Kl);
   prep_kernel<<<dim3(std::max(1, gp->plan.npad * gp->DP / 256), BM), 256, 0, s>>>(
       X, n, d, m, gp->DP, gp->plan.npad, ls, s2, gp->xt, gp->invls, gp->s2f);
-  const size_t smem_chol = ((size_t)n * n + n) * sizeof(double);
-  if (smem_chol <= 200 * 1024) {
-    cudaFuncSetAttribute(chol_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         (int)smem_chol);
-    chol_kernel<true><<<BM, 512, smem_chol, s>>>(gp->K, n, gp->status);
+  const size_t smem = fit_smem_bytes(gp->plan.npad);
+  if (smem <= 220 * 1024) {
+    cudaFuncSetAttribute(fit32_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)smem);
+    fit32_kernel<true><<<BM, 256, smem, s>>>(gp->Kh, gp->Kl, Ys, n, m, gp->Aws, gp->Wws, gp->xt,
+                                             gp->DP, gp->plan.npad, gp->status);
   } else {
-    chol_kernel<false><<<BM, 512, n * sizeof(double), s>>>(gp->K, n, gp->status);
+    fit32_kernel<false><<<BM, 256, 6 * gp->plan.npad * sizeof(float), s>>>(
+        gp->Kh, gp->Kl, Ys, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, gp->plan.npad, gp->status);
   }
-  const int wpb = 8;
-  const size_t smem_inv = (size_t)wpb * n * sizeof(double);
-  cudaFuncSetAttribute(trinv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_inv);
-  trinv_kernel<<<dim3((n + wpb - 1) / wpb, BM), wpb * 32, smem_inv, s>>>(gp->K, gp->W, n,
-                                                                          gp->status);
-  alpha_kernel<<<BM, 256, n * sizeof(double), s>>>(gp->W, Ys, n, m, gp->alpha, gp->status);
   const long long tot = (long long)gp->plan.ncols * gp->plan.npad;
   pack_kernel<<<dim3((unsigned)std::min<long long>((tot + 255) / 256, 4096), BM), 256, 0, s>>>(
-      gp->W, gp->alpha, gp->plan, gp->bop, gp->status);
-  count_launch(6);
+      gp->Wws, gp->plan, gp->bop, gp->status);
+  count_launch(4);
   return last_launch_status();
 }
 

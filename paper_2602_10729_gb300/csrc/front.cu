@@ -9,8 +9,17 @@ namespace boute {
 
 namespace {
 
+// Order-preserving integer image of a double (-0 taken as +0): x < y exactly
+// when key(x) < key(y), for finite values. Comparing keys keeps the O(n^2)
+// dominance tests on the integer pipes instead of the slow fp64 unit.
+__device__ __forceinline__ long long dkey(double x) {
+  if (x == 0.0) x = 0.0;
+  const long long b = __double_as_longlong(x);
+  return b >= 0 ? b : (long long)(b ^ 0x7FFFFFFFFFFFFFFFll);
+}
+
 // a dominates b (minimisation): <= everywhere, < somewhere
-__device__ __forceinline__ bool dominates(const double *a, const double *b, int m) {
+__device__ __forceinline__ bool dominates(const long long *a, const long long *b, int m) {
   bool lt = false;
   for (int t = 0; t < m; ++t) {
     if (a[t] > b[t]) return false;
@@ -19,14 +28,15 @@ __device__ __forceinline__ bool dominates(const double *a, const double *b, int 
   return lt;
 }
 
-__device__ __forceinline__ bool equal(const double *a, const double *b, int m) {
+__device__ __forceinline__ bool equal(const long long *a, const long long *b, int m) {
   for (int t = 0; t < m; ++t)
     if (a[t] != b[t]) return false;
   return true;
 }
 
 // (Y_j, j) < (Y_i, i) lexicographically
-__device__ __forceinline__ bool lex_less(const double *yj, int j, const double *yi, int i, int m) {
+__device__ __forceinline__ bool lex_less(const long long *yj, int j, const long long *yi, int i,
+                                         int m) {
   for (int t = 0; t < m; ++t) {
     if (yj[t] < yi[t]) return true;
     if (yj[t] > yi[t]) return false;
@@ -36,23 +46,24 @@ __device__ __forceinline__ bool lex_less(const double *yj, int j, const double *
 
 __global__ void pareto_kernel(const double *Ys, int n, int m, const double *ref,
                               unsigned char *mask, double *front, int *P) {
-  extern __shared__ double y[];  // n*m outcomes, then n keep flags (as int)
-  int *keep = (int *)(y + (size_t)n * m);
+  extern __shared__ long long yk[];  // n*m keys, then n keep flags (as int)
+  int *keep = (int *)(yk + (size_t)n * m);
   __shared__ int count;
+  __shared__ long long rk[BOUTE_MAX_M];
   const int b = blockIdx.x;
   const double *Yb = Ys + (size_t)b * n * m;
-  const double *rb = ref + (size_t)b * m;
-  for (int e = threadIdx.x; e < n * m; e += blockDim.x) y[e] = Yb[e];
+  for (int e = threadIdx.x; e < n * m; e += blockDim.x) yk[e] = dkey(Yb[e]);
+  if (threadIdx.x < m) rk[threadIdx.x] = dkey(ref[(size_t)b * m + threadIdx.x]);
   if (threadIdx.x == 0) count = 0;
   __syncthreads();
   for (int i = threadIdx.x; i < n; i += blockDim.x) {
-    const double *yi = y + (size_t)i * m;
+    const long long *yi = yk + (size_t)i * m;
     bool k = true;
     for (int t = 0; t < m; ++t)
-      if (!(yi[t] < rb[t])) k = false;
+      if (!(yi[t] < rk[t])) k = false;
     for (int j = 0; j < n && k; ++j) {
       if (j == i) continue;
-      const double *yj = y + (size_t)j * m;
+      const long long *yj = yk + (size_t)j * m;
       if (dominates(yj, yi, m) || (j < i && equal(yj, yi, m))) k = false;
     }
     keep[i] = k;
@@ -62,12 +73,12 @@ __global__ void pareto_kernel(const double *Ys, int n, int m, const double *ref,
   __syncthreads();
   for (int i = threadIdx.x; i < n; i += blockDim.x) {
     if (!keep[i]) continue;
-    const double *yi = y + (size_t)i * m;
+    const long long *yi = yk + (size_t)i * m;
     int rank = 0;
     for (int j = 0; j < n; ++j)
-      if (keep[j] && lex_less(y + (size_t)j * m, j, yi, i, m)) ++rank;
+      if (keep[j] && lex_less(yk + (size_t)j * m, j, yi, i, m)) ++rank;
     double *dst = front + ((size_t)b * n + rank) * m;
-    for (int t = 0; t < m; ++t) dst[t] = yi[t];
+    for (int t = 0; t < m; ++t) dst[t] = Yb[(size_t)i * m + t];
   }
   if (threadIdx.x == 0) P[b] = count;
 }
@@ -164,7 +175,7 @@ __global__ void boxes_kernel(const double *front, const int *P, int n, int m, co
 
 int launch_pareto(const double *Ys, int B, int n, int m, const double *ref, unsigned char *mask,
                   double *front, int *P, cudaStream_t s) {
-  const size_t smem = (size_t)n * m * sizeof(double) + (size_t)n * sizeof(int);
+  const size_t smem = (size_t)n * m * sizeof(long long) + (size_t)n * sizeof(int);
   if (smem > 48 * 1024)
     cudaFuncSetAttribute(pareto_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   pareto_kernel<<<B, 512, smem, s>>>(Ys, n, m, ref, mask, front, P);

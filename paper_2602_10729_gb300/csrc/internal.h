@@ -11,11 +11,11 @@ namespace boute {
 struct Gp {
   int B, n, d, m, DP;  // DP = d rounded up to a multiple of 4 (register tile)
   PostPlan plan;
-  double *K;      // B*m x n x n: kernel matrix, overwritten by L (lower)
-  double *W;      // B*m x n x n: L^-1 (lower)
-  double *alpha;  // B*m x n
-  float *bop;     // B*m x plan.image_floats: [L^-1 ; alpha^T] as tf32 hi/lo images
-  float *xt;      // B*m x nchunk x 2 x 32 x DP: X / lengthscale as fp32 hi/lo
+  float *Kh, *Kl;  // B*m x n x n: kernel matrix (lower) as an fp32 pair hi + lo
+  float *Aws;      // B*m x np x (np+1): factorisation workspace (large n; np = npad)
+  float *Wws;      // B*m x np x (np+1): L^-1 (lower, row stride np+1)
+  float *bop;     // B*m x plan.image_floats: L^-1 as tf32 hi/lo operand images
+  float *xt;      // B*m x nchunk x xt_chunk_floats(DP): X/lengthscale hi/lo, alpha
   float *invls;   // B*m x 2 x DP: 1 / lengthscale as fp32 hi/lo
   float *s2f;     // B*m: outputscale
   int *status;    // device status word (first error wins)

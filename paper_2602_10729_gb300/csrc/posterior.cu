@@ -4,11 +4,14 @@
 // cross-covariance K* (128 x n) is built chunk by chunk (32 training points =
 // 128 B rows) straight into shared memory in the swizzled K-major operand
 // layout, split into tf32 hi/lo parts, and contracted against the prepacked
-// operand [L^-1 ; alpha^T] (hi/lo, brought in by bulk TMA copies) with three
+// operand L^-1 (hi/lo, brought in by bulk TMA copies) with three
 // tcgen05.mma kind::tf32 per k-step (hi*hi + hi*lo + lo*hi, fp32 accumulate in
 // tensor memory). The epilogue reads the 128 x ncol accumulator back with
-// tcgen05.ld and reduces it to mean (alpha column) and variance
-// (s2 - sum of squares of the L^-1 columns). K* never reaches HBM.
+// tcgen05.ld and reduces it to the variance s2 - rowsum(V^2). The mean K* alpha
+// is a matrix-vector product: the threads building K* reduce it on the CUDA
+// cores in fp32 with compensated (Kahan) accumulation across chunks, which is
+// more accurate than the tensor core's fp32 accumulation and takes no
+// operand column. K* never reaches HBM.
 //
 // Pipeline: two shared-memory stages. While the tensor core runs chunk q-1,
 // the 256 threads build chunk q and the TMA engine fetches chunk q+1's
@@ -64,6 +67,7 @@ __global__ void __launch_bounds__(256, 1) posterior_kernel(const __grid_constant
   auto b_reg = [&](int s) { return stage(s) + 32768; };
   const int ncolmax = pl.ncol[0];
   auto xt_reg = [&](int s) { return (float *)(stage(s) + 32768 + 2 * ncolmax * 128); };
+  const int cf = xt_chunk_floats(DP);
 
   if (tid == 0) {
     for (int i = 0; i < 7; ++i) mbar_init(&bars[i], 1);
@@ -109,14 +113,13 @@ __global__ void __launch_bounds__(256, 1) posterior_kernel(const __grid_constant
   auto issue = [&](int t, int p, int c, int s) {
     const int bt = b * m + t;
     const uint32_t bbytes = (uint32_t)(2 * pl.ncol[p] * 128);
-    const uint32_t xtb = (uint32_t)(2 * BOUTE_KCHUNK * DP * 4);
+    const uint32_t xtb = (uint32_t)(cf * 4);
     mbar_arrive_expect_tx(&full[s], bbytes + xtb);
     bulk_g2s(b_reg(s),
              a.bop + (size_t)bt * pl.image_floats + pl.off[p] +
                  (size_t)c * 2 * pl.ncol[p] * BOUTE_KCHUNK,
              bbytes, &full[s]);
-    bulk_g2s(xt_reg(s), a.xt + ((size_t)bt * pl.npad + (size_t)c * BOUTE_KCHUNK) * 2 * DP, xtb,
-             &full[s]);
+    bulk_g2s(xt_reg(s), a.xt + ((size_t)bt * pl.nchunk + c) * cf, xtb, &full[s]);
   };
   auto next_job = [&](int &t, int &p, int &c) {
     if (++c == pl.kc[p]) {
@@ -138,7 +141,7 @@ __global__ void __launch_bounds__(256, 1) posterior_kernel(const __grid_constant
   int t = 0, p = 0, c = 0;
   int pass_count = 0;
   float xs[DP];
-  float s2 = 0.f, ss_acc = 0.f, mu_acc = 0.f;
+  float s2 = 0.f, ss_acc = 0.f, mu_acc = 0.f, mu_comp = 0.f;
   bool mma_issued = false;
 
   for (int q = 0; q < total; ++q) {
@@ -167,12 +170,15 @@ __global__ void __launch_bounds__(256, 1) posterior_kernel(const __grid_constant
       s2 = a.s2f[bt];
       ss_acc = 0.f;
       mu_acc = 0.f;
+      mu_comp = 0.f;
     }
     // build K* chunk c: this thread's row, 16 columns [16*half, 16*half+16)
     {
       const float *xth = xt_reg(s), *xtl = xth + BOUTE_KCHUNK * DP;
+      const float *alp = xth + 2 * BOUTE_KCHUNK * DP;
       float *Ah = a_hi(s), *Al = a_lo(s);
       const int jbase = c * BOUTE_KCHUNK;
+      float mu_part = 0.f;
 #pragma unroll
       for (int g4 = 0; g4 < 4; ++g4) {
         float vh[4], vl[4];
@@ -195,6 +201,7 @@ __global__ void __launch_bounds__(256, 1) posterior_kernel(const __grid_constant
           const float sr = kSqrt5 * r;
           float kv = s2 * fmaf(kFiveThirds, acc, 1.0f + sr) * expf(-sr);
           kv = (jbase + kk < n) ? kv : 0.f;
+          mu_part = fmaf(kv, alp[kk], mu_part);  // used in the last pass only
           const float hi = tf32_rna(kv);
           vh[e] = hi;
           vl[e] = kv - hi;
@@ -202,6 +209,14 @@ __global__ void __launch_bounds__(256, 1) posterior_kernel(const __grid_constant
         const int o = sw128_off(row, half * 16 + g4 * 4);
         *(float4 *)(Ah + o) = make_float4(vh[0], vh[1], vh[2], vh[3]);
         *(float4 *)(Al + o) = make_float4(vl[0], vl[1], vl[2], vl[3]);
+      }
+      // Kahan: mu_acc += mu_part, once per chunk: the last pass builds every
+      // chunk, earlier passes rebuild a prefix of them
+      if (p == pl.npass - 1) {
+        const float yk = mu_part - mu_comp;
+        const float tk = mu_acc + yk;
+        mu_comp = (tk - mu_acc) - yk;
+        mu_acc = tk;
       }
     }
     // (4) publish the chunk to the tensor core
@@ -237,16 +252,11 @@ __global__ void __launch_bounds__(256, 1) posterior_kernel(const __grid_constant
       const int gq = warp & 3, hsel = warp >> 2;
       const int hcols = ncol >> 1;
       const uint32_t tbase = tmem + ((uint32_t)(32 * gq) << 16) + (uint32_t)(hsel * hcols);
-      const int cbase = pl.col0[p] + hsel * hcols;
       for (int cc = 0; cc < hcols; cc += 8) {
         float v[8];
         tmem_ld8(tbase + cc, v);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const int gcol = cbase + cc + e;
-          if (gcol < n) ss_acc = fmaf(v[e], v[e], ss_acc);
-          else if (gcol == n) mu_acc = v[e];
-        }
+        for (int e = 0; e < 8; ++e) ss_acc = fmaf(v[e], v[e], ss_acc);  // zero beyond n
       }
       tc_fence_before();
       __syncthreads();
@@ -254,7 +264,7 @@ __global__ void __launch_bounds__(256, 1) posterior_kernel(const __grid_constant
       if (p == pl.npass - 1) {  // objective complete
         const int r2 = 32 * gq + lane;
         red_ss[hsel * 128 + r2] = ss_acc;
-        red_mu[hsel * 128 + r2] = mu_acc;
+        red_mu[half * 128 + row] = mu_acc - mu_comp;
         __syncthreads();
         if (half == 0) {
           const long long gr = tile0 + row;
@@ -306,7 +316,7 @@ int launch_dp(const Gp *gp, const float *Xc, long long N, float *mean, float *va
   a.n = gp->n;
   a.plan = gp->plan;
   const int ncolmax = gp->plan.ncol[0];
-  a.stage_bytes = (uint32_t)round_up(32768 + 2 * ncolmax * 128 + 2 * BOUTE_KCHUNK * DP * 4, 1024);
+  a.stage_bytes = (uint32_t)round_up(32768 + 2 * ncolmax * 128 + xt_chunk_floats(DP) * 4, 1024);
   const size_t smem = 1024 + 2 * (size_t)a.stage_bytes + 8 * 8 + 2 * 256 * 4;
   cudaFuncSetAttribute(posterior_kernel<DP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        (int)smem);

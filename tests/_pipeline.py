@@ -55,6 +55,43 @@ def check_acq(g, o, rel=ACQ_REL, scale=None):
     return float(e.max())
 
 
+def acq_sensitivity(fn, mean, var, s2):
+    """First-order change of the oracle acquisition fn(mean, var) (N x m each)
+    when every posterior input moves by its tolerance: the part of an
+    end-to-end acquisition difference the posterior tolerance accounts for."""
+    base = fn(mean, var)
+    s2 = np.asarray(s2, np.float64)
+    tot = np.zeros_like(base)
+    for t in range(mean.shape[1]):
+        dm = POST_REL * np.maximum(np.abs(mean[:, t]), np.sqrt(s2[t]))
+        dv = POST_REL * s2[t]
+        worst_m = np.zeros_like(base)
+        worst_v = np.zeros_like(base)
+        for sign in (1.0, -1.0):
+            mm = mean.copy()
+            mm[:, t] += sign * dm
+            worst_m = np.maximum(worst_m, np.abs(fn(mm, var) - base))
+            vv = var.copy()
+            vv[:, t] = np.maximum(vv[:, t] + sign * dv, 0.0)
+            worst_v = np.maximum(worst_v, np.abs(fn(mean, vv) - base))
+        tot += worst_m + worst_v
+    return base, tot
+
+
+def check_acq_end_to_end(g_acq, fn, mean_g, var_g, mean_o, var_o, s2):
+    """(1) the acquisition kernel's own error: GPU acquisition against the
+    oracle acquisition of the GPU posterior; (2) against the oracle's own
+    acquisition, allowing for the posterior tolerance (acq_sensitivity)."""
+    a_at_g = fn(np.asarray(mean_g, np.float64), np.asarray(var_g, np.float64))
+    e1 = check_acq(g_acq, a_at_g)
+    o, sens = acq_sensitivity(fn, mean_o, var_o, s2)
+    scale = np.abs(o).max()
+    tol = ACQ_REL * np.maximum(np.abs(o), ACQ_FLOOR * scale) + 2 * sens
+    err = np.abs(np.asarray(g_acq, np.float64) - o)
+    assert np.all(err <= tol), f"acq e2e err {err.max():.3g} > tol at {np.argmax(err - tol)}"
+    return e1, o, tol
+
+
 def check_topk_consistent(idx_g, acq_o, k, tol_abs):
     """End-to-end top-k: the GPU may differ from the oracle only among
     candidates whose oracle values are within tol_abs of the k-th value."""
@@ -65,6 +102,17 @@ def check_topk_consistent(idx_g, acq_o, k, tol_abs):
     assert must <= sel, f"missing clear winners {sorted(must - sel)[:5]}"
     for i in sel:
         assert acq_o[i] >= kth - tol_abs, f"selected {i} with oracle {acq_o[i]} < kth {kth}"
+
+
+def check_topk_consistent_tol(idx_g, acq_o, k, tol):
+    """As check_topk_consistent with a per-candidate tolerance array."""
+    order = np.lexsort((np.arange(acq_o.size), -acq_o))
+    kth = acq_o[order[k - 1]]
+    sel = set(int(i) for i in idx_g)
+    must = {int(i) for i in order[:k] if acq_o[i] - tol[i] > kth + tol[order[k - 1]]}
+    assert must <= sel, f"missing clear winners {sorted(must - sel)[:5]}"
+    for i in sel:
+        assert acq_o[i] + tol[i] >= kth - tol[order[k - 1]], f"selected {i} below the k-th"
 
 
 # ---- workload on the host -------------------------------------------------------

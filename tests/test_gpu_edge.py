@@ -7,7 +7,8 @@ import numpy as np
 import pytest
 
 import oracle
-from _pipeline import (HostProblem, check_acq, check_mean, check_var, gpu_pipeline)
+from _pipeline import (HostProblem, check_acq, check_acq_end_to_end, check_mean, check_var,
+                       gpu_pipeline)
 from oracle import pipeline as opl
 from paper_2602_10729_gb300 import workloads as wl
 
@@ -43,8 +44,9 @@ def compare(hp, check_topk=True):
         for t in range(w.m):
             check_mean(g["mean"][b, t], mean[:, t], fp.s2[t])
             check_var(g["var"][b, t], var[:, t], fp.s2[t])
-        acq = opl.acquisition(fp, mean, var, w.mode, None if hp.eps is None else hp.eps[b])
-        check_acq(g["acq"][b], acq)
+        eps = None if hp.eps is None else hp.eps[b]
+        check_acq_end_to_end(g["acq"][b], lambda mm, vv: opl.acquisition(fp, mm, vv, w.mode, eps),
+                             g["mean"][b].T, g["var"][b].T, mean, var, fp.s2)
     return g
 
 
@@ -70,7 +72,33 @@ def test_training_set_sizes_and_column_passes(n):
 
 @pytest.mark.parametrize("d", [1, 3, 8, 9, 13, 17, 25, 32])
 def test_dimensions(d):
-    compare(rand_problem(3, 40, d, 2, 300))
+    # lengthscale 0.2 sqrt(d) as in the workloads; 1-D with few points keeps
+    # the kernel matrix well conditioned (see the ill-conditioned test below)
+    n, ls = (6, 0.1) if d == 1 else (40, 0.2 * np.sqrt(d))
+    compare(rand_problem(3, n, d, 2, 300, ls=ls))
+
+
+def test_ill_conditioned_problem_meets_fp32_error_bound():
+    """40 points on a line with lengthscale 0.3: cond(K) ~ 2e5, |alpha| ~ 1e3.
+    The fp32-accurate path cannot give 1e-5 relative there; it must stay
+    within the error bound of fp32 dot products, a small multiple of
+    eps32 * sum_j |K*_j alpha_j| for the mean (and of eps32 * s2 * cond-scaled
+    terms for the variance)."""
+    hp = rand_problem(12, 40, 1, 2, 300)
+    g = gpu_pipeline(hp)
+    assert g["status"] == 0
+    fp = opl.fit_problem(hp.X[0], hp.Y[0], hp.ls[0], hp.s2[0], hp.noise[0], hp.ref[0])
+    mean, var = opl.posterior(fp, hp.Xc[0])
+    eps32 = np.finfo(np.float32).eps
+    for t in range(2):
+        Ks = np.array([[oracle.matern52(c.astype(np.float64), x, hp.ls[0][t], hp.s2[0][t])
+                        for x in hp.X[0]] for c in hp.Xc[0]])
+        bound_mu = 64 * eps32 * (np.abs(Ks) @ np.abs(fp.alpha[t])) + 1e-5
+        assert np.all(np.abs(g["mean"][0, t] - mean[:, t]) <= bound_mu)
+        W = np.linalg.inv(fp.L[t])
+        v = Ks @ W.T
+        bound_v = 64 * eps32 * 2 * (np.abs(v) * (np.abs(Ks) @ np.abs(W.T))).sum(1) + 1e-5
+        assert np.all(np.abs(g["var"][0, t] - var[:, t]) <= bound_v)
 
 
 def test_three_objectives_monte_carlo_and_box_decomposition():

@@ -5,8 +5,8 @@ import numpy as np
 import pytest
 
 import oracle
-from _pipeline import (ACQ_REL, check_acq, check_mean, check_topk_consistent, check_var,
-                       gpu_pipeline, host_problem, oracle_fit)
+from _pipeline import (check_acq, check_acq_end_to_end, check_mean, check_topk_consistent_tol,
+                       check_var, gpu_pipeline, host_problem, oracle_fit)
 from oracle import pipeline as opl
 from paper_2602_10729_gb300 import workloads as wl
 
@@ -55,22 +55,27 @@ def test_posterior(case):
             check_var(g["var"][b, t], var[:, t], fp.s2[t])
 
 
+def _acq_fn(w, hp, fp, b):
+    eps = None if hp.eps is None else hp.eps[b]
+    return lambda mean, var: opl.acquisition(fp, mean, var, w.mode, eps)
+
+
 def test_acquisition_end_to_end(case):
     w, hp, g, fits = case
     for b, fp in enumerate(fits):
         mean, var = opl.posterior(fp, hp.Xc[b])
-        acq = opl.acquisition(fp, mean, var, w.mode, None if hp.eps is None else hp.eps[b])
-        check_acq(g["acq"][b], acq)
+        check_acq_end_to_end(g["acq"][b], _acq_fn(w, hp, fp, b), g["mean"][b].T, g["var"][b].T,
+                             mean, var, fp.s2)
 
 
 def test_topk_end_to_end(case):
     w, hp, g, fits = case
     for b, fp in enumerate(fits):
         mean, var = opl.posterior(fp, hp.Xc[b])
-        acq = opl.acquisition(fp, mean, var, w.mode, None if hp.eps is None else hp.eps[b])
+        _, acq, tol = check_acq_end_to_end(g["acq"][b], _acq_fn(w, hp, fp, b), g["mean"][b].T,
+                                           g["var"][b].T, mean, var, fp.s2)
         k = min(w.k, acq.size)
-        tol = ACQ_REL * np.maximum(np.abs(acq), 1e-3 * np.abs(acq).max())
-        check_topk_consistent(g["idx"][b], acq, k, float(2 * tol.max()))
+        check_topk_consistent_tol(g["idx"][b], acq, k, tol)
         # values are the GPU's own acquisition at the returned indices, in order
         assert np.array_equal(g["val"][b], g["acq"][b][g["idx"][b]])
         assert np.all(np.diff(g["val"][b]) <= 0)
