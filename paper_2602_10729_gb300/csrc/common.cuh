@@ -36,7 +36,8 @@ struct PostPlan {
 inline __host__ __device__ int round_up(int x, int r) { return (x + r - 1) / r * r; }
 
 // Floats of one training-point chunk of the posterior's side input: X/ls as
-// fp32 hi [32][DP], lo [32][DP], then alpha [32].
+// fp32 hi [DP][32] and lo [DP][32] (dimension-major, so pairs of training
+// points load as packed f32x2), then alpha [32].
 inline __host__ __device__ int xt_chunk_floats(int DP) { return 2 * BOUTE_KCHUNK * DP + BOUTE_KCHUNK; }
 
 inline PostPlan make_post_plan(int n) {
@@ -92,6 +93,11 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t by
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
                "r"(bytes)
                : "memory");
+}
+
+// One plain arrival (release semantics at CTA scope for the calling thread).
+__device__ __forceinline__ void mbar_arrive_count(uint64_t *bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
 __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t phase) {

@@ -92,9 +92,9 @@ __global__ void prep_kernel(const double *X, int n, int d, int m, int DP, int np
     double v = (j < n && t < d) ? X[((size_t)b * n + j) * d + t] / l[t] : 0.0;
     float hi = (float)v, lo = (float)(v - (double)hi);
     const int c = j / BOUTE_KCHUNK, jj = j % BOUTE_KCHUNK;
-    float *blk = x + (size_t)c * cf;
-    blk[jj * DP + t] = hi;
-    blk[BOUTE_KCHUNK * DP + jj * DP + t] = lo;
+    float *blk = x + (size_t)c * cf;  // dimension-major: [DP][32] hi, [DP][32] lo
+    blk[t * BOUTE_KCHUNK + jj] = hi;
+    blk[BOUTE_KCHUNK * DP + t * BOUTE_KCHUNK + jj] = lo;
   }
   if (blockIdx.x == 0) {
     for (int t = threadIdx.x; t < DP; t += blockDim.x) {

@@ -6,18 +6,24 @@
 // layout, split into tf32 hi/lo parts, and contracted against the prepacked
 // operand L^-1 (hi/lo, brought in by bulk TMA copies) with three
 // tcgen05.mma kind::tf32 per k-step (hi*hi + hi*lo + lo*hi, fp32 accumulate in
-// tensor memory). The epilogue reads the 128 x ncol accumulator back with
-// tcgen05.ld and reduces it to the variance s2 - rowsum(V^2). The mean K* alpha
-// is a matrix-vector product: the threads building K* reduce it on the CUDA
-// cores in fp32 with compensated (Kahan) accumulation across chunks, which is
-// more accurate than the tensor core's fp32 accumulation and takes no
-// operand column. K* never reaches HBM.
+// tensor memory). The variance is s2 - rowsum(V^2), V = K* L^-T, read back
+// from tensor memory with tcgen05.ld. The mean K* alpha is a matrix-vector
+// product: the threads building K* reduce it on the CUDA cores in fp32 with
+// compensated (Kahan) accumulation across chunks, which is more accurate than
+// the tensor core's fp32 accumulation and takes no operand column. K* never
+// reaches HBM.
 //
-// Pipeline: two shared-memory stages. While the tensor core runs chunk q-1,
-// the 256 threads build chunk q and the TMA engine fetches chunk q+1's
-// operand image. Output columns beyond 256 are handled in passes (TMEM holds
-// the 128 x 256 fp32 accumulator); pass p skips the reduction chunks where its
-// rows of L^-1 are zero.
+// Persistent and warp-specialised: each CTA loops over (problem, tile) pairs.
+//   warp 0      bulk-TMA producer (operand images and training-point chunks)
+//   warp 1      tcgen05.mma issuer; owns the 512-column TMEM allocation
+//   warps 4-7   epilogue: one TMEM lane quarter each, sum of squares, variance
+//   warps 8-15  K* builders: 16 rows x 2 halves per warp, packed f32x2 math
+// A ring of S shared-memory stages carries (A hi/lo, B hi/lo, side input);
+// the accumulator is double-buffered in TMEM (2 x 256 columns) so the
+// epilogue of one output pass overlaps the MMAs of the next. Output columns
+// beyond 256 are handled in passes; pass p skips the reduction chunks where
+// its rows of L^-1 are zero. All waits are bounded (BOUTE_WAIT_NS): a wait
+// that gives up records BOUTE_ERR_TIMEOUT and every role stops.
 #include <math.h>
 
 #include <algorithm>
@@ -28,13 +34,21 @@ namespace boute {
 
 namespace {
 
+constexpr int kThreads = 512;
+constexpr int kEpiWarp0 = 4;
+constexpr int kBldWarp0 = 8;
+constexpr int kBldWarps = 8;
+constexpr int kEpiWarps = 4;
+constexpr int kMaxStages = 4;
+
 struct PostArgs {
   const float *Xc;
   float *mean, *var;
   const float *bop, *xt, *invls, *s2f;
   int *status;
   long long N;
-  int m, d, n;
+  int B, m, d, n;
+  int tiles_per_problem, tiles_total, stages;
   uint32_t stage_bytes;
   PostPlan plan;
 };
@@ -42,40 +56,101 @@ struct PostArgs {
 constexpr float kSqrt5 = 2.2360679774997896964f;
 constexpr float kFiveThirds = 1.6666666666666667f;
 
+// ---- packed fp32 pairs (sm_100+ f32x2 arithmetic) --------------------------------
+__device__ __forceinline__ unsigned long long f2_dup(float x) {
+  unsigned long long r;
+  asm("mov.b64 %0, {%1, %1};" : "=l"(r) : "f"(x));
+  return r;
+}
+__device__ __forceinline__ unsigned long long f2_sub(unsigned long long a, unsigned long long b) {
+  unsigned long long r;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ unsigned long long f2_fma(unsigned long long a, unsigned long long b,
+                                                     unsigned long long c) {
+  unsigned long long r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+__device__ __forceinline__ void f2_split(unsigned long long v, float &x, float &y) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(x), "=f"(y) : "l"(v));
+}
+
+// 32 lanes x 32 bit, 16 consecutive columns per thread, wait fused.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
+                 "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
+                 "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15])::"memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Bounded wait that also gives up as soon as another role has aborted.
+__device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity,
+                                              volatile int *abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 63) == 0) {
+      if (*abort) return false;
+      if (globaltimer() - t0 > BOUTE_WAIT_NS) {
+        *abort = 1;
+        return false;
+      }
+    }
+  }
+}
+
 template <int DP>
-__global__ void __launch_bounds__(256, 1) posterior_kernel(const __grid_constant__ PostArgs a) {
+__global__ void __launch_bounds__(kThreads, 1)
+    posterior_kernel(const __grid_constant__ PostArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t *sm = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int row = tid & 127, half = tid >> 7;
-  const int b = blockIdx.y;
-  const long long tile0 = (long long)blockIdx.x * BOUTE_TILE_M;
   const PostPlan &pl = a.plan;
-  const int n = a.n, m = a.m, d = a.d;
+  const int n = a.n, m = a.m, d = a.d, S = a.stages;
+  const int ncolmax = pl.ncol[0];
+  const int cf = xt_chunk_floats(DP);
 
-  uint64_t *bars = (uint64_t *)(sm + 2 * a.stage_bytes);
-  uint64_t *full = bars, *empty = bars + 2, *accb = bars + 4, *xbar = bars + 5,
-           *drain = bars + 6;
-  uint32_t *tmem_holder = (uint32_t *)(bars + 7);
-  float *red_ss = (float *)(bars + 8);  // [2][128]
-  float *red_mu = red_ss + 256;         // [2][128]
-  __shared__ int s_abort;
+  uint64_t *bars = (uint64_t *)(sm + (size_t)S * a.stage_bytes);
+  uint64_t *full_b = bars, *a_full = bars + kMaxStages, *empty = bars + 2 * kMaxStages;
+  uint64_t *acc_full = bars + 3 * kMaxStages, *acc_empty = acc_full + 2, *drain = acc_full + 4;
+  uint32_t *tmem_holder = (uint32_t *)(drain + 1);
+  volatile int *abort = (volatile int *)(tmem_holder + 1);
 
   auto stage = [&](int s) { return sm + (size_t)s * a.stage_bytes; };
   auto a_hi = [&](int s) { return (float *)stage(s); };
   auto a_lo = [&](int s) { return (float *)(stage(s) + 16384); };
   auto b_reg = [&](int s) { return stage(s) + 32768; };
-  const int ncolmax = pl.ncol[0];
   auto xt_reg = [&](int s) { return (float *)(stage(s) + 32768 + 2 * ncolmax * 128); };
-  const int cf = xt_chunk_floats(DP);
 
   if (tid == 0) {
-    for (int i = 0; i < 7; ++i) mbar_init(&bars[i], 1);
+    for (int s = 0; s < kMaxStages; ++s) {
+      mbar_init(&full_b[s], 1);
+      mbar_init(&a_full[s], kBldWarps);
+      mbar_init(&empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], kEpiWarps);
+    }
+    mbar_init(drain, 1);
+    *abort = 0;
     fence_mbar_init();
-    s_abort = 0;
   }
-  if (warp == 0) {
-    tmem_alloc(tmem_holder, 256);
+  if (warp == 1) {
+    tmem_alloc(tmem_holder, 512);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -83,219 +158,213 @@ __global__ void __launch_bounds__(256, 1) posterior_kernel(const __grid_constant
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
 
-  // ---- candidate tile -> registers (raw coordinates) -----------------------
-  const long long rows_here = std::min<long long>(BOUTE_TILE_M, a.N - tile0);
-  const float *xsrc = a.Xc + ((long long)b * a.N + tile0) * d;
-  const uint32_t xbytes = (uint32_t)(BOUTE_TILE_M * d * 4);
-  const bool x_tma = rows_here == BOUTE_TILE_M && ((uintptr_t)xsrc & 15) == 0 && (xbytes & 15) == 0;
-  float xr[DP];
-  if (x_tma) {
-    // staged through stage 1's A region, which is first written by chunk 1
-    if (tid == 0) {
-      mbar_arrive_expect_tx(xbar, xbytes);
-      bulk_g2s(a_hi(1), xsrc, xbytes, xbar);
-    }
-    if (!mbar_wait(xbar, 0)) s_abort = 1;
-    const float *xs = a_hi(1) + row * d;
-#pragma unroll
-    for (int t = 0; t < DP; ++t) xr[t] = t < d ? xs[t] : 0.f;
-  } else {
-#pragma unroll
-    for (int t = 0; t < DP; ++t) xr[t] = (t < d && row < rows_here) ? xsrc[(long long)row * d + t] : 0.f;
-  }
-  __syncthreads();
-
-  // ---- job sequence: objective t, pass p, chunk c -------------------------
-  int total = 0;
-  for (int p = 0; p < pl.npass; ++p) total += pl.kc[p];
-  total *= m;
-
-  auto issue = [&](int t, int p, int c, int s) {
-    const int bt = b * m + t;
-    const uint32_t bbytes = (uint32_t)(2 * pl.ncol[p] * 128);
-    const uint32_t xtb = (uint32_t)(cf * 4);
-    mbar_arrive_expect_tx(&full[s], bbytes + xtb);
-    bulk_g2s(b_reg(s),
-             a.bop + (size_t)bt * pl.image_floats + pl.off[p] +
-                 (size_t)c * 2 * pl.ncol[p] * BOUTE_KCHUNK,
-             bbytes, &full[s]);
-    bulk_g2s(xt_reg(s), a.xt + ((size_t)bt * pl.nchunk + c) * cf, xtb, &full[s]);
-  };
-  auto next_job = [&](int &t, int &p, int &c) {
-    if (++c == pl.kc[p]) {
-      c = 0;
-      if (++p == pl.npass) {
-        p = 0;
-        ++t;
-      }
-    }
-  };
-
-  int pend_q[2] = {-1, -1};  // thread 0: job whose TMA is issued but not yet consumed
-  if (tid == 0 && !s_abort && total > 0) {
-    issue(0, 0, 0, 0);
-    pend_q[0] = 0;
-  }
-  int nt = 0, np = 0, nc = 0;  // job q+1
-  next_job(nt, np, nc);
-  int t = 0, p = 0, c = 0;
-  int pass_count = 0;
-  float xs[DP];
-  float s2 = 0.f, ss_acc = 0.f, mu_acc = 0.f, mu_comp = 0.f;
-  bool mma_issued = false;
-
-  for (int q = 0; q < total; ++q) {
-    const int s = q & 1;
-    // (1) prefetch job q+1 into the other stage once the MMAs of job q-1 are done
-    if (tid == 0 && q + 1 < total && !s_abort) {
-      const int s1 = (q + 1) & 1;
-      bool ok = true;
-      if (q + 1 >= 2) ok = mbar_wait(&empty[s1], (((q + 1) >> 1) - 1) & 1);
-      if (ok) {
-        issue(nt, np, nc, s1);
-        pend_q[s1] = q + 1;
-      } else {
-        s_abort = 1;
-      }
-    }
-    // (2) operands of job q landed
-    if (!mbar_wait(&full[s], (q >> 1) & 1)) s_abort = 1;
-    if (tid == 0) pend_q[s] = -1;
-    // (3) new objective: scaled candidate coordinates
-    if (p == 0 && c == 0) {
-      const int bt = b * m + t;
-      const float *il = a.invls + (size_t)bt * 2 * DP;
-#pragma unroll
-      for (int k = 0; k < DP; ++k) xs[k] = fmaf(xr[k], il[k], xr[k] * il[DP + k]);
-      s2 = a.s2f[bt];
-      ss_acc = 0.f;
-      mu_acc = 0.f;
-      mu_comp = 0.f;
-    }
-    // build K* chunk c: this thread's row, 16 columns [16*half, 16*half+16)
-    {
-      const float *xth = xt_reg(s), *xtl = xth + BOUTE_KCHUNK * DP;
-      const float *alp = xth + 2 * BOUTE_KCHUNK * DP;
-      float *Ah = a_hi(s), *Al = a_lo(s);
-      const int jbase = c * BOUTE_KCHUNK;
-      float mu_part = 0.f;
-#pragma unroll
-      for (int g4 = 0; g4 < 4; ++g4) {
-        float vh[4], vl[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int kk = half * 16 + g4 * 4 + e;
-          const float4 *ph = (const float4 *)(xth + kk * DP);
-          const float4 *plo = (const float4 *)(xtl + kk * DP);
-          float acc = 0.f;
-#pragma unroll
-          for (int q4 = 0; q4 < DP / 4; ++q4) {
-            const float4 h4 = ph[q4], l4 = plo[q4];
-            float df;
-            df = (xs[4 * q4 + 0] - h4.x) - l4.x; acc = fmaf(df, df, acc);
-            df = (xs[4 * q4 + 1] - h4.y) - l4.y; acc = fmaf(df, df, acc);
-            df = (xs[4 * q4 + 2] - h4.z) - l4.z; acc = fmaf(df, df, acc);
-            df = (xs[4 * q4 + 3] - h4.w) - l4.w; acc = fmaf(df, df, acc);
-          }
-          const float r = sqrtf(acc);
-          const float sr = kSqrt5 * r;
-          float kv = s2 * fmaf(kFiveThirds, acc, 1.0f + sr) * expf(-sr);
-          kv = (jbase + kk < n) ? kv : 0.f;
-          mu_part = fmaf(kv, alp[kk], mu_part);  // used in the last pass only
-          const float hi = tf32_rna(kv);
-          vh[e] = hi;
-          vl[e] = kv - hi;
-        }
-        const int o = sw128_off(row, half * 16 + g4 * 4);
-        *(float4 *)(Ah + o) = make_float4(vh[0], vh[1], vh[2], vh[3]);
-        *(float4 *)(Al + o) = make_float4(vl[0], vl[1], vl[2], vl[3]);
-      }
-      // Kahan: mu_acc += mu_part, once per chunk: the last pass builds every
-      // chunk, earlier passes rebuild a prefix of them
-      if (p == pl.npass - 1) {
-        const float yk = mu_part - mu_comp;
-        const float tk = mu_acc + yk;
-        mu_comp = (tk - mu_acc) - yk;
-        mu_acc = tk;
-      }
-    }
-    // (4) publish the chunk to the tensor core
-    fence_proxy_async_smem();
-    __syncthreads();
-    if (s_abort) break;
-    const int ncol = pl.ncol[p];
-    const bool last_chunk = c == pl.kc[p] - 1;
-    // (5) one thread issues 4 k-steps x 3 MMAs
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t idesc = idesc_tf32(ncol);
-      const uint32_t sah = smem_u32(a_hi(s)), sal = smem_u32(a_lo(s));
-      const uint32_t sbh = smem_u32(b_reg(s)), sbl = sbh + ncol * 128;
-#pragma unroll
-      for (int ks = 0; ks < 4; ++ks) {
-        const uint64_t dah = sdesc_sw128(sah + ks * 32), dal = sdesc_sw128(sal + ks * 32);
-        const uint64_t dbh = sdesc_sw128(sbh + ks * 32), dbl = sdesc_sw128(sbl + ks * 32);
-        mma_tf32(tmem, dah, dbh, idesc, (c > 0 || ks > 0) ? 1u : 0u);
-        mma_tf32(tmem, dah, dbl, idesc, 1u);
-        mma_tf32(tmem, dal, dbh, idesc, 1u);
-      }
-      mma_commit(&empty[s]);
-      if (last_chunk) mma_commit(accb);
-      mma_issued = true;
-    }
-    // (6) end of pass: drain the accumulator
-    if (last_chunk) {
-      if (!mbar_wait(accb, pass_count & 1)) s_abort = 1;
-      __syncthreads();  // a uniform abort decision before the warp-collective loads
-      if (s_abort) break;
-      tc_fence_after();
-      const int gq = warp & 3, hsel = warp >> 2;
-      const int hcols = ncol >> 1;
-      const uint32_t tbase = tmem + ((uint32_t)(32 * gq) << 16) + (uint32_t)(hsel * hcols);
-      for (int cc = 0; cc < hcols; cc += 8) {
-        float v[8];
-        tmem_ld8(tbase + cc, v);
-#pragma unroll
-        for (int e = 0; e < 8; ++e) ss_acc = fmaf(v[e], v[e], ss_acc);  // zero beyond n
-      }
-      tc_fence_before();
-      __syncthreads();
-      ++pass_count;
-      if (p == pl.npass - 1) {  // objective complete
-        const int r2 = 32 * gq + lane;
-        red_ss[hsel * 128 + r2] = ss_acc;
-        red_mu[half * 128 + row] = mu_acc - mu_comp;
-        __syncthreads();
-        if (half == 0) {
-          const long long gr = tile0 + row;
-          if (gr < a.N) {
-            const size_t o = ((size_t)b * m + t) * a.N + gr;
-            const float vv = s2 - (red_ss[row] + red_ss[128 + row]);
-            a.mean[o] = red_mu[row] + red_mu[128 + row];
-            a.var[o] = vv > 0.f ? vv : 0.f;
+  if (warp == 0) {
+    // ---------------------------------------------------------------- producer
+    if (lane == 0) {
+      uint32_t q = 0;
+      int last_q = -1;  // last job issued
+      for (int tile = blockIdx.x; tile < a.tiles_total && !*abort; tile += gridDim.x) {
+        const int b = tile / a.tiles_per_problem;
+        for (int t = 0; t < m && !*abort; ++t) {
+          const int bt = b * m + t;
+          for (int p = 0; p < pl.npass && !*abort; ++p) {
+            const uint32_t bbytes = (uint32_t)(2 * pl.ncol[p] * 128);
+            for (int c = 0; c < pl.kc[p]; ++c, ++q) {
+              const int s = q % S;
+              const uint32_t use = q / S;
+              if (use >= 1 && !wait_or_abort(&empty[s], (use - 1) & 1, abort)) break;
+              mbar_arrive_expect_tx(&full_b[s], bbytes + (uint32_t)(cf * 4));
+              bulk_g2s(b_reg(s),
+                       a.bop + (size_t)bt * pl.image_floats + pl.off[p] +
+                           (size_t)c * 2 * pl.ncol[p] * BOUTE_KCHUNK,
+                       bbytes, &full_b[s]);
+              bulk_g2s(xt_reg(s), a.xt + ((size_t)bt * pl.nchunk + c) * cf, (uint32_t)(cf * 4),
+                       &full_b[s]);
+              last_q = (int)q;
+            }
           }
         }
-        __syncthreads();
+      }
+      if (*abort) {  // let our copies land before the block exits
+        for (int j = std::max(0, last_q - S + 1); j <= last_q; ++j)
+          mbar_wait(&full_b[j % S], (j / S) & 1);
       }
     }
-    t = nt; p = np; c = nc;
-    next_job(nt, np, nc);
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      uint32_t q = 0, u = 0;
+      bool issued = false;
+      for (int tile = blockIdx.x; tile < a.tiles_total && !*abort; tile += gridDim.x) {
+        for (int t = 0; t < m && !*abort; ++t) {
+          for (int p = 0; p < pl.npass && !*abort; ++p, ++u) {
+            const int ab = u & 1;
+            if (u >= 2 && !wait_or_abort(&acc_empty[ab], ((u >> 1) - 1) & 1, abort)) break;
+            tc_fence_after();
+            const int ncol = pl.ncol[p];
+            const uint32_t idesc = idesc_tf32(ncol);
+            const uint32_t dtm = tmem + (uint32_t)(ab * 256);
+            for (int c = 0; c < pl.kc[p]; ++c, ++q) {
+              const int s = q % S;
+              const uint32_t use = q / S;
+              if (!wait_or_abort(&full_b[s], use & 1, abort)) break;
+              if (!wait_or_abort(&a_full[s], use & 1, abort)) break;
+              tc_fence_after();
+              const uint32_t sah = smem_u32(a_hi(s)), sal = smem_u32(a_lo(s));
+              const uint32_t sbh = smem_u32(b_reg(s)), sbl = sbh + ncol * 128;
+#pragma unroll
+              for (int ks = 0; ks < 4; ++ks) {
+                const uint64_t dah = sdesc_sw128(sah + ks * 32), dal = sdesc_sw128(sal + ks * 32);
+                const uint64_t dbh = sdesc_sw128(sbh + ks * 32), dbl = sdesc_sw128(sbl + ks * 32);
+                mma_tf32(dtm, dah, dbh, idesc, (c > 0 || ks > 0) ? 1u : 0u);
+                mma_tf32(dtm, dah, dbl, idesc, 1u);
+                mma_tf32(dtm, dal, dbh, idesc, 1u);
+              }
+              mma_commit(&empty[s]);
+              issued = true;
+            }
+            mma_commit(&acc_full[ab]);
+          }
+        }
+      }
+      if (issued) {  // every MMA of ours has completed before TMEM is released
+        mma_commit(drain);
+        mbar_wait(drain, 0);
+      }
+    }
+  } else if (warp >= kEpiWarp0 && warp < kEpiWarp0 + kEpiWarps) {
+    // ---------------------------------------------------------------- epilogue
+    const int eq = warp - kEpiWarp0;  // TMEM lane quarter (warp % 4)
+    uint32_t u = 0;
+    for (int tile = blockIdx.x; tile < a.tiles_total && !*abort; tile += gridDim.x) {
+      const int b = tile / a.tiles_per_problem;
+      const long long row =
+          (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M + 32 * eq + lane;
+      for (int t = 0; t < m && !*abort; ++t) {
+        float ss = 0.f;
+        for (int p = 0; p < pl.npass; ++p, ++u) {
+          const int ab = u & 1;
+          if (!wait_or_abort(&acc_full[ab], (u >> 1) & 1, abort)) break;
+          tc_fence_after();
+          const uint32_t tb = tmem + (uint32_t)(ab * 256) + ((uint32_t)(32 * eq) << 16);
+          for (int cc = 0; cc < pl.ncol[p]; cc += 16) {
+            float v[16];
+            tmem_ld16(tb + cc, v);
+#pragma unroll
+            for (int e = 0; e < 16; ++e) ss = fmaf(v[e], v[e], ss);  // zero beyond n
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_count(&acc_empty[ab]);
+        }
+        if (*abort) break;
+        if (row < a.N) {
+          const float vv = a.s2f[b * m + t] - ss;
+          a.var[((size_t)b * m + t) * a.N + row] = vv > 0.f ? vv : 0.f;
+        }
+      }
+    }
+  } else if (warp >= kBldWarp0) {
+    // ---------------------------------------------------------------- K* builders
+    const int bw = warp - kBldWarp0;
+    const int r = bw * 16 + (lane & 15), half = lane >> 4;
+    uint32_t q = 0;
+    for (int tile = blockIdx.x; tile < a.tiles_total && !*abort; tile += gridDim.x) {
+      const int b = tile / a.tiles_per_problem;
+      const long long row = (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M + r;
+      const float *xrow = a.Xc + ((long long)b * a.N + row) * d;
+      float xr[DP];
+#pragma unroll
+      for (int k = 0; k < DP; ++k) xr[k] = (k < d && row < a.N) ? xrow[k] : 0.f;
+      for (int t = 0; t < m && !*abort; ++t) {
+        const int bt = b * m + t;
+        const float *il = a.invls + (size_t)bt * 2 * DP;
+        unsigned long long xs2[DP];
+#pragma unroll
+        for (int k = 0; k < DP; ++k) xs2[k] = f2_dup(fmaf(xr[k], il[k], xr[k] * il[DP + k]));
+        const float s2 = a.s2f[bt];
+        float mu = 0.f, comp = 0.f;
+        for (int p = 0; p < pl.npass && !*abort; ++p) {
+          const bool last_pass = p == pl.npass - 1;
+          for (int c = 0; c < pl.kc[p]; ++c, ++q) {
+            const int s = q % S;
+            const uint32_t use = q / S;
+            if (use >= 1 && !wait_or_abort(&empty[s], (use - 1) & 1, abort)) break;
+            if (!wait_or_abort(&full_b[s], use & 1, abort)) break;
+            const float *xth = xt_reg(s), *xtl = xth + BOUTE_KCHUNK * DP;
+            const float *alp = xtl + BOUTE_KCHUNK * DP;
+            // squared scaled distances to this thread's 16 training points, in
+            // pairs: (x*_k - x_hi) - x_lo, squared and accumulated
+            unsigned long long acc2[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc2[e] = 0ull;
+#pragma unroll
+            for (int k = 0; k < DP; ++k) {
+              const unsigned long long *h2 =
+                  (const unsigned long long *)(xth + k * BOUTE_KCHUNK + 16 * half);
+              const unsigned long long *l2 =
+                  (const unsigned long long *)(xtl + k * BOUTE_KCHUNK + 16 * half);
+#pragma unroll
+              for (int e = 0; e < 8; ++e) {
+                const unsigned long long df = f2_sub(f2_sub(xs2[k], h2[e]), l2[e]);
+                acc2[e] = f2_fma(df, df, acc2[e]);
+              }
+            }
+            const int jbase = c * BOUTE_KCHUNK + 16 * half;
+            float mu_part = 0.f;
+            float *Ah = a_hi(s), *Al = a_lo(s);
+#pragma unroll
+            for (int g4 = 0; g4 < 4; ++g4) {
+              float vh[4], vl[4];
+#pragma unroll
+              for (int e2 = 0; e2 < 2; ++e2) {
+                float r2[2];
+                f2_split(acc2[2 * g4 + e2], r2[0], r2[1]);
+#pragma unroll
+                for (int z = 0; z < 2; ++z) {
+                  const int e = 2 * e2 + z, kk = 4 * g4 + e;
+                  const float rr = sqrtf(r2[z]);
+                  const float sr = kSqrt5 * rr;
+                  float kv = s2 * fmaf(kFiveThirds, r2[z], 1.0f + sr) * expf(-sr);
+                  kv = (jbase + kk < n) ? kv : 0.f;
+                  mu_part = fmaf(kv, alp[16 * half + kk], mu_part);
+                  const float hi = tf32_rna(kv);
+                  vh[e] = hi;
+                  vl[e] = kv - hi;
+                }
+              }
+              const int o = sw128_off(r, half * 16 + g4 * 4);
+              *(float4 *)(Ah + o) = make_float4(vh[0], vh[1], vh[2], vh[3]);
+              *(float4 *)(Al + o) = make_float4(vl[0], vl[1], vl[2], vl[3]);
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_count(&a_full[s]);
+            if (last_pass) {  // Kahan: mu += mu_part (the last pass builds every chunk)
+              const float yk = mu_part - comp;
+              const float tk = mu + yk;
+              comp = (tk - mu) - yk;
+              mu = tk;
+            }
+          }
+        }
+        if (*abort) break;
+        float mt = mu - comp;
+        mt += __shfl_xor_sync(0xffffffffu, mt, 16);
+        if (half == 0 && row < a.N) a.mean[((size_t)b * m + t) * a.N + row] = mt;
+      }
+    }
   }
 
-  // ---- teardown: nothing of ours may still be in flight ---------------------
-  if (tid == 0) {
-    if (s_abort) set_status(a.status, BOUTE_ERR_TIMEOUT);
-    if (mma_issued) {
-      mma_commit(drain);
-      mbar_wait(drain, 0);
-    }
-    for (int s = 0; s < 2; ++s)
-      if (pend_q[s] >= 0) mbar_wait(&full[s], (pend_q[s] >> 1) & 1);
-  }
+  // ---- teardown -----------------------------------------------------------------
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (warp == 0) tmem_dealloc(tmem, 256);
+  if (tid == 0 && *abort) set_status(a.status, BOUTE_ERR_TIMEOUT);
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem, 512);
+  }
 }
 
 template <int DP>
@@ -311,17 +380,26 @@ int launch_dp(const Gp *gp, const float *Xc, long long N, float *mean, float *va
   a.s2f = gp->s2f;
   a.status = gp->status;
   a.N = N;
+  a.B = gp->B;
   a.m = gp->m;
   a.d = gp->d;
   a.n = gp->n;
   a.plan = gp->plan;
+  a.tiles_per_problem = (int)((N + BOUTE_TILE_M - 1) / BOUTE_TILE_M);
+  a.tiles_total = a.tiles_per_problem * gp->B;
   const int ncolmax = gp->plan.ncol[0];
-  a.stage_bytes = (uint32_t)round_up(32768 + 2 * ncolmax * 128 + xt_chunk_floats(DP) * 4, 1024);
-  const size_t smem = 1024 + 2 * (size_t)a.stage_bytes + 8 * 8 + 2 * 256 * 4;
+  a.stage_bytes =
+      (uint32_t)round_up(32768 + 2 * ncolmax * 128 + xt_chunk_floats(DP) * 4, 1024);
+  const size_t fixed = 1024 + 256;  // alignment slack, barriers, TMEM address, flag
+  const size_t budget = 227 * 1024 - fixed;
+  a.stages = (int)std::min<size_t>(kMaxStages, budget / a.stage_bytes);
+  const size_t smem = fixed + (size_t)a.stages * a.stage_bytes;
   cudaFuncSetAttribute(posterior_kernel<DP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        (int)smem);
-  dim3 grid((unsigned)((N + BOUTE_TILE_M - 1) / BOUTE_TILE_M), gp->B);
-  posterior_kernel<DP><<<grid, 256, smem, s>>>(a);
+  int sms = 152;
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
+  const int grid = std::max(1, std::min(a.tiles_total, sms));
+  posterior_kernel<DP><<<grid, kThreads, smem, s>>>(a);
   count_launch();
   return last_launch_status();
 }
