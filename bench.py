@@ -257,7 +257,9 @@ def main():
     idx = torch.empty((w.B, w.k), dtype=torch.int64, device=dev)
     val = torch.empty((w.B, w.k), dtype=f32, device=dev)
     args_dev = (dX, dY, dls, ds2, dnz, dref, dXc, deps, idx, val)
-    stream = torch.cuda.current_stream()
+    # a dedicated stream: the engine replays its step as a CUDA graph there
+    stream = torch.cuda.Stream(device=dev)
+    torch.cuda.set_stream(stream)
     bt.boute_engine_set_timing(e)
     flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
 

@@ -165,7 +165,10 @@ int boute_select_topk(const float *acq, int B, long long N, int k, long long *id
  *   Xc: B x N x d fp32; eps: B x N x m x S fp32 (mode MC_HVI; NULL otherwise);
  *   idx: B x k int64, val: B x k fp32.
  * boute_engine_step_async: as boute_engine_step without the final
- * synchronisation (device errors surface at the next synchronising call). */
+ * synchronisation (device errors surface at the next synchronising call).
+ * On a non-default stream the step is captured once per argument set (device
+ * or host buffers) into a CUDA graph and replayed afterwards; a first call
+ * with new pointers therefore must not itself run inside a stream capture. */
 typedef struct boute_engine boute_engine;
 int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S, int k,
                         boute_engine **out);

@@ -12,6 +12,11 @@ namespace boute {
 
 static std::atomic<unsigned long long> g_launches{0};
 void count_launch(int k) { g_launches.fetch_add((unsigned long long)k); }
+// Launches recorded while capturing a graph ran nothing; they count when the
+// graph is launched.
+static void g_launches_adjust(int captured) {
+  g_launches.fetch_sub((unsigned long long)captured);
+}
 unsigned long long launch_count() { return g_launches.load(); }
 
 int last_launch_status() {
@@ -74,6 +79,14 @@ struct boute_engine {
   int timing;                  // record one CUDA event per stage boundary
   cudaEvent_t ev[8];           // boundaries of the stages of the last step
   int nstage;
+  // the step as a CUDA graph, per argument set (two sets: device and host
+  // inputs); replay removes the host launch gaps between the kernels
+  struct Graph {
+    const void *key[11];
+    cudaGraphExec_t exec;
+    int launches;
+  } graphs[2];
+  int graph_next, graphs_off;
 };
 
 // Stage order of one step; boxes run only in Monte-Carlo mode (zero-length
@@ -232,6 +245,8 @@ void boute_engine_free(boute_engine *e) {
   boute_gp_free(e->gp);
   if (e->timing)
     for (int i = 0; i <= ST_COUNT; ++i) cudaEventDestroy(e->ev[i]);
+  for (auto &g : e->graphs)
+    if (g.exec) cudaGraphExecDestroy(g.exec);
   void *ptrs[] = {e->X, e->Y, e->Ys, e->ls, e->s2, e->noise, e->ref, e->front, e->mask, e->P,
                   e->K, e->lower, e->upper, e->Xc, e->eps, e->mean, e->var, e->acq, e->val,
                   e->idx, e->scratch};
@@ -291,7 +306,7 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
   int r;
   const int B = e->B, n = e->n, m = e->m;
   auto mark = [&](int stage) {
-    if (e->timing) cudaEventRecord(e->ev[stage], s);
+    if (e->timing) cudaEventRecordWithFlags(e->ev[stage], s, cudaEventRecordExternal);
   };
   mark(ST_STANDARDIZE);
   if ((r = launch_standardize(Y, B, n, m, e->Ys, s))) return r;
@@ -327,14 +342,67 @@ static int engine_args_ok(const boute_engine *e, const void *X, const void *Y, c
   return 1;
 }
 
+// Runs the step, through a cached CUDA graph when the stream can be captured.
+static int engine_launch(boute_engine *e, const double *X, const double *Y, const double *ls,
+                         const double *s2, const double *noise, const double *ref,
+                         const float *Xc, const float *eps, long long *idx, float *val,
+                         cudaStream_t s) {
+  const void *key[11] = {X, Y, ls, s2, noise, ref, Xc, eps, idx, val, (const void *)s};
+  if (!s || e->graphs_off)  // the legacy default stream cannot be captured
+    return engine_run(e, X, Y, ls, s2, noise, ref, Xc, eps, idx, val, s);
+  for (auto &g : e->graphs) {
+    if (g.exec && std::memcmp(g.key, key, sizeof(key)) == 0) {
+      if (cudaGraphLaunch(g.exec, s) != cudaSuccess) return last_launch_status();
+      count_launch(g.launches);
+      e->launches = g.launches;
+      return BOUTE_OK;
+    }
+  }
+  auto &g = e->graphs[e->graph_next];
+  e->graph_next ^= 1;
+  if (g.exec) {
+    cudaGraphExecDestroy(g.exec);
+    g.exec = nullptr;
+  }
+  if (cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+    cudaGetLastError();
+    return engine_run(e, X, Y, ls, s2, noise, ref, Xc, eps, idx, val, s);
+  }
+  const unsigned long long l0 = launch_count();
+  const int r = engine_run(e, X, Y, ls, s2, noise, ref, Xc, eps, idx, val, s);
+  cudaGraph_t graph = nullptr;
+  const cudaError_t ce = cudaStreamEndCapture(s, &graph);
+  const int captured = (int)(launch_count() - l0);
+  g_launches_adjust(captured);  // the capture itself ran nothing
+  if (r != BOUTE_OK || ce != cudaSuccess || !graph) {
+    if (graph) cudaGraphDestroy(graph);
+    cudaGetLastError();
+    return r != BOUTE_OK ? r : BOUTE_ERR_CUDA;
+  }
+  cudaGraphExec_t exec = nullptr;
+  const cudaError_t ie = cudaGraphInstantiate(&exec, graph, 0);
+  cudaGraphDestroy(graph);
+  if (ie != cudaSuccess) {
+    cudaGetLastError();
+    return BOUTE_ERR_CUDA;
+  }
+  std::memcpy(g.key, key, sizeof(key));
+  g.exec = exec;
+  g.launches = captured;
+  if (cudaGraphLaunch(exec, s) != cudaSuccess) return last_launch_status();
+  count_launch(captured);
+  e->launches = captured;
+  return BOUTE_OK;
+}
+
 int boute_engine_step_async(boute_engine *e, const double *X, const double *Y,
                             const double *lengthscale, const double *outputscale,
                             const double *noise, const double *ref, const float *Xc,
                             const float *eps, long long *idx, float *val, void *stream) {
   if (!engine_args_ok(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val))
     return BOUTE_ERR_INVALID_ARG;
-  return engine_run(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val,
-                    (cudaStream_t)stream);
+  return engine_launch(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val,
+                       (cudaStream_t)stream);
 }
 
 int boute_engine_step(boute_engine *e, const double *X, const double *Y,
@@ -365,8 +433,8 @@ int boute_engine_step_host(boute_engine *e, const double *X, const double *Y,
   if (e->mode == BOUTE_ACQ_MC_HVI)
     cudaMemcpyAsync(e->eps, eps, B * N * m * S * sizeof(float), cudaMemcpyHostToDevice, s);
   if (int r = last_launch_status()) return r;
-  int r = engine_run(e, e->X, e->Y, e->ls, e->s2, e->noise, e->ref, e->Xc, e->eps, e->idx,
-                     e->val, s);
+  int r = engine_launch(e, e->X, e->Y, e->ls, e->s2, e->noise, e->ref, e->Xc, e->eps, e->idx,
+                        e->val, s);
   if (r) return r;
   cudaMemcpyAsync(idx, e->idx, B * k * sizeof(long long), cudaMemcpyDeviceToHost, s);
   cudaMemcpyAsync(val, e->val, B * k * sizeof(float), cudaMemcpyDeviceToHost, s);
@@ -391,6 +459,11 @@ int boute_engine_set_timing(boute_engine *e, int on) {
     for (int i = 0; i <= ST_COUNT; ++i)
       if (cudaEventCreate(&e->ev[i]) != cudaSuccess) return last_launch_status();
     e->timing = 1;
+    for (auto &g : e->graphs)  // recapture with the event nodes
+      if (g.exec) {
+        cudaGraphExecDestroy(g.exec);
+        g.exec = nullptr;
+      }
   }
   return BOUTE_OK;
 }

@@ -142,6 +142,105 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
   }
 }
 
+// ---- Monte-Carlo HVI, two objectives: the boxes are the staircase strips
+// [a_i, b_i) x (-inf, u_i), so the f2 lower bound drops out:
+// HVI(y) = sum_i (b_i - max(a_i, y1))_+ (u_i - y2)_+.
+__global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const float *var,
+                                                     long long N, const float *lower,
+                                                     const float *upper, const int *Kc,
+                                                     int box_cap, const float *eps, int S,
+                                                     long long eps_stride, float *acq) {
+  extern __shared__ float strips[];  // a[K], b[K], u[K]
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
+  const int b = blockIdx.y;
+  const int K = Kc[b];
+  float *sa = strips, *sb = strips + box_cap, *su = strips + 2 * box_cap;
+  for (int i = threadIdx.x; i < K; i += blockDim.x) {
+    const size_t o = ((size_t)b * box_cap + i) * 2;
+    sa[i] = lower[o];
+    sb[i] = upper[o];
+    su[i] = upper[o + 1];
+  }
+  __syncthreads();
+  const float *m1 = mean + (size_t)b * 2 * N, *m2 = m1 + N;
+  const float *v1 = var + (size_t)b * 2 * N, *v2 = v1 + N;
+  const bool vec = (S == 128) && ((uintptr_t)eps & 15) == 0 && (eps_stride % 4) == 0;
+  const long long cstride = (long long)gridDim.x * wpb;
+  auto eps_of = [&](long long c) {
+    return eps + ((size_t)b * N + c) * eps_stride + (eps_stride == 0 ? (size_t)b * 2 * S : 0);
+  };
+  if (vec) {
+    // S = 128: one float4 per lane per objective; the next candidate's
+    // samples and posterior are loaded before this one is scored
+    long long c = (long long)blockIdx.x * wpb + warp;
+    float4 z1 = make_float4(0.f, 0.f, 0.f, 0.f), z2 = z1;
+    float pm1 = 0.f, pm2 = 0.f, pv1 = 0.f, pv2 = 0.f;
+    if (c < N) {
+      const float *e = eps_of(c);
+      z1 = __ldcs((const float4 *)(e + 4 * lane));
+      z2 = __ldcs((const float4 *)(e + S + 4 * lane));
+      pm1 = m1[c]; pm2 = m2[c]; pv1 = v1[c]; pv2 = v2[c];
+    }
+    for (; c < N; c += cstride) {
+      const float4 c1 = z1, c2 = z2;
+      const float mu1 = pm1, mu2 = pm2;
+      const float sg1 = sqrtf(fmaxf(pv1, 0.f)), sg2 = sqrtf(fmaxf(pv2, 0.f));
+      const long long cn = c + cstride;
+      if (cn < N) {
+        const float *e = eps_of(cn);
+        z1 = __ldcs((const float4 *)(e + 4 * lane));
+        z2 = __ldcs((const float4 *)(e + S + 4 * lane));
+        pm1 = m1[cn]; pm2 = m2[cn]; pv1 = v1[cn]; pv2 = v2[cn];
+      }
+      const float y1[4] = {fmaf(sg1, c1.x, mu1), fmaf(sg1, c1.y, mu1), fmaf(sg1, c1.z, mu1),
+                           fmaf(sg1, c1.w, mu1)};
+      const float y2[4] = {fmaf(sg2, c2.x, mu2), fmaf(sg2, c2.y, mu2), fmaf(sg2, c2.z, mu2),
+                           fmaf(sg2, c2.w, mu2)};
+      // strips no sample of this candidate can reach contribute exactly zero:
+      // b_k <= min y1 (b increasing) or u_k <= min y2 (u decreasing)
+      float lo1 = fminf(fminf(y1[0], y1[1]), fminf(y1[2], y1[3]));
+      float lo2 = fminf(fminf(y2[0], y2[1]), fminf(y2[2], y2[3]));
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        lo1 = fminf(lo1, __shfl_xor_sync(0xffffffffu, lo1, o));
+        lo2 = fminf(lo2, __shfl_xor_sync(0xffffffffu, lo2, o));
+      }
+      int k0 = 0, k1 = K;
+      while (k0 < K && sb[k0] <= lo1) ++k0;
+      while (k1 > k0 && su[k1 - 1] <= lo2) --k1;
+      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+      for (int k = k0; k < k1; ++k) {
+        const float ak = sa[k], bk = sb[k], uk = su[k];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float w = fmaxf(bk - fmaxf(ak, y1[j]), 0.f);
+          const float h = fmaxf(uk - y2[j], 0.f);
+          acc[j] = fmaf(w, h, acc[j]);
+        }
+      }
+      float sum = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+      if (lane == 0) acq[(size_t)b * N + c] = sum / (float)S;
+    }
+    return;
+  }
+  for (long long c = (long long)blockIdx.x * wpb + warp; c < N; c += cstride) {
+    const float mu1 = m1[c], mu2 = m2[c];
+    const float sg1 = sqrtf(fmaxf(v1[c], 0.f)), sg2 = sqrtf(fmaxf(v2[c], 0.f));
+    const float *e = eps_of(c);
+    float sum = 0.f;
+    for (int s = lane; s < S; s += 32) {
+      const float y1 = fmaf(sg1, e[s], mu1), y2 = fmaf(sg2, e[S + s], mu2);
+      for (int k = 0; k < K; ++k)
+        sum = fmaf(fmaxf(sb[k] - fmaxf(sa[k], y1), 0.f), fmaxf(su[k] - y2, 0.f), sum);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    if (lane == 0) acq[(size_t)b * N + c] = sum / (float)S;
+  }
+}
+
 }  // namespace
 
 int launch_ehvi(const float *mean, const float *var, int B, long long N, const double *front,
@@ -173,8 +272,8 @@ int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
     cudaFuncSetAttribute(mchvi_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   }
   if (m == 2) {
-    mchvi_kernel<2><<<dim3(gx, B), wpb * 32, smem, s>>>(mean, var, B, N, lower, upper, K, box_cap,
-                                                        eps, S, eps_stride, acq);
+    mchvi2_kernel<<<dim3(gx, B), wpb * 32, 3 * (size_t)box_cap * sizeof(float), s>>>(
+        mean, var, N, lower, upper, K, box_cap, eps, S, eps_stride, acq);
   } else if (m == 3) {
     mchvi_kernel<3><<<dim3(gx, B), wpb * 32, smem, s>>>(mean, var, B, N, lower, upper, K, box_cap,
                                                         eps, S, eps_stride, acq);

@@ -37,8 +37,12 @@ inline __host__ __device__ int round_up(int x, int r) { return (x + r - 1) / r *
 
 // Floats of one training-point chunk of the posterior's side input: X/ls as
 // fp32 hi [DP][32] and lo [DP][32] (dimension-major, so pairs of training
-// points load as packed f32x2), then alpha [32].
-inline __host__ __device__ int xt_chunk_floats(int DP) { return 2 * BOUTE_KCHUNK * DP + BOUTE_KCHUNK; }
+// points load as packed f32x2), alpha [32], then the objective's parameters
+// 1/ls hi [DP], 1/ls lo [DP], outputscale, 3 floats of padding.
+inline __host__ __device__ int xt_chunk_floats(int DP) {
+  return 2 * BOUTE_KCHUNK * DP + BOUTE_KCHUNK + 2 * DP + 4;
+}
+inline __host__ __device__ int xt_param_offset(int DP) { return 2 * BOUTE_KCHUNK * DP + BOUTE_KCHUNK; }
 
 inline PostPlan make_post_plan(int n) {
   PostPlan p{};

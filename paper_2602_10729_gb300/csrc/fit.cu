@@ -46,8 +46,9 @@ __global__ void standardize_kernel(const double *Y, int n, int m, double *Ys) {
   ss = block_sum(ss, red);
   double sd = n > 1 ? sqrt(ss / (n - 1)) : 1.0;
   if (!(sd >= 1e-8)) sd = 1.0;
+  const double isd = 1.0 / sd;  // one division; fp64 divides are slow on this part
   __syncthreads();  // every thread has read its inputs before (aliased) outputs land
-  for (int i = threadIdx.x; i < n; i += blockDim.x) ys[(size_t)i * m] = (y[(size_t)i * m] - mean) / sd;
+  for (int i = threadIdx.x; i < n; i += blockDim.x) ys[(size_t)i * m] = (y[(size_t)i * m] - mean) * isd;
 }
 
 // ---- K = s2 M52(X, X) + noise I (full, symmetric), per (problem, objective) ----
@@ -104,6 +105,22 @@ __global__ void prep_kernel(const double *X, int n, int d, int m, int DP, int np
       invls[(size_t)bt * 2 * DP + DP + t] = (float)(v - (double)hi);
     }
     if (threadIdx.x == 0) s2f[bt] = (float)s2[bt];
+  }
+  // the objective's parameters ride along in every chunk of the side input
+  const int po = xt_param_offset(DP), nch = npad / BOUTE_KCHUNK;
+  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < nch * (2 * DP + 4);
+       e += gridDim.x * blockDim.x) {
+    const int c = e / (2 * DP + 4), k = e % (2 * DP + 4);
+    float v = 0.f;
+    if (k < DP) v = k < d ? (float)(1.0 / l[k]) : 0.f;
+    else if (k < 2 * DP) {
+      const int t = k - DP;
+      if (t < d) {
+        const double iv = 1.0 / l[t];
+        v = (float)(iv - (double)(float)iv);
+      }
+    } else if (k == 2 * DP) v = (float)s2[bt];
+    x[(size_t)c * cf + po + k] = v;
   }
 }
 

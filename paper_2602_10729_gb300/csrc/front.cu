@@ -44,43 +44,64 @@ __device__ __forceinline__ bool lex_less(const long long *yj, int j, const long 
   return j < i;
 }
 
-__global__ void pareto_kernel(const double *Ys, int n, int m, const double *ref,
-                              unsigned char *mask, double *front, int *P) {
-  extern __shared__ long long yk[];  // n*m keys, then n keep flags (as int)
-  int *keep = (int *)(yk + (size_t)n * m);
+// All ordered pairs (i, j) are spread over the block's threads: a point is
+// dropped as soon as one pair shows it dominated (or a duplicate of a smaller
+// index), and its rank among the kept points is a count over pairs too.
+// smem: n*m keys, n drop flags, n ranks. Writes mask, front rows, P.
+__device__ void pareto_block(const double *Yb, int n, int m, const double *rb,
+                             unsigned char *mask, double *front, int *P, void *smem) {
+  long long *yk = (long long *)smem;
+  int *drop = (int *)(yk + (size_t)n * m);
+  int *rank = drop + n;
   __shared__ int count;
   __shared__ long long rk[BOUTE_MAX_M];
-  const int b = blockIdx.x;
-  const double *Yb = Ys + (size_t)b * n * m;
   for (int e = threadIdx.x; e < n * m; e += blockDim.x) yk[e] = dkey(Yb[e]);
-  if (threadIdx.x < m) rk[threadIdx.x] = dkey(ref[(size_t)b * m + threadIdx.x]);
+  if (threadIdx.x < m) rk[threadIdx.x] = dkey(rb[threadIdx.x]);
+  for (int i = threadIdx.x; i < n; i += blockDim.x) {
+    drop[i] = 0;
+    rank[i] = 0;
+  }
   if (threadIdx.x == 0) count = 0;
   __syncthreads();
   for (int i = threadIdx.x; i < n; i += blockDim.x) {
     const long long *yi = yk + (size_t)i * m;
-    bool k = true;
     for (int t = 0; t < m; ++t)
-      if (!(yi[t] < rk[t])) k = false;
-    for (int j = 0; j < n && k; ++j) {
-      if (j == i) continue;
-      const long long *yj = yk + (size_t)j * m;
-      if (dominates(yj, yi, m) || (j < i && equal(yj, yi, m))) k = false;
-    }
-    keep[i] = k;
-    mask[(size_t)b * n + i] = (unsigned char)k;
-    if (k) atomicAdd(&count, 1);
+      if (!(yi[t] < rk[t])) drop[i] = 1;
+  }
+  const long long nn = (long long)n * n;
+  for (long long e = threadIdx.x; e < nn; e += blockDim.x) {
+    const int i = (int)(e / n), j = (int)(e % n);
+    if (j == i) continue;
+    const long long *yi = yk + (size_t)i * m, *yj = yk + (size_t)j * m;
+    if (dominates(yj, yi, m) || (j < i && equal(yj, yi, m))) drop[i] = 1;  // benign race: all write 1
+  }
+  __syncthreads();
+  for (long long e = threadIdx.x; e < nn; e += blockDim.x) {
+    const int i = (int)(e / n), j = (int)(e % n);
+    if (drop[i] || drop[j] || j == i) continue;
+    if (lex_less(yk + (size_t)j * m, j, yk + (size_t)i * m, i, m)) atomicAdd(&rank[i], 1);
   }
   __syncthreads();
   for (int i = threadIdx.x; i < n; i += blockDim.x) {
-    if (!keep[i]) continue;
-    const long long *yi = yk + (size_t)i * m;
-    int rank = 0;
-    for (int j = 0; j < n; ++j)
-      if (keep[j] && lex_less(yk + (size_t)j * m, j, yi, i, m)) ++rank;
-    double *dst = front + ((size_t)b * n + rank) * m;
-    for (int t = 0; t < m; ++t) dst[t] = Yb[(size_t)i * m + t];
+    const bool k = !drop[i];
+    mask[i] = (unsigned char)k;
+    if (k) {
+      atomicAdd(&count, 1);
+      double *dst = front + (size_t)rank[i] * m;
+      for (int t = 0; t < m; ++t) dst[t] = Yb[(size_t)i * m + t];
+    }
   }
-  if (threadIdx.x == 0) P[b] = count;
+  __syncthreads();
+  if (threadIdx.x == 0) *P = count;
+  __syncthreads();
+}
+
+__global__ void pareto_kernel(const double *Ys, int n, int m, const double *ref,
+                              unsigned char *mask, double *front, int *P) {
+  extern __shared__ long long smem_keys[];
+  const int b = blockIdx.x;
+  pareto_block(Ys + (size_t)b * n * m, n, m, ref + (size_t)b * m, mask + (size_t)b * n,
+               front + (size_t)b * n * m, P + b, smem_keys);
 }
 
 // ---- boxes ---------------------------------------------------------------------
@@ -91,14 +112,13 @@ __global__ void pareto_kernel(const double *Ys, int n, int m, const double *ref,
 // the level where an inserted point changes it, and becomes one box
 // [a, b) x (-inf, u) x [z_birth, z_death); every insertion creates at most two
 // strips, so there are at most 2P+1 boxes.
-__global__ void boxes_kernel(const double *front, const int *P, int n, int m, const double *ref,
-                             float *lower, float *upper, int *Kout) {
-  extern __shared__ double ws[];
-  const int b = blockIdx.x, cap = 2 * n + 2;
-  const int Pb = P[b];
-  const double *F = front + (size_t)b * n * m;
-  const double *r = ref + (size_t)b * m;
-  float *lo = lower + (size_t)b * cap * m, *hi = upper + (size_t)b * cap * m;
+// One problem: F = its front (P rows), r = its reference point, lo/hi = its
+// box arrays (capacity 2n+2), *Kout = box count. smem (m = 3): 10 (n+2)
+// doubles and n+2 ints.
+__device__ void boxes_block(const double *F, int Pb, int n, int m, const double *r, float *lo,
+                            float *hi, int *Kout, void *smem) {
+  double *ws = (double *)smem;
+  const int cap = 2 * n + 2;
   if (m == 2) {
     for (int i = threadIdx.x; i <= Pb; i += blockDim.x) {
       lo[2 * i] = i == 0 ? -INFINITY : (float)F[2 * (i - 1)];
@@ -106,7 +126,7 @@ __global__ void boxes_kernel(const double *front, const int *P, int n, int m, co
       hi[2 * i] = i == Pb ? (float)r[0] : (float)F[2 * i];
       hi[2 * i + 1] = i == 0 ? (float)r[1] : (float)F[2 * (i - 1) + 1];
     }
-    if (threadIdx.x == 0) Kout[b] = Pb + 1;
+    if (threadIdx.x == 0) *Kout = Pb + 1;
     return;
   }
   // m == 3 --------------------------------------------------------------------
@@ -168,14 +188,71 @@ __global__ void boxes_kernel(const double *front, const int *P, int n, int m, co
     nc = nn;
   }
   for (int j = 0; j < nc; ++j) emit(ca[j], cb[j], cu[j], cz[j], r[2]);
-  Kout[b] = K;
+  *Kout = K;
+}
+
+__global__ void boxes_kernel(const double *front, const int *P, int n, int m, const double *ref,
+                             float *lower, float *upper, int *Kout) {
+  extern __shared__ double ws_boxes[];
+  const int b = blockIdx.x, cap = 2 * n + 2;
+  boxes_block(front + (size_t)b * n * m, P[b], n, m, ref + (size_t)b * m,
+              lower + (size_t)b * cap * m, upper + (size_t)b * cap * m, Kout + b, ws_boxes);
+}
+
+__device__ double block_sum_d(double v, double *red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  double t = 0.0;
+  for (int w = 0; w < nw; ++w) t += red[w];
+  return t;
+}
+
+// The engine's front stage, one block per problem: standardise the m outcome
+// columns, take the Pareto front, decompose the improving region into boxes.
+// It depends on the raw outcomes only, so it runs beside the GP fit.
+__global__ void front_fused_kernel(const double *Y, int n, int m, const double *ref, double *Ys,
+                                   unsigned char *mask, double *front, int *P, float *lower,
+                                   float *upper, int *Kout, int want_boxes) {
+  extern __shared__ long long smem_front[];
+  __shared__ double red[32];
+  const int b = blockIdx.x, cap = 2 * n + 2;
+  const double *Yb = Y + (size_t)b * n * m;
+  double *Ysb = Ys + (size_t)b * n * m;
+  for (int t = 0; t < m; ++t) {
+    double s = 0.0;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) s += Yb[(size_t)i * m + t];
+    const double mean = block_sum_d(s, red) / n;
+    double ss = 0.0;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+      const double z = Yb[(size_t)i * m + t] - mean;
+      ss += z * z;
+    }
+    ss = block_sum_d(ss, red);
+    double sd = n > 1 ? sqrt(ss / (n - 1)) : 1.0;
+    if (!(sd >= 1e-8)) sd = 1.0;
+    const double isd = 1.0 / sd;
+    for (int i = threadIdx.x; i < n; i += blockDim.x)
+      Ysb[(size_t)i * m + t] = (Yb[(size_t)i * m + t] - mean) * isd;
+  }
+  __syncthreads();
+  __shared__ int Pb;
+  pareto_block(Ysb, n, m, ref + (size_t)b * m, mask + (size_t)b * n, front + (size_t)b * n * m,
+               &Pb, smem_front);
+  if (threadIdx.x == 0) P[b] = Pb;
+  if (want_boxes)
+    boxes_block(front + (size_t)b * n * m, Pb, n, m, ref + (size_t)b * m,
+                lower + (size_t)b * cap * m, upper + (size_t)b * cap * m, Kout + b, smem_front);
 }
 
 }  // namespace
 
 int launch_pareto(const double *Ys, int B, int n, int m, const double *ref, unsigned char *mask,
                   double *front, int *P, cudaStream_t s) {
-  const size_t smem = (size_t)n * m * sizeof(long long) + (size_t)n * sizeof(int);
+  const size_t smem = (size_t)n * m * sizeof(long long) + 2 * (size_t)n * sizeof(int) + 16;
   if (smem > 48 * 1024)
     cudaFuncSetAttribute(pareto_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   pareto_kernel<<<B, 512, smem, s>>>(Ys, n, m, ref, mask, front, P);
@@ -191,6 +268,25 @@ int launch_boxes(const double *front, const int *P, int B, int n, int m, const d
   if (smem > 48 * 1024)
     cudaFuncSetAttribute(boxes_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   boxes_kernel<<<B, 256, smem, s>>>(front, P, n, m, ref, lower, upper, K);
+  count_launch();
+  return last_launch_status();
+}
+
+size_t front_smem_bytes(int n, int m) {
+  const size_t pk = (size_t)n * m * sizeof(long long) + 2 * (size_t)n * sizeof(int) + 16;
+  const size_t bx = m == 3 ? (size_t)10 * (n + 2) * sizeof(double) + (size_t)(n + 2) * sizeof(int) : 0;
+  return pk > bx ? pk : bx;
+}
+
+int launch_front_fused(const double *Y, int B, int n, int m, const double *ref, double *Ys,
+                       unsigned char *mask, double *front, int *P, float *lower, float *upper,
+                       int *K, int want_boxes, cudaStream_t s) {
+  const size_t smem = front_smem_bytes(n, m);
+  if (smem > 48 * 1024)
+    cudaFuncSetAttribute(front_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)smem);
+  front_fused_kernel<<<B, 512, smem, s>>>(Y, n, m, ref, Ys, mask, front, P, lower, upper, K,
+                                          want_boxes);
   count_launch();
   return last_launch_status();
 }

@@ -32,6 +32,12 @@ int launch_posterior(const Gp *gp, const float *Xc, long long N, float *mean, fl
                      cudaStream_t s);
 int launch_pareto(const double *Ys, int B, int n, int m, const double *ref, unsigned char *mask,
                   double *front, int *P, cudaStream_t s);
+size_t front_smem_bytes(int n, int m);
+int launch_front_fused(const double *Y, int B, int n, int m, const double *ref, double *Ys,
+                       unsigned char *mask, double *front, int *P, float *lower, float *upper,
+                       int *K, int want_boxes, cudaStream_t s);
+int launch_fit_raw(Gp *gp, const double *X, const double *Y, const double *ls, const double *s2,
+                   const double *noise, cudaStream_t s);
 int launch_boxes(const double *front, const int *P, int B, int n, int m, const double *ref,
                  float *lower, float *upper, int *K, cudaStream_t s);
 int launch_ehvi(const float *mean, const float *var, int B, long long N, const double *front,

@@ -34,12 +34,18 @@ namespace boute {
 
 namespace {
 
-constexpr int kThreads = 512;
-constexpr int kEpiWarp0 = 4;
-constexpr int kBldWarp0 = 8;
-constexpr int kBldWarps = 8;
+constexpr int kEpiWarp0 = 2;  // warps 2-5: epilogue, TMEM lane quarter = warp % 4
 constexpr int kEpiWarps = 4;
+constexpr int kBldWarp0 = 6;  // warps 6..: K* builders
 constexpr int kMaxStages = 4;
+// builder warps: 16 (8 elements per thread and chunk) when the candidate
+// coordinates are short enough to keep in registers, else 8 (16 elements)
+template <int DP>
+struct Layout {
+  static constexpr int kBld = DP <= 16 ? 16 : 8;
+  static constexpr int kThreads = 32 * (kBldWarp0 + kBld);
+  static constexpr int kCols = 128 / kBld;  // chunk columns per builder thread (8 or 16)
+};
 
 struct PostArgs {
   const float *Xc;
@@ -96,13 +102,20 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
 }
 
 // Bounded wait that also gives up as soon as another role has aborted.
+// Waiters that are not on the critical path back off with nanosleep so that
+// their polling does not take issue slots from the K* builders.
 __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity,
-                                              volatile int *abort) {
+                                              volatile int *abort, uint32_t max_sleep_ns = 0) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
+  uint32_t sleep = 16;
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 63) == 0) {
+    if (max_sleep_ns) {
+      __nanosleep(sleep);
+      sleep = sleep * 2 < max_sleep_ns ? sleep * 2 : max_sleep_ns;
+    }
+    if ((it & 15) == 0) {
       if (*abort) return false;
       if (globaltimer() - t0 > BOUTE_WAIT_NS) {
         *abort = 1;
@@ -113,8 +126,12 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity,
 }
 
 template <int DP>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
     posterior_kernel(const __grid_constant__ PostArgs a) {
+  constexpr int kBldWarps = Layout<DP>::kBld;
+  constexpr int COLS = Layout<DP>::kCols;   // columns of a chunk per builder thread
+  constexpr int GPR = 32 / COLS;            // column groups per row (threads per row)
+  constexpr int RPW = 32 / GPR;             // rows per builder warp
   extern __shared__ uint8_t smem_raw[];
   uint8_t *sm = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -172,7 +189,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int c = 0; c < pl.kc[p]; ++c, ++q) {
               const int s = q % S;
               const uint32_t use = q / S;
-              if (use >= 1 && !wait_or_abort(&empty[s], (use - 1) & 1, abort)) break;
+              if (use >= 1 && !wait_or_abort(&empty[s], (use - 1) & 1, abort, 128)) break;
               mbar_arrive_expect_tx(&full_b[s], bbytes + (uint32_t)(cf * 4));
               bulk_g2s(b_reg(s),
                        a.bop + (size_t)bt * pl.image_floats + pl.off[p] +
@@ -199,7 +216,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int t = 0; t < m && !*abort; ++t) {
           for (int p = 0; p < pl.npass && !*abort; ++p, ++u) {
             const int ab = u & 1;
-            if (u >= 2 && !wait_or_abort(&acc_empty[ab], ((u >> 1) - 1) & 1, abort)) break;
+            if (u >= 2 && !wait_or_abort(&acc_empty[ab], ((u >> 1) - 1) & 1, abort, 64)) break;
             tc_fence_after();
             const int ncol = pl.ncol[p];
             const uint32_t idesc = idesc_tf32(ncol);
@@ -207,8 +224,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int c = 0; c < pl.kc[p]; ++c, ++q) {
               const int s = q % S;
               const uint32_t use = q / S;
-              if (!wait_or_abort(&full_b[s], use & 1, abort)) break;
-              if (!wait_or_abort(&a_full[s], use & 1, abort)) break;
+              if (!wait_or_abort(&full_b[s], use & 1, abort, 32)) break;
+              if (!wait_or_abort(&a_full[s], use & 1, abort, 32)) break;
               tc_fence_after();
               const uint32_t sah = smem_u32(a_hi(s)), sal = smem_u32(a_lo(s));
               const uint32_t sbh = smem_u32(b_reg(s)), sbl = sbh + ncol * 128;
@@ -234,7 +251,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= kEpiWarp0 && warp < kEpiWarp0 + kEpiWarps) {
     // ---------------------------------------------------------------- epilogue
-    const int eq = warp - kEpiWarp0;  // TMEM lane quarter (warp % 4)
+    const int eq = warp & 3;  // TMEM lane quarter this warp may access
     uint32_t u = 0;
     for (int tile = blockIdx.x; tile < a.tiles_total && !*abort; tile += gridDim.x) {
       const int b = tile / a.tiles_per_problem;
@@ -244,7 +261,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         float ss = 0.f;
         for (int p = 0; p < pl.npass; ++p, ++u) {
           const int ab = u & 1;
-          if (!wait_or_abort(&acc_full[ab], (u >> 1) & 1, abort)) break;
+          if (!wait_or_abort(&acc_full[ab], (u >> 1) & 1, abort, 512)) break;
           tc_fence_after();
           const uint32_t tb = tmem + (uint32_t)(ab * 256) + ((uint32_t)(32 * eq) << 16);
           for (int cc = 0; cc < pl.ncol[p]; cc += 16) {
@@ -266,8 +283,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= kBldWarp0) {
     // ---------------------------------------------------------------- K* builders
+    // thread -> (row r, column group g): COLS consecutive columns of each chunk
     const int bw = warp - kBldWarp0;
-    const int r = bw * 16 + (lane & 15), half = lane >> 4;
+    const int r = bw * RPW + lane % RPW, g = lane / RPW;
     uint32_t q = 0;
     for (int tile = blockIdx.x; tile < a.tiles_total && !*abort; tile += gridDim.x) {
       const int b = tile / a.tiles_per_problem;
@@ -277,12 +295,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int k = 0; k < DP; ++k) xr[k] = (k < d && row < a.N) ? xrow[k] : 0.f;
       for (int t = 0; t < m && !*abort; ++t) {
-        const int bt = b * m + t;
-        const float *il = a.invls + (size_t)bt * 2 * DP;
         unsigned long long xs2[DP];
-#pragma unroll
-        for (int k = 0; k < DP; ++k) xs2[k] = f2_dup(fmaf(xr[k], il[k], xr[k] * il[DP + k]));
-        const float s2 = a.s2f[bt];
+        float s2 = 0.f;
         float mu = 0.f, comp = 0.f;
         for (int p = 0; p < pl.npass && !*abort; ++p) {
           const bool last_pass = p == pl.npass - 1;
@@ -293,28 +307,34 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!wait_or_abort(&full_b[s], use & 1, abort)) break;
             const float *xth = xt_reg(s), *xtl = xth + BOUTE_KCHUNK * DP;
             const float *alp = xtl + BOUTE_KCHUNK * DP;
-            // squared scaled distances to this thread's 16 training points, in
-            // pairs: (x*_k - x_hi) - x_lo, squared and accumulated
-            unsigned long long acc2[8];
+            if (p == 0 && c == 0) {  // new objective: its parameters came with the chunk
+              const float *il = xth + xt_param_offset(DP);
 #pragma unroll
-            for (int e = 0; e < 8; ++e) acc2[e] = 0ull;
+              for (int k = 0; k < DP; ++k) xs2[k] = f2_dup(fmaf(xr[k], il[k], xr[k] * il[DP + k]));
+              s2 = il[2 * DP];
+            }
+            // squared scaled distances to this thread's COLS training points, in
+            // pairs: (x*_k - x_hi) - x_lo, squared and accumulated
+            unsigned long long acc2[COLS / 2];
+#pragma unroll
+            for (int e = 0; e < COLS / 2; ++e) acc2[e] = 0ull;
 #pragma unroll
             for (int k = 0; k < DP; ++k) {
               const unsigned long long *h2 =
-                  (const unsigned long long *)(xth + k * BOUTE_KCHUNK + 16 * half);
+                  (const unsigned long long *)(xth + k * BOUTE_KCHUNK + COLS * g);
               const unsigned long long *l2 =
-                  (const unsigned long long *)(xtl + k * BOUTE_KCHUNK + 16 * half);
+                  (const unsigned long long *)(xtl + k * BOUTE_KCHUNK + COLS * g);
 #pragma unroll
-              for (int e = 0; e < 8; ++e) {
+              for (int e = 0; e < COLS / 2; ++e) {
                 const unsigned long long df = f2_sub(f2_sub(xs2[k], h2[e]), l2[e]);
                 acc2[e] = f2_fma(df, df, acc2[e]);
               }
             }
-            const int jbase = c * BOUTE_KCHUNK + 16 * half;
+            const int jbase = c * BOUTE_KCHUNK + COLS * g;
             float mu_part = 0.f;
             float *Ah = a_hi(s), *Al = a_lo(s);
 #pragma unroll
-            for (int g4 = 0; g4 < 4; ++g4) {
+            for (int g4 = 0; g4 < COLS / 4; ++g4) {
               float vh[4], vl[4];
 #pragma unroll
               for (int e2 = 0; e2 < 2; ++e2) {
@@ -327,13 +347,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                   const float sr = kSqrt5 * rr;
                   float kv = s2 * fmaf(kFiveThirds, r2[z], 1.0f + sr) * expf(-sr);
                   kv = (jbase + kk < n) ? kv : 0.f;
-                  mu_part = fmaf(kv, alp[16 * half + kk], mu_part);
+                  mu_part = fmaf(kv, alp[COLS * g + kk], mu_part);
                   const float hi = tf32_rna(kv);
                   vh[e] = hi;
                   vl[e] = kv - hi;
                 }
               }
-              const int o = sw128_off(r, half * 16 + g4 * 4);
+              const int o = sw128_off(r, COLS * g + g4 * 4);
               *(float4 *)(Ah + o) = make_float4(vh[0], vh[1], vh[2], vh[3]);
               *(float4 *)(Al + o) = make_float4(vl[0], vl[1], vl[2], vl[3]);
             }
@@ -349,9 +369,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         if (*abort) break;
-        float mt = mu - comp;
-        mt += __shfl_xor_sync(0xffffffffu, mt, 16);
-        if (half == 0 && row < a.N) a.mean[((size_t)b * m + t) * a.N + row] = mt;
+        float mt = mu - comp;  // sum over the GPR column groups of the row
+#pragma unroll
+        for (int o = RPW; o < 32; o <<= 1) mt += __shfl_xor_sync(0xffffffffu, mt, o);
+        if (g == 0 && row < a.N) a.mean[((size_t)b * m + t) * a.N + row] = mt;
       }
     }
   }
@@ -399,7 +420,7 @@ int launch_dp(const Gp *gp, const float *Xc, long long N, float *mean, float *va
   int sms = 152;
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
   const int grid = std::max(1, std::min(a.tiles_total, sms));
-  posterior_kernel<DP><<<grid, kThreads, smem, s>>>(a);
+  posterior_kernel<DP><<<grid, Layout<DP>::kThreads, smem, s>>>(a);
   count_launch();
   return last_launch_status();
 }
