@@ -154,6 +154,30 @@ int boute_acq_mc_hvi(const float *mean, const float *var, int B, long long N, in
 int boute_select_topk(const float *acq, int B, long long N, int k, long long *idx, float *val,
                       void *stream);
 
+/* boute_select_topk_noalloc: the same selection, bit for bit, with its
+ * intermediate keys in a fixed array compiled into the library
+ * (BOUTE_TOPK_NOALLOC_SCRATCH_BYTES of device memory, 8 MiB) instead of
+ * memory from the CUDA pool; the paper has no counterpart, it is a service to
+ * callers that must not allocate device memory on the call path: a caller
+ * whose allocator already holds the device's free memory, a latency-critical
+ * loop that cannot take the synchronisation cudaFree implies, or a fixed
+ * memory budget. The call makes no allocation of any kind.
+ *   Limit: 2 * B * ceil(N / 2048) * k * 8 bytes of scratch (0 when
+ *   N <= 2048) must not exceed BOUTE_TOPK_NOALLOC_SCRATCH_BYTES; a larger
+ *   request returns BOUTE_ERR_UNSUPPORTED before launching anything. Other
+ *   argument errors are those of boute_select_topk.
+ *   Set-up: the first call on a device, made with that device current, looks
+ *   up the array's device address (once per device, under a lock); make that
+ *   first call before any stream capture begins.
+ *   Nothing in the array has to start at zero: every level of the selection
+ *   writes all the keys the next level reads.
+ *   There is ONE array per device: calls that overlap in time on that device
+ *   (on different streams, or from different threads) race on it and may
+ *   return wrong results. Serialise them, e.g. by issuing them on one stream. */
+#define BOUTE_TOPK_NOALLOC_SCRATCH_BYTES (8u << 20)
+int boute_select_topk_noalloc(const float *acq, int B, long long N, int k, long long *idx,
+                              float *val, void *stream);
+
 /* ---- the whole scoring step ---------------------------------------------------
  * An engine owns every intermediate buffer of one workload shape and runs
  * a0..a6 as one launch sequence on one stream.

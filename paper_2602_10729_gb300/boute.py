@@ -23,7 +23,8 @@ SYMBOLS = (
     "boute_status_string", "boute_launch_count", "boute_standardize", "boute_gp_create",
     "boute_gp_fit", "boute_gp_status", "boute_gp_free", "boute_gp_posterior",
     "boute_pareto_front", "boute_box_decompose", "boute_acq_ehvi", "boute_acq_mc_hvi",
-    "boute_select_topk", "boute_engine_create", "boute_engine_step", "boute_engine_step_async",
+    "boute_select_topk", "boute_select_topk_noalloc", "boute_engine_create", "boute_engine_step",
+    "boute_engine_step_async",
     "boute_engine_step_host", "boute_engine_scores", "boute_engine_set_timing",
     "boute_engine_stage_times", "boute_engine_launches_per_step", "boute_engine_free",
 )
@@ -70,6 +71,7 @@ def load(path: str | None = None):
         "boute_acq_mc_hvi": ([_vp, _vp, _i, _ll, _i, _vp, _vp, _vp, _i, _vp, _i, _ll, _vp, _vp],
                              _i),
         "boute_select_topk": ([_vp, _i, _ll, _i, _vp, _vp, _vp], _i),
+        "boute_select_topk_noalloc": ([_vp, _i, _ll, _i, _vp, _vp, _vp], _i),
         "boute_engine_create": ([_i, _i, _i, _i, _ll, _i, _i, _i, ctypes.POINTER(_vp)], _i),
         "boute_engine_step": ([_vp] * 11 + [_vp], _i),
         "boute_engine_step_async": ([_vp] * 11 + [_vp], _i),
@@ -207,6 +209,16 @@ def boute_acq_mc_hvi(mean, var, B, N, m, lower, upper, K, box_cap, eps, S, eps_c
 def boute_select_topk(acq, B, N, k, idx, val, stream=None):
     _check(load().boute_select_topk(_p(acq, torch.float32), B, N, k, _p(idx, torch.int64),
                                     _p(val, torch.float32), _s(stream)), "boute_select_topk")
+
+
+def boute_select_topk_noalloc(acq, B, N, k, idx, val, stream=None):
+    _check(load().boute_select_topk_noalloc(_p(acq, torch.float32), B, N, k,
+                                            _p(idx, torch.int64), _p(val, torch.float32),
+                                            _s(stream)), "boute_select_topk_noalloc")
+
+
+#: bytes of the fixed scratch array behind boute_select_topk_noalloc
+TOPK_NOALLOC_SCRATCH_BYTES = 8 << 20
 
 
 class Engine:
