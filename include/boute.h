@@ -52,14 +52,14 @@ const char *boute_status_string(int status);
  * A monotone counter; differences bracket a region of work. */
 unsigned long long boute_launch_count(void);
 
-/* ---- a0: outcome standardisation -----------------------------------------
+/* ---- outcome standardisation ---------------------------------------------
  * Sec. 6 (outcome transform "Standardize", applied after Sec. 5.2 S4's
  * Log/Logit, which stay with the caller): Ys[b,:,t] = (Y[b,:,t] - mean) / std,
  * std with the n-1 denominator; a column with n < 2 or std < 1e-8 is divided
  * by 1. Y, Ys: B x n x m fp64 (may alias). */
 int boute_standardize(const double *Y, int B, int n, int m, double *Ys, void *stream);
 
-/* ---- a1: GP fit ------------------------------------------------------------
+/* ---- GP fit ----------------------------------------------------------------
  * Sec. 5.2 step (i) and Sec. 6: one exact GP per objective (SingleTaskGP
  * models combined as a ModelListGP), ARD Matern-5/2 covariance with an
  * outputscale (MaternKernel nu=2.5 in a ScaleKernel), zero prior mean on
@@ -83,7 +83,7 @@ int boute_gp_fit(boute_gp *gp, const double *X, const double *Ys, const double *
 int boute_gp_status(boute_gp *gp, void *stream);
 void boute_gp_free(boute_gp *gp);
 
-/* ---- a2 + a3: posterior -----------------------------------------------------
+/* ---- posterior ---------------------------------------------------------------
  * Latent-function posterior of every objective at N candidates per problem
  * (Sec. 5.2: the acquisition is taken over the GP posterior):
  *   mean = K* alpha,  var = max(0, s2 - rowsum((K* L^-T)^2)),
@@ -95,7 +95,7 @@ void boute_gp_free(boute_gp *gp);
 int boute_gp_posterior(const boute_gp *gp, const float *Xc, long long N, float *mean,
                        float *var, void *stream);
 
-/* ---- a4: Pareto front and box decomposition ---------------------------------
+/* ---- Pareto front and box decomposition -------------------------------------
  * Sec. 5.2 (Pareto-optimal set; Sec. 4.3, minimisation): point i of problem b
  * is on the front iff no point dominates it (<= in every objective, < in
  * one), no exact duplicate with a smaller index exists, and it is strictly
@@ -118,7 +118,7 @@ int boute_pareto_front(const double *Ys, int B, int n, int m, const double *ref,
 int boute_box_decompose(const double *front, const int *P, int B, int n, int m,
                         const double *ref, float *lower, float *upper, int *K, void *stream);
 
-/* ---- a5: acquisition ----------------------------------------------------------
+/* ---- acquisition --------------------------------------------------------------
  * Expected hypervolume improvement (Sec. 5.2, "Constrained qNEHVI": the
  * expectation of HVI over the posterior), for m = 2 independent objectives in
  * closed form over the P+1 staircase cells:
@@ -144,7 +144,7 @@ int boute_acq_mc_hvi(const float *mean, const float *var, int B, long long N, in
                      const float *eps, int S, long long eps_cand_stride, float *acq,
                      void *stream);
 
-/* ---- a6: selection ------------------------------------------------------------
+/* ---- selection ----------------------------------------------------------------
  * Sec. 5.2 step (ii): the next configuration(s) to evaluate are the best
  * scored candidates. Per problem, the k largest acq values in the order
  * (value descending, NaN as -infinity, -0 as +0, equal values by ascending
@@ -179,8 +179,10 @@ int boute_select_topk_noalloc(const float *acq, int B, long long N, int k, long 
                               float *val, void *stream);
 
 /* ---- the whole scoring step ---------------------------------------------------
- * An engine owns every intermediate buffer of one workload shape and runs
- * a0..a6 as one launch sequence on one stream.
+ * An engine owns every intermediate buffer of one workload shape and runs the
+ * whole step: GP fit, then posterior, acquisition and selection on `stream`;
+ * the front stage (standardise, Pareto front, boxes) on an internal second
+ * stream forked from `stream` and joined back before the acquisition.
  * boute_engine_step: device inputs; boute_engine_step_host: HOST inputs and
  * outputs (copied in and out on `stream` inside the call); both synchronise
  * and return the fit status or the first device error.
@@ -211,10 +213,13 @@ int boute_engine_step_host(boute_engine *e, const double *X, const double *Y,
 /* Copies the last step's per-candidate results into caller buffers (device
  * pointers; any may be NULL): acq B x N, mean and var B x m x N (fp32). */
 int boute_engine_scores(const boute_engine *e, float *acq, float *mean, float *var, void *stream);
-/* Stage timing on the engine's stream: once enabled, every step records a
- * CUDA event at each stage boundary (standardise, fit, front, boxes,
- * posterior, acquisition, top-k); boute_engine_stage_times waits for the
- * last step and writes its 7 stage durations in milliseconds (count >= 7). */
+/* Stage timing on the engine's stream: while enabled (on != 0), every step
+ * records a CUDA event at each stage boundary (fit, front = standardise +
+ * Pareto front + boxes, posterior, acquisition, top-k) and runs the front
+ * stage after the fit on the step's stream instead of beside it, so that the
+ * stages add up; boute_engine_stage_times waits for the last timed step and
+ * writes its 5 stage durations in milliseconds (count >= 5). Disabling it
+ * restores the concurrent front stage. */
 int boute_engine_set_timing(boute_engine *e, int on);
 int boute_engine_stage_times(boute_engine *e, float *ms, int count);
 /* Kernels one boute_engine_step launches. */

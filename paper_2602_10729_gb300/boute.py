@@ -29,7 +29,7 @@ SYMBOLS = (
     "boute_engine_stage_times", "boute_engine_launches_per_step", "boute_engine_free",
 )
 #: stage names of boute_engine_stage_times, in order
-STAGES = ("standardize", "fit", "front", "boxes", "posterior", "acquisition", "topk")
+STAGES = ("fit", "front", "posterior", "acquisition", "topk")
 
 _lib = None
 _vp = ctypes.c_void_p

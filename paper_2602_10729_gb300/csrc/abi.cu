@@ -87,11 +87,16 @@ struct boute_engine {
     int launches;
   } graphs[2];
   int graph_next, graphs_off;
+  // the front stage (standardise, Pareto front, boxes) depends on the raw
+  // outcomes only: it runs on a second stream, forked from and joined back
+  // into the step's stream, beside the GP fit
+  cudaStream_t side;
+  cudaEvent_t fork, join;
 };
 
-// Stage order of one step; boxes run only in Monte-Carlo mode (zero-length
-// stage otherwise).
-enum { ST_STANDARDIZE, ST_FIT, ST_FRONT, ST_BOXES, ST_POSTERIOR, ST_ACQ, ST_TOPK, ST_COUNT };
+// Stage order of one step as timed (with timing on, the front stage runs
+// after the fit on the step's stream, so the stage times add up).
+enum { ST_FIT, ST_FRONT, ST_POSTERIOR, ST_ACQ, ST_TOPK, ST_COUNT };
 
 extern "C" {
 
@@ -135,7 +140,6 @@ int boute_gp_create(int B, int n, int d, int m, boute_gp **out) {
   r |= dalloc(&g.Wws, BM * np * (np + 1));
   r |= dalloc(&g.bop, BM * (size_t)g.plan.image_floats);
   r |= dalloc(&g.xt, BM * (size_t)g.plan.nchunk * xt_chunk_floats(g.DP));
-  r |= dalloc(&g.invls, BM * 2 * g.DP);
   r |= dalloc(&g.s2f, BM);
   r |= dalloc(&g.status, 1);
   if (r != BOUTE_OK) {
@@ -170,7 +174,7 @@ void boute_gp_free(boute_gp *gp) {
   if (!gp) return;
   Gp &g = gp->g;
   cudaFree(g.Kh); cudaFree(g.Kl); cudaFree(g.Aws); cudaFree(g.Wws); cudaFree(g.bop); cudaFree(g.xt);
-  cudaFree(g.invls); cudaFree(g.s2f); cudaFree(g.status);
+  cudaFree(g.s2f); cudaFree(g.status);
   delete gp;
 }
 
@@ -243,10 +247,13 @@ int boute_select_topk(const float *acq, int B, long long N, int k, long long *id
 void boute_engine_free(boute_engine *e) {
   if (!e) return;
   boute_gp_free(e->gp);
-  if (e->timing)
+  if (e->ev[0])
     for (int i = 0; i <= ST_COUNT; ++i) cudaEventDestroy(e->ev[i]);
   for (auto &g : e->graphs)
     if (g.exec) cudaGraphExecDestroy(g.exec);
+  if (e->fork) cudaEventDestroy(e->fork);
+  if (e->join) cudaEventDestroy(e->join);
+  if (e->side) cudaStreamDestroy(e->side);
   void *ptrs[] = {e->X, e->Y, e->Ys, e->ls, e->s2, e->noise, e->ref, e->front, e->mask, e->P,
                   e->K, e->lower, e->upper, e->Xc, e->eps, e->mean, e->var, e->acq, e->val,
                   e->idx, e->scratch};
@@ -291,6 +298,13 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
   r |= dalloc(&e->idx, (size_t)B * k);
   r |= dalloc(&e->val, (size_t)B * k);
   r |= dalloc((unsigned char **)&e->scratch, topk_scratch_bytes(B, N, k));
+  if (r == BOUTE_OK &&
+      (cudaStreamCreateWithFlags(&e->side, cudaStreamNonBlocking) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->fork, cudaEventDisableTiming) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->join, cudaEventDisableTiming) != cudaSuccess)) {
+    cudaGetLastError();
+    r = BOUTE_ERR_CUDA;
+  }
   if (r != BOUTE_OK) {
     boute_engine_free(e);
     return BOUTE_ERR_OOM;
@@ -305,22 +319,31 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
   const unsigned long long l0 = launch_count();
   int r;
   const int B = e->B, n = e->n, m = e->m;
+  const int mc = e->mode == BOUTE_ACQ_MC_HVI;
   auto mark = [&](int stage) {
     if (e->timing) cudaEventRecordWithFlags(e->ev[stage], s, cudaEventRecordExternal);
   };
-  mark(ST_STANDARDIZE);
-  if ((r = launch_standardize(Y, B, n, m, e->Ys, s))) return r;
+  auto front = [&](cudaStream_t fs) {
+    return launch_front_fused(Y, B, n, m, ref, e->Ys, e->mask, e->front, e->P, e->lower,
+                              e->upper, e->K, mc, fs);
+  };
   mark(ST_FIT);
-  if ((r = launch_fit(&e->gp->g, X, e->Ys, ls, s2, noise, s))) return r;
+  if (!e->timing) {  // fork: the front stage runs beside the fit
+    if (cudaEventRecord(e->fork, s) != cudaSuccess ||
+        cudaStreamWaitEvent(e->side, e->fork, 0) != cudaSuccess)
+      return last_launch_status();
+    if ((r = front(e->side))) return r;
+    if (cudaEventRecord(e->join, e->side) != cudaSuccess) return last_launch_status();
+  }
+  if ((r = launch_fit_raw(&e->gp->g, X, Y, ls, s2, noise, s))) return r;
   mark(ST_FRONT);
-  if ((r = launch_pareto(e->Ys, B, n, m, ref, e->mask, e->front, e->P, s))) return r;
-  mark(ST_BOXES);
-  if (e->mode == BOUTE_ACQ_MC_HVI)
-    if ((r = launch_boxes(e->front, e->P, B, n, m, ref, e->lower, e->upper, e->K, s))) return r;
+  if (e->timing && (r = front(s))) return r;
   mark(ST_POSTERIOR);
   if ((r = launch_posterior(&e->gp->g, Xc, e->N, e->mean, e->var, s))) return r;
+  if (!e->timing && cudaStreamWaitEvent(s, e->join, 0) != cudaSuccess)  // join
+    return last_launch_status();
   mark(ST_ACQ);
-  if (e->mode == BOUTE_ACQ_EHVI2D) {
+  if (!mc) {
     if ((r = launch_ehvi(e->mean, e->var, B, e->N, e->front, e->P, n, ref, e->acq, s))) return r;
   } else {
     if ((r = launch_mchvi(e->mean, e->var, B, e->N, m, e->lower, e->upper, e->K, 2 * n + 2, eps,
@@ -455,21 +478,22 @@ int boute_engine_scores(const boute_engine *e, float *acq, float *mean, float *v
 
 int boute_engine_set_timing(boute_engine *e, int on) {
   if (!e) return BOUTE_ERR_INVALID_ARG;
-  if (on && !e->timing) {
+  on = on != 0;
+  if (on == e->timing) return BOUTE_OK;
+  if (on && !e->ev[0])
     for (int i = 0; i <= ST_COUNT; ++i)
       if (cudaEventCreate(&e->ev[i]) != cudaSuccess) return last_launch_status();
-    e->timing = 1;
-    for (auto &g : e->graphs)  // recapture with the event nodes
-      if (g.exec) {
-        cudaGraphExecDestroy(g.exec);
-        g.exec = nullptr;
-      }
-  }
+  e->timing = on;
+  for (auto &g : e->graphs)  // recapture: event nodes in or out, front stage placement
+    if (g.exec) {
+      cudaGraphExecDestroy(g.exec);
+      g.exec = nullptr;
+    }
   return BOUTE_OK;
 }
 
 int boute_engine_stage_times(boute_engine *e, float *ms, int count) {
-  if (!e || !ms || count < ST_COUNT || !e->timing) return BOUTE_ERR_INVALID_ARG;
+  if (!e || !ms || count < ST_COUNT || !e->ev[0]) return BOUTE_ERR_INVALID_ARG;
   if (cudaEventSynchronize(e->ev[ST_COUNT]) != cudaSuccess) return last_launch_status();
   for (int i = 0; i < ST_COUNT; ++i)
     if (cudaEventElapsedTime(&ms[i], e->ev[i], e->ev[i + 1]) != cudaSuccess)

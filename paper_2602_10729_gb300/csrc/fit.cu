@@ -29,7 +29,7 @@ __device__ double block_sum(double v, double *red) {
   return t;
 }
 
-// ---- a0: Standardize (one block per (problem, objective)) --------------------
+// ---- Standardize (one block per (problem, objective)) --------------------
 __global__ void standardize_kernel(const double *Y, int n, int m, double *Ys) {
   __shared__ double red[32];
   const int b = blockIdx.x / m, t = blockIdx.x % m;
@@ -51,18 +51,20 @@ __global__ void standardize_kernel(const double *Y, int n, int m, double *Ys) {
   for (int i = threadIdx.x; i < n; i += blockDim.x) ys[(size_t)i * m] = (y[(size_t)i * m] - mean) * isd;
 }
 
-// ---- K = s2 M52(X, X) + noise I (full, symmetric), per (problem, objective) ----
-// fp64 arithmetic, stored as an fp32 pair (hi = K rounded, lo = K - hi): the
-// factorisation works on hi, the refinement of alpha on hi + lo.
-__global__ void kernel_matrix_kernel(const double *X, int n, int d, int m, const double *ls,
-                                     const double *s2, const double *noise, float *Kh_all,
-                                     float *Kl_all) {
-  __shared__ double il[BOUTE_MAX_D];
-  const int bt = blockIdx.z, b = bt / m;
-  for (int t = threadIdx.y * blockDim.x + threadIdx.x; t < d; t += blockDim.x * blockDim.y)
-    il[t] = 1.0 / ls[(size_t)bt * d + t];
+// ---- fit set-up, one launch: K = s2 M52(X, X) + noise I and the side input --
+// Blocks [0, nkt) of problem-objective bt compute 16 x 16 tiles of K (full,
+// symmetric) in fp64, stored as an fp32 pair (hi = K rounded, lo = K - hi):
+// the factorisation works on hi, the refinement of alpha on hi + lo. The
+// remaining blocks write the posterior's side input: scaled training inputs
+// x / l as fp32 hi/lo pairs (dimension-major per 32-point chunk), and in every
+// chunk the objective's 1/l (hi, lo) and outputscale. Block 0 of the first
+// problem clears the fit status.
+__device__ void kmat_tile(const double *X, int n, int d, int b, const double *l, double s2,
+                          double noise, int tile, float *Kh, float *Kl, double *il) {
+  for (int t = threadIdx.x; t < d; t += blockDim.x) il[t] = 1.0 / l[t];
   __syncthreads();
-  const int i = blockIdx.y * blockDim.y + threadIdx.y, j = blockIdx.x * blockDim.x + threadIdx.x;
+  const int tn = (n + 15) / 16;
+  const int i = (tile / tn) * 16 + threadIdx.x / 16, j = (tile % tn) * 16 + threadIdx.x % 16;
   if (i >= n || j >= n) return;
   const double *xi = X + ((size_t)b * n + i) * d, *xj = X + ((size_t)b * n + j) * d;
   double r2 = 0.0;
@@ -71,45 +73,29 @@ __global__ void kernel_matrix_kernel(const double *X, int n, int d, int m, const
     r2 = fma(z, z, r2);
   }
   const double r = sqrt(r2), sr = sqrt(5.0) * r;
-  double k = s2[bt] * (1.0 + sr + 5.0 * r2 / 3.0) * exp(-sr);
-  if (i == j) k += noise[bt];
+  double k = s2 * (1.0 + sr + 5.0 * r2 / 3.0) * exp(-sr);
+  if (i == j) k += noise;
   const float kh = (float)k;
-  const size_t o = (size_t)bt * n * n + (size_t)i * n + j;
-  Kh_all[o] = kh;
-  Kl_all[o] = (float)(k - (double)kh);
+  const size_t o = (size_t)i * n + j;
+  Kh[o] = kh;
+  Kl[o] = (float)(k - (double)kh);
 }
 
-// ---- scaled training inputs, 1/lengthscale and outputscale in fp32 -----------
-__global__ void prep_kernel(const double *X, int n, int d, int m, int DP, int npad,
-                            const double *ls, const double *s2, float *xt, float *invls,
-                            float *s2f) {
-  const int bt = blockIdx.y, b = bt / m;
-  const double *l = ls + (size_t)bt * d;
+__device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad,
+                          const double *l, double s2, float *x, int blk, int nblk) {
   const int cf = xt_chunk_floats(DP);
-  float *x = xt + (size_t)bt * (npad / BOUTE_KCHUNK) * cf;
   const int total = npad * DP;
-  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < total; e += gridDim.x * blockDim.x) {
+  for (int e = blk * blockDim.x + threadIdx.x; e < total; e += nblk * blockDim.x) {
     const int j = e / DP, t = e % DP;
     double v = (j < n && t < d) ? X[((size_t)b * n + j) * d + t] / l[t] : 0.0;
     float hi = (float)v, lo = (float)(v - (double)hi);
     const int c = j / BOUTE_KCHUNK, jj = j % BOUTE_KCHUNK;
-    float *blk = x + (size_t)c * cf;  // dimension-major: [DP][32] hi, [DP][32] lo
-    blk[t * BOUTE_KCHUNK + jj] = hi;
-    blk[BOUTE_KCHUNK * DP + t * BOUTE_KCHUNK + jj] = lo;
+    float *q = x + (size_t)c * cf;  // dimension-major: [DP][32] hi, [DP][32] lo
+    q[t * BOUTE_KCHUNK + jj] = hi;
+    q[BOUTE_KCHUNK * DP + t * BOUTE_KCHUNK + jj] = lo;
   }
-  if (blockIdx.x == 0) {
-    for (int t = threadIdx.x; t < DP; t += blockDim.x) {
-      double v = t < d ? 1.0 / l[t] : 0.0;
-      float hi = (float)v;
-      invls[(size_t)bt * 2 * DP + t] = hi;
-      invls[(size_t)bt * 2 * DP + DP + t] = (float)(v - (double)hi);
-    }
-    if (threadIdx.x == 0) s2f[bt] = (float)s2[bt];
-  }
-  // the objective's parameters ride along in every chunk of the side input
   const int po = xt_param_offset(DP), nch = npad / BOUTE_KCHUNK;
-  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < nch * (2 * DP + 4);
-       e += gridDim.x * blockDim.x) {
+  for (int e = blk * blockDim.x + threadIdx.x; e < nch * (2 * DP + 4); e += nblk * blockDim.x) {
     const int c = e / (2 * DP + 4), k = e % (2 * DP + 4);
     float v = 0.f;
     if (k < DP) v = k < d ? (float)(1.0 / l[k]) : 0.f;
@@ -119,8 +105,48 @@ __global__ void prep_kernel(const double *X, int n, int d, int m, int DP, int np
         const double iv = 1.0 / l[t];
         v = (float)(iv - (double)(float)iv);
       }
-    } else if (k == 2 * DP) v = (float)s2[bt];
+    } else if (k == 2 * DP) v = (float)s2;
     x[(size_t)c * cf + po + k] = v;
+  }
+}
+
+__global__ void __launch_bounds__(256) fit_setup_kernel(
+    const double *X, int n, int d, int m, int DP, int npad, const double *ls, const double *s2,
+    const double *noise, float *Kh_all, float *Kl_all, float *xt, float *s2f, int nkt, int nprep,
+    int *status) {
+  __shared__ double il[BOUTE_MAX_D];
+  const int bt = blockIdx.y, b = bt / m;
+  const double *l = ls + (size_t)bt * d;
+  if (blockIdx.x == 0 && bt == 0 && threadIdx.x == 0) *status = BOUTE_OK;
+  if ((int)blockIdx.x < nkt) {
+    kmat_tile(X, n, d, b, l, s2[bt], noise[bt], blockIdx.x, Kh_all + (size_t)bt * n * n,
+              Kl_all + (size_t)bt * n * n, il);
+  } else {
+    float *x = xt + (size_t)bt * (npad / BOUTE_KCHUNK) * xt_chunk_floats(DP);
+    prep_part(X, n, d, b, DP, npad, l, s2[bt], x, blockIdx.x - nkt, nprep);
+    if (blockIdx.x == nkt && threadIdx.x == 0) s2f[bt] = (float)s2[bt];
+  }
+}
+
+// fp32 tf32 hi/lo operand images of W = L^-1 (lower, row stride ld), swizzled
+// per column pass and 32-wide K chunk, written by the threads of one block (or
+// a grid of blocks: element e in [first, total) by stride).
+__device__ __forceinline__ void pack_elems(const float *W, int ld, const PostPlan &plan,
+                                           float *img, long long first, long long stride) {
+  const int n = plan.n;
+  const long long total = (long long)plan.ncols * plan.npad;
+  for (long long e = first; e < total; e += stride) {
+    const int g = (int)(e / plan.npad), k = (int)(e % plan.npad);
+    const int p = g >> 8, c = k / BOUTE_KCHUNK;
+    if (c >= plan.kc[p]) continue;
+    const float v = (k < n && g < n && k <= g) ? W[(size_t)g * ld + k] : 0.f;
+    const float hi = tf32_rna(v);
+    const float lo = tf32_rna(v - hi);
+    const int ncol = plan.ncol[p];
+    float *blk = img + plan.off[p] + (long long)c * 2 * ncol * BOUTE_KCHUNK;
+    const int o = sw128_off(g - plan.col0[p], k % BOUTE_KCHUNK);
+    blk[o] = hi;
+    blk[ncol * BOUTE_KCHUNK + o] = lo;
   }
 }
 
@@ -151,11 +177,13 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
 // in the handle's global workspace.
 template <bool SMEM>
 __global__ void __launch_bounds__(256, 1) fit32_kernel(const float *Kh_all, const float *Kl_all,
-                                                    const double *Ys, int n, int m, float *Aws,
-                                                    float *Wws, float *xt, int DP, int npad,
+                                                    const double *Ys, int standardize, int n,
+                                                    int m, float *Aws, float *Wws, float *xt,
+                                                    int DP, int npad, PostPlan plan, float *bop,
                                                     int *status) {
   extern __shared__ float sm[];
   __shared__ int bad;
+  __shared__ double red[8], ymu, yisd;
   const int bt = blockIdx.x, b = bt / m, t = bt % m;
   const int tid = threadIdx.x, nthr = blockDim.x, lane = tid & 31, warp = tid >> 5,
             nw = nthr >> 5;
@@ -167,6 +195,30 @@ __global__ void __launch_bounds__(256, 1) fit32_kernel(const float *Kh_all, cons
   float *dg = vec + NP, *yv = vec + 2 * NP, *tv = vec + 3 * NP, *al = vec + 4 * NP,
         *rv = vec + 5 * NP;
   const double *y = Ys + (size_t)b * n * m + t;
+  // standardize != 0: Ys holds raw outcomes; this column is standardised here
+  // (zero mean, unit sample standard deviation, as standardize_kernel does)
+  if (standardize) {
+    double sum = 0.0;
+    for (int i = tid; i < n; i += nthr) sum += y[(size_t)i * m];
+    const double mean = block_sum(sum, red) / n;
+    double ss = 0.0;
+    for (int i = tid; i < n; i += nthr) {
+      const double z = y[(size_t)i * m] - mean;
+      ss += z * z;
+    }
+    ss = block_sum(ss, red);
+    double sd = n > 1 ? sqrt(ss / (n - 1)) : 1.0;
+    if (!(sd >= 1e-8)) sd = 1.0;
+    if (tid == 0) {
+      ymu = mean;
+      yisd = 1.0 / sd;
+    }
+  } else if (tid == 0) {
+    ymu = 0.0;
+    yisd = 1.0;
+  }
+  __syncthreads();
+  const double mu_y = ymu, isd_y = yisd;
 
   for (int e = tid; e < NP * ld; e += nthr) {
     const int i = e / ld, k = e % ld;
@@ -176,7 +228,7 @@ __global__ void __launch_bounds__(256, 1) fit32_kernel(const float *Kh_all, cons
     W[e] = 0.f;
   }
   for (int i = tid; i < NP; i += nthr) {
-    yv[i] = i < n ? (float)y[(size_t)i * m] : 0.f;
+    yv[i] = i < n ? (float)((y[(size_t)i * m] - mu_y) * isd_y) : 0.f;
     dg[i] = i < n ? Kh[(size_t)i * n + i] : 1.f;
   }
   if (tid == 0) bad = 0;
@@ -421,7 +473,7 @@ __global__ void __launch_bounds__(256, 1) fit32_kernel(const float *Kh_all, cons
         sl += ol + e;
       }
       if (hl == 0 && i < n) {
-        const double yi = y[(size_t)i * m];
+        const double yi = (y[(size_t)i * m] - mu_y) * isd_y;
         const float yh = (float)yi, yl = (float)(yi - (double)yh);
         rv[i] = (yh - sh) + (yl - sl);
       }
@@ -432,37 +484,23 @@ __global__ void __launch_bounds__(256, 1) fit32_kernel(const float *Kh_all, cons
   solve(rv, rv);
   for (int k = tid; k < NP; k += nthr) al[k] += rv[k];
   __syncthreads();
-  // outputs: W (row stride ld) for the operand packing, alpha into the side input
-  if (SMEM)
-    for (int e = tid; e < NP * ld; e += nthr) Wws[(size_t)bt * NP * ld + e] = W[e];
+  // outputs: the operand images of W (packed here from shared memory; the
+  // global variant leaves W in the workspace for pack_kernel), alpha into the
+  // side input
+  if (SMEM) pack_elems(W, ld, plan, bop + (size_t)bt * plan.image_floats, tid, nthr);
   const int cf = xt_chunk_floats(DP);
   float *xa = xt + (size_t)bt * (npad / BOUTE_KCHUNK) * cf + 2 * BOUTE_KCHUNK * DP;
   for (int k = tid; k < npad; k += nthr)
     xa[(size_t)(k / BOUTE_KCHUNK) * cf + k % BOUTE_KCHUNK] = k < n ? al[k] : 0.f;
 }
 
-// ---- operand images of L^-1 as tf32 hi/lo, swizzled ---------------------------
+// ---- operand images of L^-1 as tf32 hi/lo, swizzled (global-workspace fit) ----
 __global__ void pack_kernel(const float *Wws, PostPlan plan, float *bop, const int *status) {
   if (*status == BOUTE_ERR_NOT_PD) return;
   const size_t bt = blockIdx.y;
-  const int n = plan.n, ld = plan.npad + 1;
-  const float *W = Wws + bt * plan.npad * ld;
-  float *img = bop + bt * plan.image_floats;
-  const long long total = (long long)plan.ncols * plan.npad;
-  for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < total;
-       e += (long long)gridDim.x * blockDim.x) {
-    const int g = (int)(e / plan.npad), k = (int)(e % plan.npad);
-    const int p = g >> 8, c = k / BOUTE_KCHUNK;
-    if (c >= plan.kc[p]) continue;
-    const float v = (k < n && g < n && k <= g) ? W[(size_t)g * ld + k] : 0.f;
-    const float hi = tf32_rna(v);
-    const float lo = tf32_rna(v - hi);
-    const int ncol = plan.ncol[p];
-    float *blk = img + plan.off[p] + (long long)c * 2 * ncol * BOUTE_KCHUNK;
-    const int o = sw128_off(g - plan.col0[p], k % BOUTE_KCHUNK);
-    blk[o] = hi;
-    blk[ncol * BOUTE_KCHUNK + o] = lo;
-  }
+  const int ld = plan.npad + 1;
+  pack_elems(Wws + bt * plan.npad * ld, ld, plan, bop + bt * plan.image_floats,
+             (long long)blockIdx.x * blockDim.x + threadIdx.x, (long long)gridDim.x * blockDim.x);
 }
 
 }  // namespace
@@ -475,29 +513,45 @@ int launch_standardize(const double *Y, int B, int n, int m, double *Ys, cudaStr
 
 size_t fit_smem_bytes(int np) { return (2 * (size_t)np * (np + 1) + 6 * (size_t)np) * sizeof(float); }
 
-int launch_fit(Gp *gp, const double *X, const double *Ys, const double *ls, const double *s2,
-               const double *noise, cudaStream_t s) {
+// Ys: standardised outcomes, or raw outcomes when standardize != 0.
+static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standardize,
+                           const double *ls, const double *s2, const double *noise,
+                           cudaStream_t s) {
   const int n = gp->n, d = gp->d, m = gp->m, BM = gp->B * gp->m;
-  cudaMemsetAsync(gp->status, 0, sizeof(int), s);  // a new fit starts with a clean status
-  dim3 g1((n + 7) / 8, (n + 7) / 8, BM);
-  kernel_matrix_kernel<<<g1, dim3(8, 8), 0, s>>>(X, n, d, m, ls, s2, noise, gp->Kh, gp->Kl);
-  prep_kernel<<<dim3(std::max(1, gp->plan.npad * gp->DP / 256), BM), 256, 0, s>>>(
-      X, n, d, m, gp->DP, gp->plan.npad, ls, s2, gp->xt, gp->invls, gp->s2f);
-  const size_t smem = fit_smem_bytes(gp->plan.npad);
+  const int npad = gp->plan.npad;
+  const int tn = (n + 15) / 16, nkt = tn * tn;
+  const int nprep = std::max(1, std::min(8, npad * gp->DP / 256));
+  fit_setup_kernel<<<dim3(nkt + nprep, BM), 256, 0, s>>>(X, n, d, m, gp->DP, npad, ls, s2, noise,
+                                                         gp->Kh, gp->Kl, gp->xt, gp->s2f, nkt,
+                                                         nprep, gp->status);
+  const size_t smem = fit_smem_bytes(npad);
   if (smem <= 220 * 1024) {
     cudaFuncSetAttribute(fit32_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);
-    fit32_kernel<true><<<BM, 256, smem, s>>>(gp->Kh, gp->Kl, Ys, n, m, gp->Aws, gp->Wws, gp->xt,
-                                             gp->DP, gp->plan.npad, gp->status);
+    fit32_kernel<true><<<BM, 256, smem, s>>>(gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws,
+                                             gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop,
+                                             gp->status);
+    count_launch(2);
   } else {
-    fit32_kernel<false><<<BM, 256, 6 * gp->plan.npad * sizeof(float), s>>>(
-        gp->Kh, gp->Kl, Ys, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, gp->plan.npad, gp->status);
+    fit32_kernel<false><<<BM, 256, 6 * npad * sizeof(float), s>>>(
+        gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan,
+        gp->bop, gp->status);
+    const long long tot = (long long)gp->plan.ncols * npad;
+    pack_kernel<<<dim3((unsigned)std::min<long long>((tot + 255) / 256, 4096), BM), 256, 0, s>>>(
+        gp->Wws, gp->plan, gp->bop, gp->status);
+    count_launch(3);
   }
-  const long long tot = (long long)gp->plan.ncols * gp->plan.npad;
-  pack_kernel<<<dim3((unsigned)std::min<long long>((tot + 255) / 256, 4096), BM), 256, 0, s>>>(
-      gp->Wws, gp->plan, gp->bop, gp->status);
-  count_launch(4);
   return last_launch_status();
+}
+
+int launch_fit(Gp *gp, const double *X, const double *Ys, const double *ls, const double *s2,
+               const double *noise, cudaStream_t s) {
+  return launch_fit_impl(gp, X, Ys, 0, ls, s2, noise, s);
+}
+
+int launch_fit_raw(Gp *gp, const double *X, const double *Y, const double *ls, const double *s2,
+                   const double *noise, cudaStream_t s) {
+  return launch_fit_impl(gp, X, Y, 1, ls, s2, noise, s);
 }
 
 }  // namespace boute

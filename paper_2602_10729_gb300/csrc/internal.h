@@ -16,7 +16,6 @@ struct Gp {
   float *Wws;      // B*m x np x (np+1): L^-1 (lower, row stride np+1)
   float *bop;     // B*m x plan.image_floats: L^-1 as tf32 hi/lo operand images
   float *xt;      // B*m x nchunk x xt_chunk_floats(DP): X/lengthscale hi/lo, alpha
-  float *invls;   // B*m x 2 x DP: 1 / lengthscale as fp32 hi/lo
   float *s2f;     // B*m: outputscale
   int *status;    // device status word (first error wins)
 };

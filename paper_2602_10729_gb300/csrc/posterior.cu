@@ -50,7 +50,7 @@ struct Layout {
 struct PostArgs {
   const float *Xc;
   float *mean, *var;
-  const float *bop, *xt, *invls, *s2f;
+  const float *bop, *xt, *s2f;
   int *status;
   long long N;
   int B, m, d, n;
@@ -397,7 +397,6 @@ int launch_dp(const Gp *gp, const float *Xc, long long N, float *mean, float *va
   a.var = var;
   a.bop = gp->bop;
   a.xt = gp->xt;
-  a.invls = gp->invls;
   a.s2f = gp->s2f;
   a.status = gp->status;
   a.N = N;
