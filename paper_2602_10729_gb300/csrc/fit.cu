@@ -162,28 +162,34 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
 }
 
 // ---- factorisation: one block per (problem, objective) -------------------------
-// Blocked right-looking Cholesky of K (its fp32 rounding) in 32-column panels:
-// one warp factors each diagonal block in registers, then the block forms the
-// panel below it (row-parallel forward substitution) and the trailing update
-// (4 x 4 register tiles). The diagonal blocks of W = L^-1 are inverted
-// afterwards, one warp each, concurrently, and W is completed block
-// row by block row, W_IJ = -W_II sum_{K=J}^{I-1} L_IK W_KJ. fp32 arithmetic on
-// the FP32 pipes: the fp32 factor is as accurate as the posterior needs, while
-// alpha, which carries the condition number, gets one step of iterative
-// refinement against the fp64-accurate K = hi + lo with double-float
-// residuals. A pivot at or below 16 * eps32 times its original diagonal entry
-// counts as not positive. Matrix and inverse live in shared memory (row stride
-// NP+1, NP = n rounded up to 32, padded with the identity) when they fit, else
-// in the handle's global workspace.
+// Blocked right-looking Cholesky of K (its fp32 rounding) in 32-column panels,
+// with W = L^-1 formed block row by block row inside the same loop: one warp
+// factors and inverts each diagonal block in registers, the panel below is the
+// product with that inverse, W_pJ = -W_pp sum_{K=J}^{p-1} L_pK W_KJ, and the
+// trailing update uses 4 x 4 register tiles. fp32 arithmetic on the FP32
+// pipes: the fp32 factor is as accurate as the posterior needs, while alpha,
+// which carries the condition number, gets one step of iterative refinement
+// against the fp64-accurate K = hi + lo with double-float residuals. A pivot
+// at or below 16 * eps32 times its original diagonal entry counts as not
+// positive. Matrix and inverse live in shared memory (row stride NP+1, NP = n
+// rounded up to 32, padded with the identity) when they fit, else in the
+// handle's global workspace.
+// Threads per block of the two variants: the shared-memory variant runs more
+// warps to hide the latency of its short, dependent phases.
 template <bool SMEM>
-__global__ void __launch_bounds__(256, 1) fit32_kernel(const float *Kh_all, const float *Kl_all,
-                                                    const double *Ys, int standardize, int n,
-                                                    int m, float *Aws, float *Wws, float *xt,
-                                                    int DP, int npad, PostPlan plan, float *bop,
-                                                    int *status) {
-  extern __shared__ float sm[];
+constexpr int fit_threads() { return SMEM ? 384 : 256; }
+
+template <bool SMEM>
+__global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
+    const float *Kh_all, const float *Kl_all, const double *Ys, int standardize, int n, int m,
+    float *Aws, float *Wws, float *xt, int DP, int npad, PostPlan plan, float *bop, int kl_smem,
+    int *status) {
+  extern __shared__ __align__(16) float sm[];
   __shared__ int bad;
-  __shared__ double red[8], ymu, yisd;
+  __shared__ uint64_t lbar;
+  __shared__ double red[16], ymu, yisd;
+  __shared__ __align__(16) float colb[2][32];
+  __shared__ __align__(16) float wrow[2][32];
   const int bt = blockIdx.x, b = bt / m, t = bt % m;
   const int tid = threadIdx.x, nthr = blockDim.x, lane = tid & 31, warp = tid >> 5,
             nw = nthr >> 5;
@@ -191,27 +197,72 @@ __global__ void __launch_bounds__(256, 1) fit32_kernel(const float *Kh_all, cons
   const float *Kh = Kh_all + (size_t)bt * n * n, *Kl = Kl_all + (size_t)bt * n * n;
   float *A = SMEM ? sm : Aws + (size_t)bt * NP * ld;
   float *W = SMEM ? sm + (size_t)NP * ld : Wws + (size_t)bt * NP * ld;
-  float *vec = SMEM ? sm + 2 * (size_t)NP * ld : sm;  // col, dg, y, tv, al, r: 6 x NP
-  float *dg = vec + NP, *yv = vec + 2 * NP, *tv = vec + 3 * NP, *al = vec + 4 * NP,
+  float *vec = SMEM ? sm + 2 * (size_t)NP * ld : sm;  // ylo, dg, y, tv, al, r: 6 x NP
+  float *ylo = vec, *dg = vec + NP, *yv = vec + 2 * NP, *tv = vec + 3 * NP, *al = vec + 4 * NP,
         *rv = vec + 5 * NP;
   const double *y = Ys + (size_t)b * n * m + t;
+  // A = K (hi; the lower triangle becomes L, the upper triangle keeps K for the
+  // residual), padded with the identity to NP x NP. In shared memory with n
+  // even, K hi (and, for n <= 128, K lo) arrive by bulk copy, K hi staged in
+  // the W area, while the outcomes are standardised.
+  float *Kls = kl_smem ? vec + 6 * NP : nullptr;  // K lo, n x n (shared)
+  const bool bulk = SMEM && (n % 2 == 0);
+  if (bulk) {
+    if (tid == 0) {
+      mbar_init(&lbar, 1);
+      fence_mbar_init();
+    }
+    __syncthreads();
+    if (tid == 0) {
+      const uint32_t bytes = (uint32_t)n * n * sizeof(float);
+      mbar_arrive_expect_tx(&lbar, kl_smem ? 2 * bytes : bytes);
+      bulk_g2s(W, Kh, bytes, &lbar);
+      if (kl_smem) bulk_g2s(Kls, Kl, bytes, &lbar);
+    }
+  } else {  // eight independent loads per thread in flight before their stores
+    const int nn = n * n;
+    for (int base = 0; base < nn; base += 8 * nthr) {
+      float v[8], w8[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int e = base + j * nthr + tid;
+        v[j] = e < nn ? Kh[e] : 0.f;
+        w8[j] = (e < nn && kl_smem) ? Kl[e] : 0.f;
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int e = base + j * nthr + tid;
+        if (e < nn) {
+          const int i = e / n, k = e - i * n;
+          A[(size_t)i * ld + k] = v[j];
+          if (kl_smem) Kls[e] = w8[j];
+        }
+      }
+    }
+  }
+  for (int e = tid; e < (NP - n) * NP; e += nthr) {
+    const int i = n + e / NP, k = e % NP;
+    if (k <= i) A[(size_t)i * ld + k] = (k == i) ? 1.f : 0.f;
+  }
   // standardize != 0: Ys holds raw outcomes; this column is standardised here
   // (zero mean, unit sample standard deviation, as standardize_kernel does)
-  if (standardize) {
-    double sum = 0.0;
-    for (int i = tid; i < n; i += nthr) sum += y[(size_t)i * m];
-    const double mean = block_sum(sum, red) / n;
-    double ss = 0.0;
-    for (int i = tid; i < n; i += nthr) {
-      const double z = y[(size_t)i * m] - mean;
-      ss += z * z;
-    }
-    ss = block_sum(ss, red);
-    double sd = n > 1 ? sqrt(ss / (n - 1)) : 1.0;
-    if (!(sd >= 1e-8)) sd = 1.0;
-    if (tid == 0) {
-      ymu = mean;
-      yisd = 1.0 / sd;
+  if (standardize) {  // warp 0 alone: few fp64 instructions
+    if (warp == 0) {
+      double sum = 0.0;
+      for (int i = lane; i < n; i += 32) sum += y[(size_t)i * m];
+      const double mean = warp_sum(sum) / n;
+      double ss = 0.0;
+      for (int i = lane; i < n; i += 32) {
+        const double z = y[(size_t)i * m] - mean;
+        ss += z * z;
+      }
+      ss = warp_sum(ss);
+      double sd = n > 1 ? sqrt(ss / (n - 1)) : 1.0;
+      if (!(sd >= 1e-8)) sd = 1.0;
+      if (lane == 0) {
+        ymu = mean;
+        yisd = 1.0 / sd;
+      }
     }
   } else if (tid == 0) {
     ymu = 0.0;
@@ -219,190 +270,199 @@ __global__ void __launch_bounds__(256, 1) fit32_kernel(const float *Kh_all, cons
   }
   __syncthreads();
   const double mu_y = ymu, isd_y = yisd;
-
-  for (int e = tid; e < NP * ld; e += nthr) {
-    const int i = e / ld, k = e % ld;
-    float v = 0.f;
-    if (k <= i && k < NP) v = (i < n) ? Kh[(size_t)i * n + k] : (i == k ? 1.f : 0.f);
-    A[e] = v;
-    W[e] = 0.f;
+  if (bulk) {
+    if (!mbar_wait(&lbar, 0)) {  // the copy never completed: report, drain, leave
+      if (tid == 0) set_status(status, BOUTE_ERR_TIMEOUT);
+      mbar_wait(&lbar, 0);
+      return;
+    }
+    for (int e = tid; e < n * n; e += nthr) {
+      const int i = e / n, k = e - i * n;
+      A[(size_t)i * ld + k] = W[e];
+    }
+    __syncthreads();
   }
-  for (int i = tid; i < NP; i += nthr) {
-    yv[i] = i < n ? (float)((y[(size_t)i * m] - mu_y) * isd_y) : 0.f;
-    dg[i] = i < n ? Kh[(size_t)i * n + i] : 1.f;
+  for (int i = tid; i < NP; i += nthr) {  // standardised y as an fp32 pair
+    const double ys = i < n ? (y[(size_t)i * m] - mu_y) * isd_y : 0.0;
+    yv[i] = (float)ys;
+    ylo[i] = (float)(ys - (double)yv[i]);
+    dg[i] = A[(size_t)i * ld + i];
   }
   if (tid == 0) bad = 0;
   __syncthreads();
-  // ---- blocked Cholesky, 32-column panels --------------------------------------
+  // ---- blocked Cholesky and W = L^-1, 32-column panels -------------------------
+  // Iteration p: (a) warp 0 factors the diagonal block, A_pp = L_pp L_pp^T,
+  // and inverts it, W_pp = L_pp^-1, both register-resident (lane = row of the
+  // block); (b) the panel below, L_rp = A_rp W_pp^T, goes to the still-unused
+  // block column p of W, and T_pJ = sum_{K=J}^{p-1} L_pK W_KJ (J < p) is
+  // parked, transposed, in the unused upper triangle of W; (c) the trailing
+  // update A_ij -= sum_q L_iq L_jq (rows and columns below the panel), the
+  // copy of the panel into A, and W_pJ = -W_pp T_pJ. 4 x 4 register tiles.
   const int nb = NP / 32;
   const unsigned FULL = 0xffffffffu;
   for (int p = 0; p < nb; ++p) {
     const int p0 = 32 * p;
-    // (a) one warp factors the diagonal block, register-resident (lane = row):
-    //     at step c, column c of L is formed and broadcast by shuffles to
-    //     update the trailing rows of the block.
     if (warp == 0) {
-      float a[32];
+      float a[32], w[32];  // row lane of A_pp (becoming L_pp) and of R (becoming W_pp)
       float *Ar = A + (size_t)(p0 + lane) * ld + p0;
 #pragma unroll
-      for (int c = 0; c < 32; ++c) a[c] = (c <= lane) ? Ar[c] : 0.f;
+      for (int c = 0; c < 32; ++c) {
+        a[c] = (c <= lane) ? Ar[c] : 0.f;
+        w[c] = (c == lane) ? 1.f : 0.f;
+      }
       const float dgl = dg[p0 + lane];
       bool ok = true;
+      float myinv = 0.f;
+      float pivn = __shfl_sync(FULL, a[0], 0);
 #pragma unroll
       for (int c = 0; c < 32; ++c) {
-        const float piv = __shfl_sync(FULL, a[c], c);
+        const float piv = pivn;
         if (!(piv > 16.f * 1.1920929e-7f * __shfl_sync(FULL, dgl, c))) ok = false;
         float inv = rsqrtf(piv);
-        inv = inv * fmaf(-0.5f * piv * inv, inv, 1.5f);  // one Newton step
+        inv = inv * fmaf(-0.5f * piv * inv, inv, 1.5f);  // one Newton step; 1 / L_cc
         const float l = lane > c ? a[c] * inv : (lane == c ? piv * inv : 0.f);
-        a[c] = l;
-#pragma unroll
-        for (int c2 = 0; c2 < 32; ++c2) {
-          if (c2 > c) {
-            const float lc2 = __shfl_sync(FULL, l, c2);
-            if (lane >= c2) a[c2] = fmaf(-l, lc2, a[c2]);
-          }
+        if (c < 31) {  // the next pivot straight from lane c+1, ahead of the rest
+          const float an = __shfl_sync(FULL, a[c + 1], c + 1);
+          const float lc = __shfl_sync(FULL, l, c + 1);
+          pivn = fmaf(-lc, lc, an);
         }
+        a[c] = l;
+        float *cb = colb[c & 1];  // column c of L_pp
+        float *wr = wrow[c & 1];  // row c of R (W_pp's row c times L_cc)
+        cb[lane] = l;
+        if (lane == c) {
+          myinv = inv;
+#pragma unroll
+          for (int k = 0; k <= c; ++k) wr[k] = w[k];
+        }
+        __syncwarp();
+        // Entries above a lane's diagonal collect garbage that is never
+        // stored, so the updates need no predicates.
+#pragma unroll
+        for (int c2 = c + 1; c2 < 32; ++c2) a[c2] = fmaf(-l, cb[c2], a[c2]);
+        // R_i -= L_ic W_c = (L_ic / L_cc) R_c for the rows below c
+        const float lw = lane > c ? l * inv : 0.f;
+#pragma unroll
+        for (int k = 0; k <= c; ++k) w[k] = fmaf(-lw, wr[k], w[k]);
+      }
+      float *Wr = W + (size_t)(p0 + lane) * ld + p0;
+#pragma unroll
+      for (int c = 0; c < 32; ++c) {
+        if (c <= lane) Ar[c] = a[c];
+        Wr[c] = w[c] * myinv;
       }
       if (!ok && lane == 0) bad = 1;
-#pragma unroll
-      for (int c = 0; c < 32; ++c)
-        if (c <= lane) Ar[c] = a[c];
     }
     __syncthreads();
     if (bad) break;
     const int r0 = p0 + 32, rows = NP - r0;
-    const float *Lp = A + (size_t)p0 * ld + p0;  // L_pp, lower
+    // (b)
     {
-      // (b) panel below the diagonal block: row r solves x L_pp^T = A_r,p
-      //     by forward substitution (x in registers), one row per thread
-      for (int r = r0 + tid; r < NP; r += nthr) {
-        float *ar = A + (size_t)r * ld + p0;
-        float x[32];
+      const int ntr = (rows / 4) * 8, ntt = p * 64;
+      for (int tix = tid; tix < ntr + ntt; tix += nthr) {
+        float acc[4][4] = {};
+        if (tix < ntr) {  // L_rp tile: rows i0.., columns c0.. of the panel
+          const int i0 = r0 + 4 * (tix >> 3), c0 = 4 * (tix & 7);
+#pragma unroll 4
+          for (int q = 0; q < 32; ++q) {
+            float x[4], y4[4];
 #pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          float s0 = ar[c], s1 = 0.f, s2 = 0.f, s3 = 0.f;
+            for (int u = 0; u < 4; ++u) {
+              x[u] = A[(size_t)(i0 + u) * ld + p0 + q];
+              y4[u] = W[(size_t)(p0 + c0 + u) * ld + p0 + q];
+            }
 #pragma unroll
-          for (int q = 0; q < 32; q += 4) {
-            if (q < c) s0 = fmaf(-x[q], Lp[(size_t)c * ld + q], s0);
-            if (q + 1 < c) s1 = fmaf(-x[q + 1], Lp[(size_t)c * ld + q + 1], s1);
-            if (q + 2 < c) s2 = fmaf(-x[q + 2], Lp[(size_t)c * ld + q + 2], s2);
-            if (q + 3 < c) s3 = fmaf(-x[q + 3], Lp[(size_t)c * ld + q + 3], s3);
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+              for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
           }
-          x[c] = ((s0 + s1) + (s2 + s3)) / Lp[(size_t)c * ld + c];
-        }
 #pragma unroll
-        for (int c = 0; c < 32; ++c) ar[c] = x[c];
+          for (int u = 0; u < 4; ++u)
+#pragma unroll
+            for (int v = 0; v < 4; ++v) W[(size_t)(i0 + u) * ld + p0 + c0 + v] = acc[u][v];
+        } else {  // T_pJ tile (8 x 8 tiles per 32 x 32 block)
+          const int e = tix - ntr, J = e >> 6, rb = 4 * ((e >> 3) & 7), cb = 4 * (e & 7);
+#pragma unroll 4
+          for (int q = 32 * J; q < p0; ++q) {
+            float x[4], y4[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              x[u] = A[(size_t)(p0 + rb + u) * ld + q];
+              y4[u] = W[(size_t)q * ld + 32 * J + cb + u];
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+              for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+#pragma unroll
+            for (int v = 0; v < 4; ++v) W[(size_t)(32 * J + cb + v) * ld + p0 + rb + u] = acc[u][v];
+        }
       }
     }
     __syncthreads();
-    // (c) trailing update of the lower triangle, 4 x 4 register tiles:
-    //     A_ij -= sum_q L_i,p0+q L_j,p0+q for r0 <= j <= i < NP
-    const int th = rows / 4;
-    const int ntile = th * (th + 1) / 2;
-    for (int tix = tid; tix < ntile; tix += nthr) {
-      int ti = (int)((sqrtf(8.f * tix + 1.f) - 1.f) * 0.5f);
-      while (ti * (ti + 1) / 2 > tix) --ti;
-      while ((ti + 1) * (ti + 2) / 2 <= tix) ++ti;
-      const int tj = tix - ti * (ti + 1) / 2;
-      const int i0 = r0 + 4 * ti, j0 = r0 + 4 * tj;
-      float acc[4][4] = {};
+    // (c)
+    {
+      const int th = rows / 4, ntile = th * (th + 1) / 2, nwt = p * 64;
+      for (int tix = tid; tix < ntile + nwt; tix += nthr) {
+        float acc[4][4] = {};
+        if (tix < ntile) {  // trailing tile (i, j) of the lower triangle
+          int ti = (int)((sqrtf(8.f * tix + 1.f) - 1.f) * 0.5f);
+          while (ti * (ti + 1) / 2 > tix) --ti;
+          while ((ti + 1) * (ti + 2) / 2 <= tix) ++ti;
+          const int tj = tix - ti * (ti + 1) / 2;
+          const int i0 = r0 + 4 * ti, j0 = r0 + 4 * tj;
 #pragma unroll 4
-      for (int q = 0; q < 32; ++q) {
-        float x[4], y4[4];
+          for (int q = 0; q < 32; ++q) {
+            float x[4], y4[4];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          x[u] = A[(size_t)(i0 + u) * ld + p0 + q];
-          y4[u] = A[(size_t)(j0 + u) * ld + p0 + q];
+            for (int u = 0; u < 4; ++u) {
+              x[u] = W[(size_t)(i0 + u) * ld + p0 + q];
+              y4[u] = W[(size_t)(j0 + u) * ld + p0 + q];
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+              for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+              if (ti != tj || v <= u) A[(size_t)(i0 + u) * ld + j0 + v] -= acc[u][v];
+        } else {  // W_pJ tile = -W_pp T_pJ (W_pp lower, zeros above)
+          const int e = tix - ntile, J = e >> 6, rb = 4 * ((e >> 3) & 7), cb = 4 * (e & 7);
+#pragma unroll 4
+          for (int q = 0; q < 32; ++q) {
+            float x[4], y4[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              x[u] = W[(size_t)(p0 + rb + u) * ld + p0 + q];
+              y4[u] = W[(size_t)(32 * J + cb + u) * ld + p0 + q];
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+              for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+#pragma unroll
+            for (int v = 0; v < 4; ++v) W[(size_t)(p0 + rb + u) * ld + 32 * J + cb + v] = -acc[u][v];
         }
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-#pragma unroll
-          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
       }
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-#pragma unroll
-        for (int v = 0; v < 4; ++v)
-          if (ti != tj || v <= u) A[(size_t)(i0 + u) * ld + j0 + v] -= acc[u][v];
+      for (int e = tid; e < rows * 32; e += nthr) {  // the panel into A
+        const size_t o = (size_t)(r0 + (e >> 5)) * ld + p0 + (e & 31);
+        A[o] = W[o];
+      }
     }
     __syncthreads();
   }
   if (bad) {
     if (tid == 0) set_status(status, BOUTE_ERR_NOT_PD);
     return;
-  }
-  // ---- diagonal blocks of W = L^-1: warp I inverts L_II (lane = column) --------
-  for (int I = warp; I < nb; I += nw) {
-    const float *Lb = A + (size_t)(32 * I) * ld + 32 * I;
-    float w[32];
-#pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      float s0 = (i == lane) ? 1.f : 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll
-      for (int l = 0; l < 32; l += 4) {
-        if (l < i) s0 = fmaf(-Lb[(size_t)i * ld + l], w[l], s0);
-        if (l + 1 < i) s1 = fmaf(-Lb[(size_t)i * ld + l + 1], w[l + 1], s1);
-        if (l + 2 < i) s2 = fmaf(-Lb[(size_t)i * ld + l + 2], w[l + 2], s2);
-        if (l + 3 < i) s3 = fmaf(-Lb[(size_t)i * ld + l + 3], w[l + 3], s3);
-      }
-      w[i] = ((s0 + s1) + (s2 + s3)) / Lb[(size_t)i * ld + i];
-    }
-    float *Wb = W + (size_t)(32 * I) * ld + 32 * I;
-#pragma unroll
-    for (int i = 0; i < 32; ++i) Wb[(size_t)i * ld + lane] = w[i];
-  }
-  __syncthreads();
-  // ---- off-diagonal blocks of W = L^-1, block row by block row ------------------
-  // W_IJ = -W_II T_IJ, T_IJ = sum_{K=J}^{I-1} L_IK W_KJ; T is parked, transposed,
-  // in the (unused) upper triangle of W. 4 x 4 register tiles.
-  for (int I = 1; I < nb; ++I) {
-    const int nt = I * 64;  // J < I, 8 x 8 tiles per block
-    for (int tix = tid; tix < nt; tix += nthr) {
-      const int J = tix / 64, rb = 4 * ((tix / 8) % 8), cb = 4 * (tix % 8);
-      float acc[4][4] = {};
-#pragma unroll 4
-      for (int q = 32 * J; q < 32 * I; ++q) {
-        float x[4], y4[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          x[u] = A[(size_t)(32 * I + rb + u) * ld + q];
-          y4[u] = W[(size_t)q * ld + 32 * J + cb + u];
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-#pragma unroll
-          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-#pragma unroll
-        for (int v = 0; v < 4; ++v)
-          W[(size_t)(32 * J + cb + v) * ld + 32 * I + rb + u] = acc[u][v];
-    }
-    __syncthreads();
-    for (int tix = tid; tix < nt; tix += nthr) {
-      const int J = tix / 64, rb = 4 * ((tix / 8) % 8), cb = 4 * (tix % 8);
-      float acc[4][4] = {};
-#pragma unroll 4
-      for (int q = 0; q < 32; ++q) {  // W_II is lower triangular: zeros above
-        float x[4], y4[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          x[u] = W[(size_t)(32 * I + rb + u) * ld + 32 * I + q];
-          y4[u] = W[(size_t)(32 * J + cb + u) * ld + 32 * I + q];
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-#pragma unroll
-          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-#pragma unroll
-        for (int v = 0; v < 4; ++v) W[(size_t)(32 * I + rb + u) * ld + 32 * J + cb + v] = -acc[u][v];
-    }
-    __syncthreads();
   }
   // ---- alpha0 = W^T (W y), refined once against K = hi + lo ----------------------
   // out = W^T (W rhs): thread per row, then thread per column (4 accumulators)
@@ -436,32 +496,22 @@ __global__ void __launch_bounds__(256, 1) fit32_kernel(const float *Kh_all, cons
     __syncthreads();
   };
   solve(yv, al);
-  // residual r = y - K alpha0 in double-float: half a warp per row, all the
-  // row's loads issued before the arithmetic
-  {
+  // residual r = y - K alpha0 in double-float. Shared-memory variant: K hi
+  // from the upper triangle of A and its diagonal, K lo from shared memory
+  // when it fits there; half a warp per row.
+  if (SMEM) {
     const int half = lane >> 4, hl = lane & 15;
-    for (int i = 2 * warp + half; i < NP; i += 2 * nw) {
+    for (int i = 2 * warp + half; i < NP; i += 2 * nw) {  // NP: both halves, same trips
       float sh = 0.f, sl = 0.f;
-      if (i < n) {
-        const float *kh = Kh + (size_t)i * n, *kl = Kl + (size_t)i * n;
-        for (int k0 = 0; k0 < n; k0 += 128) {
-          float h8[8], l8[8], a8[8];
-#pragma unroll
-          for (int u = 0; u < 8; ++u) {
-            const int k = k0 + hl + 16 * u;
-            h8[u] = k < n ? kh[k] : 0.f;
-            l8[u] = k < n ? kl[k] : 0.f;
-            a8[u] = k < n ? al[k] : 0.f;
-          }
-#pragma unroll
-          for (int u = 0; u < 8; ++u) {
-            float pr, e, s_, e2;
-            two_prod(h8[u], a8[u], pr, e);
-            two_sum(sh, pr, s_, e2);
-            sh = s_;
-            sl += e2 + fmaf(l8[u], a8[u], e);
-          }
-        }
+      for (int k = hl; k < (i < n ? n : 0); k += 16) {
+        const float h = k < i ? A[(size_t)k * ld + i] : (k > i ? A[(size_t)i * ld + k] : dg[i]);
+        const float l = kl_smem ? Kls[(size_t)i * n + k] : Kl[(size_t)i * n + k];
+        const float a = al[k];
+        float pr, e, s_, e2;
+        two_prod(h, a, pr, e);
+        two_sum(sh, pr, s_, e2);
+        sh = s_;
+        sl += e2 + fmaf(l, a, e);
       }
 #pragma unroll
       for (int o = 8; o > 0; o >>= 1) {  // within the half warp
@@ -472,10 +522,51 @@ __global__ void __launch_bounds__(256, 1) fit32_kernel(const float *Kh_all, cons
         sh = s_;
         sl += ol + e;
       }
-      if (hl == 0 && i < n) {
-        const double yi = (y[(size_t)i * m] - mu_y) * isd_y;
-        const float yh = (float)yi, yl = (float)(yi - (double)yh);
-        rv[i] = (yh - sh) + (yl - sl);
+      if (hl == 0 && i < n) rv[i] = (yv[i] - sh) + (ylo[i] - sl);
+    }
+  } else {
+    // global variant: two rows per half warp at a time, all their loads
+    // issued before the arithmetic
+    const int half = lane >> 4, hl = lane & 15;
+    for (int i0 = 2 * warp + half; i0 < NP; i0 += 4 * nw) {
+      const int rows[2] = {i0, i0 + 2 * nw};
+      float sh[2] = {0.f, 0.f}, sl[2] = {0.f, 0.f};
+      for (int k0 = 0; k0 < n; k0 += 128) {
+        float h8[2][8], l8[2][8], a8[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int k = k0 + hl + 16 * u;
+          a8[u] = k < n ? al[k] : 0.f;
+#pragma unroll
+          for (int q = 0; q < 2; ++q) {
+            const bool ok = k < n && rows[q] < n;
+            h8[q][u] = ok ? Kh[(size_t)rows[q] * n + k] : 0.f;
+            l8[q][u] = ok ? Kl[(size_t)rows[q] * n + k] : 0.f;
+          }
+        }
+#pragma unroll
+        for (int q = 0; q < 2; ++q)
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            float pr, e, s_, e2;
+            two_prod(h8[q][u], a8[u], pr, e);
+            two_sum(sh[q], pr, s_, e2);
+            sh[q] = s_;
+            sl[q] += e2 + fmaf(l8[q][u], a8[u], e);
+          }
+      }
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+#pragma unroll
+        for (int o = 8; o > 0; o >>= 1) {  // within the half warp
+          const float oh = __shfl_xor_sync(FULL, sh[q], o);
+          const float ol = __shfl_xor_sync(FULL, sl[q], o);
+          float s_, e;
+          two_sum(sh[q], oh, s_, e);
+          sh[q] = s_;
+          sl[q] += ol + e;
+        }
+        if (hl == 0 && rows[q] < n) rv[rows[q]] = (yv[rows[q]] - sh[q]) + (ylo[rows[q]] - sl[q]);
       }
     }
   }
@@ -487,7 +578,23 @@ __global__ void __launch_bounds__(256, 1) fit32_kernel(const float *Kh_all, cons
   // outputs: the operand images of W (packed here from shared memory; the
   // global variant leaves W in the workspace for pack_kernel), alpha into the
   // side input
-  if (SMEM) pack_elems(W, ld, plan, bop + (size_t)bt * plan.image_floats, tid, nthr);
+  if (SMEM) {  // one column pass (n <= 160): warp per row g, lane = k % 32
+    float *img = bop + (size_t)bt * plan.image_floats + plan.off[0];
+    const int ncol = plan.ncol[0], kc = plan.kc[0];
+    for (int g = warp; g < ncol; g += nw) {
+      const float *wr = W + (size_t)g * ld;
+      const int o = sw128_off(g, lane);
+#pragma unroll 4
+      for (int c = 0; c < kc; ++c) {
+        const int k = c * BOUTE_KCHUNK + lane;
+        const float v = (k < n && g < n && k <= g) ? wr[k] : 0.f;
+        const float hi = tf32_rna(v), lo = tf32_rna(v - hi);
+        float *blk = img + (size_t)c * 2 * ncol * BOUTE_KCHUNK;
+        blk[o] = hi;
+        blk[ncol * BOUTE_KCHUNK + o] = lo;
+      }
+    }
+  }
   const int cf = xt_chunk_floats(DP);
   float *xa = xt + (size_t)bt * (npad / BOUTE_KCHUNK) * cf + 2 * BOUTE_KCHUNK * DP;
   for (int k = tid; k < npad; k += nthr)
@@ -511,7 +618,16 @@ int launch_standardize(const double *Y, int B, int n, int m, double *Ys, cudaStr
   return last_launch_status();
 }
 
-size_t fit_smem_bytes(int np) { return (2 * (size_t)np * (np + 1) + 6 * (size_t)np) * sizeof(float); }
+// The shared-memory variant holds n up to 160 (n rounded up to 32).
+bool fit_uses_smem(int npad) { return npad <= 160; }
+
+// Dynamic shared memory of the shared-memory fit: A and W (np x (np+1)), six
+// vectors, and K lo (n x n) when n <= 128.
+static bool fit_kl_in_smem(int n) { return n <= 128; }
+size_t fit_smem_bytes(int np, int n) {
+  return (2 * (size_t)np * (np + 1) + 6 * (size_t)np + (fit_kl_in_smem(n) ? (size_t)n * n : 0)) *
+         sizeof(float);
+}
 
 // Ys: standardised outcomes, or raw outcomes when standardize != 0.
 static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standardize,
@@ -524,18 +640,18 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
   fit_setup_kernel<<<dim3(nkt + nprep, BM), 256, 0, s>>>(X, n, d, m, gp->DP, npad, ls, s2, noise,
                                                          gp->Kh, gp->Kl, gp->xt, gp->s2f, nkt,
                                                          nprep, gp->status);
-  const size_t smem = fit_smem_bytes(npad);
-  if (smem <= 220 * 1024) {
+  if (fit_uses_smem(npad)) {
+    const size_t smem = fit_smem_bytes(npad, n);
     cudaFuncSetAttribute(fit32_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);
-    fit32_kernel<true><<<BM, 256, smem, s>>>(gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws,
-                                             gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop,
-                                             gp->status);
+    fit32_kernel<true><<<BM, fit_threads<true>(), smem, s>>>(
+        gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan,
+        gp->bop, fit_kl_in_smem(n) ? 1 : 0, gp->status);
     count_launch(2);
   } else {
-    fit32_kernel<false><<<BM, 256, 6 * npad * sizeof(float), s>>>(
+    fit32_kernel<false><<<BM, fit_threads<false>(), 6 * npad * sizeof(float), s>>>(
         gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan,
-        gp->bop, gp->status);
+        gp->bop, 0, gp->status);
     const long long tot = (long long)gp->plan.ncols * npad;
     pack_kernel<<<dim3((unsigned)std::min<long long>((tot + 255) / 256, 4096), BM), 256, 0, s>>>(
         gp->Wws, gp->plan, gp->bop, gp->status);
