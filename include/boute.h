@@ -162,7 +162,7 @@ int boute_select_topk(const float *acq, int B, long long N, int k, long long *id
  * whose allocator already holds the device's free memory, a latency-critical
  * loop that cannot take the synchronisation cudaFree implies, or a fixed
  * memory budget. The call makes no allocation of any kind.
- *   Limit: 2 * B * ceil(N / 2048) * k * 8 bytes of scratch (0 when
+ *   Limit: 2 * B * ceil(N / 2048) * max(k, 16) * 8 bytes of scratch (0 when
  *   N <= 2048) must not exceed BOUTE_TOPK_NOALLOC_SCRATCH_BYTES; a larger
  *   request returns BOUTE_ERR_UNSUPPORTED before launching anything. Other
  *   argument errors are those of boute_select_topk.

@@ -66,7 +66,8 @@ extern "C" int boute_select_topk_noalloc(const float *acq, int B, long long N, i
   if ((long long)B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;
   const long long nseg = (N + 2047) / 2048;  // first-level segments per problem
   const unsigned long long need =
-      nseg <= 1 ? 0ull : 2ull * (unsigned long long)B * nseg * k * sizeof(unsigned long long);
+      nseg <= 1 ? 0ull
+                : 2ull * (unsigned long long)B * nseg * (k < 16 ? 16 : k) * sizeof(unsigned long long);
   if (need > BOUTE_TOPK_NOALLOC_SCRATCH_BYTES) return BOUTE_ERR_UNSUPPORTED;
   if (!device_is_sm103()) return BOUTE_ERR_UNSUPPORTED;
   void *scratch = nullptr;

@@ -1,7 +1,7 @@
 // Deterministic top-k per problem. Values become 64-bit keys (order-preserving
 // float bits in the high word, the complement of the index in the low word), so
 // one unsigned comparison orders by value descending, then index ascending.
-// Level 1: every block sorts one segment of kSeg keys in shared memory
+// k <= 32 takes a warp-register path (below). Otherwise, level 1: every block sorts one segment of kSeg keys in shared memory
 // (bitonic) and keeps its k largest. Further levels apply the same segment
 // sort to the surviving keys until one segment per problem remains; the last
 // level writes indices and values. All levels are fully parallel across
@@ -85,18 +85,140 @@ __global__ void __launch_bounds__(kThreads) segment_topk_kernel(
   }
 }
 
+// ---- k <= 32: one warp holds a running top 32, one key per lane ----------------
+// Lane i holds the i-th largest key seen so far. A batch of 32 new keys is
+// rejected with one ballot when none beats the current 32nd; otherwise it is
+// sorted across the lanes (bitonic network on shuffles) and merged: the
+// element-wise maximum of the running list and the reversed batch is a bitonic
+// sequence holding the 32 largest keys of both, which five more shuffle steps
+// sort. Each block merges its warps' lists; a second launch merges the blocks'.
+constexpr int kWarpK = 32;
+constexpr int kWarpBlock = 256;  // threads; 8 warps
+constexpr int kWarpBatches = 8;  // batches of 32 keys a warp loads at once
+
+__device__ __forceinline__ unsigned long long shfl64(unsigned long long v, int src) {
+  return __shfl_sync(0xffffffffu, v, src);
+}
+__device__ __forceinline__ unsigned long long shfl_xor64(unsigned long long v, int m) {
+  return __shfl_xor_sync(0xffffffffu, v, m);
+}
+
+// Sort one key per lane, descending across the lanes.
+__device__ __forceinline__ unsigned long long warp_sort_desc(unsigned long long x, int lane) {
+#pragma unroll
+  for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      const unsigned long long y = shfl_xor64(x, stride);
+      const bool desc = (lane & size) == 0 || size == 32;
+      const bool lower = (lane & stride) == 0;
+      const unsigned long long mx = x > y ? x : y, mn = x > y ? y : x;
+      x = (lower == desc) ? mx : mn;
+    }
+  }
+  return x;
+}
+
+// top, s: descending across the lanes. Returns the 32 largest of both, descending.
+__device__ __forceinline__ unsigned long long warp_merge_desc(unsigned long long top,
+                                                              unsigned long long s, int lane) {
+  const unsigned long long r = shfl64(s, 31 - lane);
+  unsigned long long u = top > r ? top : r;
+#pragma unroll
+  for (int stride = 16; stride > 0; stride >>= 1) {
+    const unsigned long long y = shfl_xor64(u, stride);
+    const bool lower = (lane & stride) == 0;
+    u = lower ? (u > y ? u : y) : (u > y ? y : u);
+  }
+  return u;
+}
+
+// Block blockIdx.x of problem blockIdx.y covers entries [x * per_block,
+// (x+1) * per_block) of a row of `len` (values when FROM_VALUES, else sorted
+// runs of 32 keys). With idx set (one block per problem) it writes the final
+// k indices and values; otherwise its 32 keys to keys_out.
+template <bool FROM_VALUES>
+__global__ void __launch_bounds__(kWarpBlock) warp_topk_kernel(
+    const float *vals, const unsigned long long *keys_in, long long len, long long per_block,
+    unsigned long long *keys_out, const float *acq, long long N, int k, long long *idx,
+    float *val) {
+  __shared__ unsigned long long lists[kWarpBlock / 32][kWarpK];
+  const int b = blockIdx.y, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const long long lo = (long long)blockIdx.x * per_block;
+  const long long hi = std::min<long long>(len, lo + per_block);
+  const size_t row = (size_t)b * len;
+  unsigned long long top = 0ull;  // below every real key
+  for (long long base = lo + (long long)warp * 32 * kWarpBatches; base < hi;
+       base += (long long)kWarpBlock * kWarpBatches) {
+    unsigned long long x[kWarpBatches];
+#pragma unroll
+    for (int u = 0; u < kWarpBatches; ++u) {
+      const long long g = base + 32 * u + lane;
+      x[u] = 0ull;
+      if (g < hi) x[u] = FROM_VALUES ? make_key(__ldcs(vals + row + g), (unsigned)g) : keys_in[row + g];
+    }
+#pragma unroll
+    for (int u = 0; u < kWarpBatches; ++u) {
+      const unsigned long long thr = shfl64(top, 31);
+      if (__ballot_sync(0xffffffffu, x[u] > thr) == 0u) continue;
+      top = warp_merge_desc(top, FROM_VALUES ? warp_sort_desc(x[u], lane) : x[u], lane);
+    }
+  }
+  lists[warp][lane] = top;
+  __syncthreads();
+  if (warp != 0) return;
+#pragma unroll 1
+  for (int w = 1; w < kWarpBlock / 32; ++w) top = warp_merge_desc(top, lists[w][lane], lane);
+  if (idx) {
+    if (lane < k) {
+      const unsigned j = key_index(top);
+      idx[(size_t)b * k + lane] = (long long)j;
+      val[(size_t)b * k + lane] = acq[(size_t)b * N + j];
+    }
+  } else {
+    keys_out[((size_t)b * gridDim.x + blockIdx.x) * kWarpK + lane] = top;
+  }
+}
+
+int launch_topk_warp(const float *acq, int B, long long N, int k, long long *idx, float *val,
+                     void *scratch, cudaStream_t s) {
+  // at most 256 first-level blocks per problem, each a multiple of 2048 entries
+  const long long unit = (long long)kWarpBlock * kWarpBatches;
+  long long per_block = unit;
+  while ((N + per_block - 1) / per_block > 256) per_block += unit;
+  const long long G = (N + per_block - 1) / per_block;
+  if (G == 1) {
+    warp_topk_kernel<true><<<dim3(1, B), kWarpBlock, 0, s>>>(acq, nullptr, N, per_block, nullptr,
+                                                              acq, N, k, idx, val);
+    count_launch(1);
+    return last_launch_status();
+  }
+  unsigned long long *keys = (unsigned long long *)scratch;
+  warp_topk_kernel<true><<<dim3((unsigned)G, B), kWarpBlock, 0, s>>>(
+      acq, nullptr, N, per_block, keys, acq, N, k, nullptr, nullptr);
+  const long long len2 = G * kWarpK;
+  warp_topk_kernel<false><<<dim3(1, B), kWarpBlock, 0, s>>>(nullptr, keys, len2, len2, nullptr,
+                                                             acq, N, k, idx, val);
+  count_launch(2);
+  return last_launch_status();
+}
+
 }  // namespace
 
-// Scratch for the levels after the first: two ping-pong key arrays.
+// Scratch for the levels after the first: two ping-pong key arrays of
+// ceil(N / 2048) * k keys per problem (segment path), or at most
+// ceil(N / 2048) runs of 32 keys per problem (warp path, k <= 32); k is
+// counted as at least 16 so that one bound covers both.
 size_t topk_scratch_bytes(int B, long long N, int k) {
   const long long g1 = (N + kSeg - 1) / kSeg;
   if (g1 <= 1) return 16;
-  return 2 * (size_t)B * g1 * k * sizeof(unsigned long long) + 16;
+  return 2 * (size_t)B * g1 * std::max(k, 16) * sizeof(unsigned long long) + 16;
 }
 
 int launch_topk(const float *acq, int B, long long N, int k, long long *idx, float *val,
                 void *scratch, cudaStream_t s) {
   if (k > kSeg / 2) return BOUTE_ERR_UNSUPPORTED;
+  if (k <= kWarpK) return launch_topk_warp(acq, B, N, k, idx, val, scratch, s);
   long long len = N;
   long long nseg = (len + kSeg - 1) / kSeg;
   unsigned long long *ping = (unsigned long long *)scratch;

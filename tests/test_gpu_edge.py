@@ -177,17 +177,22 @@ def test_far_candidates_and_zero_variance_ehvi():
     compare(hp)
 
 
-def test_topk_ties_nan_and_negative_zero():
+# k <= 32 takes the warp-register path, larger k the segment sort; N spans one
+# block, several, and more than 256 first-level blocks (larger blocks)
+@pytest.mark.parametrize("N,k", [(5000, 40), (5000, 32), (5000, 1), (2048, 7), (40, 32),
+                                 (700_001, 32), (700_001, 17), (70_000, 33)])
+def test_topk_ties_nan_and_negative_zero(N, k):
     import torch
 
     from paper_2602_10729_gb300 import boute as bt
     rng = np.random.default_rng(11)
-    B, N, k = 3, 5000, 40
+    B = 3
     v = np.round(rng.random((B, N)), 2).astype(np.float32)
-    v[0, [3, 99]] = np.nan
+    v[0, [i for i in (3, 99) if i < N]] = np.nan
     v[1, :50] = -0.0
     v[1, 50:] = -1.0
     v[2, :] = 0.25  # all equal: the first k indices
+    v[0, -1] = 2.0  # the maximum in the ragged tail
     a = torch.as_tensor(v, device="cuda")
     idx = torch.empty((B, k), dtype=torch.int64, device="cuda")
     val = torch.empty((B, k), dtype=torch.float32, device="cuda")

@@ -19,7 +19,7 @@ CASES = [(1, 1000, 10), (1, 2048, 64), (2, 70_001, 64), (3, 300_000, 1024), (1, 
 
 def _scratch_bytes(B, N, k):
     nseg = -(-N // 2048)
-    return 0 if nseg <= 1 else 2 * B * nseg * k * 8
+    return 0 if nseg <= 1 else 2 * B * nseg * max(k, 16) * 8
 
 
 @pytest.mark.parametrize("B,N,k", CASES)
