@@ -142,24 +142,44 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
   }
 }
 
-// ---- Monte-Carlo HVI, two objectives: the boxes are the staircase strips
-// [a_i, b_i) x (-inf, u_i), so the f2 lower bound drops out:
-// HVI(y) = sum_i (b_i - max(a_i, y1))_+ (u_i - y2)_+.
+// 2-objective Monte-Carlo HVI over the strip decomposition: strips k = 0..K-1
+// with x-extent [a_k, b_k) (a_0 = -inf, a_k = b_{k-1}) and top u_k (u
+// decreasing). For a sample y the improvement is
+//   sum_k (b_k - max(a_k, y1))^+ (u_k - y2)^+
+//     = (b_0 - y1)^+ (u_0 - y2)^+ + sum_{k>=1} D_k sat((b_k - y1) / D_k) (u_k - y2)^+,
+// D_k = b_k - a_k, because (b_k - max(a_k, y1))^+ is (b_k - y1) clamped to
+// [0, D_k]. Per strip and sample: one saturating FMA, one FMA and a max for
+// the height with D_k folded in, one FMA to accumulate. One warp per
+// candidate, a float4 of base normals per lane and objective when S = 128.
+__device__ __forceinline__ float fma_sat(float a, float b, float c) {
+  float d;
+  asm("fma.rn.sat.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
 __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const float *var,
                                                      long long N, const float *lower,
                                                      const float *upper, const int *Kc,
                                                      int box_cap, const float *eps, int S,
                                                      long long eps_stride, float *acq) {
-  extern __shared__ float strips[];  // a[K], b[K], u[K]
+  extern __shared__ float4 strips4[];  // k >= 1: (b/D, 1/D, D u, D); [0]: (b_0, u_0, -, -)
+  float *sb = (float *)(strips4 + box_cap);  // b_k, for the pruning scans
+  float *su = sb + box_cap;                  // u_k
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
   const int b = blockIdx.y;
   const int K = Kc[b];
-  float *sa = strips, *sb = strips + box_cap, *su = strips + 2 * box_cap;
   for (int i = threadIdx.x; i < K; i += blockDim.x) {
     const size_t o = ((size_t)b * box_cap + i) * 2;
-    sa[i] = lower[o];
-    sb[i] = upper[o];
-    su[i] = upper[o + 1];
+    const float ai = lower[o], bi = upper[o], ui = upper[o + 1];
+    sb[i] = bi;
+    su[i] = ui;
+    if (i == 0) {
+      strips4[0] = make_float4(bi, ui, 0.f, 0.f);
+    } else {
+      const float D = bi - ai;
+      strips4[i] = D > 0.f ? make_float4(bi / D, 1.f / D, D * ui, D)
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
   }
   __syncthreads();
   const float *m1 = mean + (size_t)b * 2 * N, *m2 = m1 + N;
@@ -168,6 +188,23 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
   const long long cstride = (long long)gridDim.x * wpb;
   auto eps_of = [&](long long c) {
     return eps + ((size_t)b * N + c) * eps_stride + (eps_stride == 0 ? (size_t)b * 2 * S : 0);
+  };
+  // improvement of one sample from strips [k0, k1)
+  auto hvi = [&](float y1, float y2, int k0, int k1) {
+    float acc = 0.f;
+    int k = k0;
+    if (k == 0 && k < k1) {
+      const float4 t = strips4[0];
+      acc = fmaxf(t.x - y1, 0.f) * fmaxf(t.y - y2, 0.f);
+      k = 1;
+    }
+    for (; k < k1; ++k) {
+      const float4 t = strips4[k];
+      const float w = fma_sat(-y1, t.y, t.x);
+      const float h = fmaxf(fmaf(-y2, t.w, t.z), 0.f);
+      acc = fmaf(w, h, acc);
+    }
+    return acc;
   };
   if (vec) {
     // S = 128: one float4 per lane per objective; the next candidate's
@@ -209,12 +246,19 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
       while (k0 < K && sb[k0] <= lo1) ++k0;
       while (k1 > k0 && su[k1 - 1] <= lo2) --k1;
       float acc[4] = {0.f, 0.f, 0.f, 0.f};
-      for (int k = k0; k < k1; ++k) {
-        const float ak = sa[k], bk = sb[k], uk = su[k];
+      int k = k0;
+      if (k == 0 && k < k1) {
+        const float4 t = strips4[0];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[j] = fmaxf(t.x - y1[j], 0.f) * fmaxf(t.y - y2[j], 0.f);
+        k = 1;
+      }
+      for (; k < k1; ++k) {
+        const float4 t = strips4[k];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          const float w = fmaxf(bk - fmaxf(ak, y1[j]), 0.f);
-          const float h = fmaxf(uk - y2[j], 0.f);
+          const float w = fma_sat(-y1[j], t.y, t.x);
+          const float h = fmaxf(fmaf(-y2[j], t.w, t.z), 0.f);
           acc[j] = fmaf(w, h, acc[j]);
         }
       }
@@ -230,11 +274,8 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
     const float sg1 = sqrtf(fmaxf(v1[c], 0.f)), sg2 = sqrtf(fmaxf(v2[c], 0.f));
     const float *e = eps_of(c);
     float sum = 0.f;
-    for (int s = lane; s < S; s += 32) {
-      const float y1 = fmaf(sg1, e[s], mu1), y2 = fmaf(sg2, e[S + s], mu2);
-      for (int k = 0; k < K; ++k)
-        sum = fmaf(fmaxf(sb[k] - fmaxf(sa[k], y1), 0.f), fmaxf(su[k] - y2, 0.f), sum);
-    }
+    for (int s = lane; s < S; s += 32)
+      sum += hvi(fmaf(sg1, e[s], mu1), fmaf(sg2, e[S + s], mu2), 0, K);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
     if (lane == 0) acq[(size_t)b * N + c] = sum / (float)S;
@@ -272,7 +313,10 @@ int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
     cudaFuncSetAttribute(mchvi_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   }
   if (m == 2) {
-    mchvi2_kernel<<<dim3(gx, B), wpb * 32, 3 * (size_t)box_cap * sizeof(float), s>>>(
+    const size_t smem2 = 6 * (size_t)box_cap * sizeof(float);
+    if (smem2 > 48 * 1024)
+      cudaFuncSetAttribute(mchvi2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
+    mchvi2_kernel<<<dim3(gx, B), wpb * 32, smem2, s>>>(
         mean, var, N, lower, upper, K, box_cap, eps, S, eps_stride, acq);
   } else if (m == 3) {
     mchvi_kernel<3><<<dim3(gx, B), wpb * 32, smem, s>>>(mean, var, B, N, lower, upper, K, box_cap,

@@ -187,7 +187,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   extern __shared__ __align__(16) float sm[];
   __shared__ int bad;
   __shared__ uint64_t lbar;
-  __shared__ double red[16], ymu, yisd;
+  __shared__ double ymu, yisd;
   __shared__ __align__(16) float colb[2][32];
   __shared__ __align__(16) float wrow[2][32];
   const int bt = blockIdx.x, b = bt / m, t = bt % m;

@@ -13,13 +13,17 @@
 // the tensor core's fp32 accumulation and takes no operand column. K* never
 // reaches HBM.
 //
-// Persistent and warp-specialised: each CTA loops over (problem, tile) pairs.
-//   warp 0      bulk-TMA producer (operand images and training-point chunks)
+// Persistent and warp-specialised: each CTA loops over (tile, objective) units.
+//   warp 0      bulk-TMA producer of the operand images of L^-1 (B ring)
 //   warp 1      tcgen05.mma issuer; owns the 512-column TMEM allocation
-//   warps 4-7   epilogue: one TMEM lane quarter each, sum of squares, variance
-//   warps 8-15  K* builders: 16 rows x 2 halves per warp, packed f32x2 math
-// A ring of S shared-memory stages carries (A hi/lo, B hi/lo, side input);
-// the accumulator is double-buffered in TMEM (2 x 256 columns) so the
+//   warps 2-5   epilogue: one TMEM lane quarter each, sum of squares, variance
+//   warp 6      bulk-TMA producer of the training-point chunks (side-input ring)
+//   warps 7..   K* builders: packed f32x2 distance math, A ring
+// Three shared-memory rings with their own depths: A (K* hi/lo, builders ->
+// MMA), B (L^-1 hi/lo, TMA -> MMA) and the side input (scaled training points,
+// alpha and the objective's parameters, TMA -> builders), so that the builders
+// never wait on the operand copies of the MMA; the accumulator is
+// double-buffered in TMEM (2 x 256 columns) so the
 // epilogue of one output pass overlaps the MMAs of the next. Output columns
 // beyond 256 are handled in passes; pass p skips the reduction chunks where
 // its rows of L^-1 are zero. All waits are bounded (BOUTE_WAIT_NS): a wait
@@ -36,8 +40,10 @@ namespace {
 
 constexpr int kEpiWarp0 = 2;  // warps 2-5: epilogue, TMEM lane quarter = warp % 4
 constexpr int kEpiWarps = 4;
-constexpr int kBldWarp0 = 6;  // warps 6..: K* builders
-constexpr int kMaxStages = 4;
+constexpr int kXtWarp = 6;    // warp 6: side-input producer
+constexpr int kBldWarp0 = 7;  // warps 7..: K* builders
+constexpr int kMaxA = 4, kMaxB = 4, kMaxX = 8;  // ring depths
+constexpr uint32_t kABytes = 32768;             // one A stage: 128 x 32 fp32, hi and lo
 // builder warps: 16 (8 elements per thread and chunk) when the candidate
 // coordinates are short enough to keep in registers, else 8 (16 elements)
 template <int DP>
@@ -54,12 +60,27 @@ struct PostArgs {
   int *status;
   long long N;
   int B, m, d, n;
-  int tiles_per_problem, tiles_total, stages;
-  uint32_t stage_bytes;
+  int tiles_per_problem, tiles_total;
+  int sa, sb, sx;              // depths of the A, B and side-input rings
+  uint32_t b_bytes, x_bytes;   // one B stage, one side-input entry
   PostPlan plan;
 };
 
 constexpr float kSqrt5 = 2.2360679774997896964f;
+constexpr float kSqrt5Log2e = 3.2259641822295610f;  // sqrt(5) / ln(2)
+
+// Single hardware instructions (relative error about 2^-22), no range fix-ups:
+// arguments here are finite and non-negative (sqrt) or non-positive (ex2).
+__device__ __forceinline__ float sqrt_approx(float x) {
+  float y;
+  asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 constexpr float kFiveThirds = 1.6666666666666667f;
 
 // ---- packed fp32 pairs (sm_100+ f32x2 arithmetic) --------------------------------
@@ -136,27 +157,36 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   uint8_t *sm = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const PostPlan &pl = a.plan;
-  const int n = a.n, m = a.m, d = a.d, S = a.stages;
-  const int ncolmax = pl.ncol[0];
+  const int n = a.n, m = a.m, d = a.d, SA = a.sa, SB = a.sb, SX = a.sx;
   const int cf = xt_chunk_floats(DP);
 
-  uint64_t *bars = (uint64_t *)(sm + (size_t)S * a.stage_bytes);
-  uint64_t *full_b = bars, *a_full = bars + kMaxStages, *empty = bars + 2 * kMaxStages;
-  uint64_t *acc_full = bars + 3 * kMaxStages, *acc_empty = acc_full + 2, *drain = acc_full + 4;
+  uint8_t *ring_b = sm + (size_t)SA * kABytes;
+  uint8_t *ring_x = ring_b + (size_t)SB * a.b_bytes;
+  uint64_t *bars = (uint64_t *)(ring_x + (size_t)SX * a.x_bytes);
+  uint64_t *a_full = bars, *a_empty = bars + kMaxA;
+  uint64_t *b_full = bars + 2 * kMaxA, *b_empty = b_full + kMaxB;
+  uint64_t *x_full = b_full + 2 * kMaxB, *x_empty = x_full + kMaxX;
+  uint64_t *acc_full = x_full + 2 * kMaxX, *acc_empty = acc_full + 2, *drain = acc_full + 4;
   uint32_t *tmem_holder = (uint32_t *)(drain + 1);
   volatile int *abort = (volatile int *)(tmem_holder + 1);
 
-  auto stage = [&](int s) { return sm + (size_t)s * a.stage_bytes; };
-  auto a_hi = [&](int s) { return (float *)stage(s); };
-  auto a_lo = [&](int s) { return (float *)(stage(s) + 16384); };
-  auto b_reg = [&](int s) { return stage(s) + 32768; };
-  auto xt_reg = [&](int s) { return (float *)(stage(s) + 32768 + 2 * ncolmax * 128); };
+  auto a_hi = [&](int s) { return (float *)(sm + (size_t)s * kABytes); };
+  auto a_lo = [&](int s) { return (float *)(sm + (size_t)s * kABytes + 16384); };
+  auto b_reg = [&](int s) { return ring_b + (size_t)s * a.b_bytes; };
+  auto xt_reg = [&](int j) { return (float *)(ring_x + (size_t)j * a.x_bytes); };
 
   if (tid == 0) {
-    for (int s = 0; s < kMaxStages; ++s) {
-      mbar_init(&full_b[s], 1);
+    for (int s = 0; s < kMaxA; ++s) {
       mbar_init(&a_full[s], kBldWarps);
-      mbar_init(&empty[s], 1);
+      mbar_init(&a_empty[s], 1);
+    }
+    for (int s = 0; s < kMaxB; ++s) {
+      mbar_init(&b_full[s], 1);
+      mbar_init(&b_empty[s], 1);
+    }
+    for (int j = 0; j < kMaxX; ++j) {
+      mbar_init(&x_full[j], 1);
+      mbar_init(&x_empty[j], kBldWarps);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&acc_full[i], 1);
@@ -175,36 +205,44 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
 
-  if (warp == 0) {
-    // ---------------------------------------------------------------- producer
+  if (warp == 0 || warp == kXtWarp) {
+    // ------------------------------------------------------ producers (B / side input)
     if (lane == 0) {
+      const bool is_b = warp == 0;
+      const int R = is_b ? SB : SX;
+      uint64_t *full = is_b ? b_full : x_full, *empty = is_b ? b_empty : x_empty;
       uint32_t q = 0;
       int last_q = -1;  // last job issued
-      for (int tile = blockIdx.x; tile < a.tiles_total && !*abort; tile += gridDim.x) {
+      for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
+        const int tile = unit / m, t = unit % m;
         const int b = tile / a.tiles_per_problem;
-        for (int t = 0; t < m && !*abort; ++t) {
+        {
           const int bt = b * m + t;
           for (int p = 0; p < pl.npass && !*abort; ++p) {
             const uint32_t bbytes = (uint32_t)(2 * pl.ncol[p] * 128);
             for (int c = 0; c < pl.kc[p]; ++c, ++q) {
-              const int s = q % S;
-              const uint32_t use = q / S;
+              const int s = q % R;
+              const uint32_t use = q / R;
               if (use >= 1 && !wait_or_abort(&empty[s], (use - 1) & 1, abort, 128)) break;
-              mbar_arrive_expect_tx(&full_b[s], bbytes + (uint32_t)(cf * 4));
-              bulk_g2s(b_reg(s),
-                       a.bop + (size_t)bt * pl.image_floats + pl.off[p] +
-                           (size_t)c * 2 * pl.ncol[p] * BOUTE_KCHUNK,
-                       bbytes, &full_b[s]);
-              bulk_g2s(xt_reg(s), a.xt + ((size_t)bt * pl.nchunk + c) * cf, (uint32_t)(cf * 4),
-                       &full_b[s]);
+              if (is_b) {
+                mbar_arrive_expect_tx(&full[s], bbytes);
+                bulk_g2s(b_reg(s),
+                         a.bop + (size_t)bt * pl.image_floats + pl.off[p] +
+                             (size_t)c * 2 * pl.ncol[p] * BOUTE_KCHUNK,
+                         bbytes, &full[s]);
+              } else {
+                mbar_arrive_expect_tx(&full[s], (uint32_t)(cf * 4));
+                bulk_g2s(xt_reg(s), a.xt + ((size_t)bt * pl.nchunk + c) * cf, (uint32_t)(cf * 4),
+                         &full[s]);
+              }
               last_q = (int)q;
             }
           }
         }
       }
       if (*abort) {  // let our copies land before the block exits
-        for (int j = std::max(0, last_q - S + 1); j <= last_q; ++j)
-          mbar_wait(&full_b[j % S], (j / S) & 1);
+        for (int j = std::max(0, last_q - R + 1); j <= last_q; ++j)
+          mbar_wait(&full[j % R], (j / R) & 1);
       }
     }
   } else if (warp == 1) {
@@ -212,8 +250,8 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
     if (lane == 0) {
       uint32_t q = 0, u = 0;
       bool issued = false;
-      for (int tile = blockIdx.x; tile < a.tiles_total && !*abort; tile += gridDim.x) {
-        for (int t = 0; t < m && !*abort; ++t) {
+      for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
+        {
           for (int p = 0; p < pl.npass && !*abort; ++p, ++u) {
             const int ab = u & 1;
             if (u >= 2 && !wait_or_abort(&acc_empty[ab], ((u >> 1) - 1) & 1, abort, 64)) break;
@@ -222,13 +260,12 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
             const uint32_t idesc = idesc_tf32(ncol);
             const uint32_t dtm = tmem + (uint32_t)(ab * 256);
             for (int c = 0; c < pl.kc[p]; ++c, ++q) {
-              const int s = q % S;
-              const uint32_t use = q / S;
-              if (!wait_or_abort(&full_b[s], use & 1, abort, 32)) break;
-              if (!wait_or_abort(&a_full[s], use & 1, abort, 32)) break;
+              const int sa = q % SA, sb = q % SB;
+              if (!wait_or_abort(&b_full[sb], (q / SB) & 1, abort, 32)) break;
+              if (!wait_or_abort(&a_full[sa], (q / SA) & 1, abort, 32)) break;
               tc_fence_after();
-              const uint32_t sah = smem_u32(a_hi(s)), sal = smem_u32(a_lo(s));
-              const uint32_t sbh = smem_u32(b_reg(s)), sbl = sbh + ncol * 128;
+              const uint32_t sah = smem_u32(a_hi(sa)), sal = smem_u32(a_lo(sa));
+              const uint32_t sbh = smem_u32(b_reg(sb)), sbl = sbh + ncol * 128;
 #pragma unroll
               for (int ks = 0; ks < 4; ++ks) {
                 const uint64_t dah = sdesc_sw128(sah + ks * 32), dal = sdesc_sw128(sal + ks * 32);
@@ -237,7 +274,8 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
                 mma_tf32(dtm, dah, dbl, idesc, 1u);
                 mma_tf32(dtm, dal, dbh, idesc, 1u);
               }
-              mma_commit(&empty[s]);
+              mma_commit(&a_empty[sa]);
+              mma_commit(&b_empty[sb]);
               issued = true;
             }
             mma_commit(&acc_full[ab]);
@@ -253,11 +291,12 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
     // ---------------------------------------------------------------- epilogue
     const int eq = warp & 3;  // TMEM lane quarter this warp may access
     uint32_t u = 0;
-    for (int tile = blockIdx.x; tile < a.tiles_total && !*abort; tile += gridDim.x) {
+    for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
+      const int tile = unit / m, t = unit % m;
       const int b = tile / a.tiles_per_problem;
       const long long row =
           (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M + 32 * eq + lane;
-      for (int t = 0; t < m && !*abort; ++t) {
+      {
         float ss = 0.f;
         for (int p = 0; p < pl.npass; ++p, ++u) {
           const int ab = u & 1;
@@ -287,25 +326,25 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
     const int bw = warp - kBldWarp0;
     const int r = bw * RPW + lane % RPW, g = lane / RPW;
     uint32_t q = 0;
-    for (int tile = blockIdx.x; tile < a.tiles_total && !*abort; tile += gridDim.x) {
+    for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
+      const int tile = unit / m, t = unit % m;
       const int b = tile / a.tiles_per_problem;
       const long long row = (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M + r;
       const float *xrow = a.Xc + ((long long)b * a.N + row) * d;
       float xr[DP];
 #pragma unroll
       for (int k = 0; k < DP; ++k) xr[k] = (k < d && row < a.N) ? xrow[k] : 0.f;
-      for (int t = 0; t < m && !*abort; ++t) {
+      {
         unsigned long long xs2[DP];
         float s2 = 0.f;
         float mu = 0.f, comp = 0.f;
         for (int p = 0; p < pl.npass && !*abort; ++p) {
           const bool last_pass = p == pl.npass - 1;
           for (int c = 0; c < pl.kc[p]; ++c, ++q) {
-            const int s = q % S;
-            const uint32_t use = q / S;
-            if (use >= 1 && !wait_or_abort(&empty[s], (use - 1) & 1, abort)) break;
-            if (!wait_or_abort(&full_b[s], use & 1, abort)) break;
-            const float *xth = xt_reg(s), *xtl = xth + BOUTE_KCHUNK * DP;
+            const int s = q % SA, j = q % SX;
+            if (q >= (uint32_t)SA && !wait_or_abort(&a_empty[s], (q / SA - 1) & 1, abort)) break;
+            if (!wait_or_abort(&x_full[j], (q / SX) & 1, abort)) break;
+            const float *xth = xt_reg(j), *xtl = xth + BOUTE_KCHUNK * DP;  // x hi, x lo
             const float *alp = xtl + BOUTE_KCHUNK * DP;
             if (p == 0 && c == 0) {  // new objective: its parameters came with the chunk
               const float *il = xth + xt_param_offset(DP);
@@ -314,7 +353,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
               s2 = il[2 * DP];
             }
             // squared scaled distances to this thread's COLS training points, in
-            // pairs: (x*_k - x_hi) - x_lo, squared and accumulated
+            // pairs: x*_k - x_k (fp32 scaled coordinates), squared and accumulated
             unsigned long long acc2[COLS / 2];
 #pragma unroll
             for (int e = 0; e < COLS / 2; ++e) acc2[e] = 0ull;
@@ -322,14 +361,13 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
             for (int k = 0; k < DP; ++k) {
               const unsigned long long *h2 =
                   (const unsigned long long *)(xth + k * BOUTE_KCHUNK + COLS * g);
-              const unsigned long long *l2 =
-                  (const unsigned long long *)(xtl + k * BOUTE_KCHUNK + COLS * g);
 #pragma unroll
               for (int e = 0; e < COLS / 2; ++e) {
-                const unsigned long long df = f2_sub(f2_sub(xs2[k], h2[e]), l2[e]);
+                const unsigned long long df = f2_sub(xs2[k], h2[e]);
                 acc2[e] = f2_fma(df, df, acc2[e]);
               }
             }
+            const bool full_chunk = (c + 1) * BOUTE_KCHUNK <= n;
             const int jbase = c * BOUTE_KCHUNK + COLS * g;
             float mu_part = 0.f;
             float *Ah = a_hi(s), *Al = a_lo(s);
@@ -343,10 +381,11 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
 #pragma unroll
                 for (int z = 0; z < 2; ++z) {
                   const int e = 2 * e2 + z, kk = 4 * g4 + e;
-                  const float rr = sqrtf(r2[z]);
+                  // k = s2 (1 + sqrt5 r + 5/3 r^2) exp(-sqrt5 r), exp(-x) = 2^(-x log2 e)
+                  const float rr = sqrt_approx(r2[z]);
                   const float sr = kSqrt5 * rr;
-                  float kv = s2 * fmaf(kFiveThirds, r2[z], 1.0f + sr) * expf(-sr);
-                  kv = (jbase + kk < n) ? kv : 0.f;
+                  float kv = s2 * fmaf(kFiveThirds, r2[z], 1.0f + sr) * ex2_approx(-kSqrt5Log2e * rr);
+                  if (!full_chunk) kv = (jbase + kk < n) ? kv : 0.f;
                   mu_part = fmaf(kv, alp[COLS * g + kk], mu_part);
                   const float hi = tf32_rna(kv);
                   vh[e] = hi;
@@ -359,7 +398,10 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
             }
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive_count(&a_full[s]);
+            if (lane == 0) {
+              mbar_arrive_count(&a_full[s]);
+              mbar_arrive_count(&x_empty[j]);
+            }
             if (last_pass) {  // Kahan: mu += mu_part (the last pass builds every chunk)
               const float yk = mu_part - comp;
               const float tk = mu + yk;
@@ -408,17 +450,28 @@ int launch_dp(const Gp *gp, const float *Xc, long long N, float *mean, float *va
   a.tiles_per_problem = (int)((N + BOUTE_TILE_M - 1) / BOUTE_TILE_M);
   a.tiles_total = a.tiles_per_problem * gp->B;
   const int ncolmax = gp->plan.ncol[0];
-  a.stage_bytes =
-      (uint32_t)round_up(32768 + 2 * ncolmax * 128 + xt_chunk_floats(DP) * 4, 1024);
-  const size_t fixed = 1024 + 256;  // alignment slack, barriers, TMEM address, flag
+  a.b_bytes = (uint32_t)(2 * ncolmax * 128);  // a multiple of 1024 (ncol % 16 == 0)
+  a.x_bytes = (uint32_t)round_up(xt_chunk_floats(DP) * 4, 16);
+  const size_t fixed = 1024 + 512;  // alignment slack, barriers, TMEM address, flag
   const size_t budget = 227 * 1024 - fixed;
-  a.stages = (int)std::min<size_t>(kMaxStages, budget / a.stage_bytes);
-  const size_t smem = fixed + (size_t)a.stages * a.stage_bytes;
+  // deepest B ring first (it hides the operand copies), then A, then the side input
+  a.sx = kMaxX;
+  a.sa = 3;
+  a.sb = kMaxB;
+  while ((size_t)a.sa * kABytes + (size_t)a.sb * a.b_bytes + (size_t)a.sx * a.x_bytes > budget) {
+    if (a.sx > 4) --a.sx;
+    else if (a.sb > a.sa) --a.sb;
+    else if (a.sa > 2) --a.sa;
+    else if (a.sb > 2) --a.sb;
+    else return BOUTE_ERR_UNSUPPORTED;
+  }
+  const size_t smem =
+      fixed + (size_t)a.sa * kABytes + (size_t)a.sb * a.b_bytes + (size_t)a.sx * a.x_bytes;
   cudaFuncSetAttribute(posterior_kernel<DP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        (int)smem);
   int sms = 152;
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
-  const int grid = std::max(1, std::min(a.tiles_total, sms));
+  const int grid = std::max(1, std::min(a.tiles_total * a.m, sms));  // (tile, objective) units
   posterior_kernel<DP><<<grid, Layout<DP>::kThreads, smem, s>>>(a);
   count_launch();
   return last_launch_status();

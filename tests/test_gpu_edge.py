@@ -165,10 +165,36 @@ def test_candidates_on_training_points():
 def test_per_objective_hyperparameters():
     rng = np.random.default_rng(8)
     hp = rand_problem(9, 70, 5, 2, 333)
-    hp.ls[0] = rng.uniform(0.1, 1.5, (2, 5))
+    hp.ls[0] = rng.uniform(0.2, 0.6, (2, 5))
     hp.s2[0] = [0.5, 2.5]
-    hp.noise[0] = [1e-3, 1e-5]
+    hp.noise[0] = [1e-3, 1e-4]
     compare(hp)
+
+
+@pytest.mark.parametrize("ls_range,noise", [((0.1, 1.5), (1e-3, 1e-5)), ((0.3, 1.5), (1e-3, 1e-4))])
+def test_ill_conditioned_mean_meets_fp32_error_bound(ls_range, noise):
+    """Long lengthscales (or tiny noise) over 70 points in 5-D: the mean K*
+    alpha cancels, sum_j |K*_j alpha_j| reaching 200-270 times its scale, so
+    fp32 K* entries (relative error a few eps32) cannot give 1e-5 relative.
+    The mean must stay within a small multiple of eps32 * sum_j |K*_j alpha_j|,
+    the forward error bound of an fp32-accurate cross-covariance; the variance
+    keeps the 1e-5 tolerance."""
+    rng = np.random.default_rng(8)
+    hp = rand_problem(9, 70, 5, 2, 333)
+    hp.ls[0] = rng.uniform(*ls_range, (2, 5))
+    hp.s2[0] = [0.5, 2.5]
+    hp.noise[0] = list(noise)
+    g = gpu_pipeline(hp)
+    assert g["status"] == 0
+    fp = opl.fit_problem(hp.X[0], hp.Y[0], hp.ls[0], hp.s2[0], hp.noise[0], hp.ref[0])
+    mean, var = opl.posterior(fp, hp.Xc[0])
+    eps32 = np.finfo(np.float32).eps
+    for t in range(2):
+        Ks = np.array([[oracle.matern52(c.astype(np.float64), x, hp.ls[0][t], hp.s2[0][t])
+                        for x in hp.X[0]] for c in hp.Xc[0]])
+        bound_mu = 16 * eps32 * (np.abs(Ks) @ np.abs(fp.alpha[t])) + 1e-5 * np.sqrt(hp.s2[0][t])
+        assert np.all(np.abs(g["mean"][0, t] - mean[:, t]) <= bound_mu)
+        check_var(g["var"][0, t], var[:, t], fp.s2[t])
 
 
 def test_far_candidates_and_zero_variance_ehvi():
