@@ -123,7 +123,7 @@ def roofline(w: wl.Workload, stage: str, ms: float, hbm, bf16):
     if stage == "acquisition" and w.mode == "mc":
         byts = B * N * (m * S * 4 + 2 * m * 4 + 4)
         return dict(bound="hbm", achieved=byts / (ms * 1e-3) / 1e9, peak=hbm, unit="GB/s",
-                    per_launch=byts, kernel="mchvi_kernel")
+                    per_launch=byts, kernel="mchvi2_kernel" if m == 2 else "mchvi_kernel")
     if stage == "acquisition":
         byts = B * N * (2 * m * 4 + 4)
         return dict(bound="hbm", achieved=byts / (ms * 1e-3) / 1e9, peak=hbm, unit="GB/s",
@@ -131,7 +131,8 @@ def roofline(w: wl.Workload, stage: str, ms: float, hbm, bf16):
     if stage == "topk":
         byts = B * N * 4
         return dict(bound="hbm", achieved=byts / (ms * 1e-3) / 1e9, peak=hbm, unit="GB/s",
-                    per_launch=byts, kernel="topk_partial_kernel")
+                    per_launch=byts,
+                    kernel="warp_topk_kernel" if w.k <= 32 else "segment_topk_kernel")
     if stage == "fit":
         # Cholesky n^3/3 + triangular inverse n^3/3 flops per (problem,
         # objective), fp32 on the CUDA cores of the SMs the fit occupies (one

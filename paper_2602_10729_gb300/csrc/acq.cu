@@ -314,6 +314,7 @@ int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
   }
   if (m == 2) {
     const size_t smem2 = 6 * (size_t)box_cap * sizeof(float);
+    prefer_shared(mchvi2_kernel);
     if (smem2 > 48 * 1024)
       cudaFuncSetAttribute(mchvi2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
     mchvi2_kernel<<<dim3(gx, B), wpb * 32, smem2, s>>>(

@@ -1,7 +1,11 @@
-// GP fit on the device: standardisation, kernel matrix, Cholesky factor,
-// triangular inverse, alpha, and the prepacked tensor-core operands of the
-// posterior contraction. All factor arithmetic is fp64 (Sec. 6: the paper's
-// GP kernels run in double precision).
+// GP fit on the device (Sec. 5.2, one exact GP per objective; Sec. 6,
+// Matern-5/2 ARD kernel with outputscale on standardised outcomes):
+// standardisation, kernel matrix, Cholesky factor, triangular inverse, alpha,
+// and the prepacked tensor-core operands of the posterior contraction. The
+// kernel matrix is formed in fp64 and kept as an fp32 pair; the factor and its
+// inverse are fp32, and alpha is refined against the fp64-accurate matrix
+// with double-float residuals (the paper runs its GP kernels in double
+// precision, Appendix C; fp64 throughput is low on this part).
 #include <math.h>
 
 #include <algorithm>
@@ -637,11 +641,13 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
   const int npad = gp->plan.npad;
   const int tn = (n + 15) / 16, nkt = tn * tn;
   const int nprep = std::max(1, std::min(8, npad * gp->DP / 256));
+  prefer_shared(fit_setup_kernel);
   fit_setup_kernel<<<dim3(nkt + nprep, BM), 256, 0, s>>>(X, n, d, m, gp->DP, npad, ls, s2, noise,
                                                          gp->Kh, gp->Kl, gp->xt, gp->s2f, nkt,
                                                          nprep, gp->status);
   if (fit_uses_smem(npad)) {
     const size_t smem = fit_smem_bytes(npad, n);
+    prefer_shared(fit32_kernel<true>);
     cudaFuncSetAttribute(fit32_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);
     fit32_kernel<true><<<BM, fit_threads<true>(), smem, s>>>(

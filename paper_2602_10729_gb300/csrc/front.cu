@@ -282,6 +282,7 @@ int launch_front_fused(const double *Y, int B, int n, int m, const double *ref, 
                        unsigned char *mask, double *front, int *P, float *lower, float *upper,
                        int *K, int want_boxes, cudaStream_t s) {
   const size_t smem = front_smem_bytes(n, m);
+  prefer_shared(front_fused_kernel);
   if (smem > 48 * 1024)
     cudaFuncSetAttribute(front_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);

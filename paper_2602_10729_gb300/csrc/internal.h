@@ -20,6 +20,14 @@ struct Gp {
   int *status;    // device status word (first error wins)
 };
 
+// Every kernel of the step asks for the largest shared-memory carveout, so
+// that consecutive kernels never make an SM switch its L1 / shared split.
+template <class F>
+inline void prefer_shared(F *kernel) {
+  cudaFuncSetAttribute((const void *)kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                       (int)cudaSharedmemCarveoutMaxShared);
+}
+
 void count_launch(int k = 1);
 unsigned long long launch_count();
 int last_launch_status();  // BOUTE_OK or BOUTE_ERR_CUDA after a launch

@@ -467,6 +467,7 @@ int launch_dp(const Gp *gp, const float *Xc, long long N, float *mean, float *va
   }
   const size_t smem =
       fixed + (size_t)a.sa * kABytes + (size_t)a.sb * a.b_bytes + (size_t)a.sx * a.x_bytes;
+  prefer_shared(posterior_kernel<DP>);
   cudaFuncSetAttribute(posterior_kernel<DP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        (int)smem);
   int sms = 152;

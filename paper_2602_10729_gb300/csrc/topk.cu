@@ -187,6 +187,8 @@ int launch_topk_warp(const float *acq, int B, long long N, int k, long long *idx
   long long per_block = unit;
   while ((N + per_block - 1) / per_block > 256) per_block += unit;
   const long long G = (N + per_block - 1) / per_block;
+  prefer_shared(warp_topk_kernel<true>);
+  prefer_shared(warp_topk_kernel<false>);
   if (G == 1) {
     warp_topk_kernel<true><<<dim3(1, B), kWarpBlock, 0, s>>>(acq, nullptr, N, per_block, nullptr,
                                                               acq, N, k, idx, val);
