@@ -23,7 +23,8 @@
 // MMA), B (L^-1 hi/lo, TMA -> MMA) and the side input (scaled training points,
 // alpha and the objective's parameters, TMA -> builders), so that the builders
 // never wait on the operand copies of the MMA; the accumulator is
-// double-buffered in TMEM (2 x 256 columns) so the
+// double-buffered in TMEM (2 x 256 columns; a pass with a reduction longer
+// than 256 takes both buffers, one per half of the reduction) so the
 // epilogue of one output pass overlaps the MMAs of the next. Output columns
 // beyond 256 are handled in passes; pass p skips the reduction chunks where
 // its rows of L^-1 are zero. All waits are bounded (BOUTE_WAIT_NS): a wait
@@ -44,6 +45,13 @@ constexpr int kXtWarp = 6;    // warp 6: side-input producer
 constexpr int kBldWarp0 = 7;  // warps 7..: K* builders
 constexpr int kMaxA = 4, kMaxB = 4, kMaxX = 8;  // ring depths
 constexpr uint32_t kABytes = 32768;             // one A stage: 128 x 32 fp32, hi and lo
+
+// The tensor core's fp32 accumulator truncates after each MMA, so its error
+// grows with the number of accumulations into one output. A pass whose
+// reduction is longer than 8 chunks (256 training points) accumulates its
+// first and second halves in the two TMEM buffers, which the epilogue adds in
+// round-to-nearest; returns the chunk count of the first half (kc: no split).
+__device__ __forceinline__ int split_chunks(int kc) { return kc > 8 ? (kc + 1) / 2 : kc; }
 // builder warps: 16 (8 elements per thread and chunk) when the candidate
 // coordinates are short enough to keep in registers, else 8 (16 elements)
 template <int DP>
@@ -248,18 +256,26 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      uint32_t q = 0, u = 0;
+      uint32_t q = 0, nuse[2] = {0u, 0u};
+      int nxt = 0;
       bool issued = false;
       for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
         {
-          for (int p = 0; p < pl.npass && !*abort; ++p, ++u) {
-            const int ab = u & 1;
-            if (u >= 2 && !wait_or_abort(&acc_empty[ab], ((u >> 1) - 1) & 1, abort, 64)) break;
+          for (int p = 0; p < pl.npass && !*abort; ++p) {
+            const int kc = pl.kc[p], h = split_chunks(kc);
+            const bool split = h < kc;  // second half of the reduction -> other buffer
+            const int A = nxt, Bf = nxt ^ 1;
+            if (nuse[A] >= 1 && !wait_or_abort(&acc_empty[A], (nuse[A] - 1) & 1, abort, 64)) break;
+            if (split && nuse[Bf] >= 1 &&
+                !wait_or_abort(&acc_empty[Bf], (nuse[Bf] - 1) & 1, abort, 64))
+              break;
             tc_fence_after();
             const int ncol = pl.ncol[p];
             const uint32_t idesc = idesc_tf32(ncol);
-            const uint32_t dtm = tmem + (uint32_t)(ab * 256);
-            for (int c = 0; c < pl.kc[p]; ++c, ++q) {
+            for (int c = 0; c < kc; ++c, ++q) {
+              const bool second = split && c >= h;
+              const uint32_t dtm = tmem + (uint32_t)((second ? Bf : A) * 256);
+              const int c0 = second ? h : 0;  // first chunk of this accumulator
               const int sa = q % SA, sb = q % SB;
               if (!wait_or_abort(&b_full[sb], (q / SB) & 1, abort, 32)) break;
               if (!wait_or_abort(&a_full[sa], (q / SA) & 1, abort, 32)) break;
@@ -270,15 +286,19 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
               for (int ks = 0; ks < 4; ++ks) {
                 const uint64_t dah = sdesc_sw128(sah + ks * 32), dal = sdesc_sw128(sal + ks * 32);
                 const uint64_t dbh = sdesc_sw128(sbh + ks * 32), dbl = sdesc_sw128(sbl + ks * 32);
-                mma_tf32(dtm, dah, dbh, idesc, (c > 0 || ks > 0) ? 1u : 0u);
+                mma_tf32(dtm, dah, dbh, idesc, (c > c0 || ks > 0) ? 1u : 0u);
                 mma_tf32(dtm, dah, dbl, idesc, 1u);
                 mma_tf32(dtm, dal, dbh, idesc, 1u);
               }
               mma_commit(&a_empty[sa]);
               mma_commit(&b_empty[sb]);
+              if (split && c == h - 1) mma_commit(&acc_full[A]);
               issued = true;
             }
-            mma_commit(&acc_full[ab]);
+            mma_commit(&acc_full[split ? Bf : A]);
+            ++nuse[A];
+            if (split) ++nuse[Bf];
+            else nxt ^= 1;
           }
         }
       }
@@ -290,7 +310,8 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   } else if (warp >= kEpiWarp0 && warp < kEpiWarp0 + kEpiWarps) {
     // ---------------------------------------------------------------- epilogue
     const int eq = warp & 3;  // TMEM lane quarter this warp may access
-    uint32_t u = 0;
+    uint32_t nuse[2] = {0u, 0u};
+    int nxt = 0;
     for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
       const int tile = unit / m, t = unit % m;
       const int b = tile / a.tiles_per_problem;
@@ -298,20 +319,37 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
           (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M + 32 * eq + lane;
       {
         float ss = 0.f;
-        for (int p = 0; p < pl.npass; ++p, ++u) {
-          const int ab = u & 1;
-          if (!wait_or_abort(&acc_full[ab], (u >> 1) & 1, abort, 512)) break;
+        for (int p = 0; p < pl.npass; ++p) {
+          const int kc = pl.kc[p];
+          const bool split = split_chunks(kc) < kc;
+          const int A = nxt, Bf = nxt ^ 1;
+          if (!wait_or_abort(&acc_full[A], nuse[A] & 1, abort, 512)) break;
+          if (split && !wait_or_abort(&acc_full[Bf], nuse[Bf] & 1, abort, 512)) break;
           tc_fence_after();
-          const uint32_t tb = tmem + (uint32_t)(ab * 256) + ((uint32_t)(32 * eq) << 16);
+          const uint32_t lanes = (uint32_t)(32 * eq) << 16;
+          const uint32_t ta = tmem + (uint32_t)(A * 256) + lanes;
+          const uint32_t tbb = tmem + (uint32_t)(Bf * 256) + lanes;
           for (int cc = 0; cc < pl.ncol[p]; cc += 16) {
             float v[16];
-            tmem_ld16(tb + cc, v);
+            tmem_ld16(ta + cc, v);
+            if (split) {  // V = first half + second half of the reduction
+              float w[16];
+              tmem_ld16(tbb + cc, w);
+#pragma unroll
+              for (int e = 0; e < 16; ++e) v[e] += w[e];
+            }
 #pragma unroll
             for (int e = 0; e < 16; ++e) ss = fmaf(v[e], v[e], ss);  // zero beyond n
           }
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive_count(&acc_empty[ab]);
+          if (lane == 0) {
+            mbar_arrive_count(&acc_empty[A]);
+            if (split) mbar_arrive_count(&acc_empty[Bf]);
+          }
+          ++nuse[A];
+          if (split) ++nuse[Bf];
+          else nxt ^= 1;
         }
         if (*abort) break;
         if (row < a.N) {
