@@ -82,7 +82,7 @@ struct boute_engine {
   // the step as a CUDA graph, per argument set (two sets: device and host
   // inputs); replay removes the host launch gaps between the kernels
   struct Graph {
-    const void *key[11];
+    const void *key[12];
     cudaGraphExec_t exec;
     int launches;
   } graphs[2];
@@ -92,6 +92,11 @@ struct boute_engine {
   // into the step's stream, beside the GP fit
   cudaStream_t side;
   cudaEvent_t fork, join;
+  // host-input steps: candidates and base normals are copied on two copy
+  // streams while the fit runs; the step waits for them only where it needs
+  // them (posterior, acquisition)
+  cudaStream_t cpy[2];
+  cudaEvent_t ev_in, ev_xc, ev_eps[2];
 };
 
 // Stage order of one step as timed (with timing on, the front stage runs
@@ -254,6 +259,10 @@ void boute_engine_free(boute_engine *e) {
   if (e->fork) cudaEventDestroy(e->fork);
   if (e->join) cudaEventDestroy(e->join);
   if (e->side) cudaStreamDestroy(e->side);
+  for (cudaEvent_t ev : {e->ev_in, e->ev_xc, e->ev_eps[0], e->ev_eps[1]})
+    if (ev) cudaEventDestroy(ev);
+  for (cudaStream_t c : e->cpy)
+    if (c) cudaStreamDestroy(c);
   void *ptrs[] = {e->X, e->Y, e->Ys, e->ls, e->s2, e->noise, e->ref, e->front, e->mask, e->P,
                   e->K, e->lower, e->upper, e->Xc, e->eps, e->mean, e->var, e->acq, e->val,
                   e->idx, e->scratch};
@@ -301,7 +310,13 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
   if (r == BOUTE_OK &&
       (cudaStreamCreateWithFlags(&e->side, cudaStreamNonBlocking) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->fork, cudaEventDisableTiming) != cudaSuccess ||
-       cudaEventCreateWithFlags(&e->join, cudaEventDisableTiming) != cudaSuccess)) {
+       cudaEventCreateWithFlags(&e->join, cudaEventDisableTiming) != cudaSuccess ||
+       cudaStreamCreateWithFlags(&e->cpy[0], cudaStreamNonBlocking) != cudaSuccess ||
+       cudaStreamCreateWithFlags(&e->cpy[1], cudaStreamNonBlocking) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->ev_in, cudaEventDisableTiming) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->ev_xc, cudaEventDisableTiming) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->ev_eps[0], cudaEventDisableTiming) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->ev_eps[1], cudaEventDisableTiming) != cudaSuccess)) {
     cudaGetLastError();
     r = BOUTE_ERR_CUDA;
   }
@@ -315,7 +330,8 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
 
 static int engine_run(boute_engine *e, const double *X, const double *Y, const double *ls,
                       const double *s2, const double *noise, const double *ref, const float *Xc,
-                      const float *eps, long long *idx, float *val, cudaStream_t s) {
+                      const float *eps, long long *idx, float *val, cudaStream_t s,
+                      int host) {
   const unsigned long long l0 = launch_count();
   int r;
   const int B = e->B, n = e->n, m = e->m;
@@ -338,10 +354,21 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
   if ((r = launch_fit_raw(&e->gp->g, X, Y, ls, s2, noise, s))) return r;
   mark(ST_FRONT);
   if (e->timing && (r = front(s))) return r;
+  // waits on the host-input copies: an external-event node when captured
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (host && cudaStreamIsCapturing(s, &cap) != cudaSuccess) return last_launch_status();
+  const unsigned wait_flags =
+      cap == cudaStreamCaptureStatusActive ? cudaEventWaitExternal : cudaEventWaitDefault;
   mark(ST_POSTERIOR);
+  if (host && cudaStreamWaitEvent(s, e->ev_xc, wait_flags) != cudaSuccess)
+    return last_launch_status();
   if ((r = launch_posterior(&e->gp->g, Xc, e->N, e->mean, e->var, s))) return r;
   if (!e->timing && cudaStreamWaitEvent(s, e->join, 0) != cudaSuccess)  // join
     return last_launch_status();
+  if (host && mc)
+    for (cudaEvent_t ev : e->ev_eps)
+      if (cudaStreamWaitEvent(s, ev, wait_flags) != cudaSuccess)
+        return last_launch_status();
   mark(ST_ACQ);
   if (!mc) {
     if ((r = launch_ehvi(e->mean, e->var, B, e->N, e->front, e->P, n, ref, e->acq, s))) return r;
@@ -369,10 +396,11 @@ static int engine_args_ok(const boute_engine *e, const void *X, const void *Y, c
 static int engine_launch(boute_engine *e, const double *X, const double *Y, const double *ls,
                          const double *s2, const double *noise, const double *ref,
                          const float *Xc, const float *eps, long long *idx, float *val,
-                         cudaStream_t s) {
-  const void *key[11] = {X, Y, ls, s2, noise, ref, Xc, eps, idx, val, (const void *)s};
+                         cudaStream_t s, int host = 0) {
+  const void *key[12] = {X,   Y,   ls,  s2,  noise,           ref,
+                         Xc,  eps, idx, val, (const void *)s, (const void *)(uintptr_t)host};
   if (!s || e->graphs_off)  // the legacy default stream cannot be captured
-    return engine_run(e, X, Y, ls, s2, noise, ref, Xc, eps, idx, val, s);
+    return engine_run(e, X, Y, ls, s2, noise, ref, Xc, eps, idx, val, s, host);
   for (auto &g : e->graphs) {
     if (g.exec && std::memcmp(g.key, key, sizeof(key)) == 0) {
       if (cudaGraphLaunch(g.exec, s) != cudaSuccess) return last_launch_status();
@@ -389,10 +417,10 @@ static int engine_launch(boute_engine *e, const double *X, const double *Y, cons
   }
   if (cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
     cudaGetLastError();
-    return engine_run(e, X, Y, ls, s2, noise, ref, Xc, eps, idx, val, s);
+    return engine_run(e, X, Y, ls, s2, noise, ref, Xc, eps, idx, val, s, host);
   }
   const unsigned long long l0 = launch_count();
-  const int r = engine_run(e, X, Y, ls, s2, noise, ref, Xc, eps, idx, val, s);
+  const int r = engine_run(e, X, Y, ls, s2, noise, ref, Xc, eps, idx, val, s, host);
   cudaGraph_t graph = nullptr;
   const cudaError_t ce = cudaStreamEndCapture(s, &graph);
   const int captured = (int)(launch_count() - l0);
@@ -452,12 +480,24 @@ int boute_engine_step_host(boute_engine *e, const double *X, const double *Y,
   cudaMemcpyAsync(e->s2, outputscale, B * m * sizeof(double), cudaMemcpyHostToDevice, s);
   cudaMemcpyAsync(e->noise, noise, B * m * sizeof(double), cudaMemcpyHostToDevice, s);
   cudaMemcpyAsync(e->ref, ref, B * m * sizeof(double), cudaMemcpyHostToDevice, s);
-  cudaMemcpyAsync(e->Xc, Xc, B * N * d * sizeof(float), cudaMemcpyHostToDevice, s);
-  if (e->mode == BOUTE_ACQ_MC_HVI)
-    cudaMemcpyAsync(e->eps, eps, B * N * m * S * sizeof(float), cudaMemcpyHostToDevice, s);
+  // candidates and normals on the copy streams, ordered after everything
+  // already on `stream` (the previous step still reads these buffers), and
+  // overlapping the fit; the normals in two halves, one per copy engine
+  cudaEventRecord(e->ev_in, s);
+  for (cudaStream_t c : e->cpy) cudaStreamWaitEvent(c, e->ev_in, 0);
+  cudaMemcpyAsync(e->Xc, Xc, B * N * d * sizeof(float), cudaMemcpyHostToDevice, e->cpy[0]);
+  cudaEventRecord(e->ev_xc, e->cpy[0]);
+  const size_t eps_n = e->mode == BOUTE_ACQ_MC_HVI ? B * N * m * S : 0, half = eps_n / 2;
+  for (int i = 0; i < 2; ++i) {
+    const size_t off = i ? half : 0, cnt = i ? eps_n - half : half;
+    if (cnt)
+      cudaMemcpyAsync(e->eps + off, eps + off, cnt * sizeof(float), cudaMemcpyHostToDevice,
+                      e->cpy[i]);
+    cudaEventRecord(e->ev_eps[i], e->cpy[i]);
+  }
   if (int r = last_launch_status()) return r;
   int r = engine_launch(e, e->X, e->Y, e->ls, e->s2, e->noise, e->ref, e->Xc, e->eps, e->idx,
-                        e->val, s);
+                        e->val, s, 1);
   if (r) return r;
   cudaMemcpyAsync(idx, e->idx, B * k * sizeof(long long), cudaMemcpyDeviceToHost, s);
   cudaMemcpyAsync(val, e->val, B * k * sizeof(float), cudaMemcpyDeviceToHost, s);

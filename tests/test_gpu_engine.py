@@ -1,0 +1,114 @@
+"""The whole scoring step through the engine entry points: device inputs,
+host inputs (copies inside the call, overlapped with the fit), graph replay
+on a side stream, eager execution on the legacy default stream and the
+stage-timing mode must all give the same selection, value for value, and the
+same per-candidate scores as the step-by-step calls checked against the
+oracle elsewhere. Consecutive host-input steps with different inputs catch
+reuse of the engine's input buffers before the previous step is done."""
+import numpy as np
+import pytest
+
+from _pipeline import check_acq_end_to_end, gpu_pipeline, host_problem, oracle_fit
+from oracle import pipeline as opl
+from paper_2602_10729_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+CASES = [(0, 4096 + 77, 1), (1, 3000 + 5, 1), (4, 1500 + 1, 3)]
+
+
+def _dev(hp):
+    import torch
+    t = lambda a, dt: None if a is None else torch.as_tensor(np.ascontiguousarray(a), dtype=dt,
+                                                             device="cuda")
+    f64, f32 = torch.float64, torch.float32
+    return (t(hp.X, f64), t(hp.Y, f64), t(hp.ls, f64), t(hp.s2, f64), t(hp.noise, f64),
+            t(hp.ref, f64), t(hp.Xc, f32), t(hp.eps, f32))
+
+
+def _host(hp):
+    import torch
+    t = lambda a, dt: None if a is None else torch.as_tensor(np.ascontiguousarray(a),
+                                                             dtype=dt).pin_memory()
+    f64, f32 = torch.float64, torch.float32
+    return (t(hp.X, f64), t(hp.Y, f64), t(hp.ls, f64), t(hp.s2, f64), t(hp.noise, f64),
+            t(hp.ref, f64), t(hp.Xc, f32), t(hp.eps, f32))
+
+
+def _engine(w):
+    from paper_2602_10729_gb300 import boute as bt
+    mode = bt.BOUTE_ACQ_MC_HVI if w.mode == "mc" else bt.BOUTE_ACQ_EHVI2D
+    return bt.Engine(w.B, w.n, w.d, w.m, w.N, mode, w.S, w.k)
+
+
+def _run(e, w, inputs, how):
+    import torch
+
+    from paper_2602_10729_gb300 import boute as bt
+    if how == "host":
+        idx = torch.empty((w.B, w.k), dtype=torch.int64).pin_memory()
+        val = torch.empty((w.B, w.k), dtype=torch.float32).pin_memory()
+        bt.boute_engine_step_host(e, *inputs, idx, val)
+        return idx.numpy().copy(), val.numpy().copy()
+    idx = torch.empty((w.B, w.k), dtype=torch.int64, device="cuda")
+    val = torch.empty((w.B, w.k), dtype=torch.float32, device="cuda")
+    if how == "legacy":  # eager launches on the legacy default stream
+        torch.cuda.synchronize()
+        bt.boute_engine_step(e, *inputs, idx, val, stream=0)
+    else:
+        bt.boute_engine_step(e, *inputs, idx, val)
+    return idx.cpu().numpy(), val.cpu().numpy()
+
+
+@pytest.mark.parametrize("case", CASES, ids=lambda c: wl.WORKLOADS[c[0]].name)
+def test_engine_paths_agree_and_match_oracle(case):
+    import torch
+
+    from paper_2602_10729_gb300 import boute as bt
+    wi, N, B = case
+    w = wl.scaled(wl.WORKLOADS[wi], N=N, B=B)
+    hp = host_problem(w)
+    e = _engine(w)
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        ref_idx, ref_val = _run(e, w, _dev(hp), "device")
+        for how in ("device", "host", "legacy"):  # graph replay, host copies, eager
+            idx, val = _run(e, w, _host(hp) if how == "host" else _dev(hp), how)
+            assert np.array_equal(idx, ref_idx), how
+            assert np.array_equal(val, ref_val), how
+        bt.boute_engine_set_timing(e, True)
+        idx, val = _run(e, w, _dev(hp), "device")
+        times = bt.boute_engine_stage_times(e)
+        bt.boute_engine_set_timing(e, False)
+        assert np.array_equal(idx, ref_idx) and np.array_equal(val, ref_val)
+        assert all(v > 0 for v in times.values()), times
+        acq = torch.empty((w.B, w.N), dtype=torch.float32, device="cuda")
+        bt.boute_engine_scores(e, acq=acq)
+        torch.cuda.synchronize()
+    e.free()
+    A = acq.cpu().numpy()
+    g = gpu_pipeline(hp)  # the step-by-step calls: same scores as the engine
+    assert np.array_equal(g["acq"], A)
+    for b in range(w.B):
+        fp = oracle_fit(hp, b)
+        mean, var = opl.posterior(fp, hp.Xc[b])
+        eps = None if hp.eps is None else hp.eps[b]
+        check_acq_end_to_end(A[b], lambda mm, vv: opl.acquisition(fp, mm, vv, w.mode, eps),
+                             g["mean"][b].T, g["var"][b].T, mean, var, fp.s2)
+        assert np.array_equal(ref_val[b], A[b][ref_idx[b]])
+
+
+def test_consecutive_host_steps_with_new_inputs():
+    w = wl.scaled(wl.WORKLOADS[1], N=2000 + 7, B=1)
+    hp1 = host_problem(w)
+    hp2 = host_problem(wl.scaled(w, N=w.N), threads=4)
+    rng = np.random.default_rng(5)
+    hp2.Xc[:] = rng.random(hp2.Xc.shape).astype(np.float32)
+    hp2.eps[:] = rng.standard_normal(hp2.eps.shape).astype(np.float32)
+    e = _engine(w)
+    want = [_run(e, w, _dev(h), "device") for h in (hp1, hp2)]
+    got = [_run(e, w, _host(h), "host") for h in (hp1, hp2, hp1)]
+    e.free()
+    for (gi, gv), (wi_, wv) in zip(got, want + want[:1]):
+        assert np.array_equal(gi, wi_)
+        assert np.array_equal(gv, wv)
