@@ -30,6 +30,7 @@ __global__ void __launch_bounds__(256) ehvi2d_kernel(const float *mean, const fl
                                                      const int *P, int n, const double *ref,
                                                      float *acq) {
   extern __shared__ float cells[];  // bnd[n+1] (b_i), up[n+1] (u_i)
+  pdl_wait();
   const int b = blockIdx.y;
   const int Pb = P[b];
   float *bnd = cells, *up = cells + (n + 1);
@@ -73,6 +74,7 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
                                                     int box_cap, const float *eps, int S,
                                                     long long eps_stride, float *acq) {
   extern __shared__ float boxes[];  // per problem in this block: lo[K][M], hi[K][M]
+  pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
   const int b = blockIdx.y;
   const int K = Kc[b];
@@ -165,6 +167,7 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
   extern __shared__ float4 strips4[];  // k >= 1: (b/D, 1/D, D u, D); [0]: (b_0, u_0, -, -)
   float *sb = (float *)(strips4 + box_cap);  // b_k, for the pruning scans
   float *su = sb + box_cap;                  // u_k
+  pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
   const int b = blockIdx.y;
   const int K = Kc[b];
@@ -291,8 +294,8 @@ int launch_ehvi(const float *mean, const float *var, int B, long long N, const d
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
   const long long want = (N + 255) / 256;
   const unsigned gx = (unsigned)std::max<long long>(1, std::min<long long>(want, (long long)sms * 8 / std::max(1, B) + 1));
-  ehvi2d_kernel<<<dim3(gx, B), 256, 2 * (n + 1) * sizeof(float), s>>>(mean, var, N, front, P, n,
-                                                                     ref, acq);
+  launch_pdl(ehvi2d_kernel, dim3(gx, B), dim3(256), 2 * (n + 1) * sizeof(float), s, mean, var, N,
+             front, P, n, ref, acq);
   count_launch();
   return last_launch_status();
 }
@@ -317,11 +320,11 @@ int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
     prefer_shared(mchvi2_kernel);
     if (smem2 > 48 * 1024)
       cudaFuncSetAttribute(mchvi2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
-    mchvi2_kernel<<<dim3(gx, B), wpb * 32, smem2, s>>>(
-        mean, var, N, lower, upper, K, box_cap, eps, S, eps_stride, acq);
+    launch_pdl(mchvi2_kernel, dim3(gx, B), dim3(wpb * 32), smem2, s, mean, var, N, lower, upper, K,
+               box_cap, eps, S, eps_stride, acq);
   } else if (m == 3) {
-    mchvi_kernel<3><<<dim3(gx, B), wpb * 32, smem, s>>>(mean, var, B, N, lower, upper, K, box_cap,
-                                                        eps, S, eps_stride, acq);
+    launch_pdl(mchvi_kernel<3>, dim3(gx, B), dim3(wpb * 32), smem, s, mean, var, B, N, lower, upper,
+               K, box_cap, eps, S, eps_stride, acq);
   } else {
     return BOUTE_ERR_UNSUPPORTED;
   }

@@ -142,6 +142,17 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// ---- programmatic dependent launch -----------------------------------------------
+// A kernel launched with programmatic stream serialization may start while its
+// predecessor in the stream is still running: it must call pdl_wait() before
+// reading anything that predecessor writes. pdl_trigger() lets the successor
+// start launching; without it the successor launches when this grid's blocks
+// have exited. Both are no-ops for a grid launched without the attribute.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---- tcgen05 (5th-generation tensor cores, tensor memory) -------------------
 __device__ __forceinline__ void tmem_alloc(uint32_t *dst_smem, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(

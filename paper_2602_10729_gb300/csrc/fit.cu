@@ -117,9 +117,10 @@ __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad
 __global__ void __launch_bounds__(256) fit_setup_kernel(
     const double *X, int n, int d, int m, int DP, int npad, const double *ls, const double *s2,
     const double *noise, float *Kh_all, float *Kl_all, float *xt, float *s2f, int nkt, int nprep,
-    int *status) {
+    int early_trigger, int *status) {
   __shared__ double il[BOUTE_MAX_D];
   const int bt = blockIdx.y, b = bt / m;
+  if (early_trigger) pdl_trigger();  // the whole grid is resident: the fit may launch now
   const double *l = ls + (size_t)bt * d;
   if (blockIdx.x == 0 && bt == 0 && threadIdx.x == 0) *status = BOUTE_OK;
   if ((int)blockIdx.x < nkt) {
@@ -187,7 +188,7 @@ template <bool SMEM>
 __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     const float *Kh_all, const float *Kl_all, const double *Ys, int standardize, int n, int m,
     float *Aws, float *Wws, float *xt, int DP, int npad, PostPlan plan, float *bop, int kl_smem,
-    int *status) {
+    int early_trigger, int *status) {
   extern __shared__ __align__(16) float sm[];
   __shared__ int bad;
   __shared__ uint64_t lbar;
@@ -205,10 +206,37 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   float *ylo = vec, *dg = vec + NP, *yv = vec + 2 * NP, *tv = vec + 3 * NP, *al = vec + 4 * NP,
         *rv = vec + 5 * NP;
   const double *y = Ys + (size_t)b * n * m + t;
+  if (early_trigger) pdl_trigger();  // every block is resident: the posterior may launch
+  // standardize != 0: Ys holds raw outcomes; this column is standardised here
+  // (zero mean, unit sample standard deviation, as standardize_kernel does)
+  if (standardize) {  // warp 0 alone: few fp64 instructions
+    if (warp == 0) {
+      double sum = 0.0;
+      for (int i = lane; i < n; i += 32) sum += y[(size_t)i * m];
+      const double mean = warp_sum(sum) / n;
+      double ss = 0.0;
+      for (int i = lane; i < n; i += 32) {
+        const double z = y[(size_t)i * m] - mean;
+        ss += z * z;
+      }
+      ss = warp_sum(ss);
+      double sd = n > 1 ? sqrt(ss / (n - 1)) : 1.0;
+      if (!(sd >= 1e-8)) sd = 1.0;
+      if (lane == 0) {
+        ymu = mean;
+        yisd = 1.0 / sd;
+      }
+    }
+  } else if (tid == 0) {
+    ymu = 0.0;
+    yisd = 1.0;
+  }
+  // everything below reads what the set-up kernel wrote
+  pdl_wait();
   // A = K (hi; the lower triangle becomes L, the upper triangle keeps K for the
   // residual), padded with the identity to NP x NP. In shared memory with n
   // even, K hi (and, for n <= 128, K lo) arrive by bulk copy, K hi staged in
-  // the W area, while the outcomes are standardised.
+  // the W area.
   float *Kls = kl_smem ? vec + 6 * NP : nullptr;  // K lo, n x n (shared)
   const bool bulk = SMEM && (n % 2 == 0);
   if (bulk) {
@@ -247,30 +275,6 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   for (int e = tid; e < (NP - n) * NP; e += nthr) {
     const int i = n + e / NP, k = e % NP;
     if (k <= i) A[(size_t)i * ld + k] = (k == i) ? 1.f : 0.f;
-  }
-  // standardize != 0: Ys holds raw outcomes; this column is standardised here
-  // (zero mean, unit sample standard deviation, as standardize_kernel does)
-  if (standardize) {  // warp 0 alone: few fp64 instructions
-    if (warp == 0) {
-      double sum = 0.0;
-      for (int i = lane; i < n; i += 32) sum += y[(size_t)i * m];
-      const double mean = warp_sum(sum) / n;
-      double ss = 0.0;
-      for (int i = lane; i < n; i += 32) {
-        const double z = y[(size_t)i * m] - mean;
-        ss += z * z;
-      }
-      ss = warp_sum(ss);
-      double sd = n > 1 ? sqrt(ss / (n - 1)) : 1.0;
-      if (!(sd >= 1e-8)) sd = 1.0;
-      if (lane == 0) {
-        ymu = mean;
-        yisd = 1.0 / sd;
-      }
-    }
-  } else if (tid == 0) {
-    ymu = 0.0;
-    yisd = 1.0;
   }
   __syncthreads();
   const double mu_y = ymu, isd_y = yisd;
@@ -642,22 +646,29 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
   const int tn = (n + 15) / 16, nkt = tn * tn;
   const int nprep = std::max(1, std::min(8, npad * gp->DP / 256));
   prefer_shared(fit_setup_kernel);
+  const int sms = num_sms();
+  // early triggers only when every block of the grid is resident at once (8
+  // set-up blocks per SM beside the fit's blocks; one fit block per SM), so
+  // that waiting successors can never hold resources a later block needs
+  const long long setup_blocks = (long long)(nkt + nprep) * BM;
+  const int setup_early = setup_blocks <= 8LL * (sms - BM) ? 1 : 0;
+  const int fit_early = 2 * BM <= sms ? 1 : 0;
   fit_setup_kernel<<<dim3(nkt + nprep, BM), 256, 0, s>>>(X, n, d, m, gp->DP, npad, ls, s2, noise,
                                                          gp->Kh, gp->Kl, gp->xt, gp->s2f, nkt,
-                                                         nprep, gp->status);
+                                                         nprep, setup_early, gp->status);
   if (fit_uses_smem(npad)) {
     const size_t smem = fit_smem_bytes(npad, n);
     prefer_shared(fit32_kernel<true>);
     cudaFuncSetAttribute(fit32_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);
-    fit32_kernel<true><<<BM, fit_threads<true>(), smem, s>>>(
-        gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan,
-        gp->bop, fit_kl_in_smem(n) ? 1 : 0, gp->status);
+    launch_pdl(fit32_kernel<true>, dim3(BM), dim3(fit_threads<true>()), smem, s, gp->Kh, gp->Kl,
+               Ys, standardize, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop,
+               fit_kl_in_smem(n) ? 1 : 0, fit_early, gp->status);
     count_launch(2);
   } else {
-    fit32_kernel<false><<<BM, fit_threads<false>(), 6 * npad * sizeof(float), s>>>(
-        gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan,
-        gp->bop, 0, gp->status);
+    launch_pdl(fit32_kernel<false>, dim3(BM), dim3(fit_threads<false>()),
+               6 * npad * sizeof(float), s, gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws,
+               gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop, 0, 0, gp->status);
     const long long tot = (long long)gp->plan.ncols * npad;
     pack_kernel<<<dim3((unsigned)std::min<long long>((tot + 255) / 256, 4096), BM), 256, 0, s>>>(
         gp->Wws, gp->plan, gp->bop, gp->status);

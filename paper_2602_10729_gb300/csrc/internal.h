@@ -28,6 +28,32 @@ inline void prefer_shared(F *kernel) {
                        (int)cudaSharedmemCarveoutMaxShared);
 }
 
+// Launch with programmatic stream serialization: the kernel may begin while
+// the previous kernel on the stream finishes, and waits (pdl_wait) before
+// reading its results.
+template <class... KArgs, class... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args &&...args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
+inline int num_sms() {
+  int dev = 0, sms = 152;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  return sms;
+}
+
 void count_launch(int k = 1);
 unsigned long long launch_count();
 int last_launch_status();  // BOUTE_OK or BOUTE_ERR_CUDA after a launch

@@ -212,6 +212,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
+  pdl_wait();  // the fit's outputs (operand images, side input) are complete
 
   if (warp == 0 || warp == kXtWarp) {
     // ------------------------------------------------------ producers (B / side input)
@@ -458,6 +459,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   }
 
   // ---- teardown -----------------------------------------------------------------
+  pdl_trigger();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -511,7 +513,7 @@ int launch_dp(const Gp *gp, const float *Xc, long long N, float *mean, float *va
   int sms = 152;
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
   const int grid = std::max(1, std::min(a.tiles_total * a.m, sms));  // (tile, objective) units
-  posterior_kernel<DP><<<grid, Layout<DP>::kThreads, smem, s>>>(a);
+  launch_pdl(posterior_kernel<DP>, dim3(grid), dim3(Layout<DP>::kThreads), smem, s, a);
   count_launch();
   return last_launch_status();
 }

@@ -57,6 +57,7 @@ __global__ void __launch_bounds__(kThreads) segment_topk_kernel(
     const float *vals, const unsigned long long *keys_in, long long len, int k, int nseg,
     unsigned long long *keys_out, const float *acq, long long N, long long *idx, float *val) {
   __shared__ unsigned long long buf[kSeg];
+  pdl_wait();
   const int b = blockIdx.y, seg = blockIdx.x;
   const long long base = (long long)seg * kSeg;
   const long long n_here = std::min<long long>(kSeg, len - base);
@@ -143,6 +144,7 @@ __global__ void __launch_bounds__(kWarpBlock) warp_topk_kernel(
     unsigned long long *keys_out, const float *acq, long long N, int k, long long *idx,
     float *val) {
   __shared__ unsigned long long lists[kWarpBlock / 32][kWarpK];
+  pdl_wait();
   const int b = blockIdx.y, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const long long lo = (long long)blockIdx.x * per_block;
   const long long hi = std::min<long long>(len, lo + per_block);
@@ -189,18 +191,23 @@ int launch_topk_warp(const float *acq, int B, long long N, int k, long long *idx
   const long long G = (N + per_block - 1) / per_block;
   prefer_shared(warp_topk_kernel<true>);
   prefer_shared(warp_topk_kernel<false>);
+  const float *nf = nullptr;
+  const unsigned long long *nk = nullptr;
+  unsigned long long *nko = nullptr;
+  long long *ni = nullptr;
+  float *nv = nullptr;
   if (G == 1) {
-    warp_topk_kernel<true><<<dim3(1, B), kWarpBlock, 0, s>>>(acq, nullptr, N, per_block, nullptr,
-                                                              acq, N, k, idx, val);
+    launch_pdl(warp_topk_kernel<true>, dim3(1, B), dim3(kWarpBlock), 0, s, acq, nk, N, per_block,
+               nko, acq, N, k, idx, val);
     count_launch(1);
     return last_launch_status();
   }
   unsigned long long *keys = (unsigned long long *)scratch;
-  warp_topk_kernel<true><<<dim3((unsigned)G, B), kWarpBlock, 0, s>>>(
-      acq, nullptr, N, per_block, keys, acq, N, k, nullptr, nullptr);
+  launch_pdl(warp_topk_kernel<true>, dim3((unsigned)G, B), dim3(kWarpBlock), 0, s, acq, nk, N,
+             per_block, keys, acq, N, k, ni, nv);
   const long long len2 = G * kWarpK;
-  warp_topk_kernel<false><<<dim3(1, B), kWarpBlock, 0, s>>>(nullptr, keys, len2, len2, nullptr,
-                                                             acq, N, k, idx, val);
+  launch_pdl(warp_topk_kernel<false>, dim3(1, B), dim3(kWarpBlock), 0, s, nf, keys, len2, len2,
+             nko, acq, N, k, idx, val);
   count_launch(2);
   return last_launch_status();
 }
