@@ -146,17 +146,28 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
 
 // 2-objective Monte-Carlo HVI over the strip decomposition: strips k = 0..K-1
 // with x-extent [a_k, b_k) (a_0 = -inf, a_k = b_{k-1}) and top u_k (u
-// decreasing). For a sample y the improvement is
+// decreasing, u_0 = r2 the largest). For a sample y the improvement is
 //   sum_k (b_k - max(a_k, y1))^+ (u_k - y2)^+
-//     = (b_0 - y1)^+ (u_0 - y2)^+ + sum_{k>=1} D_k sat((b_k - y1) / D_k) (u_k - y2)^+,
-// D_k = b_k - a_k, because (b_k - max(a_k, y1))^+ is (b_k - y1) clamped to
-// [0, D_k]. Per strip and sample: one saturating FMA, one FMA and a max for
-// the height with D_k folded in, one FMA to accumulate. One warp per
-// candidate, a float4 of base normals per lane and objective when S = 128.
+//     = (b_0 - y1)^+ (u_0 - y2)^+ + H sum_{k>=1} D_k sat((b_k - y1) / D_k) sat((u_k - y2) / H)
+// with D_k = b_k - a_k, because (b_k - max(a_k, y1))^+ is (b_k - y1) clamped
+// to [0, D_k], and with H = u_0 - min y2 >= u_k - y2 over the samples a thread
+// holds, so that (u_k - y2)^+ = H sat((u_k - y2) / H). Per strip and sample:
+// two saturating FMAs and one FMA. One warp per candidate, a float4 of base
+// normals per lane and objective when S = 128.
 __device__ __forceinline__ float fma_sat(float a, float b, float c) {
   float d;
   asm("fma.rn.sat.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
   return d;
+}
+__device__ __forceinline__ float sqrt_fast(float x) {
+  float y;
+  asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float rcp_fast(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const float *var,
@@ -164,8 +175,8 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
                                                      const float *upper, const int *Kc,
                                                      int box_cap, const float *eps, int S,
                                                      long long eps_stride, float *acq) {
-  extern __shared__ float4 strips4[];  // k >= 1: (b/D, 1/D, D u, D); [0]: (b_0, u_0, -, -)
-  float *sb = (float *)(strips4 + box_cap);  // b_k, for the pruning scans
+  extern __shared__ float4 strips4[];  // k >= 1: (b/D, 1/D, u, D); [0]: (b_0, u_0, -, -)
+  float *sb = (float *)(strips4 + box_cap);  // b_k
   float *su = sb + box_cap;                  // u_k
   pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
@@ -180,8 +191,7 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
       strips4[0] = make_float4(bi, ui, 0.f, 0.f);
     } else {
       const float D = bi - ai;
-      strips4[i] = D > 0.f ? make_float4(bi / D, 1.f / D, D * ui, D)
-                           : make_float4(0.f, 0.f, 0.f, 0.f);
+      strips4[i] = D > 0.f ? make_float4(bi / D, 1.f / D, ui, D) : make_float4(0.f, 0.f, ui, 0.f);
     }
   }
   __syncthreads();
@@ -189,23 +199,21 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
   const float *v1 = var + (size_t)b * 2 * N, *v2 = v1 + N;
   const bool vec = (S == 128) && ((uintptr_t)eps & 15) == 0 && (eps_stride % 4) == 0;
   const long long cstride = (long long)gridDim.x * wpb;
+  const float inv_s = 1.f / (float)S;
   auto eps_of = [&](long long c) {
     return eps + ((size_t)b * N + c) * eps_stride + (eps_stride == 0 ? (size_t)b * 2 * S : 0);
   };
-  // improvement of one sample from strips [k0, k1)
-  auto hvi = [&](float y1, float y2, int k0, int k1) {
+  // improvement of one sample (the direct strip sum)
+  auto hvi = [&](float y1, float y2) {
     float acc = 0.f;
-    int k = k0;
-    if (k == 0 && k < k1) {
+    if (K > 0) {
       const float4 t = strips4[0];
       acc = fmaxf(t.x - y1, 0.f) * fmaxf(t.y - y2, 0.f);
-      k = 1;
     }
-    for (; k < k1; ++k) {
+    for (int k = 1; k < K; ++k) {
       const float4 t = strips4[k];
       const float w = fma_sat(-y1, t.y, t.x);
-      const float h = fmaxf(fmaf(-y2, t.w, t.z), 0.f);
-      acc = fmaf(w, h, acc);
+      acc = fmaf(w * t.w, fmaxf(t.z - y2, 0.f), acc);
     }
     return acc;
   };
@@ -221,10 +229,11 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
       z2 = __ldcs((const float4 *)(e + S + 4 * lane));
       pm1 = m1[c]; pm2 = m2[c]; pv1 = v1[c]; pv2 = v2[c];
     }
+    const float u0 = K > 0 ? su[0] : 0.f;
     for (; c < N; c += cstride) {
       const float4 c1 = z1, c2 = z2;
       const float mu1 = pm1, mu2 = pm2;
-      const float sg1 = sqrtf(fmaxf(pv1, 0.f)), sg2 = sqrtf(fmaxf(pv2, 0.f));
+      const float sg1 = sqrt_fast(fmaxf(pv1, 0.f)), sg2 = sqrt_fast(fmaxf(pv2, 0.f));
       const long long cn = c + cstride;
       if (cn < N) {
         const float *e = eps_of(cn);
@@ -236,52 +245,43 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
                            fmaf(sg1, c1.w, mu1)};
       const float y2[4] = {fmaf(sg2, c2.x, mu2), fmaf(sg2, c2.y, mu2), fmaf(sg2, c2.z, mu2),
                            fmaf(sg2, c2.w, mu2)};
-      // strips no sample of this candidate can reach contribute exactly zero:
-      // b_k <= min y1 (b increasing) or u_k <= min y2 (u decreasing)
-      float lo1 = fminf(fminf(y1[0], y1[1]), fminf(y1[2], y1[3]));
-      float lo2 = fminf(fminf(y2[0], y2[1]), fminf(y2[2], y2[3]));
+      // per lane: H = u_0 - (its lowest y2) bounds every height of its samples
+      const float lo2 = fminf(fminf(y2[0], y2[1]), fminf(y2[2], y2[3]));
+      const float H = u0 - lo2;
+      float sum = 0.f;
+      if (K > 0) {
+        const float4 t0 = strips4[0];
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        lo1 = fminf(lo1, __shfl_xor_sync(0xffffffffu, lo1, o));
-        lo2 = fminf(lo2, __shfl_xor_sync(0xffffffffu, lo2, o));
-      }
-      int k0 = 0, k1 = K;
-      while (k0 < K && sb[k0] <= lo1) ++k0;
-      while (k1 > k0 && su[k1 - 1] <= lo2) --k1;
-      float acc[4] = {0.f, 0.f, 0.f, 0.f};
-      int k = k0;
-      if (k == 0 && k < k1) {
-        const float4 t = strips4[0];
+        for (int j = 0; j < 4; ++j) sum += fmaxf(t0.x - y1[j], 0.f) * fmaxf(t0.y - y2[j], 0.f);
+        const float iH = H > 0.f ? rcp_fast(H) : 0.f;  // H <= 0: every sample dominated
+        float acc = 0.f;
+#pragma unroll 2
+        for (int k = 1; k < K; ++k) {
+          const float4 t = strips4[k];
+          const float uh = t.z * iH;
+          float tk = 0.f;
 #pragma unroll
-        for (int j = 0; j < 4; ++j) acc[j] = fmaxf(t.x - y1[j], 0.f) * fmaxf(t.y - y2[j], 0.f);
-        k = 1;
-      }
-      for (; k < k1; ++k) {
-        const float4 t = strips4[k];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const float w = fma_sat(-y1[j], t.y, t.x);
-          const float h = fmaxf(fmaf(-y2[j], t.w, t.z), 0.f);
-          acc[j] = fmaf(w, h, acc[j]);
+          for (int j = 0; j < 4; ++j)
+            tk = fmaf(fma_sat(-y1[j], t.y, t.x), fma_sat(-y2[j], iH, uh), tk);
+          acc = fmaf(t.w, tk, acc);
         }
+        sum = fmaf(fmaxf(H, 0.f), acc, sum);
       }
-      float sum = (acc[0] + acc[1]) + (acc[2] + acc[3]);
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-      if (lane == 0) acq[(size_t)b * N + c] = sum / (float)S;
+      if (lane == 0) acq[(size_t)b * N + c] = sum * inv_s;
     }
     return;
   }
   for (long long c = (long long)blockIdx.x * wpb + warp; c < N; c += cstride) {
     const float mu1 = m1[c], mu2 = m2[c];
-    const float sg1 = sqrtf(fmaxf(v1[c], 0.f)), sg2 = sqrtf(fmaxf(v2[c], 0.f));
+    const float sg1 = sqrt_fast(fmaxf(v1[c], 0.f)), sg2 = sqrt_fast(fmaxf(v2[c], 0.f));
     const float *e = eps_of(c);
     float sum = 0.f;
-    for (int s = lane; s < S; s += 32)
-      sum += hvi(fmaf(sg1, e[s], mu1), fmaf(sg2, e[S + s], mu2), 0, K);
+    for (int s = lane; s < S; s += 32) sum += hvi(fmaf(sg1, e[s], mu1), fmaf(sg2, e[S + s], mu2));
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    if (lane == 0) acq[(size_t)b * N + c] = sum / (float)S;
+    if (lane == 0) acq[(size_t)b * N + c] = sum * inv_s;
   }
 }
 
