@@ -116,6 +116,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t phase) {
   return ok != 0;
 }
 
+// As mbar_try_wait, but the thread may stay suspended in hardware for up to
+// hint_ns while the phase is incomplete (it resumes as soon as the phase
+// completes), so a waiting warp takes no issue slots from the working ones.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t *bar, uint32_t phase,
+                                                    uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(phase), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+
 // Waits for the given phase parity; gives up after BOUTE_WAIT_NS and returns
 // false so the caller can record BOUTE_ERR_TIMEOUT instead of hanging.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t phase) {

@@ -130,20 +130,29 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// Bounded wait that also gives up as soon as another role has aborted.
-// Waiters that are not on the critical path back off with nanosleep so that
-// their polling does not take issue slots from the K* builders.
+// Position in a ring of R stages: the stage index and the parity of the
+// stage's use count (the mbarrier phase a consumer waits for), advanced
+// without integer division.
+struct RingPos {
+  int idx = 0;
+  uint32_t phase = 0;
+  __device__ __forceinline__ void advance(int R) {
+    if (++idx == R) {
+      idx = 0;
+      phase ^= 1u;
+    }
+  }
+};
+
+// Bounded wait that also gives up as soon as another role has aborted. The
+// waiting thread sleeps in hardware until the phase completes (at most 2 us
+// per try), so waiting warps take no issue slots from the K* builders.
 __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity,
-                                              volatile int *abort, uint32_t max_sleep_ns = 0) {
+                                              volatile int *abort) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
-  uint32_t sleep = 16;
   for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if (max_sleep_ns) {
-      __nanosleep(sleep);
-      sleep = sleep * 2 < max_sleep_ns ? sleep * 2 : max_sleep_ns;
-    }
+    if (mbar_try_wait_sleep(bar, parity, 2000)) return true;
     if ((it & 15) == 0) {
       if (*abort) return false;
       if (globaltimer() - t0 > BOUTE_WAIT_NS) {
@@ -161,8 +170,10 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   constexpr int COLS = Layout<DP>::kCols;   // columns of a chunk per builder thread
   constexpr int GPR = 32 / COLS;            // column groups per row (threads per row)
   constexpr int RPW = 32 / GPR;             // rows per builder warp
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t *sm = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  // 1024-byte alignment (the 128-byte swizzle atom) as an offset from the
+  // shared array, so that every access below stays a shared-memory access
+  uint8_t *sm = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const PostPlan &pl = a.plan;
   const int n = a.n, m = a.m, d = a.d, SA = a.sa, SB = a.sb, SX = a.sx;
@@ -221,6 +232,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       const int R = is_b ? SB : SX;
       uint64_t *full = is_b ? b_full : x_full, *empty = is_b ? b_empty : x_empty;
       uint32_t q = 0;
+      RingPos rp;
       int last_q = -1;  // last job issued
       for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
         const int tile = unit / m, t = unit % m;
@@ -229,10 +241,9 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
           const int bt = b * m + t;
           for (int p = 0; p < pl.npass && !*abort; ++p) {
             const uint32_t bbytes = (uint32_t)(2 * pl.ncol[p] * 128);
-            for (int c = 0; c < pl.kc[p]; ++c, ++q) {
-              const int s = q % R;
-              const uint32_t use = q / R;
-              if (use >= 1 && !wait_or_abort(&empty[s], (use - 1) & 1, abort, 128)) break;
+            for (int c = 0; c < pl.kc[p]; ++c, ++q, rp.advance(R)) {
+              const int s = rp.idx;
+              if (q >= (uint32_t)R && !wait_or_abort(&empty[s], rp.phase ^ 1u, abort)) break;
               if (is_b) {
                 mbar_arrive_expect_tx(&full[s], bbytes);
                 bulk_g2s(b_reg(s),
@@ -260,26 +271,27 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       uint32_t q = 0, nuse[2] = {0u, 0u};
       int nxt = 0;
       bool issued = false;
+      RingPos pa, pb;
       for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
         {
           for (int p = 0; p < pl.npass && !*abort; ++p) {
             const int kc = pl.kc[p], h = split_chunks(kc);
             const bool split = h < kc;  // second half of the reduction -> other buffer
             const int A = nxt, Bf = nxt ^ 1;
-            if (nuse[A] >= 1 && !wait_or_abort(&acc_empty[A], (nuse[A] - 1) & 1, abort, 64)) break;
+            if (nuse[A] >= 1 && !wait_or_abort(&acc_empty[A], (nuse[A] - 1) & 1, abort)) break;
             if (split && nuse[Bf] >= 1 &&
-                !wait_or_abort(&acc_empty[Bf], (nuse[Bf] - 1) & 1, abort, 64))
+                !wait_or_abort(&acc_empty[Bf], (nuse[Bf] - 1) & 1, abort))
               break;
             tc_fence_after();
             const int ncol = pl.ncol[p];
             const uint32_t idesc = idesc_tf32(ncol);
-            for (int c = 0; c < kc; ++c, ++q) {
+            for (int c = 0; c < kc; ++c, ++q, pa.advance(SA), pb.advance(SB)) {
               const bool second = split && c >= h;
               const uint32_t dtm = tmem + (uint32_t)((second ? Bf : A) * 256);
               const int c0 = second ? h : 0;  // first chunk of this accumulator
-              const int sa = q % SA, sb = q % SB;
-              if (!wait_or_abort(&b_full[sb], (q / SB) & 1, abort, 32)) break;
-              if (!wait_or_abort(&a_full[sa], (q / SA) & 1, abort, 32)) break;
+              const int sa = pa.idx, sb = pb.idx;
+              if (!wait_or_abort(&b_full[sb], pb.phase, abort)) break;
+              if (!wait_or_abort(&a_full[sa], pa.phase, abort)) break;
               tc_fence_after();
               const uint32_t sah = smem_u32(a_hi(sa)), sal = smem_u32(a_lo(sa));
               const uint32_t sbh = smem_u32(b_reg(sb)), sbl = sbh + ncol * 128;
@@ -324,8 +336,8 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
           const int kc = pl.kc[p];
           const bool split = split_chunks(kc) < kc;
           const int A = nxt, Bf = nxt ^ 1;
-          if (!wait_or_abort(&acc_full[A], nuse[A] & 1, abort, 512)) break;
-          if (split && !wait_or_abort(&acc_full[Bf], nuse[Bf] & 1, abort, 512)) break;
+          if (!wait_or_abort(&acc_full[A], nuse[A] & 1, abort)) break;
+          if (split && !wait_or_abort(&acc_full[Bf], nuse[Bf] & 1, abort)) break;
           tc_fence_after();
           const uint32_t lanes = (uint32_t)(32 * eq) << 16;
           const uint32_t ta = tmem + (uint32_t)(A * 256) + lanes;
@@ -365,6 +377,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
     const int bw = warp - kBldWarp0;
     const int r = bw * RPW + lane % RPW, g = lane / RPW;
     uint32_t q = 0;
+    RingPos pa, px;
     for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
       const int tile = unit / m, t = unit % m;
       const int b = tile / a.tiles_per_problem;
@@ -379,10 +392,10 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
         float mu = 0.f, comp = 0.f;
         for (int p = 0; p < pl.npass && !*abort; ++p) {
           const bool last_pass = p == pl.npass - 1;
-          for (int c = 0; c < pl.kc[p]; ++c, ++q) {
-            const int s = q % SA, j = q % SX;
-            if (q >= (uint32_t)SA && !wait_or_abort(&a_empty[s], (q / SA - 1) & 1, abort)) break;
-            if (!wait_or_abort(&x_full[j], (q / SX) & 1, abort)) break;
+          for (int c = 0; c < pl.kc[p]; ++c, ++q, pa.advance(SA), px.advance(SX)) {
+            const int s = pa.idx, j = px.idx;
+            if (q >= (uint32_t)SA && !wait_or_abort(&a_empty[s], pa.phase ^ 1u, abort)) break;
+            if (!wait_or_abort(&x_full[j], px.phase, abort)) break;
             const float *xth = xt_reg(j), *xtl = xth + BOUTE_KCHUNK * DP;  // x hi, x lo
             const float *alp = xtl + BOUTE_KCHUNK * DP;
             if (p == 0 && c == 0) {  // new objective: its parameters came with the chunk
