@@ -193,8 +193,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   __shared__ int bad;
   __shared__ uint64_t lbar;
   __shared__ double ymu, yisd;
-  __shared__ __align__(16) float colb[2][32];
-  __shared__ __align__(16) float wrow[2][32];
+  __shared__ __align__(16) float colz[64];  // a column of L_pp, zero-padded
   const int bt = blockIdx.x, b = bt / m, t = bt % m;
   const int tid = threadIdx.x, nthr = blockDim.x, lane = tid & 31, warp = tid >> 5,
             nw = nthr >> 5;
@@ -297,6 +296,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     dg[i] = A[(size_t)i * ld + i];
   }
   if (tid == 0) bad = 0;
+  if (tid < 64) colz[tid] = 0.f;
   __syncthreads();
   // ---- blocked Cholesky and W = L^-1, 32-column panels -------------------------
   // Iteration p: (a) warp 0 factors the diagonal block, A_pp = L_pp L_pp^T,
@@ -311,7 +311,11 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   for (int p = 0; p < nb; ++p) {
     const int p0 = 32 * p;
     if (warp == 0) {
-      float a[32], w[32];  // row lane of A_pp (becoming L_pp) and of R (becoming W_pp)
+      // Lane = row of the block. a[] is a window on the lane's row that moves
+      // one column right every step (a[0] is always column c), so the step
+      // loop runs with static register indices and stays small enough for
+      // the instruction cache. w[] is the lane's row of R (becoming W_pp).
+      float a[32], w[32];
       float *Ar = A + (size_t)(p0 + lane) * ld + p0;
 #pragma unroll
       for (int c = 0; c < 32; ++c) {
@@ -321,44 +325,32 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
       const float dgl = dg[p0 + lane];
       bool ok = true;
       float myinv = 0.f;
-      float pivn = __shfl_sync(FULL, a[0], 0);
-#pragma unroll
+#pragma unroll 1
       for (int c = 0; c < 32; ++c) {
-        const float piv = pivn;
+        const float piv = __shfl_sync(FULL, a[0], c);
         if (!(piv > 16.f * 1.1920929e-7f * __shfl_sync(FULL, dgl, c))) ok = false;
         float inv = rsqrtf(piv);
         inv = inv * fmaf(-0.5f * piv * inv, inv, 1.5f);  // one Newton step; 1 / L_cc
-        const float l = lane > c ? a[c] * inv : (lane == c ? piv * inv : 0.f);
-        if (c < 31) {  // the next pivot straight from lane c+1, ahead of the rest
-          const float an = __shfl_sync(FULL, a[c + 1], c + 1);
-          const float lc = __shfl_sync(FULL, l, c + 1);
-          pivn = fmaf(-lc, lc, an);
-        }
-        a[c] = l;
-        float *cb = colb[c & 1];  // column c of L_pp
-        float *wr = wrow[c & 1];  // row c of R (W_pp's row c times L_cc)
-        cb[lane] = l;
-        if (lane == c) {
-          myinv = inv;
-#pragma unroll
-          for (int k = 0; k <= c; ++k) wr[k] = w[k];
-        }
-        __syncwarp();
-        // Entries above a lane's diagonal collect garbage that is never
-        // stored, so the updates need no predicates.
-#pragma unroll
-        for (int c2 = c + 1; c2 < 32; ++c2) a[c2] = fmaf(-l, cb[c2], a[c2]);
-        // R_i -= L_ic W_c = (L_ic / L_cc) R_c for the rows below c
+        const float l = lane > c ? a[0] * inv : (lane == c ? piv * inv : 0.f);
+        if (lane >= c) Ar[c] = l;
+        colz[lane] = l;  // column c of L_pp; colz[32..63] stay zero
+        if (lane == c) myinv = inv;
+        // R_i -= L_ic W_c = (L_ic / L_cc) R_c for the rows below c; R_c has no
+        // entries right of c, so the full-width update is exact
         const float lw = lane > c ? l * inv : 0.f;
 #pragma unroll
-        for (int k = 0; k <= c; ++k) w[k] = fmaf(-lw, wr[k], w[k]);
+        for (int k = 0; k < 32; ++k) w[k] = fmaf(-lw, __shfl_sync(FULL, w[k], c), w[k]);
+        __syncwarp();
+        // trailing update of the lane's row, shifted one column: entries right
+        // of the block or above the lane's diagonal collect values never stored
+#pragma unroll
+        for (int k = 0; k < 31; ++k) a[k] = fmaf(-l, colz[c + 1 + k], a[k + 1]);
+        a[31] = 0.f;
+        __syncwarp();
       }
       float *Wr = W + (size_t)(p0 + lane) * ld + p0;
 #pragma unroll
-      for (int c = 0; c < 32; ++c) {
-        if (c <= lane) Ar[c] = a[c];
-        Wr[c] = w[c] * myinv;
-      }
+      for (int c = 0; c < 32; ++c) Wr[c] = w[c] * myinv;
       if (!ok && lane == 0) bad = 1;
     }
     __syncthreads();
