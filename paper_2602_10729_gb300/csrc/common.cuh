@@ -158,6 +158,12 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// Named CTA barrier `id` (1..15; 0 is __syncthreads) over `count` threads, a
+// multiple of 32; every warp taking part calls it the same number of times.
+__device__ __forceinline__ void named_barrier_sync(int id, int count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 // ---- programmatic dependent launch -----------------------------------------------
 // A kernel launched with programmatic stream serialization may start while its
 // predecessor in the stream is still running: it must call pdl_wait() before

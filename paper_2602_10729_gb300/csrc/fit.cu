@@ -193,7 +193,8 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   __shared__ int bad;
   __shared__ uint64_t lbar;
   __shared__ double ymu, yisd;
-  __shared__ __align__(16) float colz[64];  // a column of L_pp, zero-padded
+  __shared__ __align__(16) float colL[32][64];  // columns of L_pp, zero-padded
+  __shared__ float invs[32];                    // 1 / L_cc
   const int bt = blockIdx.x, b = bt / m, t = bt % m;
   const int tid = threadIdx.x, nthr = blockDim.x, lane = tid & 31, warp = tid >> 5,
             nw = nthr >> 5;
@@ -296,12 +297,12 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     dg[i] = A[(size_t)i * ld + i];
   }
   if (tid == 0) bad = 0;
-  if (tid < 64) colz[tid] = 0.f;
+  for (int e = tid; e < 32 * 64; e += nthr) (&colL[0][0])[e] = 0.f;
   __syncthreads();
   // ---- blocked Cholesky and W = L^-1, 32-column panels -------------------------
   // Iteration p: (a) warp 0 factors the diagonal block, A_pp = L_pp L_pp^T,
-  // and inverts it, W_pp = L_pp^-1, both register-resident (lane = row of the
-  // block); (b) the panel below, L_rp = A_rp W_pp^T, goes to the still-unused
+  // and warp 1 inverts it one column behind, W_pp = L_pp^-1, both
+  // register-resident (lane = row of the block); (b) the panel below, L_rp = A_rp W_pp^T, goes to the still-unused
   // block column p of W, and T_pJ = sum_{K=J}^{p-1} L_pK W_KJ (J < p) is
   // parked, transposed, in the unused upper triangle of W; (c) the trailing
   // update A_ij -= sum_q L_iq L_jq (rows and columns below the panel), the
@@ -311,20 +312,17 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   for (int p = 0; p < nb; ++p) {
     const int p0 = 32 * p;
     if (warp == 0) {
-      // Lane = row of the block. a[] is a window on the lane's row that moves
-      // one column right every step (a[0] is always column c), so the step
-      // loop runs with static register indices and stays small enough for
-      // the instruction cache. w[] is the lane's row of R (becoming W_pp).
-      float a[32], w[32];
+      // Factor. Lane = row of the block. a[] is a window on the lane's row
+      // that moves one column right every step (a[0] is always column c), so
+      // the step loop runs with static register indices and stays small.
+      // Each column of L_pp and 1 / L_cc go to warp 1 through shared memory,
+      // one named-barrier handshake per step.
+      float a[32];
       float *Ar = A + (size_t)(p0 + lane) * ld + p0;
 #pragma unroll
-      for (int c = 0; c < 32; ++c) {
-        a[c] = (c <= lane) ? Ar[c] : 0.f;
-        w[c] = (c == lane) ? 1.f : 0.f;
-      }
+      for (int c = 0; c < 32; ++c) a[c] = (c <= lane) ? Ar[c] : 0.f;
       const float dgl = dg[p0 + lane];
       bool ok = true;
-      float myinv = 0.f;
 #pragma unroll 1
       for (int c = 0; c < 32; ++c) {
         const float piv = __shfl_sync(FULL, a[0], c);
@@ -333,25 +331,38 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
         inv = inv * fmaf(-0.5f * piv * inv, inv, 1.5f);  // one Newton step; 1 / L_cc
         const float l = lane > c ? a[0] * inv : (lane == c ? piv * inv : 0.f);
         if (lane >= c) Ar[c] = l;
-        colz[lane] = l;  // column c of L_pp; colz[32..63] stay zero
-        if (lane == c) myinv = inv;
-        // R_i -= L_ic W_c = (L_ic / L_cc) R_c for the rows below c; R_c has no
-        // entries right of c, so the full-width update is exact
-        const float lw = lane > c ? l * inv : 0.f;
-#pragma unroll
-        for (int k = 0; k < 32; ++k) w[k] = fmaf(-lw, __shfl_sync(FULL, w[k], c), w[k]);
+        colL[c][lane] = l;  // colL[c][32..63] stay zero
+        if (lane == 0) invs[c] = inv;
         __syncwarp();
+        named_barrier_sync(1, 64);  // column c is ready for warp 1
         // trailing update of the lane's row, shifted one column: entries right
         // of the block or above the lane's diagonal collect values never stored
 #pragma unroll
-        for (int k = 0; k < 31; ++k) a[k] = fmaf(-l, colz[c + 1 + k], a[k + 1]);
+        for (int k = 0; k < 31; ++k) a[k] = fmaf(-l, colL[c][c + 1 + k], a[k + 1]);
         a[31] = 0.f;
-        __syncwarp();
+      }
+      if (!ok && lane == 0) bad = 1;
+    } else if (warp == 1) {
+      // Inverse, one column behind the factor. w[] is the lane's row of
+      // R = e_lane - sum_{j<c} L_lane,j W_j, which becomes W_pp's row after
+      // the division by L_lane,lane. R_c has no entries right of c, so the
+      // full-width update below is exact.
+      float w[32];
+#pragma unroll
+      for (int c = 0; c < 32; ++c) w[c] = (c == lane) ? 1.f : 0.f;
+      float myinv = 0.f;
+#pragma unroll 1
+      for (int c = 0; c < 32; ++c) {
+        named_barrier_sync(1, 64);  // wait for column c
+        const float l = colL[c][lane], inv = invs[c];
+        if (lane == c) myinv = inv;
+        const float lw = lane > c ? l * inv : 0.f;  // R_i -= (L_ic / L_cc) R_c, rows below c
+#pragma unroll
+        for (int k = 0; k < 32; ++k) w[k] = fmaf(-lw, __shfl_sync(FULL, w[k], c), w[k]);
       }
       float *Wr = W + (size_t)(p0 + lane) * ld + p0;
 #pragma unroll
       for (int c = 0; c < 32; ++c) Wr[c] = w[c] * myinv;
-      if (!ok && lane == 0) bad = 1;
     }
     __syncthreads();
     if (bad) break;
