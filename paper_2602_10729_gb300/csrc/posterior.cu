@@ -32,6 +32,7 @@
 #include <math.h>
 
 #include <algorithm>
+#include <type_traits>
 
 #include "internal.h"
 
@@ -411,8 +412,15 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
             for (int e = 0; e < COLS / 2; ++e) acc2[e] = 0ull;
 #pragma unroll
             for (int k = 0; k < DP; ++k) {
-              const unsigned long long *h2 =
-                  (const unsigned long long *)(xth + k * BOUTE_KCHUNK + COLS * g);
+              // 16-byte loads: two training points' coordinate pairs each
+              const ulonglong2 *h4 = (const ulonglong2 *)(xth + k * BOUTE_KCHUNK + COLS * g);
+              unsigned long long h2[COLS / 2];
+#pragma unroll
+              for (int e = 0; e < COLS / 4; ++e) {
+                const ulonglong2 v = h4[e];
+                h2[2 * e] = v.x;
+                h2[2 * e + 1] = v.y;
+              }
 #pragma unroll
               for (int e = 0; e < COLS / 2; ++e) {
                 const unsigned long long df = f2_sub(xs2[k], h2[e]);
@@ -421,33 +429,43 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
             }
             const bool full_chunk = (c + 1) * BOUTE_KCHUNK <= n;
             const int jbase = c * BOUTE_KCHUNK + COLS * g;
+            const float *alg = alp + COLS * g;
             float mu_part = 0.f;
             float *Ah = a_hi(s), *Al = a_lo(s);
+            // kernel values of this thread's COLS columns into the A stage; the
+            // last chunk of a ragged n zeroes the columns beyond n
+            auto emit = [&](auto ragged) {
 #pragma unroll
-            for (int g4 = 0; g4 < COLS / 4; ++g4) {
-              float vh[4], vl[4];
+              for (int g4 = 0; g4 < COLS / 4; ++g4) {
+                float vh[4], vl[4];
 #pragma unroll
-              for (int e2 = 0; e2 < 2; ++e2) {
-                float r2[2];
-                f2_split(acc2[2 * g4 + e2], r2[0], r2[1]);
+                for (int e2 = 0; e2 < 2; ++e2) {
+                  float r2[2];
+                  f2_split(acc2[2 * g4 + e2], r2[0], r2[1]);
 #pragma unroll
-                for (int z = 0; z < 2; ++z) {
-                  const int e = 2 * e2 + z, kk = 4 * g4 + e;
-                  // k = s2 (1 + sqrt5 r + 5/3 r^2) exp(-sqrt5 r), exp(-x) = 2^(-x log2 e)
-                  const float rr = sqrt_approx(r2[z]);
-                  const float sr = kSqrt5 * rr;
-                  float kv = s2 * fmaf(kFiveThirds, r2[z], 1.0f + sr) * ex2_approx(-kSqrt5Log2e * rr);
-                  if (!full_chunk) kv = (jbase + kk < n) ? kv : 0.f;
-                  mu_part = fmaf(kv, alp[COLS * g + kk], mu_part);
-                  const float hi = tf32_rna(kv);
-                  vh[e] = hi;
-                  vl[e] = kv - hi;
+                  for (int z = 0; z < 2; ++z) {
+                    const int e = 2 * e2 + z, kk = 4 * g4 + e;
+                    // k = s2 (1 + sqrt5 r + 5/3 r^2) exp(-sqrt5 r), exp(-x) = 2^(-x log2 e)
+                    const float rr = sqrt_approx(r2[z]);
+                    const float sr = kSqrt5 * rr;
+                    float kv =
+                        s2 * fmaf(kFiveThirds, r2[z], 1.0f + sr) * ex2_approx(-kSqrt5Log2e * rr);
+                    if (decltype(ragged)::value) kv = (jbase + kk < n) ? kv : 0.f;
+                    mu_part = fmaf(kv, alg[kk], mu_part);
+                    // hi keeps the 19 bits the tensor core reads (it truncates
+                    // an fp32 operand to tf32); lo = kv - hi exactly
+                    const float hi = __uint_as_float(__float_as_uint(kv) & 0xFFFFE000u);
+                    vh[e] = hi;
+                    vl[e] = kv - hi;
+                  }
                 }
+                const int o = sw128_off(r, COLS * g + g4 * 4);
+                *(float4 *)(Ah + o) = make_float4(vh[0], vh[1], vh[2], vh[3]);
+                *(float4 *)(Al + o) = make_float4(vl[0], vl[1], vl[2], vl[3]);
               }
-              const int o = sw128_off(r, COLS * g + g4 * 4);
-              *(float4 *)(Ah + o) = make_float4(vh[0], vh[1], vh[2], vh[3]);
-              *(float4 *)(Al + o) = make_float4(vl[0], vl[1], vl[2], vl[3]);
-            }
+            };
+            if (full_chunk) emit(std::false_type{});
+            else emit(std::true_type{});
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) {
