@@ -162,15 +162,16 @@ int boute_select_topk(const float *acq, int B, long long N, int k, long long *id
  * whose allocator already holds the device's free memory, a latency-critical
  * loop that cannot take the synchronisation cudaFree implies, or a fixed
  * memory budget. The call makes no allocation of any kind.
- *   Limit: 2 * B * ceil(N / 2048) * max(k, 16) * 8 bytes of scratch (0 when
+ *   Limit: 2 * B * ceil(N / 2048) * max(k, 32) * 8 bytes of scratch (0 when
  *   N <= 2048) must not exceed BOUTE_TOPK_NOALLOC_SCRATCH_BYTES; a larger
  *   request returns BOUTE_ERR_UNSUPPORTED before launching anything. Other
  *   argument errors are those of boute_select_topk.
  *   Set-up: the first call on a device, made with that device current, looks
  *   up the array's device address (once per device, under a lock); make that
  *   first call before any stream capture begins.
- *   Nothing in the array has to start at zero: every level of the selection
- *   writes all the keys the next level reads.
+ *   The few words of the array that must start at zero (one counter per
+ *   problem) are cleared by the call itself, on `stream`, before its kernel
+ *   runs; every key is written before it is read.
  *   There is ONE array per device: calls that overlap in time on that device
  *   (on different streams, or from different threads) race on it and may
  *   return wrong results. Serialise them, e.g. by issuing them on one stream. */

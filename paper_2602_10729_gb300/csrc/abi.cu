@@ -307,6 +307,11 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
   r |= dalloc(&e->idx, (size_t)B * k);
   r |= dalloc(&e->val, (size_t)B * k);
   r |= dalloc((unsigned char **)&e->scratch, topk_scratch_bytes(B, N, k));
+  // the top-k counters in the scratch start at zero; every step leaves them zero
+  if (r == BOUTE_OK && cudaMemset(e->scratch, 0, topk_scratch_bytes(B, N, k)) != cudaSuccess) {
+    cudaGetLastError();
+    r = BOUTE_ERR_CUDA;
+  }
   if (r == BOUTE_OK &&
       (cudaStreamCreateWithFlags(&e->side, cudaStreamNonBlocking) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->fork, cudaEventDisableTiming) != cudaSuccess ||
@@ -378,7 +383,7 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
       return r;
   }
   mark(ST_TOPK);
-  if ((r = launch_topk(e->acq, B, e->N, e->k, idx, val, e->scratch, s))) return r;
+  if ((r = launch_topk(e->acq, B, e->N, e->k, idx, val, e->scratch, s, true))) return r;
   mark(ST_COUNT);
   e->launches = (int)(launch_count() - l0);
   return BOUTE_OK;

@@ -79,7 +79,10 @@ int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
                  const float *lower, const float *upper, const int *K, int box_cap,
                  const float *eps, int S, long long eps_stride, float *acq, cudaStream_t s);
 size_t topk_scratch_bytes(int B, long long N, int k);
+// counters_zeroed: the scratch's per-problem counters are known to be zero
+// (an engine's scratch: zeroed at creation, and every call leaves them zero);
+// otherwise the call clears them first.
 int launch_topk(const float *acq, int B, long long N, int k, long long *idx, float *val,
-                void *scratch, cudaStream_t s);
+                void *scratch, cudaStream_t s, bool counters_zeroed = false);
 
 }  // namespace boute

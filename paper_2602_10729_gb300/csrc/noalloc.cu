@@ -13,8 +13,9 @@ namespace boute {
 namespace {
 
 // Scratch of the levels after the first: two ping-pong arrays of 64-bit keys.
-// Nothing in it has to start at zero: each level writes every key the next
-// level reads before that level runs.
+// The only words that must start at zero (one counter per problem, on the
+// k <= 32 path) are cleared by every call before its kernel runs; every key
+// is written before it is read.
 static __device__ __align__(256) unsigned char g_topk_scratch[BOUTE_TOPK_NOALLOC_SCRATCH_BYTES];
 
 constexpr int kMaxDevices = 64;
@@ -67,7 +68,7 @@ extern "C" int boute_select_topk_noalloc(const float *acq, int B, long long N, i
   const long long nseg = (N + 2047) / 2048;  // first-level segments per problem
   const unsigned long long need =
       nseg <= 1 ? 0ull
-                : 2ull * (unsigned long long)B * nseg * (k < 16 ? 16 : k) * sizeof(unsigned long long);
+                : 2ull * (unsigned long long)B * nseg * (k < 32 ? 32 : k) * sizeof(unsigned long long);
   if (need > BOUTE_TOPK_NOALLOC_SCRATCH_BYTES) return BOUTE_ERR_UNSUPPORTED;
   if (!device_is_sm103()) return BOUTE_ERR_UNSUPPORTED;
   void *scratch = nullptr;

@@ -1,7 +1,7 @@
 // Deterministic top-k per problem. Values become 64-bit keys (order-preserving
 // float bits in the high word, the complement of the index in the low word), so
 // one unsigned comparison orders by value descending, then index ascending.
-// k <= 32 takes a warp-register path (below). Otherwise, level 1: every block sorts one segment of kSeg keys in shared memory
+// k <= 32 takes a warp-register path in one launch (below). Otherwise, level 1: every block sorts one segment of kSeg keys in shared memory
 // (bitonic) and keeps its k largest. Further levels apply the same segment
 // sort to the surviving keys until one segment per problem remains; the last
 // level writes indices and values. All levels are fully parallel across
@@ -134,21 +134,24 @@ __device__ __forceinline__ unsigned long long warp_merge_desc(unsigned long long
   return u;
 }
 
-// Block blockIdx.x of problem blockIdx.y covers entries [x * per_block,
-// (x+1) * per_block) of a row of `len` (values when FROM_VALUES, else sorted
-// runs of 32 keys). With idx set (one block per problem) it writes the final
-// k indices and values; otherwise its 32 keys to keys_out.
-template <bool FROM_VALUES>
+// Block blockIdx.x of problem blockIdx.y takes entries [x * per_block,
+// (x+1) * per_block) of the problem's N values and forms their 32 largest
+// keys. With one block per problem it writes the final k indices and values.
+// Otherwise each block stores its 32 keys in `keys` and counts itself done on
+// the problem's counter; the block that finishes last merges all the blocks'
+// lists (eight warps, then one) and writes the result, and sets the counter
+// back to zero for the next call.
 __global__ void __launch_bounds__(kWarpBlock) warp_topk_kernel(
-    const float *vals, const unsigned long long *keys_in, long long len, long long per_block,
-    unsigned long long *keys_out, const float *acq, long long N, int k, long long *idx,
-    float *val) {
+    const float *vals, long long N, long long per_block, unsigned long long *keys,
+    unsigned *counter, int k, long long *idx, float *val) {
   __shared__ unsigned long long lists[kWarpBlock / 32][kWarpK];
+  __shared__ int is_last;
   pdl_wait();
   const int b = blockIdx.y, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int G = gridDim.x;
   const long long lo = (long long)blockIdx.x * per_block;
-  const long long hi = std::min<long long>(len, lo + per_block);
-  const size_t row = (size_t)b * len;
+  const long long hi = std::min<long long>(N, lo + per_block);
+  const size_t row = (size_t)b * N;
   unsigned long long top = 0ull;  // below every real key
   for (long long base = lo + (long long)warp * 32 * kWarpBatches; base < hi;
        base += (long long)kWarpBlock * kWarpBatches) {
@@ -156,59 +159,66 @@ __global__ void __launch_bounds__(kWarpBlock) warp_topk_kernel(
 #pragma unroll
     for (int u = 0; u < kWarpBatches; ++u) {
       const long long g = base + 32 * u + lane;
-      x[u] = 0ull;
-      if (g < hi) x[u] = FROM_VALUES ? make_key(__ldcs(vals + row + g), (unsigned)g) : keys_in[row + g];
+      x[u] = g < hi ? make_key(__ldcs(vals + row + g), (unsigned)g) : 0ull;
     }
 #pragma unroll
     for (int u = 0; u < kWarpBatches; ++u) {
       const unsigned long long thr = shfl64(top, 31);
       if (__ballot_sync(0xffffffffu, x[u] > thr) == 0u) continue;
-      top = warp_merge_desc(top, FROM_VALUES ? warp_sort_desc(x[u], lane) : x[u], lane);
+      top = warp_merge_desc(top, warp_sort_desc(x[u], lane), lane);
     }
   }
   lists[warp][lane] = top;
   __syncthreads();
-  if (warp != 0) return;
+  if (warp == 0) {
 #pragma unroll 1
-  for (int w = 1; w < kWarpBlock / 32; ++w) top = warp_merge_desc(top, lists[w][lane], lane);
-  if (idx) {
-    if (lane < k) {
-      const unsigned j = key_index(top);
-      idx[(size_t)b * k + lane] = (long long)j;
-      val[(size_t)b * k + lane] = acq[(size_t)b * N + j];
+    for (int w = 1; w < kWarpBlock / 32; ++w) top = warp_merge_desc(top, lists[w][lane], lane);
+    if (G > 1) {
+      keys[((size_t)b * G + blockIdx.x) * kWarpK + lane] = top;
+      __threadfence();  // the list is visible before the block counts itself done
+      __syncwarp();
+      if (lane == 0) is_last = atomicAdd(&counter[b], 1u) == (unsigned)(G - 1);
     }
-  } else {
-    keys_out[((size_t)b * gridDim.x + blockIdx.x) * kWarpK + lane] = top;
+  }
+  if (G > 1) {
+    __syncthreads();
+    if (!is_last) return;
+    __threadfence();
+    top = 0ull;
+    for (int l = warp; l < G; l += kWarpBlock / 32)
+      top = warp_merge_desc(top, __ldcg(keys + ((size_t)b * G + l) * kWarpK + lane), lane);
+    lists[warp][lane] = top;
+    __syncthreads();
+    if (warp != 0) return;
+#pragma unroll 1
+    for (int w = 1; w < kWarpBlock / 32; ++w) top = warp_merge_desc(top, lists[w][lane], lane);
+    if (lane == 0) counter[b] = 0u;
+  } else if (warp != 0) {
+    return;
+  }
+  if (lane < k) {
+    const unsigned j = key_index(top);
+    idx[(size_t)b * k + lane] = (long long)j;
+    val[(size_t)b * k + lane] = vals[row + j];
   }
 }
 
+// scratch: B x G x 32 keys, then B counters (zero on entry, zero on exit)
 int launch_topk_warp(const float *acq, int B, long long N, int k, long long *idx, float *val,
-                     void *scratch, cudaStream_t s) {
+                     void *scratch, bool counters_zeroed, cudaStream_t s) {
   // at most 256 first-level blocks per problem, each a multiple of 2048 entries
   const long long unit = (long long)kWarpBlock * kWarpBatches;
   long long per_block = unit;
   while ((N + per_block - 1) / per_block > 256) per_block += unit;
   const long long G = (N + per_block - 1) / per_block;
-  prefer_shared(warp_topk_kernel<true>);
-  prefer_shared(warp_topk_kernel<false>);
-  const float *nf = nullptr;
-  const unsigned long long *nk = nullptr;
-  unsigned long long *nko = nullptr;
-  long long *ni = nullptr;
-  float *nv = nullptr;
-  if (G == 1) {
-    launch_pdl(warp_topk_kernel<true>, dim3(1, B), dim3(kWarpBlock), 0, s, acq, nk, N, per_block,
-               nko, acq, N, k, idx, val);
-    count_launch(1);
+  prefer_shared(warp_topk_kernel);
+  unsigned long long *keys = G > 1 ? (unsigned long long *)scratch : nullptr;
+  unsigned *counter = G > 1 ? (unsigned *)(keys + (size_t)B * G * kWarpK) : nullptr;
+  if (G > 1 && !counters_zeroed && cudaMemsetAsync(counter, 0, B * sizeof(unsigned), s) != cudaSuccess)
     return last_launch_status();
-  }
-  unsigned long long *keys = (unsigned long long *)scratch;
-  launch_pdl(warp_topk_kernel<true>, dim3((unsigned)G, B), dim3(kWarpBlock), 0, s, acq, nk, N,
-             per_block, keys, acq, N, k, ni, nv);
-  const long long len2 = G * kWarpK;
-  launch_pdl(warp_topk_kernel<false>, dim3(1, B), dim3(kWarpBlock), 0, s, nf, keys, len2, len2,
-             nko, acq, N, k, idx, val);
-  count_launch(2);
+  launch_pdl(warp_topk_kernel, dim3((unsigned)G, B), dim3(kWarpBlock), 0, s, acq, N, per_block,
+             keys, counter, k, idx, val);
+  count_launch(1);
   return last_launch_status();
 }
 
@@ -216,18 +226,20 @@ int launch_topk_warp(const float *acq, int B, long long N, int k, long long *idx
 
 // Scratch for the levels after the first: two ping-pong key arrays of
 // ceil(N / 2048) * k keys per problem (segment path), or at most
-// ceil(N / 2048) runs of 32 keys per problem (warp path, k <= 32); k is
-// counted as at least 16 so that one bound covers both.
+// ceil(N / 2048) runs of 32 keys per problem and one counter per problem
+// (warp path, k <= 32); k is counted as at least 32 so that one bound covers
+// both.
 size_t topk_scratch_bytes(int B, long long N, int k) {
   const long long g1 = (N + kSeg - 1) / kSeg;
   if (g1 <= 1) return 16;
-  return 2 * (size_t)B * g1 * std::max(k, 16) * sizeof(unsigned long long) + 16;
+  return 2 * (size_t)B * g1 * std::max(k, 32) * sizeof(unsigned long long) + 16;
 }
 
 int launch_topk(const float *acq, int B, long long N, int k, long long *idx, float *val,
-                void *scratch, cudaStream_t s) {
+                void *scratch, cudaStream_t s, bool counters_zeroed) {
   if (k > kSeg / 2) return BOUTE_ERR_UNSUPPORTED;
-  if (k <= kWarpK) return launch_topk_warp(acq, B, N, k, idx, val, scratch, s);
+  if (k <= kWarpK)
+    return launch_topk_warp(acq, B, N, k, idx, val, scratch, counters_zeroed, s);
   long long len = N;
   long long nseg = (len + kSeg - 1) / kSeg;
   unsigned long long *ping = (unsigned long long *)scratch;

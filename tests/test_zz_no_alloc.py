@@ -14,12 +14,12 @@ pytestmark = pytest.mark.gpu
 # (B, N, k): one segment, two levels, a ragged last segment, several problems,
 # the largest k, and a request that fills the array exactly
 CASES = [(1, 1000, 10), (1, 2048, 64), (2, 70_001, 64), (3, 300_000, 1024), (1, 1, 1),
-         (4, 1 << 22, 64)]
+         (4, 1 << 22, 64), (3, 700_001, 17)]
 
 
 def _scratch_bytes(B, N, k):
     nseg = -(-N // 2048)
-    return 0 if nseg <= 1 else 2 * B * nseg * max(k, 16) * 8
+    return 0 if nseg <= 1 else 2 * B * nseg * max(k, 32) * 8
 
 
 @pytest.mark.parametrize("B,N,k", CASES)
