@@ -75,6 +75,10 @@ struct boute_engine {
   float *lower, *upper, *Xc, *eps, *mean, *var, *acq, *val;
   long long *idx;
   void *scratch;
+  // 2-objective Monte-Carlo steps with k <= 32 select in the acquisition
+  // kernel: its lists of keys and counters (zero between steps)
+  unsigned char *sel;
+  bool fuse_sel;
   int launches;
   int timing;                  // record one CUDA event per stage boundary
   cudaEvent_t ev[8];           // boundaries of the stages of the last step
@@ -265,9 +269,17 @@ void boute_engine_free(boute_engine *e) {
     if (c) cudaStreamDestroy(c);
   void *ptrs[] = {e->X, e->Y, e->Ys, e->ls, e->s2, e->noise, e->ref, e->front, e->mask, e->P,
                   e->K, e->lower, e->upper, e->Xc, e->eps, e->mean, e->var, e->acq, e->val,
-                  e->idx, e->scratch};
+                  e->idx, e->scratch, e->sel};
   for (void *p : ptrs) cudaFree(p);
   delete e;
+}
+
+// The selection runs inside the acquisition kernel for 2-objective
+// Monte-Carlo steps with k <= 32 (not in stage-timing mode, which times the
+// selection as a stage of its own).
+static bool engine_fuses_selection(const boute_engine *e) {
+  return e->mode == BOUTE_ACQ_MC_HVI && e->m == 2 && e->k <= 32 &&
+         mchvi2_select_grid_x(e->B, e->N, 2 * e->n + 2) <= 32 * 32;
 }
 
 int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S, int k,
@@ -312,6 +324,15 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
     cudaGetLastError();
     r = BOUTE_ERR_CUDA;
   }
+  e->fuse_sel = engine_fuses_selection(e);
+  if (r == BOUTE_OK && e->fuse_sel) {
+    const size_t bytes = mchvi2_select_scratch_bytes(B, N, 2 * n + 2);
+    r |= dalloc(&e->sel, bytes);
+    if (r == BOUTE_OK && cudaMemset(e->sel, 0, bytes) != cudaSuccess) {
+      cudaGetLastError();
+      r = BOUTE_ERR_CUDA;
+    }
+  }
   if (r == BOUTE_OK &&
       (cudaStreamCreateWithFlags(&e->side, cudaStreamNonBlocking) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->fork, cudaEventDisableTiming) != cudaSuccess ||
@@ -341,8 +362,16 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
   int r;
   const int B = e->B, n = e->n, m = e->m;
   const int mc = e->mode == BOUTE_ACQ_MC_HVI;
+  // stage boundaries: event-record nodes when captured, plain records when eager
+  cudaStreamCaptureStatus run_cap = cudaStreamCaptureStatusNone;
+  if (e->timing && s && cudaStreamIsCapturing(s, &run_cap) != cudaSuccess)
+    return last_launch_status();
   auto mark = [&](int stage) {
-    if (e->timing) cudaEventRecordWithFlags(e->ev[stage], s, cudaEventRecordExternal);
+    if (!e->timing) return;
+    if (run_cap == cudaStreamCaptureStatusActive)
+      cudaEventRecordWithFlags(e->ev[stage], s, cudaEventRecordExternal);
+    else
+      cudaEventRecord(e->ev[stage], s);
   };
   auto front = [&](cudaStream_t fs) {
     return launch_front_fused(Y, B, n, m, ref, e->Ys, e->mask, e->front, e->P, e->lower,
@@ -375,15 +404,21 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
       if (cudaStreamWaitEvent(s, ev, wait_flags) != cudaSuccess)
         return last_launch_status();
   mark(ST_ACQ);
-  if (!mc) {
+  if (e->fuse_sel && !e->timing) {
+    if ((r = launch_mchvi2_select(e->mean, e->var, B, e->N, e->lower, e->upper, e->K, 2 * n + 2,
+                                  eps, e->S, 2ll * e->S, e->acq, e->k, e->sel, idx, val, s)))
+      return r;
+  } else if (!mc) {
     if ((r = launch_ehvi(e->mean, e->var, B, e->N, e->front, e->P, n, ref, e->acq, s))) return r;
   } else {
     if ((r = launch_mchvi(e->mean, e->var, B, e->N, m, e->lower, e->upper, e->K, 2 * n + 2, eps,
                           e->S, (long long)m * e->S, e->acq, s)))
       return r;
   }
-  mark(ST_TOPK);
-  if ((r = launch_topk(e->acq, B, e->N, e->k, idx, val, e->scratch, s, true))) return r;
+  if (!e->fuse_sel || e->timing) {
+    mark(ST_TOPK);
+    if ((r = launch_topk(e->acq, B, e->N, e->k, idx, val, e->scratch, s, true))) return r;
+  }
   mark(ST_COUNT);
   e->launches = (int)(launch_count() - l0);
   return BOUTE_OK;

@@ -5,6 +5,7 @@
 #include <algorithm>
 
 #include "internal.h"
+#include "warp_select.cuh"
 
 namespace boute {
 
@@ -170,11 +171,21 @@ __device__ __forceinline__ float rcp_fast(float x) {
   return y;
 }
 
+// SEL: also select the ksel <= 32 best candidates of each problem as they are
+// scored: every warp keeps a running top-32 of its candidates, each block
+// merges its warps' lists into sel_keys, and the last block of a problem to
+// finish (sel_cnt) merges all the blocks' lists, writes idx / val and sets
+// the counter back to zero.
+constexpr int kSelGroup = 32;  // blocks per selection group
+
+template <bool SEL>
 __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const float *var,
                                                      long long N, const float *lower,
                                                      const float *upper, const int *Kc,
                                                      int box_cap, const float *eps, int S,
-                                                     long long eps_stride, float *acq) {
+                                                     long long eps_stride, float *acq, int ksel,
+                                                     unsigned long long *sel_keys,
+                                                     long long *idx, float *val) {
   extern __shared__ float4 strips4[];  // k >= 1: (b/D, 1/D, u, D); [0]: (b_0, u_0, -, -)
   float *sb = (float *)(strips4 + box_cap);  // b_k
   float *su = sb + box_cap;                  // u_k
@@ -200,6 +211,7 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
   const bool vec = (S == 128) && ((uintptr_t)eps & 15) == 0 && (eps_stride % 4) == 0;
   const long long cstride = (long long)gridDim.x * wpb;
   const float inv_s = 1.f / (float)S;
+  unsigned long long top = 0ull;  // this warp's running top-32 (SEL)
   auto eps_of = [&](long long c) {
     return eps + ((size_t)b * N + c) * eps_stride + (eps_stride == 0 ? (size_t)b * 2 * S : 0);
   };
@@ -270,9 +282,9 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
       if (lane == 0) acq[(size_t)b * N + c] = sum * inv_s;
+      if (SEL) top = warp_insert_desc(top, make_key(sum * inv_s, (unsigned)c), lane);
     }
-    return;
-  }
+  } else {
   for (long long c = (long long)blockIdx.x * wpb + warp; c < N; c += cstride) {
     const float mu1 = m1[c], mu2 = m2[c];
     const float sg1 = sqrt_fast(fmaxf(v1[c], 0.f)), sg2 = sqrt_fast(fmaxf(v2[c], 0.f));
@@ -282,6 +294,62 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
     if (lane == 0) acq[(size_t)b * N + c] = sum * inv_s;
+    if (SEL) top = warp_insert_desc(top, make_key(sum * inv_s, (unsigned)c), lane);
+  }
+  }
+  if (!SEL) return;
+  // ---- selection. Block list (tree over the 16 warps); with several blocks
+  // per problem, blocks form groups of kSelGroup: the last block of a group to
+  // finish merges the group's lists, and the last group of the problem to
+  // finish merges the group lists. Counters are set back to zero by the block
+  // that consumed them.
+  __shared__ unsigned long long lists[16][kWarpK];
+  __shared__ int is_last;
+  const int G = gridDim.x, Bp = gridDim.y;
+  const int ng = (G + kSelGroup - 1) / kSelGroup, grp = blockIdx.x / kSelGroup;
+  const int gsize = min(kSelGroup, G - grp * kSelGroup);
+  unsigned long long *blk_keys = sel_keys;                           // Bp x G x 32
+  unsigned long long *grp_keys = blk_keys + (size_t)Bp * G * kWarpK;  // Bp x ng x 32
+  unsigned *grp_cnt = (unsigned *)(grp_keys + (size_t)Bp * ng * kWarpK);  // Bp x ng
+  unsigned *prob_cnt = grp_cnt + (size_t)Bp * ng;                         // Bp
+  // merges n <= 32 lists at src (32 keys each) with the whole block
+  auto merge_lists = [&](const unsigned long long *src, int n) {
+    const unsigned long long x0 = warp < n ? __ldcg(src + (size_t)warp * kWarpK + lane) : 0ull;
+    const unsigned long long x1 =
+        warp + 16 < n ? __ldcg(src + (size_t)(warp + 16) * kWarpK + lane) : 0ull;
+    __syncthreads();  // `lists` free again
+    return block_merge16(lists, warp_merge_desc(x0, x1, lane), warp, lane);
+  };
+  // publishes warp 0's list at dst and counts the block in on *cnt; true in
+  // every thread of the block that completes the count of `total`
+  // (the count is a release: it carries the list and, through the block's
+  // barriers, every acquisition value the block wrote)
+  auto publish = [&](unsigned long long *dst, unsigned *cnt, int total) {
+    if (warp == 0) {
+      dst[lane] = top;
+      __syncwarp();
+      if (lane == 0) is_last = atomic_add_acq_rel_gpu(cnt, 1u) == (unsigned)(total - 1);
+    }
+    __syncthreads();
+    return is_last != 0;
+  };
+  top = block_merge16(lists, top, warp, lane);
+  if (G > 1) {
+    if (!publish(blk_keys + ((size_t)b * G + blockIdx.x) * kWarpK, &grp_cnt[(size_t)b * ng + grp],
+                 gsize))
+      return;
+    top = merge_lists(blk_keys + ((size_t)b * G + (size_t)grp * kSelGroup) * kWarpK, gsize);
+    if (threadIdx.x == 0) grp_cnt[(size_t)b * ng + grp] = 0u;
+    if (ng > 1) {
+      if (!publish(grp_keys + ((size_t)b * ng + grp) * kWarpK, &prob_cnt[b], ng)) return;
+      top = merge_lists(grp_keys + (size_t)b * ng * kWarpK, ng);
+      if (threadIdx.x == 0) prob_cnt[b] = 0u;
+    }
+  }
+  if (warp == 0 && lane < ksel) {
+    const unsigned j = key_index(top);
+    idx[(size_t)b * ksel + lane] = (long long)j;
+    val[(size_t)b * ksel + lane] = __ldcg(acq + (size_t)b * N + j);
   }
 }
 
@@ -300,31 +368,94 @@ int launch_ehvi(const float *mean, const float *var, int B, long long N, const d
   return last_launch_status();
 }
 
+namespace {
+
+// Blocks per problem for a kernel of 512-thread blocks that scores one
+// candidate per warp: as many as are resident on the device at once, split
+// over the B problems, so that the grid is one wave.
+template <class Kern>
+unsigned resident_grid_x(Kern kernel, size_t smem, int B, long long N) {
+  int occ = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kernel, 512, smem) != cudaSuccess) {
+    cudaGetLastError();
+    occ = 1;
+  }
+  const long long want = (N + 15) / 16;
+  const long long fit = (long long)num_sms() * std::max(occ, 1) / std::max(1, B);
+  return (unsigned)std::max<long long>(1, std::min(want, fit));
+}
+
+size_t mchvi2_smem(int box_cap) { return 6 * (size_t)box_cap * sizeof(float); }
+
+void mchvi2_configure(bool sel, int box_cap) {
+  const size_t smem = mchvi2_smem(box_cap);
+  if (sel) {
+    prefer_shared(mchvi2_kernel<true>);
+    if (smem > 48 * 1024)
+      cudaFuncSetAttribute(mchvi2_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem);
+  } else {
+    prefer_shared(mchvi2_kernel<false>);
+    if (smem > 48 * 1024)
+      cudaFuncSetAttribute(mchvi2_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem);
+  }
+}
+
+}  // namespace
+
+unsigned mchvi2_select_grid_x(int B, long long N, int box_cap) {
+  mchvi2_configure(true, box_cap);
+  return resident_grid_x(mchvi2_kernel<true>, mchvi2_smem(box_cap), B, N);
+}
+
+// Bytes of the selection scratch of launch_mchvi2_select: per problem, one
+// list of 32 keys per block and per group of kSelGroup blocks, then one
+// counter per group and per problem (zero on entry, zero on exit).
+size_t mchvi2_select_scratch_bytes(int B, long long N, int box_cap) {
+  const size_t G = mchvi2_select_grid_x(B, N, box_cap), ng = (G + kSelGroup - 1) / kSelGroup;
+  return (size_t)B * (G + ng) * kWarpK * sizeof(unsigned long long) +
+         (size_t)B * (ng + 1) * sizeof(unsigned);
+}
+
+// 2-objective Monte-Carlo HVI with the k <= 32 best candidates selected in the
+// same launch; sel: mchvi2_select_scratch_bytes(B, N, box_cap) bytes whose
+// counters are zero (they are zero again when the kernel ends).
+int launch_mchvi2_select(const float *mean, const float *var, int B, long long N,
+                         const float *lower, const float *upper, const int *K, int box_cap,
+                         const float *eps, int S, long long eps_stride, float *acq, int k,
+                         void *sel, long long *idx, float *val, cudaStream_t s) {
+  if (N <= 0 || k < 1 || k > kWarpK || k > N) return BOUTE_ERR_INVALID_ARG;
+  const unsigned gx = mchvi2_select_grid_x(B, N, box_cap);
+  if (gx > (unsigned)(kSelGroup * kSelGroup)) return BOUTE_ERR_UNSUPPORTED;
+  launch_pdl(mchvi2_kernel<true>, dim3(gx, B), dim3(16 * 32), mchvi2_smem(box_cap), s, mean, var,
+             N, lower, upper, K, box_cap, eps, S, eps_stride, acq, k,
+             (unsigned long long *)sel, idx, val);
+  count_launch();
+  return last_launch_status();
+}
+
 int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
                  const float *lower, const float *upper, const int *K, int box_cap,
                  const float *eps, int S, long long eps_stride, float *acq, cudaStream_t s) {
   if (N <= 0) return BOUTE_OK;
-  int sms = 152;
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
-  const int wpb = 16;
-  const long long want = (N + wpb - 1) / wpb;
-  const unsigned gx =
-      (unsigned)std::max<long long>(1, std::min<long long>(want, (long long)sms * 4 / std::max(1, B) + 1));
-  const size_t smem = 2 * (size_t)box_cap * m * sizeof(float);
-  if (smem > 48 * 1024) {
-    cudaFuncSetAttribute(mchvi_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    cudaFuncSetAttribute(mchvi_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  }
   if (m == 2) {
-    const size_t smem2 = 6 * (size_t)box_cap * sizeof(float);
-    prefer_shared(mchvi2_kernel);
-    if (smem2 > 48 * 1024)
-      cudaFuncSetAttribute(mchvi2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
-    launch_pdl(mchvi2_kernel, dim3(gx, B), dim3(wpb * 32), smem2, s, mean, var, N, lower, upper, K,
-               box_cap, eps, S, eps_stride, acq);
+    mchvi2_configure(false, box_cap);
+    const size_t smem2 = mchvi2_smem(box_cap);
+    const unsigned gx = resident_grid_x(mchvi2_kernel<false>, smem2, B, N);
+    unsigned long long *nk = nullptr;
+    long long *ni = nullptr;
+    float *nv = nullptr;
+    launch_pdl(mchvi2_kernel<false>, dim3(gx, B), dim3(16 * 32), smem2, s, mean, var, N, lower,
+               upper, K, box_cap, eps, S, eps_stride, acq, 0, nk, ni, nv);
   } else if (m == 3) {
-    launch_pdl(mchvi_kernel<3>, dim3(gx, B), dim3(wpb * 32), smem, s, mean, var, B, N, lower, upper,
-               K, box_cap, eps, S, eps_stride, acq);
+    const size_t smem = 2 * (size_t)box_cap * m * sizeof(float);
+    if (smem > 48 * 1024)
+      cudaFuncSetAttribute(mchvi_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem);
+    const unsigned gx = resident_grid_x(mchvi_kernel<3>, smem, B, N);
+    launch_pdl(mchvi_kernel<3>, dim3(gx, B), dim3(16 * 32), smem, s, mean, var, B, N, lower,
+               upper, K, box_cap, eps, S, eps_stride, acq);
   } else {
     return BOUTE_ERR_UNSUPPORTED;
   }

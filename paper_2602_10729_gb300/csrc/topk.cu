@@ -11,6 +11,7 @@
 #include <algorithm>
 
 #include "internal.h"
+#include "warp_select.cuh"
 
 namespace boute {
 
@@ -18,18 +19,6 @@ namespace {
 
 constexpr int kThreads = 512;
 constexpr int kSeg = 2048;  // keys per segment (16 KB of shared memory)
-
-__device__ __forceinline__ unsigned long long make_key(float v, unsigned idx) {
-  if (isnan(v)) v = -INFINITY;
-  if (v == 0.f) v = 0.f;  // -0 sorts as +0
-  unsigned u = __float_as_uint(v);
-  u = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-  return ((unsigned long long)u << 32) | (unsigned long long)(0xFFFFFFFFu - idx);
-}
-
-__device__ __forceinline__ unsigned key_index(unsigned long long key) {
-  return 0xFFFFFFFFu - (unsigned)(key & 0xFFFFFFFFull);
-}
 
 // Sort buf[0, L) descending, L a power of two.
 __device__ void bitonic_desc(unsigned long long *buf, int L) {
@@ -93,46 +82,8 @@ __global__ void __launch_bounds__(kThreads) segment_topk_kernel(
 // element-wise maximum of the running list and the reversed batch is a bitonic
 // sequence holding the 32 largest keys of both, which five more shuffle steps
 // sort. Each block merges its warps' lists; a second launch merges the blocks'.
-constexpr int kWarpK = 32;
 constexpr int kWarpBlock = 256;  // threads; 8 warps
 constexpr int kWarpBatches = 8;  // batches of 32 keys a warp loads at once
-
-__device__ __forceinline__ unsigned long long shfl64(unsigned long long v, int src) {
-  return __shfl_sync(0xffffffffu, v, src);
-}
-__device__ __forceinline__ unsigned long long shfl_xor64(unsigned long long v, int m) {
-  return __shfl_xor_sync(0xffffffffu, v, m);
-}
-
-// Sort one key per lane, descending across the lanes.
-__device__ __forceinline__ unsigned long long warp_sort_desc(unsigned long long x, int lane) {
-#pragma unroll
-  for (int size = 2; size <= 32; size <<= 1) {
-#pragma unroll
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      const unsigned long long y = shfl_xor64(x, stride);
-      const bool desc = (lane & size) == 0 || size == 32;
-      const bool lower = (lane & stride) == 0;
-      const unsigned long long mx = x > y ? x : y, mn = x > y ? y : x;
-      x = (lower == desc) ? mx : mn;
-    }
-  }
-  return x;
-}
-
-// top, s: descending across the lanes. Returns the 32 largest of both, descending.
-__device__ __forceinline__ unsigned long long warp_merge_desc(unsigned long long top,
-                                                              unsigned long long s, int lane) {
-  const unsigned long long r = shfl64(s, 31 - lane);
-  unsigned long long u = top > r ? top : r;
-#pragma unroll
-  for (int stride = 16; stride > 0; stride >>= 1) {
-    const unsigned long long y = shfl_xor64(u, stride);
-    const bool lower = (lane & stride) == 0;
-    u = lower ? (u > y ? u : y) : (u > y ? y : u);
-  }
-  return u;
-}
 
 // Block blockIdx.x of problem blockIdx.y takes entries [x * per_block,
 // (x+1) * per_block) of the problem's N values and forms their 32 largest

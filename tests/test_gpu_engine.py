@@ -5,6 +5,8 @@ stage-timing mode must all give the same selection, value for value, and the
 same per-candidate scores as the step-by-step calls checked against the
 oracle elsewhere. Consecutive host-input steps with different inputs catch
 reuse of the engine's input buffers before the previous step is done."""
+import dataclasses
+
 import numpy as np
 import pytest
 
@@ -112,3 +114,37 @@ def test_consecutive_host_steps_with_new_inputs():
     for (gi, gv), (wi_, wv) in zip(got, want + want[:1]):
         assert np.array_equal(gi, wi_)
         assert np.array_equal(gv, wv)
+
+
+# 2-objective Monte-Carlo steps with k <= 32 select inside the acquisition
+# kernel; the stage-timing mode runs the separate selection launch instead.
+# (B, N, S, k): the vectorised S = 128 path with many blocks per problem,
+# the general S path, several problems, k = 1 and a ragged N.
+FUSED = [(1, 65536 + 3, 128, 32), (3, 20000 + 11, 100, 17), (2, 5000, 128, 1), (1, 97, 33, 32)]
+
+
+@pytest.mark.parametrize("B,N,S,k", FUSED)
+def test_selection_in_acquisition_kernel_matches_separate_selection(B, N, S, k):
+    import torch
+
+    from paper_2602_10729_gb300 import boute as bt
+    base = wl.WORKLOADS[1]
+    w = dataclasses.replace(wl.scaled(base, N=N, n=64, S=S), B=B, k=k,
+                            seeds=tuple(range(1, B + 1)))
+    hp = host_problem(w)
+    e = _engine(w)
+    got = [_run(e, w, _dev(hp), "device") for _ in range(3)]  # counters reset each step
+    bt.boute_engine_set_timing(e, True)
+    want = _run(e, w, _dev(hp), "device")  # eager on the legacy stream: plain event records
+    assert all(v > 0 for v in bt.boute_engine_stage_times(e).values())
+    acq = torch.empty((w.B, w.N), dtype=torch.float32, device="cuda")
+    bt.boute_engine_scores(e, acq=acq)
+    torch.cuda.synchronize()
+    e.free()
+    A = acq.cpu().numpy()
+    for gi, gv in got:
+        assert np.array_equal(gi, want[0])
+        assert np.array_equal(gv, want[1])
+    for b in range(w.B):  # values descending, ties by index
+        order = np.lexsort((np.arange(w.N), -A[b]))[:k]
+        assert want[0][b].tolist() == order.tolist()
