@@ -355,35 +355,37 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
 
 }  // namespace
 
+namespace {
+
+// Blocks per problem for a grid-stride kernel whose blocks of `threads`
+// threads score `per_block` candidates per pass: as many as are resident on
+// the device at once, split over the B problems, so that the grid is one wave.
+template <class Kern>
+unsigned resident_grid_x(Kern kernel, int threads, size_t smem, int B, long long N,
+                         int per_block) {
+  int occ = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kernel, threads, smem) != cudaSuccess) {
+    cudaGetLastError();
+    occ = 1;
+  }
+  const long long want = (N + per_block - 1) / per_block;
+  const long long fit = (long long)num_sms() * std::max(occ, 1) / std::max(1, B);
+  return (unsigned)std::max<long long>(1, std::min(want, fit));
+}
+
+}  // namespace
+
 int launch_ehvi(const float *mean, const float *var, int B, long long N, const double *front,
                 const int *P, int n, const double *ref, float *acq, cudaStream_t s) {
   if (N <= 0) return BOUTE_OK;
-  int sms = 152;
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
-  const long long want = (N + 255) / 256;
-  const unsigned gx = (unsigned)std::max<long long>(1, std::min<long long>(want, (long long)sms * 8 / std::max(1, B) + 1));
-  launch_pdl(ehvi2d_kernel, dim3(gx, B), dim3(256), 2 * (n + 1) * sizeof(float), s, mean, var, N,
-             front, P, n, ref, acq);
+  const size_t smem = 2 * (size_t)(n + 1) * sizeof(float);
+  const unsigned gx = resident_grid_x(ehvi2d_kernel, 256, smem, B, N, 256);
+  launch_pdl(ehvi2d_kernel, dim3(gx, B), dim3(256), smem, s, mean, var, N, front, P, n, ref, acq);
   count_launch();
   return last_launch_status();
 }
 
 namespace {
-
-// Blocks per problem for a kernel of 512-thread blocks that scores one
-// candidate per warp: as many as are resident on the device at once, split
-// over the B problems, so that the grid is one wave.
-template <class Kern>
-unsigned resident_grid_x(Kern kernel, size_t smem, int B, long long N) {
-  int occ = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kernel, 512, smem) != cudaSuccess) {
-    cudaGetLastError();
-    occ = 1;
-  }
-  const long long want = (N + 15) / 16;
-  const long long fit = (long long)num_sms() * std::max(occ, 1) / std::max(1, B);
-  return (unsigned)std::max<long long>(1, std::min(want, fit));
-}
 
 size_t mchvi2_smem(int box_cap) { return 6 * (size_t)box_cap * sizeof(float); }
 
@@ -406,7 +408,7 @@ void mchvi2_configure(bool sel, int box_cap) {
 
 unsigned mchvi2_select_grid_x(int B, long long N, int box_cap) {
   mchvi2_configure(true, box_cap);
-  return resident_grid_x(mchvi2_kernel<true>, mchvi2_smem(box_cap), B, N);
+  return resident_grid_x(mchvi2_kernel<true>, 512, mchvi2_smem(box_cap), B, N, 16);
 }
 
 // Bytes of the selection scratch of launch_mchvi2_select: per problem, one
@@ -442,7 +444,7 @@ int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
   if (m == 2) {
     mchvi2_configure(false, box_cap);
     const size_t smem2 = mchvi2_smem(box_cap);
-    const unsigned gx = resident_grid_x(mchvi2_kernel<false>, smem2, B, N);
+    const unsigned gx = resident_grid_x(mchvi2_kernel<false>, 512, smem2, B, N, 16);
     unsigned long long *nk = nullptr;
     long long *ni = nullptr;
     float *nv = nullptr;
@@ -453,7 +455,7 @@ int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
     if (smem > 48 * 1024)
       cudaFuncSetAttribute(mchvi_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            (int)smem);
-    const unsigned gx = resident_grid_x(mchvi_kernel<3>, smem, B, N);
+    const unsigned gx = resident_grid_x(mchvi_kernel<3>, 512, smem, B, N, 16);
     launch_pdl(mchvi_kernel<3>, dim3(gx, B), dim3(16 * 32), smem, s, mean, var, B, N, lower,
                upper, K, box_cap, eps, S, eps_stride, acq);
   } else {
