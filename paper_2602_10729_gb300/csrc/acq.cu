@@ -179,25 +179,28 @@ __device__ __forceinline__ float rcp_fast(float x) {
 constexpr int kSelGroup = 32;  // blocks per selection group
 
 template <bool SEL>
-__global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const float *var,
+__global__ void __launch_bounds__(512, 2) mchvi2_kernel(const float *mean, const float *var,
                                                      long long N, const float *lower,
                                                      const float *upper, const int *Kc,
                                                      int box_cap, const float *eps, int S,
                                                      long long eps_stride, float *acq, int ksel,
                                                      unsigned long long *sel_keys,
                                                      long long *idx, float *val) {
-  extern __shared__ float4 strips4[];  // k >= 1: (b/D, 1/D, u, D); [0]: (b_0, u_0, -, -)
-  float *sb = (float *)(strips4 + box_cap);  // b_k
-  float *su = sb + box_cap;                  // u_k
+  // k >= 1: (b/D, 1/D, u, D); [0]: (b_0, u_0, -, -); then zero strips up to
+  // 1 + a multiple of 4 (they add exactly nothing), box_cap + 4 in all
+  extern __shared__ float4 strips4[];
   pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
   const int b = blockIdx.y;
   const int K = Kc[b];
-  for (int i = threadIdx.x; i < K; i += blockDim.x) {
+  const int Kp = K > 0 ? 1 + ((K + 2) & ~3) : 0;
+  for (int i = threadIdx.x; i < Kp; i += blockDim.x) {
+    if (i >= K) {
+      strips4[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      continue;
+    }
     const size_t o = ((size_t)b * box_cap + i) * 2;
     const float ai = lower[o], bi = upper[o], ui = upper[o + 1];
-    sb[i] = bi;
-    su[i] = ui;
     if (i == 0) {
       strips4[0] = make_float4(bi, ui, 0.f, 0.f);
     } else {
@@ -232,27 +235,31 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
   if (vec) {
     // S = 128: one float4 per lane per objective; the next candidate's
     // samples and posterior are loaded before this one is scored
-    long long c = (long long)blockIdx.x * wpb + warp;
+    // (B N < 2^31: candidate indices in 32 bits; the samples' pointer advances
+    // by a fixed step; the last prefetch repeats the current candidate)
+    const int Ni = (int)N, cs = (int)cstride;
+    int c = blockIdx.x * wpb + warp;
+    const size_t estep = (size_t)cs * eps_stride;
+    const float *ep = eps_of(c < Ni ? c : 0) + 4 * lane;
     float4 z1 = make_float4(0.f, 0.f, 0.f, 0.f), z2 = z1;
     float pm1 = 0.f, pm2 = 0.f, pv1 = 0.f, pv2 = 0.f;
-    if (c < N) {
-      const float *e = eps_of(c);
-      z1 = __ldcs((const float4 *)(e + 4 * lane));
-      z2 = __ldcs((const float4 *)(e + S + 4 * lane));
+    if (c < Ni) {
+      z1 = __ldcs((const float4 *)ep);
+      z2 = __ldcs((const float4 *)(ep + S));
       pm1 = m1[c]; pm2 = m2[c]; pv1 = v1[c]; pv2 = v2[c];
     }
-    const float u0 = K > 0 ? su[0] : 0.f;
-    for (; c < N; c += cstride) {
+    const float4 t0 = K > 0 ? strips4[0] : make_float4(0.f, 0.f, 0.f, 0.f);
+    const float u0 = t0.y;
+    for (; c < Ni; c += cs) {
       const float4 c1 = z1, c2 = z2;
       const float mu1 = pm1, mu2 = pm2;
       const float sg1 = sqrt_fast(fmaxf(pv1, 0.f)), sg2 = sqrt_fast(fmaxf(pv2, 0.f));
-      const long long cn = c + cstride;
-      if (cn < N) {
-        const float *e = eps_of(cn);
-        z1 = __ldcs((const float4 *)(e + 4 * lane));
-        z2 = __ldcs((const float4 *)(e + S + 4 * lane));
-        pm1 = m1[cn]; pm2 = m2[cn]; pv1 = v1[cn]; pv2 = v2[cn];
-      }
+      const bool more = c + cs < Ni;
+      const int cn = more ? c + cs : c;
+      ep = more ? ep + estep : ep;
+      z1 = __ldcs((const float4 *)ep);
+      z2 = __ldcs((const float4 *)(ep + S));
+      pm1 = m1[cn]; pm2 = m2[cn]; pv1 = v1[cn]; pv2 = v2[cn];
       const float y1[4] = {fmaf(sg1, c1.x, mu1), fmaf(sg1, c1.y, mu1), fmaf(sg1, c1.z, mu1),
                            fmaf(sg1, c1.w, mu1)};
       const float y2[4] = {fmaf(sg2, c2.x, mu2), fmaf(sg2, c2.y, mu2), fmaf(sg2, c2.z, mu2),
@@ -262,20 +269,22 @@ __global__ void __launch_bounds__(512) mchvi2_kernel(const float *mean, const fl
       const float H = u0 - lo2;
       float sum = 0.f;
       if (K > 0) {
-        const float4 t0 = strips4[0];
 #pragma unroll
         for (int j = 0; j < 4; ++j) sum += fmaxf(t0.x - y1[j], 0.f) * fmaxf(t0.y - y2[j], 0.f);
         const float iH = H > 0.f ? rcp_fast(H) : 0.f;  // H <= 0: every sample dominated
         float acc = 0.f;
-#pragma unroll 2
-        for (int k = 1; k < K; ++k) {
-          const float4 t = strips4[k];
-          const float uh = t.z * iH;
-          float tk = 0.f;
+#pragma unroll 1
+        for (int k = 1; k < Kp; k += 4) {
 #pragma unroll
-          for (int j = 0; j < 4; ++j)
-            tk = fmaf(fma_sat(-y1[j], t.y, t.x), fma_sat(-y2[j], iH, uh), tk);
-          acc = fmaf(t.w, tk, acc);
+          for (int q = 0; q < 4; ++q) {
+            const float4 t = strips4[k + q];
+            const float uh = t.z * iH;
+            float tk = 0.f;
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              tk = fmaf(fma_sat(-y1[j], t.y, t.x), fma_sat(-y2[j], iH, uh), tk);
+            acc = fmaf(t.w, tk, acc);
+          }
         }
         sum = fmaf(fmaxf(H, 0.f), acc, sum);
       }
@@ -387,7 +396,7 @@ int launch_ehvi(const float *mean, const float *var, int B, long long N, const d
 
 namespace {
 
-size_t mchvi2_smem(int box_cap) { return 6 * (size_t)box_cap * sizeof(float); }
+size_t mchvi2_smem(int box_cap) { return ((size_t)box_cap + 4) * sizeof(float4); }
 
 void mchvi2_configure(bool sel, int box_cap) {
   const size_t smem = mchvi2_smem(box_cap);

@@ -10,6 +10,8 @@
 
 #include <algorithm>
 
+#include <type_traits>
+
 #include "internal.h"
 
 namespace boute {
@@ -323,43 +325,63 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
       for (int c = 0; c < 32; ++c) a[c] = (c <= lane) ? Ar[c] : 0.f;
       const float dgl = dg[p0 + lane];
       bool ok = true;
+      // steps c0 .. c0 + 7; after step c only a[0 .. 30 - c] still lie in the
+      // block, so each quarter of the panel shifts and updates NK entries
+      // (the rest are right of the block: never stored, left as they are)
+      // The pivot of step c + 1 is lane c + 1's entry after step c, which
+      // needs only that lane's own l: it is formed and broadcast before the
+      // stores and the row update, whose issue then hides its latency.
+      float piv = __shfl_sync(FULL, a[0], 0);
+      auto quarter = [&](auto nk, int c0) {
+        constexpr int NK = decltype(nk)::value;
 #pragma unroll 1
-      for (int c = 0; c < 32; ++c) {
-        const float piv = __shfl_sync(FULL, a[0], c);
-        if (!(piv > 16.f * 1.1920929e-7f * __shfl_sync(FULL, dgl, c))) ok = false;
-        float inv = rsqrtf(piv);
-        inv = inv * fmaf(-0.5f * piv * inv, inv, 1.5f);  // one Newton step; 1 / L_cc
-        const float l = lane > c ? a[0] * inv : (lane == c ? piv * inv : 0.f);
-        if (lane >= c) Ar[c] = l;
-        colL[c][lane] = l;  // colL[c][32..63] stay zero
-        if (lane == 0) invs[c] = inv;
-        __syncwarp();
-        named_barrier_sync(1, 64);  // column c is ready for warp 1
-        // trailing update of the lane's row, shifted one column: entries right
-        // of the block or above the lane's diagonal collect values never stored
+        for (int c = c0; c < c0 + 8; ++c) {
+          if (!(piv > 16.f * 1.1920929e-7f * __shfl_sync(FULL, dgl, c))) ok = false;
+          float inv = rsqrtf(piv);
+          inv = inv * fmaf(-0.5f * piv * inv, inv, 1.5f);  // one Newton step; 1 / L_cc
+          const float l = lane > c ? a[0] * inv : (lane == c ? piv * inv : 0.f);
+          piv = __shfl_sync(FULL, fmaf(-l, l, a[1]), (c + 1) & 31);  // (unused after c = 31)
+          if (lane >= c) Ar[c] = l;
+          colL[c][lane] = l;  // colL[c][32..63] stay zero
+          if (lane == 0) invs[c] = inv;
+          __syncwarp();
+          named_barrier_sync(1, 64);  // column c is ready for warp 1
+          // trailing update of the lane's row, shifted one column: entries
+          // above the lane's diagonal collect values never stored
 #pragma unroll
-        for (int k = 0; k < 31; ++k) a[k] = fmaf(-l, colL[c][c + 1 + k], a[k + 1]);
-        a[31] = 0.f;
-      }
+          for (int k = 0; k < NK; ++k) a[k] = fmaf(-l, colL[c][c + 1 + k], a[k + 1]);
+        }
+      };
+      quarter(std::integral_constant<int, 31>{}, 0);
+      quarter(std::integral_constant<int, 23>{}, 8);
+      quarter(std::integral_constant<int, 15>{}, 16);
+      quarter(std::integral_constant<int, 7>{}, 24);
       if (!ok && lane == 0) bad = 1;
     } else if (warp == 1) {
       // Inverse, one column behind the factor. w[] is the lane's row of
       // R = e_lane - sum_{j<c} L_lane,j W_j, which becomes W_pp's row after
       // the division by L_lane,lane. R_c has no entries right of c, so the
-      // full-width update below is exact.
+      // update at step c touches w[0 .. c] only (NK per quarter of the panel).
       float w[32];
 #pragma unroll
       for (int c = 0; c < 32; ++c) w[c] = (c == lane) ? 1.f : 0.f;
       float myinv = 0.f;
+      auto quarter = [&](auto nk, int c0) {
+        constexpr int NK = decltype(nk)::value;
 #pragma unroll 1
-      for (int c = 0; c < 32; ++c) {
-        named_barrier_sync(1, 64);  // wait for column c
-        const float l = colL[c][lane], inv = invs[c];
-        if (lane == c) myinv = inv;
-        const float lw = lane > c ? l * inv : 0.f;  // R_i -= (L_ic / L_cc) R_c, rows below c
+        for (int c = c0; c < c0 + 8; ++c) {
+          named_barrier_sync(1, 64);  // wait for column c
+          const float l = colL[c][lane], inv = invs[c];
+          if (lane == c) myinv = inv;
+          const float lw = lane > c ? l * inv : 0.f;  // R_i -= (L_ic / L_cc) R_c, rows below c
 #pragma unroll
-        for (int k = 0; k < 32; ++k) w[k] = fmaf(-lw, __shfl_sync(FULL, w[k], c), w[k]);
-      }
+          for (int k = 0; k < NK; ++k) w[k] = fmaf(-lw, __shfl_sync(FULL, w[k], c), w[k]);
+        }
+      };
+      quarter(std::integral_constant<int, 8>{}, 0);
+      quarter(std::integral_constant<int, 16>{}, 8);
+      quarter(std::integral_constant<int, 24>{}, 16);
+      quarter(std::integral_constant<int, 32>{}, 24);
       float *Wr = W + (size_t)(p0 + lane) * ld + p0;
 #pragma unroll
       for (int c = 0; c < 32; ++c) Wr[c] = w[c] * myinv;
