@@ -79,6 +79,12 @@ struct boute_engine {
   // kernel: its lists of keys and counters (zero between steps)
   unsigned char *sel;
   bool fuse_sel;
+  // K* of the candidates, computed on a second side stream while the fit
+  // runs (it needs the fit's set-up, not its results); the posterior then
+  // only contracts it. Null when it would take more than kKstarMaxBytes.
+  float *kst;
+  cudaStream_t side2;
+  cudaEvent_t ev_setup, join2;
   int launches;
   int timing;                  // record one CUDA event per stage boundary
   cudaEvent_t ev[8];           // boundaries of the stages of the last step
@@ -263,16 +269,21 @@ void boute_engine_free(boute_engine *e) {
   if (e->fork) cudaEventDestroy(e->fork);
   if (e->join) cudaEventDestroy(e->join);
   if (e->side) cudaStreamDestroy(e->side);
-  for (cudaEvent_t ev : {e->ev_in, e->ev_xc, e->ev_eps[0], e->ev_eps[1]})
+  for (cudaEvent_t ev : {e->ev_in, e->ev_xc, e->ev_eps[0], e->ev_eps[1], e->ev_setup, e->join2})
     if (ev) cudaEventDestroy(ev);
+  if (e->side2) cudaStreamDestroy(e->side2);
   for (cudaStream_t c : e->cpy)
     if (c) cudaStreamDestroy(c);
   void *ptrs[] = {e->X, e->Y, e->Ys, e->ls, e->s2, e->noise, e->ref, e->front, e->mask, e->P,
                   e->K, e->lower, e->upper, e->Xc, e->eps, e->mean, e->var, e->acq, e->val,
-                  e->idx, e->scratch, e->sel};
+                  e->idx, e->scratch, e->sel, e->kst};
   for (void *p : ptrs) cudaFree(p);
   delete e;
 }
+
+// Largest K* buffer an engine keeps (it lets the posterior's K* be computed
+// beside the fit); larger workloads build K* inside the posterior.
+constexpr size_t kKstarMaxBytes = size_t(512) << 20;
 
 // The selection runs inside the acquisition kernel for 2-objective
 // Monte-Carlo steps with k <= 32 (not in stage-timing mode, which times the
@@ -333,8 +344,13 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
       r = BOUTE_ERR_CUDA;
     }
   }
+  if (r == BOUTE_OK && kstar_floats(&e->gp->g, N) * sizeof(float) <= kKstarMaxBytes)
+    r |= dalloc(&e->kst, kstar_floats(&e->gp->g, N));
   if (r == BOUTE_OK &&
       (cudaStreamCreateWithFlags(&e->side, cudaStreamNonBlocking) != cudaSuccess ||
+       cudaStreamCreateWithFlags(&e->side2, cudaStreamNonBlocking) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->ev_setup, cudaEventDisableTiming) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->join2, cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->fork, cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->join, cudaEventDisableTiming) != cudaSuccess ||
        cudaStreamCreateWithFlags(&e->cpy[0], cudaStreamNonBlocking) != cudaSuccess ||
@@ -385,18 +401,29 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
     if ((r = front(e->side))) return r;
     if (cudaEventRecord(e->join, e->side) != cudaSuccess) return last_launch_status();
   }
-  if ((r = launch_fit_raw(&e->gp->g, X, Y, ls, s2, noise, s))) return r;
-  mark(ST_FRONT);
-  if (e->timing && (r = front(s))) return r;
   // waits on the host-input copies: an external-event node when captured
   cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
   if (host && cudaStreamIsCapturing(s, &cap) != cudaSuccess) return last_launch_status();
   const unsigned wait_flags =
       cap == cudaStreamCaptureStatusActive ? cudaEventWaitExternal : cudaEventWaitDefault;
+  // K* beside the fit (not in stage-timing mode, where the posterior builds it)
+  const float *kst = e->timing ? nullptr : e->kst;
+  if ((r = launch_fit_raw(&e->gp->g, X, Y, ls, s2, noise, s, kst ? e->ev_setup : nullptr)))
+    return r;
+  if (kst) {
+    if (cudaStreamWaitEvent(e->side2, e->ev_setup, 0) != cudaSuccess ||
+        (host && cudaStreamWaitEvent(e->side2, e->ev_xc, wait_flags) != cudaSuccess))
+      return last_launch_status();
+    if ((r = launch_kstar(&e->gp->g, Xc, e->N, e->kst, e->side2))) return r;
+    if (cudaEventRecord(e->join2, e->side2) != cudaSuccess) return last_launch_status();
+  }
+  mark(ST_FRONT);
+  if (e->timing && (r = front(s))) return r;
   mark(ST_POSTERIOR);
   if (host && cudaStreamWaitEvent(s, e->ev_xc, wait_flags) != cudaSuccess)
     return last_launch_status();
-  if ((r = launch_posterior(&e->gp->g, Xc, e->N, e->mean, e->var, s))) return r;
+  if (kst && cudaStreamWaitEvent(s, e->join2, 0) != cudaSuccess) return last_launch_status();
+  if ((r = launch_posterior(&e->gp->g, Xc, e->N, e->mean, e->var, s, kst))) return r;
   if (!e->timing && cudaStreamWaitEvent(s, e->join, 0) != cudaSuccess)  // join
     return last_launch_status();
   if (host && mc)

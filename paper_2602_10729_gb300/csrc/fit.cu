@@ -665,7 +665,7 @@ size_t fit_smem_bytes(int np, int n) {
 // Ys: standardised outcomes, or raw outcomes when standardize != 0.
 static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standardize,
                            const double *ls, const double *s2, const double *noise,
-                           cudaStream_t s) {
+                           cudaStream_t s, cudaEvent_t setup_done = nullptr) {
   const int n = gp->n, d = gp->d, m = gp->m, BM = gp->B * gp->m;
   const int npad = gp->plan.npad;
   const int tn = (n + 15) / 16, nkt = tn * tn;
@@ -681,6 +681,7 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
   fit_setup_kernel<<<dim3(nkt + nprep, BM), 256, 0, s>>>(X, n, d, m, gp->DP, npad, ls, s2, noise,
                                                          gp->Kh, gp->Kl, gp->xt, gp->s2f, nkt,
                                                          nprep, setup_early, gp->status);
+  if (setup_done && cudaEventRecord(setup_done, s) != cudaSuccess) return last_launch_status();
   if (fit_uses_smem(npad)) {
     const size_t smem = fit_smem_bytes(npad, n);
     prefer_shared(fit32_kernel<true>);
@@ -708,8 +709,8 @@ int launch_fit(Gp *gp, const double *X, const double *Ys, const double *ls, cons
 }
 
 int launch_fit_raw(Gp *gp, const double *X, const double *Y, const double *ls, const double *s2,
-                   const double *noise, cudaStream_t s) {
-  return launch_fit_impl(gp, X, Y, 1, ls, s2, noise, s);
+                   const double *noise, cudaStream_t s, cudaEvent_t setup_done) {
+  return launch_fit_impl(gp, X, Y, 1, ls, s2, noise, s, setup_done);
 }
 
 }  // namespace boute

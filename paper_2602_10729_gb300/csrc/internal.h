@@ -61,16 +61,24 @@ int last_launch_status();  // BOUTE_OK or BOUTE_ERR_CUDA after a launch
 int launch_standardize(const double *Y, int B, int n, int m, double *Ys, cudaStream_t s);
 int launch_fit(Gp *gp, const double *X, const double *Ys, const double *ls, const double *s2,
                const double *noise, cudaStream_t s);
+// kst: K* precomputed by launch_kstar (the posterior then builds no K*), or null.
 int launch_posterior(const Gp *gp, const float *Xc, long long N, float *mean, float *var,
-                     cudaStream_t s);
+                     cudaStream_t s, const float *kst = nullptr);
+// K* of all candidates, per (128-candidate tile, objective) and 32-point chunk
+// as 128 x 32 fp32: kstar_floats(gp, N) floats. Reads the fit set-up's side
+// input (not the fit's results) and the candidates.
+size_t kstar_floats(const Gp *gp, long long N);
+int launch_kstar(const Gp *gp, const float *Xc, long long N, float *kst, cudaStream_t s);
 int launch_pareto(const double *Ys, int B, int n, int m, const double *ref, unsigned char *mask,
                   double *front, int *P, cudaStream_t s);
 size_t front_smem_bytes(int n, int m);
 int launch_front_fused(const double *Y, int B, int n, int m, const double *ref, double *Ys,
                        unsigned char *mask, double *front, int *P, float *lower, float *upper,
                        int *K, int want_boxes, cudaStream_t s);
+// setup_done (optional) is recorded on s after the set-up kernel, before the fit.
 int launch_fit_raw(Gp *gp, const double *X, const double *Y, const double *ls, const double *s2,
-                   const double *noise, cudaStream_t s);
+                   const double *noise, cudaStream_t s,
+                   cudaEvent_t setup_done = nullptr);
 int launch_boxes(const double *front, const int *P, int B, int n, int m, const double *ref,
                  float *lower, float *upper, int *K, cudaStream_t s);
 int launch_ehvi(const float *mean, const float *var, int B, long long N, const double *front,

@@ -64,6 +64,7 @@ struct Layout {
 
 struct PostArgs {
   const float *Xc;
+  const float *kst;  // precomputed K* (PRE variant), else unused
   float *mean, *var;
   const float *bop, *xt, *s2f;
   int *status;
@@ -131,6 +132,57 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// The K* values of one builder thread's COLS columns of a 32-point chunk:
+// squared scaled distances in packed pairs (candidate x*_k / l_k as a
+// duplicated pair, minus the chunk's training coordinates x_k / l_k), then
+// k = s2 (1 + sqrt5 r + 5/3 r^2) exp(-sqrt5 r) with exp(-x) = 2^(-x log2 e).
+// Both the fused builders and the stand-alone K* kernel use this, so their
+// values are identical.
+template <int DP, int COLS>
+__device__ __forceinline__ void kstar_cols(const unsigned long long (&xs2)[DP], const float *xth,
+                                           int g, float s2, float (&kv)[COLS]) {
+  unsigned long long acc2[COLS / 2];
+#pragma unroll
+  for (int e = 0; e < COLS / 2; ++e) acc2[e] = 0ull;
+#pragma unroll
+  for (int k = 0; k < DP; ++k) {
+    // 16-byte loads: two training points' coordinate pairs each
+    const ulonglong2 *h4 = (const ulonglong2 *)(xth + k * BOUTE_KCHUNK + COLS * g);
+    unsigned long long h2[COLS / 2];
+#pragma unroll
+    for (int e = 0; e < COLS / 4; ++e) {
+      const ulonglong2 v = h4[e];
+      h2[2 * e] = v.x;
+      h2[2 * e + 1] = v.y;
+    }
+#pragma unroll
+    for (int e = 0; e < COLS / 2; ++e) {
+      const unsigned long long df = f2_sub(xs2[k], h2[e]);
+      acc2[e] = f2_fma(df, df, acc2[e]);
+    }
+  }
+#pragma unroll
+  for (int e = 0; e < COLS / 2; ++e) {
+    float r2[2];
+    f2_split(acc2[e], r2[0], r2[1]);
+#pragma unroll
+    for (int z = 0; z < 2; ++z) {
+      const float rr = sqrt_approx(r2[z]);
+      const float sr = kSqrt5 * rr;
+      kv[2 * e + z] = s2 * fmaf(kFiveThirds, r2[z], 1.0f + sr) * ex2_approx(-kSqrt5Log2e * rr);
+    }
+  }
+}
+
+// A candidate's scaled coordinates as duplicated pairs, x*_k (1/l_k hi + lo),
+// from the objective's parameters (1/l hi [DP], 1/l lo [DP], s2) of a chunk.
+template <int DP>
+__device__ __forceinline__ void scaled_candidate(const float (&xr)[DP], const float *il,
+                                                 unsigned long long (&xs2)[DP]) {
+#pragma unroll
+  for (int k = 0; k < DP; ++k) xs2[k] = f2_dup(fmaf(xr[k], il[k], xr[k] * il[DP + k]));
+}
+
 // Position in a ring of R stages: the stage index and the parity of the
 // stage's use count (the mbarrier phase a consumer waits for), advanced
 // without integer division.
@@ -164,7 +216,9 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity,
   }
 }
 
-template <int DP>
+// PRE: the K* values come precomputed (kstar_kernel) instead of being built
+// here; everything else is the same.
+template <int DP, bool PRE>
 __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
     posterior_kernel(const __grid_constant__ PostArgs a) {
   constexpr int kBldWarps = Layout<DP>::kBld;
@@ -187,7 +241,8 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   uint64_t *b_full = bars + 2 * kMaxA, *b_empty = b_full + kMaxB;
   uint64_t *x_full = b_full + 2 * kMaxB, *x_empty = x_full + kMaxX;
   uint64_t *acc_full = x_full + 2 * kMaxX, *acc_empty = acc_full + 2, *drain = acc_full + 4;
-  uint32_t *tmem_holder = (uint32_t *)(drain + 1);
+  uint64_t *ahi_full = drain + 1;  // PRE: the K* image of an A stage has landed
+  uint32_t *tmem_holder = (uint32_t *)(ahi_full + kMaxA);
   volatile int *abort = (volatile int *)(tmem_holder + 1);
 
   auto a_hi = [&](int s) { return (float *)(sm + (size_t)s * kABytes); };
@@ -213,6 +268,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       mbar_init(&acc_empty[i], kEpiWarps);
     }
     mbar_init(drain, 1);
+    for (int s = 0; s < kMaxA; ++s) mbar_init(&ahi_full[s], 1);
     *abort = 0;
     fence_mbar_init();
   }
@@ -232,9 +288,12 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       const bool is_b = warp == 0;
       const int R = is_b ? SB : SX;
       uint64_t *full = is_b ? b_full : x_full, *empty = is_b ? b_empty : x_empty;
+      // PRE: the side-input producer also brings each A stage's K* image (the
+      // stage is free once the MMAs that read it have completed)
+      const bool with_a = PRE && !is_b;
       uint32_t q = 0;
-      RingPos rp;
-      int last_q = -1;  // last job issued
+      RingPos rp, ra;
+      int last_q = -1, last_qa = -1;  // last jobs issued
       for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
         const int tile = unit / m, t = unit % m;
         const int b = tile / a.tiles_per_problem;
@@ -242,7 +301,16 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
           const int bt = b * m + t;
           for (int p = 0; p < pl.npass && !*abort; ++p) {
             const uint32_t bbytes = (uint32_t)(2 * pl.ncol[p] * 128);
-            for (int c = 0; c < pl.kc[p]; ++c, ++q, rp.advance(R)) {
+            for (int c = 0; c < pl.kc[p]; ++c, ++q, rp.advance(R), ra.advance(SA)) {
+              if (with_a) {
+                const int sa = ra.idx;
+                if (q >= (uint32_t)SA && !wait_or_abort(&a_empty[sa], ra.phase ^ 1u, abort)) break;
+                mbar_arrive_expect_tx(&ahi_full[sa], kABytes / 2);
+                bulk_g2s(a_hi(sa),
+                         a.kst + ((size_t)unit * pl.nchunk + c) * BOUTE_TILE_M * BOUTE_KCHUNK,
+                         kABytes / 2, &ahi_full[sa]);
+                last_qa = (int)q;
+              }
               const int s = rp.idx;
               if (q >= (uint32_t)R && !wait_or_abort(&empty[s], rp.phase ^ 1u, abort)) break;
               if (is_b) {
@@ -264,6 +332,8 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       if (*abort) {  // let our copies land before the block exits
         for (int j = std::max(0, last_q - R + 1); j <= last_q; ++j)
           mbar_wait(&full[j % R], (j / R) & 1);
+        for (int j = std::max(0, last_qa - SA + 1); j <= last_qa; ++j)
+          mbar_wait(&ahi_full[j % SA], (j / SA) & 1);
       }
     }
   } else if (warp == 1) {
@@ -383,10 +453,12 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       const int tile = unit / m, t = unit % m;
       const int b = tile / a.tiles_per_problem;
       const long long row = (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M + r;
-      const float *xrow = a.Xc + ((long long)b * a.N + row) * d;
       float xr[DP];
+      if (!PRE) {
+        const float *xrow = a.Xc + ((long long)b * a.N + row) * d;
 #pragma unroll
-      for (int k = 0; k < DP; ++k) xr[k] = (k < d && row < a.N) ? xrow[k] : 0.f;
+        for (int k = 0; k < DP; ++k) xr[k] = (k < d && row < a.N) ? xrow[k] : 0.f;
+      }
       {
         unsigned long long xs2[DP];
         float s2 = 0.f;
@@ -395,37 +467,31 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
           const bool last_pass = p == pl.npass - 1;
           for (int c = 0; c < pl.kc[p]; ++c, ++q, pa.advance(SA), px.advance(SX)) {
             const int s = pa.idx, j = px.idx;
-            if (q >= (uint32_t)SA && !wait_or_abort(&a_empty[s], pa.phase ^ 1u, abort)) break;
+            if (PRE) {
+              if (!wait_or_abort(&ahi_full[s], pa.phase, abort)) break;
+            } else if (q >= (uint32_t)SA && !wait_or_abort(&a_empty[s], pa.phase ^ 1u, abort)) {
+              break;
+            }
             if (!wait_or_abort(&x_full[j], px.phase, abort)) break;
             const float *xth = xt_reg(j), *xtl = xth + BOUTE_KCHUNK * DP;  // x hi, x lo
             const float *alp = xtl + BOUTE_KCHUNK * DP;
-            if (p == 0 && c == 0) {  // new objective: its parameters came with the chunk
+            if (!PRE && p == 0 && c == 0) {  // new objective: its parameters came with the chunk
               const float *il = xth + xt_param_offset(DP);
-#pragma unroll
-              for (int k = 0; k < DP; ++k) xs2[k] = f2_dup(fmaf(xr[k], il[k], xr[k] * il[DP + k]));
+              scaled_candidate<DP>(xr, il, xs2);
               s2 = il[2 * DP];
             }
-            // squared scaled distances to this thread's COLS training points, in
-            // pairs: x*_k - x_k (fp32 scaled coordinates), squared and accumulated
-            unsigned long long acc2[COLS / 2];
-#pragma unroll
-            for (int e = 0; e < COLS / 2; ++e) acc2[e] = 0ull;
-#pragma unroll
-            for (int k = 0; k < DP; ++k) {
-              // 16-byte loads: two training points' coordinate pairs each
-              const ulonglong2 *h4 = (const ulonglong2 *)(xth + k * BOUTE_KCHUNK + COLS * g);
-              unsigned long long h2[COLS / 2];
+            float kv[COLS];
+            if (PRE) {  // this thread's COLS values of chunk c, from the stage's image
 #pragma unroll
               for (int e = 0; e < COLS / 4; ++e) {
-                const ulonglong2 v = h4[e];
-                h2[2 * e] = v.x;
-                h2[2 * e + 1] = v.y;
+                const float4 v = *(const float4 *)(a_hi(s) + sw128_off(r, COLS * g + 4 * e));
+                kv[4 * e] = v.x;
+                kv[4 * e + 1] = v.y;
+                kv[4 * e + 2] = v.z;
+                kv[4 * e + 3] = v.w;
               }
-#pragma unroll
-              for (int e = 0; e < COLS / 2; ++e) {
-                const unsigned long long df = f2_sub(xs2[k], h2[e]);
-                acc2[e] = f2_fma(df, df, acc2[e]);
-              }
+            } else {
+              kstar_cols<DP, COLS>(xs2, xth, g, s2, kv);
             }
             const bool full_chunk = (c + 1) * BOUTE_KCHUNK <= n;
             const int jbase = c * BOUTE_KCHUNK + COLS * g;
@@ -439,28 +505,21 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
               for (int g4 = 0; g4 < COLS / 4; ++g4) {
                 float vh[4], vl[4];
 #pragma unroll
-                for (int e2 = 0; e2 < 2; ++e2) {
-                  float r2[2];
-                  f2_split(acc2[2 * g4 + e2], r2[0], r2[1]);
-#pragma unroll
-                  for (int z = 0; z < 2; ++z) {
-                    const int e = 2 * e2 + z, kk = 4 * g4 + e;
-                    // k = s2 (1 + sqrt5 r + 5/3 r^2) exp(-sqrt5 r), exp(-x) = 2^(-x log2 e)
-                    const float rr = sqrt_approx(r2[z]);
-                    const float sr = kSqrt5 * rr;
-                    float kv =
-                        s2 * fmaf(kFiveThirds, r2[z], 1.0f + sr) * ex2_approx(-kSqrt5Log2e * rr);
-                    if (decltype(ragged)::value) kv = (jbase + kk < n) ? kv : 0.f;
-                    mu_part = fmaf(kv, alg[kk], mu_part);
-                    // hi keeps the 19 bits the tensor core reads (it truncates
-                    // an fp32 operand to tf32); lo = kv - hi exactly
-                    const float hi = __uint_as_float(__float_as_uint(kv) & 0xFFFFE000u);
-                    vh[e] = hi;
-                    vl[e] = kv - hi;
-                  }
+                for (int e = 0; e < 4; ++e) {
+                  const int kk = 4 * g4 + e;
+                  float v = kv[kk];
+                  if (decltype(ragged)::value) v = (jbase + kk < n) ? v : 0.f;
+                  mu_part = fmaf(v, alg[kk], mu_part);
+                  // hi keeps the 19 bits the tensor core reads (it truncates an
+                  // fp32 operand to tf32); lo = v - hi exactly
+                  const float hi = __uint_as_float(__float_as_uint(v) & 0xFFFFE000u);
+                  vh[e] = hi;
+                  vl[e] = v - hi;
                 }
                 const int o = sw128_off(r, COLS * g + g4 * 4);
-                *(float4 *)(Ah + o) = make_float4(vh[0], vh[1], vh[2], vh[3]);
+                // (PRE: the stage already holds the full values, which the
+                // tensor core reads as their hi parts)
+                if (!PRE) *(float4 *)(Ah + o) = make_float4(vh[0], vh[1], vh[2], vh[3]);
                 *(float4 *)(Al + o) = make_float4(vl[0], vl[1], vl[2], vl[3]);
               }
             };
@@ -502,10 +561,11 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
 }
 
 template <int DP>
-int launch_dp(const Gp *gp, const float *Xc, long long N, float *mean, float *var,
-              cudaStream_t s) {
+int launch_dp(const Gp *gp, const float *Xc, const float *kst, long long N, float *mean,
+              float *var, cudaStream_t s) {
   PostArgs a;
   a.Xc = Xc;
+  a.kst = kst;
   a.mean = mean;
   a.var = var;
   a.bop = gp->bop;
@@ -538,13 +598,75 @@ int launch_dp(const Gp *gp, const float *Xc, long long N, float *mean, float *va
   }
   const size_t smem =
       fixed + (size_t)a.sa * kABytes + (size_t)a.sb * a.b_bytes + (size_t)a.sx * a.x_bytes;
-  prefer_shared(posterior_kernel<DP>);
-  cudaFuncSetAttribute(posterior_kernel<DP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                       (int)smem);
-  int sms = 152;
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, 0);
-  const int grid = std::max(1, std::min(a.tiles_total * a.m, sms));  // (tile, objective) units
-  launch_pdl(posterior_kernel<DP>, dim3(grid), dim3(Layout<DP>::kThreads), smem, s, a);
+  const int grid = std::max(1, std::min(a.tiles_total * a.m, num_sms()));  // (tile, objective) units
+  auto go = [&](auto kern) {
+    prefer_shared(kern);
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    launch_pdl(kern, dim3(grid), dim3(Layout<DP>::kThreads), smem, s, a);
+  };
+  if (kst) go(posterior_kernel<DP, true>);
+  else go(posterior_kernel<DP, false>);
+  count_launch();
+  return last_launch_status();
+}
+
+// ---- K* ahead of the fit's results ------------------------------------------------
+// One block per (tile, objective) unit, threads laid out as the posterior's
+// builders: all n training points' K* values of the tile's 128 candidates, in
+// the builders' arithmetic, zero beyond n. Each 32-point chunk is stored as
+// the 16 KB image of an A stage (128 rows x 32 fp32, K-major, 128-byte
+// swizzle), so that the posterior brings it in with one bulk copy; the tensor
+// core reads an fp32 operand truncated to tf32, so the full value serves as
+// the hi part. The training points' side input is staged in shared memory.
+// It needs the set-up's side input (not the fit's results) and the candidates.
+template <int DP>
+__global__ void __launch_bounds__(Layout<DP>::kBld * 32) kstar_kernel(
+    const float *Xc, const float *xt, long long N, int d, int m, int n, int tiles_per_problem,
+    int nchunk, float *kst) {
+  constexpr int COLS = Layout<DP>::kCols, GPR = 32 / COLS, RPW = 32 / GPR;
+  extern __shared__ __align__(16) float xs[];  // nchunk side-input chunks
+  const int unit = blockIdx.x, tile = unit / m, t = unit % m, b = tile / tiles_per_problem;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = warp * RPW + lane % RPW, g = lane / RPW;
+  const long long row = (long long)(tile % tiles_per_problem) * BOUTE_TILE_M + r;
+  const int cf = xt_chunk_floats(DP);  // a multiple of 4
+  const float4 *x4 = (const float4 *)(xt + (size_t)(b * m + t) * nchunk * cf);
+  for (int e = threadIdx.x; e < nchunk * cf / 4; e += blockDim.x) ((float4 *)xs)[e] = x4[e];
+  const float *xrow = Xc + ((long long)b * N + row) * d;
+  float xr[DP];
+#pragma unroll
+  for (int k = 0; k < DP; ++k) xr[k] = (k < d && row < N) ? xrow[k] : 0.f;
+  __syncthreads();
+  const float *il = xs + xt_param_offset(DP);
+  unsigned long long xs2[DP];
+  scaled_candidate<DP>(xr, il, xs2);
+  const float s2 = il[2 * DP];
+  for (int c = 0; c < nchunk; ++c) {
+    float kv[COLS];
+    kstar_cols<DP, COLS>(xs2, xs + (size_t)c * cf, g, s2, kv);
+    const int jbase = c * BOUTE_KCHUNK + COLS * g;
+#pragma unroll
+    for (int kk = 0; kk < COLS; ++kk) kv[kk] = (jbase + kk < n) ? kv[kk] : 0.f;
+    float *img = kst + ((size_t)unit * nchunk + c) * BOUTE_TILE_M * BOUTE_KCHUNK;
+#pragma unroll
+    for (int g4 = 0; g4 < COLS / 4; ++g4)
+      *(float4 *)(img + sw128_off(r, COLS * g + 4 * g4)) =
+          make_float4(kv[4 * g4], kv[4 * g4 + 1], kv[4 * g4 + 2], kv[4 * g4 + 3]);
+  }
+}
+
+template <int DP>
+int launch_kstar_dp(const Gp *gp, const float *Xc, long long N, float *kst, cudaStream_t s) {
+  const int tpp = (int)((N + BOUTE_TILE_M - 1) / BOUTE_TILE_M);
+  const int units = tpp * gp->B * gp->m;
+  const size_t smem = (size_t)gp->plan.nchunk * xt_chunk_floats(DP) * sizeof(float);
+  prefer_shared(kstar_kernel<DP>);
+  if (smem > 48 * 1024 &&
+      cudaFuncSetAttribute(kstar_kernel<DP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem) != cudaSuccess)
+    return last_launch_status();
+  kstar_kernel<DP><<<units, Layout<DP>::kBld * 32, smem, s>>>(Xc, gp->xt, N, gp->d, gp->m,
+                                                             gp->n, tpp, gp->plan.nchunk, kst);
   count_launch();
   return last_launch_status();
 }
@@ -552,14 +674,31 @@ int launch_dp(const Gp *gp, const float *Xc, long long N, float *mean, float *va
 }  // namespace
 
 int launch_posterior(const Gp *gp, const float *Xc, long long N, float *mean, float *var,
-                     cudaStream_t s) {
+                     cudaStream_t s, const float *kst) {
   if (N <= 0) return BOUTE_OK;
   switch (gp->DP) {
-    case 8: return launch_dp<8>(gp, Xc, N, mean, var, s);
-    case 12: return launch_dp<12>(gp, Xc, N, mean, var, s);
-    case 16: return launch_dp<16>(gp, Xc, N, mean, var, s);
-    case 24: return launch_dp<24>(gp, Xc, N, mean, var, s);
-    case 32: return launch_dp<32>(gp, Xc, N, mean, var, s);
+    case 8: return launch_dp<8>(gp, Xc, kst, N, mean, var, s);
+    case 12: return launch_dp<12>(gp, Xc, kst, N, mean, var, s);
+    case 16: return launch_dp<16>(gp, Xc, kst, N, mean, var, s);
+    case 24: return launch_dp<24>(gp, Xc, kst, N, mean, var, s);
+    case 32: return launch_dp<32>(gp, Xc, kst, N, mean, var, s);
+  }
+  return BOUTE_ERR_UNSUPPORTED;
+}
+
+size_t kstar_floats(const Gp *gp, long long N) {
+  const size_t tpp = (size_t)((N + BOUTE_TILE_M - 1) / BOUTE_TILE_M);
+  return tpp * gp->B * gp->m * gp->plan.nchunk * BOUTE_TILE_M * BOUTE_KCHUNK;
+}
+
+int launch_kstar(const Gp *gp, const float *Xc, long long N, float *kst, cudaStream_t s) {
+  if (N <= 0) return BOUTE_OK;
+  switch (gp->DP) {
+    case 8: return launch_kstar_dp<8>(gp, Xc, N, kst, s);
+    case 12: return launch_kstar_dp<12>(gp, Xc, N, kst, s);
+    case 16: return launch_kstar_dp<16>(gp, Xc, N, kst, s);
+    case 24: return launch_kstar_dp<24>(gp, Xc, N, kst, s);
+    case 32: return launch_kstar_dp<32>(gp, Xc, N, kst, s);
   }
   return BOUTE_ERR_UNSUPPORTED;
 }

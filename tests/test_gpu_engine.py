@@ -148,3 +148,35 @@ def test_selection_in_acquisition_kernel_matches_separate_selection(B, N, S, k):
     for b in range(w.B):  # values descending, ties by index
         order = np.lexsort((np.arange(w.N), -A[b]))[:k]
         assert want[0][b].tolist() == order.tolist()
+
+
+# Graph replay computes K* on a second stream beside the fit and the posterior
+# only contracts it; stage-timing mode builds K* inside the posterior. Mean,
+# variance, scores and selection must agree bit for bit. (workload, n, N, B):
+# a ragged last chunk of training points, several problems, both
+# acquisition modes.
+TWO_PHASE = [(1, 77, 3000 + 5, 1), (4, 100, 1500 + 1, 3), (0, 32, 4096 + 77, 2)]
+
+
+@pytest.mark.parametrize("wi,n,N,B", TWO_PHASE)
+def test_posterior_from_precomputed_kstar_matches_fused(wi, n, N, B):
+    import torch
+
+    from paper_2602_10729_gb300 import boute as bt
+    base = wl.WORKLOADS[wi]
+    w = dataclasses.replace(wl.scaled(base, N=N, n=n), B=B, seeds=tuple(range(11, 11 + B)))
+    hp = host_problem(w)
+    e = _engine(w)
+    out = []
+    for timing in (False, True):
+        bt.boute_engine_set_timing(e, timing)
+        idx, val = _run(e, w, _dev(hp), "device")
+        mean = torch.empty((w.B, w.m, w.N), dtype=torch.float32, device="cuda")
+        var = torch.empty_like(mean)
+        acq = torch.empty((w.B, w.N), dtype=torch.float32, device="cuda")
+        bt.boute_engine_scores(e, acq=acq, mean=mean, var=var)
+        torch.cuda.synchronize()
+        out.append((idx, val, acq.cpu().numpy(), mean.cpu().numpy(), var.cpu().numpy()))
+    e.free()
+    for a, b in zip(*out):
+        assert np.array_equal(a, b)
