@@ -58,19 +58,31 @@ __global__ void standardize_kernel(const double *Y, int n, int m, double *Ys) {
 }
 
 // ---- fit set-up, one launch: K = s2 M52(X, X) + noise I and the side input --
-// Blocks [0, nkt) of problem-objective bt compute 16 x 16 tiles of K (full,
-// symmetric) in fp64, stored as an fp32 pair (hi = K rounded, lo = K - hi):
-// the factorisation works on hi, the refinement of alpha on hi + lo. The
-// remaining blocks write the posterior's side input: scaled training inputs
-// x / l as fp32 hi/lo pairs (dimension-major per 32-point chunk), and in every
-// chunk the objective's 1/l (hi, lo) and outputscale. Block 0 of the first
-// problem clears the fit status.
+// Blocks [0, nkt) of problem-objective bt compute K in fp64, one half (16 x 8)
+// of a 16 x 16 tile on or below the diagonal per block of 128 threads, each
+// value written to both (i, j) and (j, i), stored as an fp32 pair (hi = K
+// rounded, lo = K - hi): the factorisation works on hi, the refinement of
+// alpha on hi + lo. (The set-up is bound by fp64 throughput: the lower
+// triangle alone, spread over as many SMs as possible.) The remaining blocks
+// write the posterior's side input: scaled training inputs x / l as fp32
+// hi/lo pairs (dimension-major per 32-point chunk), and in every chunk the
+// objective's 1/l (hi, lo) and outputscale. Block 0 of the first problem
+// clears the fit status.
+constexpr int kSetupThreads = 128;
+__host__ __device__ inline int kmat_units(int n) {
+  const int tn = (n + 15) / 16;
+  return tn * (tn + 1);  // tiles on or below the diagonal, two halves each
+}
 __device__ void kmat_tile(const double *X, int n, int d, int b, const double *l, double s2,
-                          double noise, int tile, float *Kh, float *Kl, double *il) {
+                          double noise, int unit, float *Kh, float *Kl, double *il) {
   for (int t = threadIdx.x; t < d; t += blockDim.x) il[t] = 1.0 / l[t];
   __syncthreads();
-  const int tn = (n + 15) / 16;
-  const int i = (tile / tn) * 16 + threadIdx.x / 16, j = (tile % tn) * 16 + threadIdx.x % 16;
+  const int tile = unit >> 1, half = unit & 1;
+  int ti = (int)((sqrtf(8.f * tile + 1.f) - 1.f) * 0.5f);  // tile = ti (ti + 1) / 2 + tj
+  while (ti * (ti + 1) / 2 > tile) --ti;
+  while ((ti + 1) * (ti + 2) / 2 <= tile) ++ti;
+  const int tj = tile - ti * (ti + 1) / 2;
+  const int i = ti * 16 + threadIdx.x / 8, j = tj * 16 + half * 8 + threadIdx.x % 8;
   if (i >= n || j >= n) return;
   const double *xi = X + ((size_t)b * n + i) * d, *xj = X + ((size_t)b * n + j) * d;
   double r2 = 0.0;
@@ -81,10 +93,13 @@ __device__ void kmat_tile(const double *X, int n, int d, int b, const double *l,
   const double r = sqrt(r2), sr = sqrt(5.0) * r;
   double k = s2 * (1.0 + sr + 5.0 * r2 / 3.0) * exp(-sr);
   if (i == j) k += noise;
-  const float kh = (float)k;
-  const size_t o = (size_t)i * n + j;
-  Kh[o] = kh;
-  Kl[o] = (float)(k - (double)kh);
+  const float kh = (float)k, kl = (float)(k - (double)kh);
+  Kh[(size_t)i * n + j] = kh;
+  Kl[(size_t)i * n + j] = kl;
+  if (i != j) {  // (the same value: the squared differences are symmetric)
+    Kh[(size_t)j * n + i] = kh;
+    Kl[(size_t)j * n + i] = kl;
+  }
 }
 
 __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad,
@@ -116,7 +131,7 @@ __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad
   }
 }
 
-__global__ void __launch_bounds__(256) fit_setup_kernel(
+__global__ void __launch_bounds__(kSetupThreads) fit_setup_kernel(
     const double *X, int n, int d, int m, int DP, int npad, const double *ls, const double *s2,
     const double *noise, float *Kh_all, float *Kl_all, float *xt, float *s2f, int nkt, int nprep,
     int early_trigger, int *status) {
@@ -668,17 +683,18 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
                            cudaStream_t s, cudaEvent_t setup_done = nullptr) {
   const int n = gp->n, d = gp->d, m = gp->m, BM = gp->B * gp->m;
   const int npad = gp->plan.npad;
-  const int tn = (n + 15) / 16, nkt = tn * tn;
-  const int nprep = std::max(1, std::min(8, npad * gp->DP / 256));
-  prefer_shared(fit_setup_kernel);
+  const int nkt = kmat_units(n);
   const int sms = num_sms();
+  // side-input blocks: as many as leave one block per SM (K blocks first), 2 .. 16
+  const int nprep = std::max(2, std::min(16, sms / BM - nkt));
+  prefer_shared(fit_setup_kernel);
   // early triggers only when every block of the grid is resident at once (8
   // set-up blocks per SM beside the fit's blocks; one fit block per SM), so
   // that waiting successors can never hold resources a later block needs
   const long long setup_blocks = (long long)(nkt + nprep) * BM;
   const int setup_early = setup_blocks <= 8LL * (sms - BM) ? 1 : 0;
   const int fit_early = 2 * BM <= sms ? 1 : 0;
-  fit_setup_kernel<<<dim3(nkt + nprep, BM), 256, 0, s>>>(X, n, d, m, gp->DP, npad, ls, s2, noise,
+  fit_setup_kernel<<<dim3(nkt + nprep, BM), kSetupThreads, 0, s>>>(X, n, d, m, gp->DP, npad, ls, s2, noise,
                                                          gp->Kh, gp->Kl, gp->xt, gp->s2f, nkt,
                                                          nprep, setup_early, gp->status);
   if (setup_done && cudaEventRecord(setup_done, s) != cudaSuccess) return last_launch_status();
