@@ -208,7 +208,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     int early_trigger, int *status) {
   extern __shared__ __align__(16) float sm[];
   __shared__ int bad;
-  __shared__ uint64_t lbar;
+  __shared__ uint64_t lbar, lbar_lo;  // K hi; K lo (needed only by the residual)
   __shared__ double ymu, yisd;
   __shared__ __align__(16) float colL[32][64];  // columns of L_pp, zero-padded
   __shared__ float invs[32];                    // 1 / L_cc
@@ -259,14 +259,18 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   if (bulk) {
     if (tid == 0) {
       mbar_init(&lbar, 1);
+      mbar_init(&lbar_lo, 1);
       fence_mbar_init();
     }
     __syncthreads();
     if (tid == 0) {
       const uint32_t bytes = (uint32_t)n * n * sizeof(float);
-      mbar_arrive_expect_tx(&lbar, kl_smem ? 2 * bytes : bytes);
+      mbar_arrive_expect_tx(&lbar, bytes);
       bulk_g2s(W, Kh, bytes, &lbar);
-      if (kl_smem) bulk_g2s(Kls, Kl, bytes, &lbar);
+      if (kl_smem) {  // lands while the factorisation runs
+        mbar_arrive_expect_tx(&lbar_lo, bytes);
+        bulk_g2s(Kls, Kl, bytes, &lbar_lo);
+      }
     }
   } else {  // eight independent loads per thread in flight before their stores
     const int nn = n * n;
@@ -299,6 +303,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     if (!mbar_wait(&lbar, 0)) {  // the copy never completed: report, drain, leave
       if (tid == 0) set_status(status, BOUTE_ERR_TIMEOUT);
       mbar_wait(&lbar, 0);
+      if (kl_smem) mbar_wait(&lbar_lo, 0);
       return;
     }
     for (int e = tid; e < n * n; e += nthr) {
@@ -316,6 +321,26 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   if (tid == 0) bad = 0;
   for (int e = tid; e < 32 * 64; e += nthr) (&colL[0][0])[e] = 0.f;
   __syncthreads();
+  // Operand images of W for the posterior (one column pass, n <= 160): rows
+  // [g_lo, g_hi) of W, warps w0, w0 + nws, ... one row each, lane = k % 32.
+  // A block row of W is final once its panel's trailing update is done.
+  auto pack_rows = [&](int g_lo, int g_hi, int w0, int nws) {
+    float *img = bop + (size_t)bt * plan.image_floats + plan.off[0];
+    const int ncol = plan.ncol[0], kc = plan.kc[0];
+    for (int g = g_lo + w0; g < g_hi && g < ncol; g += nws) {
+      const float *wr = W + (size_t)g * ld;
+      const int o = sw128_off(g, lane);
+#pragma unroll 4
+      for (int c = 0; c < kc; ++c) {
+        const int k = c * BOUTE_KCHUNK + lane;
+        const float v = (k < n && g < n && k <= g) ? wr[k] : 0.f;
+        const float hi = tf32_rna(v), lo = tf32_rna(v - hi);
+        float *blk = img + (size_t)c * 2 * ncol * BOUTE_KCHUNK;
+        blk[o] = hi;
+        blk[ncol * BOUTE_KCHUNK + o] = lo;
+      }
+    }
+  };
   // ---- blocked Cholesky and W = L^-1, 32-column panels -------------------------
   // Iteration p: (a) warp 0 factors the diagonal block, A_pp = L_pp L_pp^T,
   // and warp 1 inverts it one column behind, W_pp = L_pp^-1, both
@@ -400,6 +425,9 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
       float *Wr = W + (size_t)(p0 + lane) * ld + p0;
 #pragma unroll
       for (int c = 0; c < 32; ++c) Wr[c] = w[c] * myinv;
+    } else if (SMEM && p > 0) {
+      // the other warps pack the previous block row of W meanwhile
+      pack_rows(p0 - 32, p0, warp - 2, nw - 2);
     }
     __syncthreads();
     if (bad) break;
@@ -508,8 +536,10 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     }
     __syncthreads();
   }
+  const bool lo_copy = bulk && kl_smem;  // K lo is on its way by bulk copy
   if (bad) {
     if (tid == 0) set_status(status, BOUTE_ERR_NOT_PD);
+    if (lo_copy) mbar_wait(&lbar_lo, 0);  // let it land before the block exits
     return;
   }
   // ---- alpha0 = W^T (W y), refined once against K = hi + lo ----------------------
@@ -544,6 +574,11 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     __syncthreads();
   };
   solve(yv, al);
+  if (lo_copy && !mbar_wait(&lbar_lo, 0)) {  // the copy never completed: report, drain, leave
+    if (tid == 0) set_status(status, BOUTE_ERR_TIMEOUT);
+    mbar_wait(&lbar_lo, 0);
+    return;
+  }
   // residual r = y - K alpha0 in double-float. Shared-memory variant: K hi
   // from the upper triangle of A and its diagonal, K lo from shared memory
   // when it fits there; half a warp per row.
@@ -626,23 +661,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   // outputs: the operand images of W (packed here from shared memory; the
   // global variant leaves W in the workspace for pack_kernel), alpha into the
   // side input
-  if (SMEM) {  // one column pass (n <= 160): warp per row g, lane = k % 32
-    float *img = bop + (size_t)bt * plan.image_floats + plan.off[0];
-    const int ncol = plan.ncol[0], kc = plan.kc[0];
-    for (int g = warp; g < ncol; g += nw) {
-      const float *wr = W + (size_t)g * ld;
-      const int o = sw128_off(g, lane);
-#pragma unroll 4
-      for (int c = 0; c < kc; ++c) {
-        const int k = c * BOUTE_KCHUNK + lane;
-        const float v = (k < n && g < n && k <= g) ? wr[k] : 0.f;
-        const float hi = tf32_rna(v), lo = tf32_rna(v - hi);
-        float *blk = img + (size_t)c * 2 * ncol * BOUTE_KCHUNK;
-        blk[o] = hi;
-        blk[ncol * BOUTE_KCHUNK + o] = lo;
-      }
-    }
-  }
+  if (SMEM) pack_rows(NP - 32, NP, warp, nw);  // the last block row (the others: above)
   const int cf = xt_chunk_floats(DP);
   float *xa = xt + (size_t)bt * (npad / BOUTE_KCHUNK) * cf + 2 * BOUTE_KCHUNK * DP;
   for (int k = tid; k < npad; k += nthr)
