@@ -214,7 +214,7 @@ __global__ void __launch_bounds__(512, 2) mchvi2_kernel(const float *mean, const
   const bool vec = (S == 128) && ((uintptr_t)eps & 15) == 0 && (eps_stride % 4) == 0;
   const long long cstride = (long long)gridDim.x * wpb;
   const float inv_s = 1.f / (float)S;
-  unsigned long long top = 0ull;  // this warp's running top-32 (SEL)
+  WarpTopBatch sel;  // this warp's running top-32 (SEL)
   auto eps_of = [&](long long c) {
     return eps + ((size_t)b * N + c) * eps_stride + (eps_stride == 0 ? (size_t)b * 2 * S : 0);
   };
@@ -272,17 +272,18 @@ __global__ void __launch_bounds__(512, 2) mchvi2_kernel(const float *mean, const
 #pragma unroll
         for (int j = 0; j < 4; ++j) sum += fmaxf(t0.x - y1[j], 0.f) * fmaxf(t0.y - y2[j], 0.f);
         const float iH = H > 0.f ? rcp_fast(H) : 0.f;  // H <= 0: every sample dominated
+        // height of strip k for sample j: sat(u_k / H - y2_j / H)
+        const float ny2[4] = {-y2[0] * iH, -y2[1] * iH, -y2[2] * iH, -y2[3] * iH};
         float acc = 0.f;
 #pragma unroll 1
         for (int k = 1; k < Kp; k += 4) {
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
             const float4 t = strips4[k + q];
-            const float uh = t.z * iH;
             float tk = 0.f;
 #pragma unroll
             for (int j = 0; j < 4; ++j)
-              tk = fmaf(fma_sat(-y1[j], t.y, t.x), fma_sat(-y2[j], iH, uh), tk);
+              tk = fmaf(fma_sat(-y1[j], t.y, t.x), fma_sat(t.z, iH, ny2[j]), tk);
             acc = fmaf(t.w, tk, acc);
           }
         }
@@ -291,7 +292,7 @@ __global__ void __launch_bounds__(512, 2) mchvi2_kernel(const float *mean, const
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
       if (lane == 0) acq[(size_t)b * N + c] = sum * inv_s;
-      if (SEL) top = warp_insert_desc(top, make_key(sum * inv_s, (unsigned)c), lane);
+      if (SEL) sel.add(make_key(sum * inv_s, (unsigned)c), lane);
     }
   } else {
   for (long long c = (long long)blockIdx.x * wpb + warp; c < N; c += cstride) {
@@ -303,10 +304,12 @@ __global__ void __launch_bounds__(512, 2) mchvi2_kernel(const float *mean, const
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
     if (lane == 0) acq[(size_t)b * N + c] = sum * inv_s;
-    if (SEL) top = warp_insert_desc(top, make_key(sum * inv_s, (unsigned)c), lane);
+    if (SEL) sel.add(make_key(sum * inv_s, (unsigned)c), lane);
   }
   }
   if (!SEL) return;
+  sel.flush(lane);
+  unsigned long long top = sel.top;
   // ---- selection. Block list (tree over the 16 warps); with several blocks
   // per problem, blocks form groups of kSelGroup: the last block of a group to
   // finish merges the group's lists, and the last group of the problem to

@@ -71,6 +71,26 @@ __device__ __forceinline__ unsigned long long warp_insert_desc(unsigned long lon
   return lane < pos ? top : (lane == pos ? key : up);
 }
 
+// A warp's running top-32 fed one key at a time (the same key in every lane):
+// keys wait in a lane each (lane i holds the i-th since the last merge) and
+// are sorted and merged into the list 32 at a time, so that adding a key
+// costs a select. flush() merges what is pending; top then holds the 32
+// largest keys added, descending (zero where fewer were added).
+struct WarpTopBatch {
+  unsigned long long top = 0ull, pend = 0ull;
+  int count = 0;  // pending keys (the same in every lane)
+  __device__ __forceinline__ void add(unsigned long long key, int lane) {
+    if (lane == count) pend = key;
+    if (++count == kWarpK) flush(lane);
+  }
+  __device__ __forceinline__ void flush(int lane) {
+    if (count == 0) return;
+    top = warp_merge_desc(top, warp_sort_desc(pend, lane), lane);
+    pend = 0ull;
+    count = 0;
+  }
+};
+
 // Counts a block in on *p at GPU scope with acquire-release order. Release:
 // what this thread wrote, or observed before a barrier it passed, is visible
 // to whoever observes the new count. Acquire: a thread that observes the
