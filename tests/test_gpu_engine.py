@@ -154,8 +154,9 @@ def test_selection_in_acquisition_kernel_matches_separate_selection(B, N, S, k):
 # only contracts it; stage-timing mode builds K* inside the posterior. Mean,
 # variance, scores and selection must agree bit for bit. (workload, n, N, B):
 # a ragged last chunk of training points, several problems, both
-# acquisition modes.
-TWO_PHASE = [(1, 77, 3000 + 5, 1), (4, 100, 1500 + 1, 3), (0, 32, 4096 + 77, 2)]
+# acquisition modes, more than 256 training points.
+TWO_PHASE = [(1, 77, 3000 + 5, 1), (4, 100, 1500 + 1, 3), (0, 32, 4096 + 77, 2),
+             (1, 300, 700 + 3, 1), (4, 288, 500, 2)]  # (two column passes, split reduction)
 
 
 @pytest.mark.parametrize("wi,n,N,B", TWO_PHASE)
