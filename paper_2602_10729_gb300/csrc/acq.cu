@@ -5,6 +5,7 @@
 #include <algorithm>
 
 #include "internal.h"
+#include "mc2.cuh"
 #include "warp_select.cuh"
 
 namespace boute {
@@ -145,32 +146,9 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
   }
 }
 
-// 2-objective Monte-Carlo HVI over the strip decomposition: strips k = 0..K-1
-// with x-extent [a_k, b_k) (a_0 = -inf, a_k = b_{k-1}) and top u_k (u
-// decreasing, u_0 = r2 the largest). For a sample y the improvement is
-//   sum_k (b_k - max(a_k, y1))^+ (u_k - y2)^+
-//     = (b_0 - y1)^+ (u_0 - y2)^+ + H sum_{k>=1} D_k sat((b_k - y1) / D_k) sat((u_k - y2) / H)
-// with D_k = b_k - a_k, because (b_k - max(a_k, y1))^+ is (b_k - y1) clamped
-// to [0, D_k], and with H = u_0 - min y2 >= u_k - y2 over the samples a thread
-// holds, so that (u_k - y2)^+ = H sat((u_k - y2) / H). Per strip and sample:
-// two saturating FMAs and one FMA. One warp per candidate, a float4 of base
-// normals per lane and objective when S = 128.
-__device__ __forceinline__ float fma_sat(float a, float b, float c) {
-  float d;
-  asm("fma.rn.sat.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
-  return d;
-}
-__device__ __forceinline__ float sqrt_fast(float x) {
-  float y;
-  asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-__device__ __forceinline__ float rcp_fast(float x) {
-  float y;
-  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
+// 2-objective Monte-Carlo HVI over the strip decomposition (mc2.cuh): one
+// warp per candidate, a float4 of base normals per lane and objective when
+// S = 128.
 // SEL: also select the ksel <= 32 best candidates of each problem as they are
 // scored: every warp keeps a running top-32 of its candidates, each block
 // merges its warps' lists into sel_keys, and the last block of a problem to
@@ -192,22 +170,8 @@ __global__ void __launch_bounds__(512, 2) mchvi2_kernel(const float *mean, const
   pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
   const int b = blockIdx.y;
-  const int K = Kc[b];
-  const int Kp = K > 0 ? 1 + ((K + 2) & ~3) : 0;
-  for (int i = threadIdx.x; i < Kp; i += blockDim.x) {
-    if (i >= K) {
-      strips4[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-      continue;
-    }
-    const size_t o = ((size_t)b * box_cap + i) * 2;
-    const float ai = lower[o], bi = upper[o], ui = upper[o + 1];
-    if (i == 0) {
-      strips4[0] = make_float4(bi, ui, 0.f, 0.f);
-    } else {
-      const float D = bi - ai;
-      strips4[i] = D > 0.f ? make_float4(bi / D, 1.f / D, ui, D) : make_float4(0.f, 0.f, ui, 0.f);
-    }
-  }
+  const int K = mc2_load_strips(strips4, lower, upper, Kc, b, box_cap, threadIdx.x, blockDim.x);
+  const int Kp = mc2_padded(K);
   __syncthreads();
   const float *m1 = mean + (size_t)b * 2 * N, *m2 = m1 + N;
   const float *v1 = var + (size_t)b * 2 * N, *v2 = v1 + N;
@@ -249,48 +213,16 @@ __global__ void __launch_bounds__(512, 2) mchvi2_kernel(const float *mean, const
       pm1 = m1[c]; pm2 = m2[c]; pv1 = v1[c]; pv2 = v2[c];
     }
     const float4 t0 = K > 0 ? strips4[0] : make_float4(0.f, 0.f, 0.f, 0.f);
-    const float u0 = t0.y;
     for (; c < Ni; c += cs) {
       const float4 c1 = z1, c2 = z2;
-      const float mu1 = pm1, mu2 = pm2;
-      const float sg1 = sqrt_fast(fmaxf(pv1, 0.f)), sg2 = sqrt_fast(fmaxf(pv2, 0.f));
+      const float mu1 = pm1, mu2 = pm2, qv1 = pv1, qv2 = pv2;
       const bool more = c + cs < Ni;
       const int cn = more ? c + cs : c;
       ep = more ? ep + estep : ep;
       z1 = __ldcs((const float4 *)ep);
       z2 = __ldcs((const float4 *)(ep + S));
       pm1 = m1[cn]; pm2 = m2[cn]; pv1 = v1[cn]; pv2 = v2[cn];
-      const float y1[4] = {fmaf(sg1, c1.x, mu1), fmaf(sg1, c1.y, mu1), fmaf(sg1, c1.z, mu1),
-                           fmaf(sg1, c1.w, mu1)};
-      const float y2[4] = {fmaf(sg2, c2.x, mu2), fmaf(sg2, c2.y, mu2), fmaf(sg2, c2.z, mu2),
-                           fmaf(sg2, c2.w, mu2)};
-      // per lane: H = u_0 - (its lowest y2) bounds every height of its samples
-      const float lo2 = fminf(fminf(y2[0], y2[1]), fminf(y2[2], y2[3]));
-      const float H = u0 - lo2;
-      float sum = 0.f;
-      if (K > 0) {
-#pragma unroll
-        for (int j = 0; j < 4; ++j) sum += fmaxf(t0.x - y1[j], 0.f) * fmaxf(t0.y - y2[j], 0.f);
-        const float iH = H > 0.f ? rcp_fast(H) : 0.f;  // H <= 0: every sample dominated
-        // height of strip k for sample j: sat(u_k / H - y2_j / H)
-        const float ny2[4] = {-y2[0] * iH, -y2[1] * iH, -y2[2] * iH, -y2[3] * iH};
-        float acc = 0.f;
-#pragma unroll 1
-        for (int k = 1; k < Kp; k += 4) {
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const float4 t = strips4[k + q];
-            float tk = 0.f;
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-              tk = fmaf(fma_sat(-y1[j], t.y, t.x), fma_sat(t.z, iH, ny2[j]), tk);
-            acc = fmaf(t.w, tk, acc);
-          }
-        }
-        sum = fmaf(fmaxf(H, 0.f), acc, sum);
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+      const float sum = mc2_warp_total(mc2_lane_sum(strips4, K, Kp, t0, c1, c2, mu1, mu2, qv1, qv2));
       if (lane == 0) acq[(size_t)b * N + c] = sum * inv_s;
       if (SEL) sel.add(make_key(sum * inv_s, (unsigned)c), lane);
     }
