@@ -98,10 +98,10 @@ struct boute_engine {
   } graphs[2];
   int graph_next, graphs_off;
   // the front stage (standardise, Pareto front, boxes) depends on the raw
-  // outcomes only: it runs on a second stream, forked from and joined back
-  // into the step's stream, beside the GP fit
+  // outcomes only: it runs on a second stream, forked after the fit's set-up
+  // (ev_setup) and joined back into the step's stream, beside the GP fit
   cudaStream_t side;
-  cudaEvent_t fork, join;
+  cudaEvent_t join;
   // host-input steps: candidates and base normals are copied on two copy
   // streams while the fit runs; the step waits for them only where it needs
   // them (posterior, acquisition)
@@ -266,7 +266,6 @@ void boute_engine_free(boute_engine *e) {
     for (int i = 0; i <= ST_COUNT; ++i) cudaEventDestroy(e->ev[i]);
   for (auto &g : e->graphs)
     if (g.exec) cudaGraphExecDestroy(g.exec);
-  if (e->fork) cudaEventDestroy(e->fork);
   if (e->join) cudaEventDestroy(e->join);
   if (e->side) cudaStreamDestroy(e->side);
   for (cudaEvent_t ev : {e->ev_in, e->ev_xc, e->ev_eps[0], e->ev_eps[1], e->ev_setup, e->join2})
@@ -351,7 +350,6 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
        cudaStreamCreateWithFlags(&e->side2, cudaStreamNonBlocking) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->ev_setup, cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->join2, cudaEventDisableTiming) != cudaSuccess ||
-       cudaEventCreateWithFlags(&e->fork, cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->join, cudaEventDisableTiming) != cudaSuccess ||
        cudaStreamCreateWithFlags(&e->cpy[0], cudaStreamNonBlocking) != cudaSuccess ||
        cudaStreamCreateWithFlags(&e->cpy[1], cudaStreamNonBlocking) != cudaSuccess ||
@@ -394,13 +392,6 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
                               e->upper, e->K, mc, fs);
   };
   mark(ST_FIT);
-  if (!e->timing) {  // fork: the front stage runs beside the fit
-    if (cudaEventRecord(e->fork, s) != cudaSuccess ||
-        cudaStreamWaitEvent(e->side, e->fork, 0) != cudaSuccess)
-      return last_launch_status();
-    if ((r = front(e->side))) return r;
-    if (cudaEventRecord(e->join, e->side) != cudaSuccess) return last_launch_status();
-  }
   // waits on the host-input copies: an external-event node when captured
   cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
   if (host && cudaStreamIsCapturing(s, &cap) != cudaSuccess) return last_launch_status();
@@ -408,8 +399,16 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
       cap == cudaStreamCaptureStatusActive ? cudaEventWaitExternal : cudaEventWaitDefault;
   // K* beside the fit (not in stage-timing mode, where the posterior builds it)
   const float *kst = e->timing ? nullptr : e->kst;
-  if ((r = launch_fit_raw(&e->gp->g, X, Y, ls, s2, noise, s, kst ? e->ev_setup : nullptr)))
+  // The graph has one root, the fit's set-up: the front stage (which needs
+  // the raw outcomes only) and K* (which needs the set-up's side input) fork
+  // after it and run beside the fit (one root launches sooner than two).
+  if ((r = launch_fit_raw(&e->gp->g, X, Y, ls, s2, noise, s, e->timing ? nullptr : e->ev_setup)))
     return r;
+  if (!e->timing) {
+    if (cudaStreamWaitEvent(e->side, e->ev_setup, 0) != cudaSuccess) return last_launch_status();
+    if ((r = front(e->side))) return r;
+    if (cudaEventRecord(e->join, e->side) != cudaSuccess) return last_launch_status();
+  }
   if (kst) {
     if (cudaStreamWaitEvent(e->side2, e->ev_setup, 0) != cudaSuccess ||
         (host && cudaStreamWaitEvent(e->side2, e->ev_xc, wait_flags) != cudaSuccess))
