@@ -193,6 +193,15 @@ int boute_select_topk_noalloc(const float *acq, int B, long long N, int k, long 
  *   idx: B x k int64, val: B x k fp32.
  * boute_engine_step_async: as boute_engine_step without the final
  * synchronisation (device errors surface at the next synchronising call).
+ * boute_engine_step_host_async: as boute_engine_step_host without the final
+ * synchronisation, for a stream of steps: consecutive calls alternate between
+ * two sets of device input buffers, so that one step's host-to-device copies
+ * overlap the previous step's computation. Until the step has completed
+ * (boute_engine_sync, or a synchronisation of `stream`) its host inputs must
+ * stay unchanged and its idx / val must not be read. The second input set is
+ * allocated by the first call (B x N x (d + m S) fp32 and the small inputs).
+ * boute_engine_sync: waits for every step issued on `stream` and returns the
+ * fit status or the first device error.
  * On a non-default stream the step is captured once per argument set (device
  * or host buffers) into a CUDA graph and replayed afterwards; a first call
  * with new pointers therefore must not itself run inside a stream capture. */
@@ -211,6 +220,11 @@ int boute_engine_step_host(boute_engine *e, const double *X, const double *Y,
                            const double *lengthscale, const double *outputscale,
                            const double *noise, const double *ref, const float *Xc,
                            const float *eps, long long *idx, float *val, void *stream);
+int boute_engine_step_host_async(boute_engine *e, const double *X, const double *Y,
+                                 const double *lengthscale, const double *outputscale,
+                                 const double *noise, const double *ref, const float *Xc,
+                                 const float *eps, long long *idx, float *val, void *stream);
+int boute_engine_sync(boute_engine *e, void *stream);
 /* Copies the last step's per-candidate results into caller buffers (device
  * pointers; any may be NULL): acq B x N, mean and var B x m x N (fp32). */
 int boute_engine_scores(const boute_engine *e, float *acq, float *mean, float *var, void *stream);

@@ -25,7 +25,8 @@ SYMBOLS = (
     "boute_pareto_front", "boute_box_decompose", "boute_acq_ehvi", "boute_acq_mc_hvi",
     "boute_select_topk", "boute_select_topk_noalloc", "boute_engine_create", "boute_engine_step",
     "boute_engine_step_async",
-    "boute_engine_step_host", "boute_engine_scores", "boute_engine_set_timing",
+    "boute_engine_step_host", "boute_engine_step_host_async", "boute_engine_sync",
+    "boute_engine_scores", "boute_engine_set_timing",
     "boute_engine_stage_times", "boute_engine_launches_per_step", "boute_engine_free",
 )
 #: stage names of boute_engine_stage_times, in order
@@ -76,6 +77,8 @@ def load(path: str | None = None):
         "boute_engine_step": ([_vp] * 11 + [_vp], _i),
         "boute_engine_step_async": ([_vp] * 11 + [_vp], _i),
         "boute_engine_step_host": ([_vp] * 11 + [_vp], _i),
+        "boute_engine_step_host_async": ([_vp] * 11 + [_vp], _i),
+        "boute_engine_sync": ([_vp, _vp], _i),
         "boute_engine_scores": ([_vp, _vp, _vp, _vp, _vp], _i),
         "boute_engine_set_timing": ([_vp, _i], _i),
         "boute_engine_stage_times": ([_vp, ctypes.POINTER(ctypes.c_float), _i], _i),
@@ -271,6 +274,20 @@ def boute_engine_step_host(e: Engine, X, Y, ls, s2, noise, ref, Xc, eps, idx, va
     """HOST (CPU, ideally pinned) tensors in and out; copies inside the call."""
     _check(load().boute_engine_step_host(e.handle, *_engine_args(
         X, Y, ls, s2, noise, ref, Xc, eps, idx, val, False), _s(stream)), "boute_engine_step_host")
+
+
+def boute_engine_step_host_async(e: Engine, X, Y, ls, s2, noise, ref, Xc, eps, idx, val,
+                                 stream=None):
+    """As boute_engine_step_host without the final synchronisation; the host
+    tensors must stay as they are (inputs) and unread (idx, val) until
+    boute_engine_sync."""
+    _check(load().boute_engine_step_host_async(e.handle, *_engine_args(
+        X, Y, ls, s2, noise, ref, Xc, eps, idx, val, False), _s(stream)),
+        "boute_engine_step_host_async")
+
+
+def boute_engine_sync(e: Engine, stream=None):
+    _check(load().boute_engine_sync(e.handle, _s(stream)), "boute_engine_sync")
 
 
 def boute_engine_scores(e: Engine, acq=None, mean=None, var=None, stream=None):

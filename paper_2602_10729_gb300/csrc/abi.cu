@@ -95,7 +95,7 @@ struct boute_engine {
     const void *key[12];
     cudaGraphExec_t exec;
     int launches;
-  } graphs[2];
+  } graphs[3];
   int graph_next, graphs_off;
   // the front stage (standardise, Pareto front, boxes) depends on the raw
   // outcomes only: it runs on a second stream, forked after the fit's set-up
@@ -107,6 +107,15 @@ struct boute_engine {
   // them (posterior, acquisition)
   cudaStream_t cpy[2];
   cudaEvent_t ev_in, ev_xc, ev_eps[2];
+  // pipelined host-input steps: a second set of device input buffers (the
+  // first is X .. eps above, allocated on first use) so that one step's copies
+  // overlap the previous step's computation; in_free[s] marks the end of the
+  // last step that read set s
+  double *X1, *Y1, *ls1, *s21, *noise1, *ref1;
+  float *Xc1, *eps1;
+  cudaEvent_t ev_xc1, ev_eps1[2], in_free[2];
+  cudaEvent_t ev_small[2];  // the small inputs of set 0 / 1 are in place
+  int host_set;
 };
 
 // Stage order of one step as timed (with timing on, the front stage runs
@@ -268,14 +277,17 @@ void boute_engine_free(boute_engine *e) {
     if (g.exec) cudaGraphExecDestroy(g.exec);
   if (e->join) cudaEventDestroy(e->join);
   if (e->side) cudaStreamDestroy(e->side);
-  for (cudaEvent_t ev : {e->ev_in, e->ev_xc, e->ev_eps[0], e->ev_eps[1], e->ev_setup, e->join2})
+  for (cudaEvent_t ev : {e->ev_in, e->ev_xc, e->ev_eps[0], e->ev_eps[1], e->ev_setup, e->join2,
+                         e->ev_xc1, e->ev_eps1[0], e->ev_eps1[1], e->in_free[0], e->in_free[1],
+                         e->ev_small[0], e->ev_small[1]})
     if (ev) cudaEventDestroy(ev);
   if (e->side2) cudaStreamDestroy(e->side2);
   for (cudaStream_t c : e->cpy)
     if (c) cudaStreamDestroy(c);
   void *ptrs[] = {e->X, e->Y, e->Ys, e->ls, e->s2, e->noise, e->ref, e->front, e->mask, e->P,
                   e->K, e->lower, e->upper, e->Xc, e->eps, e->mean, e->var, e->acq, e->val,
-                  e->idx, e->scratch, e->sel, e->kst};
+                  e->idx, e->scratch, e->sel, e->kst, e->X1, e->Y1, e->ls1, e->s21,
+                  e->noise1, e->ref1, e->Xc1, e->eps1};
   for (void *p : ptrs) cudaFree(p);
   delete e;
 }
@@ -356,7 +368,14 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
        cudaEventCreateWithFlags(&e->ev_in, cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->ev_xc, cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->ev_eps[0], cudaEventDisableTiming) != cudaSuccess ||
-       cudaEventCreateWithFlags(&e->ev_eps[1], cudaEventDisableTiming) != cudaSuccess)) {
+       cudaEventCreateWithFlags(&e->ev_eps[1], cudaEventDisableTiming) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->ev_xc1, cudaEventDisableTiming) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->ev_eps1[0], cudaEventDisableTiming) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->ev_eps1[1], cudaEventDisableTiming) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->in_free[0], cudaEventDisableTiming) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->in_free[1], cudaEventDisableTiming) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->ev_small[0], cudaEventDisableTiming) != cudaSuccess ||
+       cudaEventCreateWithFlags(&e->ev_small[1], cudaEventDisableTiming) != cudaSuccess)) {
     cudaGetLastError();
     r = BOUTE_ERR_CUDA;
   }
@@ -397,6 +416,11 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
   if (host && cudaStreamIsCapturing(s, &cap) != cudaSuccess) return last_launch_status();
   const unsigned wait_flags =
       cap == cudaStreamCaptureStatusActive ? cudaEventWaitExternal : cudaEventWaitDefault;
+  // host inputs: the copy events of input set host - 1
+  const cudaEvent_t ev_xc = host == 2 ? e->ev_xc1 : e->ev_xc;
+  const cudaEvent_t *ev_eps = host == 2 ? e->ev_eps1 : e->ev_eps;
+  if (host && cudaStreamWaitEvent(s, e->ev_small[host - 1], wait_flags) != cudaSuccess)
+    return last_launch_status();
   // K* beside the fit (not in stage-timing mode, where the posterior builds it)
   const float *kst = e->timing ? nullptr : e->kst;
   // The graph has one root, the fit's set-up: the front stage (which needs
@@ -411,7 +435,7 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
   }
   if (kst) {
     if (cudaStreamWaitEvent(e->side2, e->ev_setup, 0) != cudaSuccess ||
-        (host && cudaStreamWaitEvent(e->side2, e->ev_xc, wait_flags) != cudaSuccess))
+        (host && cudaStreamWaitEvent(e->side2, ev_xc, wait_flags) != cudaSuccess))
       return last_launch_status();
     if ((r = launch_kstar(&e->gp->g, Xc, e->N, e->kst, e->side2))) return r;
     if (cudaEventRecord(e->join2, e->side2) != cudaSuccess) return last_launch_status();
@@ -419,15 +443,15 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
   mark(ST_FRONT);
   if (e->timing && (r = front(s))) return r;
   mark(ST_POSTERIOR);
-  if (host && cudaStreamWaitEvent(s, e->ev_xc, wait_flags) != cudaSuccess)
+  if (host && cudaStreamWaitEvent(s, ev_xc, wait_flags) != cudaSuccess)
     return last_launch_status();
   if (kst && cudaStreamWaitEvent(s, e->join2, 0) != cudaSuccess) return last_launch_status();
   if ((r = launch_posterior(&e->gp->g, Xc, e->N, e->mean, e->var, s, kst))) return r;
   if (!e->timing && cudaStreamWaitEvent(s, e->join, 0) != cudaSuccess)  // join
     return last_launch_status();
   if (host && mc)
-    for (cudaEvent_t ev : e->ev_eps)
-      if (cudaStreamWaitEvent(s, ev, wait_flags) != cudaSuccess)
+    for (int i = 0; i < 2; ++i)
+      if (cudaStreamWaitEvent(s, ev_eps[i], wait_flags) != cudaSuccess)
         return last_launch_status();
   mark(ST_ACQ);
   if (e->fuse_sel && !e->timing) {
@@ -476,7 +500,7 @@ static int engine_launch(boute_engine *e, const double *X, const double *Y, cons
     }
   }
   auto &g = e->graphs[e->graph_next];
-  e->graph_next ^= 1;
+  e->graph_next = (e->graph_next + 1) % 3;
   if (g.exec) {
     cudaGraphExecDestroy(g.exec);
     g.exec = nullptr;
@@ -522,14 +546,73 @@ int boute_engine_step_async(boute_engine *e, const double *X, const double *Y,
                        (cudaStream_t)stream);
 }
 
+// After a failed step the cross-block counters of the kernels that select as
+// blocks finish may be left part-way: set them back to zero.
+static void engine_reset_counters(boute_engine *e) {
+  cudaDeviceSynchronize();
+  cudaGetLastError();
+  if (e->sel) cudaMemset(e->sel, 0, mchvi2_select_scratch_bytes(e->B, e->N, 2 * e->n + 2));
+  cudaMemset(e->scratch, 0, topk_scratch_bytes(e->B, e->N, e->k));
+  cudaGetLastError();
+}
+
 int boute_engine_step(boute_engine *e, const double *X, const double *Y,
                       const double *lengthscale, const double *outputscale, const double *noise,
                       const double *ref, const float *Xc, const float *eps, long long *idx,
                       float *val, void *stream) {
   int r = boute_engine_step_async(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx,
                                   val, stream);
+  if (!r) r = boute_gp_status(e->gp, stream);
+  if (r && e) engine_reset_counters(e);
+  return r;
+}
+
+// Copies a host-input step's inputs into device input set `set` and runs the
+// step on `s`, its results copied back into idx / val (host); nothing waits.
+// The inputs go on the two copy streams, after the last step that read this
+// set (in_free), so that they overlap the previous step's computation: the
+// small ones first, then the candidates, then the base normals in halves;
+// the step waits for each only where it needs it (fit, posterior,
+// acquisition).
+static int engine_host_step(boute_engine *e, int set, const double *X, const double *Y,
+                            const double *lengthscale, const double *outputscale,
+                            const double *noise, const double *ref, const float *Xc,
+                            const float *eps, long long *idx, float *val, cudaStream_t s) {
+  const size_t B = e->B, n = e->n, d = e->d, m = e->m, N = e->N, S = e->S, k = e->k;
+  double *dX = set ? e->X1 : e->X, *dY = set ? e->Y1 : e->Y, *dls = set ? e->ls1 : e->ls;
+  double *ds2 = set ? e->s21 : e->s2, *dnz = set ? e->noise1 : e->noise;
+  double *dref = set ? e->ref1 : e->ref;
+  float *dXc = set ? e->Xc1 : e->Xc, *deps = set ? e->eps1 : e->eps;
+  const cudaEvent_t ev_xc = set ? e->ev_xc1 : e->ev_xc;
+  const cudaEvent_t *ev_eps = set ? e->ev_eps1 : e->ev_eps;
+  for (cudaStream_t c : e->cpy) cudaStreamWaitEvent(c, e->in_free[set], 0);
+  // the small inputs first, so that the step's fit never waits behind the
+  // previous copies of the normals on the copy engine
+  cudaStream_t c0 = e->cpy[0];
+  cudaMemcpyAsync(dX, X, B * n * d * sizeof(double), cudaMemcpyHostToDevice, c0);
+  cudaMemcpyAsync(dY, Y, B * n * m * sizeof(double), cudaMemcpyHostToDevice, c0);
+  cudaMemcpyAsync(dls, lengthscale, B * m * d * sizeof(double), cudaMemcpyHostToDevice, c0);
+  cudaMemcpyAsync(ds2, outputscale, B * m * sizeof(double), cudaMemcpyHostToDevice, c0);
+  cudaMemcpyAsync(dnz, noise, B * m * sizeof(double), cudaMemcpyHostToDevice, c0);
+  cudaMemcpyAsync(dref, ref, B * m * sizeof(double), cudaMemcpyHostToDevice, c0);
+  cudaEventRecord(e->ev_small[set], c0);
+  cudaMemcpyAsync(dXc, Xc, B * N * d * sizeof(float), cudaMemcpyHostToDevice, c0);
+  cudaEventRecord(ev_xc, e->cpy[0]);
+  const size_t eps_n = e->mode == BOUTE_ACQ_MC_HVI ? B * N * m * S : 0, half = eps_n / 2;
+  for (int i = 0; i < 2; ++i) {  // the normals in two halves, one per copy stream
+    const size_t off = i ? half : 0, cnt = i ? eps_n - half : half;
+    if (cnt)
+      cudaMemcpyAsync(deps + off, eps + off, cnt * sizeof(float), cudaMemcpyHostToDevice,
+                      e->cpy[i]);
+    cudaEventRecord(ev_eps[i], e->cpy[i]);
+  }
+  if (int r = last_launch_status()) return r;
+  int r = engine_launch(e, dX, dY, dls, ds2, dnz, dref, dXc, deps, e->idx, e->val, s, 1 + set);
   if (r) return r;
-  return boute_gp_status(e->gp, stream);
+  cudaEventRecord(e->in_free[set], s);  // this step has read set `set`
+  cudaMemcpyAsync(idx, e->idx, B * k * sizeof(long long), cudaMemcpyDeviceToHost, s);
+  cudaMemcpyAsync(val, e->val, B * k * sizeof(float), cudaMemcpyDeviceToHost, s);
+  return last_launch_status();
 }
 
 int boute_engine_step_host(boute_engine *e, const double *X, const double *Y,
@@ -538,37 +621,38 @@ int boute_engine_step_host(boute_engine *e, const double *X, const double *Y,
                            const float *eps, long long *idx, float *val, void *stream) {
   if (!engine_args_ok(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val))
     return BOUTE_ERR_INVALID_ARG;
-  cudaStream_t s = (cudaStream_t)stream;
-  const size_t B = e->B, n = e->n, d = e->d, m = e->m, N = e->N, S = e->S, k = e->k;
-  cudaMemcpyAsync(e->X, X, B * n * d * sizeof(double), cudaMemcpyHostToDevice, s);
-  cudaMemcpyAsync(e->Y, Y, B * n * m * sizeof(double), cudaMemcpyHostToDevice, s);
-  cudaMemcpyAsync(e->ls, lengthscale, B * m * d * sizeof(double), cudaMemcpyHostToDevice, s);
-  cudaMemcpyAsync(e->s2, outputscale, B * m * sizeof(double), cudaMemcpyHostToDevice, s);
-  cudaMemcpyAsync(e->noise, noise, B * m * sizeof(double), cudaMemcpyHostToDevice, s);
-  cudaMemcpyAsync(e->ref, ref, B * m * sizeof(double), cudaMemcpyHostToDevice, s);
-  // candidates and normals on the copy streams, ordered after everything
-  // already on `stream` (the previous step still reads these buffers), and
-  // overlapping the fit; the normals in two halves, one per copy engine
-  cudaEventRecord(e->ev_in, s);
-  for (cudaStream_t c : e->cpy) cudaStreamWaitEvent(c, e->ev_in, 0);
-  cudaMemcpyAsync(e->Xc, Xc, B * N * d * sizeof(float), cudaMemcpyHostToDevice, e->cpy[0]);
-  cudaEventRecord(e->ev_xc, e->cpy[0]);
-  const size_t eps_n = e->mode == BOUTE_ACQ_MC_HVI ? B * N * m * S : 0, half = eps_n / 2;
-  for (int i = 0; i < 2; ++i) {
-    const size_t off = i ? half : 0, cnt = i ? eps_n - half : half;
-    if (cnt)
-      cudaMemcpyAsync(e->eps + off, eps + off, cnt * sizeof(float), cudaMemcpyHostToDevice,
-                      e->cpy[i]);
-    cudaEventRecord(e->ev_eps[i], e->cpy[i]);
+  int r = engine_host_step(e, 0, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val,
+                           (cudaStream_t)stream);
+  if (!r) r = boute_gp_status(e->gp, stream);
+  if (r) engine_reset_counters(e);
+  return r;
+}
+
+int boute_engine_step_host_async(boute_engine *e, const double *X, const double *Y,
+                                 const double *lengthscale, const double *outputscale,
+                                 const double *noise, const double *ref, const float *Xc,
+                                 const float *eps, long long *idx, float *val, void *stream) {
+  if (!engine_args_ok(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val))
+    return BOUTE_ERR_INVALID_ARG;
+  if (!e->X1) {  // the second input set, on first use
+    const size_t Bn = (size_t)e->B * e->n, BN = (size_t)e->B * e->N, Bm = (size_t)e->B * e->m;
+    int r = dalloc(&e->X1, Bn * e->d) | dalloc(&e->Y1, Bn * e->m) |
+            dalloc(&e->ls1, Bm * e->d) | dalloc(&e->s21, Bm) | dalloc(&e->noise1, Bm) |
+            dalloc(&e->ref1, Bm) | dalloc(&e->Xc1, BN * e->d);
+    if (e->mode == BOUTE_ACQ_MC_HVI) r |= dalloc(&e->eps1, BN * e->m * e->S);
+    if (r) return BOUTE_ERR_OOM;
   }
-  if (int r = last_launch_status()) return r;
-  int r = engine_launch(e, e->X, e->Y, e->ls, e->s2, e->noise, e->ref, e->Xc, e->eps, e->idx,
-                        e->val, s, 1);
-  if (r) return r;
-  cudaMemcpyAsync(idx, e->idx, B * k * sizeof(long long), cudaMemcpyDeviceToHost, s);
-  cudaMemcpyAsync(val, e->val, B * k * sizeof(float), cudaMemcpyDeviceToHost, s);
-  if (int r2 = last_launch_status()) return r2;
-  return boute_gp_status(e->gp, stream);
+  const int set = e->host_set;
+  e->host_set ^= 1;
+  return engine_host_step(e, set, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val,
+                          (cudaStream_t)stream);
+}
+
+int boute_engine_sync(boute_engine *e, void *stream) {
+  if (!e) return BOUTE_ERR_INVALID_ARG;
+  const int r = boute_gp_status(e->gp, stream);
+  if (r) engine_reset_counters(e);
+  return r;
 }
 
 int boute_engine_scores(const boute_engine *e, float *acq, float *mean, float *var,

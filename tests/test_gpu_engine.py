@@ -181,3 +181,32 @@ def test_posterior_from_precomputed_kstar_matches_fused(wi, n, N, B):
     e.free()
     for a, b in zip(*out):
         assert np.array_equal(a, b)
+
+
+# Pipelined host-input steps: consecutive calls alternate between two device
+# input sets and overlap one step's copies with the previous step's
+# computation; each step's results must equal the device-input step's.
+@pytest.mark.parametrize("wi,N,B", [(1, 2000 + 7, 1), (4, 1500 + 1, 3)])
+def test_pipelined_host_steps_match_device_steps(wi, N, B):
+    import torch
+
+    from paper_2602_10729_gb300 import boute as bt
+    w = wl.scaled(wl.WORKLOADS[wi], N=N, B=B)
+    hp1 = host_problem(w)
+    hp2 = host_problem(wl.scaled(w, N=w.N), threads=4)
+    rng = np.random.default_rng(11)
+    hp2.Xc[:] = rng.random(hp2.Xc.shape).astype(np.float32)
+    if hp2.eps is not None:
+        hp2.eps[:] = rng.standard_normal(hp2.eps.shape).astype(np.float32)
+    e = _engine(w)
+    want = [_run(e, w, _dev(h), "device") for h in (hp1, hp2)]
+    inputs = [_host(h) for h in (hp1, hp2, hp1, hp2, hp1)]
+    outs = [(torch.empty((w.B, w.k), dtype=torch.int64).pin_memory(),
+             torch.empty((w.B, w.k), dtype=torch.float32).pin_memory()) for _ in inputs]
+    for inp, (i, v) in zip(inputs, outs):
+        bt.boute_engine_step_host_async(e, *inp, i, v)
+    bt.boute_engine_sync(e)
+    e.free()
+    for (i, v), (wi_, wv) in zip(outs, want + want + want[:1]):
+        assert np.array_equal(i.numpy(), wi_)
+        assert np.array_equal(v.numpy(), wv)
