@@ -59,11 +59,12 @@ def lib():
         L.bo_hv.restype = ctypes.c_double
         L.bo_hvi.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp, _dp]
         L.bo_hvi.restype = ctypes.c_double
-        L.bo_ehvi2d.argtypes = [_dp, _dp, ctypes.c_longlong, _dp, ctypes.c_int, _dp, _dp,
+        L.bo_ehvi2d.argtypes = [_dp, _dp, ctypes.c_longlong, _dp, ctypes.c_int, _dp, _dp, _dp,
                                 ctypes.c_int]
         L.bo_ehvi2d.restype = None
         L.bo_mc_hvi.argtypes = [_dp, _dp, ctypes.c_longlong, ctypes.c_int, _fp, ctypes.c_int,
-                                ctypes.c_longlong, _dp, ctypes.c_int, _dp, _dp, ctypes.c_int]
+                                ctypes.c_longlong, _dp, ctypes.c_int, _dp, _dp, _dp,
+                                ctypes.c_int]
         L.bo_mc_hvi.restype = None
         L.bo_topk.argtypes = [_dp, ctypes.c_longlong, ctypes.c_int, _lp, _dp]
         L.bo_topk.restype = None
@@ -164,20 +165,31 @@ def hvi(F, ref, y) -> float:
     return float(lib().bo_hvi(pF, F.shape[0], F.shape[1], pr, py))
 
 
-def ehvi2d(mean, var, F, ref, threads: int = 0):
-    """mean, var: N x 2; F: P x 2 sorted by f1 ascending."""
+def _cons(cons):
+    """Constraint thresholds (one per objective) or None."""
+    if cons is None:
+        return None, None
+    c, pc = _d(cons)
+    return c, pc
+
+
+def ehvi2d(mean, var, F, ref, threads: int = 0, cons=None):
+    """mean, var: N x 2; F: P x 2 sorted by f1 ascending; cons: 2 thresholds
+    on the minimised objectives (feasibility indicator) or None."""
     mean, pm = _d(mean)
     var, pv = _d(var)
     F, pF = _d(np.asarray(F, dtype=np.float64).reshape(-1, 2))
     ref, pr = _d(ref)
+    c, pc = _cons(cons)
     N = mean.shape[0]
     acq = np.empty(N)
-    lib().bo_ehvi2d(pm, pv, N, pF, F.shape[0], pr, acq.ctypes.data_as(_dp), threads)
+    lib().bo_ehvi2d(pm, pv, N, pF, F.shape[0], pr, pc, acq.ctypes.data_as(_dp), threads)
     return acq
 
 
-def mc_hvi(mean, var, eps, F, ref, eps_stride: int | None = None, threads: int = 0):
-    """mean, var: N x m; eps: float32 (N, m, S) (or (1, m, S) with eps_stride=0)."""
+def mc_hvi(mean, var, eps, F, ref, eps_stride: int | None = None, threads: int = 0, cons=None):
+    """mean, var: N x m; eps: float32 (N, m, S) (or (1, m, S) with eps_stride=0);
+    cons: m thresholds on the minimised objectives (feasibility indicator) or None."""
     mean, pm = _d(mean)
     var, pv = _d(var)
     eps, pe = _f(eps)
@@ -186,10 +198,11 @@ def mc_hvi(mean, var, eps, F, ref, eps_stride: int | None = None, threads: int =
     stride = m * S if eps_stride is None else eps_stride
     F, pF = _d(np.asarray(F, dtype=np.float64).reshape(-1, m))
     ref, pr = _d(ref)
+    c, pc = _cons(cons)
     N = mean.shape[0]
     acq = np.empty(N)
-    lib().bo_mc_hvi(pm, pv, N, m, pe, S, stride, pF, F.shape[0], pr, acq.ctypes.data_as(_dp),
-                    threads)
+    lib().bo_mc_hvi(pm, pv, N, m, pe, S, stride, pF, F.shape[0], pr, pc,
+                    acq.ctypes.data_as(_dp), threads)
     return acq
 
 

@@ -266,20 +266,38 @@ static double psi(double c, double mu, double sigma) {
   return (c - mu) * std_cdf(z) + sigma * std_pdf(z);
 }
 
+/* Constrained (Sec. 5.2 "Constrained qNEHVI", feasibility g_t = Y_t - c_t <= 0
+ * on the minimised objectives): psi_c(v) = E[(v - Y)_+ 1[Y <= c]]. Since
+ * (v - Y)_+ 1[Y <= c] = (v - Y) 1[Y <= w] with w = min(v, c),
+ * psi_c(v) = (v - mu) Phi(z) + sigma phi(z), z = (w - mu) / sigma;
+ * c = +infinity gives psi(v). */
+static double psi_c(double v, double cons, double mu, double sigma) {
+  if (isinf(v) && v < 0) return 0.0;
+  double w = v < cons ? v : cons;
+  if (!(sigma > 0.0)) return mu <= w ? v - mu : 0.0;
+  double z = (w - mu) / sigma;
+  return (v - mu) * std_cdf(z) + sigma * std_pdf(z);
+}
+
 void bo_ehvi2d(const double *mean, const double *var, long long N, const double *F,
-               int P, const double *ref, double *acq, int nthreads) {
+               int P, const double *ref, const double *cons, double *acq, int nthreads) {
   int nt = nthreads_or_default(nthreads);
+  const double c1 = cons ? cons[0] : INFINITY, c2 = cons ? cons[1] : INFINITY;
 #pragma omp parallel for schedule(static) num_threads(nt)
   for (long long c = 0; c < N; ++c) {
     double mu1 = mean[2 * c], mu2 = mean[2 * c + 1];
     double sg1 = sqrt(var[2 * c]), sg2 = sqrt(var[2 * c + 1]);
     double e = 0.0;
     for (int i = 0; i <= P; ++i) {
-      /* cell i: f1 in [a_i, b_i), f2 below u_i */
+      /* cell i: f1 in [a_i, b_i), f2 below u_i; with independent objectives
+       * E[HVI 1[Y <= c]] factors per cell into the two objectives' terms */
       double a = i == 0 ? -INFINITY : F[2 * (i - 1)];
       double b = i == P ? ref[0] : F[2 * i];
       double u = i == 0 ? ref[1] : F[2 * (i - 1) + 1];
-      e += (psi(b, mu1, sg1) - psi(a, mu1, sg1)) * psi(u, mu2, sg2);
+      if (cons)
+        e += (psi_c(b, c1, mu1, sg1) - psi_c(a, c1, mu1, sg1)) * psi_c(u, c2, mu2, sg2);
+      else
+        e += (psi(b, mu1, sg1) - psi(a, mu1, sg1)) * psi(u, mu2, sg2);
     }
     acq[c] = e;
   }
@@ -288,7 +306,7 @@ void bo_ehvi2d(const double *mean, const double *var, long long N, const double 
 /* ---- Monte-Carlo HVI ------------------------------------------------------ */
 void bo_mc_hvi(const double *mean, const double *var, long long N, int m,
                const float *eps, int S, long long eps_stride, const double *F,
-               int P, const double *ref, double *acq, int nthreads) {
+               int P, const double *ref, const double *cons, double *acq, int nthreads) {
   int nt = nthreads_or_default(nthreads);
   double hvF = bo_hv(F, P, m, ref, NULL);
   long long scr = bo_hv_scratch_size(P + 1, m);
@@ -302,10 +320,13 @@ void bo_mc_hvi(const double *mean, const double *var, long long N, int m,
       for (int t = 0; t < m; ++t) sg[t] = sqrt(var[c * m + t]);
       double sum = 0.0;
       for (int s = 0; s < S; ++s) {
-        for (int t = 0; t < m; ++t)
+        int feasible = 1;
+        for (int t = 0; t < m; ++t) {
           all[(long)P * m + t] =
               mean[c * m + t] + sg[t] * (double)eps[c * eps_stride + (long long)t * S + s];
-        sum += bo_hv(all, P + 1, m, ref, scratch) - hvF;
+          if (cons && !(all[(long)P * m + t] <= cons[t])) feasible = 0;
+        }
+        if (feasible) sum += bo_hv(all, P + 1, m, ref, scratch) - hvF;  /* else HVI x 0 */
       }
       acq[c] = sum / S;
     }

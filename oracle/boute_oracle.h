@@ -67,17 +67,22 @@ double bo_hvi(const double *F, int P, int m, const double *ref, const double *y)
  * in closed form over the P+1 cells of the sorted 2-D front):
  * EHVI = sum_i [psi1(b_i) - psi1(a_i)] psi2(u_i),
  * psi(c) = E[(c - Y)_+] = (c - mu) Phi(z) + sigma phi(z), z = (c - mu)/sigma.
+ * cons (2 thresholds on the minimised objectives, or NULL): the feasibility
+ * indicator 1[Y_1 <= c_1, Y_2 <= c_2] inside the expectation, which turns psi
+ * into psi_c(v) = E[(v - Y)_+ 1[Y <= c]].
  * mean, var: N x 2; F: P x 2 sorted by f1 ascending; acq: N. */
 void bo_ehvi2d(const double *mean, const double *var, long long N, const double *F,
-               int P, const double *ref, double *acq, int nthreads);
+               int P, const double *ref, const double *cons, double *acq, int nthreads);
 
 /* Monte-Carlo hypervolume improvement (Sec. 5.2: expectation of HVI over
  * posterior samples, by Monte-Carlo integration): sample s of candidate c is
  * y_t = mean_t + sqrt(var_t) eps[c*eps_stride + t*S + s]; acq = mean over the
- * S samples of HV(F u {y}) - HV(F). mean, var: N x m; eps: float. */
+ * S samples of HV(F u {y}) - HV(F), each multiplied by the feasibility
+ * indicator 1[y_t <= cons_t for every t] when cons (m thresholds) is given.
+ * mean, var: N x m; eps: float. */
 void bo_mc_hvi(const double *mean, const double *var, long long N, int m,
                const float *eps, int S, long long eps_stride, const double *F,
-               int P, const double *ref, double *acq, int nthreads);
+               int P, const double *ref, const double *cons, double *acq, int nthreads);
 
 /* Top-k selection (Sec. 5.2 step (ii): the next configuration is the best
  * scored candidate): the first k entries of the order (value descending, NaN

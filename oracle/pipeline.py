@@ -54,11 +54,13 @@ def posterior(fp: FittedProblem, Xc, threads: int = 0):
     return mean, var
 
 
-def acquisition(fp: FittedProblem, mean, var, mode: str, eps=None, threads: int = 0):
+def acquisition(fp: FittedProblem, mean, var, mode: str, eps=None, threads: int = 0,
+                cons=None):
+    """cons: per-objective feasibility thresholds (standardised units) or None."""
     if mode == "ehvi":
-        return ehvi2d(mean, var, fp.front, fp.ref, threads)
+        return ehvi2d(mean, var, fp.front, fp.ref, threads, cons=cons)
     if mode == "mc":
-        return mc_hvi(mean, var, eps, fp.front, fp.ref, threads=threads)
+        return mc_hvi(mean, var, eps, fp.front, fp.ref, threads=threads, cons=cons)
     raise ValueError(mode)
 
 

@@ -416,3 +416,126 @@ def test_pipeline_config0_end_to_end_shapes_and_topk_consistency():
     assert mean.shape == (w.N, 2) and acq.shape == (w.N,) and idx.shape == (w.k,)
     assert np.all(acq >= 0) and np.all(np.diff(val) <= 0)
     assert fp.front.shape[0] == int(fp.mask.sum())
+
+
+# ------------------------------------------------------------ constrained acquisition
+# Sec. 5.2 "Constrained qNEHVI": the expectation of HVI times the feasibility
+# indicator 1[g_t <= 0], g_t = Y_t - c_t on the minimised objectives.
+def test_constraints_at_infinity_change_nothing():
+    F = _front2d(61, 6)
+    ref = np.array([1.1, 1.1])
+    rng = np.random.default_rng(62)
+    mu = rng.uniform(-2, 2, (50, 2))
+    var = rng.uniform(0, 1, (50, 2))
+    inf = np.array([np.inf, np.inf])
+    np.testing.assert_array_equal(oracle.ehvi2d(mu, var, F, ref, cons=inf),
+                                  oracle.ehvi2d(mu, var, F, ref))
+    eps = rng.standard_normal((50, 2, 32)).astype(np.float32)
+    np.testing.assert_array_equal(oracle.mc_hvi(mu, var, eps, F, ref, cons=inf),
+                                  oracle.mc_hvi(mu, var, eps, F, ref))
+
+
+def test_constrained_ehvi_empty_front_by_quadrature():
+    ref = np.array([1.1, 1.1])
+    mean = np.array([[0.3, 1.5], [-2.0, 0.9], [0.0, 0.0]])
+    var = np.array([[0.49, 0.25], [1.7, 0.01], [0.3, 0.2]])
+    cons = np.array([0.4, 2.0])  # the first cuts below r1, the second is above r2
+
+    def e_pos(r, c, mu, s):  # E[(r - Y)_+ 1[Y <= c]] by quadrature over y <= min(r, c)
+        f = lambda y: (r - y) * math.exp(-0.5 * ((y - mu) / s) ** 2) / (s * math.sqrt(2 * math.pi))
+        return scipy.integrate.quad(f, mu - 40 * s, min(r, c), epsabs=1e-14, epsrel=1e-12,
+                                    limit=200)[0]
+
+    got = oracle.ehvi2d(mean, var, np.zeros((0, 2)), ref, cons=cons)
+    for c in range(3):
+        want = (e_pos(ref[0], cons[0], mean[c, 0], math.sqrt(var[c, 0])) *
+                e_pos(ref[1], cons[1], mean[c, 1], math.sqrt(var[c, 1])))
+        assert got[c] == pytest.approx(want, rel=1e-9, abs=1e-300)
+
+
+@pytest.mark.parametrize("case", range(3))
+def test_constrained_ehvi_matches_brute_force_monte_carlo(case):
+    """1e6 samples per candidate with the feasibility indicator applied."""
+    F = _front2d(71 + case, 6)
+    ref = np.array([1.1, 1.1])
+    rng = np.random.default_rng(170 + case)
+    mu = F.min(0) + rng.uniform(-0.6, 0.3, 2)
+    sd = rng.uniform(0.08, 0.2, 2)
+    cons = mu + sd * rng.uniform(-0.3, 0.8, 2)  # cuts inside each objective's spread
+    got = oracle.ehvi2d(mu[None], (sd ** 2)[None], F, ref, cons=cons)[0]
+    cuts = np.concatenate([F[:, 0], [ref[0]]])
+    lefts = np.concatenate([[-np.inf], F[:, 0]])
+    heights = np.concatenate([[ref[1]], F[:, 1]])
+    sums = []
+    for _ in range(8):  # 8 x 5e5 antithetic pairs
+        Z = rng.standard_normal((500_000, 2))
+        pair = []
+        for Ysmp in (mu + sd * Z, mu - sd * Z):
+            w = np.clip(cuts[None, :] - np.maximum(lefts[None, :], Ysmp[:, :1]), 0, None)
+            h = np.clip(heights[None, :] - Ysmp[:, 1:], 0, None)
+            pair.append((w * h).sum(1) * np.all(Ysmp <= cons, axis=1))
+        sums.append(0.5 * (pair[0] + pair[1]))
+    mc = np.concatenate(sums)
+    se = mc.std() / math.sqrt(mc.size)
+    assert se < 1e-3 * got  # resolves errors of a few tenths of a percent
+    assert abs(got - mc.mean()) < 4 * se
+
+
+def test_constrained_ehvi_by_2d_quadrature_against_exact_hvi():
+    F = _front2d(81, 4)
+    ref = np.array([1.1, 1.1])
+    mu, sd = np.array([0.0, -0.2]), np.array([0.4, 0.3])
+    cons = np.array([0.1, -0.1])
+    got = oracle.ehvi2d(mu[None], (sd ** 2)[None], F, ref, cons=cons)[0]
+    pdf = lambda y, m, s: math.exp(-0.5 * ((y - m) / s) ** 2) / (s * math.sqrt(2 * math.pi))
+    breaks = sorted(set(F[:, 0].tolist() + [ref[0], cons[0]]))
+    tot = 0.0
+    lo = mu[0] - 9 * sd[0]
+    for a, b in zip([lo] + breaks[:-1], breaks):
+        if b <= lo or a >= cons[0]:
+            continue
+        tot += scipy.integrate.dblquad(
+            lambda y2, y1: oracle.hvi(F, ref, np.array([y1, y2])) * pdf(y1, mu[0], sd[0]) *
+            pdf(y2, mu[1], sd[1]), max(a, lo), min(b, cons[0]), mu[1] - 9 * sd[1],
+            min(ref[1], cons[1]), epsabs=1e-10, epsrel=1e-8)[0]
+    assert got == pytest.approx(tot, rel=1e-5)
+
+
+@pytest.mark.parametrize("m", [2, 3])
+def test_constrained_mc_hvi_is_the_sample_mean_of_feasible_hvi(m):
+    rng = np.random.default_rng(90 + m)
+    ref = np.full(m, 1.1)
+    Yobs = rng.normal(size=(60, m))
+    mask, order = oracle.pareto_front(Yobs, ref)
+    F = Yobs[order]
+    N, S = 7, 16
+    mean = rng.normal(size=(N, m))
+    var = rng.uniform(0, 0.5, (N, m))
+    eps = rng.standard_normal((N, m, S)).astype(np.float32)
+    cons = rng.uniform(-0.5, 0.8, m)
+    got = oracle.mc_hvi(mean, var, eps, F, ref, cons=cons)
+    for c in range(N):
+        ys = mean[c][:, None] + np.sqrt(var[c])[:, None] * eps[c].astype(np.float64)
+        vals = []
+        for s in range(S):
+            y = ys[:, s]
+            hv = _hvi_staircase_integral(F, ref, y) if m == 2 else oracle.hvi(F, ref, y)
+            vals.append(hv if np.all(y <= cons) else 0.0)
+        assert got[c] == pytest.approx(np.mean(vals), rel=1e-12, abs=1e-15)
+
+
+def test_constrained_acquisition_limits():
+    F = _front2d(95, 5)
+    ref = np.array([1.1, 1.1])
+    rng = np.random.default_rng(96)
+    mu = rng.uniform(-1.5, 1.0, (200, 2))
+    var = rng.uniform(0.01, 0.5, (200, 2))
+    free = oracle.ehvi2d(mu, var, F, ref)
+    prev = np.zeros(200)
+    for c in (-40.0, -1.0, -0.3, 0.2, 0.8, 5.0):  # non-decreasing in the thresholds
+        e = oracle.ehvi2d(mu, var, F, ref, cons=np.array([c, c]))
+        assert np.all(e >= -1e-15) and np.all(e <= free + 1e-12)
+        assert np.all(e >= prev - 1e-12)
+        prev = e
+    assert np.all(oracle.ehvi2d(mu, var, F, ref, cons=np.array([-40.0, 0.0])) < 1e-300)
+    np.testing.assert_allclose(prev, free, rtol=1e-12, atol=1e-15)  # c far above every sample
