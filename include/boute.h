@@ -125,9 +125,15 @@ int boute_box_decompose(const double *front, const int *P, int B, int n, int m,
  *   EHVI = sum_i [psi1(b_i) - psi1(a_i)] psi2(u_i),  psi(c) = E[(c - Y)_+].
  *   mean, var: B x 2 x N fp32 (boute_gp_posterior's layout);
  *   front, P: boute_pareto_front's output, n = its row capacity; ref: B x 2;
+ *   cons: NULL, or B x 2 fp64 device thresholds k_t on the minimised
+ *         (standardised) objectives, in the units of ref: the constrained
+ *         acquisition of Sec. 5.2, E[HVI(Y) 1[Y_1 <= k_1] 1[Y_2 <= k_2]], which
+ *         replaces psi_t by psi_t^c(c) = E[(c - Y_t)_+ 1[Y_t <= k_t]]; an
+ *         infinite threshold constrains nothing;
  *   acq: B x N fp32. */
 int boute_acq_ehvi(const float *mean, const float *var, int B, long long N, const double *front,
-                   const int *P, int n, const double *ref, float *acq, void *stream);
+                   const int *P, int n, const double *ref, const double *cons, float *acq,
+                   void *stream);
 
 /* Monte-Carlo hypervolume improvement (Sec. 5.2: the expectation estimated by Monte-Carlo
  * integration over posterior samples): sample s of candidate c is
@@ -138,11 +144,15 @@ int boute_acq_ehvi(const float *mean, const float *var, int B, long long N, cons
  *        eps + (b*N + c) * eps_cand_stride, laid out m x S; eps_cand_stride =
  *        m*S for per-candidate normals, 0 for normals shared by all candidates
  *        of a problem (then problem b's block is at eps + b*m*S);
+ *   cons: NULL, or B x m fp64 device thresholds (as for boute_acq_ehvi): a
+ *         sample with some y_t > k_t contributes zero (HVI times the
+ *         feasibility indicator, the constrained estimate of Sec. 5.2); the
+ *         comparison is made in fp32;
  *   acq: B x N fp32. 2 <= m <= 3, 1 <= S. */
 int boute_acq_mc_hvi(const float *mean, const float *var, int B, long long N, int m,
                      const float *lower, const float *upper, const int *K, int box_cap,
-                     const float *eps, int S, long long eps_cand_stride, float *acq,
-                     void *stream);
+                     const float *eps, int S, long long eps_cand_stride, const double *cons,
+                     float *acq, void *stream);
 
 /* ---- selection ----------------------------------------------------------------
  * Sec. 5.2 step (ii): the next configuration(s) to evaluate are the best
@@ -239,6 +249,15 @@ int boute_engine_set_timing(boute_engine *e, int on);
 int boute_engine_stage_times(boute_engine *e, float *ms, int count);
 /* Kernels one boute_engine_step launches. */
 int boute_engine_launches_per_step(const boute_engine *e);
+/* Constrained acquisition for the engine's later steps (Sec. 5.2,
+ * "Constrained qNEHVI"): cons is a HOST array of B x m fp64 thresholds on the
+ * standardised, minimised outcomes (the units of the steps' ref), copied into
+ * the engine; the steps' acquisition becomes E[HVI 1[Y <= cons]] (see
+ * boute_acq_ehvi, boute_acq_mc_hvi). cons = NULL returns to the unconstrained
+ * acquisition. Waits for all work on the device first (no step may be
+ * running); the engine's cached step graphs are rebuilt on the next step when
+ * constraints are switched on or off. */
+int boute_engine_set_constraints(boute_engine *e, const double *cons);
 void boute_engine_free(boute_engine *e);
 
 #ifdef __cplusplus

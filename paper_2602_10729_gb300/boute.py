@@ -27,7 +27,8 @@ SYMBOLS = (
     "boute_engine_step_async",
     "boute_engine_step_host", "boute_engine_step_host_async", "boute_engine_sync",
     "boute_engine_scores", "boute_engine_set_timing",
-    "boute_engine_stage_times", "boute_engine_launches_per_step", "boute_engine_free",
+    "boute_engine_stage_times", "boute_engine_launches_per_step", "boute_engine_set_constraints",
+    "boute_engine_free",
 )
 #: stage names of boute_engine_stage_times, in order
 STAGES = ("fit", "front", "posterior", "acquisition", "topk")
@@ -68,9 +69,9 @@ def load(path: str | None = None):
         "boute_gp_posterior": ([_vp, _vp, _ll, _vp, _vp, _vp], _i),
         "boute_pareto_front": ([_vp, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
         "boute_box_decompose": ([_vp, _vp, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
-        "boute_acq_ehvi": ([_vp, _vp, _i, _ll, _vp, _vp, _i, _vp, _vp, _vp], _i),
-        "boute_acq_mc_hvi": ([_vp, _vp, _i, _ll, _i, _vp, _vp, _vp, _i, _vp, _i, _ll, _vp, _vp],
-                             _i),
+        "boute_acq_ehvi": ([_vp, _vp, _i, _ll, _vp, _vp, _i, _vp, _vp, _vp, _vp], _i),
+        "boute_acq_mc_hvi": ([_vp, _vp, _i, _ll, _i, _vp, _vp, _vp, _i, _vp, _i, _ll, _vp, _vp,
+                              _vp], _i),
         "boute_select_topk": ([_vp, _i, _ll, _i, _vp, _vp, _vp], _i),
         "boute_select_topk_noalloc": ([_vp, _i, _ll, _i, _vp, _vp, _vp], _i),
         "boute_engine_create": ([_i, _i, _i, _i, _ll, _i, _i, _i, ctypes.POINTER(_vp)], _i),
@@ -83,6 +84,7 @@ def load(path: str | None = None):
         "boute_engine_set_timing": ([_vp, _i], _i),
         "boute_engine_stage_times": ([_vp, ctypes.POINTER(ctypes.c_float), _i], _i),
         "boute_engine_launches_per_step": ([_vp], _i),
+        "boute_engine_set_constraints": ([_vp, _vp], _i),
         "boute_engine_free": ([_vp], None),
     }
     for name, (args, res) in sig.items():
@@ -194,19 +196,22 @@ def boute_box_decompose(front, P, B, n, m, ref, lower, upper, K, stream=None):
            "boute_box_decompose")
 
 
-def boute_acq_ehvi(mean, var, B, N, front, P, n, ref, acq, stream=None):
-    f32 = torch.float32
-    _check(load().boute_acq_ehvi(_p(mean, f32), _p(var, f32), B, N, _p(front, torch.float64),
-                                 _p(P, torch.int32), n, _p(ref, torch.float64), _p(acq, f32),
-                                 _s(stream)), "boute_acq_ehvi")
+def boute_acq_ehvi(mean, var, B, N, front, P, n, ref, acq, stream=None, cons=None):
+    """cons: None or a B x 2 fp64 CUDA tensor of thresholds (constrained EHVI)."""
+    f32, f64 = torch.float32, torch.float64
+    _check(load().boute_acq_ehvi(_p(mean, f32), _p(var, f32), B, N, _p(front, f64),
+                                 _p(P, torch.int32), n, _p(ref, f64), _p(cons, f64),
+                                 _p(acq, f32), _s(stream)), "boute_acq_ehvi")
 
 
 def boute_acq_mc_hvi(mean, var, B, N, m, lower, upper, K, box_cap, eps, S, eps_cand_stride, acq,
-                     stream=None):
+                     stream=None, cons=None):
+    """cons: None or a B x m fp64 CUDA tensor of thresholds (constrained MC HVI)."""
     f32 = torch.float32
     _check(load().boute_acq_mc_hvi(_p(mean, f32), _p(var, f32), B, N, m, _p(lower, f32),
                                    _p(upper, f32), _p(K, torch.int32), box_cap, _p(eps, f32), S,
-                                   eps_cand_stride, _p(acq, f32), _s(stream)), "boute_acq_mc_hvi")
+                                   eps_cand_stride, _p(cons, torch.float64), _p(acq, f32),
+                                   _s(stream)), "boute_acq_mc_hvi")
 
 
 def boute_select_topk(acq, B, N, k, idx, val, stream=None):
@@ -308,6 +313,13 @@ def boute_engine_stage_times(e: Engine) -> dict:
 
 def boute_engine_launches_per_step(e: Engine) -> int:
     return int(load().boute_engine_launches_per_step(e.handle))
+
+
+def boute_engine_set_constraints(e: Engine, cons=None):
+    """cons: None (unconstrained) or a contiguous B x m fp64 CPU tensor of
+    thresholds on the standardised, minimised outcomes (the units of ref)."""
+    _check(load().boute_engine_set_constraints(e.handle, _p(cons, torch.float64, False)),
+           "boute_engine_set_constraints")
 
 
 def boute_engine_free(e: Engine):

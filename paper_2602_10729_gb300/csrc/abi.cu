@@ -116,6 +116,10 @@ struct boute_engine {
   cudaEvent_t ev_xc1, ev_eps1[2], in_free[2];
   cudaEvent_t ev_small[2];  // the small inputs of set 0 / 1 are in place
   int host_set;
+  // constrained acquisition (boute_engine_set_constraints): B x m thresholds,
+  // allocated on first use; used while has_cons
+  double *cons;
+  int has_cons;
 };
 
 // Stage order of one step as timed (with timing on, the front stage runs
@@ -226,19 +230,20 @@ int boute_box_decompose(const double *front, const int *P, int B, int n, int m, 
 }
 
 int boute_acq_ehvi(const float *mean, const float *var, int B, long long N, const double *front,
-                   const int *P, int n, const double *ref, float *acq, void *stream) {
+                   const int *P, int n, const double *ref, const double *cons, float *acq,
+                   void *stream) {
   if (B < 1 || N < 0 || n < 1 || n > BOUTE_MAX_N || !front || !P || !ref ||
       (N > 0 && (!mean || !var || !acq)))
     return BOUTE_ERR_INVALID_ARG;
   if ((long long)B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;
   if (int r = device_ok()) return r;
-  return launch_ehvi(mean, var, B, N, front, P, n, ref, acq, (cudaStream_t)stream);
+  return launch_ehvi(mean, var, B, N, front, P, n, ref, cons, acq, (cudaStream_t)stream);
 }
 
 int boute_acq_mc_hvi(const float *mean, const float *var, int B, long long N, int m,
                      const float *lower, const float *upper, const int *K, int box_cap,
-                     const float *eps, int S, long long eps_cand_stride, float *acq,
-                     void *stream) {
+                     const float *eps, int S, long long eps_cand_stride, const double *cons,
+                     float *acq, void *stream) {
   if (B < 1 || N < 0 || S < 1 || box_cap < 1 || eps_cand_stride < 0 || !lower || !upper || !K ||
       (N > 0 && (!mean || !var || !acq || !eps)))
     return BOUTE_ERR_INVALID_ARG;
@@ -246,8 +251,8 @@ int boute_acq_mc_hvi(const float *mean, const float *var, int B, long long N, in
   if ((long long)B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;
   if ((size_t)box_cap * m * 2 * sizeof(float) > 200 * 1024) return BOUTE_ERR_UNSUPPORTED;
   if (int r = device_ok()) return r;
-  return launch_mchvi(mean, var, B, N, m, lower, upper, K, box_cap, eps, S, eps_cand_stride, acq,
-                      (cudaStream_t)stream);
+  return launch_mchvi(mean, var, B, N, m, lower, upper, K, box_cap, eps, S, eps_cand_stride, cons,
+                      acq, (cudaStream_t)stream);
 }
 
 int boute_select_topk(const float *acq, int B, long long N, int k, long long *idx, float *val,
@@ -287,7 +292,7 @@ void boute_engine_free(boute_engine *e) {
   void *ptrs[] = {e->X, e->Y, e->Ys, e->ls, e->s2, e->noise, e->ref, e->front, e->mask, e->P,
                   e->K, e->lower, e->upper, e->Xc, e->eps, e->mean, e->var, e->acq, e->val,
                   e->idx, e->scratch, e->sel, e->kst, e->X1, e->Y1, e->ls1, e->s21,
-                  e->noise1, e->ref1, e->Xc1, e->eps1};
+                  e->noise1, e->ref1, e->Xc1, e->eps1, e->cons};
   for (void *p : ptrs) cudaFree(p);
   delete e;
 }
@@ -454,15 +459,18 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
       if (cudaStreamWaitEvent(s, ev_eps[i], wait_flags) != cudaSuccess)
         return last_launch_status();
   mark(ST_ACQ);
+  const double *cons = e->has_cons ? e->cons : nullptr;
   if (e->fuse_sel && !e->timing) {
     if ((r = launch_mchvi2_select(e->mean, e->var, B, e->N, e->lower, e->upper, e->K, 2 * n + 2,
-                                  eps, e->S, 2ll * e->S, e->acq, e->k, e->sel, idx, val, s)))
+                                  eps, e->S, 2ll * e->S, cons, e->acq, e->k, e->sel, idx, val,
+                                  s)))
       return r;
   } else if (!mc) {
-    if ((r = launch_ehvi(e->mean, e->var, B, e->N, e->front, e->P, n, ref, e->acq, s))) return r;
+    if ((r = launch_ehvi(e->mean, e->var, B, e->N, e->front, e->P, n, ref, cons, e->acq, s)))
+      return r;
   } else {
     if ((r = launch_mchvi(e->mean, e->var, B, e->N, m, e->lower, e->upper, e->K, 2 * n + 2, eps,
-                          e->S, (long long)m * e->S, e->acq, s)))
+                          e->S, (long long)m * e->S, cons, e->acq, s)))
       return r;
   }
   if (!e->fuse_sel || e->timing) {
@@ -692,5 +700,27 @@ int boute_engine_stage_times(boute_engine *e, float *ms, int count) {
 }
 
 int boute_engine_launches_per_step(const boute_engine *e) { return e ? e->launches : 0; }
+
+int boute_engine_set_constraints(boute_engine *e, const double *cons) {
+  if (!e) return BOUTE_ERR_INVALID_ARG;
+  const size_t count = (size_t)e->B * e->m;
+  // no step of this engine may be reading the thresholds while they change
+  if (cudaDeviceSynchronize() != cudaSuccess) return last_launch_status();
+  if (cons) {
+    if (!e->cons && dalloc(&e->cons, count) != BOUTE_OK) return BOUTE_ERR_OOM;
+    if (cudaMemcpy(e->cons, cons, count * sizeof(double), cudaMemcpyHostToDevice) != cudaSuccess)
+      return last_launch_status();
+  }
+  const int on = cons != nullptr;
+  if (on != e->has_cons) {  // the step's acquisition kernel changes: recapture
+    e->has_cons = on;
+    for (auto &g : e->graphs)
+      if (g.exec) {
+        cudaGraphExecDestroy(g.exec);
+        g.exec = nullptr;
+      }
+  }
+  return BOUTE_OK;
+}
 
 }  // extern "C"

@@ -1,5 +1,6 @@
 // Acquisition kernels: closed-form 2-objective EHVI and Monte-Carlo
 // hypervolume improvement over the box decomposition of the front.
+#include <float.h>
 #include <math.h>
 
 #include <algorithm>
@@ -18,19 +19,35 @@ constexpr float kInvSqrt2 = 0.7071067811865476f;
 // Small part of psi: with z = (x - mu)/sigma, E[(x - Y)_+] = max(x - mu, 0) +
 // sigma * gm(z), gm(z) = phi(|z|) - |z| Phi(-|z|) >= 0 (the identity
 // G(z) = z + G(-z) for G(z) = z Phi(z) + phi(z)). Keeping the linear part
-// apart avoids cancellation for points far to either side of x.
+// apart avoids cancellation for points far to either side of x. |z| is
+// capped where gm is already zero, so that infinite z gives 0, not NaN.
 __device__ __forceinline__ float gm(float z) {
-  const float t = fabsf(z);
+  const float t = fminf(fabsf(z), 1.0e4f);
   return expf(-0.5f * t * t) * kInvSqrt2Pi - t * (0.5f * erfcf(t * kInvSqrt2));
+}
+
+__device__ __forceinline__ float std_cdf(float z) { return 0.5f * erfcf(-z * kInvSqrt2); }
+
+// A threshold as a finite float (an infinite threshold constrains nothing:
+// FLT_MAX is above every finite value and keeps the differences below finite).
+__device__ __forceinline__ float threshold(double c) {
+  return fminf(fmaxf((float)c, -FLT_MAX), FLT_MAX);
 }
 
 // ---- closed-form EHVI, m = 2 ---------------------------------------------------
 // Cells i = 0..P of the front sorted by f1: f1 in [a_i, b_i), f2 below u_i,
 // a_0 = -inf, b_P = r1, u_0 = r2. EHVI = sum_i [psi1(b_i) - psi1(a_i)] psi2(u_i).
+// CONS (Sec. 5.2, constrained qNEHVI, thresholds k_t on the minimised
+// objectives, cons: B x 2): psi_t becomes psi_t^c(v) = E[(v - Y)_+ 1[Y <= k_t]],
+// which is psi_t(min(v, k_t)) + (v - k_t)_+ Phi((k_t - mu_t) / sigma_t), since
+// below k_t the indicator is one and above it (v - Y) splits into (k_t - Y) +
+// (v - k_t). Per cell psi1^c(b) - psi1^c(a) is then the unconstrained
+// difference between the clamped bounds plus (max(b, k1) - max(a, k1)) Phi_1.
+template <bool CONS>
 __global__ void __launch_bounds__(256) ehvi2d_kernel(const float *mean, const float *var,
                                                      long long N, const double *front,
                                                      const int *P, int n, const double *ref,
-                                                     float *acq) {
+                                                     const double *cons, float *acq) {
   extern __shared__ float cells[];  // bnd[n+1] (b_i), up[n+1] (u_i)
   pdl_wait();
   const int b = blockIdx.y;
@@ -38,6 +55,7 @@ __global__ void __launch_bounds__(256) ehvi2d_kernel(const float *mean, const fl
   float *bnd = cells, *up = cells + (n + 1);
   const double *F = front + (size_t)b * n * 2;
   const float r1 = (float)ref[2 * b], r2 = (float)ref[2 * b + 1];
+  const float k1 = CONS ? threshold(cons[2 * b]) : 0.f, k2 = CONS ? threshold(cons[2 * b + 1]) : 0.f;
   for (int i = threadIdx.x; i <= Pb; i += blockDim.x) {
     bnd[i] = i == Pb ? r1 : (float)F[2 * i];
     up[i] = i == 0 ? r2 : (float)F[2 * (i - 1) + 1];
@@ -50,14 +68,26 @@ __global__ void __launch_bounds__(256) ehvi2d_kernel(const float *mean, const fl
     const float mu1 = m1[c], mu2 = m2[c];
     const float sg1 = sqrtf(fmaxf(v1[c], 0.f)), sg2 = sqrtf(fmaxf(v2[c], 0.f));
     const float is1 = sg1 > 0.f ? 1.f / sg1 : 0.f, is2 = sg2 > 0.f ? 1.f / sg2 : 0.f;
+    // CONS: P(Y_t <= k_t) (a step when sigma_t = 0) and max(a, k1) of cell 0
+    float F1 = 1.f, F2 = 1.f, ahi = k1;
+    if (CONS) {
+      F1 = sg1 > 0.f ? std_cdf((k1 - mu1) * is1) : (mu1 <= k1 ? 1.f : 0.f);
+      F2 = sg2 > 0.f ? std_cdf((k2 - mu2) * is2) : (mu2 <= k2 ? 1.f : 0.f);
+    }
     float e = 0.f, ga = 0.f, a = -INFINITY;
     for (int i = 0; i <= Pb; ++i) {
-      const float bb = bnd[i], u = up[i];
+      const float bb = CONS ? fminf(bnd[i], k1) : bnd[i], u = CONS ? fminf(up[i], k2) : up[i];
       const float gb = sg1 > 0.f ? gm((bb - mu1) * is1) : 0.f;
       const float lin = mu1 <= a ? bb - a : (mu1 <= bb ? bb - mu1 : 0.f);
-      const float D = fmaxf(fmaf(sg1, gb - ga, lin), 0.f);
+      float D = fmaxf(fmaf(sg1, gb - ga, lin), 0.f);
       const float g2 = sg2 > 0.f ? gm((u - mu2) * is2) : 0.f;
-      const float psi2 = fmaf(sg2, g2, fmaxf(u - mu2, 0.f));
+      float psi2 = fmaf(sg2, g2, fmaxf(u - mu2, 0.f));
+      if (CONS) {
+        const float bhi = fmaxf(bnd[i], k1);
+        D = fmaf(bhi - ahi, F1, D);
+        ahi = bhi;
+        psi2 = fmaf(fmaxf(up[i] - k2, 0.f), F2, psi2);
+      }
       e = fmaf(D, psi2, e);
       ga = gb;
       a = bb;
@@ -69,12 +99,15 @@ __global__ void __launch_bounds__(256) ehvi2d_kernel(const float *mean, const fl
 // ---- Monte-Carlo HVI: one warp per candidate, lanes over samples ---------------
 // Each sample's HVI is the volume of [y, ref] inside the disjoint boxes:
 // sum_k prod_t (u_kt - max(l_kt, y_t))_+.
-template <int M>
+// CONS: a sample with some y_t above its threshold (cons: B x M) counts zero
+// (its first coordinate is moved beyond every box).
+template <int M, bool CONS>
 __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const float *var, int B,
                                                     long long N, const float *lower,
                                                     const float *upper, const int *Kc,
                                                     int box_cap, const float *eps, int S,
-                                                    long long eps_stride, float *acq) {
+                                                    long long eps_stride, const double *cons,
+                                                    float *acq) {
   extern __shared__ float boxes[];  // per problem in this block: lo[K][M], hi[K][M]
   pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
@@ -86,6 +119,9 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
     hi[i] = upper[(size_t)b * box_cap * M + i];
   }
   __syncthreads();
+  float kc[M];
+#pragma unroll
+  for (int t = 0; t < M; ++t) kc[t] = CONS ? threshold(cons[(size_t)b * M + t]) : 0.f;
   const float *mb = mean + (size_t)b * M * N, *vb = var + (size_t)b * M * N;
   const bool vec = (S % 128) == 0 && ((uintptr_t)eps & 15) == 0 && (eps_stride % 4) == 0;
   for (long long c = (long long)blockIdx.x * wpb + warp; c < N; c += (long long)gridDim.x * wpb) {
@@ -111,6 +147,15 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
           y[2][t] = fmaf(sg[t], z[t].z, mu[t]);
           y[3][t] = fmaf(sg[t], z[t].w, mu[t]);
         }
+        if (CONS) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            bool ok = true;
+#pragma unroll
+            for (int t = 0; t < M; ++t) ok = ok && y[j][t] <= kc[t];
+            if (!ok) y[j][0] = kInfeasible;
+          }
+        }
         for (int k = 0; k < K; ++k) {
           float l[M], h[M];
 #pragma unroll
@@ -132,6 +177,12 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
         float y[M];
 #pragma unroll
         for (int t = 0; t < M; ++t) y[t] = fmaf(sg[t], e[(size_t)t * S + s], mu[t]);
+        if (CONS) {
+          bool ok = true;
+#pragma unroll
+          for (int t = 0; t < M; ++t) ok = ok && y[t] <= kc[t];
+          if (!ok) y[0] = kInfeasible;
+        }
         for (int k = 0; k < K; ++k) {
           float v = fmaxf(hi[k * M] - fmaxf(lo[k * M], y[0]), 0.f);
 #pragma unroll
@@ -154,14 +205,16 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
 // merges its warps' lists into sel_keys, and the last block of a problem to
 // finish (sel_cnt) merges all the blocks' lists, writes idx / val and sets
 // the counter back to zero.
+// CONS: samples above a threshold (cons: B x 2) count zero.
 constexpr int kSelGroup = 32;  // blocks per selection group
 
-template <bool SEL>
+template <bool SEL, bool CONS>
 __global__ void __launch_bounds__(512, 2) mchvi2_kernel(const float *mean, const float *var,
                                                      long long N, const float *lower,
                                                      const float *upper, const int *Kc,
                                                      int box_cap, const float *eps, int S,
-                                                     long long eps_stride, float *acq, int ksel,
+                                                     long long eps_stride, const double *cons,
+                                                     float *acq, int ksel,
                                                      unsigned long long *sel_keys,
                                                      long long *idx, float *val) {
   // k >= 1: (b/D, 1/D, u, D); [0]: (b_0, u_0, -, -); then zero strips up to
@@ -173,6 +226,7 @@ __global__ void __launch_bounds__(512, 2) mchvi2_kernel(const float *mean, const
   const int K = mc2_load_strips(strips4, lower, upper, Kc, b, box_cap, threadIdx.x, blockDim.x);
   const int Kp = mc2_padded(K);
   __syncthreads();
+  const float k1 = CONS ? threshold(cons[2 * b]) : 0.f, k2 = CONS ? threshold(cons[2 * b + 1]) : 0.f;
   const float *m1 = mean + (size_t)b * 2 * N, *m2 = m1 + N;
   const float *v1 = var + (size_t)b * 2 * N, *v2 = v1 + N;
   const bool vec = (S == 128) && ((uintptr_t)eps & 15) == 0 && (eps_stride % 4) == 0;
@@ -222,7 +276,8 @@ __global__ void __launch_bounds__(512, 2) mchvi2_kernel(const float *mean, const
       z1 = __ldcs((const float4 *)ep);
       z2 = __ldcs((const float4 *)(ep + S));
       pm1 = m1[cn]; pm2 = m2[cn]; pv1 = v1[cn]; pv2 = v2[cn];
-      const float sum = mc2_warp_total(mc2_lane_sum(strips4, K, Kp, t0, c1, c2, mu1, mu2, qv1, qv2));
+      const float sum =
+          mc2_warp_total(mc2_lane_sum<CONS>(strips4, K, Kp, t0, c1, c2, mu1, mu2, qv1, qv2, k1, k2));
       if (lane == 0) acq[(size_t)b * N + c] = sum * inv_s;
       if (SEL) sel.add(make_key(sum * inv_s, (unsigned)c), lane);
     }
@@ -232,7 +287,12 @@ __global__ void __launch_bounds__(512, 2) mchvi2_kernel(const float *mean, const
     const float sg1 = sqrt_fast(fmaxf(v1[c], 0.f)), sg2 = sqrt_fast(fmaxf(v2[c], 0.f));
     const float *e = eps_of(c);
     float sum = 0.f;
-    for (int s = lane; s < S; s += 32) sum += hvi(fmaf(sg1, e[s], mu1), fmaf(sg2, e[S + s], mu2));
+    for (int s = lane; s < S; s += 32) {
+      float y1 = fmaf(sg1, e[s], mu1);
+      const float y2 = fmaf(sg2, e[S + s], mu2);
+      if (CONS && !(y1 <= k1 && y2 <= k2)) y1 = kInfeasible;
+      sum += hvi(y1, y2);
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
     if (lane == 0) acq[(size_t)b * N + c] = sum * inv_s;
@@ -320,11 +380,19 @@ unsigned resident_grid_x(Kern kernel, int threads, size_t smem, int B, long long
 }  // namespace
 
 int launch_ehvi(const float *mean, const float *var, int B, long long N, const double *front,
-                const int *P, int n, const double *ref, float *acq, cudaStream_t s) {
+                const int *P, int n, const double *ref, const double *cons, float *acq,
+                cudaStream_t s) {
   if (N <= 0) return BOUTE_OK;
   const size_t smem = 2 * (size_t)(n + 1) * sizeof(float);
-  const unsigned gx = resident_grid_x(ehvi2d_kernel, 256, smem, B, N, 256);
-  launch_pdl(ehvi2d_kernel, dim3(gx, B), dim3(256), smem, s, mean, var, N, front, P, n, ref, acq);
+  if (cons) {
+    const unsigned gx = resident_grid_x(ehvi2d_kernel<true>, 256, smem, B, N, 256);
+    launch_pdl(ehvi2d_kernel<true>, dim3(gx, B), dim3(256), smem, s, mean, var, N, front, P, n,
+               ref, cons, acq);
+  } else {
+    const unsigned gx = resident_grid_x(ehvi2d_kernel<false>, 256, smem, B, N, 256);
+    launch_pdl(ehvi2d_kernel<false>, dim3(gx, B), dim3(256), smem, s, mean, var, N, front, P, n,
+               ref, cons, acq);
+  }
   count_launch();
   return last_launch_status();
 }
@@ -333,26 +401,28 @@ namespace {
 
 size_t mchvi2_smem(int box_cap) { return ((size_t)box_cap + 4) * sizeof(float4); }
 
-void mchvi2_configure(bool sel, int box_cap) {
+template <class Kern>
+void configure_smem(Kern kernel, size_t smem) {
+  prefer_shared(kernel);
+  if (smem > 48 * 1024)
+    cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+}
+
+void mchvi2_configure(int box_cap) {
   const size_t smem = mchvi2_smem(box_cap);
-  if (sel) {
-    prefer_shared(mchvi2_kernel<true>);
-    if (smem > 48 * 1024)
-      cudaFuncSetAttribute(mchvi2_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)smem);
-  } else {
-    prefer_shared(mchvi2_kernel<false>);
-    if (smem > 48 * 1024)
-      cudaFuncSetAttribute(mchvi2_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)smem);
-  }
+  configure_smem(mchvi2_kernel<true, false>, smem);
+  configure_smem(mchvi2_kernel<true, true>, smem);
+  configure_smem(mchvi2_kernel<false, false>, smem);
+  configure_smem(mchvi2_kernel<false, true>, smem);
 }
 
 }  // namespace
 
+// One grid for both variants of the selecting kernel (the scratch is sized by
+// it); the grid stride makes any grid correct.
 unsigned mchvi2_select_grid_x(int B, long long N, int box_cap) {
-  mchvi2_configure(true, box_cap);
-  return resident_grid_x(mchvi2_kernel<true>, 512, mchvi2_smem(box_cap), B, N, 16);
+  mchvi2_configure(box_cap);
+  return resident_grid_x(mchvi2_kernel<true, false>, 512, mchvi2_smem(box_cap), B, N, 16);
 }
 
 // Bytes of the selection scratch of launch_mchvi2_select: per problem, one
@@ -369,39 +439,76 @@ size_t mchvi2_select_scratch_bytes(int B, long long N, int box_cap) {
 // counters are zero (they are zero again when the kernel ends).
 int launch_mchvi2_select(const float *mean, const float *var, int B, long long N,
                          const float *lower, const float *upper, const int *K, int box_cap,
-                         const float *eps, int S, long long eps_stride, float *acq, int k,
-                         void *sel, long long *idx, float *val, cudaStream_t s) {
+                         const float *eps, int S, long long eps_stride, const double *cons,
+                         float *acq, int k, void *sel, long long *idx, float *val,
+                         cudaStream_t s) {
   if (N <= 0 || k < 1 || k > kWarpK || k > N) return BOUTE_ERR_INVALID_ARG;
   const unsigned gx = mchvi2_select_grid_x(B, N, box_cap);
   if (gx > (unsigned)(kSelGroup * kSelGroup)) return BOUTE_ERR_UNSUPPORTED;
-  launch_pdl(mchvi2_kernel<true>, dim3(gx, B), dim3(16 * 32), mchvi2_smem(box_cap), s, mean, var,
-             N, lower, upper, K, box_cap, eps, S, eps_stride, acq, k,
-             (unsigned long long *)sel, idx, val);
+  auto *keys = (unsigned long long *)sel;
+  if (cons)
+    launch_pdl(mchvi2_kernel<true, true>, dim3(gx, B), dim3(16 * 32), mchvi2_smem(box_cap), s,
+               mean, var, N, lower, upper, K, box_cap, eps, S, eps_stride, cons, acq, k, keys,
+               idx, val);
+  else
+    launch_pdl(mchvi2_kernel<true, false>, dim3(gx, B), dim3(16 * 32), mchvi2_smem(box_cap), s,
+               mean, var, N, lower, upper, K, box_cap, eps, S, eps_stride, cons, acq, k, keys,
+               idx, val);
   count_launch();
   return last_launch_status();
 }
 
+namespace {
+
+template <bool CONS>
+void launch_mchvi2_plain(const float *mean, const float *var, int B, long long N,
+                         const float *lower, const float *upper, const int *K, int box_cap,
+                         const float *eps, int S, long long eps_stride, const double *cons,
+                         float *acq, cudaStream_t s) {
+  mchvi2_configure(box_cap);
+  const size_t smem = mchvi2_smem(box_cap);
+  const unsigned gx = resident_grid_x(mchvi2_kernel<false, CONS>, 512, smem, B, N, 16);
+  unsigned long long *nk = nullptr;
+  long long *ni = nullptr;
+  float *nv = nullptr;
+  launch_pdl(mchvi2_kernel<false, CONS>, dim3(gx, B), dim3(16 * 32), smem, s, mean, var, N,
+             lower, upper, K, box_cap, eps, S, eps_stride, cons, acq, 0, nk, ni, nv);
+}
+
+template <bool CONS>
+void launch_mchvi3(const float *mean, const float *var, int B, long long N, const float *lower,
+                   const float *upper, const int *K, int box_cap, const float *eps, int S,
+                   long long eps_stride, const double *cons, float *acq, cudaStream_t s) {
+  const size_t smem = 2 * (size_t)box_cap * 3 * sizeof(float);
+  if (smem > 48 * 1024)
+    cudaFuncSetAttribute(mchvi_kernel<3, CONS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)smem);
+  const unsigned gx = resident_grid_x(mchvi_kernel<3, CONS>, 512, smem, B, N, 16);
+  launch_pdl(mchvi_kernel<3, CONS>, dim3(gx, B), dim3(16 * 32), smem, s, mean, var, B, N, lower,
+             upper, K, box_cap, eps, S, eps_stride, cons, acq);
+}
+
+}  // namespace
+
 int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
                  const float *lower, const float *upper, const int *K, int box_cap,
-                 const float *eps, int S, long long eps_stride, float *acq, cudaStream_t s) {
+                 const float *eps, int S, long long eps_stride, const double *cons, float *acq,
+                 cudaStream_t s) {
   if (N <= 0) return BOUTE_OK;
   if (m == 2) {
-    mchvi2_configure(false, box_cap);
-    const size_t smem2 = mchvi2_smem(box_cap);
-    const unsigned gx = resident_grid_x(mchvi2_kernel<false>, 512, smem2, B, N, 16);
-    unsigned long long *nk = nullptr;
-    long long *ni = nullptr;
-    float *nv = nullptr;
-    launch_pdl(mchvi2_kernel<false>, dim3(gx, B), dim3(16 * 32), smem2, s, mean, var, N, lower,
-               upper, K, box_cap, eps, S, eps_stride, acq, 0, nk, ni, nv);
+    if (cons)
+      launch_mchvi2_plain<true>(mean, var, B, N, lower, upper, K, box_cap, eps, S, eps_stride,
+                                cons, acq, s);
+    else
+      launch_mchvi2_plain<false>(mean, var, B, N, lower, upper, K, box_cap, eps, S, eps_stride,
+                                 cons, acq, s);
   } else if (m == 3) {
-    const size_t smem = 2 * (size_t)box_cap * m * sizeof(float);
-    if (smem > 48 * 1024)
-      cudaFuncSetAttribute(mchvi_kernel<3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)smem);
-    const unsigned gx = resident_grid_x(mchvi_kernel<3>, 512, smem, B, N, 16);
-    launch_pdl(mchvi_kernel<3>, dim3(gx, B), dim3(16 * 32), smem, s, mean, var, B, N, lower,
-               upper, K, box_cap, eps, S, eps_stride, acq);
+    if (cons)
+      launch_mchvi3<true>(mean, var, B, N, lower, upper, K, box_cap, eps, S, eps_stride, cons,
+                          acq, s);
+    else
+      launch_mchvi3<false>(mean, var, B, N, lower, upper, K, box_cap, eps, S, eps_stride, cons,
+                           acq, s);
   } else {
     return BOUTE_ERR_UNSUPPORTED;
   }

@@ -81,17 +81,21 @@ int launch_fit_raw(Gp *gp, const double *X, const double *Y, const double *ls, c
                    cudaEvent_t setup_done = nullptr);
 int launch_boxes(const double *front, const int *P, int B, int n, int m, const double *ref,
                  float *lower, float *upper, int *K, cudaStream_t s);
+// cons: per problem m thresholds on the minimised objectives (device), or null
 int launch_ehvi(const float *mean, const float *var, int B, long long N, const double *front,
-                const int *P, int n, const double *ref, float *acq, cudaStream_t s);
+                const int *P, int n, const double *ref, const double *cons, float *acq,
+                cudaStream_t s);
 unsigned mchvi2_select_grid_x(int B, long long N, int box_cap);
 size_t mchvi2_select_scratch_bytes(int B, long long N, int box_cap);
 int launch_mchvi2_select(const float *mean, const float *var, int B, long long N,
                          const float *lower, const float *upper, const int *K, int box_cap,
-                         const float *eps, int S, long long eps_stride, float *acq, int k,
-                         void *sel, long long *idx, float *val, cudaStream_t s);
+                         const float *eps, int S, long long eps_stride, const double *cons,
+                         float *acq, int k, void *sel, long long *idx, float *val,
+                         cudaStream_t s);
 int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
                  const float *lower, const float *upper, const int *K, int box_cap,
-                 const float *eps, int S, long long eps_stride, float *acq, cudaStream_t s);
+                 const float *eps, int S, long long eps_stride, const double *cons, float *acq,
+                 cudaStream_t s);
 size_t topk_scratch_bytes(int B, long long N, int k);
 // counters_zeroed: the scratch's per-problem counters are known to be zero
 // (an engine's scratch: zeroed at creation, and every call leaves them zero);

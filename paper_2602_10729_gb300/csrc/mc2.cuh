@@ -1,7 +1,6 @@
 // 2-objective Monte-Carlo hypervolume improvement (Sec. 5.2, "Constrained
-// qNEHVI": the expected improvement estimated over base normals), shared by
-// the acquisition kernel and the posterior kernel that scores candidates as
-// soon as their posterior is complete, so that both give identical values.
+// qNEHVI": the expected improvement estimated over base normals), the
+// per-candidate arithmetic of the 2-objective acquisition kernel.
 //
 // Strip decomposition: strips k = 0..K-1 with x-extent [a_k, b_k) (a_0 = -inf,
 // a_k = b_{k-1}) and top u_k (u decreasing, u_0 = r2 the largest). For a
@@ -62,19 +61,33 @@ __device__ __forceinline__ int mc2_load_strips(float4 *strips4, const float *low
 
 __device__ __forceinline__ int mc2_padded(int K) { return K > 0 ? 1 + ((K + 2) & ~3) : 0; }
 
+// A sample that violates a constraint contributes nothing (Sec. 5.2,
+// constrained qNEHVI: HVI times the feasibility indicator): its first
+// coordinate is moved beyond every strip, which makes every width term zero.
+constexpr float kInfeasible = 3.0e38f;
+
 // One lane's share of the improvement sum of a candidate, S = 128: the lane's
 // four samples per objective (c1, c2: base normals), posterior mean mu and
 // variance pv per objective. t0 = strips4[0] (zero when K = 0), u0 = t0.y.
-// The caller adds the 32 lanes' shares and divides by S.
+// CONS: samples count only if y_1 <= k1 and y_2 <= k2 (thresholds on the
+// minimised objectives). The caller adds the 32 lanes' shares and divides by S.
+template <bool CONS = false>
 __device__ __forceinline__ float mc2_lane_sum(const float4 *strips4, int K, int Kp, float4 t0,
                                               float4 c1, float4 c2, float mu1, float mu2,
-                                              float pv1, float pv2) {
+                                              float pv1, float pv2, float k1 = 0.f,
+                                              float k2 = 0.f) {
   const float u0 = t0.y;
   const float sg1 = sqrt_fast(fmaxf(pv1, 0.f)), sg2 = sqrt_fast(fmaxf(pv2, 0.f));
-  const float y1[4] = {fmaf(sg1, c1.x, mu1), fmaf(sg1, c1.y, mu1), fmaf(sg1, c1.z, mu1),
-                       fmaf(sg1, c1.w, mu1)};
+  const float y1c[4] = {fmaf(sg1, c1.x, mu1), fmaf(sg1, c1.y, mu1), fmaf(sg1, c1.z, mu1),
+                        fmaf(sg1, c1.w, mu1)};
   const float y2[4] = {fmaf(sg2, c2.x, mu2), fmaf(sg2, c2.y, mu2), fmaf(sg2, c2.z, mu2),
                        fmaf(sg2, c2.w, mu2)};
+  float y1[4] = {y1c[0], y1c[1], y1c[2], y1c[3]};
+  if (CONS) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (!(y1c[j] <= k1 && y2[j] <= k2)) y1[j] = kInfeasible;
+  }
   // per lane: H = u_0 - (its lowest y2) bounds every height of its samples
   const float lo2 = fminf(fminf(y2[0], y2[1]), fminf(y2[2], y2[3]));
   const float H = u0 - lo2;

@@ -150,11 +150,12 @@ def oracle_fit(hp: HostProblem, b: int) -> opl.FittedProblem:
 
 
 # ---- GPU: one ABI call at a time ------------------------------------------------
-def gpu_pipeline(hp: HostProblem, N: int | None = None, mean_var_in=None):
+def gpu_pipeline(hp: HostProblem, N: int | None = None, mean_var_in=None, cons=None):
     """Runs standardise -> fit -> front -> boxes -> posterior -> acq -> top-k
     through the C-ABI and returns every intermediate on the host.
     mean_var_in: optional (mean, var) B x m x N float32 fed to the
-    acquisition instead of the GPU posterior (isolated acquisition test)."""
+    acquisition instead of the GPU posterior (isolated acquisition test).
+    cons: optional B x m thresholds (constrained acquisition)."""
     import torch
 
     from paper_2602_10729_gb300 import boute as bt
@@ -190,15 +191,17 @@ def gpu_pipeline(hp: HostProblem, N: int | None = None, mean_var_in=None):
         mi, vi = mean, var
     acq = torch.empty((B, N), dtype=torch.float32, device=dev)
     cap = 2 * n + 2
+    cn = None if cons is None else t(cons, torch.float64)
     if w.mode == "ehvi":
-        bt.boute_acq_ehvi(mi, vi, B, N, front, P, n, ref, acq)
+        bt.boute_acq_ehvi(mi, vi, B, N, front, P, n, ref, acq, cons=cn)
     else:
         lower = torch.empty((B, cap, m), dtype=torch.float32, device=dev)
         upper = torch.empty_like(lower)
         K = torch.empty(B, dtype=torch.int32, device=dev)
         bt.boute_box_decompose(front, P, B, n, m, ref, lower, upper, K)
         eps = t(hp.eps[:, :N], torch.float32)
-        bt.boute_acq_mc_hvi(mi, vi, B, N, m, lower, upper, K, cap, eps, w.S, m * w.S, acq)
+        bt.boute_acq_mc_hvi(mi, vi, B, N, m, lower, upper, K, cap, eps, w.S, m * w.S, acq,
+                            cons=cn)
         out.update(lower=lower.cpu().numpy(), upper=upper.cpu().numpy(), K=K.cpu().numpy())
     k = min(w.k, N)
     idx = torch.empty((B, k), dtype=torch.int64, device=dev)

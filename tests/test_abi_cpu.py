@@ -58,8 +58,9 @@ def test_invalid_arguments_are_rejected_before_any_device_call(lib):
     assert lib.boute_select_topk(p, 1, 10, 0, p, p, None) == bt.BOUTE_ERR_INVALID_ARG
     assert lib.boute_engine_create(1, 8, 2, 3, 100, bt.BOUTE_ACQ_EHVI2D, 0, 4,
                                    ctypes.byref(h)) == bt.BOUTE_ERR_INVALID_ARG
-    assert lib.boute_acq_mc_hvi(p, p, 1, 10, 4, p, p, p, 4, p, 8, 32, p, None) in (
+    assert lib.boute_acq_mc_hvi(p, p, 1, 10, 4, p, p, p, 4, p, 8, 32, None, p, None) in (
         bt.BOUTE_ERR_UNSUPPORTED, bt.BOUTE_ERR_INVALID_ARG)
+    assert lib.boute_engine_set_constraints(None, None) == bt.BOUTE_ERR_INVALID_ARG
     assert lib.boute_gp_status(None, None) == bt.BOUTE_ERR_INVALID_ARG
 
 
