@@ -169,9 +169,10 @@ def profiled_traffic(kernel: str, workload: str):
 
 
 # ---------------------------------------------------------------- CPU oracle
-def oracle_rate(w: wl.Workload, inp, budget_s: float, threads: int = 0):
+def oracle_rate(w: wl.Workload, inp, budget_s: float, threads: int = 0, cons=None):
     """The oracle's scoring step (fit, front, posterior, acquisition, top-k)
-    on problem 0 over a candidate sample sized to about budget_s seconds."""
+    on problem 0 over a candidate sample sized to about budget_s seconds
+    (cons: the thresholds of a constrained acquisition, or None)."""
     import oracle
     from oracle import pipeline as opl
     threads = threads or oracle.default_threads()
@@ -182,14 +183,14 @@ def oracle_rate(w: wl.Workload, inp, budget_s: float, threads: int = 0):
     n_try = min(w.N, 2048)
     t0 = time.perf_counter()
     opl.score(fp, inp["Xc"][0, :n_try], w.mode, min(w.k, n_try),
-              None if inp["eps"] is None else inp["eps"][0, :n_try], threads)
+              None if inp["eps"] is None else inp["eps"][0, :n_try], threads, cons=cons)
     per = (time.perf_counter() - t0) / n_try
     sample = int(max(n_try, min(w.N, (budget_s - fit_s) / max(per, 1e-9))))
     t0 = time.perf_counter()
     fp = opl.fit_problem(inp["X"][0], inp["Y"][0], inp["ls"][0], inp["s2"][0], inp["noise"][0],
                          inp["ref"][0])
     opl.score(fp, inp["Xc"][0, :sample], w.mode, min(w.k, sample),
-              None if inp["eps"] is None else inp["eps"][0, :sample], threads)
+              None if inp["eps"] is None else inp["eps"][0, :sample], threads, cons=cons)
     dt = time.perf_counter() - t0
     return sample / dt, threads, sample, dt
 
@@ -201,7 +202,7 @@ def run_reference(args, w):
     per_step_budget = max(0.5, 150.0 / max(1, args.steps + args.warmup))
     times, samples = [], []
     for i in range(args.warmup + args.steps):
-        rate, thr, sample, dt = oracle_rate(w, inp, per_step_budget, threads)
+        rate, thr, sample, dt = oracle_rate(w, inp, per_step_budget, threads, args.cons)
         if i >= args.warmup:
             times.append(dt)
             samples.append(sample)
@@ -213,7 +214,8 @@ def run_reference(args, w):
         "ms_per_step": 1e3 * sum(times) / len(times), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": w.name, "B": w.B, "n": w.n, "d": w.d, "m": w.m, "N": w.N,
-                   "acquisition": w.mode, "S": w.S, "k": w.k, "l2": "n/a (CPU)"},
+                   "acquisition": w.mode, "S": w.S, "k": w.k, "l2": "n/a (CPU)",
+                   **({"constraints": args.constraints} if args.cons else {})},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
                          "sample": f"{samples[0]} of {w.N} candidates of problem 0 per step, "
                                    "full fit + front + posterior + acquisition + top-k"},
@@ -232,8 +234,14 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=0, help="0: same as --steps (max 200)")
+    ap.add_argument("--constraints", default="",
+                    help="comma-separated thresholds on the standardised, minimised objectives "
+                         "(constrained acquisition; 'inf' leaves an objective unconstrained)")
     args = ap.parse_args()
     w = wl.by_name(args.workload)
+    args.cons = [float(c) for c in args.constraints.split(",")] if args.constraints else None
+    if args.cons is not None and len(args.cons) != w.m:
+        ap.error(f"--constraints needs {w.m} values")
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", 1))
     local = int(os.environ.get("LOCAL_RANK", 0))
@@ -261,6 +269,8 @@ def main():
     dXc, deps = t(inp["Xc"], f32), t(inp["eps"], f32)
     mode = bt.BOUTE_ACQ_MC_HVI if w.mode == "mc" else bt.BOUTE_ACQ_EHVI2D
     e = bt.Engine(w.B, w.n, w.d, w.m, w.N, mode, w.S, w.k)
+    if args.cons is not None:
+        bt.boute_engine_set_constraints(e, torch.tensor([args.cons] * w.B, dtype=f64))
     idx = torch.empty((w.B, w.k), dtype=torch.int64, device=dev)
     val = torch.empty((w.B, w.k), dtype=f32, device=dev)
     args_dev = (dX, dY, dls, ds2, dnz, dref, dXc, deps, idx, val)
@@ -356,7 +366,7 @@ def main():
                 "algorithmic_per_launch": rf["per_launch"]}
         cpu = None
         if world == 1 and not args.no_cpu_baseline:
-            rate, thr, sample, dt = oracle_rate(w, inp, 12.0)
+            rate, thr, sample, dt = oracle_rate(w, inp, 12.0, cons=args.cons)
             cpu = {"value": rate, "unit": UNIT, "cores": thr, "kind": "oracle",
                    "sample": f"{sample} of {w.N} candidates of problem 0 ({dt:.1f} s), full fit "
                              "+ front + posterior + acquisition + top-k"}
@@ -367,7 +377,8 @@ def main():
             "data": "synthetic",
             "config": {"workload": w.name, "B": w.B, "n": w.n, "d": w.d, "m": w.m, "N": w.N,
                        "acquisition": w.mode, "S": w.S, "k": w.k,
-                       "l2": "flushed between steps (512 MB write)", "parallelism": "replicas"},
+                       "l2": "flushed between steps (512 MB write)", "parallelism": "replicas",
+                       **({"constraints": args.constraints} if args.cons else {})},
             "roofline": roof,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,

@@ -64,8 +64,8 @@ def acquisition(fp: FittedProblem, mean, var, mode: str, eps=None, threads: int 
     raise ValueError(mode)
 
 
-def score(fp: FittedProblem, Xc, mode: str, k: int, eps=None, threads: int = 0):
+def score(fp: FittedProblem, Xc, mode: str, k: int, eps=None, threads: int = 0, cons=None):
     mean, var = posterior(fp, Xc, threads)
-    acq = acquisition(fp, mean, var, mode, eps, threads)
+    acq = acquisition(fp, mean, var, mode, eps, threads, cons=cons)
     idx, val = topk(acq, k)
     return mean, var, acq, idx, val
