@@ -54,6 +54,19 @@ def lib():
         L.bo_gp_posterior.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp, ctypes.c_double,
                                       _dp, _dp, _fp, ctypes.c_longlong, _dp, _dp, ctypes.c_int]
         L.bo_gp_posterior.restype = None
+        L.bo_matern32.argtypes = [_dp, _dp, ctypes.c_int, _dp, ctypes.c_double]
+        L.bo_matern32.restype = ctypes.c_double
+        L.bo_pref_weight.argtypes = [_dp, ctypes.c_int, ctypes.c_double, _dp]
+        L.bo_pref_weight.restype = ctypes.c_double
+        L.bo_kernel.argtypes = [_dp, _dp, ctypes.c_int, _dp, ctypes.c_double, ctypes.c_int, _dp]
+        L.bo_kernel.restype = ctypes.c_double
+        L.bo_outcome_transform.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _ip, _dp]
+        L.bo_gp_fit_k.argtypes = [_dp, _dp, ctypes.c_int, ctypes.c_int, _dp, ctypes.c_double,
+                                  ctypes.c_double, ctypes.c_int, _dp, _dp, _dp]
+        L.bo_gp_posterior_k.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp, ctypes.c_double,
+                                        ctypes.c_int, _dp, _dp, _dp, _fp, ctypes.c_longlong, _dp,
+                                        _dp, ctypes.c_int]
+        L.bo_gp_posterior_k.restype = None
         L.bo_pareto_front.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp, _bp, _ip]
         L.bo_hv.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp, _dp]
         L.bo_hv.restype = ctypes.c_double
@@ -108,16 +121,67 @@ def matern52(a, b, ls, s2=1.0) -> float:
     return float(lib().bo_matern52(pa, pb, a.size, pl, s2))
 
 
-def gp_fit(X, y, ls, s2, noise):
-    """Returns (L, alpha); raises NotPositiveDefinite on a failed pivot."""
+def matern32(a, b, ls, s2=1.0) -> float:
+    a, pa = _d(a)
+    b, pb = _d(b)
+    ls, pl = _d(ls)
+    return float(lib().bo_matern32(pa, pb, a.size, pl, s2))
+
+
+def pref_weight(c, beta, pref) -> float:
+    c, pc = _d(c)
+    pref, pp = _d(pref)
+    return float(lib().bo_pref_weight(pc, c.size, float(beta), pp))
+
+
+def _kern(kernel):
+    """kernel: None (Matern-5/2) or (dtau, kc) with kc = [s2_c, s2_x, beta, pref...]."""
+    if kernel is None:
+        return 0, None, None
+    dtau, kc = kernel
+    kc, pk = _d(kc)
+    return int(dtau), kc, pk
+
+
+def kernel(a, b, ls, s2=1.0, kernel=None) -> float:
+    """The GP's kernel k(a, b): Matern-5/2 (kernel None) or the composite
+    kernel (dtau, kc) of Sec. 5.2."""
+    a, pa = _d(a)
+    b, pb = _d(b)
+    ls, pl = _d(ls)
+    dtau, kc, pk = _kern(kernel)
+    return float(lib().bo_kernel(pa, pb, a.size, pl, float(s2), dtau, pk))
+
+
+def outcome_transform(Y, codes):
+    """Per-objective transforms before Standardize: codes[t] & 3 = 0 identity,
+    1 log, 2 logit; bit 4 negates."""
+    Y, pY = _d(Y)
+    n, m = Y.shape
+    codes = np.ascontiguousarray(codes, np.int32)
+    out = np.empty_like(Y)
+    rc = lib().bo_outcome_transform(pY, n, m, codes.ctypes.data_as(_ip), out.ctypes.data_as(_dp))
+    if rc:
+        raise ValueError(rc)
+    return out
+
+
+def gp_fit(X, y, ls, s2, noise, kernel=None):
+    """Returns (L, alpha); raises NotPositiveDefinite on a failed pivot.
+    kernel: None (Matern-5/2) or (dtau, kc), the composite kernel."""
     X, pX = _d(X)
     y, py = _d(y)
     ls, pl = _d(ls)
     n, d = X.shape
     L = np.empty((n, n))
     alpha = np.empty(n)
-    rc = lib().bo_gp_fit(pX, py, n, d, pl, float(s2), float(noise), L.ctypes.data_as(_dp),
-                         alpha.ctypes.data_as(_dp))
+    dtau, kc, pk = _kern(kernel)
+    if kc is None:
+        rc = lib().bo_gp_fit(pX, py, n, d, pl, float(s2), float(noise), L.ctypes.data_as(_dp),
+                             alpha.ctypes.data_as(_dp))
+    else:
+        rc = lib().bo_gp_fit_k(pX, py, n, d, pl, float(s2), float(noise), dtau, pk,
+                               L.ctypes.data_as(_dp), alpha.ctypes.data_as(_dp))
     if rc == 2:
         raise NotPositiveDefinite("kernel matrix not positive definite")
     if rc:
@@ -125,7 +189,7 @@ def gp_fit(X, y, ls, s2, noise):
     return L, alpha
 
 
-def gp_posterior(X, ls, s2, L, alpha, Xc, threads: int = 0):
+def gp_posterior(X, ls, s2, L, alpha, Xc, threads: int = 0, kernel=None):
     """Posterior mean and variance (fp64) at fp32 candidates Xc (N x d)."""
     X, pX = _d(X)
     ls, pl = _d(ls)
@@ -136,8 +200,13 @@ def gp_posterior(X, ls, s2, L, alpha, Xc, threads: int = 0):
     N = Xc.shape[0]
     mean = np.empty(N)
     var = np.empty(N)
-    lib().bo_gp_posterior(pX, n, d, pl, float(s2), pL, pa, pc, N, mean.ctypes.data_as(_dp),
-                          var.ctypes.data_as(_dp), threads)
+    dtau, kc, pk = _kern(kernel)
+    if kc is None:
+        lib().bo_gp_posterior(pX, n, d, pl, float(s2), pL, pa, pc, N, mean.ctypes.data_as(_dp),
+                              var.ctypes.data_as(_dp), threads)
+    else:
+        lib().bo_gp_posterior_k(pX, n, d, pl, float(s2), dtau, pk, pL, pa, pc, N,
+                                mean.ctypes.data_as(_dp), var.ctypes.data_as(_dp), threads)
     return mean, var
 
 

@@ -56,16 +56,71 @@ double bo_matern52(const double *a, const double *b, int d, const double *ls, do
   return s2 * (1.0 + sr + 5.0 * r2 / 3.0) * exp(-sr);
 }
 
+/* ---- Sec. 6 (ii): ARD Matern-3/2 with ScaleKernel ------------------------ */
+double bo_matern32(const double *a, const double *b, int d, const double *ls, double s2) {
+  double r2 = 0.0;
+  for (int t = 0; t < d; ++t) {
+    double z = (a[t] - b[t]) / ls[t];
+    r2 += z * z;
+  }
+  double sr = sqrt(3.0) * sqrt(r2);
+  return s2 * (1.0 + sr) * exp(-sr);
+}
+
+/* ---- Sec. 5.2 S1-S3 / S5: preference weight of a deployment --------------- */
+double bo_pref_weight(const double *c, int dc, double beta, const double *pref) {
+  double e = 0.0;
+  for (int k = 0; k < dc; ++k) e += pref[k] * c[k];
+  return exp(beta * e);
+}
+
+/* ---- Sec. 5.2 "Additive kernels" and Sec. 6 (i)-(iv): the GP's kernel ------ */
+double bo_kernel(const double *a, const double *b, int d, const double *ls, double s2,
+                 int dtau, const double *kc) {
+  if (!kc) return bo_matern52(a, b, d, ls, s2);
+  const int dc = d - dtau;
+  /* the base kernels, unscaled: k_tau over the routing features, k_c over the
+   * deployment features (ProductKernel(k_tau, k_c) reuses both) */
+  double ktau = bo_matern52(a, b, dtau, ls, 1.0);
+  double kcd = bo_matern32(a + dtau, b + dtau, dc, ls + dtau, 1.0);
+  double wa = bo_pref_weight(a + dtau, dc, kc[2], kc + 3);
+  double wb = bo_pref_weight(b + dtau, dc, kc[2], kc + 3);
+  return s2 * ktau + kc[0] * wa * wb * kcd + kc[1] * ktau * kcd;
+}
+
+/* ---- Sec. 5.2 S4: outcome transforms applied before Standardize ----------- */
+int bo_outcome_transform(const double *Y, int n, int m, const int *codes, double *Yt) {
+  if (n < 0 || m < 1 || (n > 0 && (!Y || !Yt))) return 1;
+  for (int i = 0; i < n; ++i)
+    for (int t = 0; t < m; ++t) {
+      double y = Y[(long)i * m + t];
+      int c = codes ? codes[t] : 0;
+      double v = y;
+      if ((c & 3) == 1) v = log(y);                  /* latency: log */
+      else if ((c & 3) == 2) v = log(y / (1.0 - y)); /* quality: logit */
+      if (c & 4) v = -v;                             /* a maximised outcome, minimised */
+      Yt[(long)i * m + t] = v;
+    }
+  return 0;
+}
+
 /* ---- Sec. 5.2 (i) / Sec. 6: exact GP fit --------------------------------- */
 int bo_gp_fit(const double *X, const double *y, int n, int d, const double *ls,
               double s2, double noise, double *L, double *alpha) {
+  return bo_gp_fit_k(X, y, n, d, ls, s2, noise, d, NULL, L, alpha);
+}
+
+int bo_gp_fit_k(const double *X, const double *y, int n, int d, const double *ls, double s2,
+                double noise, int dtau, const double *kc, double *L, double *alpha) {
   if (n < 1 || d < 1 || !X || !y || !ls || !L || !alpha) return 1;
-  /* K = s2 M52(X, X) + noise I, lower triangle written straight into L */
+  if (kc && (dtau < 0 || dtau > d)) return 1;
+  /* K = k(X, X) + noise I, lower triangle written straight into L */
   for (int i = 0; i < n; ++i)
     for (int j = 0; j < n; ++j)
-      L[(long)i * n + j] = j <= i ? bo_matern52(X + (long)i * d, X + (long)j * d, d, ls, s2) +
-                                        (i == j ? noise : 0.0)
-                                  : 0.0;
+      L[(long)i * n + j] =
+          j <= i ? bo_kernel(X + (long)i * d, X + (long)j * d, d, ls, s2, dtau, kc) +
+                       (i == j ? noise : 0.0)
+                 : 0.0;
   /* Cholesky-Banachiewicz, row by row, in place */
   for (int i = 0; i < n; ++i) {
     for (int j = 0; j <= i; ++j) {
@@ -96,7 +151,15 @@ int bo_gp_fit(const double *X, const double *y, int n, int d, const double *ls,
 void bo_gp_posterior(const double *X, int n, int d, const double *ls, double s2,
                      const double *L, const double *alpha, const float *Xc,
                      long long N, double *mean, double *var, int nthreads) {
+  bo_gp_posterior_k(X, n, d, ls, s2, d, NULL, L, alpha, Xc, N, mean, var, nthreads);
+}
+
+void bo_gp_posterior_k(const double *X, int n, int d, const double *ls, double s2, int dtau,
+                       const double *kc, const double *L, const double *alpha, const float *Xc,
+                       long long N, double *mean, double *var, int nthreads) {
   int nt = nthreads_or_default(nthreads);
+  /* prior variance k(x, x): s2 for the Matern-5/2 kernel; for the composite
+   * kernel it depends on x through the preference weight */
 #pragma omp parallel num_threads(nt)
   {
     double *kv = (double *)malloc(sizeof(double) * (size_t)(2 * n + d));
@@ -106,7 +169,7 @@ void bo_gp_posterior(const double *X, int n, int d, const double *ls, double s2,
       for (int t = 0; t < d; ++t) xc[t] = (double)Xc[c * d + t];
       double mu = 0.0;
       for (int j = 0; j < n; ++j) {
-        kv[j] = bo_matern52(xc, X + (long)j * d, d, ls, s2);
+        kv[j] = bo_kernel(xc, X + (long)j * d, d, ls, s2, dtau, kc);
         mu += kv[j] * alpha[j];
       }
       double vv = 0.0;
@@ -116,7 +179,7 @@ void bo_gp_posterior(const double *X, int n, int d, const double *ls, double s2,
         v[i] = s / L[(long)i * n + i];
         vv += v[i] * v[i];
       }
-      double s2v = s2 - vv;
+      double s2v = bo_kernel(xc, xc, d, ls, s2, dtau, kc) - vv;
       mean[c] = mu;
       var[c] = s2v > 0.0 ? s2v : 0.0;
     }

@@ -28,6 +28,33 @@ int bo_standardize(const double *Y, int n, int m, double *Ys);
  * r^2 = sum_t ((a_t - b_t) / ls_t)^2. */
 double bo_matern52(const double *a, const double *b, int d, const double *ls, double s2);
 
+/* ARD Matern-3/2 kernel with outputscale (Sec. 6 (ii): MaternKernel nu=1.5):
+ * s2 (1 + sqrt3 r) exp(-sqrt3 r), r as for bo_matern52. */
+double bo_matern32(const double *a, const double *b, int d, const double *ls, double s2);
+
+/* Preference weight of a deployment (Sec. 5.2 S5): w(c) = exp(beta sum_k
+ * pref_k c_k), with c the allocation counts a_{m,n} flattened (dc entries) and
+ * pref the matching entries s_{m,n} of the preference matrix. */
+double bo_pref_weight(const double *c, int dc, double beta, const double *pref);
+
+/* The GP's kernel. kc = NULL: the ARD Matern-5/2 kernel above (s2). Otherwise
+ * the composite kernel of Sec. 5.2 ("Additive kernels", S5) as Sec. 6
+ * assembles it, the routing features tau = x[0, dtau), the deployment
+ * features c = x[dtau, d):
+ *   k = s2 k52(tau, tau*) + kc[0] w(c) w(c*) k32(c, c*) + kc[1] k52(tau, tau*) k32(c, c*)
+ * with k52, k32 the unscaled ARD Matern kernels (lengthscales ls[0, dtau) and
+ * ls[dtau, d)), kc[0] and kc[1] the outputscales of the preference-weighted
+ * deployment kernel and of the interaction (phi), kc[2] = beta and
+ * kc[3 .. 3 + d - dtau) = pref. */
+double bo_kernel(const double *a, const double *b, int d, const double *ls, double s2,
+                 int dtau, const double *kc);
+
+/* Outcome transforms before Standardize (Sec. 5.2 S4; Sec. 6): per objective
+ * t, codes[t] & 3 = 0 identity, 1 log (latency), 2 logit (quality); bit 4
+ * negates (a maximised outcome becomes a minimised one). codes = NULL: all
+ * identity. Y, Yt: n x m. Values outside a transform's domain give NaN. */
+int bo_outcome_transform(const double *Y, int n, int m, const int *codes, double *Yt);
+
 /* Exact GP fit with fixed hyperparameters (Sec. 5.2 step (i); Sec. 6
  * SingleTaskGP, zero prior mean on standardised outcomes):
  * K = s2 M52(X, X) + noise I, L = chol(K) (Cholesky-Banachiewicz, no jitter),
@@ -36,6 +63,9 @@ double bo_matern52(const double *a, const double *b, int d, const double *ls, do
  * Returns 2 when a pivot is not positive. */
 int bo_gp_fit(const double *X, const double *y, int n, int d, const double *ls,
               double s2, double noise, double *L, double *alpha);
+/* The same with the kernel bo_kernel(., ., d, ls, s2, dtau, kc). */
+int bo_gp_fit_k(const double *X, const double *y, int n, int d, const double *ls, double s2,
+                double noise, int dtau, const double *kc, double *L, double *alpha);
 
 /* Latent-function posterior at fp32 candidates (cast to double):
  * mean = k*^T alpha, var = max(0, s2 - v^T v) with v = L^-1 k* by forward
@@ -43,6 +73,11 @@ int bo_gp_fit(const double *X, const double *y, int n, int d, const double *ls,
 void bo_gp_posterior(const double *X, int n, int d, const double *ls, double s2,
                      const double *L, const double *alpha, const float *Xc,
                      long long N, double *mean, double *var, int nthreads);
+/* The same with the kernel bo_kernel(., ., d, ls, s2, dtau, kc); the prior
+ * variance is k(x, x), which depends on x through the preference weight. */
+void bo_gp_posterior_k(const double *X, int n, int d, const double *ls, double s2, int dtau,
+                       const double *kc, const double *L, const double *alpha, const float *Xc,
+                       long long N, double *mean, double *var, int nthreads);
 
 /* Pareto front of observed outcomes (Sec. 5.2, Pareto-optimal set; all
  * objectives minimised): point i is kept iff no j dominates it (Y_j <= Y_i in

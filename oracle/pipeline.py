@@ -12,7 +12,8 @@ from dataclasses import dataclass
 
 import numpy as np
 
-from . import (ehvi2d, gp_fit, gp_posterior, mc_hvi, pareto_front, standardize, topk)
+from . import (ehvi2d, gp_fit, gp_posterior, mc_hvi, outcome_transform, pareto_front, standardize,
+               topk)
 
 
 @dataclass
@@ -27,19 +28,27 @@ class FittedProblem:
     ref: np.ndarray
     mask: np.ndarray  # front membership (n,)
     front: np.ndarray  # P x m, sorted
+    kernel: list | None = None  # per objective (dtau, kc) of the composite kernel, or None
 
 
-def fit_problem(X, Y, ls, s2, noise, ref) -> FittedProblem:
+def fit_problem(X, Y, ls, s2, noise, ref, kernel=None, transforms=None) -> FittedProblem:
+    """kernel: None (Matern-5/2) or (dtau, kc) with kc m x (3 + d - dtau), one
+    row [s2_c, s2_x, beta, pref...] per objective (the composite kernel);
+    transforms: None or m outcome-transform codes applied before Standardize."""
+    if transforms is not None:
+        Y = outcome_transform(Y, transforms)
     Ys = standardize(Y)
+    kern = None if kernel is None else [(kernel[0], np.asarray(kernel[1], np.float64)[t])
+                                        for t in range(Ys.shape[1])]
     Ls, alphas = [], []
     for t in range(Ys.shape[1]):
-        L, a = gp_fit(X, Ys[:, t], ls[t], s2[t], noise[t])
+        L, a = gp_fit(X, Ys[:, t], ls[t], s2[t], noise[t], None if kern is None else kern[t])
         Ls.append(L)
         alphas.append(a)
     mask, order = pareto_front(Ys, ref)
     return FittedProblem(np.asarray(X, np.float64), Ys, np.asarray(ls, np.float64),
                          np.asarray(s2, np.float64), np.asarray(noise, np.float64), Ls, alphas,
-                         np.asarray(ref, np.float64), mask, Ys[order])
+                         np.asarray(ref, np.float64), mask, Ys[order], kern)
 
 
 def posterior(fp: FittedProblem, Xc, threads: int = 0):
@@ -50,7 +59,7 @@ def posterior(fp: FittedProblem, Xc, threads: int = 0):
     var = np.empty((Xc.shape[0], m))
     for t in range(m):
         mean[:, t], var[:, t] = gp_posterior(fp.X, fp.ls[t], fp.s2[t], fp.L[t], fp.alpha[t], Xc,
-                                             threads)
+                                             threads, None if fp.kernel is None else fp.kernel[t])
     return mean, var
 
 

@@ -19,6 +19,17 @@ large 2-objective workload adds 0.1 sin(2 pi x_0) to f1, and the 3-objective
 workload adds f3(x) = 1 - exp(-||x - 0.5 1||^2 / (0.1 d)). The noise term
 "N(0, 1e-4)" is read as variance 1e-4 (standard deviation 0.01).
 
+Composite-kernel variants (`composite(w)`) stand in for the paper's decision
+vector theta = (tau, c) more closely: the first d_tau = d // 2 features are
+routing features in [0, 1], the rest are deployment features, GPU counts in
+{0, .., 4} (the allocations a_{m,n} of Sec. 5.2 S5), and the outcomes are a
+positive latency L = exp(f1 + e1) and a quality Q = 1 / (1 + exp(f2 + e2)) in
+(0, 1) (to be maximised), with f1, f2 evaluated at x with the counts divided
+by 4. The GP then uses the composite kernel with the Log and negated Logit
+outcome transforms; its extra hyperparameters (interaction and deployment
+outputscales, preference strength beta, preference entries s_{m,n} ~ U[0, 1])
+come from `kernel_params`.
+
 Random-access generation: candidates and base normals are drawn in blocks of
 CHUNK candidates, block j from SeedSequence([seed, stream, j]), so any slice
 of a multi-gigabyte input can be regenerated on its own (the oracle checks
@@ -26,6 +37,7 @@ sampled candidates of full-size workloads that way).
 """
 from __future__ import annotations
 
+import dataclasses
 import math
 from concurrent.futures import ThreadPoolExecutor
 from dataclasses import dataclass, field
@@ -35,7 +47,8 @@ import numpy as np
 CHUNK = 8192  # candidates per independently seeded block
 
 # stream ids within one seed
-_S_TRAIN_X, _S_NOISE, _S_CAND, _S_EPS, _S_SHIFT = 0, 1, 2, 3, 4
+_S_TRAIN_X, _S_NOISE, _S_CAND, _S_EPS, _S_SHIFT, _S_PREF = 0, 1, 2, 3, 4, 5
+MAX_COUNT = 4  # deployment features of composite variants: GPU counts 0 .. MAX_COUNT
 
 
 @dataclass(frozen=True)
@@ -57,6 +70,8 @@ class Workload:
     sine_term: bool = False  # add 0.1 sin(2 pi x_0) to f1
     shifted: bool = False  # per-problem shift c_i ~ U[0.1, 0.4]
     ref: tuple = field(default=())  # reference point in standardised units
+    d_tau: int = 0  # composite kernel: routing features [0, d_tau); 0 = Matern-5/2 kernel
+    transforms: tuple = field(default=())  # outcome-transform codes per objective, or ()
 
     def lengthscale(self) -> float:
         return 0.2 * math.sqrt(self.d)
@@ -79,10 +94,19 @@ WORKLOADS = [
 ]
 
 
+def composite(w: Workload) -> Workload:
+    """The same shapes with the composite kernel's decision vectors and
+    outcomes (routing + deployment features, latency and quality)."""
+    codes = (1, 6) + (0,) * (w.m - 2)  # log latency, negated logit quality
+    return dataclasses.replace(w, name=w.name + "-composite", d_tau=w.d // 2, transforms=codes)
+
+
 def by_name(name: str) -> Workload:
     for w in WORKLOADS:
         if w.name == name:
             return w
+        if w.name + "-composite" == name:
+            return composite(w)
     raise KeyError(name)
 
 
@@ -93,7 +117,7 @@ def scaled(w: Workload, *, N: int | None = None, B: int | None = None,
     return Workload(w.name + "-scaled", B2, w.n if n is None else n, w.d, w.m,
                     w.N if N is None else N, w.mode, w.S if S is None else S,
                     min(w.k, w.N if N is None else N), w.seeds[:B2], w.eps_seed,
-                    w.sine_term, w.shifted, w.ref)
+                    w.sine_term, w.shifted, w.ref, w.d_tau, w.transforms)
 
 
 def _rng(*key) -> np.random.Generator:
@@ -122,18 +146,48 @@ def objectives(w: Workload, b: int, X: np.ndarray) -> np.ndarray:
     return np.stack(cols, 1)
 
 
+def _counts(U: np.ndarray, w: Workload) -> np.ndarray:
+    """Composite variants: uniform draws in [0, 1) of the deployment features
+    become GPU counts 0 .. MAX_COUNT (in place)."""
+    if w.d_tau:
+        U[:, w.d_tau:] = np.floor(U[:, w.d_tau:] * (MAX_COUNT + 1))
+    return U
+
+
 def training_set(w: Workload, b: int = 0):
     """Observed points of problem b: X (n x d fp64), raw noisy Y (n x m fp64)."""
-    X = _rng(w.seeds[b], _S_TRAIN_X).random((w.n, w.d))
+    X = _counts(_rng(w.seeds[b], _S_TRAIN_X).random((w.n, w.d)), w)
     noise = _rng(w.seeds[b], _S_NOISE).normal(0.0, 0.01, (w.n, w.m))
-    return X, objectives(w, b, X) + noise
+    if not w.d_tau:
+        return X, objectives(w, b, X) + noise
+    Xh = X.copy()
+    Xh[:, w.d_tau:] /= MAX_COUNT
+    F = objectives(w, b, Xh) + noise
+    Y = F.copy()
+    Y[:, 0] = np.exp(F[:, 0])  # latency
+    Y[:, 1] = 1.0 / (1.0 + np.exp(F[:, 1]))  # quality, to be maximised
+    return X, Y
 
 
 def hyperparameters(w: Workload, b: int = 0):
     """Fixed GP hyperparameters per objective: ARD lengthscales (m x d),
     outputscale (m,), noise variance (m,), in standardised units."""
     ls = np.full((w.m, w.d), w.lengthscale())
+    if w.d_tau:
+        ls[:, w.d_tau:] *= MAX_COUNT  # the deployment features span 0 .. MAX_COUNT
     return ls, np.ones(w.m), np.full(w.m, 1e-4)
+
+
+def kernel_params(w: Workload, b: int = 0):
+    """Composite variants: (d_tau, kc), kc m x (3 + d - d_tau), per objective
+    [deployment outputscale, interaction outputscale (phi), beta, preference
+    entries ~ U[0, 1]]; None for the Matern-5/2 workloads."""
+    if not w.d_tau:
+        return None
+    dc = w.d - w.d_tau
+    pref = _rng(w.seeds[b], _S_PREF).random((w.m, dc))
+    kc = np.concatenate([np.tile([0.5, 0.1, 0.05], (w.m, 1)), pref], 1)
+    return w.d_tau, kc
 
 
 def ref_point(w: Workload) -> np.ndarray:
@@ -172,8 +226,8 @@ def candidates(w: Workload, b: int, start: int = 0, count: int | None = None,
     count = w.N - start if count is None else count
     out = np.empty((count, w.d), np.float32)
     return _fill(out, start, count,
-                 lambda j: _rng(w.seeds[b], _S_CAND, j).random((CHUNK, w.d)).astype(np.float32),
-                 threads)
+                 lambda j: _counts(_rng(w.seeds[b], _S_CAND, j).random((CHUNK, w.d)),
+                                   w).astype(np.float32), threads)
 
 
 def base_normals(w: Workload, b: int, start: int = 0, count: int | None = None,

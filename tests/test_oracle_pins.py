@@ -539,3 +539,145 @@ def test_constrained_acquisition_limits():
         prev = e
     assert np.all(oracle.ehvi2d(mu, var, F, ref, cons=np.array([-40.0, 0.0])) < 1e-300)
     np.testing.assert_allclose(prev, free, rtol=1e-12, atol=1e-15)  # c far above every sample
+
+
+# ------------------------------- composite kernel and outcome transforms (Sec. 5.2, Sec. 6)
+def _kc(s2_c, s2_x, beta, pref):
+    return np.concatenate([[s2_c, s2_x, beta], np.asarray(pref, np.float64)])
+
+
+@pytest.mark.parametrize("r", [0.0, 1e-3, 0.3, 1.0, 2.5, 6.0])
+def test_matern32_equals_general_matern_at_nu_1p5(r):
+    ls = np.array([0.8, 2.0, 1.3])
+    u = np.array([-0.4, 0.3, 0.7])
+    u = u / np.linalg.norm(u / ls) * r if r > 0 else np.zeros(3)
+    a = np.array([1.0, 2.0, 0.5])
+    got = oracle.matern32(a, a + u, ls, 0.6)
+    assert got == pytest.approx(_matern_bessel(r, 1.5, 0.6), rel=1e-12, abs=1e-300)
+
+
+def test_preference_weight_hand_values():
+    # w(c) = exp(beta <s, a>): allocations (2, 4) with suitabilities (0.5, 0.25)
+    assert oracle.pref_weight([2.0, 4.0], 0.1, [0.5, 0.25]) == pytest.approx(math.exp(0.2),
+                                                                             rel=1e-15)
+    assert oracle.pref_weight([2.0, 4.0], 0.0, [0.5, 0.25]) == 1.0
+
+
+def test_composite_routing_term_alone_is_matern52_of_the_routing_features():
+    rng = np.random.default_rng(21)
+    a, b, ls = rng.random(5), rng.random(5), rng.random(5) + 0.3
+    kc = _kc(0.0, 0.0, 0.3, [0.2, 0.9])
+    got = oracle.kernel(a, b, ls, 1.3, (3, kc))
+    assert got == pytest.approx(oracle.matern52(a[:3], b[:3], ls[:3], 1.3), rel=1e-15)
+    b2 = b.copy(); b2[3:] += 5.0  # the deployment features do not enter this term
+    assert oracle.kernel(a, b2, ls, 1.3, (3, kc)) == pytest.approx(got, rel=1e-15)
+    # every feature a routing feature: the plain Matern-5/2 kernel
+    assert oracle.kernel(a, b, ls, 1.3, (5, _kc(0.0, 0.0, 0.0, []))) == pytest.approx(
+        oracle.kernel(a, b, ls, 1.3), rel=1e-15)
+
+
+def test_composite_deployment_term_worked_example():
+    # k~_c = s2_c w(c) w(c*) k32(c, c*), routing features irrelevant:
+    # c = (2, 1), c* = (0, 3), lengthscales (2, 1): r^2 = 1 + 4 = 5;
+    # w(c) = exp(0.1 (0.5*2 + 0.25*1)) = exp(0.125), w(c*) = exp(0.075)
+    a = np.array([0.3, 2.0, 1.0])
+    b = np.array([0.9, 0.0, 3.0])
+    ls = np.array([0.5, 2.0, 1.0])
+    kc = _kc(0.7, 0.0, 0.1, [0.5, 0.25])
+    sr = math.sqrt(3.0 * 5.0)
+    want = 0.7 * math.exp(0.2) * (1.0 + sr) * math.exp(-sr)
+    assert oracle.kernel(a, b, ls, 0.0, (1, kc)) == pytest.approx(want, rel=1e-14)
+    b2 = b.copy(); b2[0] = -4.0
+    assert oracle.kernel(a, b2, ls, 0.0, (1, kc)) == pytest.approx(want, rel=1e-14)
+    # at zero distance: s2_c w(c)^2
+    assert oracle.kernel(a, a, ls, 0.0, (1, kc)) == pytest.approx(0.7 * math.exp(0.25),
+                                                                  rel=1e-15)
+
+
+def test_composite_interaction_term_is_a_product():
+    # s2_x alone: k(a, b) = k52(tau, tau*) k32(c, c*), so it factorises into
+    # the value with only the routing features moved times the value with
+    # only the deployment features moved; each factor is pinned above
+    rng = np.random.default_rng(22)
+    a, b, ls = rng.random(6), rng.random(6) * 3, rng.random(6) + 0.4
+    kc = _kc(0.0, 0.35, 0.2, rng.random(2))
+    dt = 4
+    ab_tau = np.concatenate([b[:dt], a[dt:]])
+    ab_c = np.concatenate([a[:dt], b[dt:]])
+    k = lambda u, v: oracle.kernel(u, v, ls, 0.0, (dt, kc))
+    assert k(a, b) == pytest.approx(k(a, ab_tau) * k(a, ab_c) / 0.35, rel=1e-13)
+    assert k(a, ab_c) == pytest.approx(0.35 * oracle.matern32(a[dt:], b[dt:], ls[dt:]),
+                                       rel=1e-14)
+    assert k(a, ab_tau) == pytest.approx(0.35 * oracle.matern52(a[:dt], b[:dt], ls[:dt]),
+                                         rel=1e-14)
+
+
+def test_composite_terms_add_with_their_own_scales():
+    rng = np.random.default_rng(23)
+    a, b, ls = rng.random(5), rng.random(5) * 2, rng.random(5) + 0.3
+    pref = rng.random(2)
+    k = lambda s2, sc, sx: oracle.kernel(a, b, ls, s2, (3, _kc(sc, sx, 0.15, pref)))
+    assert k(1.1, 0.4, 0.07) == pytest.approx(k(1.1, 0, 0) + k(0, 0.4, 0) + k(0, 0, 0.07),
+                                              rel=1e-14)
+
+
+def test_composite_gram_matrix_is_positive_semidefinite():
+    rng = np.random.default_rng(24)
+    X = np.concatenate([rng.random((60, 3)), rng.integers(0, 5, (60, 4))], 1).astype(float)
+    ls = np.array([0.4, 0.5, 0.6, 1.5, 2.0, 1.0, 1.8])
+    kc = _kc(0.5, 0.1, 0.05, rng.random(4))
+    K = np.array([[oracle.kernel(x, y, ls, 1.0, (3, kc)) for y in X] for x in X])
+    np.testing.assert_allclose(K, K.T, rtol=0, atol=0)
+    ev = np.linalg.eigvalsh(K)
+    assert ev.min() > -1e-12 * ev.max()
+
+
+def test_composite_posterior_matches_schur_complement_by_library_solve():
+    # the pipeline's fit and posterior with the composite kernel and outcome
+    # transforms, against a library solve on the same kernel's Gram matrices
+    # (prior variance k(x, x), which varies with the preference weight)
+    rng = np.random.default_rng(25)
+    n, dt, dc = 40, 3, 3
+    X = np.concatenate([rng.random((n, dt)), rng.integers(0, 5, (n, dc))], 1).astype(float)
+    lat = np.exp(rng.normal(0, 0.5, n))
+    qual = 1.0 / (1.0 + np.exp(-rng.normal(0, 1.0, n)))
+    Y = np.stack([lat, qual], 1)
+    ls = np.tile(np.array([0.4, 0.5, 0.6, 1.5, 2.0, 1.0]), (2, 1))
+    s2, noise = np.array([1.0, 0.8]), np.array([1e-3, 2e-3])
+    kc = np.stack([_kc(0.5, 0.1, 0.05, rng.random(dc)), _kc(0.3, 0.2, -0.04, rng.random(dc))])
+    fp = pipeline.fit_problem(X, Y, ls, s2, noise, np.array([2.0, 2.0]), kernel=(dt, kc),
+                              transforms=[1, 6])
+    y = oracle.standardize(np.stack([np.log(lat), -np.log(qual / (1 - qual))], 1))
+    np.testing.assert_allclose(fp.Ys, y, rtol=1e-12, atol=1e-12)
+    Xc = np.concatenate([rng.random((25, dt)), rng.integers(0, 5, (25, dc))], 1)
+    Xc = Xc.astype(np.float32)
+    mean, var = pipeline.posterior(fp, Xc)
+    for t in range(2):
+        k = lambda u, v: oracle.kernel(u, v, ls[t], s2[t], (dt, kc[t]))
+        K = np.array([[k(u, v) for v in X] for u in X]) + noise[t] * np.eye(n)
+        Ks = np.array([[k(c.astype(np.float64), x) for x in X] for c in Xc])
+        prior = np.array([k(c.astype(np.float64), c.astype(np.float64)) for c in Xc])
+        np.testing.assert_allclose(mean[:, t], Ks @ scipy.linalg.solve(K, y[:, t]), rtol=1e-9,
+                                   atol=1e-10)
+        sol = scipy.linalg.solve(K, Ks.T)
+        np.testing.assert_allclose(var[:, t], prior - np.einsum("ij,ji->i", Ks, sol), rtol=1e-8,
+                                   atol=1e-10)
+        assert np.all(var[:, t] <= prior + 1e-12)
+
+
+def test_outcome_transforms():
+    rng = np.random.default_rng(26)
+    lat = rng.uniform(0.1, 20.0, 30)
+    q = rng.uniform(0.01, 0.99, 30)
+    Y = np.stack([lat, q, q, 1 - q, lat], 1)
+    T = oracle.outcome_transform(Y, [1, 2, 6, 2, 0])
+    np.testing.assert_allclose(T[:, 0], np.log(lat), rtol=1e-15)
+    np.testing.assert_allclose(T[:, 1], scipy.special.logit(q), rtol=1e-13, atol=1e-15)
+    # logit(1 - q) = -logit(q): the negated transform of q equals the plain
+    # transform of 1 - q
+    np.testing.assert_allclose(T[:, 2], T[:, 3], rtol=1e-12, atol=1e-14)
+    np.testing.assert_allclose(T[:, 2], -T[:, 1], rtol=0, atol=0)
+    np.testing.assert_array_equal(T[:, 4], lat)
+    # outside the domain: NaN
+    bad = oracle.outcome_transform(np.array([[-1.0, 1.5]]), [1, 2])
+    assert np.isnan(bad).all()
