@@ -52,12 +52,22 @@ const char *boute_status_string(int status);
  * A monotone counter; differences bracket a region of work. */
 unsigned long long boute_launch_count(void);
 
-/* ---- outcome standardisation ---------------------------------------------
- * Sec. 6 (outcome transform "Standardize", applied after Sec. 5.2 S4's
- * Log/Logit, which stay with the caller): Ys[b,:,t] = (Y[b,:,t] - mean) / std,
- * std with the n-1 denominator; a column with n < 2 or std < 1e-8 is divided
- * by 1. Y, Ys: B x n x m fp64 (may alias). */
-int boute_standardize(const double *Y, int B, int n, int m, double *Ys, void *stream);
+/* ---- outcome transforms and standardisation ------------------------------
+ * Sec. 5.2 S4 and Sec. 6 (outcome transforms Log / Logit, then "Standardize"):
+ * each raw outcome is first transformed per objective, transforms[t] & 3 =
+ * BOUTE_TF_IDENTITY (0), BOUTE_TF_LOG (1, latency) or BOUTE_TF_LOGIT (2,
+ * quality, log(y / (1 - y))), | BOUTE_TF_NEGATE (4) to minimise a maximised
+ * outcome; then Ys[b,:,t] = (z[b,:,t] - mean) / std, std with the n-1
+ * denominator; a column with n < 2 or std < 1e-8 is divided by 1.
+ * transforms: HOST array of m codes, or NULL (all identity); an unknown code
+ * is INVALID_ARG; outcomes outside a transform's domain give NaN.
+ * Y, Ys: B x n x m fp64 (may alias). m <= 4. */
+#define BOUTE_TF_IDENTITY 0
+#define BOUTE_TF_LOG 1
+#define BOUTE_TF_LOGIT 2
+#define BOUTE_TF_NEGATE 4
+int boute_standardize(const double *Y, int B, int n, int m, const int *transforms, double *Ys,
+                      void *stream);
 
 /* ---- GP fit ----------------------------------------------------------------
  * Sec. 5.2 step (i) and Sec. 6: one exact GP per objective (SingleTaskGP
@@ -82,6 +92,23 @@ int boute_gp_fit(boute_gp *gp, const double *X, const double *Ys, const double *
                  const double *outputscale, const double *noise, void *stream);
 int boute_gp_status(boute_gp *gp, void *stream);
 void boute_gp_free(boute_gp *gp);
+/* The paper's composite kernel for the handle's later fits and posteriors
+ * (Sec. 5.2 "Additive kernels" with the preference weighting of S5, as
+ * Sec. 6 assembles it: k_tau + k~_c + k_x, each in its own ScaleKernel):
+ * the first d_tau features are routing features tau, the other d - d_tau
+ * deployment features c (GPU counts a_{m,n}, flattened), and
+ *   k(x, x*) = s2 k52(tau, tau*) + s2_c w(c) w(c*) k32(c, c*)
+ *              + s2_x k52(tau, tau*) k32(c, c*),
+ *   w(c) = exp(beta sum_k s_k c_k),
+ * k52 / k32 the unscaled ARD Matern-5/2 / 3/2 kernels with the fit's
+ * lengthscales of the respective features, s2 the fit's outputscale.
+ * params: HOST array B x m x (3 + d - d_tau) fp64, per problem-objective
+ * [s2_c, s2_x (the interaction weight phi), beta, s_0 .. s_{d-d_tau-1}]
+ * (the preference-matrix entries matching the deployment features); copied
+ * into the handle. params = NULL restores the Matern-5/2 kernel. The prior
+ * variance k(x, x) = s2 + s2_x + s2_c w(c)^2 depends on the candidate.
+ * Waits for all work on the device first. */
+int boute_gp_set_kernel(boute_gp *gp, int d_tau, const double *params);
 
 /* ---- posterior ---------------------------------------------------------------
  * Latent-function posterior of every objective at N candidates per problem
@@ -258,6 +285,14 @@ int boute_engine_launches_per_step(const boute_engine *e);
  * running); the engine's cached step graphs are rebuilt on the next step when
  * constraints are switched on or off. */
 int boute_engine_set_constraints(boute_engine *e, const double *cons);
+/* Outcome transforms for the engine's later steps (see boute_standardize):
+ * codes is a HOST array of m codes, or NULL for none. The steps' raw outcomes
+ * Y are transformed before they are standardised, for the fit and the front
+ * alike. Waits for all work on the device when the codes change. */
+int boute_engine_set_outcome_transforms(boute_engine *e, const int *codes);
+/* The composite kernel for the engine's later steps (see boute_gp_set_kernel;
+ * params is a HOST array, NULL restores the Matern-5/2 kernel). */
+int boute_engine_set_kernel(boute_engine *e, int d_tau, const double *params);
 void boute_engine_free(boute_engine *e);
 
 #ifdef __cplusplus

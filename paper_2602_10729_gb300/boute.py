@@ -17,6 +17,7 @@ from . import build as _build
 BOUTE_OK, BOUTE_ERR_INVALID_ARG, BOUTE_ERR_NOT_PD, BOUTE_ERR_CUDA = 0, 1, 2, 3
 BOUTE_ERR_OOM, BOUTE_ERR_UNSUPPORTED, BOUTE_ERR_TIMEOUT = 4, 5, 6
 BOUTE_ACQ_EHVI2D, BOUTE_ACQ_MC_HVI = 0, 1
+BOUTE_TF_IDENTITY, BOUTE_TF_LOG, BOUTE_TF_LOGIT, BOUTE_TF_NEGATE = 0, 1, 2, 4
 
 #: exported symbols declared in include/boute.h
 SYMBOLS = (
@@ -28,6 +29,7 @@ SYMBOLS = (
     "boute_engine_step_host", "boute_engine_step_host_async", "boute_engine_sync",
     "boute_engine_scores", "boute_engine_set_timing",
     "boute_engine_stage_times", "boute_engine_launches_per_step", "boute_engine_set_constraints",
+    "boute_engine_set_outcome_transforms", "boute_engine_set_kernel", "boute_gp_set_kernel",
     "boute_engine_free",
 )
 #: stage names of boute_engine_stage_times, in order
@@ -61,7 +63,7 @@ def load(path: str | None = None):
     sig = {
         "boute_status_string": ([_i], ctypes.c_char_p),
         "boute_launch_count": ([], ctypes.c_ulonglong),
-        "boute_standardize": ([_vp, _i, _i, _i, _vp, _vp], _i),
+        "boute_standardize": ([_vp, _i, _i, _i, _vp, _vp, _vp], _i),
         "boute_gp_create": ([_i, _i, _i, _i, ctypes.POINTER(_vp)], _i),
         "boute_gp_fit": ([_vp, _vp, _vp, _vp, _vp, _vp, _vp], _i),
         "boute_gp_status": ([_vp, _vp], _i),
@@ -85,6 +87,9 @@ def load(path: str | None = None):
         "boute_engine_stage_times": ([_vp, ctypes.POINTER(ctypes.c_float), _i], _i),
         "boute_engine_launches_per_step": ([_vp], _i),
         "boute_engine_set_constraints": ([_vp, _vp], _i),
+        "boute_engine_set_outcome_transforms": ([_vp, _vp], _i),
+        "boute_engine_set_kernel": ([_vp, _i, _vp], _i),
+        "boute_gp_set_kernel": ([_vp, _i, _vp], _i),
         "boute_engine_free": ([_vp], None),
     }
     for name, (args, res) in sig.items():
@@ -131,10 +136,18 @@ def boute_launch_count() -> int:
     return int(load().boute_launch_count())
 
 
-def boute_standardize(Y, Ys, stream=None):
+def _codes(codes):
+    """A host int array of outcome-transform codes (or None)."""
+    if codes is None:
+        return None
+    return (ctypes.c_int * len(codes))(*[int(c) for c in codes])
+
+
+def boute_standardize(Y, Ys, stream=None, transforms=None):
+    """transforms: None or m outcome-transform codes (BOUTE_TF_*)."""
     B, n, m = Y.shape
-    _check(load().boute_standardize(_p(Y, torch.float64), B, n, m, _p(Ys, torch.float64),
-                                    _s(stream)), "boute_standardize")
+    _check(load().boute_standardize(_p(Y, torch.float64), B, n, m, _codes(transforms),
+                                    _p(Ys, torch.float64), _s(stream)), "boute_standardize")
 
 
 class Gp:
@@ -174,6 +187,19 @@ def boute_gp_status(gp: Gp, stream=None) -> int:
 
 def boute_gp_free(gp: Gp):
     gp.free()
+
+
+def _host_f64(a):
+    import numpy as np
+    return None if a is None else torch.as_tensor(np.ascontiguousarray(a, np.float64))
+
+
+def boute_gp_set_kernel(gp: Gp, d_tau: int = 0, params=None):
+    """params: None (Matern-5/2) or B x m x (3 + d - d_tau) host values
+    [s2_c, s2_x, beta, preference entries...] of the composite kernel."""
+    p = _host_f64(params)
+    _check(load().boute_gp_set_kernel(gp.handle, int(d_tau), _p(p, torch.float64, False)),
+           "boute_gp_set_kernel")
 
 
 def boute_gp_posterior(gp: Gp, Xc, N: int, mean, var, stream=None):
@@ -313,6 +339,19 @@ def boute_engine_stage_times(e: Engine) -> dict:
 
 def boute_engine_launches_per_step(e: Engine) -> int:
     return int(load().boute_engine_launches_per_step(e.handle))
+
+
+def boute_engine_set_kernel(e: Engine, d_tau: int = 0, params=None):
+    """As boute_gp_set_kernel, for the engine's steps."""
+    p = _host_f64(params)
+    _check(load().boute_engine_set_kernel(e.handle, int(d_tau), _p(p, torch.float64, False)),
+           "boute_engine_set_kernel")
+
+
+def boute_engine_set_outcome_transforms(e: Engine, codes=None):
+    """codes: None or m outcome-transform codes (BOUTE_TF_*)."""
+    _check(load().boute_engine_set_outcome_transforms(e.handle, _codes(codes)),
+           "boute_engine_set_outcome_transforms")
 
 
 def boute_engine_set_constraints(e: Engine, cons=None):

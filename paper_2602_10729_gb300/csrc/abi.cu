@@ -5,6 +5,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <new>
+#include <vector>
 
 #include "internal.h"
 
@@ -143,10 +144,26 @@ const char *boute_status_string(int s) {
 
 unsigned long long boute_launch_count(void) { return launch_count(); }
 
-int boute_standardize(const double *Y, int B, int n, int m, double *Ys, void *stream) {
-  if (!Y || !Ys || B < 1 || n < 1 || m < 1) return BOUTE_ERR_INVALID_ARG;
+// m per-objective transform codes (host, or null = identity) packed 3 bits
+// apiece; false for an unknown code
+static bool pack_codes(const int *codes, int m, int *packed) {
+  *packed = 0;
+  if (!codes) return true;
+  for (int t = 0; t < m; ++t) {
+    const int c = codes[t];
+    if (c < 0 || c > 7 || (c & 3) == 3) return false;
+    *packed |= c << (3 * t);
+  }
+  return true;
+}
+
+int boute_standardize(const double *Y, int B, int n, int m, const int *transforms, double *Ys,
+                      void *stream) {
+  int codes = 0;
+  if (!Y || !Ys || B < 1 || n < 1 || m < 1 || m > BOUTE_MAX_M || !pack_codes(transforms, m, &codes))
+    return BOUTE_ERR_INVALID_ARG;
   if (int r = device_ok()) return r;
-  return launch_standardize(Y, B, n, m, Ys, (cudaStream_t)stream);
+  return launch_standardize(Y, B, n, m, codes, Ys, (cudaStream_t)stream);
 }
 
 int boute_gp_create(int B, int n, int d, int m, boute_gp **out) {
@@ -202,8 +219,37 @@ void boute_gp_free(boute_gp *gp) {
   if (!gp) return;
   Gp &g = gp->g;
   cudaFree(g.Kh); cudaFree(g.Kl); cudaFree(g.Aws); cudaFree(g.Wws); cudaFree(g.bop); cudaFree(g.xt);
-  cudaFree(g.s2f); cudaFree(g.status);
+  cudaFree(g.s2f); cudaFree(g.status); cudaFree(g.kpar);
   delete gp;
+}
+
+int boute_gp_set_kernel(boute_gp *gp, int d_tau, const double *params) {
+  if (!gp) return BOUTE_ERR_INVALID_ARG;
+  Gp &g = gp->g;
+  if (!params) {
+    g.kern = 0;
+    return BOUTE_OK;
+  }
+  if (d_tau < 0 || d_tau > g.d) return BOUTE_ERR_INVALID_ARG;
+  const int BM = g.B * g.m, dc = g.d - d_tau, in = 3 + dc, out = 3 + g.d;
+  std::vector<double> h((size_t)BM * out, 0.0);
+  for (int bt = 0; bt < BM; ++bt) {
+    const double *p = params + (size_t)bt * in;
+    double *q = h.data() + (size_t)bt * out;
+    q[0] = p[0];
+    q[1] = p[1];
+    q[2] = p[2];
+    for (int k = 0; k < dc; ++k) q[3 + d_tau + k] = p[3 + k];
+  }
+  // no fit of this handle may be reading the parameters while they change
+  if (cudaDeviceSynchronize() != cudaSuccess) return last_launch_status();
+  if (!g.kpar && dalloc(&g.kpar, h.size()) != BOUTE_OK) return BOUTE_ERR_OOM;
+  if (cudaMemcpy(g.kpar, h.data(), h.size() * sizeof(double), cudaMemcpyHostToDevice) !=
+      cudaSuccess)
+    return last_launch_status();
+  g.kern = 1;
+  g.dtau = d_tau;
+  return BOUTE_OK;
 }
 
 int boute_gp_posterior(const boute_gp *gp, const float *Xc, long long N, float *mean, float *var,
@@ -412,8 +458,8 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
       cudaEventRecord(e->ev[stage], s);
   };
   auto front = [&](cudaStream_t fs) {
-    return launch_front_fused(Y, B, n, m, ref, e->Ys, e->mask, e->front, e->P, e->lower,
-                              e->upper, e->K, mc, fs);
+    return launch_front_fused(Y, B, n, m, e->gp->g.tcodes, ref, e->Ys, e->mask, e->front, e->P,
+                              e->lower, e->upper, e->K, mc, fs);
   };
   mark(ST_FIT);
   // waits on the host-input copies: an external-event node when captured
@@ -701,6 +747,33 @@ int boute_engine_stage_times(boute_engine *e, float *ms, int count) {
 
 int boute_engine_launches_per_step(const boute_engine *e) { return e ? e->launches : 0; }
 
+// the cached step graphs hold kernel arguments and kernel choices: drop them
+static void engine_drop_graphs(boute_engine *e) {
+  for (auto &g : e->graphs)
+    if (g.exec) {
+      cudaGraphExecDestroy(g.exec);
+      g.exec = nullptr;
+    }
+}
+
+int boute_engine_set_kernel(boute_engine *e, int d_tau, const double *params) {
+  if (!e) return BOUTE_ERR_INVALID_ARG;
+  const int r = boute_gp_set_kernel(e->gp, d_tau, params);
+  engine_drop_graphs(e);  // the step's kernel choices change
+  return r;
+}
+
+int boute_engine_set_outcome_transforms(boute_engine *e, const int *codes) {
+  int packed = 0;
+  if (!e || !pack_codes(codes, e->m, &packed)) return BOUTE_ERR_INVALID_ARG;
+  if (packed != e->gp->g.tcodes) {
+    if (cudaDeviceSynchronize() != cudaSuccess) return last_launch_status();
+    e->gp->g.tcodes = packed;
+    engine_drop_graphs(e);
+  }
+  return BOUTE_OK;
+}
+
 int boute_engine_set_constraints(boute_engine *e, const double *cons) {
   if (!e) return BOUTE_ERR_INVALID_ARG;
   const size_t count = (size_t)e->B * e->m;
@@ -714,11 +787,7 @@ int boute_engine_set_constraints(boute_engine *e, const double *cons) {
   const int on = cons != nullptr;
   if (on != e->has_cons) {  // the step's acquisition kernel changes: recapture
     e->has_cons = on;
-    for (auto &g : e->graphs)
-      if (g.exec) {
-        cudaGraphExecDestroy(g.exec);
-        g.exec = nullptr;
-      }
+    engine_drop_graphs(e);
   }
   return BOUTE_OK;
 }

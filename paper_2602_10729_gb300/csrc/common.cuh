@@ -35,6 +35,20 @@ struct PostPlan {
 
 inline __host__ __device__ int round_up(int x, int r) { return (x + r - 1) / r * r; }
 
+// Outcome transforms applied before Standardize (Sec. 5.2 S4): per objective
+// a 3-bit code, code & 3 = 0 identity, 1 log (latency), 2 logit (quality);
+// code & 4 negates (a maximised outcome becomes a minimised one). Several
+// objectives' codes are packed 3 bits apiece, objective t at bit 3t.
+inline __host__ __device__ int objective_code(int codes, int t) { return (codes >> (3 * t)) & 7; }
+#ifdef __CUDACC__
+__device__ __forceinline__ double outcome_transform(double y, int code) {
+  double v = y;
+  if ((code & 3) == 1) v = log(y);
+  else if ((code & 3) == 2) v = log(y / (1.0 - y));
+  return (code & 4) ? -v : v;
+}
+#endif
+
 // Floats of one training-point chunk of the posterior's side input: X/ls as
 // fp32 hi [DP][32] and lo [DP][32] (dimension-major, so pairs of training
 // points load as packed f32x2), alpha [32], then the objective's parameters

@@ -36,17 +36,19 @@ __device__ double block_sum(double v, double *red) {
 }
 
 // ---- Standardize (one block per (problem, objective)) --------------------
-__global__ void standardize_kernel(const double *Y, int n, int m, double *Ys) {
+// (codes: outcome transforms, objective_code)
+__global__ void standardize_kernel(const double *Y, int n, int m, int codes, double *Ys) {
   __shared__ double red[32];
   const int b = blockIdx.x / m, t = blockIdx.x % m;
+  const int code = objective_code(codes, t);
   const double *y = Y + (size_t)b * n * m + t;
   double *ys = Ys + (size_t)b * n * m + t;
   double s = 0.0;
-  for (int i = threadIdx.x; i < n; i += blockDim.x) s += y[(size_t)i * m];
+  for (int i = threadIdx.x; i < n; i += blockDim.x) s += outcome_transform(y[(size_t)i * m], code);
   const double mean = block_sum(s, red) / n;
   double ss = 0.0;
   for (int i = threadIdx.x; i < n; i += blockDim.x) {
-    double z = y[(size_t)i * m] - mean;
+    double z = outcome_transform(y[(size_t)i * m], code) - mean;
     ss += z * z;
   }
   ss = block_sum(ss, red);
@@ -54,7 +56,8 @@ __global__ void standardize_kernel(const double *Y, int n, int m, double *Ys) {
   if (!(sd >= 1e-8)) sd = 1.0;
   const double isd = 1.0 / sd;  // one division; fp64 divides are slow on this part
   __syncthreads();  // every thread has read its inputs before (aliased) outputs land
-  for (int i = threadIdx.x; i < n; i += blockDim.x) ys[(size_t)i * m] = (y[(size_t)i * m] - mean) * isd;
+  for (int i = threadIdx.x; i < n; i += blockDim.x)
+    ys[(size_t)i * m] = (outcome_transform(y[(size_t)i * m], code) - mean) * isd;
 }
 
 // ---- fit set-up, one launch: K = s2 M52(X, X) + noise I and the side input --
@@ -68,13 +71,22 @@ __global__ void standardize_kernel(const double *Y, int n, int m, double *Ys) {
 // hi/lo pairs (dimension-major per 32-point chunk), and in every chunk the
 // objective's 1/l (hi, lo) and outputscale. Block 0 of the first problem
 // clears the fit status.
+// Composite kernel (kp != null: [s2_c, s2_x, beta, s_0 .. s_{d-1}] of this
+// problem-objective, s_k = 0 for the routing features [0, dtau)), Sec. 5.2
+// "Additive kernels" and S5 as Sec. 6 assembles them:
+//   k = s2 k52(r_t) + s2_c w_i w_j k32(r_c) + s2_x k52(r_t) k32(r_c),
+// r_t over the routing features, r_c over the deployment features,
+// w = exp(beta sum_k s_k x_k). Its side input holds, in place of the
+// coordinates' lo parts, the training points' weights w_j and beta s_k, and
+// s2_c, s2_x, dtau after the outputscale.
 constexpr int kSetupThreads = 128;
 __host__ __device__ inline int kmat_units(int n) {
   const int tn = (n + 15) / 16;
   return tn * (tn + 1);  // tiles on or below the diagonal, two halves each
 }
 __device__ void kmat_tile(const double *X, int n, int d, int b, const double *l, double s2,
-                          double noise, int unit, float *Kh, float *Kl, double *il) {
+                          double noise, int unit, float *Kh, float *Kl, double *il,
+                          const double *kp, int dtau) {
   for (int t = threadIdx.x; t < d; t += blockDim.x) il[t] = 1.0 / l[t];
   __syncthreads();
   const int tile = unit >> 1, half = unit & 1;
@@ -85,13 +97,30 @@ __device__ void kmat_tile(const double *X, int n, int d, int b, const double *l,
   const int i = ti * 16 + threadIdx.x / 8, j = tj * 16 + half * 8 + threadIdx.x % 8;
   if (i >= n || j >= n) return;
   const double *xi = X + ((size_t)b * n + i) * d, *xj = X + ((size_t)b * n + j) * d;
-  double r2 = 0.0;
-  for (int t = 0; t < d; ++t) {
+  double r2 = 0.0, r2c = 0.0;
+  const int dt = kp ? dtau : d;
+  for (int t = 0; t < dt; ++t) {
     const double z = (xi[t] - xj[t]) * il[t];
     r2 = fma(z, z, r2);
   }
+  for (int t = dt; t < d; ++t) {
+    const double z = (xi[t] - xj[t]) * il[t];
+    r2c = fma(z, z, r2c);
+  }
   const double r = sqrt(r2), sr = sqrt(5.0) * r;
-  double k = s2 * (1.0 + sr + 5.0 * r2 / 3.0) * exp(-sr);
+  double k;
+  if (!kp) {
+    k = s2 * (1.0 + sr + 5.0 * r2 / 3.0) * exp(-sr);
+  } else {
+    const double k52 = (1.0 + sr + 5.0 * r2 / 3.0) * exp(-sr);
+    const double sc = sqrt(3.0) * sqrt(r2c), k32 = (1.0 + sc) * exp(-sc);
+    double ei = 0.0, ej = 0.0;
+    for (int t = dtau; t < d; ++t) {
+      ei = fma(kp[3 + t], xi[t], ei);
+      ej = fma(kp[3 + t], xj[t], ej);
+    }
+    k = s2 * k52 + kp[0] * exp(kp[2] * (ei + ej)) * k32 + kp[1] * k52 * k32;
+  }
   if (i == j) k += noise;
   const float kh = (float)k, kl = (float)(k - (double)kh);
   Kh[(size_t)i * n + j] = kh;
@@ -103,7 +132,8 @@ __device__ void kmat_tile(const double *X, int n, int d, int b, const double *l,
 }
 
 __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad,
-                          const double *l, double s2, float *x, int blk, int nblk) {
+                          const double *l, double s2, float *x, int blk, int nblk,
+                          const double *kp, int dtau) {
   const int cf = xt_chunk_floats(DP);
   const int total = npad * DP;
   for (int e = blk * blockDim.x + threadIdx.x; e < total; e += nblk * blockDim.x) {
@@ -113,7 +143,22 @@ __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad
     const int c = j / BOUTE_KCHUNK, jj = j % BOUTE_KCHUNK;
     float *q = x + (size_t)c * cf;  // dimension-major: [DP][32] hi, [DP][32] lo
     q[t * BOUTE_KCHUNK + jj] = hi;
-    q[BOUTE_KCHUNK * DP + t * BOUTE_KCHUNK + jj] = lo;
+    if (!kp) q[BOUTE_KCHUNK * DP + t * BOUTE_KCHUNK + jj] = lo;
+  }
+  if (kp) {  // composite kernel: w_j (row 0 of the lo block), beta s_k (row 1)
+    for (int e = blk * blockDim.x + threadIdx.x; e < npad; e += nblk * blockDim.x) {
+      double ej = 0.0;
+      if (e < n)
+        for (int t = dtau; t < d; ++t) ej = fma(kp[3 + t], X[((size_t)b * n + e) * d + t], ej);
+      x[(size_t)(e / BOUTE_KCHUNK) * cf + BOUTE_KCHUNK * DP + e % BOUTE_KCHUNK] =
+          e < n ? (float)exp(kp[2] * ej) : 0.f;
+    }
+    for (int e = blk * blockDim.x + threadIdx.x; e < (npad / BOUTE_KCHUNK) * DP;
+         e += nblk * blockDim.x) {
+      const int c = e / DP, k = e % DP;
+      x[(size_t)c * cf + BOUTE_KCHUNK * DP + BOUTE_KCHUNK + k] =
+          (k >= dtau && k < d) ? (float)(kp[2] * kp[3 + k]) : 0.f;
+    }
   }
   const int po = xt_param_offset(DP), nch = npad / BOUTE_KCHUNK;
   for (int e = blk * blockDim.x + threadIdx.x; e < nch * (2 * DP + 4); e += nblk * blockDim.x) {
@@ -127,6 +172,9 @@ __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad
         v = (float)(iv - (double)(float)iv);
       }
     } else if (k == 2 * DP) v = (float)s2;
+    else if (kp && k == 2 * DP + 1) v = (float)kp[0];
+    else if (kp && k == 2 * DP + 2) v = (float)kp[1];
+    else if (kp && k == 2 * DP + 3) v = (float)dtau;
     x[(size_t)c * cf + po + k] = v;
   }
 }
@@ -134,19 +182,22 @@ __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad
 __global__ void __launch_bounds__(kSetupThreads) fit_setup_kernel(
     const double *X, int n, int d, int m, int DP, int npad, const double *ls, const double *s2,
     const double *noise, float *Kh_all, float *Kl_all, float *xt, float *s2f, int nkt, int nprep,
-    int early_trigger, int *status) {
+    int early_trigger, int *status, const double *kpar, int dtau) {
   __shared__ double il[BOUTE_MAX_D];
   const int bt = blockIdx.y, b = bt / m;
   if (early_trigger) pdl_trigger();  // the whole grid is resident: the fit may launch now
   const double *l = ls + (size_t)bt * d;
+  const double *kp = kpar ? kpar + (size_t)bt * (3 + d) : nullptr;
   if (blockIdx.x == 0 && bt == 0 && threadIdx.x == 0) *status = BOUTE_OK;
   if ((int)blockIdx.x < nkt) {
     kmat_tile(X, n, d, b, l, s2[bt], noise[bt], blockIdx.x, Kh_all + (size_t)bt * n * n,
-              Kl_all + (size_t)bt * n * n, il);
+              Kl_all + (size_t)bt * n * n, il, kp, dtau);
   } else {
     float *x = xt + (size_t)bt * (npad / BOUTE_KCHUNK) * xt_chunk_floats(DP);
-    prep_part(X, n, d, b, DP, npad, l, s2[bt], x, blockIdx.x - nkt, nprep);
-    if (blockIdx.x == nkt && threadIdx.x == 0) s2f[bt] = (float)s2[bt];
+    prep_part(X, n, d, b, DP, npad, l, s2[bt], x, blockIdx.x - nkt, nprep, kp, dtau);
+    // the prior variance's constant part (composite: s2 + s2_x; the
+    // posterior adds s2_c w(x)^2)
+    if (blockIdx.x == nkt && threadIdx.x == 0) s2f[bt] = (float)(s2[bt] + (kp ? kp[1] : 0.0));
   }
 }
 
@@ -203,9 +254,9 @@ constexpr int fit_threads() { return SMEM ? 384 : 256; }
 
 template <bool SMEM>
 __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
-    const float *Kh_all, const float *Kl_all, const double *Ys, int standardize, int n, int m,
-    float *Aws, float *Wws, float *xt, int DP, int npad, PostPlan plan, float *bop, int kl_smem,
-    int early_trigger, int *status) {
+    const float *Kh_all, const float *Kl_all, const double *Ys, int standardize, int tcodes,
+    int n, int m, float *Aws, float *Wws, float *xt, int DP, int npad, PostPlan plan, float *bop,
+    int kl_smem, int early_trigger, int *status) {
   extern __shared__ __align__(16) float sm[];
   __shared__ int bad;
   __shared__ uint64_t lbar, lbar_lo;  // K hi; K lo (needed only by the residual)
@@ -224,16 +275,18 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
         *rv = vec + 5 * NP;
   const double *y = Ys + (size_t)b * n * m + t;
   if (early_trigger) pdl_trigger();  // every block is resident: the posterior may launch
-  // standardize != 0: Ys holds raw outcomes; this column is standardised here
-  // (zero mean, unit sample standard deviation, as standardize_kernel does)
+  // standardize != 0: Ys holds raw outcomes; this column is transformed
+  // (tcodes) and standardised here (zero mean, unit sample standard deviation,
+  // as standardize_kernel does)
+  const int tcode = standardize ? objective_code(tcodes, t) : 0;
   if (standardize) {  // warp 0 alone: few fp64 instructions
     if (warp == 0) {
       double sum = 0.0;
-      for (int i = lane; i < n; i += 32) sum += y[(size_t)i * m];
+      for (int i = lane; i < n; i += 32) sum += outcome_transform(y[(size_t)i * m], tcode);
       const double mean = warp_sum(sum) / n;
       double ss = 0.0;
       for (int i = lane; i < n; i += 32) {
-        const double z = y[(size_t)i * m] - mean;
+        const double z = outcome_transform(y[(size_t)i * m], tcode) - mean;
         ss += z * z;
       }
       ss = warp_sum(ss);
@@ -313,7 +366,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     __syncthreads();
   }
   for (int i = tid; i < NP; i += nthr) {  // standardised y as an fp32 pair
-    const double ys = i < n ? (y[(size_t)i * m] - mu_y) * isd_y : 0.0;
+    const double ys = i < n ? (outcome_transform(y[(size_t)i * m], tcode) - mu_y) * isd_y : 0.0;
     yv[i] = (float)ys;
     ylo[i] = (float)(ys - (double)yv[i]);
     dg[i] = A[(size_t)i * ld + i];
@@ -679,8 +732,9 @@ __global__ void pack_kernel(const float *Wws, PostPlan plan, float *bop, const i
 
 }  // namespace
 
-int launch_standardize(const double *Y, int B, int n, int m, double *Ys, cudaStream_t s) {
-  standardize_kernel<<<B * m, 256, 0, s>>>(Y, n, m, Ys);
+int launch_standardize(const double *Y, int B, int n, int m, int codes, double *Ys,
+                       cudaStream_t s) {
+  standardize_kernel<<<B * m, 256, 0, s>>>(Y, n, m, codes, Ys);
   count_launch();
   return last_launch_status();
 }
@@ -715,7 +769,8 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
   const int fit_early = 2 * BM <= sms ? 1 : 0;
   fit_setup_kernel<<<dim3(nkt + nprep, BM), kSetupThreads, 0, s>>>(X, n, d, m, gp->DP, npad, ls, s2, noise,
                                                          gp->Kh, gp->Kl, gp->xt, gp->s2f, nkt,
-                                                         nprep, setup_early, gp->status);
+                                                         nprep, setup_early, gp->status,
+                                                         gp->kern ? gp->kpar : nullptr, gp->dtau);
   if (setup_done && cudaEventRecord(setup_done, s) != cudaSuccess) return last_launch_status();
   if (fit_uses_smem(npad)) {
     const size_t smem = fit_smem_bytes(npad, n);
@@ -723,13 +778,13 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
     cudaFuncSetAttribute(fit32_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);
     launch_pdl(fit32_kernel<true>, dim3(BM), dim3(fit_threads<true>()), smem, s, gp->Kh, gp->Kl,
-               Ys, standardize, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop,
-               fit_kl_in_smem(n) ? 1 : 0, fit_early, gp->status);
+               Ys, standardize, gp->tcodes, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad,
+               gp->plan, gp->bop, fit_kl_in_smem(n) ? 1 : 0, fit_early, gp->status);
     count_launch(2);
   } else {
     launch_pdl(fit32_kernel<false>, dim3(BM), dim3(fit_threads<false>()),
-               6 * npad * sizeof(float), s, gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws,
-               gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop, 0, 0, gp->status);
+               6 * npad * sizeof(float), s, gp->Kh, gp->Kl, Ys, standardize, gp->tcodes, n, m,
+               gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop, 0, 0, gp->status);
     const long long tot = (long long)gp->plan.ncols * npad;
     pack_kernel<<<dim3((unsigned)std::min<long long>((tot + 255) / 256, 4096), BM), 256, 0, s>>>(
         gp->Wws, gp->plan, gp->bop, gp->status);

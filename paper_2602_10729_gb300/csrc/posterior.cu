@@ -73,11 +73,14 @@ struct PostArgs {
   int tiles_per_problem, tiles_total;
   int sa, sb, sx;              // depths of the A, B and side-input rings
   uint32_t b_bytes, x_bytes;   // one B stage, one side-input entry
+  int kern;                    // 1: the composite kernel (prior variance per candidate)
   PostPlan plan;
 };
 
 constexpr float kSqrt5 = 2.2360679774997896964f;
 constexpr float kSqrt5Log2e = 3.2259641822295610f;  // sqrt(5) / ln(2)
+constexpr float kSqrt3 = 1.7320508075688772f;
+constexpr float kSqrt3Log2e = 2.4988211106473432f;  // sqrt(3) / ln(2)
 
 // Single hardware instructions (relative error about 2^-22), no range fix-ups:
 // arguments here are finite and non-negative (sqrt) or non-positive (ex2).
@@ -132,18 +135,59 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// The composite kernel's per-candidate inputs (Sec. 5.2 "Additive kernels"
+// and S5, as Sec. 6 assembles them): the routing features are dimensions
+// [0, dtau), the candidate's preference weight w* = exp(beta <s, c*>), the
+// outputscales of the weighted deployment term and of the interaction term.
+struct CompIn {
+  int dtau;
+  float ws, s2c, s2x;
+};
+
+// The side input's composite-kernel entries within a chunk (the block after
+// the scaled coordinates): row 0 the chunk's training-point preference weights
+// w_j, row 1 beta * s_k per dimension (zero for routing features); the
+// parameter block holds s2_c, s2_x and dtau after the outputscale.
+__device__ __forceinline__ const float *chunk_weights(const float *chunk, int DP) {
+  return chunk + BOUTE_KCHUNK * DP;
+}
+__device__ __forceinline__ const float *chunk_pref(const float *chunk, int DP) {
+  return chunk + BOUTE_KCHUNK * DP + BOUTE_KCHUNK;
+}
+__device__ __forceinline__ CompIn chunk_comp(const float *chunk, int DP) {
+  const float *pb = chunk + xt_param_offset(DP) + 2 * DP;
+  return CompIn{(int)pb[3], 0.f, pb[1], pb[2]};
+}
+
+// A candidate's preference weight from its raw coordinates.
+template <int DP>
+__device__ __forceinline__ float cand_weight(const float (&xr)[DP], const float *bp) {
+  float e = 0.f;
+#pragma unroll
+  for (int k = 0; k < DP; ++k) e = fmaf(bp[k], xr[k], e);
+  return expf(e);
+}
+
 // The K* values of one builder thread's COLS columns of a 32-point chunk:
 // squared scaled distances in packed pairs (candidate x*_k / l_k as a
 // duplicated pair, minus the chunk's training coordinates x_k / l_k), then
 // k = s2 (1 + sqrt5 r + 5/3 r^2) exp(-sqrt5 r) with exp(-x) = 2^(-x log2 e).
+// KERN = 1, the composite kernel: the distances over the routing features
+// (r_t) and the deployment features (r_c) are accumulated apart, and
+//   k = k52(r_t) (s2 + s2_x k32(r_c)) + s2_c w_j w* k32(r_c),
+//   k52(r) = (1 + sqrt5 r + 5/3 r^2) e^(-sqrt5 r), k32(r) = (1 + sqrt3 r) e^(-sqrt3 r).
 // Both the fused builders and the stand-alone K* kernel use this, so their
 // values are identical.
-template <int DP, int COLS>
+template <int DP, int COLS, int KERN = 0>
 __device__ __forceinline__ void kstar_cols(const unsigned long long (&xs2)[DP], const float *xth,
-                                           int g, float s2, float (&kv)[COLS]) {
-  unsigned long long acc2[COLS / 2];
+                                           int g, float s2, float (&kv)[COLS],
+                                           const CompIn &ci = CompIn{}) {
+  unsigned long long acc2[COLS / 2], accc[COLS / 2];
 #pragma unroll
-  for (int e = 0; e < COLS / 2; ++e) acc2[e] = 0ull;
+  for (int e = 0; e < COLS / 2; ++e) {
+    acc2[e] = 0ull;
+    accc[e] = 0ull;
+  }
 #pragma unroll
   for (int k = 0; k < DP; ++k) {
     // 16-byte loads: two training points' coordinate pairs each
@@ -155,11 +199,38 @@ __device__ __forceinline__ void kstar_cols(const unsigned long long (&xs2)[DP], 
       h2[2 * e] = v.x;
       h2[2 * e + 1] = v.y;
     }
+    if (KERN == 1 && k >= ci.dtau) {  // a deployment feature (uniform branch)
+#pragma unroll
+      for (int e = 0; e < COLS / 2; ++e) {
+        const unsigned long long df = f2_sub(xs2[k], h2[e]);
+        accc[e] = f2_fma(df, df, accc[e]);
+      }
+    } else {
+#pragma unroll
+      for (int e = 0; e < COLS / 2; ++e) {
+        const unsigned long long df = f2_sub(xs2[k], h2[e]);
+        acc2[e] = f2_fma(df, df, acc2[e]);
+      }
+    }
+  }
+  if (KERN == 1) {
+    const float *wj = chunk_weights(xth, DP) + COLS * g;
 #pragma unroll
     for (int e = 0; e < COLS / 2; ++e) {
-      const unsigned long long df = f2_sub(xs2[k], h2[e]);
-      acc2[e] = f2_fma(df, df, acc2[e]);
+      float r2[2], c2[2];
+      f2_split(acc2[e], r2[0], r2[1]);
+      f2_split(accc[e], c2[0], c2[1]);
+#pragma unroll
+      for (int z = 0; z < 2; ++z) {
+        const float rr = sqrt_approx(r2[z]);
+        const float k52 =
+            fmaf(kFiveThirds, r2[z], fmaf(kSqrt5, rr, 1.0f)) * ex2_approx(-kSqrt5Log2e * rr);
+        const float rc = sqrt_approx(c2[z]);
+        const float k32 = fmaf(kSqrt3, rc, 1.0f) * ex2_approx(-kSqrt3Log2e * rc);
+        kv[2 * e + z] = fmaf(k52, fmaf(ci.s2x, k32, s2), ci.s2c * (wj[2 * e + z] * ci.ws) * k32);
+      }
     }
+    return;
   }
 #pragma unroll
   for (int e = 0; e < COLS / 2; ++e) {
@@ -217,8 +288,9 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity,
 }
 
 // PRE: the K* values come precomputed (kstar_kernel) instead of being built
-// here; everything else is the same.
-template <int DP, bool PRE>
+// here; everything else is the same. KERN: the kernel the builders evaluate
+// (0 Matern-5/2, 1 composite; only when !PRE).
+template <int DP, bool PRE, int KERN = 0>
 __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
     posterior_kernel(const __grid_constant__ PostArgs a) {
   constexpr int kBldWarps = Layout<DP>::kBld;
@@ -437,7 +509,16 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
         }
         if (*abort) break;
         if (row < a.N) {
-          const float vv = a.s2f[b * m + t] - ss;
+          float prior = a.s2f[b * m + t];
+          if (a.kern) {  // composite kernel: k(x, x) = s2 + s2_x + s2_c w(x)^2
+            const float *c0 = a.xt + (size_t)(b * m + t) * pl.nchunk * cf;
+            const float *bp = chunk_pref(c0, DP), *xrow = a.Xc + ((size_t)b * a.N + row) * d;
+            float e = 0.f;
+            for (int k = 0; k < d; ++k) e = fmaf(bp[k], xrow[k], e);
+            const float w = expf(e);
+            prior = fmaf(chunk_comp(c0, DP).s2c * w, w, prior);
+          }
+          const float vv = prior - ss;
           a.var[((size_t)b * m + t) * a.N + row] = vv > 0.f ? vv : 0.f;
         }
       }
@@ -462,6 +543,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       {
         unsigned long long xs2[DP];
         float s2 = 0.f;
+        CompIn ci{};
         float mu = 0.f, comp = 0.f;
         for (int p = 0; p < pl.npass && !*abort; ++p) {
           const bool last_pass = p == pl.npass - 1;
@@ -479,6 +561,10 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
               const float *il = xth + xt_param_offset(DP);
               scaled_candidate<DP>(xr, il, xs2);
               s2 = il[2 * DP];
+              if (KERN == 1) {
+                ci = chunk_comp(xth, DP);
+                ci.ws = cand_weight<DP>(xr, chunk_pref(xth, DP));
+              }
             }
             float kv[COLS];
             if (PRE) {  // this thread's COLS values of chunk c, from the stage's image
@@ -491,7 +577,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
                 kv[4 * e + 3] = v.w;
               }
             } else {
-              kstar_cols<DP, COLS>(xs2, xth, g, s2, kv);
+              kstar_cols<DP, COLS, KERN>(xs2, xth, g, s2, kv, ci);
             }
             const bool full_chunk = (c + 1) * BOUTE_KCHUNK <= n;
             const int jbase = c * BOUTE_KCHUNK + COLS * g;
@@ -578,6 +664,7 @@ int launch_dp(const Gp *gp, const float *Xc, const float *kst, long long N, floa
   a.d = gp->d;
   a.n = gp->n;
   a.plan = gp->plan;
+  a.kern = gp->kern;
   a.tiles_per_problem = (int)((N + BOUTE_TILE_M - 1) / BOUTE_TILE_M);
   a.tiles_total = a.tiles_per_problem * gp->B;
   const int ncolmax = gp->plan.ncol[0];
@@ -605,6 +692,7 @@ int launch_dp(const Gp *gp, const float *Xc, const float *kst, long long N, floa
     launch_pdl(kern, dim3(grid), dim3(Layout<DP>::kThreads), smem, s, a);
   };
   if (kst) go(posterior_kernel<DP, true>);
+  else if (gp->kern) go(posterior_kernel<DP, false, 1>);
   else go(posterior_kernel<DP, false>);
   count_launch();
   return last_launch_status();
@@ -619,7 +707,7 @@ int launch_dp(const Gp *gp, const float *Xc, const float *kst, long long N, floa
 // core reads an fp32 operand truncated to tf32, so the full value serves as
 // the hi part. The training points' side input is staged in shared memory.
 // It needs the set-up's side input (not the fit's results) and the candidates.
-template <int DP>
+template <int DP, int KERN>
 __global__ void __launch_bounds__(Layout<DP>::kBld * 32) kstar_kernel(
     const float *Xc, const float *xt, long long N, int d, int m, int n, int tiles_per_problem,
     int nchunk, float *kst) {
@@ -641,9 +729,14 @@ __global__ void __launch_bounds__(Layout<DP>::kBld * 32) kstar_kernel(
   unsigned long long xs2[DP];
   scaled_candidate<DP>(xr, il, xs2);
   const float s2 = il[2 * DP];
+  CompIn ci{};
+  if (KERN == 1) {
+    ci = chunk_comp(xs, DP);
+    ci.ws = cand_weight<DP>(xr, chunk_pref(xs, DP));
+  }
   for (int c = 0; c < nchunk; ++c) {
     float kv[COLS];
-    kstar_cols<DP, COLS>(xs2, xs + (size_t)c * cf, g, s2, kv);
+    kstar_cols<DP, COLS, KERN>(xs2, xs + (size_t)c * cf, g, s2, kv, ci);
     const int jbase = c * BOUTE_KCHUNK + COLS * g;
 #pragma unroll
     for (int kk = 0; kk < COLS; ++kk) kv[kk] = (jbase + kk < n) ? kv[kk] : 0.f;
@@ -660,13 +753,17 @@ int launch_kstar_dp(const Gp *gp, const float *Xc, long long N, float *kst, cuda
   const int tpp = (int)((N + BOUTE_TILE_M - 1) / BOUTE_TILE_M);
   const int units = tpp * gp->B * gp->m;
   const size_t smem = (size_t)gp->plan.nchunk * xt_chunk_floats(DP) * sizeof(float);
-  prefer_shared(kstar_kernel<DP>);
-  if (smem > 48 * 1024 &&
-      cudaFuncSetAttribute(kstar_kernel<DP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)smem) != cudaSuccess)
-    return last_launch_status();
-  kstar_kernel<DP><<<units, Layout<DP>::kBld * 32, smem, s>>>(Xc, gp->xt, N, gp->d, gp->m,
-                                                             gp->n, tpp, gp->plan.nchunk, kst);
+  auto go = [&](auto kern) {
+    prefer_shared(kern);
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+            cudaSuccess)
+      return last_launch_status();
+    kern<<<units, Layout<DP>::kBld * 32, smem, s>>>(Xc, gp->xt, N, gp->d, gp->m, gp->n, tpp,
+                                                    gp->plan.nchunk, kst);
+    return (int)BOUTE_OK;
+  };
+  if (int r = gp->kern ? go(kstar_kernel<DP, 1>) : go(kstar_kernel<DP, 0>)) return r;
   count_launch();
   return last_launch_status();
 }

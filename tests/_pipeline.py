@@ -127,6 +127,13 @@ class HostProblem:
     ref: np.ndarray  # B x m
     Xc: np.ndarray  # B x N x d float32
     eps: np.ndarray | None  # B x N x m x S float32
+    d_tau: int = 0  # composite kernel: routing features [0, d_tau), kc below
+    kc: np.ndarray | None = None  # B x m x (3 + d - d_tau) composite-kernel parameters
+    transforms: tuple = ()  # outcome-transform codes per objective
+
+    def kernel(self, b: int):
+        """The oracle's kernel argument for problem b."""
+        return None if self.kc is None else (self.d_tau, self.kc[b])
 
 
 def host_problem(w: wl.Workload, N: int | None = None, threads: int = 8) -> HostProblem:
@@ -141,12 +148,16 @@ def host_problem(w: wl.Workload, N: int | None = None, threads: int = 8) -> Host
     if w.mode == "mc":
         eps = np.stack([wl.base_normals(w, b, 0, N, threads) for b in range(w.B)])
     ref = np.tile(wl.ref_point(w), (w.B, 1))
+    kc = None
+    if w.d_tau:
+        kc = np.stack([wl.kernel_params(w, b)[1] for b in range(w.B)])
     return HostProblem(w, np.stack(Xs), np.stack(Ys), np.stack(L), np.stack(S2), np.stack(NZ),
-                       ref, Xc, eps)
+                       ref, Xc, eps, w.d_tau, kc, tuple(w.transforms))
 
 
 def oracle_fit(hp: HostProblem, b: int) -> opl.FittedProblem:
-    return opl.fit_problem(hp.X[b], hp.Y[b], hp.ls[b], hp.s2[b], hp.noise[b], hp.ref[b])
+    return opl.fit_problem(hp.X[b], hp.Y[b], hp.ls[b], hp.s2[b], hp.noise[b], hp.ref[b],
+                           kernel=hp.kernel(b), transforms=hp.transforms or None)
 
 
 # ---- GPU: one ABI call at a time ------------------------------------------------
@@ -169,8 +180,10 @@ def gpu_pipeline(hp: HostProblem, N: int | None = None, mean_var_in=None, cons=N
                        t(hp.noise, torch.float64), t(hp.ref, torch.float64))
     Xc = t(hp.Xc[:, :N], torch.float32)
     Ys = torch.empty_like(Y)
-    bt.boute_standardize(Y, Ys)
+    bt.boute_standardize(Y, Ys, transforms=hp.transforms or None)
     gp = bt.boute_gp_create(B, n, d, m)
+    if hp.kc is not None:
+        bt.boute_gp_set_kernel(gp, hp.d_tau, hp.kc)
     bt.boute_gp_fit(gp, X, Ys, ls, s2, nz)
     st = bt.boute_gp_status(gp)
     mask = torch.empty((B, n), dtype=torch.uint8, device=dev)
