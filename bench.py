@@ -64,8 +64,9 @@ def host_inputs(w: wl.Workload, threads: int = 16):
     eps = (np.stack([wl.base_normals(w, b, 0, w.N, threads) for b in range(w.B)])
            if w.mode == "mc" else None)
     ref = np.tile(wl.ref_point(w), (w.B, 1))
+    kc = np.stack([wl.kernel_params(w, b)[1] for b in range(w.B)]) if w.d_tau else None
     return dict(X=np.stack(X), Y=np.stack(Y), ls=np.stack(L), s2=np.stack(S2),
-                noise=np.stack(NZ), ref=ref, Xc=Xc, eps=eps)
+                noise=np.stack(NZ), ref=ref, Xc=Xc, eps=eps, kc=kc)
 
 
 # ---------------------------------------------------------------- clocks
@@ -176,9 +177,11 @@ def oracle_rate(w: wl.Workload, inp, budget_s: float, threads: int = 0, cons=Non
     import oracle
     from oracle import pipeline as opl
     threads = threads or oracle.default_threads()
+    kern = None if inp["kc"] is None else (w.d_tau, inp["kc"][0])
+    tfs = list(w.transforms) or None
     t0 = time.perf_counter()
     fp = opl.fit_problem(inp["X"][0], inp["Y"][0], inp["ls"][0], inp["s2"][0], inp["noise"][0],
-                         inp["ref"][0])
+                         inp["ref"][0], kernel=kern, transforms=tfs)
     fit_s = time.perf_counter() - t0
     n_try = min(w.N, 2048)
     t0 = time.perf_counter()
@@ -188,7 +191,7 @@ def oracle_rate(w: wl.Workload, inp, budget_s: float, threads: int = 0, cons=Non
     sample = int(max(n_try, min(w.N, (budget_s - fit_s) / max(per, 1e-9))))
     t0 = time.perf_counter()
     fp = opl.fit_problem(inp["X"][0], inp["Y"][0], inp["ls"][0], inp["s2"][0], inp["noise"][0],
-                         inp["ref"][0])
+                         inp["ref"][0], kernel=kern, transforms=tfs)
     opl.score(fp, inp["Xc"][0, :sample], w.mode, min(w.k, sample),
               None if inp["eps"] is None else inp["eps"][0, :sample], threads, cons=cons)
     dt = time.perf_counter() - t0
@@ -271,6 +274,9 @@ def main():
     e = bt.Engine(w.B, w.n, w.d, w.m, w.N, mode, w.S, w.k)
     if args.cons is not None:
         bt.boute_engine_set_constraints(e, torch.tensor([args.cons] * w.B, dtype=f64))
+    if w.d_tau:  # composite-kernel variant: the paper's kernel and outcome transforms
+        bt.boute_engine_set_kernel(e, w.d_tau, inp["kc"])
+        bt.boute_engine_set_outcome_transforms(e, list(w.transforms))
     idx = torch.empty((w.B, w.k), dtype=torch.int64, device=dev)
     val = torch.empty((w.B, w.k), dtype=f32, device=dev)
     args_dev = (dX, dY, dls, ds2, dnz, dref, dXc, deps, idx, val)
@@ -378,6 +384,7 @@ def main():
             "config": {"workload": w.name, "B": w.B, "n": w.n, "d": w.d, "m": w.m, "N": w.N,
                        "acquisition": w.mode, "S": w.S, "k": w.k,
                        "l2": "flushed between steps (512 MB write)", "parallelism": "replicas",
+                       "kernel": "composite" if w.d_tau else "matern52",
                        **({"constraints": args.constraints} if args.cons else {})},
             "roofline": roof,
             "cpu_baseline": cpu,
