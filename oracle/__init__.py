@@ -13,6 +13,7 @@ independent pin: none.
 from __future__ import annotations
 
 import ctypes
+import math
 import os
 import subprocess
 
@@ -67,6 +68,11 @@ def lib():
                                         ctypes.c_int, _dp, _dp, _dp, _fp, ctypes.c_longlong, _dp,
                                         _dp, ctypes.c_int]
         L.bo_gp_posterior_k.restype = None
+        L.bo_gp_mll.argtypes = [_dp, _dp, ctypes.c_int, ctypes.c_int, _dp, ctypes.c_double,
+                                ctypes.c_double, _dp]
+        L.bo_gp_mll.restype = ctypes.c_double
+        L.bo_gp_learn.argtypes = [_dp, _dp, ctypes.c_int, ctypes.c_int, _dp, ctypes.c_int,
+                                  ctypes.c_int, ctypes.c_double, _dp, _dp, _dp]
         L.bo_pareto_front.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp, _bp, _ip]
         L.bo_hv.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp, _dp]
         L.bo_hv.restype = ctypes.c_double
@@ -208,6 +214,43 @@ def gp_posterior(X, ls, s2, L, alpha, Xc, threads: int = 0, kernel=None):
         lib().bo_gp_posterior_k(pX, n, d, pl, float(s2), dtau, pk, pL, pa, pc, N,
                                 mean.ctypes.data_as(_dp), var.ctypes.data_as(_dp), threads)
     return mean, var
+
+
+def gp_mll(X, y, ls, s2, noise, grad: bool = False):
+    """Log marginal likelihood of the Matern-5/2 GP (and its gradient with
+    respect to (log l, log s2, log noise) when grad)."""
+    X, pX = _d(X)
+    y, py = _d(y)
+    ls, pl = _d(ls)
+    n, d = X.shape
+    g = np.empty(d + 2) if grad else None
+    v = lib().bo_gp_mll(pX, py, n, d, pl, float(s2), float(noise),
+                        None if g is None else g.ctypes.data_as(_dp))
+    return (v, g) if grad else v
+
+
+#: bounds of the learned log-parameters (log l, log s2, log noise)
+LOG_LS_BOUNDS = (math.log(1e-3), math.log(1e3))
+LOG_S2_BOUNDS = (math.log(1e-3), math.log(1e3))
+LOG_NOISE_BOUNDS = (math.log(1e-4), math.log(10.0))
+
+
+def gp_learn(X, y, theta0, iters: int, lr: float, grad: bool = False):
+    """Adam ascent on the log marginal likelihood from R starting points
+    theta0 (R x (d + 2) log-parameters). Returns (theta, mll[, grad])."""
+    X, pX = _d(X)
+    y, py = _d(y)
+    th0, pt = _d(np.atleast_2d(theta0))
+    n, d = X.shape
+    R = th0.shape[0]
+    theta = np.empty_like(th0)
+    mll = np.empty(R)
+    g = np.empty_like(th0) if grad else None
+    rc = lib().bo_gp_learn(pX, py, n, d, pt, R, int(iters), float(lr), theta.ctypes.data_as(_dp),
+                           mll.ctypes.data_as(_dp), None if g is None else g.ctypes.data_as(_dp))
+    if rc:
+        raise ValueError(rc)
+    return (theta, mll, g) if grad else (theta, mll)
 
 
 def pareto_front(Y, ref):

@@ -187,6 +187,105 @@ void bo_gp_posterior_k(const double *X, int n, int d, const double *ls, double s
   }
 }
 
+/* ---- Sec. 6: hyperparameters learned by maximising the marginal likelihood */
+double bo_gp_mll(const double *X, const double *y, int n, int d, const double *ls, double s2,
+                 double noise, double *grad) {
+  double *L = (double *)malloc(sizeof(double) * ((size_t)n * n * 2 + 2 * (size_t)n));
+  double *Ki = L + (size_t)n * n, *alpha = Ki + (size_t)n * n, *col = alpha + n;
+  double mll = NAN;
+  if (bo_gp_fit(X, y, n, d, ls, s2, noise, L, alpha) != 0) goto done;
+  /* log p(y) = -1/2 y^T alpha - sum_i log L_ii - n/2 log(2 pi) */
+  mll = -0.5 * (double)n * log(2.0 * M_PI);
+  for (int i = 0; i < n; ++i) mll += -0.5 * y[i] * alpha[i] - log(L[(long)i * n + i]);
+  if (grad) {
+    /* K^-1 column by column: solve L L^T x = e_j */
+    for (int j = 0; j < n; ++j) {
+      for (int i = 0; i < n; ++i) {
+        double s = i == j ? 1.0 : 0.0;
+        for (int k = 0; k < i; ++k) s -= L[(long)i * n + k] * col[k];
+        col[i] = s / L[(long)i * n + i];
+      }
+      for (int i = n - 1; i >= 0; --i) {
+        double s = col[i];
+        for (int k = i + 1; k < n; ++k) s -= L[(long)k * n + i] * col[k];
+        col[i] = s / L[(long)i * n + i];
+      }
+      for (int i = 0; i < n; ++i) Ki[(long)i * n + j] = col[i];
+    }
+    /* d log p / d theta = 1/2 tr((alpha alpha^T - K^-1) dK/dtheta), theta the
+     * log-parameters: dK/dlog s2 = s2 M52; dK/dlog noise = noise I;
+     * dK_ij/dlog l_t = s2 (5/3) (1 + sqrt5 r) exp(-sqrt5 r) (dx_t / l_t)^2 */
+    for (int q = 0; q < d + 2; ++q) grad[q] = 0.0;
+    for (int i = 0; i < n; ++i)
+      for (int j = 0; j < n; ++j) {
+        const double Q = alpha[i] * alpha[j] - Ki[(long)i * n + j];
+        const double *xi = X + (long)i * d, *xj = X + (long)j * d;
+        double r2 = 0.0;
+        for (int t = 0; t < d; ++t) {
+          double z = (xi[t] - xj[t]) / ls[t];
+          r2 += z * z;
+        }
+        const double r = sqrt(r2), e = exp(-sqrt(5.0) * r);
+        const double f = s2 * (5.0 / 3.0) * (1.0 + sqrt(5.0) * r) * e;
+        for (int t = 0; t < d; ++t) {
+          double z = (xi[t] - xj[t]) / ls[t];
+          grad[t] += 0.5 * Q * f * z * z;
+        }
+        grad[d] += 0.5 * Q * s2 * (1.0 + sqrt(5.0) * r + 5.0 * r2 / 3.0) * e;
+        if (i == j) grad[d + 1] += 0.5 * Q * noise;
+      }
+  }
+done:
+  free(L);
+  return mll;
+}
+
+/* Log-parameter bounds of the learner (theta = log l_1..log l_d, log s2, log noise). */
+static double clampd(double v, double lo, double hi) { return v < lo ? lo : (v > hi ? hi : v); }
+static void learn_clamp(double *th, int d) {
+  for (int t = 0; t < d; ++t) th[t] = clampd(th[t], BO_LOG_LS_MIN, BO_LOG_LS_MAX);
+  th[d] = clampd(th[d], BO_LOG_S2_MIN, BO_LOG_S2_MAX);
+  th[d + 1] = clampd(th[d + 1], BO_LOG_NOISE_MIN, BO_LOG_NOISE_MAX);
+}
+
+static double mll_at(const double *X, const double *y, int n, int d, const double *th,
+                     double *grad, double *ls) {
+  for (int t = 0; t < d; ++t) ls[t] = exp(th[t]);
+  return bo_gp_mll(X, y, n, d, ls, exp(th[d]), exp(th[d + 1]), grad);
+}
+
+int bo_gp_learn(const double *X, const double *y, int n, int d, const double *theta0, int R,
+                int iters, double lr, double *theta, double *mll, double *grad) {
+  if (n < 1 || d < 1 || R < 1 || iters < 0 || !X || !y || !theta0 || !theta || !mll) return 1;
+  const int P = d + 2;
+  double *buf = (double *)malloc(sizeof(double) * (size_t)(4 * P + d));
+  double *g = buf, *m1 = g + P, *m2 = m1 + P, *ls = m2 + P;
+  for (int r = 0; r < R; ++r) {
+    double *th = theta + (size_t)r * P;
+    memcpy(th, theta0 + (size_t)r * P, sizeof(double) * P);
+    learn_clamp(th, d);
+    for (int q = 0; q < P; ++q) m1[q] = m2[q] = 0.0;
+    double b1t = 1.0, b2t = 1.0;
+    for (int it = 0; it < iters; ++it) {
+      /* Adam ascent on the log marginal likelihood, bias-corrected moments */
+      const double v = mll_at(X, y, n, d, th, g, ls);
+      if (v != v) break; /* not positive definite: keep the last theta */
+      b1t *= BO_ADAM_B1;
+      b2t *= BO_ADAM_B2;
+      for (int q = 0; q < P; ++q) {
+        m1[q] = BO_ADAM_B1 * m1[q] + (1.0 - BO_ADAM_B1) * g[q];
+        m2[q] = BO_ADAM_B2 * m2[q] + (1.0 - BO_ADAM_B2) * g[q] * g[q];
+        const double mh = m1[q] / (1.0 - b1t), vh = m2[q] / (1.0 - b2t);
+        th[q] += lr * mh / (sqrt(vh) + BO_ADAM_EPS);
+      }
+      learn_clamp(th, d);
+    }
+    mll[r] = mll_at(X, y, n, d, th, grad ? grad + (size_t)r * P : NULL, ls);
+  }
+  free(buf);
+  return 0;
+}
+
 /* ---- Sec. 5.2: Pareto-optimal set (minimisation) ------------------------- */
 static _Thread_local const double *g_sortY;
 static _Thread_local int g_sortM;

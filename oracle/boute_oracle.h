@@ -79,6 +79,36 @@ void bo_gp_posterior_k(const double *X, int n, int d, const double *ls, double s
                        const double *kc, const double *L, const double *alpha, const float *Xc,
                        long long N, double *mean, double *var, int nthreads);
 
+/* Log marginal likelihood log p(y | X, theta) of the zero-mean GP with the
+ * Matern-5/2 kernel above (Sec. 6: the hyperparameters are learned by
+ * maximising it), -1/2 y^T K^-1 y - 1/2 log det K - n/2 log 2 pi, K = s2
+ * M52(X, X) + noise I; NaN when K is not positive definite. grad (d + 2, or
+ * NULL): its gradient with respect to theta = (log l_1 .. log l_d, log s2,
+ * log noise), 1/2 tr((alpha alpha^T - K^-1) dK/dtheta_q). */
+double bo_gp_mll(const double *X, const double *y, int n, int d, const double *ls, double s2,
+                 double noise, double *grad);
+
+/* Bounds of the learned log-parameters and the Adam constants of bo_gp_learn. */
+#define BO_LOG_LS_MIN (-6.907755278982137)    /* log 1e-3 */
+#define BO_LOG_LS_MAX (6.907755278982137)     /* log 1e3 */
+#define BO_LOG_S2_MIN (-6.907755278982137)    /* log 1e-3 */
+#define BO_LOG_S2_MAX (6.907755278982137)     /* log 1e3 */
+#define BO_LOG_NOISE_MIN (-9.210340371976182) /* log 1e-4 */
+#define BO_LOG_NOISE_MAX (2.302585092994046)  /* log 10 */
+#define BO_ADAM_B1 0.9
+#define BO_ADAM_B2 0.999
+#define BO_ADAM_EPS 1e-8
+
+/* Hyperparameter learning (Sec. 6): from each of R starting points
+ * theta0[r] (d + 2 log-parameters, clamped to the bounds above), `iters`
+ * steps of Adam ascent on bo_gp_mll with step size lr (bias-corrected first
+ * and second moments, BO_ADAM_*), each step followed by the clamp. Writes the
+ * final theta (R x (d + 2)), its log marginal likelihood mll (R) and, when
+ * grad is not NULL, the gradient there (R x (d + 2)). A restart whose K stops
+ * being positive definite keeps its last theta (mll NaN). */
+int bo_gp_learn(const double *X, const double *y, int n, int d, const double *theta0, int R,
+                int iters, double lr, double *theta, double *mll, double *grad);
+
 /* Pareto front of observed outcomes (Sec. 5.2, Pareto-optimal set; all
  * objectives minimised): point i is kept iff no j dominates it (Y_j <= Y_i in
  * every objective, < in one), no exact duplicate j < i exists, and

@@ -681,3 +681,74 @@ def test_outcome_transforms():
     # outside the domain: NaN
     bad = oracle.outcome_transform(np.array([[-1.0, 1.5]]), [1, 2])
     assert np.isnan(bad).all()
+
+
+# --------------------------- hyperparameters by marginal likelihood (Sec. 6)
+def _mll_library(X, y, th):
+    """log N(y; 0, K) by scipy on the Gram matrix of the (separately pinned)
+    Matern-5/2 kernel; th = (log l_1..log l_d, log s2, log noise)."""
+    import scipy.stats
+    d = X.shape[1]
+    ls, s2, noise = np.exp(th[:d]), math.exp(th[d]), math.exp(th[d + 1])
+    K = np.array([[oracle.matern52(a, b, ls, s2) for b in X] for a in X]) + noise * np.eye(len(X))
+    return scipy.stats.multivariate_normal(np.zeros(len(X)), K).logpdf(y)
+
+
+def _mll_problem(seed, n=24, d=3):
+    rng = np.random.default_rng(seed)
+    X = rng.random((n, d))
+    y = oracle.standardize((np.sin(3 * X[:, :1]) + X[:, 1:2] ** 2 + 0.05 * rng.normal(size=(n, 1))))
+    return X, y[:, 0]
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_mll_equals_library_logpdf(seed):
+    X, y = _mll_problem(seed)
+    th = np.array([-0.7, 0.2, -0.1, 0.3, math.log(2e-3)])
+    got = oracle.gp_mll(X, y, np.exp(th[:3]), math.exp(th[3]), math.exp(th[4]))
+    assert got == pytest.approx(_mll_library(X, y, th), rel=1e-11, abs=1e-10)
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_mll_gradient_matches_finite_differences_of_library_logpdf(seed):
+    X, y = _mll_problem(seed)
+    th = np.array([-0.7, 0.2, -0.1, 0.3, math.log(2e-3)])
+    _, g = oracle.gp_mll(X, y, np.exp(th[:3]), math.exp(th[3]), math.exp(th[4]), grad=True)
+    h = 1e-5
+    for q in range(len(th)):
+        e = np.zeros_like(th); e[q] = h
+        fd = (_mll_library(X, y, th + e) - _mll_library(X, y, th - e)) / (2 * h)
+        assert g[q] == pytest.approx(fd, rel=1e-6, abs=1e-6), q
+
+
+def test_learner_first_step_and_bounds():
+    X, y = _mll_problem(2)
+    th0 = np.array([[-0.7, 0.2, -0.1, 0.3, math.log(2e-3)],
+                    [20.0, -20.0, 0.0, 50.0, -50.0]])  # the second starts out of bounds
+    _, g = oracle.gp_mll(X, y, np.exp(th0[0, :3]), math.exp(th0[0, 3]), math.exp(th0[0, 4]),
+                         grad=True)
+    lr = 0.05
+    th1, _ = oracle.gp_learn(X, y, th0, 1, lr)
+    # Adam's first bias-corrected step: lr * g / (|g| + eps)
+    np.testing.assert_allclose(th1[0], th0[0] + lr * g / (np.abs(g) + 1e-8), rtol=0, atol=1e-12)
+    th_c, _ = oracle.gp_learn(X, y, th0[1:], 0, lr)
+    np.testing.assert_allclose(th_c[0], [oracle.LOG_LS_BOUNDS[1], oracle.LOG_LS_BOUNDS[0], 0.0,
+                                         oracle.LOG_S2_BOUNDS[1], oracle.LOG_NOISE_BOUNDS[0]])
+
+
+def test_learner_reaches_the_grid_search_optimum():
+    # one feature: a grid over (log l, log s2, log noise) of the library
+    # log-likelihood; the learner must end at least as high, near the argmax
+    rng = np.random.default_rng(5)
+    X = rng.random((20, 1))
+    y = oracle.standardize(np.sin(4 * X) + 0.1 * rng.normal(size=(20, 1)))[:, 0]
+    grid = [(a, b, c) for a in np.linspace(-2.5, 0.5, 25) for b in np.linspace(-1.5, 2.0, 15)
+            for c in np.linspace(-8.0, -1.0, 15)]
+    vals = np.array([oracle.gp_mll(X, y, [math.exp(a)], math.exp(b), math.exp(c))
+                     for a, b, c in grid])
+    best = int(np.argmax(vals))
+    assert _mll_library(X, y, np.array(grid[best])) == pytest.approx(vals[best], rel=1e-10)
+    th, mll = oracle.gp_learn(X, y, np.array([[-0.5, 0.0, -4.0], [-2.0, 1.0, -2.0]]), 1500, 0.02)
+    assert mll.max() >= vals[best] - 1e-3
+    r = int(np.argmax(mll))
+    assert abs(th[r, 0] - grid[best][0]) < 0.25
