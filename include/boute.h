@@ -110,6 +110,39 @@ void boute_gp_free(boute_gp *gp);
  * Waits for all work on the device first. */
 int boute_gp_set_kernel(boute_gp *gp, int d_tau, const double *params);
 
+/* ---- hyperparameters ----------------------------------------------------------
+ * Sec. 6: the lengthscales, outputscale and noise are learned by maximising
+ * the GP's log marginal likelihood (in double precision):
+ *   log p(y | theta) = -1/2 y^T K^-1 y - 1/2 log det K - n/2 log 2 pi,
+ *   K = s2 M52(X, X) + noise I,
+ * over theta = (log l_1 .. log l_d, log s2, log noise). For every problem b,
+ * objective t and restart r, `iters` steps of Adam ascent (bias-corrected
+ * moments, BOUTE_ADAM_B1 / B2 / EPS, step size lr) from theta0, each step
+ * followed by a clamp to the BOUTE_LOG_* bounds; then the log likelihood at
+ * the final theta. The gradient is
+ *   1/2 sum_ij (alpha_i alpha_j - K^-1_ij) dK_ij / dtheta_q,  alpha = K^-1 y.
+ *   X: B x n x d fp64; Ys: B x n x m fp64 (standardised outcomes);
+ *   theta0: B x m x R x (d + 2) fp64 starting points; theta (out, same
+ *   layout): the final log-parameters; mll (out): B x m x R; grad (out,
+ *   optional, same layout as theta): the gradient at the final theta.
+ *   All device pointers; iters >= 0 (0: evaluate at theta0); R >= 1.
+ * A restart whose K is not positive definite stops there: its theta is kept
+ * and its mll (and grad) are NaN. One block per (b, t, r); a block's n x n
+ * workspace is in shared memory up to n = 150 or so, else in stream-ordered
+ * pool memory. Asynchronous on `stream`. */
+#define BOUTE_LOG_LS_MIN (-6.907755278982137)    /* log 1e-3 */
+#define BOUTE_LOG_LS_MAX (6.907755278982137)     /* log 1e3 */
+#define BOUTE_LOG_S2_MIN (-6.907755278982137)    /* log 1e-3 */
+#define BOUTE_LOG_S2_MAX (6.907755278982137)     /* log 1e3 */
+#define BOUTE_LOG_NOISE_MIN (-9.210340371976182) /* log 1e-4 */
+#define BOUTE_LOG_NOISE_MAX (2.302585092994046)  /* log 10 */
+#define BOUTE_ADAM_B1 0.9
+#define BOUTE_ADAM_B2 0.999
+#define BOUTE_ADAM_EPS 1e-8
+int boute_gp_learn(const double *X, const double *Ys, int B, int n, int d, int m,
+                   const double *theta0, int R, int iters, double lr, double *theta,
+                   double *mll, double *grad, void *stream);
+
 /* ---- posterior ---------------------------------------------------------------
  * Latent-function posterior of every objective at N candidates per problem
  * (Sec. 5.2: the acquisition is taken over the GP posterior):

@@ -30,6 +30,7 @@ SYMBOLS = (
     "boute_engine_scores", "boute_engine_set_timing",
     "boute_engine_stage_times", "boute_engine_launches_per_step", "boute_engine_set_constraints",
     "boute_engine_set_outcome_transforms", "boute_engine_set_kernel", "boute_gp_set_kernel",
+    "boute_gp_learn",
     "boute_engine_free",
 )
 #: stage names of boute_engine_stage_times, in order
@@ -90,6 +91,8 @@ def load(path: str | None = None):
         "boute_engine_set_outcome_transforms": ([_vp, _vp], _i),
         "boute_engine_set_kernel": ([_vp, _i, _vp], _i),
         "boute_gp_set_kernel": ([_vp, _i, _vp], _i),
+        "boute_gp_learn": ([_vp, _vp, _i, _i, _i, _i, _vp, _i, _i, ctypes.c_double, _vp, _vp, _vp,
+                            _vp], _i),
         "boute_engine_free": ([_vp], None),
     }
     for name, (args, res) in sig.items():
@@ -187,6 +190,18 @@ def boute_gp_status(gp: Gp, stream=None) -> int:
 
 def boute_gp_free(gp: Gp):
     gp.free()
+
+
+def boute_gp_learn(X, Ys, theta0, iters: int, lr: float, theta, mll, grad=None, stream=None):
+    """X: B x n x d, Ys: B x n x m, theta0 / theta / grad: B x m x R x (d + 2),
+    mll: B x m x R (fp64 CUDA tensors)."""
+    f64 = torch.float64
+    B, n, d = X.shape
+    m = Ys.shape[2]
+    R = theta0.shape[2]
+    _check(load().boute_gp_learn(_p(X, f64), _p(Ys, f64), B, n, d, m, _p(theta0, f64), R,
+                                 int(iters), float(lr), _p(theta, f64), _p(mll, f64),
+                                 _p(grad, f64), _s(stream)), "boute_gp_learn")
 
 
 def _host_f64(a):

@@ -223,6 +223,18 @@ void boute_gp_free(boute_gp *gp) {
   delete gp;
 }
 
+int boute_gp_learn(const double *X, const double *Ys, int B, int n, int d, int m,
+                   const double *theta0, int R, int iters, double lr, double *theta,
+                   double *mll, double *grad, void *stream) {
+  if (!X || !Ys || !theta0 || !theta || !mll || !shape_ok(B, n, d, m) || R < 1 || iters < 0 ||
+      !(lr >= 0.0))
+    return BOUTE_ERR_INVALID_ARG;
+  if ((long long)B * m * R > (1ll << 30)) return BOUTE_ERR_INVALID_ARG;
+  if (int r = device_ok()) return r;
+  return launch_learn(X, Ys, B, n, d, m, theta0, R, iters, lr, theta, mll, grad,
+                      (cudaStream_t)stream);
+}
+
 int boute_gp_set_kernel(boute_gp *gp, int d_tau, const double *params) {
   if (!gp) return BOUTE_ERR_INVALID_ARG;
   Gp &g = gp->g;

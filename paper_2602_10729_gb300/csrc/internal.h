@@ -103,6 +103,11 @@ int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
                  const float *lower, const float *upper, const int *K, int box_cap,
                  const float *eps, int S, long long eps_stride, const double *cons, float *acq,
                  cudaStream_t s);
+// hyperparameter learning (learn.cu): B*m*R blocks, fp64; workspace from the
+// stream-ordered pool when a block's does not fit in shared memory
+int launch_learn(const double *X, const double *Ys, int B, int n, int d, int m,
+                 const double *theta0, int R, int iters, double lr, double *theta, double *mll,
+                 double *grad, cudaStream_t s);
 size_t topk_scratch_bytes(int B, long long N, int k);
 // counters_zeroed: the scratch's per-problem counters are known to be zero
 // (an engine's scratch: zeroed at creation, and every call leaves them zero);

@@ -1,0 +1,264 @@
+// Hyperparameter learning by maximising the GP's log marginal likelihood
+// (Sec. 6: the ARD lengthscales and outputscale are learned jointly by
+// maximising the marginal likelihood; all kernels in double precision).
+//
+// One block per (problem, objective, restart) runs the whole optimisation:
+// per Adam step it builds K = s2 M52(X, X) + noise I in fp64, factors it in
+// place (right-looking Cholesky), inverts the factor in place, forms K^-1 in
+// place, alpha = K^-1 y, the log likelihood and its gradient with respect to
+// theta = (log l_1 .. log l_d, log s2, log noise),
+//   d log p / d theta_q = 1/2 sum_ij (alpha_i alpha_j - K^-1_ij) dK_ij / dtheta_q,
+// then takes a bias-corrected Adam ascent step and clamps theta to its
+// bounds. The lower triangle of the n x n workspace holds K, then L, then
+// L^-1, then K^-1; the upper triangle keeps exp(-sqrt5 r_ij) for the gradient.
+// The workspace is in shared memory when it fits, else in global memory
+// (one slice per block, L2-resident).
+#include <math.h>
+
+#include "internal.h"
+
+namespace boute {
+
+namespace {
+
+constexpr int kLearnThreads = 256;
+constexpr int kLearnWarps = kLearnThreads / 32;
+constexpr double kSqrt5d = 2.23606797749978969641;
+constexpr double kLog2Pi = 1.83787706640934548356;
+
+__device__ __forceinline__ double warp_sum_d(double v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ double clamp_d(double v, double lo, double hi) {
+  return v < lo ? lo : (v > hi ? hi : v);
+}
+
+// Doubles of one block's workspace: A (n x n), X (n x d), y, alpha, tmp (n each).
+__host__ __device__ inline size_t learn_ws_doubles(int n, int d) {
+  return (size_t)n * n + (size_t)n * d + 3 * (size_t)n;
+}
+
+__global__ void __launch_bounds__(kLearnThreads) learn_kernel(
+    const double *X, const double *Ys, int n, int d, int m, int R, const double *theta0,
+    int iters, double lr, double *theta_out, double *mll_out, double *grad_out, double *ws,
+    int use_smem) {
+  extern __shared__ __align__(16) double lsm[];
+  __shared__ double th[BOUTE_MAX_D + 2], m1[BOUTE_MAX_D + 2], m2[BOUTE_MAX_D + 2];
+  __shared__ double il[BOUTE_MAX_D], red[kLearnWarps][BOUTE_MAX_D + 2];
+  __shared__ double logdet, mll_s;
+  __shared__ int bad;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int blk = blockIdx.x, r = blk % R, bt = blk / R, b = bt / m, t = bt % m;
+  const int P = d + 2;
+  double *A = use_smem ? lsm : ws + (size_t)blk * learn_ws_doubles(n, d);
+  double *xs = A + (size_t)n * n, *yv = xs + (size_t)n * d, *av = yv + n, *tmp = av + n;
+  for (int e = tid; e < n * d; e += kLearnThreads) xs[e] = X[(size_t)b * n * d + e];
+  for (int i = tid; i < n; i += kLearnThreads) yv[i] = Ys[((size_t)b * n + i) * m + t];
+  const double *th0 = theta0 + (size_t)blk * P;
+  if (tid < P) {
+    const double v = th0[tid];
+    th[tid] = tid < d ? clamp_d(v, BOUTE_LOG_LS_MIN, BOUTE_LOG_LS_MAX)
+              : tid == d ? clamp_d(v, BOUTE_LOG_S2_MIN, BOUTE_LOG_S2_MAX)
+                         : clamp_d(v, BOUTE_LOG_NOISE_MIN, BOUTE_LOG_NOISE_MAX);
+    m1[tid] = 0.0;
+    m2[tid] = 0.0;
+  }
+  double b1t = 1.0, b2t = 1.0;
+  __syncthreads();
+
+  for (int it = 0; it <= iters; ++it) {
+    const bool last = it == iters;
+    const bool want_grad = !last || grad_out != nullptr;
+    // ---- K (lower) and exp(-sqrt5 r) (upper) at theta
+    if (tid < d) il[tid] = exp(-th[tid]);
+    if (tid == 0) {
+      bad = 0;
+      logdet = 0.0;
+    }
+    __syncthreads();
+    const double s2 = exp(th[d]), nz = exp(th[d + 1]);
+    for (int e = tid; e < n * n; e += kLearnThreads) {
+      const int i = e / n, j = e - i * n;
+      if (j > i) continue;
+      double r2 = 0.0;
+      for (int q = 0; q < d; ++q) {
+        const double z = (xs[i * d + q] - xs[j * d + q]) * il[q];
+        r2 = fma(z, z, r2);
+      }
+      const double rr = sqrt(r2), sr = kSqrt5d * rr, ex = exp(-sr);
+      A[(size_t)i * n + j] = s2 * (1.0 + sr + 5.0 * r2 / 3.0) * ex + (i == j ? nz : 0.0);
+      if (i != j) A[(size_t)j * n + i] = ex;
+    }
+    // ---- Cholesky in place (lower), column by column
+    for (int j = 0; j < n; ++j) {
+      __syncthreads();
+      const double djj = A[(size_t)j * n + j];
+      if (!(djj > 0.0)) {  // not positive definite (every thread sees the same value)
+        if (tid == 0) bad = 1;
+        break;
+      }
+      const double Ljj = sqrt(djj), inv = 1.0 / Ljj;
+      for (int i = j + 1 + tid; i < n; i += kLearnThreads) A[(size_t)i * n + j] *= inv;
+      __syncthreads();
+      // (the diagonal entry is replaced only now: every thread has read it)
+      if (tid == 0) {
+        A[(size_t)j * n + j] = Ljj;
+        logdet += log(Ljj);
+      }
+      for (int i = j + 1 + warp; i < n; i += kLearnWarps) {
+        const double lij = A[(size_t)i * n + j];
+        for (int k = j + 1 + lane; k <= i; k += 32) A[(size_t)i * n + k] -= lij * A[(size_t)k * n + j];
+      }
+    }
+    __syncthreads();
+    if (bad) break;  // keeps theta; the evaluation after the loop reports NaN
+    // ---- L^-1 in place, last column first: column j needs the columns > j of
+    // L^-1 and column j of L
+    for (int j = n - 1; j >= 0; --j) {
+      const double ijj = 1.0 / A[(size_t)j * n + j];
+      for (int i = j + 1 + warp; i < n; i += kLearnWarps) {
+        double s = 0.0;
+        for (int k = j + 1 + lane; k <= i; k += 32) s = fma(A[(size_t)i * n + k], A[(size_t)k * n + j], s);
+        s = warp_sum_d(s);
+        if (lane == 0) tmp[i] = -s * ijj;
+      }
+      __syncthreads();
+      for (int i = j + 1 + tid; i < n; i += kLearnThreads) A[(size_t)i * n + j] = tmp[i];
+      if (tid == 0) A[(size_t)j * n + j] = ijj;
+      __syncthreads();
+    }
+    // ---- K^-1 = L^-T L^-1 in place, row by row: row i needs rows >= i of L^-1
+    for (int i = 0; i < n; ++i) {
+      for (int j = warp; j <= i; j += kLearnWarps) {
+        double s = 0.0;
+        for (int k = i + lane; k < n; k += 32) s = fma(A[(size_t)k * n + i], A[(size_t)k * n + j], s);
+        s = warp_sum_d(s);
+        if (lane == 0) tmp[j] = s;
+      }
+      __syncthreads();
+      for (int j = tid; j <= i; j += kLearnThreads) A[(size_t)i * n + j] = tmp[j];
+      __syncthreads();
+    }
+    // ---- alpha = K^-1 y and the log likelihood
+    for (int i = warp; i < n; i += kLearnWarps) {
+      double s = 0.0;
+      for (int j = lane; j < n; j += 32) {
+        const double kij = j <= i ? A[(size_t)i * n + j] : A[(size_t)j * n + i];
+        s = fma(kij, yv[j], s);
+      }
+      s = warp_sum_d(s);
+      if (lane == 0) av[i] = s;
+    }
+    __syncthreads();
+    if (tid < 32) {
+      double s = 0.0;
+      for (int i = lane; i < n; i += 32) s = fma(yv[i], av[i], s);
+      s = warp_sum_d(s);
+      if (lane == 0) mll_s = -0.5 * s - logdet - 0.5 * (double)n * kLog2Pi;
+    }
+    if (!want_grad) break;
+    // ---- gradient: pairs i >= j (an off-diagonal pair stands for two
+    // entries); per pair f = s2 (5/3) (1 + sqrt5 r) e^(-sqrt5 r) multiplies
+    // (dx_q / l_q)^2 in the lengthscale terms
+    double g[BOUTE_MAX_D], gs2 = 0.0, gnz = 0.0;
+#pragma unroll
+    for (int q = 0; q < BOUTE_MAX_D; ++q) g[q] = 0.0;
+    for (int e = tid; e < n * n; e += kLearnThreads) {
+      const int i = e / n, j = e - i * n;
+      if (j > i) continue;
+      const double Q = (i == j ? 0.5 : 1.0) * (av[i] * av[j] - A[(size_t)i * n + j]);
+      const double *xi = xs + (size_t)i * d, *xj = xs + (size_t)j * d;
+      double r2 = 0.0;
+      for (int q = 0; q < d; ++q) {
+        const double z = (xi[q] - xj[q]) * il[q];
+        r2 = fma(z, z, r2);
+      }
+      const double rr = sqrt(r2), sr = kSqrt5d * rr;
+      const double ex = i == j ? 1.0 : A[(size_t)j * n + i];
+      const double Qf = Q * s2 * (5.0 / 3.0) * (1.0 + sr) * ex;
+#pragma unroll
+      for (int q = 0; q < BOUTE_MAX_D; ++q) {
+        if (q < d) {
+          const double z = (xi[q] - xj[q]) * il[q];
+          g[q] = fma(Qf, z * z, g[q]);
+        }
+      }
+      gs2 = fma(Q, s2 * (1.0 + sr + 5.0 * r2 / 3.0) * ex, gs2);
+      if (i == j) gnz = fma(Q, nz, gnz);
+    }
+    // block sums of the d + 2 components (the pair sums already carry the 1/2)
+#pragma unroll
+    for (int q = 0; q < BOUTE_MAX_D; ++q) {
+      if (q < d) {
+        const double v = warp_sum_d(g[q]);
+        if (lane == 0) red[warp][q] = v;
+      }
+    }
+    {
+      const double a = warp_sum_d(gs2), c = warp_sum_d(gnz);
+      if (lane == 0) {
+        red[warp][d] = a;
+        red[warp][d + 1] = c;
+      }
+    }
+    __syncthreads();
+    if (tid < P) {
+      double v = 0.0;
+      for (int w = 0; w < kLearnWarps; ++w) v += red[w][tid];
+      if (last) {
+        grad_out[(size_t)blk * P + tid] = v;
+      } else {
+        // Adam ascent step, bias-corrected moments, then the bounds
+        b1t *= BOUTE_ADAM_B1;
+        b2t *= BOUTE_ADAM_B2;
+        m1[tid] = BOUTE_ADAM_B1 * m1[tid] + (1.0 - BOUTE_ADAM_B1) * v;
+        m2[tid] = BOUTE_ADAM_B2 * m2[tid] + (1.0 - BOUTE_ADAM_B2) * v * v;
+        const double mh = m1[tid] / (1.0 - b1t), vh = m2[tid] / (1.0 - b2t);
+        const double nt = th[tid] + lr * mh / (sqrt(vh) + BOUTE_ADAM_EPS);
+        th[tid] = tid < d ? clamp_d(nt, BOUTE_LOG_LS_MIN, BOUTE_LOG_LS_MAX)
+                  : tid == d ? clamp_d(nt, BOUTE_LOG_S2_MIN, BOUTE_LOG_S2_MAX)
+                             : clamp_d(nt, BOUTE_LOG_NOISE_MIN, BOUTE_LOG_NOISE_MAX);
+      }
+    }
+    __syncthreads();
+  }
+  __syncthreads();
+  if (tid < P) theta_out[(size_t)blk * P + tid] = th[tid];
+  if (tid == 0) mll_out[blk] = bad ? nan("") : mll_s;
+  if (bad && grad_out && tid < P) grad_out[(size_t)blk * P + tid] = nan("");
+}
+
+}  // namespace
+
+size_t learn_smem_limit() { return 200 * 1024; }
+
+int launch_learn(const double *X, const double *Ys, int B, int n, int d, int m,
+                 const double *theta0, int R, int iters, double lr, double *theta, double *mll,
+                 double *grad, cudaStream_t s) {
+  const size_t per = learn_ws_doubles(n, d) * sizeof(double);
+  const int blocks = B * m * R;
+  const bool smem = per <= learn_smem_limit();
+  double *ws = nullptr;
+  if (!smem) {
+    if (cudaMallocAsync((void **)&ws, per * blocks, s) != cudaSuccess) {
+      cudaGetLastError();
+      return BOUTE_ERR_OOM;
+    }
+  } else {
+    prefer_shared(learn_kernel);
+    if (cudaFuncSetAttribute(learn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)per) != cudaSuccess)
+      return last_launch_status();
+  }
+  learn_kernel<<<blocks, kLearnThreads, smem ? per : 0, s>>>(X, Ys, n, d, m, R, theta0, iters, lr,
+                                                             theta, mll, grad, ws, smem ? 1 : 0);
+  count_launch();
+  const int st = last_launch_status();
+  if (ws) cudaFreeAsync(ws, s);
+  return st;
+}
+
+}  // namespace boute
