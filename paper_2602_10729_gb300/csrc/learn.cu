@@ -23,6 +23,7 @@ namespace {
 
 constexpr int kLearnThreads = 256;
 constexpr int kLearnWarps = kLearnThreads / 32;
+constexpr int kLearnRows = 8;  // rows of K^-1 formed per pass
 constexpr double kSqrt5d = 2.23606797749978969641;
 constexpr double kLog2Pi = 1.83787706640934548356;
 
@@ -32,13 +33,27 @@ __device__ __forceinline__ double warp_sum_d(double v) {
   return v;
 }
 
+// Entry e of a lower triangle (diagonal included, row by row) -> (i, j).
+__device__ __forceinline__ void tri_index(int e, int &i, int &j) {
+  int r = (int)((sqrtf(8.f * (float)e + 1.f) - 1.f) * 0.5f);
+  while (r * (r + 1) / 2 > e) --r;
+  while ((r + 1) * (r + 2) / 2 <= e) ++r;
+  i = r;
+  j = e - r * (r + 1) / 2;
+}
+
 __device__ __forceinline__ double clamp_d(double v, double lo, double hi) {
   return v < lo ? lo : (v > hi ? hi : v);
 }
 
-// Doubles of one block's workspace: A (n x n), X (n x d), y, alpha, tmp (n each).
+// Row stride of the n x n workspace: odd, so that a column's 64-bit entries
+// fall in different shared-memory banks.
+__host__ __device__ inline int learn_ld(int n) { return n | 1; }
+
+// Doubles of one block's workspace: A (n x ld), X (n x d), y, alpha, tmp,
+// 1 / L_jj (n each), tmp2 (kLearnRows rows of K^-1).
 __host__ __device__ inline size_t learn_ws_doubles(int n, int d) {
-  return (size_t)n * n + (size_t)n * d + 3 * (size_t)n;
+  return (size_t)n * learn_ld(n) + (size_t)n * d + 4 * (size_t)n + (size_t)kLearnRows * n;
 }
 
 __global__ void __launch_bounds__(kLearnThreads) learn_kernel(
@@ -52,9 +67,10 @@ __global__ void __launch_bounds__(kLearnThreads) learn_kernel(
   __shared__ int bad;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int blk = blockIdx.x, r = blk % R, bt = blk / R, b = bt / m, t = bt % m;
-  const int P = d + 2;
+  const int P = d + 2, ld = learn_ld(n);
   double *A = use_smem ? lsm : ws + (size_t)blk * learn_ws_doubles(n, d);
-  double *xs = A + (size_t)n * n, *yv = xs + (size_t)n * d, *av = yv + n, *tmp = av + n;
+  double *xs = A + (size_t)n * ld, *yv = xs + (size_t)n * d, *av = yv + n, *tmp = av + n, *dinv = tmp + n,
+         *tmp2 = dinv + n;
   for (int e = tid; e < n * d; e += kLearnThreads) xs[e] = X[(size_t)b * n * d + e];
   for (int i = tid; i < n; i += kLearnThreads) yv[i] = Ys[((size_t)b * n + i) * m + t];
   const double *th0 = theta0 + (size_t)blk * P;
@@ -74,79 +90,108 @@ __global__ void __launch_bounds__(kLearnThreads) learn_kernel(
     const bool want_grad = !last || grad_out != nullptr;
     // ---- K (lower) and exp(-sqrt5 r) (upper) at theta
     if (tid < d) il[tid] = exp(-th[tid]);
-    if (tid == 0) {
-      bad = 0;
-      logdet = 0.0;
-    }
+    if (tid == 0) bad = 0;
     __syncthreads();
     const double s2 = exp(th[d]), nz = exp(th[d + 1]);
-    for (int e = tid; e < n * n; e += kLearnThreads) {
-      const int i = e / n, j = e - i * n;
-      if (j > i) continue;
+    const int npair = n * (n + 1) / 2;  // pairs i >= j, one thread each
+    for (int e = tid; e < npair; e += kLearnThreads) {
+      int i, j;
+      tri_index(e, i, j);
       double r2 = 0.0;
       for (int q = 0; q < d; ++q) {
         const double z = (xs[i * d + q] - xs[j * d + q]) * il[q];
         r2 = fma(z, z, r2);
       }
       const double rr = sqrt(r2), sr = kSqrt5d * rr, ex = exp(-sr);
-      A[(size_t)i * n + j] = s2 * (1.0 + sr + 5.0 * r2 / 3.0) * ex + (i == j ? nz : 0.0);
-      if (i != j) A[(size_t)j * n + i] = ex;
+      A[(size_t)i * ld + j] = s2 * (1.0 + sr + 5.0 * r2 / 3.0) * ex + (i == j ? nz : 0.0);
+      if (i != j) A[(size_t)j * ld + i] = ex;
     }
     // ---- Cholesky in place (lower), column by column
     for (int j = 0; j < n; ++j) {
       __syncthreads();
-      const double djj = A[(size_t)j * n + j];
+      const double djj = A[(size_t)j * ld + j];
       if (!(djj > 0.0)) {  // not positive definite (every thread sees the same value)
         if (tid == 0) bad = 1;
         break;
       }
-      const double Ljj = sqrt(djj), inv = 1.0 / Ljj;
-      for (int i = j + 1 + tid; i < n; i += kLearnThreads) A[(size_t)i * n + j] *= inv;
+      // one reciprocal square root on the column's critical path
+      const double inv = rsqrt(djj), Ljj = djj * inv;
+      for (int i = j + 1 + tid; i < n; i += kLearnThreads) A[(size_t)i * ld + j] *= inv;
       __syncthreads();
       // (the diagonal entry is replaced only now: every thread has read it)
-      if (tid == 0) {
-        A[(size_t)j * n + j] = Ljj;
-        logdet += log(Ljj);
-      }
+      if (tid == 0) A[(size_t)j * ld + j] = Ljj;
       for (int i = j + 1 + warp; i < n; i += kLearnWarps) {
-        const double lij = A[(size_t)i * n + j];
-        for (int k = j + 1 + lane; k <= i; k += 32) A[(size_t)i * n + k] -= lij * A[(size_t)k * n + j];
+        const double lij = A[(size_t)i * ld + j];
+        for (int k = j + 1 + lane; k <= i; k += 32)
+          A[(size_t)i * ld + k] = fma(-lij, A[(size_t)k * ld + j], A[(size_t)i * ld + k]);
       }
     }
     __syncthreads();
     if (bad) break;  // keeps theta; the evaluation after the loop reports NaN
-    // ---- L^-1 in place, last column first: column j needs the columns > j of
-    // L^-1 and column j of L
-    for (int j = n - 1; j >= 0; --j) {
-      const double ijj = 1.0 / A[(size_t)j * n + j];
-      for (int i = j + 1 + warp; i < n; i += kLearnWarps) {
-        double s = 0.0;
-        for (int k = j + 1 + lane; k <= i; k += 32) s = fma(A[(size_t)i * n + k], A[(size_t)k * n + j], s);
-        s = warp_sum_d(s);
-        if (lane == 0) tmp[i] = -s * ijj;
-      }
-      __syncthreads();
-      for (int i = j + 1 + tid; i < n; i += kLearnThreads) A[(size_t)i * n + j] = tmp[i];
-      if (tid == 0) A[(size_t)j * n + j] = ijj;
-      __syncthreads();
+    // log det K = 2 sum_j log L_jj (off the factorisation's critical path),
+    // and the reciprocals of the diagonal for the inversion
+    if (warp == 0) {
+      double s = 0.0;
+      for (int j = lane; j < n; j += 32) s += log(A[(size_t)j * ld + j]);
+      s = warp_sum_d(s);
+      if (lane == 0) logdet = s;
     }
-    // ---- K^-1 = L^-T L^-1 in place, row by row: row i needs rows >= i of L^-1
-    for (int i = 0; i < n; ++i) {
-      for (int j = warp; j <= i; j += kLearnWarps) {
+    for (int j = tid; j < n; j += kLearnThreads) dinv[j] = 1.0 / A[(size_t)j * ld + j];
+    __syncthreads();
+    // ---- L^-1 in place by forward substitution of L X = I, right-looking:
+    // step k finishes row k of X (row k of B divided by L_kk) and subtracts
+    // L_ik times it from the rows i > k of B (B = I initially). Entry (i, c)
+    // holds L_ic until step c has used it, then B_ic, then X_ic.
+    for (int k = 0; k < n; ++k) {
+      const double ikk = dinv[k];
+      for (int i = k + 1 + tid; i < n; i += kLearnThreads) tmp[i] = A[(size_t)i * ld + k];
+      __syncthreads();  // column k of L saved; every thread has read L_kk
+      for (int c = tid; c <= k; c += kLearnThreads)
+        A[(size_t)k * ld + c] = c == k ? ikk : A[(size_t)k * ld + c] * ikk;
+      __syncthreads();
+      const int w = k + 1;  // entries per row to update: columns 0 .. k
+      for (int e = tid; e < (n - k - 1) * w; e += kLearnThreads) {
+        const int i = k + 1 + e / w, c = e - (e / w) * w;
+        const double xkc = A[(size_t)k * ld + c];
+        A[(size_t)i * ld + c] = c == k ? -tmp[i] * xkc : fma(-tmp[i], xkc, A[(size_t)i * ld + c]);
+      }
+      __syncthreads();  // tmp is rewritten by the next step
+    }
+    // ---- K^-1 = X^T X in place (X = L^-1 lower), kLearnRows rows at a time:
+    // entry (i, j <= i) is sum_{k >= i} X_ki X_kj, which needs only rows >= i
+    // of X, so a batch of rows is computed into tmp2 and written back after
+    __syncthreads();
+    for (int i0 = 0; i0 < n; i0 += kLearnRows) {
+      const int i1 = min(n, i0 + kLearnRows);
+      const int cnt = (i1 - i0) * i0 + (i1 - i0) * (i1 - i0 + 1) / 2;  // entries j <= i
+      for (int e = tid; e < cnt; e += kLearnThreads) {
+        // entry e -> (i, j): rows of i0 + 1, i0 + 2, ... entries
+        int i = i0, base = 0;
+        while (base + i + 1 <= e) {
+          base += i + 1;
+          ++i;
+        }
+        const int j = e - base;
         double s = 0.0;
-        for (int k = i + lane; k < n; k += 32) s = fma(A[(size_t)k * n + i], A[(size_t)k * n + j], s);
-        s = warp_sum_d(s);
-        if (lane == 0) tmp[j] = s;
+        for (int k = i; k < n; ++k) s = fma(A[(size_t)k * ld + i], A[(size_t)k * ld + j], s);
+        tmp2[e] = s;
       }
       __syncthreads();
-      for (int j = tid; j <= i; j += kLearnThreads) A[(size_t)i * n + j] = tmp[j];
+      for (int e = tid; e < cnt; e += kLearnThreads) {
+        int i = i0, base = 0;
+        while (base + i + 1 <= e) {
+          base += i + 1;
+          ++i;
+        }
+        A[(size_t)i * ld + (e - base)] = tmp2[e];
+      }
       __syncthreads();
     }
     // ---- alpha = K^-1 y and the log likelihood
     for (int i = warp; i < n; i += kLearnWarps) {
       double s = 0.0;
       for (int j = lane; j < n; j += 32) {
-        const double kij = j <= i ? A[(size_t)i * n + j] : A[(size_t)j * n + i];
+        const double kij = j <= i ? A[(size_t)i * ld + j] : A[(size_t)j * ld + i];
         s = fma(kij, yv[j], s);
       }
       s = warp_sum_d(s);
@@ -166,10 +211,10 @@ __global__ void __launch_bounds__(kLearnThreads) learn_kernel(
     double g[BOUTE_MAX_D], gs2 = 0.0, gnz = 0.0;
 #pragma unroll
     for (int q = 0; q < BOUTE_MAX_D; ++q) g[q] = 0.0;
-    for (int e = tid; e < n * n; e += kLearnThreads) {
-      const int i = e / n, j = e - i * n;
-      if (j > i) continue;
-      const double Q = (i == j ? 0.5 : 1.0) * (av[i] * av[j] - A[(size_t)i * n + j]);
+    for (int e = tid; e < npair; e += kLearnThreads) {
+      int i, j;
+      tri_index(e, i, j);
+      const double Q = (i == j ? 0.5 : 1.0) * (av[i] * av[j] - A[(size_t)i * ld + j]);
       const double *xi = xs + (size_t)i * d, *xj = xs + (size_t)j * d;
       double r2 = 0.0;
       for (int q = 0; q < d; ++q) {
@@ -177,7 +222,7 @@ __global__ void __launch_bounds__(kLearnThreads) learn_kernel(
         r2 = fma(z, z, r2);
       }
       const double rr = sqrt(r2), sr = kSqrt5d * rr;
-      const double ex = i == j ? 1.0 : A[(size_t)j * n + i];
+      const double ex = i == j ? 1.0 : A[(size_t)j * ld + i];
       const double Qf = Q * s2 * (5.0 / 3.0) * (1.0 + sr) * ex;
 #pragma unroll
       for (int q = 0; q < BOUTE_MAX_D; ++q) {
