@@ -328,6 +328,48 @@ int boute_engine_set_outcome_transforms(boute_engine *e, const int *codes);
 int boute_engine_set_kernel(boute_engine *e, int d_tau, const double *params);
 void boute_engine_free(boute_engine *e);
 
+/* ---- the optimisation loop ------------------------------------------------------
+ * Sec. 5.2 "Overall MOBO workflow" (i)-(iii), on one problem over a fixed
+ * candidate pool: each iteration (i) takes the n observations so far and,
+ * when learn_iters > 0, learns the hyperparameters by learn_iters Adam steps
+ * from the current ones (boute_gp_learn, one restart; an objective whose
+ * kernel matrix is not positive definite keeps its hyperparameters);
+ * (ii) scores the pool with the engine (boute_engine_step, k = 1) and
+ * (iii) evaluates the best candidate with `f` and adds it to X, Y. It stops
+ * when n reaches max_evals or when the observed Pareto set (the observations
+ * not dominated after the outcome transforms) has stayed the same for
+ * `patience` consecutive iterations (Sec. 7 counts the algorithm converged
+ * when the solution is stable for more than 20 consecutive iterations).
+ *   f: returns 0 and writes y (m outcomes, raw: before transforms) for x
+ *      (d features); a nonzero return stops the loop with INVALID_ARG.
+ *   cand: HOST N x d fp32 pool; eps: HOST N x m x S fp32 base normals
+ *      (mode BOUTE_ACQ_MC_HVI, reused every iteration), else NULL;
+ *   ref: m reference point (standardised units); transforms: m codes or
+ *      NULL; cons: m thresholds or NULL (the constrained acquisition);
+ *   ls (m x d), s2 (m), noise (m): HOST hyperparameters, updated in place
+ *      when learning;
+ *   X (max_evals x d), Y (max_evals x m): HOST, the first n0 rows given;
+ *   sel (out, max_evals - n0): the candidate index chosen per iteration;
+ *   theta_hist (out, optional, (max_evals - n0) x m x (d + 2)): the
+ *      log-hyperparameters each iteration scored with;
+ *   n_out: observations at the end; converged: 1 if the stability test
+ *      stopped the loop.
+ * Synchronous; allocates its device buffers and one engine per iteration. */
+typedef int (*boute_objective_fn)(const double *x, int d, double *y, int m, void *user);
+typedef struct {
+  int mode;         /* BOUTE_ACQ_EHVI2D or BOUTE_ACQ_MC_HVI */
+  int S;            /* Monte-Carlo samples (BOUTE_ACQ_MC_HVI) */
+  int max_evals;    /* observations at which the loop stops */
+  int patience;     /* consecutive iterations of an unchanged Pareto set */
+  int learn_iters;  /* Adam steps per iteration; 0 keeps the hyperparameters */
+  double learn_lr;  /* Adam step size */
+} boute_mobo_config;
+int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const float *cand, long long N,
+                   const float *eps, const double *ref, const int *transforms,
+                   const double *cons, double *ls, double *s2, double *noise, double *X,
+                   double *Y, int n0, boute_objective_fn f, void *user, long long *sel,
+                   double *theta_hist, int *n_out, int *converged);
+
 #ifdef __cplusplus
 }
 #endif

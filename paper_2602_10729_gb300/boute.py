@@ -30,7 +30,7 @@ SYMBOLS = (
     "boute_engine_scores", "boute_engine_set_timing",
     "boute_engine_stage_times", "boute_engine_launches_per_step", "boute_engine_set_constraints",
     "boute_engine_set_outcome_transforms", "boute_engine_set_kernel", "boute_gp_set_kernel",
-    "boute_gp_learn",
+    "boute_gp_learn", "boute_mobo_run",
     "boute_engine_free",
 )
 #: stage names of boute_engine_stage_times, in order
@@ -40,6 +40,18 @@ _lib = None
 _vp = ctypes.c_void_p
 _i = ctypes.c_int
 _ll = ctypes.c_longlong
+
+
+class MoboConfig(ctypes.Structure):
+    """boute_mobo_config."""
+    _fields_ = [("mode", ctypes.c_int), ("S", ctypes.c_int), ("max_evals", ctypes.c_int),
+                ("patience", ctypes.c_int), ("learn_iters", ctypes.c_int),
+                ("learn_lr", ctypes.c_double)]
+
+
+#: boute_objective_fn
+ObjectiveFn = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.POINTER(ctypes.c_double), ctypes.c_int,
+                               ctypes.POINTER(ctypes.c_double), ctypes.c_int, ctypes.c_void_p)
 
 
 class BouteError(RuntimeError):
@@ -93,6 +105,9 @@ def load(path: str | None = None):
         "boute_gp_set_kernel": ([_vp, _i, _vp], _i),
         "boute_gp_learn": ([_vp, _vp, _i, _i, _i, _i, _vp, _i, _i, ctypes.c_double, _vp, _vp, _vp,
                             _vp], _i),
+        "boute_mobo_run": ([ctypes.POINTER(MoboConfig), _i, _i, _vp, _ll, _vp, _vp, _vp, _vp, _vp,
+                            _vp, _vp, _vp, _vp, _i, ObjectiveFn, _vp, _vp, _vp,
+                            ctypes.POINTER(_i), ctypes.POINTER(_i)], _i),
         "boute_engine_free": ([_vp], None),
     }
     for name, (args, res) in sig.items():
@@ -202,6 +217,61 @@ def boute_gp_learn(X, Ys, theta0, iters: int, lr: float, theta, mll, grad=None, 
     _check(load().boute_gp_learn(_p(X, f64), _p(Ys, f64), B, n, d, m, _p(theta0, f64), R,
                                  int(iters), float(lr), _p(theta, f64), _p(mll, f64),
                                  _p(grad, f64), _s(stream)), "boute_gp_learn")
+
+
+def boute_mobo_run(objective, cand, ref, ls, s2, noise, X0, Y0, *, mode=BOUTE_ACQ_EHVI2D, S=0,
+                   eps=None, max_evals=50, patience=20, learn_iters=0, learn_lr=0.05,
+                   transforms=None, cons=None):
+    """The optimisation loop. objective(x: (d,) float64 array) -> m outcomes.
+    cand: N x d; eps: N x m x S (mode MC); ls: m x d, s2, noise: m (initial
+    hyperparameters); X0 / Y0: the first observations. Returns a dict with X,
+    Y (the n observations), sel (the chosen candidate per iteration), theta
+    (the log-hyperparameters of each iteration), ls, s2, noise (final),
+    converged."""
+    import numpy as np
+    cand = np.ascontiguousarray(cand, np.float32)
+    N, d = cand.shape
+    X0 = np.asarray(X0, np.float64)
+    Y0 = np.asarray(Y0, np.float64)
+    n0, m = Y0.shape
+    X = np.zeros((max_evals, d))
+    Y = np.zeros((max_evals, m))
+    X[:n0], Y[:n0] = X0, Y0
+    ls = np.ascontiguousarray(ls, np.float64).copy()
+    s2 = np.ascontiguousarray(s2, np.float64).copy()
+    noise = np.ascontiguousarray(noise, np.float64).copy()
+    iters = max(max_evals - n0, 1)
+    sel = np.zeros(iters, np.int64)
+    theta = np.zeros((iters, m, d + 2))
+    ref = np.ascontiguousarray(ref, np.float64)
+    eps = None if eps is None else np.ascontiguousarray(eps, np.float32)
+    tf = None if transforms is None else np.ascontiguousarray(transforms, np.int32)
+    cs = None if cons is None else np.ascontiguousarray(cons, np.float64)
+    errors = []
+
+    def cb(xp, dd, yp, mm, user):
+        try:
+            y = np.asarray(objective(np.ctypeslib.as_array(xp, (dd,)).copy()), np.float64)
+            for t in range(mm):
+                yp[t] = float(y[t])
+            return 0
+        except Exception as exc:  # reported after the loop returns
+            errors.append(exc)
+            return 1
+
+    fn = ObjectiveFn(cb)
+    cfg = MoboConfig(mode, S, max_evals, patience, learn_iters, learn_lr)
+    n_out, conv = ctypes.c_int(0), ctypes.c_int(0)
+    a = lambda v: None if v is None else v.ctypes.data
+    rc = load().boute_mobo_run(ctypes.byref(cfg), d, m, a(cand), N, a(eps), a(ref), a(tf), a(cs),
+                               a(ls), a(s2), a(noise), a(X), a(Y), n0, fn, None, a(sel), a(theta),
+                               ctypes.byref(n_out), ctypes.byref(conv))
+    if errors:
+        raise errors[0]
+    _check(rc, "boute_mobo_run")
+    n = n_out.value
+    return dict(X=X[:n], Y=Y[:n], sel=sel[:n - n0], theta=theta[:n - n0], ls=ls, s2=s2,
+                noise=noise, converged=bool(conv.value))
 
 
 def _host_f64(a):

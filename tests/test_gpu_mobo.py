@@ -1,0 +1,105 @@
+"""The optimisation loop (Sec. 5.2 "Overall MOBO workflow" (i)-(iii), stopped
+by the stability rule of Sec. 7) on the GPU against the oracle: every
+iteration's choice must be a best candidate of the oracle's acquisition on
+the same observations and hyperparameters, the learned hyperparameters must
+be the oracle learner's from the same start, the observations must be the
+objective at the chosen candidates, and the loop must stop exactly when the
+observed Pareto set has been stable for `patience` iterations."""
+import numpy as np
+import pytest
+
+import oracle
+from oracle import pipeline as opl
+
+pytestmark = pytest.mark.gpu
+
+
+def _objective(x):
+    d = x.size
+    return np.array([((x - 0.25) ** 2).sum() / d, ((x - 0.75) ** 2).sum() / d])
+
+
+def _pareto_set(Y):
+    mask, _ = oracle.pareto_front(Y, np.full(Y.shape[1], np.inf))
+    return set(np.flatnonzero(mask).tolist())
+
+
+def _check_run(res, cand, n0, patience, max_evals, mode, eps, ls0, s2, noise, learn):
+    X, Y, sel, theta = res["X"], res["Y"], res["sel"], res["theta"]
+    n = len(X)
+    assert n == n0 + len(sel)
+    ref = np.array([1.1, 1.1])
+    d = cand.shape[1]
+    th_prev = np.concatenate([np.log(ls0), np.log(s2)[:, None], np.log(noise)[:, None]], 1)
+    for t, pick in enumerate(sel):
+        nt = n0 + t
+        np.testing.assert_array_equal(X[nt], cand[pick].astype(np.float64))
+        np.testing.assert_array_equal(Y[nt], _objective(X[nt]))
+        th = theta[t]
+        if learn:  # the oracle learner from the previous iteration's parameters
+            ys = oracle.standardize(Y[:nt])
+            for obj in range(2):
+                th_o, mll_o = oracle.gp_learn(X[:nt], ys[:, obj], th_prev[obj][None], learn[0],
+                                              learn[1])
+                np.testing.assert_allclose(th[obj], th_o[0], rtol=0, atol=1e-6)
+        else:
+            np.testing.assert_allclose(th, th_prev, rtol=0, atol=0)
+        th_prev = th
+        fp = opl.fit_problem(X[:nt], Y[:nt], np.exp(th[:, :d]), np.exp(th[:, d]),
+                             np.exp(th[:, d + 1]), ref)
+        mean, var = opl.posterior(fp, cand)
+        acq = opl.acquisition(fp, mean, var, mode, eps)
+        best = acq.max()
+        assert acq[pick] >= best - 1e-3 * max(abs(best), 1e-6), (t, acq[pick], best)
+    # stopping rule
+    sets = [_pareto_set(Y[:k]) for k in range(n0, n + 1)]
+    stable = 0
+    for k in range(1, len(sets)):
+        stable = stable + 1 if sets[k] == sets[k - 1] else 0
+        if k < len(sets) - 1:
+            assert stable < patience  # it would have stopped here
+    assert res["converged"] == (stable >= patience)
+    if not res["converged"]:
+        assert n == max_evals
+
+
+@pytest.mark.parametrize("learn", [None, (15, 0.05)], ids=["fixed", "learned"])
+def test_loop_choices_match_oracle(learn):
+    from paper_2602_10729_gb300 import boute as bt
+    rng = np.random.default_rng(7)
+    d, N, n0 = 4, 1536, 6
+    cand = rng.random((N, d)).astype(np.float32)
+    X0 = cand[:n0].astype(np.float64)
+    Y0 = np.stack([_objective(x) for x in X0])
+    ls0 = np.full((2, d), 0.4)
+    s2, noise = np.ones(2), np.full(2, 1e-4)
+    mode = "mc" if learn else "ehvi"
+    S = 128
+    eps = rng.standard_normal((N, 2, S), dtype=np.float32) if mode == "mc" else None
+    max_evals, patience = 24, 4
+    res = bt.boute_mobo_run(_objective, cand, [1.1, 1.1], ls0, s2, noise, X0, Y0,
+                            mode=bt.BOUTE_ACQ_MC_HVI if mode == "mc" else bt.BOUTE_ACQ_EHVI2D,
+                            S=S if mode == "mc" else 0, eps=eps, max_evals=max_evals,
+                            patience=patience, learn_iters=learn[0] if learn else 0,
+                            learn_lr=learn[1] if learn else 0.05)
+    assert len(res["sel"]) >= patience  # converged (stable that long) or ran out of budget
+    _check_run(res, cand, n0, patience, max_evals, mode, eps, ls0, s2, noise, learn)
+    # the loop improves the observed front: its hypervolume never falls
+    hv = [oracle.hv(Y[list(_pareto_set(Y))], np.array([1.0, 1.0]))
+          for Y in (res["Y"][:k] for k in range(n0, len(res["Y"]) + 1))]
+    assert all(b >= a - 1e-12 for a, b in zip(hv, hv[1:]))
+
+
+def test_objective_errors_stop_the_loop():
+    from paper_2602_10729_gb300 import boute as bt
+    rng = np.random.default_rng(8)
+    cand = rng.random((256, 3)).astype(np.float32)
+    X0 = cand[:4].astype(np.float64)
+    Y0 = np.stack([_objective(x) for x in X0])
+
+    def bad(x):
+        raise ValueError("evaluation failed")
+
+    with pytest.raises(ValueError):
+        bt.boute_mobo_run(bad, cand, [1.1, 1.1], np.full((2, 3), 0.4), np.ones(2),
+                          np.full(2, 1e-4), X0, Y0, max_evals=8, patience=3)
