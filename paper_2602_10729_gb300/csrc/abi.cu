@@ -121,6 +121,10 @@ struct boute_engine {
   // allocated on first use; used while has_cons
   double *cons;
   int has_cons;
+  // outcome transforms (boute_engine_set_outcome_transforms): the step first
+  // writes the transformed outcomes to Yt, which the fit and the front read
+  int tcodes;
+  double *Yt;
 };
 
 // Stage order of one step as timed (with timing on, the front stage runs
@@ -350,7 +354,7 @@ void boute_engine_free(boute_engine *e) {
   void *ptrs[] = {e->X, e->Y, e->Ys, e->ls, e->s2, e->noise, e->ref, e->front, e->mask, e->P,
                   e->K, e->lower, e->upper, e->Xc, e->eps, e->mean, e->var, e->acq, e->val,
                   e->idx, e->scratch, e->sel, e->kst, e->X1, e->Y1, e->ls1, e->s21,
-                  e->noise1, e->ref1, e->Xc1, e->eps1, e->cons};
+                  e->noise1, e->ref1, e->Xc1, e->eps1, e->cons, e->Yt};
   for (void *p : ptrs) cudaFree(p);
   delete e;
 }
@@ -470,8 +474,8 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
       cudaEventRecord(e->ev[stage], s);
   };
   auto front = [&](cudaStream_t fs) {
-    return launch_front_fused(Y, B, n, m, e->gp->g.tcodes, ref, e->Ys, e->mask, e->front, e->P,
-                              e->lower, e->upper, e->K, mc, fs);
+    return launch_front_fused(Y, B, n, m, ref, e->Ys, e->mask, e->front, e->P, e->lower,
+                              e->upper, e->K, mc, fs);
   };
   mark(ST_FIT);
   // waits on the host-input copies: an external-event node when captured
@@ -484,6 +488,12 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
   const cudaEvent_t *ev_eps = host == 2 ? e->ev_eps1 : e->ev_eps;
   if (host && cudaStreamWaitEvent(s, e->ev_small[host - 1], wait_flags) != cudaSuccess)
     return last_launch_status();
+  // outcome transforms: one elementwise pass first (the kernels after it see
+  // transformed outcomes; without transforms the step does not have it)
+  if (e->tcodes) {
+    if ((r = launch_outcome_transform(Y, (long long)B * n * m, m, e->tcodes, e->Yt, s))) return r;
+    Y = e->Yt;
+  }
   // K* beside the fit (not in stage-timing mode, where the posterior builds it)
   const float *kst = e->timing ? nullptr : e->kst;
   // The graph has one root, the fit's set-up: the front stage (which needs
@@ -778,9 +788,11 @@ int boute_engine_set_kernel(boute_engine *e, int d_tau, const double *params) {
 int boute_engine_set_outcome_transforms(boute_engine *e, const int *codes) {
   int packed = 0;
   if (!e || !pack_codes(codes, e->m, &packed)) return BOUTE_ERR_INVALID_ARG;
-  if (packed != e->gp->g.tcodes) {
+  if (packed != e->tcodes) {
     if (cudaDeviceSynchronize() != cudaSuccess) return last_launch_status();
-    e->gp->g.tcodes = packed;
+    if (packed && !e->Yt && dalloc(&e->Yt, (size_t)e->B * e->n * e->m) != BOUTE_OK)
+      return BOUTE_ERR_OOM;
+    e->tcodes = packed;
     engine_drop_graphs(e);
   }
   return BOUTE_OK;

@@ -41,11 +41,16 @@ inline __host__ __device__ int round_up(int x, int r) { return (x + r - 1) / r *
 // objectives' codes are packed 3 bits apiece, objective t at bit 3t.
 inline __host__ __device__ int objective_code(int codes, int t) { return (codes >> (3 * t)) & 7; }
 #ifdef __CUDACC__
-__device__ __forceinline__ double outcome_transform(double y, int code) {
+// (out of line: the transforms' fp64 logarithm stays out of the kernels'
+// register allocation; the identity costs a test)
+static __device__ __noinline__ double outcome_transform_call(double y, int code) {
   double v = y;
   if ((code & 3) == 1) v = log(y);
   else if ((code & 3) == 2) v = log(y / (1.0 - y));
   return (code & 4) ? -v : v;
+}
+__device__ __forceinline__ double outcome_transform(double y, int code) {
+  return code ? outcome_transform_call(y, code) : y;
 }
 #endif
 

@@ -84,6 +84,9 @@ __host__ __device__ inline int kmat_units(int n) {
   const int tn = (n + 15) / 16;
   return tn * (tn + 1);  // tiles on or below the diagonal, two halves each
 }
+// COMP: the composite kernel (kp its parameters); the Matern-5/2
+// instantiation carries none of its code.
+template <bool COMP>
 __device__ void kmat_tile(const double *X, int n, int d, int b, const double *l, double s2,
                           double noise, int unit, float *Kh, float *Kl, double *il,
                           const double *kp, int dtau) {
@@ -98,18 +101,20 @@ __device__ void kmat_tile(const double *X, int n, int d, int b, const double *l,
   if (i >= n || j >= n) return;
   const double *xi = X + ((size_t)b * n + i) * d, *xj = X + ((size_t)b * n + j) * d;
   double r2 = 0.0, r2c = 0.0;
-  const int dt = kp ? dtau : d;
+  const int dt = COMP ? dtau : d;
   for (int t = 0; t < dt; ++t) {
     const double z = (xi[t] - xj[t]) * il[t];
     r2 = fma(z, z, r2);
   }
-  for (int t = dt; t < d; ++t) {
-    const double z = (xi[t] - xj[t]) * il[t];
-    r2c = fma(z, z, r2c);
+  if (COMP) {
+    for (int t = dt; t < d; ++t) {
+      const double z = (xi[t] - xj[t]) * il[t];
+      r2c = fma(z, z, r2c);
+    }
   }
   const double r = sqrt(r2), sr = sqrt(5.0) * r;
   double k;
-  if (!kp) {
+  if (!COMP) {
     k = s2 * (1.0 + sr + 5.0 * r2 / 3.0) * exp(-sr);
   } else {
     const double k52 = (1.0 + sr + 5.0 * r2 / 3.0) * exp(-sr);
@@ -131,6 +136,7 @@ __device__ void kmat_tile(const double *X, int n, int d, int b, const double *l,
   }
 }
 
+template <bool COMP>
 __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad,
                           const double *l, double s2, float *x, int blk, int nblk,
                           const double *kp, int dtau) {
@@ -143,9 +149,9 @@ __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad
     const int c = j / BOUTE_KCHUNK, jj = j % BOUTE_KCHUNK;
     float *q = x + (size_t)c * cf;  // dimension-major: [DP][32] hi, [DP][32] lo
     q[t * BOUTE_KCHUNK + jj] = hi;
-    if (!kp) q[BOUTE_KCHUNK * DP + t * BOUTE_KCHUNK + jj] = lo;
+    if (!COMP) q[BOUTE_KCHUNK * DP + t * BOUTE_KCHUNK + jj] = lo;
   }
-  if (kp) {  // composite kernel: w_j (row 0 of the lo block), beta s_k (row 1)
+  if (COMP) {  // composite kernel: w_j (row 0 of the lo block), beta s_k (row 1)
     for (int e = blk * blockDim.x + threadIdx.x; e < npad; e += nblk * blockDim.x) {
       double ej = 0.0;
       if (e < n)
@@ -172,13 +178,14 @@ __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad
         v = (float)(iv - (double)(float)iv);
       }
     } else if (k == 2 * DP) v = (float)s2;
-    else if (kp && k == 2 * DP + 1) v = (float)kp[0];
-    else if (kp && k == 2 * DP + 2) v = (float)kp[1];
-    else if (kp && k == 2 * DP + 3) v = (float)dtau;
+    else if (COMP && k == 2 * DP + 1) v = (float)kp[0];
+    else if (COMP && k == 2 * DP + 2) v = (float)kp[1];
+    else if (COMP && k == 2 * DP + 3) v = (float)dtau;
     x[(size_t)c * cf + po + k] = v;
   }
 }
 
+template <bool COMP>
 __global__ void __launch_bounds__(kSetupThreads) fit_setup_kernel(
     const double *X, int n, int d, int m, int DP, int npad, const double *ls, const double *s2,
     const double *noise, float *Kh_all, float *Kl_all, float *xt, float *s2f, int nkt, int nprep,
@@ -187,17 +194,17 @@ __global__ void __launch_bounds__(kSetupThreads) fit_setup_kernel(
   const int bt = blockIdx.y, b = bt / m;
   if (early_trigger) pdl_trigger();  // the whole grid is resident: the fit may launch now
   const double *l = ls + (size_t)bt * d;
-  const double *kp = kpar ? kpar + (size_t)bt * (3 + d) : nullptr;
+  const double *kp = COMP ? kpar + (size_t)bt * (3 + d) : nullptr;
   if (blockIdx.x == 0 && bt == 0 && threadIdx.x == 0) *status = BOUTE_OK;
   if ((int)blockIdx.x < nkt) {
-    kmat_tile(X, n, d, b, l, s2[bt], noise[bt], blockIdx.x, Kh_all + (size_t)bt * n * n,
-              Kl_all + (size_t)bt * n * n, il, kp, dtau);
+    kmat_tile<COMP>(X, n, d, b, l, s2[bt], noise[bt], blockIdx.x, Kh_all + (size_t)bt * n * n,
+                    Kl_all + (size_t)bt * n * n, il, kp, dtau);
   } else {
     float *x = xt + (size_t)bt * (npad / BOUTE_KCHUNK) * xt_chunk_floats(DP);
-    prep_part(X, n, d, b, DP, npad, l, s2[bt], x, blockIdx.x - nkt, nprep, kp, dtau);
+    prep_part<COMP>(X, n, d, b, DP, npad, l, s2[bt], x, blockIdx.x - nkt, nprep, kp, dtau);
     // the prior variance's constant part (composite: s2 + s2_x; the
     // posterior adds s2_c w(x)^2)
-    if (blockIdx.x == nkt && threadIdx.x == 0) s2f[bt] = (float)(s2[bt] + (kp ? kp[1] : 0.0));
+    if (blockIdx.x == nkt && threadIdx.x == 0) s2f[bt] = (float)(COMP ? s2[bt] + kp[1] : s2[bt]);
   }
 }
 
@@ -254,9 +261,9 @@ constexpr int fit_threads() { return SMEM ? 384 : 256; }
 
 template <bool SMEM>
 __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
-    const float *Kh_all, const float *Kl_all, const double *Ys, int standardize, int tcodes,
-    int n, int m, float *Aws, float *Wws, float *xt, int DP, int npad, PostPlan plan, float *bop,
-    int kl_smem, int early_trigger, int *status) {
+    const float *Kh_all, const float *Kl_all, const double *Ys, int standardize, int n, int m,
+    float *Aws, float *Wws, float *xt, int DP, int npad, PostPlan plan, float *bop, int kl_smem,
+    int early_trigger, int *status) {
   extern __shared__ __align__(16) float sm[];
   __shared__ int bad;
   __shared__ uint64_t lbar, lbar_lo;  // K hi; K lo (needed only by the residual)
@@ -275,18 +282,16 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
         *rv = vec + 5 * NP;
   const double *y = Ys + (size_t)b * n * m + t;
   if (early_trigger) pdl_trigger();  // every block is resident: the posterior may launch
-  // standardize != 0: Ys holds raw outcomes; this column is transformed
-  // (tcodes) and standardised here (zero mean, unit sample standard deviation,
-  // as standardize_kernel does)
-  const int tcode = standardize ? objective_code(tcodes, t) : 0;
+  // standardize != 0: Ys holds raw outcomes; this column is standardised here
+  // (zero mean, unit sample standard deviation, as standardize_kernel does)
   if (standardize) {  // warp 0 alone: few fp64 instructions
     if (warp == 0) {
       double sum = 0.0;
-      for (int i = lane; i < n; i += 32) sum += outcome_transform(y[(size_t)i * m], tcode);
+      for (int i = lane; i < n; i += 32) sum += y[(size_t)i * m];
       const double mean = warp_sum(sum) / n;
       double ss = 0.0;
       for (int i = lane; i < n; i += 32) {
-        const double z = outcome_transform(y[(size_t)i * m], tcode) - mean;
+        const double z = y[(size_t)i * m] - mean;
         ss += z * z;
       }
       ss = warp_sum(ss);
@@ -366,7 +371,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     __syncthreads();
   }
   for (int i = tid; i < NP; i += nthr) {  // standardised y as an fp32 pair
-    const double ys = i < n ? (outcome_transform(y[(size_t)i * m], tcode) - mu_y) * isd_y : 0.0;
+    const double ys = i < n ? (y[(size_t)i * m] - mu_y) * isd_y : 0.0;
     yv[i] = (float)ys;
     ylo[i] = (float)(ys - (double)yv[i]);
     dg[i] = A[(size_t)i * ld + i];
@@ -732,6 +737,22 @@ __global__ void pack_kernel(const float *Wws, PostPlan plan, float *bop, const i
 
 }  // namespace
 
+// Outcome transforms alone (codes != 0), elementwise: Yt = t(Y), count
+// values of m objectives.
+__global__ void transform_kernel(const double *Y, long long count, int m, int codes, double *Yt) {
+  for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < count;
+       e += (long long)gridDim.x * blockDim.x)
+    Yt[e] = outcome_transform(Y[e], objective_code(codes, (int)(e % m)));
+}
+
+int launch_outcome_transform(const double *Y, long long count, int m, int codes, double *Yt,
+                             cudaStream_t s) {
+  const int blocks = (int)std::min<long long>((count + 255) / 256, 1024);
+  transform_kernel<<<std::max(blocks, 1), 256, 0, s>>>(Y, count, m, codes, Yt);
+  count_launch();
+  return last_launch_status();
+}
+
 int launch_standardize(const double *Y, int B, int n, int m, int codes, double *Ys,
                        cudaStream_t s) {
   standardize_kernel<<<B * m, 256, 0, s>>>(Y, n, m, codes, Ys);
@@ -760,17 +781,21 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
   const int sms = num_sms();
   // side-input blocks: as many as leave one block per SM (K blocks first), 2 .. 16
   const int nprep = std::max(2, std::min(16, sms / BM - nkt));
-  prefer_shared(fit_setup_kernel);
   // early triggers only when every block of the grid is resident at once (8
   // set-up blocks per SM beside the fit's blocks; one fit block per SM), so
   // that waiting successors can never hold resources a later block needs
   const long long setup_blocks = (long long)(nkt + nprep) * BM;
   const int setup_early = setup_blocks <= 8LL * (sms - BM) ? 1 : 0;
   const int fit_early = 2 * BM <= sms ? 1 : 0;
-  fit_setup_kernel<<<dim3(nkt + nprep, BM), kSetupThreads, 0, s>>>(X, n, d, m, gp->DP, npad, ls, s2, noise,
+  auto setup = [&](auto kern) {
+    prefer_shared(kern);
+    kern<<<dim3(nkt + nprep, BM), kSetupThreads, 0, s>>>(X, n, d, m, gp->DP, npad, ls, s2, noise,
                                                          gp->Kh, gp->Kl, gp->xt, gp->s2f, nkt,
                                                          nprep, setup_early, gp->status,
-                                                         gp->kern ? gp->kpar : nullptr, gp->dtau);
+                                                         gp->kpar, gp->dtau);
+  };
+  if (gp->kern) setup(fit_setup_kernel<true>);
+  else setup(fit_setup_kernel<false>);
   if (setup_done && cudaEventRecord(setup_done, s) != cudaSuccess) return last_launch_status();
   if (fit_uses_smem(npad)) {
     const size_t smem = fit_smem_bytes(npad, n);
@@ -778,13 +803,13 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
     cudaFuncSetAttribute(fit32_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);
     launch_pdl(fit32_kernel<true>, dim3(BM), dim3(fit_threads<true>()), smem, s, gp->Kh, gp->Kl,
-               Ys, standardize, gp->tcodes, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad,
-               gp->plan, gp->bop, fit_kl_in_smem(n) ? 1 : 0, fit_early, gp->status);
+               Ys, standardize, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop,
+               fit_kl_in_smem(n) ? 1 : 0, fit_early, gp->status);
     count_launch(2);
   } else {
     launch_pdl(fit32_kernel<false>, dim3(BM), dim3(fit_threads<false>()),
-               6 * npad * sizeof(float), s, gp->Kh, gp->Kl, Ys, standardize, gp->tcodes, n, m,
-               gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop, 0, 0, gp->status);
+               6 * npad * sizeof(float), s, gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws,
+               gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop, 0, 0, gp->status);
     const long long tot = (long long)gp->plan.ncols * npad;
     pack_kernel<<<dim3((unsigned)std::min<long long>((tot + 255) / 256, 4096), BM), 256, 0, s>>>(
         gp->Wws, gp->plan, gp->bop, gp->status);

@@ -214,23 +214,21 @@ __device__ double block_sum_d(double v, double *red) {
 // The engine's front stage, one block per problem: standardise the m outcome
 // columns, take the Pareto front, decompose the improving region into boxes.
 // It depends on the raw outcomes only, so it runs beside the GP fit.
-__global__ void front_fused_kernel(const double *Y, int n, int m, int codes, const double *ref,
-                                   double *Ys, unsigned char *mask, double *front, int *P,
-                                   float *lower, float *upper, int *Kout, int want_boxes) {
+__global__ void front_fused_kernel(const double *Y, int n, int m, const double *ref, double *Ys,
+                                   unsigned char *mask, double *front, int *P, float *lower,
+                                   float *upper, int *Kout, int want_boxes) {
   extern __shared__ long long smem_front[];
   __shared__ double red[32];
   const int b = blockIdx.x, cap = 2 * n + 2;
   const double *Yb = Y + (size_t)b * n * m;
   double *Ysb = Ys + (size_t)b * n * m;
   for (int t = 0; t < m; ++t) {
-    const int code = objective_code(codes, t);
     double s = 0.0;
-    for (int i = threadIdx.x; i < n; i += blockDim.x)
-      s += outcome_transform(Yb[(size_t)i * m + t], code);
+    for (int i = threadIdx.x; i < n; i += blockDim.x) s += Yb[(size_t)i * m + t];
     const double mean = block_sum_d(s, red) / n;
     double ss = 0.0;
     for (int i = threadIdx.x; i < n; i += blockDim.x) {
-      const double z = outcome_transform(Yb[(size_t)i * m + t], code) - mean;
+      const double z = Yb[(size_t)i * m + t] - mean;
       ss += z * z;
     }
     ss = block_sum_d(ss, red);
@@ -238,7 +236,7 @@ __global__ void front_fused_kernel(const double *Y, int n, int m, int codes, con
     if (!(sd >= 1e-8)) sd = 1.0;
     const double isd = 1.0 / sd;
     for (int i = threadIdx.x; i < n; i += blockDim.x)
-      Ysb[(size_t)i * m + t] = (outcome_transform(Yb[(size_t)i * m + t], code) - mean) * isd;
+      Ysb[(size_t)i * m + t] = (Yb[(size_t)i * m + t] - mean) * isd;
   }
   __syncthreads();
   __shared__ int Pb;
@@ -280,16 +278,16 @@ size_t front_smem_bytes(int n, int m) {
   return pk > bx ? pk : bx;
 }
 
-int launch_front_fused(const double *Y, int B, int n, int m, int codes, const double *ref,
-                       double *Ys, unsigned char *mask, double *front, int *P, float *lower,
-                       float *upper, int *K, int want_boxes, cudaStream_t s) {
+int launch_front_fused(const double *Y, int B, int n, int m, const double *ref, double *Ys,
+                       unsigned char *mask, double *front, int *P, float *lower, float *upper,
+                       int *K, int want_boxes, cudaStream_t s) {
   const size_t smem = front_smem_bytes(n, m);
   prefer_shared(front_fused_kernel);
   if (smem > 48 * 1024)
     cudaFuncSetAttribute(front_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);
-  front_fused_kernel<<<B, 512, smem, s>>>(Y, n, m, codes, ref, Ys, mask, front, P, lower, upper,
-                                          K, want_boxes);
+  front_fused_kernel<<<B, 512, smem, s>>>(Y, n, m, ref, Ys, mask, front, P, lower, upper, K,
+                                          want_boxes);
   count_launch();
   return last_launch_status();
 }

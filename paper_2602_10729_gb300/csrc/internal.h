@@ -18,7 +18,6 @@ struct Gp {
   float *xt;      // B*m x nchunk x xt_chunk_floats(DP): X/lengthscale hi/lo, alpha
   float *s2f;     // B*m: outputscale
   int *status;    // device status word (first error wins)
-  int tcodes;     // outcome transforms of a fit from raw outcomes (objective_code)
   // the composite kernel (kern = 1): routing features [0, dtau) and per
   // problem-objective [s2_c, s2_x, beta, s_0 .. s_{d-1}] (B*m x (3 + d))
   int kern, dtau;
@@ -79,9 +78,12 @@ int launch_kstar(const Gp *gp, const float *Xc, long long N, float *kst, cudaStr
 int launch_pareto(const double *Ys, int B, int n, int m, const double *ref, unsigned char *mask,
                   double *front, int *P, cudaStream_t s);
 size_t front_smem_bytes(int n, int m);
-int launch_front_fused(const double *Y, int B, int n, int m, int codes, const double *ref,
-                       double *Ys, unsigned char *mask, double *front, int *P, float *lower,
-                       float *upper, int *K, int want_boxes, cudaStream_t s);
+int launch_front_fused(const double *Y, int B, int n, int m, const double *ref, double *Ys,
+                       unsigned char *mask, double *front, int *P, float *lower, float *upper,
+                       int *K, int want_boxes, cudaStream_t s);
+// Yt = outcome transforms (objective_code) of Y, count values, m objectives
+int launch_outcome_transform(const double *Y, long long count, int m, int codes, double *Yt,
+                             cudaStream_t s);
 // setup_done (optional) is recorded on s after the set-up kernel, before the fit.
 int launch_fit_raw(Gp *gp, const double *X, const double *Y, const double *ls, const double *s2,
                    const double *noise, cudaStream_t s,
