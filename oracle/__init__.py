@@ -73,6 +73,11 @@ def lib():
         L.bo_gp_mll.restype = ctypes.c_double
         L.bo_gp_learn.argtypes = [_dp, _dp, ctypes.c_int, ctypes.c_int, _dp, ctypes.c_int,
                                   ctypes.c_int, ctypes.c_double, _dp, _dp, _dp]
+        L.bo_gp_mll_k.argtypes = [_dp, _dp, ctypes.c_int, ctypes.c_int, _dp, ctypes.c_double,
+                                  ctypes.c_double, ctypes.c_int, _dp, _dp]
+        L.bo_gp_mll_k.restype = ctypes.c_double
+        L.bo_gp_learn_k.argtypes = [_dp, _dp, ctypes.c_int, ctypes.c_int, ctypes.c_int, _dp, _dp,
+                                    ctypes.c_int, ctypes.c_int, ctypes.c_double, _dp, _dp, _dp]
         L.bo_pareto_front.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp, _bp, _ip]
         L.bo_hv.argtypes = [_dp, ctypes.c_int, ctypes.c_int, _dp, _dp]
         L.bo_hv.restype = ctypes.c_double
@@ -216,16 +221,24 @@ def gp_posterior(X, ls, s2, L, alpha, Xc, threads: int = 0, kernel=None):
     return mean, var
 
 
-def gp_mll(X, y, ls, s2, noise, grad: bool = False):
-    """Log marginal likelihood of the Matern-5/2 GP (and its gradient with
-    respect to (log l, log s2, log noise) when grad)."""
+def gp_mll(X, y, ls, s2, noise, grad: bool = False, kernel=None):
+    """Log marginal likelihood of the GP (and its gradient when grad): the
+    Matern-5/2 kernel, gradient over (log l, log s2, log noise); or the
+    composite kernel kernel = (dtau, kc), gradient over (log l, log s2,
+    log noise, log s2_c, log s2_x, beta)."""
     X, pX = _d(X)
     y, py = _d(y)
     ls, pl = _d(ls)
     n, d = X.shape
-    g = np.empty(d + 2) if grad else None
-    v = lib().bo_gp_mll(pX, py, n, d, pl, float(s2), float(noise),
-                        None if g is None else g.ctypes.data_as(_dp))
+    if kernel is None:
+        g = np.empty(d + 2) if grad else None
+        v = lib().bo_gp_mll(pX, py, n, d, pl, float(s2), float(noise),
+                            None if g is None else g.ctypes.data_as(_dp))
+    else:
+        dtau, kc, pk = _kern(kernel)
+        g = np.empty(d + 5) if grad else None
+        v = lib().bo_gp_mll_k(pX, py, n, d, pl, float(s2), float(noise), dtau, pk,
+                              None if g is None else g.ctypes.data_as(_dp))
     return (v, g) if grad else v
 
 
@@ -235,9 +248,14 @@ LOG_S2_BOUNDS = (math.log(1e-3), math.log(1e3))
 LOG_NOISE_BOUNDS = (math.log(1e-4), math.log(10.0))
 
 
-def gp_learn(X, y, theta0, iters: int, lr: float, grad: bool = False):
+LOG_SC_BOUNDS = (math.log(1e-4), math.log(1e3))
+BETA_BOUNDS = (-3.0, 3.0)
+
+
+def gp_learn(X, y, theta0, iters: int, lr: float, grad: bool = False, kernel=None):
     """Adam ascent on the log marginal likelihood from R starting points
-    theta0 (R x (d + 2) log-parameters). Returns (theta, mll[, grad])."""
+    theta0 (R x (d + 2) log-parameters; with kernel = (dtau, pref), the
+    composite kernel, R x (d + 5)). Returns (theta, mll[, grad])."""
     X, pX = _d(X)
     y, py = _d(y)
     th0, pt = _d(np.atleast_2d(theta0))
@@ -246,8 +264,14 @@ def gp_learn(X, y, theta0, iters: int, lr: float, grad: bool = False):
     theta = np.empty_like(th0)
     mll = np.empty(R)
     g = np.empty_like(th0) if grad else None
-    rc = lib().bo_gp_learn(pX, py, n, d, pt, R, int(iters), float(lr), theta.ctypes.data_as(_dp),
-                           mll.ctypes.data_as(_dp), None if g is None else g.ctypes.data_as(_dp))
+    gp = None if g is None else g.ctypes.data_as(_dp)
+    if kernel is None:
+        rc = lib().bo_gp_learn(pX, py, n, d, pt, R, int(iters), float(lr),
+                               theta.ctypes.data_as(_dp), mll.ctypes.data_as(_dp), gp)
+    else:
+        pref, pp = _d(kernel[1])
+        rc = lib().bo_gp_learn_k(pX, py, n, d, int(kernel[0]), pp, pt, R, int(iters), float(lr),
+                                 theta.ctypes.data_as(_dp), mll.ctypes.data_as(_dp), gp)
     if rc:
         raise ValueError(rc)
     return (theta, mll, g) if grad else (theta, mll)

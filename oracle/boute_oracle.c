@@ -240,12 +240,90 @@ done:
   return mll;
 }
 
+/* The composite kernel's log marginal likelihood and its gradient with respect
+ * to theta = (log l_1..log l_d, log s2, log noise, log s2_c, log s2_x, beta).
+ * Per entry, with the routing distance r_t, the deployment distance r_c,
+ * e5 = exp(-sqrt5 r_t), e3 = exp(-sqrt3 r_c) and ww = w_i w_j:
+ *   dK/dlog l_q (routing)    = (5/3)(1 + sqrt5 r_t) e5 z_q^2 (s2 + s2_x k32)
+ *   dK/dlog l_q (deployment) = 3 e3 z_q^2 (s2_c ww + s2_x k52)
+ *   dK/dlog s2 = s2 k52, dK/dlog s2_c = s2_c ww k32, dK/dlog s2_x = s2_x k52 k32,
+ *   dK/dbeta = s2_c ww k32 (<s, c_i> + <s, c_j>), dK/dlog noise = noise I. */
+double bo_gp_mll_k(const double *X, const double *y, int n, int d, const double *ls, double s2,
+                   double noise, int dtau, const double *kc, double *grad) {
+  double *L = (double *)malloc(sizeof(double) * ((size_t)n * n * 2 + 3 * (size_t)n));
+  double *Ki = L + (size_t)n * n, *alpha = Ki + (size_t)n * n, *col = alpha + n, *pc = col + n;
+  double mll = NAN;
+  const int dc = d - dtau;
+  if (bo_gp_fit_k(X, y, n, d, ls, s2, noise, dtau, kc, L, alpha) != 0) goto done;
+  mll = -0.5 * (double)n * log(2.0 * M_PI);
+  for (int i = 0; i < n; ++i) mll += -0.5 * y[i] * alpha[i] - log(L[(long)i * n + i]);
+  if (grad) {
+    for (int j = 0; j < n; ++j) {
+      for (int i = 0; i < n; ++i) {
+        double s = i == j ? 1.0 : 0.0;
+        for (int k = 0; k < i; ++k) s -= L[(long)i * n + k] * col[k];
+        col[i] = s / L[(long)i * n + i];
+      }
+      for (int i = n - 1; i >= 0; --i) {
+        double s = col[i];
+        for (int k = i + 1; k < n; ++k) s -= L[(long)k * n + i] * col[k];
+        col[i] = s / L[(long)i * n + i];
+      }
+      for (int i = 0; i < n; ++i) Ki[(long)i * n + j] = col[i];
+    }
+    for (int i = 0; i < n; ++i) { /* <s, c_i> */
+      double e = 0.0;
+      for (int k = 0; k < dc; ++k) e += kc[3 + k] * X[(long)i * d + dtau + k];
+      pc[i] = e;
+    }
+    const double s2c = kc[0], s2x = kc[1], beta = kc[2];
+    for (int q = 0; q < d + 5; ++q) grad[q] = 0.0;
+    for (int i = 0; i < n; ++i)
+      for (int j = 0; j < n; ++j) {
+        const double Q = 0.5 * (alpha[i] * alpha[j] - Ki[(long)i * n + j]);
+        const double *xi = X + (long)i * d, *xj = X + (long)j * d;
+        double rt2 = 0.0, rc2 = 0.0;
+        for (int t = 0; t < d; ++t) {
+          double z = (xi[t] - xj[t]) / ls[t];
+          if (t < dtau) rt2 += z * z;
+          else rc2 += z * z;
+        }
+        const double rt = sqrt(rt2), rc = sqrt(rc2);
+        const double e5 = exp(-sqrt(5.0) * rt), e3 = exp(-sqrt(3.0) * rc);
+        const double k52 = (1.0 + sqrt(5.0) * rt + 5.0 * rt2 / 3.0) * e5;
+        const double k32 = (1.0 + sqrt(3.0) * rc) * e3;
+        const double ww = exp(beta * (pc[i] + pc[j]));
+        for (int t = 0; t < d; ++t) {
+          double z = (xi[t] - xj[t]) / ls[t];
+          if (t < dtau)
+            grad[t] += Q * (5.0 / 3.0) * (1.0 + sqrt(5.0) * rt) * e5 * z * z * (s2 + s2x * k32);
+          else
+            grad[t] += Q * 3.0 * e3 * z * z * (s2c * ww + s2x * k52);
+        }
+        grad[d] += Q * s2 * k52;
+        if (i == j) grad[d + 1] += Q * noise;
+        grad[d + 2] += Q * s2c * ww * k32;
+        grad[d + 3] += Q * s2x * k52 * k32;
+        grad[d + 4] += Q * s2c * ww * k32 * (pc[i] + pc[j]);
+      }
+  }
+done:
+  free(L);
+  return mll;
+}
+
 /* Log-parameter bounds of the learner (theta = log l_1..log l_d, log s2, log noise). */
 static double clampd(double v, double lo, double hi) { return v < lo ? lo : (v > hi ? hi : v); }
 static void learn_clamp(double *th, int d) {
   for (int t = 0; t < d; ++t) th[t] = clampd(th[t], BO_LOG_LS_MIN, BO_LOG_LS_MAX);
   th[d] = clampd(th[d], BO_LOG_S2_MIN, BO_LOG_S2_MAX);
   th[d + 1] = clampd(th[d + 1], BO_LOG_NOISE_MIN, BO_LOG_NOISE_MAX);
+}
+/* the composite kernel's extra parameters (log s2_c, log s2_x, beta) */
+static void learn_clamp_k(double *th, int d) {
+  th[d + 2] = clampd(th[d + 2], BO_LOG_SC_MIN, BO_LOG_SC_MAX);
+  th[d + 3] = clampd(th[d + 3], BO_LOG_SC_MIN, BO_LOG_SC_MAX);
+  th[d + 4] = clampd(th[d + 4], BO_BETA_MIN, BO_BETA_MAX);
 }
 
 static double mll_at(const double *X, const double *y, int n, int d, const double *th,
@@ -281,6 +359,53 @@ int bo_gp_learn(const double *X, const double *y, int n, int d, const double *th
       learn_clamp(th, d);
     }
     mll[r] = mll_at(X, y, n, d, th, grad ? grad + (size_t)r * P : NULL, ls);
+  }
+  free(buf);
+  return 0;
+}
+
+static double mll_at_k(const double *X, const double *y, int n, int d, int dtau,
+                       const double *pref, const double *th, double *grad, double *ls,
+                       double *kc) {
+  for (int t = 0; t < d; ++t) ls[t] = exp(th[t]);
+  kc[0] = exp(th[d + 2]);
+  kc[1] = exp(th[d + 3]);
+  kc[2] = th[d + 4];
+  for (int k = 0; k < d - dtau; ++k) kc[3 + k] = pref[k];
+  return bo_gp_mll_k(X, y, n, d, ls, exp(th[d]), exp(th[d + 1]), dtau, kc, grad);
+}
+
+int bo_gp_learn_k(const double *X, const double *y, int n, int d, int dtau, const double *pref,
+                  const double *theta0, int R, int iters, double lr, double *theta, double *mll,
+                  double *grad) {
+  if (n < 1 || d < 1 || dtau < 0 || dtau > d || R < 1 || iters < 0 || !X || !y || !pref ||
+      !theta0 || !theta || !mll)
+    return 1;
+  const int P = d + 5;
+  double *buf = (double *)malloc(sizeof(double) * (size_t)(3 * P + d + 3 + d));
+  double *g = buf, *m1 = g + P, *m2 = m1 + P, *ls = m2 + P, *kc = ls + d;
+  for (int r = 0; r < R; ++r) {
+    double *th = theta + (size_t)r * P;
+    memcpy(th, theta0 + (size_t)r * P, sizeof(double) * P);
+    learn_clamp(th, d);
+    learn_clamp_k(th, d);
+    for (int q = 0; q < P; ++q) m1[q] = m2[q] = 0.0;
+    double b1t = 1.0, b2t = 1.0;
+    for (int it = 0; it < iters; ++it) {
+      const double v = mll_at_k(X, y, n, d, dtau, pref, th, g, ls, kc);
+      if (v != v) break; /* not positive definite: keep the last theta */
+      b1t *= BO_ADAM_B1;
+      b2t *= BO_ADAM_B2;
+      for (int q = 0; q < P; ++q) {
+        m1[q] = BO_ADAM_B1 * m1[q] + (1.0 - BO_ADAM_B1) * g[q];
+        m2[q] = BO_ADAM_B2 * m2[q] + (1.0 - BO_ADAM_B2) * g[q] * g[q];
+        const double mh = m1[q] / (1.0 - b1t), vh = m2[q] / (1.0 - b2t);
+        th[q] += lr * mh / (sqrt(vh) + BO_ADAM_EPS);
+      }
+      learn_clamp(th, d);
+      learn_clamp_k(th, d);
+    }
+    mll[r] = mll_at_k(X, y, n, d, dtau, pref, th, grad ? grad + (size_t)r * P : NULL, ls, kc);
   }
   free(buf);
   return 0;

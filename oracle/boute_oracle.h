@@ -95,6 +95,10 @@ double bo_gp_mll(const double *X, const double *y, int n, int d, const double *l
 #define BO_LOG_S2_MAX (6.907755278982137)     /* log 1e3 */
 #define BO_LOG_NOISE_MIN (-9.210340371976182) /* log 1e-4 */
 #define BO_LOG_NOISE_MAX (2.302585092994046)  /* log 10 */
+#define BO_LOG_SC_MIN (-9.210340371976182)    /* log 1e-4: s2_c, s2_x */
+#define BO_LOG_SC_MAX (6.907755278982137)     /* log 1e3 */
+#define BO_BETA_MIN (-3.0)
+#define BO_BETA_MAX (3.0)
 #define BO_ADAM_B1 0.9
 #define BO_ADAM_B2 0.999
 #define BO_ADAM_EPS 1e-8
@@ -108,6 +112,16 @@ double bo_gp_mll(const double *X, const double *y, int n, int d, const double *l
  * being positive definite keeps its last theta (mll NaN). */
 int bo_gp_learn(const double *X, const double *y, int n, int d, const double *theta0, int R,
                 int iters, double lr, double *theta, double *mll, double *grad);
+
+/* The same two for the composite kernel (bo_kernel with kc): theta = (log
+ * l_1..log l_d, log s2, log noise, log s2_c, log s2_x, beta), d + 5 values;
+ * kc = [s2_c, s2_x, beta, pref...]; the extra bounds BO_LOG_SC_*, BO_BETA_*;
+ * pref (d - dtau preference entries) stays fixed. grad: d + 5 values. */
+double bo_gp_mll_k(const double *X, const double *y, int n, int d, const double *ls, double s2,
+                   double noise, int dtau, const double *kc, double *grad);
+int bo_gp_learn_k(const double *X, const double *y, int n, int d, int dtau, const double *pref,
+                  const double *theta0, int R, int iters, double lr, double *theta, double *mll,
+                  double *grad);
 
 /* Pareto front of observed outcomes (Sec. 5.2, Pareto-optimal set; all
  * objectives minimised): point i is kept iff no j dominates it (Y_j <= Y_i in

@@ -752,3 +752,57 @@ def test_learner_reaches_the_grid_search_optimum():
     assert mll.max() >= vals[best] - 1e-3
     r = int(np.argmax(mll))
     assert abs(th[r, 0] - grid[best][0]) < 0.25
+
+
+def _mll_library_k(X, y, th, dtau, pref):
+    """log N(y; 0, K) by scipy on the composite kernel's Gram matrix;
+    th = (log l_1..log l_d, log s2, log noise, log s2_c, log s2_x, beta)."""
+    import scipy.stats
+    d = X.shape[1]
+    kc = np.concatenate([[math.exp(th[d + 2]), math.exp(th[d + 3]), th[d + 4]], pref])
+    ls, s2, noise = np.exp(th[:d]), math.exp(th[d]), math.exp(th[d + 1])
+    K = np.array([[oracle.kernel(a, b, ls, s2, (dtau, kc)) for b in X] for a in X])
+    K += noise * np.eye(len(X))
+    return scipy.stats.multivariate_normal(np.zeros(len(X)), K).logpdf(y)
+
+
+def _composite_mll_problem(seed, n=22):
+    rng = np.random.default_rng(seed)
+    X = np.concatenate([rng.random((n, 2)), rng.integers(0, 5, (n, 2))], 1).astype(float)
+    y = oracle.standardize((np.sin(3 * X[:, :1]) + 0.2 * X[:, 2:3] - 0.1 * X[:, 3:4]
+                            + 0.05 * rng.normal(size=(n, 1))))[:, 0]
+    return X, y, 2, rng.random(2)
+
+
+def test_composite_mll_and_gradient_match_library():
+    X, y, dtau, pref = _composite_mll_problem(30)
+    th = np.array([-0.8, -0.3, 0.5, 0.9, 0.1, math.log(2e-3), math.log(0.4), math.log(0.05), 0.2])
+    d = X.shape[1]
+    kc = np.concatenate([[math.exp(th[d + 2]), math.exp(th[d + 3]), th[d + 4]], pref])
+    v, g = oracle.gp_mll(X, y, np.exp(th[:d]), math.exp(th[d]), math.exp(th[d + 1]), grad=True,
+                         kernel=(dtau, kc))
+    assert v == pytest.approx(_mll_library_k(X, y, th, dtau, pref), rel=1e-11, abs=1e-10)
+    h = 1e-5
+    for q in range(len(th)):
+        e = np.zeros_like(th); e[q] = h
+        fd = (_mll_library_k(X, y, th + e, dtau, pref)
+              - _mll_library_k(X, y, th - e, dtau, pref)) / (2 * h)
+        assert g[q] == pytest.approx(fd, rel=1e-6, abs=1e-6), q
+
+
+def test_composite_learner_first_step_and_bounds():
+    X, y, dtau, pref = _composite_mll_problem(31)
+    d = X.shape[1]
+    th0 = np.array([[-0.8, -0.3, 0.5, 0.9, 0.1, math.log(2e-3), math.log(0.4), math.log(0.05), 0.2],
+                    [0.0, 0.0, 0.0, 0.0, 0.0, -5.0, -20.0, 20.0, 9.0]])
+    kc = np.concatenate([[math.exp(th0[0, d + 2]), math.exp(th0[0, d + 3]), th0[0, d + 4]], pref])
+    _, g = oracle.gp_mll(X, y, np.exp(th0[0, :d]), math.exp(th0[0, d]), math.exp(th0[0, d + 1]),
+                         grad=True, kernel=(dtau, kc))
+    lr = 0.05
+    th1, _ = oracle.gp_learn(X, y, th0[:1], 1, lr, kernel=(dtau, pref))
+    np.testing.assert_allclose(th1[0], th0[0] + lr * g / (np.abs(g) + 1e-8), rtol=0, atol=1e-12)
+    th_c, _ = oracle.gp_learn(X, y, th0[1:], 0, lr, kernel=(dtau, pref))
+    np.testing.assert_allclose(th_c[0, d + 2:], [oracle.LOG_SC_BOUNDS[0], oracle.LOG_SC_BOUNDS[1],
+                                                 oracle.BETA_BOUNDS[1]])
+    th2, mll2 = oracle.gp_learn(X, y, th0[:1], 200, lr, kernel=(dtau, pref))
+    assert mll2[0] > _mll_library_k(X, y, th0[0], dtau, pref)
