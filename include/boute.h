@@ -136,12 +136,28 @@ int boute_gp_set_kernel(boute_gp *gp, int d_tau, const double *params);
 #define BOUTE_LOG_S2_MAX (6.907755278982137)     /* log 1e3 */
 #define BOUTE_LOG_NOISE_MIN (-9.210340371976182) /* log 1e-4 */
 #define BOUTE_LOG_NOISE_MAX (2.302585092994046)  /* log 10 */
+#define BOUTE_LOG_SC_MIN (-9.210340371976182)    /* log 1e-4: s2_c, s2_x */
+#define BOUTE_LOG_SC_MAX (6.907755278982137)     /* log 1e3 */
+#define BOUTE_BETA_MIN (-3.0)
+#define BOUTE_BETA_MAX (3.0)
 #define BOUTE_ADAM_B1 0.9
 #define BOUTE_ADAM_B2 0.999
 #define BOUTE_ADAM_EPS 1e-8
 int boute_gp_learn(const double *X, const double *Ys, int B, int n, int d, int m,
                    const double *theta0, int R, int iters, double lr, double *theta,
                    double *mll, double *grad, void *stream);
+/* The same for the composite kernel (boute_gp_set_kernel): theta = (log l_1
+ * .. log l_d, log s2, log noise, log s2_c, log s2_x, beta), d + 5 values per
+ * (b, t, r), the extra ones clamped to BOUTE_LOG_SC_* and BOUTE_BETA_*;
+ * pref: B x m x (d - d_tau) fp64 device preference entries (held fixed). The
+ * gradient adds
+ *   dK/dlog l_q = (5/3)(1 + sqrt5 r_t) e^(-sqrt5 r_t) z_q^2 (s2 + s2_x k32)  (routing)
+ *               = 3 e^(-sqrt3 r_c) z_q^2 (s2_c w_i w_j + s2_x k52)        (deployment),
+ *   dK/dlog s2_c = s2_c w_i w_j k32, dK/dlog s2_x = s2_x k52 k32,
+ *   dK/dbeta = s2_c w_i w_j k32 (<s, c_i> + <s, c_j>). */
+int boute_gp_learn_k(const double *X, const double *Ys, int B, int n, int d, int m, int d_tau,
+                     const double *pref, const double *theta0, int R, int iters, double lr,
+                     double *theta, double *mll, double *grad, void *stream);
 
 /* ---- posterior ---------------------------------------------------------------
  * Latent-function posterior of every objective at N candidates per problem

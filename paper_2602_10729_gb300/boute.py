@@ -30,7 +30,7 @@ SYMBOLS = (
     "boute_engine_scores", "boute_engine_set_timing",
     "boute_engine_stage_times", "boute_engine_launches_per_step", "boute_engine_set_constraints",
     "boute_engine_set_outcome_transforms", "boute_engine_set_kernel", "boute_gp_set_kernel",
-    "boute_gp_learn", "boute_mobo_run",
+    "boute_gp_learn", "boute_gp_learn_k", "boute_mobo_run",
     "boute_engine_free",
 )
 #: stage names of boute_engine_stage_times, in order
@@ -105,6 +105,8 @@ def load(path: str | None = None):
         "boute_gp_set_kernel": ([_vp, _i, _vp], _i),
         "boute_gp_learn": ([_vp, _vp, _i, _i, _i, _i, _vp, _i, _i, ctypes.c_double, _vp, _vp, _vp,
                             _vp], _i),
+        "boute_gp_learn_k": ([_vp, _vp, _i, _i, _i, _i, _i, _vp, _vp, _i, _i, ctypes.c_double, _vp,
+                              _vp, _vp, _vp], _i),
         "boute_mobo_run": ([ctypes.POINTER(MoboConfig), _i, _i, _vp, _ll, _vp, _vp, _vp, _vp, _vp,
                             _vp, _vp, _vp, _vp, _i, ObjectiveFn, _vp, _vp, _vp,
                             ctypes.POINTER(_i), ctypes.POINTER(_i)], _i),
@@ -272,6 +274,19 @@ def boute_mobo_run(objective, cand, ref, ls, s2, noise, X0, Y0, *, mode=BOUTE_AC
     n = n_out.value
     return dict(X=X[:n], Y=Y[:n], sel=sel[:n - n0], theta=theta[:n - n0], ls=ls, s2=s2,
                 noise=noise, converged=bool(conv.value))
+
+
+def boute_gp_learn_k(X, Ys, d_tau, pref, theta0, iters: int, lr: float, theta, mll, grad=None,
+                     stream=None):
+    """The composite kernel's learner: pref B x m x (d - d_tau); theta0 /
+    theta / grad B x m x R x (d + 5) (fp64 CUDA tensors)."""
+    f64 = torch.float64
+    B, n, d = X.shape
+    m = Ys.shape[2]
+    R = theta0.shape[2]
+    _check(load().boute_gp_learn_k(_p(X, f64), _p(Ys, f64), B, n, d, m, int(d_tau), _p(pref, f64),
+                                   _p(theta0, f64), R, int(iters), float(lr), _p(theta, f64),
+                                   _p(mll, f64), _p(grad, f64), _s(stream)), "boute_gp_learn_k")
 
 
 def _host_f64(a):

@@ -235,7 +235,19 @@ int boute_gp_learn(const double *X, const double *Ys, int B, int n, int d, int m
     return BOUTE_ERR_INVALID_ARG;
   if ((long long)B * m * R > (1ll << 30)) return BOUTE_ERR_INVALID_ARG;
   if (int r = device_ok()) return r;
-  return launch_learn(X, Ys, B, n, d, m, theta0, R, iters, lr, theta, mll, grad,
+  return launch_learn(X, Ys, B, n, d, m, theta0, R, iters, lr, theta, mll, grad, d, nullptr,
+                      (cudaStream_t)stream);
+}
+
+int boute_gp_learn_k(const double *X, const double *Ys, int B, int n, int d, int m, int d_tau,
+                     const double *pref, const double *theta0, int R, int iters, double lr,
+                     double *theta, double *mll, double *grad, void *stream) {
+  if (!X || !Ys || !pref || !theta0 || !theta || !mll || !shape_ok(B, n, d, m) || R < 1 ||
+      iters < 0 || !(lr >= 0.0) || d_tau < 0 || d_tau > d)
+    return BOUTE_ERR_INVALID_ARG;
+  if ((long long)B * m * R > (1ll << 30)) return BOUTE_ERR_INVALID_ARG;
+  if (int r = device_ok()) return r;
+  return launch_learn(X, Ys, B, n, d, m, theta0, R, iters, lr, theta, mll, grad, d_tau, pref,
                       (cudaStream_t)stream);
 }
 

@@ -107,9 +107,11 @@ int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
                  cudaStream_t s);
 // hyperparameter learning (learn.cu): B*m*R blocks, fp64; workspace from the
 // stream-ordered pool when a block's does not fit in shared memory
+// dtau, pref: the composite kernel's routing features and preference entries
+// (B x m x (d - dtau)); pref null: the Matern-5/2 kernel
 int launch_learn(const double *X, const double *Ys, int B, int n, int d, int m,
                  const double *theta0, int R, int iters, double lr, double *theta, double *mll,
-                 double *grad, cudaStream_t s);
+                 double *grad, int dtau, const double *pref, cudaStream_t s);
 size_t topk_scratch_bytes(int B, long long N, int k);
 // counters_zeroed: the scratch's per-problem counters are known to be zero
 // (an engine's scratch: zeroed at creation, and every call leaves them zero);

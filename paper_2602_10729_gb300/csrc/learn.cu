@@ -25,6 +25,7 @@ constexpr int kLearnThreads = 256;
 constexpr int kLearnWarps = kLearnThreads / 32;
 constexpr int kLearnRows = 8;  // rows of K^-1 formed per pass
 constexpr double kSqrt5d = 2.23606797749978969641;
+constexpr double kSqrt3d = 1.73205080756887729353;
 constexpr double kLog2Pi = 1.83787706640934548356;
 
 __device__ __forceinline__ double warp_sum_d(double v) {
@@ -46,41 +47,68 @@ __device__ __forceinline__ double clamp_d(double v, double lo, double hi) {
   return v < lo ? lo : (v > hi ? hi : v);
 }
 
+// theta_q clamped to its bound: q < d log l, d log s2, d + 1 log noise, then
+// (composite kernel) d + 2 log s2_c, d + 3 log s2_x, d + 4 beta
+__device__ __forceinline__ double clamp_param(int q, int d, double v) {
+  if (q < d) return clamp_d(v, BOUTE_LOG_LS_MIN, BOUTE_LOG_LS_MAX);
+  if (q == d) return clamp_d(v, BOUTE_LOG_S2_MIN, BOUTE_LOG_S2_MAX);
+  if (q == d + 1) return clamp_d(v, BOUTE_LOG_NOISE_MIN, BOUTE_LOG_NOISE_MAX);
+  if (q < d + 4) return clamp_d(v, BOUTE_LOG_SC_MIN, BOUTE_LOG_SC_MAX);
+  return clamp_d(v, BOUTE_BETA_MIN, BOUTE_BETA_MAX);
+}
+
 // Row stride of the n x n workspace: odd, so that a column's 64-bit entries
 // fall in different shared-memory banks.
 __host__ __device__ inline int learn_ld(int n) { return n | 1; }
 
 // Doubles of one block's workspace: A (n x ld), X (n x d), y, alpha, tmp,
-// 1 / L_jj (n each), tmp2 (kLearnRows rows of K^-1).
+// 1 / L_jj (n each), tmp2 (kLearnRows rows of K^-1), and for the composite
+// kernel <s, c_i> and w_i (n each).
 __host__ __device__ inline size_t learn_ws_doubles(int n, int d) {
-  return (size_t)n * learn_ld(n) + (size_t)n * d + 4 * (size_t)n + (size_t)kLearnRows * n;
+  return (size_t)n * learn_ld(n) + (size_t)n * d + 6 * (size_t)n + (size_t)kLearnRows * n;
 }
 
+constexpr int kMaxP = BOUTE_MAX_D + 5;  // parameters of the composite kernel
+
+// COMP: the composite kernel (routing features [0, dtau), preference entries
+// pref: B x m x (d - dtau)), theta extended by (log s2_c, log s2_x, beta):
+//   K = s2 k52(r_t) + s2_c w_i w_j k32(r_c) + s2_x k52 k32 + noise I,
+//   dK/dlog l_q = (5/3)(1 + sqrt5 r_t) e^(-sqrt5 r_t) z_q^2 (s2 + s2_x k32)  (routing)
+//               = 3 e^(-sqrt3 r_c) z_q^2 (s2_c w_i w_j + s2_x k52)        (deployment)
+//   dK/dlog s2_c = s2_c w_i w_j k32, dK/dlog s2_x = s2_x k52 k32,
+//   dK/dbeta = s2_c w_i w_j k32 (<s, c_i> + <s, c_j>).
+template <bool COMP>
 __global__ void __launch_bounds__(kLearnThreads) learn_kernel(
     const double *X, const double *Ys, int n, int d, int m, int R, const double *theta0,
     int iters, double lr, double *theta_out, double *mll_out, double *grad_out, double *ws,
-    int use_smem) {
+    int use_smem, int dtau, const double *pref) {
   extern __shared__ __align__(16) double lsm[];
-  __shared__ double th[BOUTE_MAX_D + 2], m1[BOUTE_MAX_D + 2], m2[BOUTE_MAX_D + 2];
-  __shared__ double il[BOUTE_MAX_D], red[kLearnWarps][BOUTE_MAX_D + 2];
+  __shared__ double th[kMaxP], m1[kMaxP], m2[kMaxP];
+  __shared__ double il[BOUTE_MAX_D], red[kLearnWarps][kMaxP];
   __shared__ double logdet, mll_s;
   __shared__ int bad;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int blk = blockIdx.x, r = blk % R, bt = blk / R, b = bt / m, t = bt % m;
-  const int P = d + 2, ld = learn_ld(n);
+  const int P = d + (COMP ? 5 : 2), ld = learn_ld(n), dc = d - dtau;
   double *A = use_smem ? lsm : ws + (size_t)blk * learn_ws_doubles(n, d);
   double *xs = A + (size_t)n * ld, *yv = xs + (size_t)n * d, *av = yv + n, *tmp = av + n, *dinv = tmp + n,
-         *tmp2 = dinv + n;
+         *tmp2 = dinv + n, *pc = tmp2 + (size_t)kLearnRows * n, *wv = pc + n;
   for (int e = tid; e < n * d; e += kLearnThreads) xs[e] = X[(size_t)b * n * d + e];
   for (int i = tid; i < n; i += kLearnThreads) yv[i] = Ys[((size_t)b * n + i) * m + t];
   const double *th0 = theta0 + (size_t)blk * P;
   if (tid < P) {
-    const double v = th0[tid];
-    th[tid] = tid < d ? clamp_d(v, BOUTE_LOG_LS_MIN, BOUTE_LOG_LS_MAX)
-              : tid == d ? clamp_d(v, BOUTE_LOG_S2_MIN, BOUTE_LOG_S2_MAX)
-                         : clamp_d(v, BOUTE_LOG_NOISE_MIN, BOUTE_LOG_NOISE_MAX);
+    th[tid] = clamp_param(tid, d, th0[tid]);
     m1[tid] = 0.0;
     m2[tid] = 0.0;
+  }
+  if (COMP) {  // <s, c_i> of the training points (s fixed)
+    __syncthreads();
+    const double *pb = pref + (size_t)bt * dc;
+    for (int i = tid; i < n; i += kLearnThreads) {
+      double e = 0.0;
+      for (int k = 0; k < dc; ++k) e = fma(pb[k], xs[(size_t)i * d + dtau + k], e);
+      pc[i] = e;
+    }
   }
   double b1t = 1.0, b2t = 1.0;
   __syncthreads();
@@ -91,12 +119,28 @@ __global__ void __launch_bounds__(kLearnThreads) learn_kernel(
     // ---- K (lower) and exp(-sqrt5 r) (upper) at theta
     if (tid < d) il[tid] = exp(-th[tid]);
     if (tid == 0) bad = 0;
+    if (COMP)
+      for (int i = tid; i < n; i += kLearnThreads) wv[i] = exp(th[d + 4] * pc[i]);
     __syncthreads();
     const double s2 = exp(th[d]), nz = exp(th[d + 1]);
+    const double s2c = COMP ? exp(th[d + 2]) : 0.0, s2x = COMP ? exp(th[d + 3]) : 0.0;
     const int npair = n * (n + 1) / 2;  // pairs i >= j, one thread each
     for (int e = tid; e < npair; e += kLearnThreads) {
       int i, j;
       tri_index(e, i, j);
+      if (COMP) {  // (the gradient recomputes the exponentials)
+        double rt2 = 0.0, rc2 = 0.0;
+        for (int q = 0; q < d; ++q) {
+          const double z = (xs[i * d + q] - xs[j * d + q]) * il[q];
+          if (q < dtau) rt2 = fma(z, z, rt2);
+          else rc2 = fma(z, z, rc2);
+        }
+        const double st = kSqrt5d * sqrt(rt2), sc = kSqrt3d * sqrt(rc2);
+        const double k52 = (1.0 + st + 5.0 * rt2 / 3.0) * exp(-st), k32 = (1.0 + sc) * exp(-sc);
+        A[(size_t)i * ld + j] =
+            s2 * k52 + s2c * wv[i] * wv[j] * k32 + s2x * k52 * k32 + (i == j ? nz : 0.0);
+        continue;
+      }
       double r2 = 0.0;
       for (int q = 0; q < d; ++q) {
         const double z = (xs[i * d + q] - xs[j * d + q]) * il[q];
@@ -208,7 +252,7 @@ __global__ void __launch_bounds__(kLearnThreads) learn_kernel(
     // ---- gradient: pairs i >= j (an off-diagonal pair stands for two
     // entries); per pair f = s2 (5/3) (1 + sqrt5 r) e^(-sqrt5 r) multiplies
     // (dx_q / l_q)^2 in the lengthscale terms
-    double g[BOUTE_MAX_D], gs2 = 0.0, gnz = 0.0;
+    double g[BOUTE_MAX_D], gs2 = 0.0, gnz = 0.0, gsc = 0.0, gsx = 0.0, gbe = 0.0;
 #pragma unroll
     for (int q = 0; q < BOUTE_MAX_D; ++q) g[q] = 0.0;
     for (int e = tid; e < npair; e += kLearnThreads) {
@@ -216,6 +260,34 @@ __global__ void __launch_bounds__(kLearnThreads) learn_kernel(
       tri_index(e, i, j);
       const double Q = (i == j ? 0.5 : 1.0) * (av[i] * av[j] - A[(size_t)i * ld + j]);
       const double *xi = xs + (size_t)i * d, *xj = xs + (size_t)j * d;
+      if (COMP) {
+        double rt2 = 0.0, rc2 = 0.0;
+        for (int q = 0; q < d; ++q) {
+          const double z = (xi[q] - xj[q]) * il[q];
+          if (q < dtau) rt2 = fma(z, z, rt2);
+          else rc2 = fma(z, z, rc2);
+        }
+        const double st = kSqrt5d * sqrt(rt2), sc = kSqrt3d * sqrt(rc2);
+        const double e5 = exp(-st), e3 = exp(-sc);
+        const double k52 = (1.0 + st + 5.0 * rt2 / 3.0) * e5, k32 = (1.0 + sc) * e3;
+        const double ww = wv[i] * wv[j];
+        const double ft = Q * (5.0 / 3.0) * (1.0 + st) * e5 * (s2 + s2x * k32);
+        const double fc = Q * 3.0 * e3 * (s2c * ww + s2x * k52);
+#pragma unroll
+        for (int q = 0; q < BOUTE_MAX_D; ++q) {
+          if (q < d) {
+            const double z = (xi[q] - xj[q]) * il[q];
+            g[q] = fma(q < dtau ? ft : fc, z * z, g[q]);
+          }
+        }
+        gs2 = fma(Q, s2 * k52, gs2);
+        if (i == j) gnz = fma(Q, nz, gnz);
+        const double tc = Q * s2c * ww * k32;
+        gsc += tc;
+        gsx = fma(Q, s2x * k52 * k32, gsx);
+        gbe = fma(tc, pc[i] + pc[j], gbe);
+        continue;
+      }
       double r2 = 0.0;
       for (int q = 0; q < d; ++q) {
         const double z = (xi[q] - xj[q]) * il[q];
@@ -248,6 +320,14 @@ __global__ void __launch_bounds__(kLearnThreads) learn_kernel(
         red[warp][d] = a;
         red[warp][d + 1] = c;
       }
+      if (COMP) {
+        const double u = warp_sum_d(gsc), v2 = warp_sum_d(gsx), w2 = warp_sum_d(gbe);
+        if (lane == 0) {
+          red[warp][d + 2] = u;
+          red[warp][d + 3] = v2;
+          red[warp][d + 4] = w2;
+        }
+      }
     }
     __syncthreads();
     if (tid < P) {
@@ -262,10 +342,7 @@ __global__ void __launch_bounds__(kLearnThreads) learn_kernel(
         m1[tid] = BOUTE_ADAM_B1 * m1[tid] + (1.0 - BOUTE_ADAM_B1) * v;
         m2[tid] = BOUTE_ADAM_B2 * m2[tid] + (1.0 - BOUTE_ADAM_B2) * v * v;
         const double mh = m1[tid] / (1.0 - b1t), vh = m2[tid] / (1.0 - b2t);
-        const double nt = th[tid] + lr * mh / (sqrt(vh) + BOUTE_ADAM_EPS);
-        th[tid] = tid < d ? clamp_d(nt, BOUTE_LOG_LS_MIN, BOUTE_LOG_LS_MAX)
-                  : tid == d ? clamp_d(nt, BOUTE_LOG_S2_MIN, BOUTE_LOG_S2_MAX)
-                             : clamp_d(nt, BOUTE_LOG_NOISE_MIN, BOUTE_LOG_NOISE_MAX);
+        th[tid] = clamp_param(tid, d, th[tid] + lr * mh / (sqrt(vh) + BOUTE_ADAM_EPS));
       }
     }
     __syncthreads();
@@ -280,26 +357,31 @@ __global__ void __launch_bounds__(kLearnThreads) learn_kernel(
 
 size_t learn_smem_limit() { return 200 * 1024; }
 
+// dtau, pref: the composite kernel (pref null: the Matern-5/2 kernel)
 int launch_learn(const double *X, const double *Ys, int B, int n, int d, int m,
                  const double *theta0, int R, int iters, double lr, double *theta, double *mll,
-                 double *grad, cudaStream_t s) {
+                 double *grad, int dtau, const double *pref, cudaStream_t s) {
   const size_t per = learn_ws_doubles(n, d) * sizeof(double);
   const int blocks = B * m * R;
   const bool smem = per <= learn_smem_limit();
   double *ws = nullptr;
-  if (!smem) {
-    if (cudaMallocAsync((void **)&ws, per * blocks, s) != cudaSuccess) {
-      cudaGetLastError();
-      return BOUTE_ERR_OOM;
-    }
-  } else {
-    prefer_shared(learn_kernel);
-    if (cudaFuncSetAttribute(learn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)per) != cudaSuccess)
-      return last_launch_status();
+  if (!smem && cudaMallocAsync((void **)&ws, per * blocks, s) != cudaSuccess) {
+    cudaGetLastError();
+    return BOUTE_ERR_OOM;
   }
-  learn_kernel<<<blocks, kLearnThreads, smem ? per : 0, s>>>(X, Ys, n, d, m, R, theta0, iters, lr,
-                                                             theta, mll, grad, ws, smem ? 1 : 0);
+  auto go = [&](auto kern) {
+    if (smem) {
+      prefer_shared(kern);
+      if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)per) !=
+          cudaSuccess)
+        return;
+    }
+    kern<<<blocks, kLearnThreads, smem ? per : 0, s>>>(X, Ys, n, d, m, R, theta0, iters, lr,
+                                                       theta, mll, grad, ws, smem ? 1 : 0, dtau,
+                                                       pref);
+  };
+  if (pref) go(learn_kernel<true>);
+  else go(learn_kernel<false>);
   count_launch();
   const int st = last_launch_status();
   if (ws) cudaFreeAsync(ws, s);

@@ -92,3 +92,54 @@ def test_invalid_arguments():
         bt.boute_gp_learn(X, Ys, th, -1, 0.1, th.clone(), mll)
     with pytest.raises(bt.BouteError):
         bt.boute_gp_learn(X, Ys, th, 5, float("nan"), th.clone(), mll)
+
+
+# ---- the composite kernel's learner ---------------------------------------------
+def _composite_problem(wi, n, R, seed=2):
+    w = wl.composite(wl.scaled(wl.WORKLOADS[wi], B=1, n=n))
+    X, Y = wl.training_set(w, 0)
+    Ys = oracle.standardize(oracle.outcome_transform(Y, list(w.transforms)))
+    dtau, kc = wl.kernel_params(w, 0)
+    ls, s2, nz = wl.hyperparameters(w, 0)
+    base = np.r_[np.log(ls[0]), np.log(s2[0]), np.log(1e-3), np.log(kc[0, 0]), np.log(kc[0, 1]),
+                 kc[0, 2]]
+    rng = np.random.default_rng(seed)
+    theta0 = base + rng.normal(0.0, 0.3, (1, w.m, R, w.d + 5))
+    pref = kc[None, :, 3:]  # B x m x (d - dtau)
+    return w, X[None], Ys[None], theta0, dtau, pref
+
+
+def _gpu_k(X, Ys, dtau, pref, theta0, iters, lr):
+    import torch
+
+    from paper_2602_10729_gb300 import boute as bt
+    t = lambda a: torch.as_tensor(np.ascontiguousarray(a), dtype=torch.float64, device="cuda")
+    th0 = t(theta0)
+    theta = torch.empty_like(th0)
+    grad = torch.empty_like(th0)
+    mll = torch.empty(theta0.shape[:3], dtype=torch.float64, device="cuda")
+    bt.boute_gp_learn_k(t(X), t(Ys), dtau, t(pref), th0, iters, lr, theta, mll, grad)
+    torch.cuda.synchronize()
+    return theta.cpu().numpy(), mll.cpu().numpy(), grad.cpu().numpy()
+
+
+@pytest.mark.parametrize("wi,n,R", [(1, 128, 2), (2, 200, 1)], ids=["n128", "n200-global"])
+def test_composite_likelihood_gradient_and_trajectory_match_oracle(wi, n, R):
+    w, X, Ys, theta0, dtau, pref = _composite_problem(wi, n, R)
+    d = w.d
+    theta, mll, grad = _gpu_k(X, Ys, dtau, pref, theta0, 0, 0.05)
+    for t in range(w.m):
+        for r in range(R):
+            th = theta0[0, t, r]
+            kc = np.concatenate([[np.exp(th[d + 2]), np.exp(th[d + 3]), th[d + 4]], pref[0, t]])
+            v, g = oracle.gp_mll(X[0], Ys[0][:, t], np.exp(th[:d]), np.exp(th[d]),
+                                 np.exp(th[d + 1]), grad=True, kernel=(dtau, kc))
+            assert mll[0, t, r] == pytest.approx(v, rel=1e-10, abs=1e-9)
+            np.testing.assert_allclose(grad[0, t, r], g, rtol=1e-7, atol=1e-9 * np.abs(g).max())
+    iters, lr = 12, 0.05
+    theta, mll, _ = _gpu_k(X, Ys, dtau, pref, theta0, iters, lr)
+    for t in range(w.m):
+        th_o, mll_o = oracle.gp_learn(X[0], Ys[0][:, t], theta0[0, t], iters, lr,
+                                      kernel=(dtau, pref[0, t]))
+        np.testing.assert_allclose(theta[0, t], th_o, rtol=0, atol=1e-7)
+        np.testing.assert_allclose(mll[0, t], mll_o, rtol=1e-9, atol=1e-8)
