@@ -362,12 +362,17 @@ void boute_engine_free(boute_engine *e);
  *      (mode BOUTE_ACQ_MC_HVI, reused every iteration), else NULL;
  *   ref: m reference point (standardised units); transforms: m codes or
  *      NULL; cons: m thresholds or NULL (the constrained acquisition);
+ *   d_tau, kc: the composite kernel (boute_gp_set_kernel's parameters of one
+ *      problem, HOST m x (3 + d - d_tau), updated in place when learning:
+ *      s2_c, s2_x and beta are learned, the preference entries held), or
+ *      kc = NULL for the Matern-5/2 kernel;
  *   ls (m x d), s2 (m), noise (m): HOST hyperparameters, updated in place
  *      when learning;
  *   X (max_evals x d), Y (max_evals x m): HOST, the first n0 rows given;
  *   sel (out, max_evals - n0): the candidate index chosen per iteration;
- *   theta_hist (out, optional, (max_evals - n0) x m x (d + 2)): the
- *      log-hyperparameters each iteration scored with;
+ *   theta_hist (out, optional, (max_evals - n0) x m x P): the parameters
+ *      each iteration scored with (P = d + 2, or d + 5 with the composite
+ *      kernel, as for boute_gp_learn / boute_gp_learn_k);
  *   n_out: observations at the end; converged: 1 if the stability test
  *      stopped the loop.
  * Synchronous; allocates its device buffers and one engine per iteration. */
@@ -382,9 +387,9 @@ typedef struct {
 } boute_mobo_config;
 int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const float *cand, long long N,
                    const float *eps, const double *ref, const int *transforms,
-                   const double *cons, double *ls, double *s2, double *noise, double *X,
-                   double *Y, int n0, boute_objective_fn f, void *user, long long *sel,
-                   double *theta_hist, int *n_out, int *converged);
+                   const double *cons, int d_tau, double *kc, double *ls, double *s2,
+                   double *noise, double *X, double *Y, int n0, boute_objective_fn f, void *user,
+                   long long *sel, double *theta_hist, int *n_out, int *converged);
 
 #ifdef __cplusplus
 }

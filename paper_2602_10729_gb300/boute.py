@@ -107,8 +107,8 @@ def load(path: str | None = None):
                             _vp], _i),
         "boute_gp_learn_k": ([_vp, _vp, _i, _i, _i, _i, _i, _vp, _vp, _i, _i, ctypes.c_double, _vp,
                               _vp, _vp, _vp], _i),
-        "boute_mobo_run": ([ctypes.POINTER(MoboConfig), _i, _i, _vp, _ll, _vp, _vp, _vp, _vp, _vp,
-                            _vp, _vp, _vp, _vp, _i, ObjectiveFn, _vp, _vp, _vp,
+        "boute_mobo_run": ([ctypes.POINTER(MoboConfig), _i, _i, _vp, _ll, _vp, _vp, _vp, _vp, _i,
+                            _vp, _vp, _vp, _vp, _vp, _vp, _i, ObjectiveFn, _vp, _vp, _vp,
                             ctypes.POINTER(_i), ctypes.POINTER(_i)], _i),
         "boute_engine_free": ([_vp], None),
     }
@@ -223,13 +223,13 @@ def boute_gp_learn(X, Ys, theta0, iters: int, lr: float, theta, mll, grad=None, 
 
 def boute_mobo_run(objective, cand, ref, ls, s2, noise, X0, Y0, *, mode=BOUTE_ACQ_EHVI2D, S=0,
                    eps=None, max_evals=50, patience=20, learn_iters=0, learn_lr=0.05,
-                   transforms=None, cons=None):
+                   transforms=None, cons=None, d_tau=0, kc=None):
     """The optimisation loop. objective(x: (d,) float64 array) -> m outcomes.
     cand: N x d; eps: N x m x S (mode MC); ls: m x d, s2, noise: m (initial
     hyperparameters); X0 / Y0: the first observations. Returns a dict with X,
     Y (the n observations), sel (the chosen candidate per iteration), theta
-    (the log-hyperparameters of each iteration), ls, s2, noise (final),
-    converged."""
+    (the log-hyperparameters of each iteration), ls, s2, noise, kc (final),
+    converged. d_tau, kc: the composite kernel (m x (3 + d - d_tau))."""
     import numpy as np
     cand = np.ascontiguousarray(cand, np.float32)
     N, d = cand.shape
@@ -244,7 +244,8 @@ def boute_mobo_run(objective, cand, ref, ls, s2, noise, X0, Y0, *, mode=BOUTE_AC
     noise = np.ascontiguousarray(noise, np.float64).copy()
     iters = max(max_evals - n0, 1)
     sel = np.zeros(iters, np.int64)
-    theta = np.zeros((iters, m, d + 2))
+    kc = None if kc is None else np.ascontiguousarray(kc, np.float64).copy()
+    theta = np.zeros((iters, m, d + (2 if kc is None else 5)))
     ref = np.ascontiguousarray(ref, np.float64)
     eps = None if eps is None else np.ascontiguousarray(eps, np.float32)
     tf = None if transforms is None else np.ascontiguousarray(transforms, np.int32)
@@ -266,14 +267,14 @@ def boute_mobo_run(objective, cand, ref, ls, s2, noise, X0, Y0, *, mode=BOUTE_AC
     n_out, conv = ctypes.c_int(0), ctypes.c_int(0)
     a = lambda v: None if v is None else v.ctypes.data
     rc = load().boute_mobo_run(ctypes.byref(cfg), d, m, a(cand), N, a(eps), a(ref), a(tf), a(cs),
-                               a(ls), a(s2), a(noise), a(X), a(Y), n0, fn, None, a(sel), a(theta),
-                               ctypes.byref(n_out), ctypes.byref(conv))
+                               int(d_tau), a(kc), a(ls), a(s2), a(noise), a(X), a(Y), n0, fn, None,
+                               a(sel), a(theta), ctypes.byref(n_out), ctypes.byref(conv))
     if errors:
         raise errors[0]
     _check(rc, "boute_mobo_run")
     n = n_out.value
     return dict(X=X[:n], Y=Y[:n], sel=sel[:n - n0], theta=theta[:n - n0], ls=ls, s2=s2,
-                noise=noise, converged=bool(conv.value))
+                noise=noise, kc=kc, converged=bool(conv.value))
 
 
 def boute_gp_learn_k(X, Ys, d_tau, pref, theta0, iters: int, lr: float, theta, mll, grad=None,

@@ -70,8 +70,8 @@ int copy_in(void *dst, const void *src, size_t bytes) {
 
 extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const float *cand,
                               long long N, const float *eps, const double *ref,
-                              const int *transforms, const double *cons, double *ls, double *s2,
-                              double *noise, double *X, double *Y, int n0,
+                              const int *transforms, const double *cons, int d_tau, double *kc,
+                              double *ls, double *s2, double *noise, double *X, double *Y, int n0,
                               boute_objective_fn f, void *user, long long *sel,
                               double *theta_hist, int *n_out, int *converged) {
   if (!cfg || !cand || !ref || !ls || !s2 || !noise || !X || !Y || !f || !sel || !n_out ||
@@ -79,11 +79,17 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
       cfg->patience < 1 || cfg->learn_iters < 0)
     return BOUTE_ERR_INVALID_ARG;
   if (cfg->mode == BOUTE_ACQ_MC_HVI && (!eps || cfg->S < 1)) return BOUTE_ERR_INVALID_ARG;
-  const int nmax = cfg->max_evals, P = d + 2, S = cfg->mode == BOUTE_ACQ_MC_HVI ? cfg->S : 0;
+  if (kc && (d_tau < 0 || d_tau > d)) return BOUTE_ERR_INVALID_ARG;
+  // the composite kernel (kc: m x (3 + dc) [s2_c, s2_x, beta, s...]) adds
+  // (log s2_c, log s2_x, beta) to the learned parameters
+  const int dc = d - d_tau, KC = 3 + dc;
+  const int nmax = cfg->max_evals, P = d + (kc ? 5 : 2),
+            S = cfg->mode == BOUTE_ACQ_MC_HVI ? cfg->S : 0;
   *n_out = n0;
   *converged = 0;
   double *dX = nullptr, *dY = nullptr, *dYs = nullptr, *dls = nullptr, *ds2 = nullptr,
-         *dnz = nullptr, *dref = nullptr, *dth0 = nullptr, *dth = nullptr, *dmll = nullptr;
+         *dnz = nullptr, *dref = nullptr, *dth0 = nullptr, *dth = nullptr, *dmll = nullptr,
+         *dpref = nullptr;
   float *dXc = nullptr, *deps = nullptr, *dval = nullptr;
   long long *didx = nullptr;
   int r = BOUTE_OK;
@@ -97,6 +103,7 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
   r |= dmalloc(&dth0, (size_t)m * P);
   r |= dmalloc(&dth, (size_t)m * P);
   r |= dmalloc(&dmll, (size_t)m);
+  if (kc) r |= dmalloc(&dpref, (size_t)m * dc);
   r |= dmalloc(&dXc, (size_t)N * d);
   if (S) r |= dmalloc(&deps, (size_t)N * m * S);
   r |= dmalloc(&didx, 1);
@@ -104,6 +111,12 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
   if (!r) r = copy_in(dXc, cand, sizeof(float) * N * d);
   if (!r && S) r = copy_in(deps, eps, sizeof(float) * N * m * S);
   if (!r) r = copy_in(dref, ref, sizeof(double) * m);
+  if (!r && kc) {  // the preference entries (held fixed)
+    std::vector<double> pr((size_t)m * dc);
+    for (int t = 0; t < m; ++t)
+      for (int k = 0; k < dc; ++k) pr[(size_t)t * dc + k] = kc[(size_t)t * KC + 3 + k];
+    r = copy_in(dpref, pr.data(), sizeof(double) * m * dc);
+  }
   std::vector<int> front = pareto_set(Y, n0, m, transforms);
   int n = n0, stable = 0, it = 0;
   std::vector<double> th((size_t)m * P);
@@ -116,13 +129,20 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
       for (int q = 0; q < d; ++q) th[(size_t)t * P + q] = log(ls[(size_t)t * d + q]);
       th[(size_t)t * P + d] = log(s2[t]);
       th[(size_t)t * P + d + 1] = log(noise[t]);
+      if (kc) {
+        th[(size_t)t * P + d + 2] = log(kc[(size_t)t * KC]);
+        th[(size_t)t * P + d + 3] = log(kc[(size_t)t * KC + 1]);
+        th[(size_t)t * P + d + 4] = kc[(size_t)t * KC + 2];
+      }
     }
     if (!r && cfg->learn_iters > 0) {
       r = boute_standardize(dY, 1, n, m, transforms, dYs, nullptr);
       if (!r) r = copy_in(dth0, th.data(), sizeof(double) * m * P);
       if (!r)
-        r = boute_gp_learn(dX, dYs, 1, n, d, m, dth0, 1, cfg->learn_iters, cfg->learn_lr, dth,
-                           dmll, nullptr, nullptr);
+        r = kc ? boute_gp_learn_k(dX, dYs, 1, n, d, m, d_tau, dpref, dth0, 1, cfg->learn_iters,
+                                  cfg->learn_lr, dth, dmll, nullptr, nullptr)
+               : boute_gp_learn(dX, dYs, 1, n, d, m, dth0, 1, cfg->learn_iters, cfg->learn_lr,
+                                dth, dmll, nullptr, nullptr);
       std::vector<double> thn((size_t)m * P), mll(m);
       if (!r && (cudaMemcpy(thn.data(), dth, sizeof(double) * m * P, cudaMemcpyDeviceToHost) !=
                      cudaSuccess ||
@@ -135,6 +155,11 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
         for (int q = 0; q < d; ++q) ls[(size_t)t * d + q] = exp(th[(size_t)t * P + q]);
         s2[t] = exp(th[(size_t)t * P + d]);
         noise[t] = exp(th[(size_t)t * P + d + 1]);
+        if (kc) {
+          kc[(size_t)t * KC] = exp(th[(size_t)t * P + d + 2]);
+          kc[(size_t)t * KC + 1] = exp(th[(size_t)t * P + d + 3]);
+          kc[(size_t)t * KC + 2] = th[(size_t)t * P + d + 4];
+        }
       }
     }
     if (theta_hist) std::memcpy(theta_hist + (size_t)it * m * P, th.data(), sizeof(double) * m * P);
@@ -146,6 +171,7 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
     if (!r) r = boute_engine_create(1, n, d, m, N, cfg->mode, S, 1, &e);
     if (!r && transforms) r = boute_engine_set_outcome_transforms(e, transforms);
     if (!r && cons) r = boute_engine_set_constraints(e, cons);
+    if (!r && kc) r = boute_engine_set_kernel(e, d_tau, kc);
     if (!r) r = boute_engine_step(e, dX, dY, dls, ds2, dnz, dref, dXc, deps, didx, dval, nullptr);
     boute_engine_free(e);
     long long pick = -1;
@@ -171,7 +197,7 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
     }
   }
   *n_out = n;
-  void *bufs[] = {dX, dY, dYs, dls, ds2, dnz, dref, dth0, dth, dmll, dXc, deps, didx, dval};
+  void *bufs[] = {dX, dY, dYs, dls, ds2, dnz, dref, dth0, dth, dmll, dXc, deps, didx, dval, dpref};
   for (void *p : bufs) cudaFree(p);
   return r;
 }

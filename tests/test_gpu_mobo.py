@@ -19,40 +19,61 @@ def _objective(x):
     return np.array([((x - 0.25) ** 2).sum() / d, ((x - 0.75) ** 2).sum() / d])
 
 
-def _pareto_set(Y):
-    mask, _ = oracle.pareto_front(Y, np.full(Y.shape[1], np.inf))
+def _objective_lq(x):
+    """Latency and quality of a routing (x[:2]) + deployment (x[2:], GPU
+    counts) configuration."""
+    xh = x.copy()
+    xh[2:] /= 4.0
+    f1, f2 = _objective(xh)
+    return np.array([np.exp(f1), 1.0 / (1.0 + np.exp(4.0 * f2 - 0.5))])
+
+
+def _pareto_set(Y, codes=None):
+    Z = Y if codes is None else oracle.outcome_transform(Y, codes)
+    mask, _ = oracle.pareto_front(Z, np.full(Y.shape[1], np.inf))
     return set(np.flatnonzero(mask).tolist())
 
 
-def _check_run(res, cand, n0, patience, max_evals, mode, eps, ls0, s2, noise, learn):
+def _check_run(res, cand, n0, patience, max_evals, mode, eps, ls0, s2, noise, learn,
+               objective=_objective, codes=None, comp=None):
+    """comp: (d_tau, kc0) of the composite kernel, else None."""
     X, Y, sel, theta = res["X"], res["Y"], res["sel"], res["theta"]
     n = len(X)
     assert n == n0 + len(sel)
     ref = np.array([1.1, 1.1])
     d = cand.shape[1]
     th_prev = np.concatenate([np.log(ls0), np.log(s2)[:, None], np.log(noise)[:, None]], 1)
+    if comp:
+        kc0 = comp[1]
+        th_prev = np.concatenate([th_prev, np.log(kc0[:, :2]), kc0[:, 2:3]], 1)
     for t, pick in enumerate(sel):
         nt = n0 + t
         np.testing.assert_array_equal(X[nt], cand[pick].astype(np.float64))
-        np.testing.assert_array_equal(Y[nt], _objective(X[nt]))
+        np.testing.assert_array_equal(Y[nt], objective(X[nt]))
         th = theta[t]
         if learn:  # the oracle learner from the previous iteration's parameters
-            ys = oracle.standardize(Y[:nt])
+            Z = Y[:nt] if codes is None else oracle.outcome_transform(Y[:nt], codes)
+            ys = oracle.standardize(Z)
             for obj in range(2):
+                kern = None if comp is None else (comp[0], comp[1][obj, 3:])
                 th_o, mll_o = oracle.gp_learn(X[:nt], ys[:, obj], th_prev[obj][None], learn[0],
-                                              learn[1])
+                                              learn[1], kernel=kern)
                 np.testing.assert_allclose(th[obj], th_o[0], rtol=0, atol=1e-6)
         else:
             np.testing.assert_allclose(th, th_prev, rtol=0, atol=0)
         th_prev = th
+        kernel = None
+        if comp:
+            kc_t = np.concatenate([np.exp(th[:, d + 2:d + 4]), th[:, d + 4:d + 5], comp[1][:, 3:]], 1)
+            kernel = (comp[0], kc_t)
         fp = opl.fit_problem(X[:nt], Y[:nt], np.exp(th[:, :d]), np.exp(th[:, d]),
-                             np.exp(th[:, d + 1]), ref)
+                             np.exp(th[:, d + 1]), ref, kernel=kernel, transforms=codes)
         mean, var = opl.posterior(fp, cand)
         acq = opl.acquisition(fp, mean, var, mode, eps)
         best = acq.max()
         assert acq[pick] >= best - 1e-3 * max(abs(best), 1e-6), (t, acq[pick], best)
     # stopping rule
-    sets = [_pareto_set(Y[:k]) for k in range(n0, n + 1)]
+    sets = [_pareto_set(Y[:k], codes) for k in range(n0, n + 1)]
     stable = 0
     for k in range(1, len(sets)):
         stable = stable + 1 if sets[k] == sets[k - 1] else 0
@@ -88,6 +109,28 @@ def test_loop_choices_match_oracle(learn):
     hv = [oracle.hv(Y[list(_pareto_set(Y))], np.array([1.0, 1.0]))
           for Y in (res["Y"][:k] for k in range(n0, len(res["Y"]) + 1))]
     assert all(b >= a - 1e-12 for a, b in zip(hv, hv[1:]))
+
+
+def test_loop_with_composite_kernel_transforms_and_learning():
+    from paper_2602_10729_gb300 import boute as bt
+    rng = np.random.default_rng(9)
+    N, n0, dtau = 1024, 8, 2
+    cand = np.concatenate([rng.random((N, 2)), rng.integers(0, 5, (N, 2))], 1).astype(np.float32)
+    X0 = cand[:n0].astype(np.float64)
+    Y0 = np.stack([_objective_lq(x) for x in X0])
+    ls0 = np.tile([0.4, 0.4, 1.6, 1.6], (2, 1))
+    s2, noise = np.ones(2), np.full(2, 1e-3)
+    kc0 = np.concatenate([np.tile([0.5, 0.1, 0.05], (2, 1)), rng.random((2, 2))], 1)
+    codes = [bt.BOUTE_TF_LOG, bt.BOUTE_TF_LOGIT | bt.BOUTE_TF_NEGATE]
+    learn = (10, 0.05)
+    max_evals, patience = 20, 4
+    res = bt.boute_mobo_run(_objective_lq, cand, [1.1, 1.1], ls0, s2, noise, X0, Y0,
+                            max_evals=max_evals, patience=patience, learn_iters=learn[0],
+                            learn_lr=learn[1], transforms=codes, d_tau=dtau, kc=kc0)
+    assert len(res["sel"]) >= patience
+    _check_run(res, cand, n0, patience, max_evals, "ehvi", None, ls0, s2, noise, learn,
+               objective=_objective_lq, codes=codes, comp=(dtau, kc0))
+    assert res["theta"].shape[2] == cand.shape[1] + 5
 
 
 def test_objective_errors_stop_the_loop():
