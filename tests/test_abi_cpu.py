@@ -62,6 +62,38 @@ def test_invalid_arguments_are_rejected_before_any_device_call(lib):
         bt.BOUTE_ERR_UNSUPPORTED, bt.BOUTE_ERR_INVALID_ARG)
     assert lib.boute_engine_set_constraints(None, None) == bt.BOUTE_ERR_INVALID_ARG
     assert lib.boute_gp_status(None, None) == bt.BOUTE_ERR_INVALID_ARG
+    # outcome transforms: unknown codes (3: both log and logit; 8: no such bit)
+    for codes in ([3, 0], [0, 8], [-1, 0]):
+        arr = (ctypes.c_int * 2)(*codes)
+        assert lib.boute_standardize(p, 1, 4, 2, arr, p, None) == bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_engine_set_outcome_transforms(None, None) == bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_engine_set_kernel(None, 0, None) == bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_gp_set_kernel(None, 0, None) == bt.BOUTE_ERR_INVALID_ARG
+    # hyperparameter learning: restarts, steps, step size, d_tau
+    assert lib.boute_gp_learn(p, p, 1, 8, 2, 2, p, 0, 5, 0.1, p, p, None, None) == \
+        bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_gp_learn(p, p, 1, 8, 2, 2, p, 1, -1, 0.1, p, p, None, None) == \
+        bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_gp_learn(p, p, 1, 8, 2, 2, p, 1, 5, float("nan"), p, p, None, None) == \
+        bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_gp_learn_k(p, p, 1, 8, 2, 2, 3, p, p, 1, 5, 0.1, p, p, None, None) == \
+        bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_gp_learn_k(p, p, 1, 8, 2, 2, 1, None, p, 1, 5, 0.1, p, p, None, None) == \
+        bt.BOUTE_ERR_INVALID_ARG
+    # the loop: no configuration, a budget below the initial observations
+    n_out, conv = ctypes.c_int(), ctypes.c_int()
+    fn = bt.ObjectiveFn(lambda *a: 0)
+    assert lib.boute_mobo_run(None, 2, 2, p, 10, None, p, None, None, 0, None, p, p, p, p, p, 4,
+                              fn, None, p, None, ctypes.byref(n_out),
+                              ctypes.byref(conv)) == bt.BOUTE_ERR_INVALID_ARG
+    cfg = bt.MoboConfig(bt.BOUTE_ACQ_EHVI2D, 0, 3, 5, 0, 0.05)
+    assert lib.boute_mobo_run(ctypes.byref(cfg), 2, 2, p, 10, None, p, None, None, 0, None, p, p,
+                              p, p, p, 4, fn, None, p, None, ctypes.byref(n_out),
+                              ctypes.byref(conv)) == bt.BOUTE_ERR_INVALID_ARG
+    cfg = bt.MoboConfig(bt.BOUTE_ACQ_MC_HVI, 0, 8, 5, 0, 0.05)  # MC without normals
+    assert lib.boute_mobo_run(ctypes.byref(cfg), 2, 2, p, 10, None, p, None, None, 0, None, p, p,
+                              p, p, p, 4, fn, None, p, None, ctypes.byref(n_out),
+                              ctypes.byref(conv)) == bt.BOUTE_ERR_INVALID_ARG
 
 
 def test_valid_calls_without_a_device_report_unsupported(lib):
