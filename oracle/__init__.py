@@ -73,6 +73,13 @@ def lib():
         L.bo_gp_mll.restype = ctypes.c_double
         L.bo_gp_learn.argtypes = [_dp, _dp, ctypes.c_int, ctypes.c_int, _dp, ctypes.c_int,
                                   ctypes.c_int, ctypes.c_double, _dp, _dp, _dp]
+        L.bo_philox4x64.argtypes = [ctypes.POINTER(ctypes.c_ulonglong),
+                                    ctypes.POINTER(ctypes.c_ulonglong),
+                                    ctypes.POINTER(ctypes.c_ulonglong)]
+        L.bo_philox4x64.restype = None
+        L.bo_base_normals.argtypes = [ctypes.c_ulonglong, ctypes.c_int, ctypes.c_longlong,
+                                      ctypes.c_int, ctypes.c_int, _fp]
+        L.bo_base_normals.restype = None
         L.bo_gp_mll_k.argtypes = [_dp, _dp, ctypes.c_int, ctypes.c_int, _dp, ctypes.c_double,
                                   ctypes.c_double, ctypes.c_int, _dp, _dp]
         L.bo_gp_mll_k.restype = ctypes.c_double
@@ -275,6 +282,21 @@ def gp_learn(X, y, theta0, iters: int, lr: float, grad: bool = False, kernel=Non
     if rc:
         raise ValueError(rc)
     return (theta, mll, g) if grad else (theta, mll)
+
+
+def philox4x64(ctr, key):
+    """Philox4x64-10 of a 4-word counter and a 2-word key (4 uint64)."""
+    U = ctypes.c_ulonglong
+    c, k, o = (U * 4)(*[int(x) for x in ctr]), (U * 2)(*[int(x) for x in key]), (U * 4)()
+    lib().bo_philox4x64(c, k, o)
+    return [int(x) for x in o]
+
+
+def base_normals(seed: int, B: int, N: int, m: int, S: int):
+    """B x N x m x S fp32 standard normals from the counter-based generator."""
+    out = np.empty((B, N, m, S), np.float32)
+    lib().bo_base_normals(int(seed), B, N, m, S, out.ctypes.data_as(_fp))
+    return out
 
 
 def pareto_front(Y, ref):

@@ -411,6 +411,61 @@ int bo_gp_learn_k(const double *X, const double *y, int n, int d, int dtau, cons
   return 0;
 }
 
+/* ---- Monte-Carlo base normals from a counter-based generator ------------
+ * Philox4x64-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two
+ * 64 x 64 -> 128-bit products with a Weyl key schedule; normals by the
+ * Box-Muller transform of its 53-bit uniforms. */
+static void mulhilo64(unsigned long long a, unsigned long long b, unsigned long long *hi,
+                      unsigned long long *lo) {
+  const unsigned __int128 p = (unsigned __int128)a * b;
+  *hi = (unsigned long long)(p >> 64);
+  *lo = (unsigned long long)p;
+}
+
+void bo_philox4x64(const unsigned long long ctr[4], const unsigned long long key[2],
+                   unsigned long long out[4]) {
+  unsigned long long c0 = ctr[0], c1 = ctr[1], c2 = ctr[2], c3 = ctr[3], k0 = key[0],
+                     k1 = key[1];
+  for (int r = 0; r < 10; ++r) {
+    unsigned long long hi0, lo0, hi1, lo1;
+    mulhilo64(0xD2E7470EE14C6C93ull, c0, &hi0, &lo0);
+    mulhilo64(0xCA5A826395121157ull, c2, &hi1, &lo1);
+    const unsigned long long n0 = hi1 ^ c1 ^ k0, n2 = hi0 ^ c3 ^ k1;
+    c0 = n0;
+    c1 = lo1;
+    c2 = n2;
+    c3 = lo0;
+    k0 += 0x9E3779B97F4A7C15ull;
+    k1 += 0xBB67AE8584CAA73Bull;
+  }
+  out[0] = c0;
+  out[1] = c1;
+  out[2] = c2;
+  out[3] = c3;
+}
+
+void bo_base_normals(unsigned long long seed, int B, long long N, int m, int S, float *eps) {
+  const unsigned long long key[2] = {seed, 0ull};
+  for (int b = 0; b < B; ++b)
+    for (long long c = 0; c < N; ++c)
+      for (int t = 0; t < m; ++t) {
+        float *e = eps + (((size_t)b * N + c) * m + t) * S;
+        for (int j = 0; 4 * j < S; ++j) {
+          const unsigned long long ctr[4] = {(unsigned long long)j, (unsigned long long)c,
+                                             (unsigned long long)b * m + t, 0ull};
+          unsigned long long w[4];
+          bo_philox4x64(ctr, key, w);
+          double u[4];
+          for (int q = 0; q < 4; ++q) u[q] = ((double)(w[q] >> 11) + 0.5) * 0x1p-53;
+          for (int q = 0; q < 2; ++q) {
+            const double rad = sqrt(-2.0 * log(u[2 * q])), ang = 2.0 * M_PI * u[2 * q + 1];
+            if (4 * j + 2 * q < S) e[4 * j + 2 * q] = (float)(rad * cos(ang));
+            if (4 * j + 2 * q + 1 < S) e[4 * j + 2 * q + 1] = (float)(rad * sin(ang));
+          }
+        }
+      }
+}
+
 /* ---- Sec. 5.2: Pareto-optimal set (minimisation) ------------------------- */
 static _Thread_local const double *g_sortY;
 static _Thread_local int g_sortM;

@@ -123,6 +123,19 @@ int bo_gp_learn_k(const double *X, const double *y, int n, int d, int dtau, cons
                   const double *theta0, int R, int iters, double lr, double *theta, double *mll,
                   double *grad);
 
+/* Monte-Carlo base normals from a counter-based generator (the MC estimate of
+ * Sec. 5.2 needs standard normals; these are drawn reproducibly from a seed):
+ * Philox4x64-10 (Salmon et al., SC'11) maps a 4 x 64-bit counter and a
+ * 2 x 64-bit key to 4 x 64-bit words; bo_base_normals fills eps (B x N x m x
+ * S fp32, the layout of boute_acq_mc_hvi) block by block: samples 4j..4j+3 of
+ * candidate c, objective t, problem b come from counter (j, c, b m + t, 0)
+ * and key (seed, 0), each word w giving the uniform ((w >> 11) + 1/2) 2^-53,
+ * each pair (u1, u2) the normals sqrt(-2 ln u1) (cos 2 pi u2, sin 2 pi u2),
+ * computed in fp64 and rounded to fp32. */
+void bo_philox4x64(const unsigned long long ctr[4], const unsigned long long key[2],
+                   unsigned long long out[4]);
+void bo_base_normals(unsigned long long seed, int B, long long N, int m, int S, float *eps);
+
 /* Pareto front of observed outcomes (Sec. 5.2, Pareto-optimal set; all
  * objectives minimised): point i is kept iff no j dominates it (Y_j <= Y_i in
  * every objective, < in one), no exact duplicate j < i exists, and

@@ -806,3 +806,40 @@ def test_composite_learner_first_step_and_bounds():
                                                  oracle.BETA_BOUNDS[1]])
     th2, mll2 = oracle.gp_learn(X, y, th0[:1], 200, lr, kernel=(dtau, pref))
     assert mll2[0] > _mll_library_k(X, y, th0[0], dtau, pref)
+
+
+# --------------------------------- Monte-Carlo base normals (counter-based generator)
+@pytest.mark.parametrize("key,ctr", [((0, 0), (0, 0, 0, 0)), ((123456789, 987654321), (5, 7, 2, 0)),
+                                     ((2**64 - 1, 2**63 + 11), (2**64 - 2, 2**64 - 1, 3, 2**62))])
+def test_philox_matches_numpy_bit_generator(key, ctr):
+    # numpy's Philox (4 x 64-bit, 10 rounds) is the same generator; it
+    # advances the counter by one before each block of four words
+    bg = np.random.Philox(key=np.array(key, dtype=np.uint64),
+                          counter=np.array(ctr, dtype=np.uint64))
+    raw = [int(x) for x in bg.random_raw(8)]
+    nxt = list(ctr)
+    for i in range(4):  # the counter plus one, with carries
+        nxt[i] = (nxt[i] + 1) % 2**64
+        if nxt[i] != 0:
+            break
+    assert oracle.philox4x64(nxt, key) == raw[:4]
+
+
+def test_base_normals_layout_and_distribution():
+    eps = oracle.base_normals(7, 2, 3000, 2, 128)
+    # the layout: candidate c, objective t, samples 4j..4j+3 from counter (j, c, b m + t, 0)
+    w = oracle.philox4x64((5, 17, 1 * 2 + 1, 0), (7, 0))
+    u = [((x >> 11) + 0.5) * 2.0 ** -53 for x in w]
+    want = [math.sqrt(-2 * math.log(u[0])) * math.cos(2 * math.pi * u[1]),
+            math.sqrt(-2 * math.log(u[0])) * math.sin(2 * math.pi * u[1]),
+            math.sqrt(-2 * math.log(u[2])) * math.cos(2 * math.pi * u[3]),
+            math.sqrt(-2 * math.log(u[2])) * math.sin(2 * math.pi * u[3])]
+    np.testing.assert_allclose(eps[1, 17, 1, 20:24], want, rtol=1e-6, atol=1e-7)
+    z = eps.astype(np.float64).ravel()
+    se = 1 / math.sqrt(z.size)
+    assert abs(z.mean()) < 5 * se and abs(z.var() - 1) < 5 * math.sqrt(2) * se
+    assert abs((z ** 4).mean() - 3) < 0.05  # normal kurtosis
+    # distinct seeds, problems and objectives give different streams
+    assert not np.array_equal(eps[0, :, 0], eps[0, :, 1])
+    assert not np.array_equal(eps[0], eps[1])
+    assert not np.array_equal(oracle.base_normals(8, 1, 10, 2, 8), eps[:1, :10, :, :8])
