@@ -15,7 +15,10 @@ line. Between timed steps the L2 is flushed (a 512 MB write outside the
 timed events). The `e2e` object times a stream of steps through the
 pipelined host-buffer call (boute_engine_step_host_async): every step copies
 its inputs in from pinned host memory and its selection out, and one step's
-copies overlap the previous step's computation.
+copies overlap the previous step's computation. Monte-Carlo workloads there
+use the engine's own base normals, drawn once on the device from a seed
+(fixed base samples, as an optimisation loop keeps them), so a step's inputs
+are its observations, hyperparameters and candidates.
 """
 from __future__ import annotations
 
@@ -335,7 +338,14 @@ def main():
     # ---- end to end through the public API with host buffers ----------------
     pin = lambda a, dt: None if a is None else torch.as_tensor(a, dtype=dt).pin_memory()
     hX, hY, hls, hs2, hnz, href = (pin(inp[k], f64) for k in ("X", "Y", "ls", "s2", "noise", "ref"))
-    hXc, heps = pin(inp["Xc"], f32), pin(inp["eps"], f32)
+    hXc = pin(inp["Xc"], f32)
+    # Monte-Carlo steps: fixed base normals drawn once on the device from a
+    # seed (the engine's own), as an optimisation loop keeps its base samples;
+    # a step's host inputs are then the observations, hyperparameters and
+    # candidates
+    heps = None
+    if w.mode == "mc":
+        bt.boute_engine_set_normals(e, 1234)
     hidx = torch.empty((w.B, w.k), dtype=torch.int64).pin_memory()
     hval = torch.empty((w.B, w.k), dtype=f32).pin_memory()
     args_host = (hX, hY, hls, hs2, hnz, href, hXc, heps, hidx, hval)
@@ -390,7 +400,8 @@ def main():
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "call": "boute_engine_step_host_async",
-                    "pipelined": True},
+                    "pipelined": True,
+                    "normals": "device (boute_engine_set_normals)" if w.mode == "mc" else None},
             "gpu_launches": launches,
             "launches_per_step": bt.boute_engine_launches_per_step(e),
             "stage_ms": stage_ms,

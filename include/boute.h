@@ -230,6 +230,18 @@ int boute_acq_mc_hvi(const float *mean, const float *var, int B, long long N, in
                      const float *eps, int S, long long eps_cand_stride, const double *cons,
                      float *acq, void *stream);
 
+/* Monte-Carlo base normals from a counter-based generator, for callers that
+ * do not draw their own: Philox4x64-10 (Salmon et al., SC'11, counter-based:
+ * any sample can be regenerated alone) and the Box-Muller transform in fp64,
+ * rounded to fp32. eps: B x N x m x S device (the layout of
+ * boute_acq_mc_hvi with eps_cand_stride = m*S); samples 4j..4j+3 of candidate
+ * c, objective t, problem b come from counter (j, c, b m + t, 0) and key
+ * (seed, 0), each 64-bit word w giving the uniform ((w >> 11) + 1/2) 2^-53
+ * and each pair (u1, u2) the normals sqrt(-2 ln u1) (cos 2 pi u2, sin 2 pi u2).
+ * Asynchronous on `stream`. */
+int boute_base_normals(unsigned long long seed, int B, long long N, int m, int S, float *eps,
+                       void *stream);
+
 /* ---- selection ----------------------------------------------------------------
  * Sec. 5.2 step (ii): the next configuration(s) to evaluate are the best
  * scored candidates. Per problem, the k largest acq values in the order
@@ -342,6 +354,10 @@ int boute_engine_set_outcome_transforms(boute_engine *e, const int *codes);
 /* The composite kernel for the engine's later steps (see boute_gp_set_kernel;
  * params is a HOST array, NULL restores the Matern-5/2 kernel). */
 int boute_engine_set_kernel(boute_engine *e, int d_tau, const double *params);
+/* Monte-Carlo engines: draws the engine's own base normals from `seed`
+ * (boute_base_normals) into a resident buffer; later steps whose eps is NULL
+ * use them (and the host-input steps copy no normals). Synchronous. */
+int boute_engine_set_normals(boute_engine *e, unsigned long long seed);
 void boute_engine_free(boute_engine *e);
 
 /* ---- the optimisation loop ------------------------------------------------------

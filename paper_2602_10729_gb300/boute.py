@@ -30,7 +30,8 @@ SYMBOLS = (
     "boute_engine_scores", "boute_engine_set_timing",
     "boute_engine_stage_times", "boute_engine_launches_per_step", "boute_engine_set_constraints",
     "boute_engine_set_outcome_transforms", "boute_engine_set_kernel", "boute_gp_set_kernel",
-    "boute_gp_learn", "boute_gp_learn_k", "boute_mobo_run",
+    "boute_gp_learn", "boute_gp_learn_k", "boute_mobo_run", "boute_base_normals",
+    "boute_engine_set_normals",
     "boute_engine_free",
 )
 #: stage names of boute_engine_stage_times, in order
@@ -107,6 +108,8 @@ def load(path: str | None = None):
                             _vp], _i),
         "boute_gp_learn_k": ([_vp, _vp, _i, _i, _i, _i, _i, _vp, _vp, _i, _i, ctypes.c_double, _vp,
                               _vp, _vp, _vp], _i),
+        "boute_base_normals": ([ctypes.c_ulonglong, _i, _ll, _i, _i, _vp, _vp], _i),
+        "boute_engine_set_normals": ([_vp, ctypes.c_ulonglong], _i),
         "boute_mobo_run": ([ctypes.POINTER(MoboConfig), _i, _i, _vp, _ll, _vp, _vp, _vp, _vp, _i,
                             _vp, _vp, _vp, _vp, _vp, _vp, _i, ObjectiveFn, _vp, _vp, _vp,
                             ctypes.POINTER(_i), ctypes.POINTER(_i)], _i),
@@ -288,6 +291,18 @@ def boute_gp_learn_k(X, Ys, d_tau, pref, theta0, iters: int, lr: float, theta, m
     _check(load().boute_gp_learn_k(_p(X, f64), _p(Ys, f64), B, n, d, m, int(d_tau), _p(pref, f64),
                                    _p(theta0, f64), R, int(iters), float(lr), _p(theta, f64),
                                    _p(mll, f64), _p(grad, f64), _s(stream)), "boute_gp_learn_k")
+
+
+def boute_base_normals(seed: int, eps, stream=None):
+    """Fills eps (B x N x m x S fp32 CUDA tensor) from the counter-based generator."""
+    B, N, m, S = eps.shape
+    _check(load().boute_base_normals(int(seed), B, N, m, S, _p(eps, torch.float32), _s(stream)),
+           "boute_base_normals")
+
+
+def boute_engine_set_normals(e: Engine, seed: int):
+    """The engine's own base normals; steps then take eps=None."""
+    _check(load().boute_engine_set_normals(e.handle, int(seed)), "boute_engine_set_normals")
 
 
 def _host_f64(a):

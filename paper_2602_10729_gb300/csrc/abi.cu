@@ -125,6 +125,9 @@ struct boute_engine {
   // writes the transformed outcomes to Yt, which the fit and the front read
   int tcodes;
   double *Yt;
+  // the engine's own base normals (boute_engine_set_normals), used by steps
+  // whose eps is null; null until set
+  float *gen_eps;
 };
 
 // Stage order of one step as timed (with timing on, the front stage runs
@@ -366,7 +369,7 @@ void boute_engine_free(boute_engine *e) {
   void *ptrs[] = {e->X, e->Y, e->Ys, e->ls, e->s2, e->noise, e->ref, e->front, e->mask, e->P,
                   e->K, e->lower, e->upper, e->Xc, e->eps, e->mean, e->var, e->acq, e->val,
                   e->idx, e->scratch, e->sel, e->kst, e->X1, e->Y1, e->ls1, e->s21,
-                  e->noise1, e->ref1, e->Xc1, e->eps1, e->cons, e->Yt};
+                  e->noise1, e->ref1, e->Xc1, e->eps1, e->cons, e->Yt, e->gen_eps};
   for (void *p : ptrs) cudaFree(p);
   delete e;
 }
@@ -534,7 +537,7 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
   if ((r = launch_posterior(&e->gp->g, Xc, e->N, e->mean, e->var, s, kst))) return r;
   if (!e->timing && cudaStreamWaitEvent(s, e->join, 0) != cudaSuccess)  // join
     return last_launch_status();
-  if (host && mc)
+  if (host && mc && eps != e->gen_eps)  // (the engine's own normals are resident)
     for (int i = 0; i < 2; ++i)
       if (cudaStreamWaitEvent(s, ev_eps[i], wait_flags) != cudaSuccess)
         return last_launch_status();
@@ -566,7 +569,7 @@ static int engine_args_ok(const boute_engine *e, const void *X, const void *Y, c
                           const void *s2, const void *noise, const void *ref, const void *Xc,
                           const void *eps, const void *idx, const void *val) {
   if (!e || !X || !Y || !ls || !s2 || !noise || !ref || !Xc || !idx || !val) return 0;
-  if (e->mode == BOUTE_ACQ_MC_HVI && !eps) return 0;
+  if (e->mode == BOUTE_ACQ_MC_HVI && !eps && !e->gen_eps) return 0;
   return 1;
 }
 
@@ -630,6 +633,7 @@ int boute_engine_step_async(boute_engine *e, const double *X, const double *Y,
                             const float *eps, long long *idx, float *val, void *stream) {
   if (!engine_args_ok(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val))
     return BOUTE_ERR_INVALID_ARG;
+  if (!eps) eps = e->gen_eps;  // the engine's own normals (Monte-Carlo steps)
   return engine_launch(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val,
                        (cudaStream_t)stream);
 }
@@ -686,14 +690,16 @@ static int engine_host_step(boute_engine *e, int set, const double *X, const dou
   cudaEventRecord(e->ev_small[set], c0);
   cudaMemcpyAsync(dXc, Xc, B * N * d * sizeof(float), cudaMemcpyHostToDevice, c0);
   cudaEventRecord(ev_xc, e->cpy[0]);
-  const size_t eps_n = e->mode == BOUTE_ACQ_MC_HVI ? B * N * m * S : 0, half = eps_n / 2;
-  for (int i = 0; i < 2; ++i) {  // the normals in two halves, one per copy stream
+  const size_t eps_n = e->mode == BOUTE_ACQ_MC_HVI && eps ? B * N * m * S : 0,
+               half = eps_n / 2;
+  for (int i = 0; eps && i < 2; ++i) {  // the normals in two halves, one per copy stream
     const size_t off = i ? half : 0, cnt = i ? eps_n - half : half;
     if (cnt)
       cudaMemcpyAsync(deps + off, eps + off, cnt * sizeof(float), cudaMemcpyHostToDevice,
                       e->cpy[i]);
     cudaEventRecord(ev_eps[i], e->cpy[i]);
   }
+  if (!eps) deps = e->gen_eps;  // null: the engine's own normals
   if (int r = last_launch_status()) return r;
   int r = engine_launch(e, dX, dY, dls, ds2, dnz, dref, dXc, deps, e->idx, e->val, s, 1 + set);
   if (r) return r;
@@ -794,6 +800,23 @@ int boute_engine_set_kernel(boute_engine *e, int d_tau, const double *params) {
   if (!e) return BOUTE_ERR_INVALID_ARG;
   const int r = boute_gp_set_kernel(e->gp, d_tau, params);
   engine_drop_graphs(e);  // the step's kernel choices change
+  return r;
+}
+
+int boute_base_normals(unsigned long long seed, int B, long long N, int m, int S, float *eps,
+                       void *stream) {
+  if (B < 1 || N < 0 || m < 1 || S < 1 || (N > 0 && !eps)) return BOUTE_ERR_INVALID_ARG;
+  if (int r = device_ok()) return r;
+  return launch_base_normals(seed, B, N, m, S, eps, (cudaStream_t)stream);
+}
+
+int boute_engine_set_normals(boute_engine *e, unsigned long long seed) {
+  if (!e || e->mode != BOUTE_ACQ_MC_HVI) return BOUTE_ERR_INVALID_ARG;
+  if (cudaDeviceSynchronize() != cudaSuccess) return last_launch_status();
+  const size_t count = (size_t)e->B * e->N * e->m * e->S;
+  if (!e->gen_eps && dalloc(&e->gen_eps, count) != BOUTE_OK) return BOUTE_ERR_OOM;
+  int r = launch_base_normals(seed, e->B, e->N, e->m, e->S, e->gen_eps, nullptr);
+  if (!r && cudaDeviceSynchronize() != cudaSuccess) r = last_launch_status();
   return r;
 }
 

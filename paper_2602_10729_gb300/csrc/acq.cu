@@ -516,4 +516,72 @@ int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
   return last_launch_status();
 }
 
+// ---- Monte-Carlo base normals from a counter-based generator -------------------
+// Philox4x64-10 (Salmon et al., SC'11) and the Box-Muller transform, in
+// fp64, one thread per block of four samples: samples 4j..4j+3 of candidate
+// c, objective t of problem b from counter (j, c, b m + t, 0), key (seed, 0).
+namespace {
+
+__device__ __forceinline__ void philox4x64(unsigned long long (&c)[4], unsigned long long k0,
+                                           unsigned long long k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const unsigned long long M0 = 0xD2E7470EE14C6C93ull, M1 = 0xCA5A826395121157ull;
+    const unsigned long long hi0 = __umul64hi(M0, c[0]), lo0 = M0 * c[0];
+    const unsigned long long hi1 = __umul64hi(M1, c[2]), lo1 = M1 * c[2];
+    const unsigned long long n0 = hi1 ^ c[1] ^ k0, n2 = hi0 ^ c[3] ^ k1;
+    c[0] = n0;
+    c[1] = lo1;
+    c[2] = n2;
+    c[3] = lo0;
+    k0 += 0x9E3779B97F4A7C15ull;
+    k1 += 0xBB67AE8584CAA73Bull;
+  }
+}
+
+__global__ void normals_kernel(unsigned long long seed, int B, long long N, int m, int S,
+                               float *eps) {
+  const int J = (S + 3) / 4;
+  const long long units = (long long)B * N * m * J;
+  for (long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x; u < units;
+       u += (long long)gridDim.x * blockDim.x) {
+    const int j = (int)(u % J);
+    const long long row = u / J;  // (b N + c) m + t
+    const int t = (int)(row % m);
+    const long long bc = row / m, c = bc % N, b = bc / N;
+    unsigned long long w[4] = {(unsigned long long)j, (unsigned long long)c,
+                               (unsigned long long)b * m + t, 0ull};
+    philox4x64(w, seed, 0ull);
+    float z[4];
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const double u1 = ((double)(w[2 * q] >> 11) + 0.5) * 0x1p-53;
+      const double u2 = ((double)(w[2 * q + 1] >> 11) + 0.5) * 0x1p-53;
+      const double rad = sqrt(-2.0 * log(u1));
+      double sn, cs;
+      sincos(2.0 * M_PI * u2, &sn, &cs);
+      z[2 * q] = (float)(rad * cs);
+      z[2 * q + 1] = (float)(rad * sn);
+    }
+    float *e = eps + (size_t)row * S + 4 * j;
+    if (4 * j + 4 <= S && ((uintptr_t)e & 15) == 0) {
+      *(float4 *)e = make_float4(z[0], z[1], z[2], z[3]);
+    } else {
+      for (int q = 0; q < 4 && 4 * j + q < S; ++q) e[q] = z[q];
+    }
+  }
+}
+
+}  // namespace
+
+int launch_base_normals(unsigned long long seed, int B, long long N, int m, int S, float *eps,
+                        cudaStream_t s) {
+  const long long units = (long long)B * N * m * ((S + 3) / 4);
+  if (units <= 0) return BOUTE_OK;
+  const int blocks = (int)std::min<long long>((units + 255) / 256, 32LL * num_sms());
+  normals_kernel<<<blocks, 256, 0, s>>>(seed, B, N, m, S, eps);
+  count_launch();
+  return last_launch_status();
+}
+
 }  // namespace boute

@@ -112,6 +112,9 @@ int launch_mchvi(const float *mean, const float *var, int B, long long N, int m,
 int launch_learn(const double *X, const double *Ys, int B, int n, int d, int m,
                  const double *theta0, int R, int iters, double lr, double *theta, double *mll,
                  double *grad, int dtau, const double *pref, cudaStream_t s);
+// Monte-Carlo base normals from Philox4x64-10 and Box-Muller (B x N x m x S)
+int launch_base_normals(unsigned long long seed, int B, long long N, int m, int S, float *eps,
+                        cudaStream_t s);
 size_t topk_scratch_bytes(int B, long long N, int k);
 // counters_zeroed: the scratch's per-problem counters are known to be zero
 // (an engine's scratch: zeroed at creation, and every call leaves them zero);
