@@ -172,6 +172,22 @@ def profiled_traffic(kernel: str, workload: str):
     return float(mt.group(1))
 
 
+# ---------------------------------------------------------------- ranks
+def max_over_ranks(x: float, dist=None, device="cpu") -> float:
+    """The largest value of x over all ranks (x itself without a process group)."""
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    if dist is not None:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world: int, w: wl.Workload, seconds: float) -> float:
+    """Candidates per second over all ranks, each scoring its own replica of
+    the workload (B N candidates) in `seconds` (the slowest rank's time)."""
+    return world * w.B * w.N / seconds
+
+
 # ---------------------------------------------------------------- CPU oracle
 def oracle_rate(w: wl.Workload, inp, budget_s: float, threads: int = 0, cons=None):
     """The oracle's scoring step (fit, front, posterior, acquisition, top-k)
@@ -315,11 +331,8 @@ def main():
     clk = clocks.stop() if clocks else None
     bt.boute_engine_step(e, *args_dev)  # synchronising step: raises on any recorded device error
     ms = sum(a.elapsed_time(b) for a, b in ev) / args.steps
-    ms_all = torch.tensor([ms], dtype=torch.float64, device=dev)
-    if dist:
-        dist.all_reduce(ms_all, op=dist.ReduceOp.MAX)
-    ms_max = float(ms_all.item())
-    value = world * w.B * w.N / (ms_max * 1e-3)
+    ms_max = max_over_ranks(ms, dist, dev)
+    value = whole_job_rate(world, w, ms_max * 1e-3)
 
     # ---- per-stage breakdown: separate steps with stage events (front stage
     # serialised after the fit so that the stages add up) -----------------------
@@ -365,10 +378,7 @@ def main():
         bt.boute_engine_step_host_async(e, *args_host)
     bt.boute_engine_sync(e)
     e2e_s = (time.perf_counter() - t0) / n_e2e
-    e2e_all = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
-    if dist:
-        dist.all_reduce(e2e_all, op=dist.ReduceOp.MAX)
-    e2e_value = world * w.B * w.N / float(e2e_all.item())
+    e2e_value = whole_job_rate(world, w, max_over_ranks(e2e_s, dist, dev))
 
     if rank == 0:
         hbm, bf16, bf16s, src = peaks()
