@@ -230,6 +230,15 @@ int boute_acq_mc_hvi(const float *mean, const float *var, int B, long long N, in
                      const float *eps, int S, long long eps_cand_stride, const double *cons,
                      float *acq, void *stream);
 
+/* Failure detection: every device-side wait of the library is bounded (about
+ * 2 s) and a wait that runs out records BOUTE_ERR_TIMEOUT in the call's
+ * status instead of hanging. This self-test runs one such bounded wait on
+ * an mbarrier with limit_ns (<= 2e9) and returns BOUTE_ERR_TIMEOUT when the
+ * wait ran out (complete = 0: nothing arrives) or BOUTE_OK when it
+ * completed (complete != 0: the one expected arrival is made). Synchronous;
+ * the device stays usable either way. */
+int boute_selftest_wait(int complete, unsigned long long limit_ns, void *stream);
+
 /* Monte-Carlo base normals from a counter-based generator, for callers that
  * do not draw their own: Philox4x64-10 (Salmon et al., SC'11, counter-based:
  * any sample can be regenerated alone) and the Box-Muller transform in fp64,

@@ -31,7 +31,7 @@ SYMBOLS = (
     "boute_engine_stage_times", "boute_engine_launches_per_step", "boute_engine_set_constraints",
     "boute_engine_set_outcome_transforms", "boute_engine_set_kernel", "boute_gp_set_kernel",
     "boute_gp_learn", "boute_gp_learn_k", "boute_mobo_run", "boute_base_normals",
-    "boute_engine_set_normals",
+    "boute_engine_set_normals", "boute_selftest_wait",
     "boute_engine_free",
 )
 #: stage names of boute_engine_stage_times, in order
@@ -110,6 +110,7 @@ def load(path: str | None = None):
                               _vp, _vp, _vp], _i),
         "boute_base_normals": ([ctypes.c_ulonglong, _i, _ll, _i, _i, _vp, _vp], _i),
         "boute_engine_set_normals": ([_vp, ctypes.c_ulonglong], _i),
+        "boute_selftest_wait": ([_i, ctypes.c_ulonglong, _vp], _i),
         "boute_mobo_run": ([ctypes.POINTER(MoboConfig), _i, _i, _vp, _ll, _vp, _vp, _vp, _vp, _i,
                             _vp, _vp, _vp, _vp, _vp, _vp, _i, ObjectiveFn, _vp, _vp, _vp,
                             ctypes.POINTER(_i), ctypes.POINTER(_i)], _i),
@@ -303,6 +304,11 @@ def boute_base_normals(seed: int, eps, stream=None):
 def boute_engine_set_normals(e: Engine, seed: int):
     """The engine's own base normals; steps then take eps=None."""
     _check(load().boute_engine_set_normals(e.handle, int(seed)), "boute_engine_set_normals")
+
+
+def boute_selftest_wait(complete: bool, limit_ns: int, stream=None) -> int:
+    """Status of one bounded device-side wait (BOUTE_ERR_TIMEOUT if it ran out)."""
+    return int(load().boute_selftest_wait(int(complete), int(limit_ns), _s(stream)))
 
 
 def _host_f64(a):

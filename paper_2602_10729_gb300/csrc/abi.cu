@@ -166,6 +166,7 @@ static bool pack_codes(const int *codes, int m, int *packed) {
 
 int boute_standardize(const double *Y, int B, int n, int m, const int *transforms, double *Ys,
                       void *stream) {
+  BOUTE_TRACE();
   int codes = 0;
   if (!Y || !Ys || B < 1 || n < 1 || m < 1 || m > BOUTE_MAX_M || !pack_codes(transforms, m, &codes))
     return BOUTE_ERR_INVALID_ARG;
@@ -174,6 +175,7 @@ int boute_standardize(const double *Y, int B, int n, int m, const int *transform
 }
 
 int boute_gp_create(int B, int n, int d, int m, boute_gp **out) {
+  BOUTE_TRACE();
   if (!out) return BOUTE_ERR_INVALID_ARG;
   *out = nullptr;
   if (!shape_ok(B, n, d, m)) return BOUTE_ERR_INVALID_ARG;
@@ -208,11 +210,13 @@ int boute_gp_create(int B, int n, int d, int m, boute_gp **out) {
 
 int boute_gp_fit(boute_gp *gp, const double *X, const double *Ys, const double *lengthscale,
                  const double *outputscale, const double *noise, void *stream) {
+  BOUTE_TRACE();
   if (!gp || !X || !Ys || !lengthscale || !outputscale || !noise) return BOUTE_ERR_INVALID_ARG;
   return launch_fit(&gp->g, X, Ys, lengthscale, outputscale, noise, (cudaStream_t)stream);
 }
 
 int boute_gp_status(boute_gp *gp, void *stream) {
+  BOUTE_TRACE();
   if (!gp) return BOUTE_ERR_INVALID_ARG;
   if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return last_launch_status();
   int st = 0;
@@ -223,6 +227,7 @@ int boute_gp_status(boute_gp *gp, void *stream) {
 }
 
 void boute_gp_free(boute_gp *gp) {
+  BOUTE_TRACE();
   if (!gp) return;
   Gp &g = gp->g;
   cudaFree(g.Kh); cudaFree(g.Kl); cudaFree(g.Aws); cudaFree(g.Wws); cudaFree(g.bop); cudaFree(g.xt);
@@ -233,6 +238,7 @@ void boute_gp_free(boute_gp *gp) {
 int boute_gp_learn(const double *X, const double *Ys, int B, int n, int d, int m,
                    const double *theta0, int R, int iters, double lr, double *theta,
                    double *mll, double *grad, void *stream) {
+  BOUTE_TRACE();
   if (!X || !Ys || !theta0 || !theta || !mll || !shape_ok(B, n, d, m) || R < 1 || iters < 0 ||
       !(lr >= 0.0))
     return BOUTE_ERR_INVALID_ARG;
@@ -245,6 +251,7 @@ int boute_gp_learn(const double *X, const double *Ys, int B, int n, int d, int m
 int boute_gp_learn_k(const double *X, const double *Ys, int B, int n, int d, int m, int d_tau,
                      const double *pref, const double *theta0, int R, int iters, double lr,
                      double *theta, double *mll, double *grad, void *stream) {
+  BOUTE_TRACE();
   if (!X || !Ys || !pref || !theta0 || !theta || !mll || !shape_ok(B, n, d, m) || R < 1 ||
       iters < 0 || !(lr >= 0.0) || d_tau < 0 || d_tau > d)
     return BOUTE_ERR_INVALID_ARG;
@@ -255,6 +262,7 @@ int boute_gp_learn_k(const double *X, const double *Ys, int B, int n, int d, int
 }
 
 int boute_gp_set_kernel(boute_gp *gp, int d_tau, const double *params) {
+  BOUTE_TRACE();
   if (!gp) return BOUTE_ERR_INVALID_ARG;
   Gp &g = gp->g;
   if (!params) {
@@ -285,6 +293,7 @@ int boute_gp_set_kernel(boute_gp *gp, int d_tau, const double *params) {
 
 int boute_gp_posterior(const boute_gp *gp, const float *Xc, long long N, float *mean, float *var,
                        void *stream) {
+  BOUTE_TRACE();
   if (!gp || N < 0 || (N > 0 && (!Xc || !mean || !var))) return BOUTE_ERR_INVALID_ARG;
   if ((long long)gp->g.B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;
   return launch_posterior(&gp->g, Xc, N, mean, var, (cudaStream_t)stream);
@@ -292,6 +301,7 @@ int boute_gp_posterior(const boute_gp *gp, const float *Xc, long long N, float *
 
 int boute_pareto_front(const double *Ys, int B, int n, int m, const double *ref,
                        unsigned char *mask, double *front, int *P, void *stream) {
+  BOUTE_TRACE();
   if (!Ys || !ref || !mask || !front || !P || !shape_ok(B, n, 1, m)) return BOUTE_ERR_INVALID_ARG;
   if (int r = device_ok()) return r;
   return launch_pareto(Ys, B, n, m, ref, mask, front, P, (cudaStream_t)stream);
@@ -299,6 +309,7 @@ int boute_pareto_front(const double *Ys, int B, int n, int m, const double *ref,
 
 int boute_box_decompose(const double *front, const int *P, int B, int n, int m, const double *ref,
                         float *lower, float *upper, int *K, void *stream) {
+  BOUTE_TRACE();
   if (!front || !P || !ref || !lower || !upper || !K || !shape_ok(B, n, 1, m))
     return BOUTE_ERR_INVALID_ARG;
   if (m < 2 || m > 3) return BOUTE_ERR_UNSUPPORTED;
@@ -309,6 +320,7 @@ int boute_box_decompose(const double *front, const int *P, int B, int n, int m, 
 int boute_acq_ehvi(const float *mean, const float *var, int B, long long N, const double *front,
                    const int *P, int n, const double *ref, const double *cons, float *acq,
                    void *stream) {
+  BOUTE_TRACE();
   if (B < 1 || N < 0 || n < 1 || n > BOUTE_MAX_N || !front || !P || !ref ||
       (N > 0 && (!mean || !var || !acq)))
     return BOUTE_ERR_INVALID_ARG;
@@ -321,6 +333,7 @@ int boute_acq_mc_hvi(const float *mean, const float *var, int B, long long N, in
                      const float *lower, const float *upper, const int *K, int box_cap,
                      const float *eps, int S, long long eps_cand_stride, const double *cons,
                      float *acq, void *stream) {
+  BOUTE_TRACE();
   if (B < 1 || N < 0 || S < 1 || box_cap < 1 || eps_cand_stride < 0 || !lower || !upper || !K ||
       (N > 0 && (!mean || !var || !acq || !eps)))
     return BOUTE_ERR_INVALID_ARG;
@@ -334,6 +347,7 @@ int boute_acq_mc_hvi(const float *mean, const float *var, int B, long long N, in
 
 int boute_select_topk(const float *acq, int B, long long N, int k, long long *idx, float *val,
                       void *stream) {
+  BOUTE_TRACE();
   if (!acq || !idx || !val || B < 1 || N < 1 || k < 1 || k > 1024 || k > N)
     return BOUTE_ERR_INVALID_ARG;
   if ((long long)B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;
@@ -351,6 +365,7 @@ int boute_select_topk(const float *acq, int B, long long N, int k, long long *id
 
 // ---- engine -------------------------------------------------------------------
 void boute_engine_free(boute_engine *e) {
+  BOUTE_TRACE();
   if (!e) return;
   boute_gp_free(e->gp);
   if (e->ev[0])
@@ -388,6 +403,7 @@ static bool engine_fuses_selection(const boute_engine *e) {
 
 int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S, int k,
                         boute_engine **out) {
+  BOUTE_TRACE();
   if (!out) return BOUTE_ERR_INVALID_ARG;
   *out = nullptr;
   if (!shape_ok(B, n, d, m) || N < 1 || k < 1 || k > 1024 || k > N) return BOUTE_ERR_INVALID_ARG;
@@ -631,6 +647,7 @@ int boute_engine_step_async(boute_engine *e, const double *X, const double *Y,
                             const double *lengthscale, const double *outputscale,
                             const double *noise, const double *ref, const float *Xc,
                             const float *eps, long long *idx, float *val, void *stream) {
+  BOUTE_TRACE();
   if (!engine_args_ok(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val))
     return BOUTE_ERR_INVALID_ARG;
   if (!eps) eps = e->gen_eps;  // the engine's own normals (Monte-Carlo steps)
@@ -652,6 +669,7 @@ int boute_engine_step(boute_engine *e, const double *X, const double *Y,
                       const double *lengthscale, const double *outputscale, const double *noise,
                       const double *ref, const float *Xc, const float *eps, long long *idx,
                       float *val, void *stream) {
+  BOUTE_TRACE();
   int r = boute_engine_step_async(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx,
                                   val, stream);
   if (!r) r = boute_gp_status(e->gp, stream);
@@ -713,6 +731,7 @@ int boute_engine_step_host(boute_engine *e, const double *X, const double *Y,
                            const double *lengthscale, const double *outputscale,
                            const double *noise, const double *ref, const float *Xc,
                            const float *eps, long long *idx, float *val, void *stream) {
+  BOUTE_TRACE();
   if (!engine_args_ok(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val))
     return BOUTE_ERR_INVALID_ARG;
   int r = engine_host_step(e, 0, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val,
@@ -726,6 +745,7 @@ int boute_engine_step_host_async(boute_engine *e, const double *X, const double 
                                  const double *lengthscale, const double *outputscale,
                                  const double *noise, const double *ref, const float *Xc,
                                  const float *eps, long long *idx, float *val, void *stream) {
+  BOUTE_TRACE();
   if (!engine_args_ok(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val))
     return BOUTE_ERR_INVALID_ARG;
   if (!e->X1) {  // the second input set, on first use
@@ -743,6 +763,7 @@ int boute_engine_step_host_async(boute_engine *e, const double *X, const double 
 }
 
 int boute_engine_sync(boute_engine *e, void *stream) {
+  BOUTE_TRACE();
   if (!e) return BOUTE_ERR_INVALID_ARG;
   const int r = boute_gp_status(e->gp, stream);
   if (r) engine_reset_counters(e);
@@ -751,6 +772,7 @@ int boute_engine_sync(boute_engine *e, void *stream) {
 
 int boute_engine_scores(const boute_engine *e, float *acq, float *mean, float *var,
                         void *stream) {
+  BOUTE_TRACE();
   if (!e) return BOUTE_ERR_INVALID_ARG;
   cudaStream_t s = (cudaStream_t)stream;
   const size_t BN = (size_t)e->B * e->N;
@@ -761,6 +783,7 @@ int boute_engine_scores(const boute_engine *e, float *acq, float *mean, float *v
 }
 
 int boute_engine_set_timing(boute_engine *e, int on) {
+  BOUTE_TRACE();
   if (!e) return BOUTE_ERR_INVALID_ARG;
   on = on != 0;
   if (on == e->timing) return BOUTE_OK;
@@ -777,6 +800,7 @@ int boute_engine_set_timing(boute_engine *e, int on) {
 }
 
 int boute_engine_stage_times(boute_engine *e, float *ms, int count) {
+  BOUTE_TRACE();
   if (!e || !ms || count < ST_COUNT || !e->ev[0]) return BOUTE_ERR_INVALID_ARG;
   if (cudaEventSynchronize(e->ev[ST_COUNT]) != cudaSuccess) return last_launch_status();
   for (int i = 0; i < ST_COUNT; ++i)
@@ -797,20 +821,40 @@ static void engine_drop_graphs(boute_engine *e) {
 }
 
 int boute_engine_set_kernel(boute_engine *e, int d_tau, const double *params) {
+  BOUTE_TRACE();
   if (!e) return BOUTE_ERR_INVALID_ARG;
   const int r = boute_gp_set_kernel(e->gp, d_tau, params);
   engine_drop_graphs(e);  // the step's kernel choices change
   return r;
 }
 
+int boute_selftest_wait(int complete, unsigned long long limit_ns, void *stream) {
+  BOUTE_TRACE();
+  if (limit_ns > BOUTE_WAIT_NS) return BOUTE_ERR_INVALID_ARG;
+  if (int r = device_ok()) return r;
+  cudaStream_t s = (cudaStream_t)stream;
+  int *status = nullptr;
+  if (dalloc(&status, 1) != BOUTE_OK) return BOUTE_ERR_OOM;
+  int r = cudaMemsetAsync(status, 0, sizeof(int), s) == cudaSuccess ? BOUTE_OK : BOUTE_ERR_CUDA;
+  if (!r) r = launch_wait_selftest(complete, limit_ns, status, s);
+  int st = BOUTE_OK;
+  if (!r && (cudaStreamSynchronize(s) != cudaSuccess ||
+             cudaMemcpy(&st, status, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess))
+    r = last_launch_status();
+  cudaFree(status);
+  return r ? r : st;
+}
+
 int boute_base_normals(unsigned long long seed, int B, long long N, int m, int S, float *eps,
                        void *stream) {
+  BOUTE_TRACE();
   if (B < 1 || N < 0 || m < 1 || S < 1 || (N > 0 && !eps)) return BOUTE_ERR_INVALID_ARG;
   if (int r = device_ok()) return r;
   return launch_base_normals(seed, B, N, m, S, eps, (cudaStream_t)stream);
 }
 
 int boute_engine_set_normals(boute_engine *e, unsigned long long seed) {
+  BOUTE_TRACE();
   if (!e || e->mode != BOUTE_ACQ_MC_HVI) return BOUTE_ERR_INVALID_ARG;
   if (cudaDeviceSynchronize() != cudaSuccess) return last_launch_status();
   const size_t count = (size_t)e->B * e->N * e->m * e->S;
@@ -821,6 +865,7 @@ int boute_engine_set_normals(boute_engine *e, unsigned long long seed) {
 }
 
 int boute_engine_set_outcome_transforms(boute_engine *e, const int *codes) {
+  BOUTE_TRACE();
   int packed = 0;
   if (!e || !pack_codes(codes, e->m, &packed)) return BOUTE_ERR_INVALID_ARG;
   if (packed != e->tcodes) {
@@ -834,6 +879,7 @@ int boute_engine_set_outcome_transforms(boute_engine *e, const int *codes) {
 }
 
 int boute_engine_set_constraints(boute_engine *e, const double *cons) {
+  BOUTE_TRACE();
   if (!e) return BOUTE_ERR_INVALID_ARG;
   const size_t count = (size_t)e->B * e->m;
   // no step of this engine may be reading the thresholds while they change

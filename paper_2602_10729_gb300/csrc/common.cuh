@@ -151,15 +151,18 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t *bar, uint32_t phas
   return ok != 0;
 }
 
-// Waits for the given phase parity; gives up after BOUTE_WAIT_NS and returns
+// Waits for the given phase parity; gives up after limit_ns and returns
 // false so the caller can record BOUTE_ERR_TIMEOUT instead of hanging.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t phase) {
+__device__ __forceinline__ bool mbar_wait_ns(uint64_t *bar, uint32_t phase, uint64_t limit_ns) {
   if (mbar_try_wait(bar, phase)) return true;
   const uint64_t t0 = globaltimer();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, phase)) return true;
-    if ((it & 63) == 0 && globaltimer() - t0 > BOUTE_WAIT_NS) return false;
+    if ((it & 63) == 0 && globaltimer() - t0 > limit_ns) return false;
   }
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t phase) {
+  return mbar_wait_ns(bar, phase, BOUTE_WAIT_NS);
 }
 
 // Bulk copy global -> shared through the TMA engine; completion is counted

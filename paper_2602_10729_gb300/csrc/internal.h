@@ -5,6 +5,8 @@
 
 #include "common.cuh"
 
+#include <nvtx3/nvToolsExt.h>
+
 namespace boute {
 
 // The boute_gp handle: fp64 factors plus the prepacked tensor-core operands.
@@ -23,6 +25,16 @@ struct Gp {
   int kern, dtau;
   double *kpar;
 };
+
+// An NVTX range over one call of the C-ABI (visible in a profiler's timeline;
+// a few nanoseconds when no tool is attached).
+struct TraceRange {
+  explicit TraceRange(const char *name) { nvtxRangePushA(name); }
+  ~TraceRange() { nvtxRangePop(); }
+  TraceRange(const TraceRange &) = delete;
+  TraceRange &operator=(const TraceRange &) = delete;
+};
+#define BOUTE_TRACE() ::boute::TraceRange boute_trace_range_(__func__)
 
 // Every kernel of the step asks for the largest shared-memory carveout, so
 // that consecutive kernels never make an SM switch its L1 / shared split.
@@ -115,6 +127,8 @@ int launch_learn(const double *X, const double *Ys, int B, int n, int d, int m,
 // Monte-Carlo base normals from Philox4x64-10 and Box-Muller (B x N x m x S)
 int launch_base_normals(unsigned long long seed, int B, long long N, int m, int S, float *eps,
                         cudaStream_t s);
+// a bounded device-side wait that runs out unless `complete` (selftest.cu)
+int launch_wait_selftest(int complete, unsigned long long limit_ns, int *status, cudaStream_t s);
 size_t topk_scratch_bytes(int B, long long N, int k);
 // counters_zeroed: the scratch's per-problem counters are known to be zero
 // (an engine's scratch: zeroed at creation, and every call leaves them zero);

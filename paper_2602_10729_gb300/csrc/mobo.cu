@@ -16,6 +16,7 @@
 #include <vector>
 
 #include "boute.h"
+#include "internal.h"
 
 namespace {
 
@@ -74,6 +75,7 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
                               double *ls, double *s2, double *noise, double *X, double *Y, int n0,
                               boute_objective_fn f, void *user, long long *sel,
                               double *theta_hist, int *n_out, int *converged) {
+  BOUTE_TRACE();
   if (!cfg || !cand || !ref || !ls || !s2 || !noise || !X || !Y || !f || !sel || !n_out ||
       !converged || d < 1 || m < 2 || N < 1 || n0 < 1 || cfg->max_evals < n0 ||
       cfg->patience < 1 || cfg->learn_iters < 0)

@@ -62,6 +62,7 @@ using namespace boute;
 
 extern "C" int boute_select_topk_noalloc(const float *acq, int B, long long N, int k,
                                          long long *idx, float *val, void *stream) {
+  BOUTE_TRACE();
   if (!acq || !idx || !val || B < 1 || N < 1 || k < 1 || k > 1024 || k > N)
     return BOUTE_ERR_INVALID_ARG;
   if ((long long)B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;

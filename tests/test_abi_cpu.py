@@ -67,6 +67,7 @@ def test_invalid_arguments_are_rejected_before_any_device_call(lib):
         arr = (ctypes.c_int * 2)(*codes)
         assert lib.boute_standardize(p, 1, 4, 2, arr, p, None) == bt.BOUTE_ERR_INVALID_ARG
     assert lib.boute_engine_set_outcome_transforms(None, None) == bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_selftest_wait(0, 3_000_000_000, None) == bt.BOUTE_ERR_INVALID_ARG
     assert lib.boute_engine_set_kernel(None, 0, None) == bt.BOUTE_ERR_INVALID_ARG
     assert lib.boute_gp_set_kernel(None, 0, None) == bt.BOUTE_ERR_INVALID_ARG
     # hyperparameter learning: restarts, steps, step size, d_tau
