@@ -205,7 +205,8 @@ int boute_box_decompose(const double *front, const int *P, int B, int n, int m,
  *         (standardised) objectives, in the units of ref: the constrained
  *         acquisition of Sec. 5.2, E[HVI(Y) 1[Y_1 <= k_1] 1[Y_2 <= k_2]], which
  *         replaces psi_t by psi_t^c(c) = E[(c - Y_t)_+ 1[Y_t <= k_t]]; an
- *         infinite threshold constrains nothing;
+ *         infinite threshold constrains nothing; NaN is not a threshold (not
+ *         checked on the device);
  *   acq: B x N fp32. */
 int boute_acq_ehvi(const float *mean, const float *var, int B, long long N, const double *front,
                    const int *P, int n, const double *ref, const double *cons, float *acq,
@@ -349,7 +350,7 @@ int boute_engine_launches_per_step(const boute_engine *e);
 /* Constrained acquisition for the engine's later steps (Sec. 5.2,
  * "Constrained qNEHVI"): cons is a HOST array of B x m fp64 thresholds on the
  * standardised, minimised outcomes (the units of the steps' ref), copied into
- * the engine; the steps' acquisition becomes E[HVI 1[Y <= cons]] (see
+ * the engine (a NaN threshold is INVALID_ARG); the steps' acquisition becomes E[HVI 1[Y <= cons]] (see
  * boute_acq_ehvi, boute_acq_mc_hvi). cons = NULL returns to the unconstrained
  * acquisition. Waits for all work on the device first (no step may be
  * running); the engine's cached step graphs are rebuilt on the next step when

@@ -882,6 +882,8 @@ int boute_engine_set_constraints(boute_engine *e, const double *cons) {
   BOUTE_TRACE();
   if (!e) return BOUTE_ERR_INVALID_ARG;
   const size_t count = (size_t)e->B * e->m;
+  for (size_t i = 0; cons && i < count; ++i)
+    if (cons[i] != cons[i]) return BOUTE_ERR_INVALID_ARG;  // NaN: no threshold
   // no step of this engine may be reading the thresholds while they change
   if (cudaDeviceSynchronize() != cudaSuccess) return last_launch_status();
   if (cons) {

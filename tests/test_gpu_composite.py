@@ -157,3 +157,29 @@ def test_composite_engine_steps(wi, N, B):
         tol = ACQ_REL * np.maximum(np.abs(want), ACQ_FLOOR * np.abs(want).max())
         check_topk_consistent_tol(s1["idx"][b], want, w.k, tol)
         assert np.array_equal(s1["val"][b], s1["acq"][b][s1["idx"][b]])
+
+
+@pytest.mark.parametrize("dtau", [0, 6], ids=["all-deployment", "all-routing"])
+def test_composite_degenerate_splits(dtau):
+    """d_tau = 0 (no routing features: k = s2 + s2_c w w* k32 + s2_x k32) and
+    d_tau = d (no deployment features: k = (s2 + s2_x) k52 + s2_c)."""
+    w = dataclasses.replace(_variant(0, 777, 1, 40), d_tau=dtau)
+    hp = host_problem(w)
+    dc = w.d - dtau
+    rng = np.random.default_rng(12)
+    hp = dataclasses.replace(hp, d_tau=dtau,
+                             kc=np.concatenate([np.tile([0.5, 0.1, 0.05], (1, w.m, 1)),
+                                                rng.random((1, w.m, dc))], 2))
+    g = gpu_pipeline(hp)
+    assert g["status"] == 0
+    fp = oracle_fit(hp, 0)
+    mean, var = opl.posterior(fp, hp.Xc[0])
+    for t in range(w.m):
+        kern = (hp.d_tau, hp.kc[0][t])
+        prior = np.array([oracle.kernel(c, c, hp.ls[0][t], hp.s2[0][t], kern)
+                          for c in hp.Xc[0].astype(np.float64)])
+        Ks = np.array([[oracle.kernel(c, x, hp.ls[0][t], hp.s2[0][t], kern) for x in hp.X[0]]
+                       for c in hp.Xc[0].astype(np.float64)])
+        bound = 16 * EPS32 * (np.abs(Ks) @ np.abs(fp.alpha[t])) + POST_REL * np.sqrt(prior.max())
+        assert np.all(np.abs(g["mean"][0, t] - mean[:, t]) <= bound)
+        assert np.abs(g["var"][0, t] - var[:, t]).max() <= POST_REL * prior.max()
