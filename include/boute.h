@@ -350,8 +350,9 @@ int boute_engine_launches_per_step(const boute_engine *e);
 /* Constrained acquisition for the engine's later steps (Sec. 5.2,
  * "Constrained qNEHVI"): cons is a HOST array of B x m fp64 thresholds on the
  * standardised, minimised outcomes (the units of the steps' ref), copied into
- * the engine (a NaN threshold is INVALID_ARG); the steps' acquisition becomes E[HVI 1[Y <= cons]] (see
- * boute_acq_ehvi, boute_acq_mc_hvi). cons = NULL returns to the unconstrained
+ * the engine (a NaN threshold is INVALID_ARG); the steps' acquisition becomes
+ * E[HVI 1[Y <= cons]] (see boute_acq_ehvi, boute_acq_mc_hvi). cons = NULL
+ * returns to the unconstrained
  * acquisition. Waits for all work on the device first (no step may be
  * running); the engine's cached step graphs are rebuilt on the next step when
  * constraints are switched on or off. */
