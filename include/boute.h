@@ -352,10 +352,9 @@ int boute_engine_launches_per_step(const boute_engine *e);
  * standardised, minimised outcomes (the units of the steps' ref), copied into
  * the engine (a NaN threshold is INVALID_ARG); the steps' acquisition becomes
  * E[HVI 1[Y <= cons]] (see boute_acq_ehvi, boute_acq_mc_hvi). cons = NULL
- * returns to the unconstrained
- * acquisition. Waits for all work on the device first (no step may be
- * running); the engine's cached step graphs are rebuilt on the next step when
- * constraints are switched on or off. */
+ * returns to the unconstrained acquisition. Waits for all work on the device
+ * first (no step may be running); the engine's cached step graphs are rebuilt
+ * on the next step when constraints are switched on or off. */
 int boute_engine_set_constraints(boute_engine *e, const double *cons);
 /* Outcome transforms for the engine's later steps (see boute_standardize):
  * codes is a HOST array of m codes, or NULL for none. The steps' raw outcomes
