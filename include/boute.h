@@ -385,7 +385,8 @@ void boute_engine_free(boute_engine *e);
  *   f: returns 0 and writes y (m outcomes, raw: before transforms) for x
  *      (d features); a nonzero return stops the loop with INVALID_ARG.
  *   cand: HOST N x d fp32 pool; eps: HOST N x m x S fp32 base normals
- *      (mode BOUTE_ACQ_MC_HVI, reused every iteration), else NULL;
+ *      (mode BOUTE_ACQ_MC_HVI, reused every iteration), or NULL: the
+ *      engine's own normals drawn from cfg->seed (the same every iteration);
  *   ref: m reference point (standardised units); transforms: m codes or
  *      NULL; cons: m thresholds or NULL (the constrained acquisition);
  *   d_tau, kc: the composite kernel (boute_gp_set_kernel's parameters of one
@@ -410,6 +411,7 @@ typedef struct {
   int patience;     /* consecutive iterations of an unchanged Pareto set */
   int learn_iters;  /* Adam steps per iteration; 0 keeps the hyperparameters */
   double learn_lr;  /* Adam step size */
+  unsigned long long seed;  /* base normals when eps is NULL (boute_engine_set_normals) */
 } boute_mobo_config;
 int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const float *cand, long long N,
                    const float *eps, const double *ref, const int *transforms,

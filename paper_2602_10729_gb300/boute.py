@@ -47,7 +47,7 @@ class MoboConfig(ctypes.Structure):
     """boute_mobo_config."""
     _fields_ = [("mode", ctypes.c_int), ("S", ctypes.c_int), ("max_evals", ctypes.c_int),
                 ("patience", ctypes.c_int), ("learn_iters", ctypes.c_int),
-                ("learn_lr", ctypes.c_double)]
+                ("learn_lr", ctypes.c_double), ("seed", ctypes.c_ulonglong)]
 
 
 #: boute_objective_fn
@@ -227,13 +227,14 @@ def boute_gp_learn(X, Ys, theta0, iters: int, lr: float, theta, mll, grad=None, 
 
 def boute_mobo_run(objective, cand, ref, ls, s2, noise, X0, Y0, *, mode=BOUTE_ACQ_EHVI2D, S=0,
                    eps=None, max_evals=50, patience=20, learn_iters=0, learn_lr=0.05,
-                   transforms=None, cons=None, d_tau=0, kc=None):
+                   transforms=None, cons=None, d_tau=0, kc=None, seed=0):
     """The optimisation loop. objective(x: (d,) float64 array) -> m outcomes.
     cand: N x d; eps: N x m x S (mode MC); ls: m x d, s2, noise: m (initial
     hyperparameters); X0 / Y0: the first observations. Returns a dict with X,
     Y (the n observations), sel (the chosen candidate per iteration), theta
     (the log-hyperparameters of each iteration), ls, s2, noise, kc (final),
-    converged. d_tau, kc: the composite kernel (m x (3 + d - d_tau))."""
+    converged. d_tau, kc: the composite kernel (m x (3 + d - d_tau)); mode MC
+    with eps None: the engine's own normals drawn from seed."""
     import numpy as np
     cand = np.ascontiguousarray(cand, np.float32)
     N, d = cand.shape
@@ -267,7 +268,7 @@ def boute_mobo_run(objective, cand, ref, ls, s2, noise, X0, Y0, *, mode=BOUTE_AC
             return 1
 
     fn = ObjectiveFn(cb)
-    cfg = MoboConfig(mode, S, max_evals, patience, learn_iters, learn_lr)
+    cfg = MoboConfig(mode, S, max_evals, patience, learn_iters, learn_lr, int(seed))
     n_out, conv = ctypes.c_int(0), ctypes.c_int(0)
     a = lambda v: None if v is None else v.ctypes.data
     rc = load().boute_mobo_run(ctypes.byref(cfg), d, m, a(cand), N, a(eps), a(ref), a(tf), a(cs),

@@ -80,7 +80,7 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
       !converged || d < 1 || m < 2 || N < 1 || n0 < 1 || cfg->max_evals < n0 ||
       cfg->patience < 1 || cfg->learn_iters < 0)
     return BOUTE_ERR_INVALID_ARG;
-  if (cfg->mode == BOUTE_ACQ_MC_HVI && (!eps || cfg->S < 1)) return BOUTE_ERR_INVALID_ARG;
+  if (cfg->mode == BOUTE_ACQ_MC_HVI && cfg->S < 1) return BOUTE_ERR_INVALID_ARG;
   if (kc && (d_tau < 0 || d_tau > d)) return BOUTE_ERR_INVALID_ARG;
   // the composite kernel (kc: m x (3 + dc) [s2_c, s2_x, beta, s...]) adds
   // (log s2_c, log s2_x, beta) to the learned parameters
@@ -107,11 +107,11 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
   r |= dmalloc(&dmll, (size_t)m);
   if (kc) r |= dmalloc(&dpref, (size_t)m * dc);
   r |= dmalloc(&dXc, (size_t)N * d);
-  if (S) r |= dmalloc(&deps, (size_t)N * m * S);
+  if (S && eps) r |= dmalloc(&deps, (size_t)N * m * S);
   r |= dmalloc(&didx, 1);
   r |= dmalloc(&dval, 1);
   if (!r) r = copy_in(dXc, cand, sizeof(float) * N * d);
-  if (!r && S) r = copy_in(deps, eps, sizeof(float) * N * m * S);
+  if (!r && S && eps) r = copy_in(deps, eps, sizeof(float) * N * m * S);
   if (!r) r = copy_in(dref, ref, sizeof(double) * m);
   if (!r && kc) {  // the preference entries (held fixed)
     std::vector<double> pr((size_t)m * dc);
@@ -174,6 +174,7 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
     if (!r && transforms) r = boute_engine_set_outcome_transforms(e, transforms);
     if (!r && cons) r = boute_engine_set_constraints(e, cons);
     if (!r && kc) r = boute_engine_set_kernel(e, d_tau, kc);
+    if (!r && S && !eps) r = boute_engine_set_normals(e, cfg->seed);  // eps null: own normals
     if (!r) r = boute_engine_step(e, dX, dY, dls, ds2, dnz, dref, dXc, deps, didx, dval, nullptr);
     boute_engine_free(e);
     long long pick = -1;

@@ -87,11 +87,11 @@ def test_invalid_arguments_are_rejected_before_any_device_call(lib):
     assert lib.boute_mobo_run(None, 2, 2, p, 10, None, p, None, None, 0, None, p, p, p, p, p, 4,
                               fn, None, p, None, ctypes.byref(n_out),
                               ctypes.byref(conv)) == bt.BOUTE_ERR_INVALID_ARG
-    cfg = bt.MoboConfig(bt.BOUTE_ACQ_EHVI2D, 0, 3, 5, 0, 0.05)
+    cfg = bt.MoboConfig(bt.BOUTE_ACQ_EHVI2D, 0, 3, 5, 0, 0.05, 0)
     assert lib.boute_mobo_run(ctypes.byref(cfg), 2, 2, p, 10, None, p, None, None, 0, None, p, p,
                               p, p, p, 4, fn, None, p, None, ctypes.byref(n_out),
                               ctypes.byref(conv)) == bt.BOUTE_ERR_INVALID_ARG
-    cfg = bt.MoboConfig(bt.BOUTE_ACQ_MC_HVI, 0, 8, 5, 0, 0.05)  # MC without normals
+    cfg = bt.MoboConfig(bt.BOUTE_ACQ_MC_HVI, 0, 8, 5, 0, 0.05, 0)  # MC without samples
     assert lib.boute_mobo_run(ctypes.byref(cfg), 2, 2, p, 10, None, p, None, None, 0, None, p, p,
                               p, p, p, 4, fn, None, p, None, ctypes.byref(n_out),
                               ctypes.byref(conv)) == bt.BOUTE_ERR_INVALID_ARG

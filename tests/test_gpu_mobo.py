@@ -96,11 +96,13 @@ def test_loop_choices_match_oracle(learn):
     s2, noise = np.ones(2), np.full(2, 1e-4)
     mode = "mc" if learn else "ehvi"
     S = 128
-    eps = rng.standard_normal((N, 2, S), dtype=np.float32) if mode == "mc" else None
+    # Monte-Carlo: the engine's own normals from a seed, regenerated here by
+    # the oracle's implementation of the same generator
+    eps = oracle.base_normals(31, 1, N, 2, S)[0] if mode == "mc" else None
     max_evals, patience = 24, 4
     res = bt.boute_mobo_run(_objective, cand, [1.1, 1.1], ls0, s2, noise, X0, Y0,
                             mode=bt.BOUTE_ACQ_MC_HVI if mode == "mc" else bt.BOUTE_ACQ_EHVI2D,
-                            S=S if mode == "mc" else 0, eps=eps, max_evals=max_evals,
+                            S=S if mode == "mc" else 0, eps=None, seed=31, max_evals=max_evals,
                             patience=patience, learn_iters=learn[0] if learn else 0,
                             learn_lr=learn[1] if learn else 0.05)
     assert len(res["sel"]) >= patience  # converged (stable that long) or ran out of budget
