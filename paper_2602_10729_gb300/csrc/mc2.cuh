@@ -35,13 +35,14 @@ __device__ __forceinline__ float rcp_fast(float x) {
 
 // Strips of problem b into shared memory, written by `nthr` threads (thread
 // index `t`): [0] = (b_0, u_0, 0, 0), [k >= 1] = (b_k / D_k, 1 / D_k, u_k, D_k)
-// (zero width: (0, 0, u_k, 0)), then zero strips up to Kp = 1 + a multiple of
-// 4 (they add exactly nothing). lower / upper: B x box_cap x 2. Returns K.
+// (zero width: (0, 0, u_k, 0)), then at most one zero strip so that Kp = 1 + an
+// even number (it adds exactly nothing). lower / upper: B x box_cap x 2.
+// Returns K.
 __device__ __forceinline__ int mc2_load_strips(float4 *strips4, const float *lower,
                                                const float *upper, const int *Kc, int b,
                                                int box_cap, int t, int nthr) {
   const int K = Kc[b];
-  const int Kp = K > 0 ? 1 + ((K + 2) & ~3) : 0;
+  const int Kp = K > 0 ? 1 + (K & ~1) : 0;
   for (int i = t; i < Kp; i += nthr) {
     if (i >= K) {
       strips4[i] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -59,7 +60,7 @@ __device__ __forceinline__ int mc2_load_strips(float4 *strips4, const float *low
   return K;
 }
 
-__device__ __forceinline__ int mc2_padded(int K) { return K > 0 ? 1 + ((K + 2) & ~3) : 0; }
+__device__ __forceinline__ int mc2_padded(int K) { return K > 0 ? 1 + (K & ~1) : 0; }
 
 // A sample that violates a constraint contributes nothing (Sec. 5.2,
 // constrained qNEHVI: HVI times the feasibility indicator): its first
@@ -99,17 +100,22 @@ __device__ __forceinline__ float mc2_lane_sum(const float4 *strips4, int K, int 
     // height of strip k for sample j: sat(u_k / H - y2_j / H)
     const float ny2[4] = {-y2[0] * iH, -y2[1] * iH, -y2[2] * iH, -y2[3] * iH};
     float acc = 0.f;
+    auto strip = [&](const float4 t) {
+      float tk = 0.f;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        tk = fmaf(fma_sat(-y1[j], t.y, t.x), fma_sat(t.z, iH, ny2[j]), tk);
+      acc = fmaf(t.w, tk, acc);
+    };
+    int k = 1;
 #pragma unroll 1
-    for (int k = 1; k < Kp; k += 4) {
+    for (; k + 3 < Kp; k += 4) {
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float4 t = strips4[k + q];
-        float tk = 0.f;
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-          tk = fmaf(fma_sat(-y1[j], t.y, t.x), fma_sat(t.z, iH, ny2[j]), tk);
-        acc = fmaf(t.w, tk, acc);
-      }
+      for (int q = 0; q < 4; ++q) strip(strips4[k + q]);
+    }
+    if (k < Kp) {  // Kp - 1 is even: two strips remain
+      strip(strips4[k]);
+      strip(strips4[k + 1]);
     }
     sum = fmaf(fmaxf(H, 0.f), acc, sum);
   }
