@@ -257,7 +257,7 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
 // Threads per block of the two variants: the shared-memory variant runs more
 // warps to hide the latency of its short, dependent phases.
 template <bool SMEM>
-constexpr int fit_threads() { return SMEM ? 384 : 256; }
+constexpr int fit_threads() { return SMEM ? 512 : 256; }
 
 template <bool SMEM>
 __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
@@ -364,9 +364,11 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
       if (kl_smem) mbar_wait(&lbar_lo, 0);
       return;
     }
-    for (int e = tid; e < n * n; e += nthr) {
-      const int i = e / n, k = e - i * n;
-      A[(size_t)i * ld + k] = W[e];
+    for (int i = warp; i < n; i += nw) {  // a warp per row: no division per entry
+      const float *src = W + (size_t)i * n;
+      float *dst = A + (size_t)i * ld;
+#pragma unroll 4
+      for (int k = lane; k < n; k += 32) dst[k] = src[k];
     }
     __syncthreads();
   }
@@ -601,8 +603,63 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     return;
   }
   // ---- alpha0 = W^T (W y), refined once against K = hi + lo ----------------------
-  // out = W^T (W rhs): thread per row, then thread per column (4 accumulators)
+  // out = W^T (W rhs). Shared-memory variant: the 32 x 32 blocks (I >= J) of
+  // W, one warp per block (the diagonal blocks hold zeros above the diagonal,
+  // the padding the identity), with the block partial sums in the space of
+  // colL (free after the factorisation), added in a fixed order.
+  auto solve_blocks = [&](const float *rhs, float *out) {
+    float *pw = &colL[0][0], *pt = pw + nb * NP;  // nb x NP each (nb <= 5, NP <= 160)
+    const int nblk = nb * (nb + 1) / 2;
+    auto block = [&](int e, int &I, int &J) {
+      I = 0;
+      while ((I + 1) * (I + 2) / 2 <= e) ++I;
+      J = e - I * (I + 1) / 2;
+    };
+    for (int e = warp; e < nblk; e += nw) {  // (W rhs) restricted to block (I, J): lane = row
+      int I, J;
+      block(e, I, J);
+      const float *wr = W + (size_t)(32 * I + lane) * ld + 32 * J;
+      const float *x = rhs + 32 * J;
+      float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+      for (int k = 0; k < 32; k += 4) {
+        s0 = fmaf(wr[k], x[k], s0);
+        s1 = fmaf(wr[k + 1], x[k + 1], s1);
+        s2 = fmaf(wr[k + 2], x[k + 2], s2);
+        s3 = fmaf(wr[k + 3], x[k + 3], s3);
+      }
+      pw[J * NP + 32 * I + lane] = (s0 + s1) + (s2 + s3);
+    }
+    __syncthreads();
+    for (int e = warp; e < nblk; e += nw) {  // W^T (W rhs) restricted to block (I, J): lane = column
+      int I, J;
+      block(e, I, J);
+      float v = 0.f;  // (W rhs) of row 32 I + lane
+      for (int q = 0; q <= I; ++q) v += pw[q * NP + 32 * I + lane];
+      const float *wc = W + (size_t)(32 * I) * ld + 32 * J + lane;
+      float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+      for (int r = 0; r < 32; r += 4) {
+        s0 = fmaf(wc[(size_t)r * ld], __shfl_sync(FULL, v, r), s0);
+        s1 = fmaf(wc[(size_t)(r + 1) * ld], __shfl_sync(FULL, v, r + 1), s1);
+        s2 = fmaf(wc[(size_t)(r + 2) * ld], __shfl_sync(FULL, v, r + 2), s2);
+        s3 = fmaf(wc[(size_t)(r + 3) * ld], __shfl_sync(FULL, v, r + 3), s3);
+      }
+      pt[I * NP + 32 * J + lane] = (s0 + s1) + (s2 + s3);
+    }
+    __syncthreads();
+    for (int k = tid; k < NP; k += nthr) {
+      float v = 0.f;
+      for (int q = k >> 5; q < nb; ++q) v += pt[q * NP + k];
+      out[k] = v;
+    }
+    __syncthreads();
+  };
+  // global variant: thread per row, then thread per column (4 accumulators)
   auto solve = [&](const float *rhs, float *out) {
+    if constexpr (SMEM) {
+      solve_blocks(rhs, out);
+    } else {
     for (int i = tid; i < NP; i += nthr) {
       const float *wr = W + (size_t)i * ld;
       float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
@@ -630,6 +687,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
       out[k] = (s0 + s1) + (s2 + s3);
     }
     __syncthreads();
+    }
   };
   solve(yv, al);
   if (lo_copy && !mbar_wait(&lbar_lo, 0)) {  // the copy never completed: report, drain, leave
@@ -637,33 +695,72 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     mbar_wait(&lbar_lo, 0);
     return;
   }
-  // residual r = y - K alpha0 in double-float. Shared-memory variant: K hi
-  // from the upper triangle of A and its diagonal, K lo from shared memory
-  // when it fits there; half a warp per row.
+  // residual r = y - K alpha0 in double-float. Shared-memory variant: one
+  // warp per 32 x 32 block (I, J) of K, lane = row, two independent chains per
+  // lane; K lo through its symmetry (K lo[k][i], conflict-free across the
+  // lanes), from shared memory when it fits there; K hi from the upper
+  // triangle of A: at (k, i) below the diagonal blocks, at (i, k) above them,
+  // each with one fixed load form (a per-entry choice of address costs more
+  // than the arithmetic), and in the diagonal blocks both loaded and the
+  // value selected, the diagonal from dg. Indices past n are clamped and
+  // alpha is zero there (padding), so those terms add exact zeros. The block
+  // partial sums (hi, lo) go to the space of colL and are added per row in a
+  // fixed order.
   if (SMEM) {
-    const int half = lane >> 4, hl = lane & 15;
-    for (int i = 2 * warp + half; i < NP; i += 2 * nw) {  // NP: both halves, same trips
+    float *ph = &colL[0][0], *pl = ph + nb * NP;  // nb x NP each
+    const float *Klsm = vec + 6 * NP;  // = Kls when kl_smem (shared-space pointer)
+    for (int e = warp; e < nb * nb; e += nw) {
+      const int I = e / nb, J = e - I * nb, ci = min(32 * I + lane, n - 1);
+      const float *alJ = al + 32 * J;
+      float sh[2] = {0.f, 0.f}, sl[2] = {0.f, 0.f};
+      auto run = [&](auto form, auto lo_smem) {
+        constexpr int F = decltype(form)::value;  // 0: below, 1: above, 2: diagonal block
+        constexpr bool LS = decltype(lo_smem)::value;
+        const float di = dg[ci];
+#pragma unroll 8
+        for (int kk = 0; kk < 32; ++kk) {
+          const int kc = min(32 * J + kk, n - 1);
+          float h;
+          if (F == 0) {
+            h = A[kc * ld + ci];
+          } else if (F == 1) {
+            h = A[ci * ld + kc];
+          } else {
+            const float x = A[kc * ld + ci], y = A[ci * ld + kc];
+            h = kc < ci ? x : y;
+            h = kc == ci ? di : h;
+          }
+          const float l = LS ? Klsm[kc * n + ci] : Kl[(size_t)kc * n + ci];
+          const float a = alJ[kk];  // zero from n on
+          float pr, er, s_, e2;
+          two_prod(h, a, pr, er);
+          two_sum(sh[kk & 1], pr, s_, e2);
+          sh[kk & 1] = s_;
+          sl[kk & 1] += e2 + fmaf(l, a, er);
+        }
+      };
+      auto pick = [&](auto lo_smem) {
+        if (I > J) run(std::integral_constant<int, 0>{}, lo_smem);
+        else if (I < J) run(std::integral_constant<int, 1>{}, lo_smem);
+        else run(std::integral_constant<int, 2>{}, lo_smem);
+      };
+      if (kl_smem) pick(std::true_type{});
+      else pick(std::false_type{});
+      float s_, e2;
+      two_sum(sh[0], sh[1], s_, e2);
+      ph[J * NP + 32 * I + lane] = s_;
+      pl[J * NP + 32 * I + lane] = (sl[0] + sl[1]) + e2;
+    }
+    __syncthreads();
+    for (int i = tid; i < NP; i += nthr) {
       float sh = 0.f, sl = 0.f;
-      for (int k = hl; k < (i < n ? n : 0); k += 16) {
-        const float h = k < i ? A[(size_t)k * ld + i] : (k > i ? A[(size_t)i * ld + k] : dg[i]);
-        const float l = kl_smem ? Kls[(size_t)i * n + k] : Kl[(size_t)i * n + k];
-        const float a = al[k];
-        float pr, e, s_, e2;
-        two_prod(h, a, pr, e);
-        two_sum(sh, pr, s_, e2);
+      for (int J = 0; J < nb; ++J) {
+        float s_, e2;
+        two_sum(sh, ph[J * NP + i], s_, e2);
         sh = s_;
-        sl += e2 + fmaf(l, a, e);
+        sl += pl[J * NP + i] + e2;
       }
-#pragma unroll
-      for (int o = 8; o > 0; o >>= 1) {  // within the half warp
-        const float oh = __shfl_xor_sync(FULL, sh, o);
-        const float ol = __shfl_xor_sync(FULL, sl, o);
-        float s_, e;
-        two_sum(sh, oh, s_, e);
-        sh = s_;
-        sl += ol + e;
-      }
-      if (hl == 0 && i < n) rv[i] = (yv[i] - sh) + (ylo[i] - sl);
+      if (i < n) rv[i] = (yv[i] - sh) + (ylo[i] - sl);
     }
   } else {
     // global variant: two rows per half warp at a time, all their loads

@@ -65,7 +65,7 @@ def test_ragged_candidate_counts(N):
     compare(rand_problem(1, 20, 4, 2, N))
 
 
-@pytest.mark.parametrize("n", [1, 2, 31, 33, 255, 257, 600])
+@pytest.mark.parametrize("n", [1, 2, 31, 33, 97, 129, 150, 160, 161, 255, 257, 600])
 def test_training_set_sizes_and_column_passes(n):
     compare(rand_problem(2, n, 5, 2, 400))
 
