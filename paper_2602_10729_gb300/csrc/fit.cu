@@ -408,7 +408,8 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   // block column p of W, and T_pJ = sum_{K=J}^{p-1} L_pK W_KJ (J < p) is
   // parked, transposed, in the unused upper triangle of W; (c) the trailing
   // update A_ij -= sum_q L_iq L_jq (rows and columns below the panel), the
-  // copy of the panel into A, and W_pJ = -W_pp T_pJ. 4 x 4 register tiles.
+  // copy of the panel into A, and W_pJ = -W_pp T_pJ. 4 x 4 register tiles (4 x 2
+  // for T_pJ and W_pJ).
   const int nb = NP / 32;
   const unsigned FULL = 0xffffffffu;
   for (int p = 0; p < nb; ++p) {
@@ -494,7 +495,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     const int r0 = p0 + 32, rows = NP - r0;
     // (b)
     {
-      const int ntr = (rows / 4) * 8, ntt = p * 64;
+      const int ntr = (rows / 4) * 8, ntt = p * 128;
       for (int tix = tid; tix < ntr + ntt; tix += nthr) {
         float acc[4][4] = {};
         if (tix < ntr) {  // L_rp tile: rows i0.., columns c0.. of the panel
@@ -516,32 +517,34 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
           for (int u = 0; u < 4; ++u)
 #pragma unroll
             for (int v = 0; v < 4; ++v) W[(size_t)(i0 + u) * ld + p0 + c0 + v] = acc[u][v];
-        } else {  // T_pJ tile (8 x 8 tiles per 32 x 32 block)
-          const int e = tix - ntr, J = e >> 6, rb = 4 * ((e >> 3) & 7), cb = 4 * (e & 7);
+        } else {
+          // T_pJ tile of 4 rows x 2 columns (8 x 16 tiles per 32 x 32 block):
+          // the sums run over 32 (p - J) terms, so the long ones get twice
+          // the threads that 4 x 4 tiles would give them
+          const int e = tix - ntr, J = e >> 7, rb = 4 * ((e >> 4) & 7), cb = 2 * (e & 15);
 #pragma unroll 4
           for (int q = 32 * J; q < p0; ++q) {
-            float x[4], y4[4];
+            float x[4], y2[2];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              x[u] = A[(size_t)(p0 + rb + u) * ld + q];
-              y4[u] = W[(size_t)q * ld + 32 * J + cb + u];
-            }
+            for (int u = 0; u < 4; ++u) x[u] = A[(size_t)(p0 + rb + u) * ld + q];
+#pragma unroll
+            for (int v = 0; v < 2; ++v) y2[v] = W[(size_t)q * ld + 32 * J + cb + v];
 #pragma unroll
             for (int u = 0; u < 4; ++u)
 #pragma unroll
-              for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
+              for (int v = 0; v < 2; ++v) acc[u][v] = fmaf(x[u], y2[v], acc[u][v]);
           }
 #pragma unroll
           for (int u = 0; u < 4; ++u)
 #pragma unroll
-            for (int v = 0; v < 4; ++v) W[(size_t)(32 * J + cb + v) * ld + p0 + rb + u] = acc[u][v];
+            for (int v = 0; v < 2; ++v) W[(size_t)(32 * J + cb + v) * ld + p0 + rb + u] = acc[u][v];
         }
       }
     }
     __syncthreads();
     // (c)
     {
-      const int th = rows / 4, ntile = th * (th + 1) / 2, nwt = p * 64;
+      const int th = rows / 4, ntile = th * (th + 1) / 2, nwt = p * 128;
       for (int tix = tid; tix < ntile + nwt; tix += nthr) {
         float acc[4][4] = {};
         if (tix < ntile) {  // trailing tile (i, j) of the lower triangle
@@ -568,25 +571,24 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
 #pragma unroll
             for (int v = 0; v < 4; ++v)
               if (ti != tj || v <= u) A[(size_t)(i0 + u) * ld + j0 + v] -= acc[u][v];
-        } else {  // W_pJ tile = -W_pp T_pJ (W_pp lower, zeros above)
-          const int e = tix - ntile, J = e >> 6, rb = 4 * ((e >> 3) & 7), cb = 4 * (e & 7);
+        } else {  // W_pJ tile = -W_pp T_pJ (W_pp lower, zeros above), 4 rows x 2 columns
+          const int e = tix - ntile, J = e >> 7, rb = 4 * ((e >> 4) & 7), cb = 2 * (e & 15);
 #pragma unroll 4
           for (int q = 0; q < 32; ++q) {
-            float x[4], y4[4];
+            float x[4], y2[2];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              x[u] = W[(size_t)(p0 + rb + u) * ld + p0 + q];
-              y4[u] = W[(size_t)(32 * J + cb + u) * ld + p0 + q];
-            }
+            for (int u = 0; u < 4; ++u) x[u] = W[(size_t)(p0 + rb + u) * ld + p0 + q];
+#pragma unroll
+            for (int v = 0; v < 2; ++v) y2[v] = W[(size_t)(32 * J + cb + v) * ld + p0 + q];
 #pragma unroll
             for (int u = 0; u < 4; ++u)
 #pragma unroll
-              for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
+              for (int v = 0; v < 2; ++v) acc[u][v] = fmaf(x[u], y2[v], acc[u][v]);
           }
 #pragma unroll
           for (int u = 0; u < 4; ++u)
 #pragma unroll
-            for (int v = 0; v < 4; ++v) W[(size_t)(p0 + rb + u) * ld + 32 * J + cb + v] = -acc[u][v];
+            for (int v = 0; v < 2; ++v) W[(size_t)(p0 + rb + u) * ld + 32 * J + cb + v] = -acc[u][v];
         }
       }
       for (int e = tid; e < rows * 32; e += nthr) {  // the panel into A
