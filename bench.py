@@ -4,7 +4,9 @@
 One step = one pass of the whole scoring path over one batch of synthetic
 input: standardise -> GP fit -> Pareto front (-> boxes) -> posterior ->
 acquisition -> top-k, launched by the C-ABI engine on one stream, inputs
-resident in HBM. Metric: candidates scored per second (whole job).
+resident in HBM. Metric: candidates scored per second (whole job). The
+default workload is the largest single-GPU one, the 3-objective Monte-Carlo
+step (n = 1024, d = 24, N = 4 Mi, S = 256).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
     python bench.py --impl reference ...   # the CPU oracle on the same workload
@@ -12,13 +14,19 @@ resident in HBM. Metric: candidates scored per second (whole job).
 Under torchrun each rank scores its own replica of the workload on its own
 GPU (no collective on the data path; weak scaling); rank 0 prints one JSON
 line. Between timed steps the L2 is flushed (a 512 MB write outside the
-timed events). The `e2e` object times a stream of steps through the
-pipelined host-buffer call (boute_engine_step_host_async): every step copies
-its inputs in from pinned host memory and its selection out, and one step's
-copies overlap the previous step's computation. Monte-Carlo workloads there
-use the engine's own base normals, drawn once on the device from a seed
-(fixed base samples, as an optimisation loop keeps them), so a step's inputs
-are its observations, hyperparameters and candidates.
+timed events). During the timed steps the engine records live stage events
+(its normal concurrent schedule, events on the step's stream only), from
+which the scoring pass (posterior + acquisition + top-k) and the dominant
+kernel are timed for the `roofline` object.
+
+The `e2e` object times a stream of steps through the pipelined host-buffer
+call (boute_engine_step_host_async): every step copies its inputs in from
+pinned host memory and its selection out, and one step's copies overlap the
+previous step's computation. Its value has the Monte-Carlo base normals
+passed in as data with every step (copied from the host); `device_normals`
+beside it is the same stream of steps with the engine's own base normals,
+drawn once on the device from a seed and held fixed, as an optimisation loop
+keeps them.
 """
 from __future__ import annotations
 
@@ -39,12 +47,16 @@ sys.path.insert(0, ROOT)
 
 from paper_2602_10729_gb300 import workloads as wl  # noqa: E402
 
-DEFAULT_WORKLOAD = wl.WORKLOADS[1].name
+DEFAULT_WORKLOAD = wl.WORKLOADS[3].name
 METRIC = "candidates scored/sec (GP posterior + EHVI) at 1 GB300; % of roofline"
 UNIT = "candidates/s"
-# nominal dense tensor throughput ratio tf32 : bf16 (1.1 : 2.25 PFLOP/s)
-TF32_PER_BF16 = 1.1 / 2.25
+# The posterior contraction's operand type and products per algorithmic
+# product: tf32 hi/lo operands, three tcgen05.mma per product (hi*hi + hi*lo +
+# lo*hi). Its peak is the measured bf16 peak times the nominal dense ratio of
+# the operand type to bf16 (tf32 1.1 : 2.25 PFLOP/s).
+CONTRACTION = {"dtype": "tf32", "products": 3, "per_bf16": 1.1 / 2.25}
 NUM_SMS = 152
+FMA_LANES_PER_SM = 128
 
 
 def peaks():
@@ -57,14 +69,17 @@ def peaks():
 
 
 # ---------------------------------------------------------------- inputs
-def host_inputs(w: wl.Workload, threads: int = 16):
+def host_inputs(w: wl.Workload, threads: int = 16, count: int | None = None):
+    """The workload's inputs on the host; count: only the first `count`
+    candidates (and their normals) of each problem."""
+    count = w.N if count is None else min(count, w.N)
     X, Y, L, S2, NZ = [], [], [], [], []
     for b in range(w.B):
         x, y = wl.training_set(w, b)
         ls, s2, nz = wl.hyperparameters(w, b)
         X.append(x); Y.append(y); L.append(ls); S2.append(s2); NZ.append(nz)
-    Xc = np.stack([wl.candidates(w, b, 0, w.N, threads) for b in range(w.B)])
-    eps = (np.stack([wl.base_normals(w, b, 0, w.N, threads) for b in range(w.B)])
+    Xc = np.stack([wl.candidates(w, b, 0, count, threads) for b in range(w.B)])
+    eps = (np.stack([wl.base_normals(w, b, 0, count, threads) for b in range(w.B)])
            if w.mode == "mc" else None)
     ref = np.tile(wl.ref_point(w), (w.B, 1))
     kc = np.stack([wl.kernel_params(w, b)[1] for b in range(w.B)]) if w.d_tau else None
@@ -118,44 +133,78 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- roofline
-def roofline(w: wl.Workload, stage: str, ms: float, hbm, bf16):
-    """Algorithmic work of one launch of the stage's dominant kernel."""
+def tensor_peak(bf16_tflops: float) -> float:
+    """Effective dense peak of the posterior contraction in algorithmic
+    TFLOP/s: the operand type's peak (measured bf16 x nominal ratio) divided
+    by the tensor-core products issued per algorithmic product."""
+    return bf16_tflops * CONTRACTION["per_bf16"] / CONTRACTION["products"]
+
+
+def contraction_flops(w: wl.Workload) -> float:
+    """Algorithmic flops of the posterior: V = K* (L^-1)^T over the lower
+    triangle (n(n+1)/2 multiply-adds per candidate and objective) and the mean
+    K* alpha (n multiply-adds)."""
+    return float(w.B) * w.N * w.m * (w.n * (w.n + 1) + 2 * w.n)
+
+
+def pass_bytes(w: wl.Workload) -> float:
+    """HBM bytes the scoring pass must move per step: each candidate's
+    coordinates (4d), its base normals (4mS, Monte-Carlo) and its score (4)."""
+    per = 4 * w.d + (4 * w.m * w.S if w.mode == "mc" else 0) + 4
+    return float(w.B) * w.N * per
+
+
+def stage_roofline(w: wl.Workload, stage: str, ms: float, hbm, tens, sm_mhz):
+    """Roofline of one stage's kernel from its algorithmic work per launch and
+    its measured duration (ms)."""
     B, n, d, m, N, S = w.B, w.n, w.d, w.m, w.N, w.S
     if stage == "posterior":
-        # triangular L^-1 contraction (n(n+1)/2 MACs) plus the mean column (n MACs)
-        flops = B * N * m * (n * (n + 1) + 2 * n)
-        peak = bf16 * TF32_PER_BF16
-        return dict(bound="tensor", achieved=flops / (ms * 1e-3) / 1e12, peak=peak,
+        flops = contraction_flops(w)
+        return dict(bound="tensor", achieved=flops / (ms * 1e-3) / 1e12, peak=tens,
                     unit="TFLOP/s", per_launch=flops, kernel="posterior_kernel")
-    if stage == "acquisition" and w.mode == "mc":
-        byts = B * N * (m * S * 4 + 2 * m * 4 + 4)
-        return dict(bound="hbm", achieved=byts / (ms * 1e-3) / 1e9, peak=hbm, unit="GB/s",
-                    per_launch=byts, kernel="mchvi2_kernel" if m == 2 else "mchvi_kernel")
     if stage == "acquisition":
-        byts = B * N * (2 * m * 4 + 4)
+        per = (m * S * 4 if w.mode == "mc" else 0) + 2 * m * 4 + 4
+        byts = float(B) * N * per
+        kern = ("ehvi2d_kernel" if w.mode != "mc" else
+                "mchvi2_kernel" if m == 2 else "mchvi_kernel")
         return dict(bound="hbm", achieved=byts / (ms * 1e-3) / 1e9, peak=hbm, unit="GB/s",
-                    per_launch=byts, kernel="ehvi2d_kernel")
+                    per_launch=byts, kernel=kern)
     if stage == "topk":
-        byts = B * N * 4
+        byts = float(B) * N * 4
         return dict(bound="hbm", achieved=byts / (ms * 1e-3) / 1e9, peak=hbm, unit="GB/s",
                     per_launch=byts,
                     kernel="warp_topk_kernel" if w.k <= 32 else "segment_topk_kernel")
-    if stage == "fit":
-        # Cholesky n^3/3 + triangular inverse n^3/3 flops per (problem,
-        # objective), fp32 on the CUDA cores of the SMs the fit occupies (one
-        # block per problem-objective): 128 FMA lanes x 2 flops x 2.07 GHz each
-        flops = B * m * 2 * n ** 3 / 3
-        peak = min(B * m, NUM_SMS) * 128 * 2 * 2.07e9 / 1e12
-        return dict(bound="alu", achieved=flops / (ms * 1e-3) / 1e12, peak=peak,
-                    unit="TFLOP/s", per_launch=flops, kernel="fit32_kernel")
-    byts = B * n * m * 8
-    return dict(bound="hbm", achieved=byts / (ms * 1e-3) / 1e9, peak=hbm, unit="GB/s",
-                per_launch=byts, kernel=stage)
+    # the fit: Cholesky n^3/3 + triangular inverse n^3/3 flops per (problem,
+    # objective) in fp32 on the CUDA cores, against the whole GPU's FP32 FMA
+    # peak at the clock measured during the run
+    flops = float(B) * m * 2 * n ** 3 / 3
+    peak = NUM_SMS * FMA_LANES_PER_SM * 2 * (sm_mhz or 2070.0) * 1e6 / 1e12
+    return dict(bound="alu", achieved=flops / (ms * 1e-3) / 1e12, peak=peak, unit="TFLOP/s",
+                per_launch=flops, kernel="fit32_kernel")
 
 
-def profiled_traffic(kernel: str, workload: str):
+def pass_roofline(w: wl.Workload, ms_pass: float, hbm, tens, tens_tf32):
+    """The scoring pass (posterior + acquisition + top-k) against its
+    roofline, the slower of the tensor bound (algorithmic contraction flops at
+    the contraction's effective peak) and the HBM bound (pass_bytes)."""
+    t_tensor = contraction_flops(w) / (tens * 1e12) * 1e3
+    t_tf32 = contraction_flops(w) / (tens_tf32 * 1e12) * 1e3
+    t_hbm = pass_bytes(w) / (hbm * 1e9) * 1e3
+    t_roof = max(t_tensor, t_hbm)
+    return {"ms": ms_pass, "bound": "tensor" if t_tensor >= t_hbm else "hbm",
+            "t_tensor_ms": t_tensor, "t_hbm_ms": t_hbm, "t_roof_ms": t_roof,
+            "frac": t_roof / ms_pass,
+            "frac_vs_tf32_over_3": max(t_tf32, t_hbm) / ms_pass,
+            "contraction": dict(CONTRACTION)}
+
+
+def profiled_traffic(kernel: str, workload: str, candidates: int):
     """dram bytes per launch from the committed ncu summary of this kernel and
-    workload, if that summary was taken on the current kernel source."""
+    workload, if that summary was taken on the current kernel source. A
+    summary captured on fewer candidates than the workload's (its
+    `captured_candidates`) is scaled to `candidates` in proportion: the
+    kernel's DRAM traffic is per candidate (coordinates and normals in,
+    results out) plus operands that stay in L2."""
     path = os.path.join(ROOT, "profiles", f"{kernel}__{workload}.md")
     if not os.path.exists(path):
         return None
@@ -169,7 +218,9 @@ def profiled_traffic(kernel: str, workload: str):
         h = hashlib.sha256(open(os.path.join(ROOT, src.group(1)), "rb").read()).hexdigest()
         if not h.startswith(ms.group(1)):
             return None
-    return float(mt.group(1))
+    cap = re.search(r"captured_candidates\s*[:=]\s*([0-9]+)", txt)
+    scale = candidates / float(cap.group(1)) if cap else 1.0
+    return float(mt.group(1)) * scale
 
 
 # ---------------------------------------------------------------- ranks
@@ -189,25 +240,34 @@ def whole_job_rate(world: int, w: wl.Workload, seconds: float) -> float:
 
 
 # ---------------------------------------------------------------- CPU oracle
-def oracle_rate(w: wl.Workload, inp, budget_s: float, threads: int = 0, cons=None):
+# candidates of each problem generated for the CPU legs (a bounded sample)
+CPU_PREFIX = 1 << 18
+
+
+def oracle_rate(w: wl.Workload, inp, budget_s: float, threads: int = 0, cons=None,
+                sample: int | None = None):
     """The oracle's scoring step (fit, front, posterior, acquisition, top-k)
-    on problem 0 over a candidate sample sized to about budget_s seconds
-    (cons: the thresholds of a constrained acquisition, or None)."""
+    on problem 0 over a candidate sample sized to about budget_s seconds (or
+    `sample` candidates) of the ones in inp (cons: the thresholds of a
+    constrained acquisition, or None)."""
     import oracle
     from oracle import pipeline as opl
     threads = threads or oracle.default_threads()
     kern = None if inp["kc"] is None else (w.d_tau, inp["kc"][0])
     tfs = list(w.transforms) or None
-    t0 = time.perf_counter()
-    fp = opl.fit_problem(inp["X"][0], inp["Y"][0], inp["ls"][0], inp["s2"][0], inp["noise"][0],
-                         inp["ref"][0], kernel=kern, transforms=tfs)
-    fit_s = time.perf_counter() - t0
-    n_try = min(w.N, 2048)
-    t0 = time.perf_counter()
-    opl.score(fp, inp["Xc"][0, :n_try], w.mode, min(w.k, n_try),
-              None if inp["eps"] is None else inp["eps"][0, :n_try], threads, cons=cons)
-    per = (time.perf_counter() - t0) / n_try
-    sample = int(max(n_try, min(w.N, (budget_s - fit_s) / max(per, 1e-9))))
+    avail = inp["Xc"].shape[1]
+    if sample is None:
+        t0 = time.perf_counter()
+        fp = opl.fit_problem(inp["X"][0], inp["Y"][0], inp["ls"][0], inp["s2"][0],
+                             inp["noise"][0], inp["ref"][0], kernel=kern, transforms=tfs)
+        fit_s = time.perf_counter() - t0
+        n_try = min(avail, 2048)
+        t0 = time.perf_counter()
+        opl.score(fp, inp["Xc"][0, :n_try], w.mode, min(w.k, n_try),
+                  None if inp["eps"] is None else inp["eps"][0, :n_try], threads, cons=cons)
+        per = (time.perf_counter() - t0) / n_try
+        sample = int(max(n_try, min(avail, (budget_s - fit_s) / max(per, 1e-9))))
+    sample = min(sample, avail)
     t0 = time.perf_counter()
     fp = opl.fit_problem(inp["X"][0], inp["Y"][0], inp["ls"][0], inp["s2"][0], inp["noise"][0],
                          inp["ref"][0], kernel=kern, transforms=tfs)
@@ -218,14 +278,15 @@ def oracle_rate(w: wl.Workload, inp, budget_s: float, threads: int = 0, cons=Non
 
 
 def run_reference(args, w):
-    inp = host_inputs(w)
+    inp = host_inputs(w, count=CPU_PREFIX)
     import oracle
     threads = oracle.default_threads()
     per_step_budget = max(0.5, 150.0 / max(1, args.steps + args.warmup))
     times, samples = [], []
-    for i in range(args.warmup + args.steps):
-        rate, thr, sample, dt = oracle_rate(w, inp, per_step_budget, threads, args.cons)
-        if i >= args.warmup:
+    sample = None  # sized on the first (warm-up) step, then held fixed
+    for i in range(max(1, args.warmup) + args.steps):
+        rate, thr, sample, dt = oracle_rate(w, inp, per_step_budget, threads, args.cons, sample)
+        if i >= max(1, args.warmup):
             times.append(dt)
             samples.append(sample)
     total = sum(samples)
@@ -250,11 +311,14 @@ def run_reference(args, w):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=2000)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=0,
+                    help="timed steps (0: as many as take about 10 s, 20 to 2000)")
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-serial-stages", action="store_true",
+                    help="skip the serialised per-stage breakdown")
     ap.add_argument("--e2e-steps", type=int, default=0, help="0: same as --steps (max 200)")
     ap.add_argument("--constraints", default="",
                     help="comma-separated thresholds on the standardised, minimised objectives "
@@ -268,6 +332,8 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", 1))
     local = int(os.environ.get("LOCAL_RANK", 0))
     if args.impl == "reference":
+        if not args.steps:
+            args.steps = 20
         if rank == 0:
             run_reference(args, w)
         return
@@ -304,9 +370,21 @@ def main():
     torch.cuda.set_stream(stream)
     flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
 
+    # live stage events in the timed steps (the normal concurrent schedule)
+    bt.boute_engine_set_timing(e, bt.TIMING_LIVE)
     for _ in range(max(3, args.warmup)):
+        flush.zero_()
         bt.boute_engine_step(e, *args_dev)
     torch.cuda.synchronize()
+    if not args.steps:  # about 10 s of timed steps
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        bt.boute_engine_step_async(e, *args_dev)
+        a1.record(stream)
+        torch.cuda.synchronize()
+        args.steps = int(max(20, min(2000, 10.0 / max(a0.elapsed_time(a1) * 1e-3, 1e-6))))
+        if dist:  # every rank times the same number of steps
+            args.steps = int(max_over_ranks(args.steps, dist, dev))
 
     def barrier():
         if dist:
@@ -314,6 +392,7 @@ def main():
 
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(args.steps)]
+    live = {s_: 0.0 for s_ in bt.STAGES}
     clocks = ClockSampler(torch.cuda.current_device()) if rank == 0 else None
     barrier()
     torch.cuda.synchronize()
@@ -324,75 +403,105 @@ def main():
         ev[i][0].record(stream)
         bt.boute_engine_step_async(e, *args_dev)
         ev[i][1].record(stream)
+        # this step's stage events (read before the next step records them;
+        # the wait falls between the step's events, outside its device time)
+        for s_, v in bt.boute_engine_stage_times(e).items():
+            live[s_] += v
     torch.cuda.synchronize()
     barrier()
     wall = time.perf_counter() - wall0
     launches = bt.boute_launch_count() - l0
     clk = clocks.stop() if clocks else None
+    bt.boute_engine_set_timing(e, False)
     bt.boute_engine_step(e, *args_dev)  # synchronising step: raises on any recorded device error
     ms = sum(a.elapsed_time(b) for a, b in ev) / args.steps
     ms_max = max_over_ranks(ms, dist, dev)
     value = whole_job_rate(world, w, ms_max * 1e-3)
+    live = {s_: v / args.steps for s_, v in live.items()}
+    live.pop("front", None)  # (beside the fit in the normal schedule)
 
-    # ---- per-stage breakdown: separate steps with stage events (front stage
-    # serialised after the fit so that the stages add up) -----------------------
-    bt.boute_engine_set_timing(e, True)
-    n_stage = min(args.steps, 200)
-    stage_ms = {s: 0.0 for s in bt.STAGES}
-    for i in range(n_stage + 3):
-        flush.zero_()
-        bt.boute_engine_step_async(e, *args_dev)
-        if i >= 3:
-            for s, v in bt.boute_engine_stage_times(e).items():
-                stage_ms[s] += v
-    stage_ms = {s: v / n_stage for s, v in stage_ms.items()}
-    bt.boute_engine_set_timing(e, False)
+    # ---- serialised per-stage breakdown: separate steps with stage events
+    # (front stage after the fit, K* built inside the posterior, selection as
+    # a launch of its own) so that the stages add up ---------------------------
+    stage_ms = None
+    if not args.no_serial_stages:
+        bt.boute_engine_set_timing(e, bt.TIMING_SERIAL)
+        n_stage = min(args.steps, 20)
+        stage_ms = {s_: 0.0 for s_ in bt.STAGES}
+        for i in range(n_stage + 3):
+            flush.zero_()
+            bt.boute_engine_step_async(e, *args_dev)
+            if i >= 3:
+                for s_, v in bt.boute_engine_stage_times(e).items():
+                    stage_ms[s_] += v
+        stage_ms = {s_: v / n_stage for s_, v in stage_ms.items()}
+        bt.boute_engine_set_timing(e, False)
+    del deps  # (the resident normals are not needed by the host-input steps)
+    args_dev = None
 
     # ---- end to end through the public API with host buffers ----------------
     pin = lambda a, dt: None if a is None else torch.as_tensor(a, dtype=dt).pin_memory()
     hX, hY, hls, hs2, hnz, href = (pin(inp[k], f64) for k in ("X", "Y", "ls", "s2", "noise", "ref"))
     hXc = pin(inp["Xc"], f32)
-    # Monte-Carlo steps: fixed base normals drawn once on the device from a
-    # seed (the engine's own), as an optimisation loop keeps its base samples;
-    # a step's host inputs are then the observations, hyperparameters and
-    # candidates
-    heps = None
-    if w.mode == "mc":
-        bt.boute_engine_set_normals(e, 1234)
     hidx = torch.empty((w.B, w.k), dtype=torch.int64).pin_memory()
     hval = torch.empty((w.B, w.k), dtype=f32).pin_memory()
-    args_host = (hX, hY, hls, hs2, hnz, href, hXc, heps, hidx, hval)
-    h2d = sum(a.numel() * a.element_size() for a in args_host[:8] if a is not None)
-    d2h = hidx.numel() * 8 + hval.numel() * 4
-    # a stream of steps through the pipelined host-input call: each step's
-    # copies in overlap the previous step's computation (two device input
-    # sets); every step copies its inputs in and its selection out
-    bt.boute_engine_step_host(e, *args_host)
-    for _ in range(2):  # (captures the graph of each input set)
-        bt.boute_engine_step_host_async(e, *args_host)
-    bt.boute_engine_sync(e)
     n_e2e = args.e2e_steps or min(args.steps, 200)
-    barrier()
-    t0 = time.perf_counter()
-    for _ in range(n_e2e):
-        bt.boute_engine_step_host_async(e, *args_host)
-    bt.boute_engine_sync(e)
-    e2e_s = (time.perf_counter() - t0) / n_e2e
-    e2e_value = whole_job_rate(world, w, max_over_ranks(e2e_s, dist, dev))
+
+    def e2e_stream(heps):
+        """Candidates per second of a pipelined stream of host-input steps,
+        and the bytes each step copies in."""
+        args_host = (hX, hY, hls, hs2, hnz, href, hXc, heps, hidx, hval)
+        h2d = sum(a.numel() * a.element_size() for a in args_host[:8] if a is not None)
+        bt.boute_engine_step_host(e, *args_host)
+        for _ in range(2):  # (captures the graph of each input set)
+            bt.boute_engine_step_host_async(e, *args_host)
+        bt.boute_engine_sync(e)
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(n_e2e):
+            bt.boute_engine_step_host_async(e, *args_host)
+        bt.boute_engine_sync(e)
+        sec = (time.perf_counter() - t0) / n_e2e
+        return whole_job_rate(world, w, max_over_ranks(sec, dist, dev)), h2d
+
+    d2h = hidx.numel() * 8 + hval.numel() * 4
+    e2e_value, h2d = e2e_stream(pin(inp["eps"], f32))  # normals passed in every step
+    e2e = {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
+           "d2h_bytes_per_step": d2h, "call": "boute_engine_step_host_async",
+           "pipelined": True, "steps": n_e2e,
+           "normals": "host (copied every step)" if w.mode == "mc" else None}
+    if w.mode == "mc":
+        # the engine's own base normals, drawn once on the device from a seed
+        bt.boute_engine_set_normals(e, 1234)
+        dn_value, dn_h2d = e2e_stream(None)
+        e2e["device_normals"] = {"value": dn_value, "unit": UNIT,
+                                 "h2d_bytes_per_step": dn_h2d, "d2h_bytes_per_step": d2h,
+                                 "normals": "device (boute_engine_set_normals, fixed)"}
 
     if rank == 0:
         hbm, bf16, bf16s, src = peaks()
-        dom = max((s for s in stage_ms if s in ("fit", "posterior", "acquisition", "topk")),
-                  key=lambda s: stage_ms[s])
-        rf = roofline(w, dom, stage_ms[dom], hbm, bf16)
+        # a kernel inside a long step of back-to-back steps: the sustained peak
+        tens = tensor_peak(bf16s)
+        tens_tf32 = bf16s * (1.1 / 2.25) / 3
+        sm_mhz = (clk or {}).get("sm_mhz")
+        dom = max(("fit", "posterior", "acquisition", "topk"), key=lambda s_: live[s_])
+        rf = stage_roofline(w, dom, live[dom], hbm, tens, sm_mhz)
         roof = {"bound": rf["bound"], "achieved": rf["achieved"], "peak": rf["peak"],
                 "unit": rf["unit"], "frac": rf["achieved"] / rf["peak"],
-                "traffic": profiled_traffic(rf["kernel"], w.name), "kernel": rf["kernel"],
-                "stage": dom, "peak_source": src if rf["bound"] != "alu" else "nominal",
-                "algorithmic_per_launch": rf["per_launch"]}
+                "traffic": profiled_traffic(rf["kernel"], w.name, w.B * w.N),
+                "kernel": rf["kernel"], "stage": dom, "ms": live[dom],
+                "algorithmic_per_launch": rf["per_launch"],
+                "peak_source": (f"{src} bf16 sustained x {CONTRACTION['per_bf16']:.4f} "
+                                f"({CONTRACTION['dtype']}) / {CONTRACTION['products']} products"
+                                if rf["bound"] == "tensor" else
+                                f"{src} hbm copy" if rf["bound"] == "hbm" else
+                                "nominal: 152 SMs x 128 FMA lanes x 2 x measured SM clock"),
+                "pass": pass_roofline(w, live["posterior"] + live["acquisition"] + live["topk"],
+                                      hbm, tens, tens_tf32)}
         cpu = None
         if world == 1 and not args.no_cpu_baseline:
-            rate, thr, sample, dt = oracle_rate(w, inp, 12.0, cons=args.cons)
+            cin = host_inputs(w, count=CPU_PREFIX)
+            rate, thr, sample, dt = oracle_rate(w, cin, 12.0, cons=args.cons)
             cpu = {"value": rate, "unit": UNIT, "cores": thr, "kind": "oracle",
                    "sample": f"{sample} of {w.N} candidates of problem 0 ({dt:.1f} s), full fit "
                              "+ front + posterior + acquisition + top-k"}
@@ -408,13 +517,11 @@ def main():
                        **({"constraints": args.constraints} if args.cons else {})},
             "roofline": roof,
             "cpu_baseline": cpu,
-            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h, "call": "boute_engine_step_host_async",
-                    "pipelined": True,
-                    "normals": "device (boute_engine_set_normals)" if w.mode == "mc" else None},
+            "e2e": e2e,
             "gpu_launches": launches,
             "launches_per_step": bt.boute_engine_launches_per_step(e),
-            "stage_ms": stage_ms,
+            "stage_ms_live": live,
+            "stage_ms_serial": stage_ms,
             "wall_s": wall,
             "clocks": clk,
         }

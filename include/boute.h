@@ -336,13 +336,18 @@ int boute_engine_sync(boute_engine *e, void *stream);
 /* Copies the last step's per-candidate results into caller buffers (device
  * pointers; any may be NULL): acq B x N, mean and var B x m x N (fp32). */
 int boute_engine_scores(const boute_engine *e, float *acq, float *mean, float *var, void *stream);
-/* Stage timing on the engine's stream: while enabled (on != 0), every step
+/* Stage timing on the engine's stream. on = 1 (serialised): every step
  * records a CUDA event at each stage boundary (fit, front = standardise +
  * Pareto front + boxes, posterior, acquisition, top-k) and runs the front
- * stage after the fit on the step's stream instead of beside it, so that the
- * stages add up; boute_engine_stage_times waits for the last timed step and
- * writes its 5 stage durations in milliseconds (count >= 5). Disabling it
- * restores the concurrent front stage. */
+ * stage after the fit on the step's stream instead of beside it, with K*
+ * built inside the posterior, so that the stages add up. on = 2 (live): the
+ * step keeps its normal concurrent schedule and records events only on the
+ * step's stream: "fit" is then everything before the posterior starts (set-up,
+ * fit, and any wait for K* built beside it), "front" is 0 (it runs beside the
+ * fit), and posterior, acquisition and top-k are the three launches of the
+ * scoring pass (top-k is 0 where the acquisition kernel selects). on = 0
+ * disables timing. boute_engine_stage_times waits for the last timed step
+ * and writes its 5 stage durations in milliseconds (count >= 5). */
 int boute_engine_set_timing(boute_engine *e, int on);
 int boute_engine_stage_times(boute_engine *e, float *ms, int count);
 /* Kernels one boute_engine_step launches. */

@@ -450,7 +450,11 @@ def boute_engine_scores(e: Engine, acq=None, mean=None, var=None, stream=None):
                                       _s(stream)), "boute_engine_scores")
 
 
-def boute_engine_set_timing(e: Engine, on: bool = True):
+TIMING_OFF, TIMING_SERIAL, TIMING_LIVE = 0, 1, 2
+
+
+def boute_engine_set_timing(e: Engine, on=True):
+    """on: False/0 off, True/1 serialised stages, 2 live (normal schedule)."""
     _check(load().boute_engine_set_timing(e.handle, int(on)), "boute_engine_set_timing")
 
 

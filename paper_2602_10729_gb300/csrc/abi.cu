@@ -497,6 +497,8 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
   cudaStreamCaptureStatus run_cap = cudaStreamCaptureStatusNone;
   if (e->timing && s && cudaStreamIsCapturing(s, &run_cap) != cudaSuccess)
     return last_launch_status();
+  // live timing (2): the normal schedule, events on the step's stream only
+  const int serial = e->timing == 1, live = e->timing == 2;
   auto mark = [&](int stage) {
     if (!e->timing) return;
     if (run_cap == cudaStreamCaptureStatusActive)
@@ -525,14 +527,14 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
     if ((r = launch_outcome_transform(Y, (long long)B * n * m, m, e->tcodes, e->Yt, s))) return r;
     Y = e->Yt;
   }
-  // K* beside the fit (not in stage-timing mode, where the posterior builds it)
-  const float *kst = e->timing ? nullptr : e->kst;
+  // K* beside the fit (not in serialised timing, where the posterior builds it)
+  const float *kst = serial ? nullptr : e->kst;
   // The graph has one root, the fit's set-up: the front stage (which needs
   // the raw outcomes only) and K* (which needs the set-up's side input) fork
   // after it and run beside the fit (one root launches sooner than two).
-  if ((r = launch_fit_raw(&e->gp->g, X, Y, ls, s2, noise, s, e->timing ? nullptr : e->ev_setup)))
+  if ((r = launch_fit_raw(&e->gp->g, X, Y, ls, s2, noise, s, serial ? nullptr : e->ev_setup)))
     return r;
-  if (!e->timing) {
+  if (!serial) {
     if (cudaStreamWaitEvent(e->side, e->ev_setup, 0) != cudaSuccess) return last_launch_status();
     if ((r = front(e->side))) return r;
     if (cudaEventRecord(e->join, e->side) != cudaSuccess) return last_launch_status();
@@ -544,22 +546,29 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
     if ((r = launch_kstar(&e->gp->g, Xc, e->N, e->kst, e->side2))) return r;
     if (cudaEventRecord(e->join2, e->side2) != cudaSuccess) return last_launch_status();
   }
-  mark(ST_FRONT);
-  if (e->timing && (r = front(s))) return r;
-  mark(ST_POSTERIOR);
+  if (serial) {
+    mark(ST_FRONT);
+    if ((r = front(s))) return r;
+    mark(ST_POSTERIOR);
+  }
   if (host && cudaStreamWaitEvent(s, ev_xc, wait_flags) != cudaSuccess)
     return last_launch_status();
   if (kst && cudaStreamWaitEvent(s, e->join2, 0) != cudaSuccess) return last_launch_status();
+  if (live) {  // the posterior starts here; the front ran beside the fit
+    mark(ST_FRONT);
+    mark(ST_POSTERIOR);
+  }
   if ((r = launch_posterior(&e->gp->g, Xc, e->N, e->mean, e->var, s, kst))) return r;
-  if (!e->timing && cudaStreamWaitEvent(s, e->join, 0) != cudaSuccess)  // join
+  if (live) mark(ST_ACQ);
+  if (!serial && cudaStreamWaitEvent(s, e->join, 0) != cudaSuccess)  // join
     return last_launch_status();
   if (host && mc && eps != e->gen_eps)  // (the engine's own normals are resident)
     for (int i = 0; i < 2; ++i)
       if (cudaStreamWaitEvent(s, ev_eps[i], wait_flags) != cudaSuccess)
         return last_launch_status();
-  mark(ST_ACQ);
+  if (!live) mark(ST_ACQ);
   const double *cons = e->has_cons ? e->cons : nullptr;
-  if (e->fuse_sel && !e->timing) {
+  if (e->fuse_sel && !serial) {
     if ((r = launch_mchvi2_select(e->mean, e->var, B, e->N, e->lower, e->upper, e->K, 2 * n + 2,
                                   eps, e->S, 2ll * e->S, cons, e->acq, e->k, e->sel, idx, val,
                                   s)))
@@ -572,7 +581,8 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
                           e->S, (long long)m * e->S, cons, e->acq, s)))
       return r;
   }
-  if (!e->fuse_sel || e->timing) {
+  if (live && e->fuse_sel) mark(ST_TOPK);  // (the acquisition kernel selected)
+  if (!e->fuse_sel || serial) {
     mark(ST_TOPK);
     if ((r = launch_topk(e->acq, B, e->N, e->k, idx, val, e->scratch, s, true))) return r;
   }
@@ -785,7 +795,7 @@ int boute_engine_scores(const boute_engine *e, float *acq, float *mean, float *v
 int boute_engine_set_timing(boute_engine *e, int on) {
   BOUTE_TRACE();
   if (!e) return BOUTE_ERR_INVALID_ARG;
-  on = on != 0;
+  if (on < 0 || on > 2) return BOUTE_ERR_INVALID_ARG;
   if (on == e->timing) return BOUTE_OK;
   if (on && !e->ev[0])
     for (int i = 0; i <= ST_COUNT; ++i)

@@ -81,9 +81,16 @@ def test_engine_paths_agree_and_match_oracle(case):
         bt.boute_engine_set_timing(e, True)
         idx, val = _run(e, w, _dev(hp), "device")
         times = bt.boute_engine_stage_times(e)
-        bt.boute_engine_set_timing(e, False)
         assert np.array_equal(idx, ref_idx) and np.array_equal(val, ref_val)
         assert all(v > 0 for v in times.values()), times
+        # live timing: the normal schedule with events on the step's stream
+        bt.boute_engine_set_timing(e, bt.TIMING_LIVE)
+        idx, val = _run(e, w, _dev(hp), "device")
+        live = bt.boute_engine_stage_times(e)
+        bt.boute_engine_set_timing(e, False)
+        assert np.array_equal(idx, ref_idx) and np.array_equal(val, ref_val)
+        assert live["front"] == 0 and live["fit"] > 0 and live["posterior"] > 0, live
+        assert live["acquisition"] > 0 and live["topk"] >= 0, live
         acq = torch.empty((w.B, w.N), dtype=torch.float32, device="cuda")
         bt.boute_engine_scores(e, acq=acq)
         torch.cuda.synchronize()
@@ -169,7 +176,7 @@ def test_posterior_from_precomputed_kstar_matches_fused(wi, n, N, B):
     hp = host_problem(w)
     e = _engine(w)
     out = []
-    for timing in (False, True):
+    for timing in (False, True, bt.TIMING_LIVE):
         bt.boute_engine_set_timing(e, timing)
         idx, val = _run(e, w, _dev(hp), "device")
         mean = torch.empty((w.B, w.m, w.N), dtype=torch.float32, device="cuda")
@@ -179,8 +186,9 @@ def test_posterior_from_precomputed_kstar_matches_fused(wi, n, N, B):
         torch.cuda.synchronize()
         out.append((idx, val, acq.cpu().numpy(), mean.cpu().numpy(), var.cpu().numpy()))
     e.free()
-    for a, b in zip(*out):
-        assert np.array_equal(a, b)
+    for other in out[1:]:
+        for a, b in zip(out[0], other):
+            assert np.array_equal(a, b)
 
 
 # Pipelined host-input steps: consecutive calls alternate between two device
