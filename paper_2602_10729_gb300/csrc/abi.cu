@@ -554,10 +554,7 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
   if (host && cudaStreamWaitEvent(s, ev_xc, wait_flags) != cudaSuccess)
     return last_launch_status();
   if (kst && cudaStreamWaitEvent(s, e->join2, 0) != cudaSuccess) return last_launch_status();
-  if (live) {  // the posterior starts here; the front ran beside the fit
-    mark(ST_FRONT);
-    mark(ST_POSTERIOR);
-  }
+  if (live) mark(ST_POSTERIOR);  // the posterior starts here (the front ran beside the fit)
   if ((r = launch_posterior(&e->gp->g, Xc, e->N, e->mean, e->var, s, kst))) return r;
   if (live) mark(ST_ACQ);
   if (!serial && cudaStreamWaitEvent(s, e->join, 0) != cudaSuccess)  // join
@@ -581,7 +578,6 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
                           e->S, (long long)m * e->S, cons, e->acq, s)))
       return r;
   }
-  if (live && e->fuse_sel) mark(ST_TOPK);  // (the acquisition kernel selected)
   if (!e->fuse_sel || serial) {
     mark(ST_TOPK);
     if ((r = launch_topk(e->acq, B, e->N, e->k, idx, val, e->scratch, s, true))) return r;
@@ -813,6 +809,22 @@ int boute_engine_stage_times(boute_engine *e, float *ms, int count) {
   BOUTE_TRACE();
   if (!e || !ms || count < ST_COUNT || !e->ev[0]) return BOUTE_ERR_INVALID_ARG;
   if (cudaEventSynchronize(e->ev[ST_COUNT]) != cudaSuccess) return last_launch_status();
+  if (e->timing == 2) {
+    // live: no front boundary (it ran beside the fit); with the selection
+    // inside the acquisition kernel no top-k boundary either
+    const bool sel = e->fuse_sel != 0;
+    const int acq_end = sel ? ST_COUNT : ST_TOPK;
+    ms[ST_FRONT] = 0.f;
+    if (sel) ms[ST_TOPK] = 0.f;
+    if (cudaEventElapsedTime(&ms[ST_FIT], e->ev[ST_FIT], e->ev[ST_POSTERIOR]) != cudaSuccess ||
+        cudaEventElapsedTime(&ms[ST_POSTERIOR], e->ev[ST_POSTERIOR], e->ev[ST_ACQ]) !=
+            cudaSuccess ||
+        cudaEventElapsedTime(&ms[ST_ACQ], e->ev[ST_ACQ], e->ev[acq_end]) != cudaSuccess ||
+        (!sel &&
+         cudaEventElapsedTime(&ms[ST_TOPK], e->ev[ST_TOPK], e->ev[ST_COUNT]) != cudaSuccess))
+      return last_launch_status();
+    return BOUTE_OK;
+  }
   for (int i = 0; i < ST_COUNT; ++i)
     if (cudaEventElapsedTime(&ms[i], e->ev[i], e->ev[i + 1]) != cudaSuccess)
       return last_launch_status();
