@@ -192,8 +192,8 @@ int boute_gp_create(int B, int n, int d, int m, boute_gp **out) {
   const size_t np = g.plan.npad;
   r |= dalloc(&g.Aws, BM * np * (np + 1));
   r |= dalloc(&g.Wws, BM * np * (np + 1));
-  r |= dalloc(&g.bop, BM * (size_t)g.plan.image_floats);
-  r |= dalloc(&g.xt, BM * (size_t)g.plan.nchunk * xt_chunk_floats(g.DP));
+  r |= dalloc(&g.bop, BM * (size_t)g.plan.image_halves);
+  r |= dalloc(&g.xt, BM * (size_t)g.plan.nxt * xt_chunk_floats(g.DP));
   r |= dalloc(&g.s2f, BM);
   r |= dalloc(&g.status, 1);
   if (r != BOUTE_OK) {
@@ -203,7 +203,8 @@ int boute_gp_create(int B, int n, int d, int m, boute_gp **out) {
   cudaMemset(g.status, 0, sizeof(int));
   // operand images are fully rewritten by every fit; zero them once so that
   // padding never holds stale bits
-  cudaMemset(g.bop, 0, BM * (size_t)g.plan.image_floats * sizeof(float));
+  cudaMemset(g.bop, 0, BM * (size_t)g.plan.image_halves * sizeof(uint16_t));
+  cudaMemset(g.xt, 0, BM * (size_t)g.plan.nxt * xt_chunk_floats(g.DP) * sizeof(float));
   *out = h;
   return BOUTE_OK;
 }

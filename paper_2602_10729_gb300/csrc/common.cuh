@@ -5,6 +5,7 @@
 #pragma once
 
 #include <cuda_runtime.h>
+#include <math.h>
 #include <stdint.h>
 
 #include "boute.h"
@@ -12,25 +13,33 @@
 #define BOUTE_MAX_D 32       // candidate dimension limit (registers per thread)
 #define BOUTE_MAX_M 4        // objectives per problem
 #define BOUTE_MAX_N 2048     // training points per problem
-#define BOUTE_MAX_PASS 12    // 256-column passes of the posterior contraction
+#define BOUTE_MAX_BLK 16     // 128-column output blocks of the posterior contraction
 #define BOUTE_TILE_M 128     // candidates per posterior tile (MMA M)
-#define BOUTE_KCHUNK 32      // reduction columns per operand chunk (128 B of fp32)
+#define BOUTE_KCHUNK 32      // training points per side-input chunk
+#define BOUTE_ACHUNK 64      // reduction columns per operand chunk (128 B of fp16)
+#define BOUTE_BLKCOLS 128    // output columns per accumulator block (one TMEM slot)
 #define BOUTE_WAIT_NS 2000000000ull  // bound on any single device-side wait
 
 namespace boute {
 
 // ---------------------------------------------------------------- host/device
-// Operand-image plan of the posterior contraction for one (problem, objective):
-// output columns [0, n) are the rows of L^-1, padded with zero rows to a
-// multiple of 16. Columns are processed in passes of at most 256 (one
-// tcgen05.mma N); pass p needs the reduction chunks [0, kc[p]) only, because
-// row j of L^-1 is zero beyond column j. (The mean K* alpha is reduced on the
+// Operand plan of the posterior contraction V = K* W^T, W = L^-1, for one
+// (problem, objective): output column i of V is row i of W. Output columns
+// come in blocks of 128 (one tensor-memory accumulator slot each; the last
+// block's width is n rounded up to 16); the reduction over the training
+// points comes in chunks of 64 (one 128-byte row of fp16 per operand row).
+// Block q needs the chunks [0, kc[q]) only, because row i of W is zero beyond
+// column i. Its operand images follow one another: for each chunk, W's rows of
+// the block as fp16 hi then fp16 lo parts (ncol[q] rows x 64 halves each) in
+// the swizzled K-major layout tcgen05.mma reads. npad (n rounded up to 32) is
+// the fit's padded size; nxt side-input chunks of 32 points (n rounded up to
+// 64) cover the nchunk operand chunks. (The mean K* alpha is reduced on the
 // CUDA cores while K* is built, in compensated fp32.)
 struct PostPlan {
-  int n, npad, ncols, npass, nchunk;
-  int col0[BOUTE_MAX_PASS], ncol[BOUTE_MAX_PASS], kc[BOUTE_MAX_PASS];
-  long long off[BOUTE_MAX_PASS];  // float offset of the pass's first chunk image
-  long long image_floats;         // per (problem, objective)
+  int n, npad, nxt, nchunk, nblk;
+  int ncol[BOUTE_MAX_BLK], kc[BOUTE_MAX_BLK];
+  long long off[BOUTE_MAX_BLK];  // half offset of block q's first chunk image
+  long long image_halves;        // per (problem, objective)
 };
 
 inline __host__ __device__ int round_up(int x, int r) { return (x + r - 1) / r * r; }
@@ -57,38 +66,56 @@ __device__ __forceinline__ double outcome_transform(double y, int code) {
 // Floats of one training-point chunk of the posterior's side input: X/ls as
 // fp32 hi [DP][32] and lo [DP][32] (dimension-major, so pairs of training
 // points load as packed f32x2), alpha [32], then the objective's parameters
-// 1/ls hi [DP], 1/ls lo [DP], outputscale, 3 floats of padding.
+// 1/ls hi [DP], 1/ls lo [DP], and 8 scalars (kParS2 .. below).
 inline __host__ __device__ int xt_chunk_floats(int DP) {
-  return 2 * BOUTE_KCHUNK * DP + BOUTE_KCHUNK + 2 * DP + 4;
+  return 2 * BOUTE_KCHUNK * DP + BOUTE_KCHUNK + 2 * DP + 8;
 }
 inline __host__ __device__ int xt_param_offset(int DP) { return 2 * BOUTE_KCHUNK * DP + BOUTE_KCHUNK; }
+// The scalars after 1/ls hi and lo: outputscale; the composite kernel's s2_c,
+// s2_x and d_tau; the power-of-two exponent e_W of W's operand scale; the
+// composite kernel's largest training-point preference weight (written by the
+// fit, in chunk 0 only).
+enum { kParS2 = 0, kParS2c = 1, kParS2x = 2, kParDtau = 3, kParEW = 4, kParWmax = 5 };
+
+// Operand scales. The contraction runs on fp16 hi/lo parts, whose normal
+// range is [2^-14, 65504]: K* is scaled by 2^e_r so that its bound lies in
+// [2^14, 2^15), and W by 2^e_W with |W| <= 1/sigma_n (the smallest eigenvalue
+// of K = K0 + sigma_n^2 I is at least sigma_n^2, so ||L^-1||_2 <= 1/sigma_n)
+// mapped below 2^14, leaving a factor 4 of headroom for the rounding of the
+// fp32 factor. Powers of two scale exactly; the epilogue divides the sum of
+// squares by 2^(2 (e_r + e_W)).
+inline __host__ __device__ int kstar_scale_exp(float bound) { return 14 - ilogbf(bound); }
+inline __host__ __device__ int w_scale_exp(double noise, double s2) {
+  // (noise floored at 1e-12 s2: a smaller noise leaves K numerically singular in fp32)
+  const double v = noise > 1e-12 * s2 ? noise : 1e-12 * s2;
+  return 13 - ilogb(1.0 / sqrt(v));
+}
 
 inline PostPlan make_post_plan(int n) {
   PostPlan p{};
   p.n = n;
   p.npad = round_up(n, BOUTE_KCHUNK);
-  p.nchunk = p.npad / BOUTE_KCHUNK;
-  p.ncols = round_up(n, 16);
-  p.npass = (p.ncols + 255) / 256;
+  p.nxt = round_up(n, BOUTE_ACHUNK) / BOUTE_KCHUNK;
+  p.nchunk = p.nxt / 2;
+  p.nblk = (n + BOUTE_BLKCOLS - 1) / BOUTE_BLKCOLS;
   long long off = 0;
-  for (int q = 0; q < p.npass; ++q) {
-    p.col0[q] = 256 * q;
-    p.ncol[q] = (p.ncols - p.col0[q]) < 256 ? (p.ncols - p.col0[q]) : 256;
-    const int last_col = p.col0[q] + p.ncol[q] - 1;
-    const int need = round_up(last_col + 1, BOUTE_KCHUNK);
-    p.kc[q] = (need < p.npad ? need : p.npad) / BOUTE_KCHUNK;
+  for (int q = 0; q < p.nblk; ++q) {
+    const int c0 = BOUTE_BLKCOLS * q;
+    const int w = n - c0 < BOUTE_BLKCOLS ? n - c0 : BOUTE_BLKCOLS;
+    p.ncol[q] = round_up(w, 16);
+    p.kc[q] = (c0 + w + BOUTE_ACHUNK - 1) / BOUTE_ACHUNK;  // rows < c0 + w need columns < c0 + w
     p.off[q] = off;
-    off += (long long)p.kc[q] * 2 * p.ncol[q] * BOUTE_KCHUNK;
+    off += (long long)p.kc[q] * 2 * p.ncol[q] * BOUTE_ACHUNK;
   }
-  p.image_floats = off;
+  p.image_halves = off;
   return p;
 }
 
-// Float offset, inside a [rows x 32] fp32 block laid out for a K-major
+// Half offset, inside a [rows x 64] fp16 block laid out for a K-major
 // tcgen05 operand with the 128-byte swizzle, of element (row, kk): each row
-// is 128 B, 16-byte groups permuted by XOR with (row mod 8).
-inline __host__ __device__ int sw128_off(int row, int kk) {
-  return row * 32 + ((((kk >> 2) ^ (row & 7))) << 2) + (kk & 3);
+// is 128 B, its 16-byte groups of 8 halves permuted by XOR with (row mod 8).
+inline __host__ __device__ int sw128_off16(int row, int kk) {
+  return row * 64 + ((((kk >> 3) ^ (row & 7))) << 3) + (kk & 7);
 }
 
 #ifdef __CUDACC__
@@ -230,18 +257,20 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
   return d;
 }
 
-// Instruction descriptor: kind::tf32, fp32 accumulate, A and B K-major, M=128.
-__host__ __device__ constexpr uint32_t idesc_tf32(int N) {
-  return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(N >> 3) << 17) |
-         ((uint32_t)(BOUTE_TILE_M >> 4) << 24);
+// Instruction descriptor: kind::f16 with fp16 A and B, fp32 accumulate, A
+// and B K-major, M = 128, N = n (a multiple of 16, at most 256).
+__host__ __device__ constexpr uint32_t idesc_f16(int N) {
+  return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(BOUTE_TILE_M >> 4) << 24);
 }
 
-__device__ __forceinline__ void mma_tf32(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
-                                         uint32_t idesc, uint32_t accumulate) {
+// D (tensor memory) += A (shared) x B (shared)^T, or D = A x B^T when
+// accumulate is 0; issued by one thread.
+__device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                        uint32_t idesc, uint32_t accumulate) {
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
       "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
@@ -269,12 +298,30 @@ __device__ __forceinline__ void tmem_ld8(uint32_t taddr, float (&v)[8]) {
   for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// Round to the nearest tf32 value (ties away), kept in fp32 layout.
-__device__ __forceinline__ float tf32_rna(float x) {
+// Two fp32 values as packed fp16 (round to nearest even): element `a` in the
+// low half (the lower address in memory), `b` in the high half.
+__device__ __forceinline__ uint32_t pack_f16x2(float a, float b) {
   uint32_t r;
-  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
-  return __uint_as_float(r);
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(b), "f"(a));
+  return r;
 }
+__device__ __forceinline__ void unpack_f16x2(uint32_t v, float &a, float &b) {
+  asm("{\n\t.reg .b16 l, h;\n\tmov.b32 {l, h}, %2;\n\t"
+      "cvt.f32.f16 %0, l;\n\tcvt.f32.f16 %1, h;\n\t}"
+      : "=f"(a), "=f"(b)
+      : "r"(v));
+}
+// The fp16 hi/lo split of a pair: hi = fp16(x), lo = fp16(x - hi), so that
+// hi + lo carries 22 significant bits of x (x within the fp16 normal range).
+__device__ __forceinline__ void split_f16x2(float x0, float x1, uint32_t &hi, uint32_t &lo) {
+  hi = pack_f16x2(x0, x1);
+  float h0, h1;
+  unpack_f16x2(hi, h0, h1);
+  lo = pack_f16x2(x0 - h0, x1 - h1);
+}
+
+// 2^k as an fp32 value, k in the normal range [-126, 127].
+__device__ __forceinline__ float exp2i(int k) { return __int_as_float((127 + k) << 23); }
 
 __device__ __forceinline__ void set_status(int *status, int code) {
   if (status) atomicCAS(status, 0, code);

@@ -138,7 +138,7 @@ __device__ void kmat_tile(const double *X, int n, int d, int b, const double *l,
 
 template <bool COMP>
 __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad,
-                          const double *l, double s2, float *x, int blk, int nblk,
+                          const double *l, double s2, double noise, float *x, int blk, int nblk,
                           const double *kp, int dtau) {
   const int cf = xt_chunk_floats(DP);
   const int total = npad * DP;
@@ -166,9 +166,9 @@ __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad
           (k >= dtau && k < d) ? (float)(kp[2] * kp[3 + k]) : 0.f;
     }
   }
-  const int po = xt_param_offset(DP), nch = npad / BOUTE_KCHUNK;
-  for (int e = blk * blockDim.x + threadIdx.x; e < nch * (2 * DP + 4); e += nblk * blockDim.x) {
-    const int c = e / (2 * DP + 4), k = e % (2 * DP + 4);
+  const int po = xt_param_offset(DP), nch = npad / BOUTE_KCHUNK, np = 2 * DP + 8;
+  for (int e = blk * blockDim.x + threadIdx.x; e < nch * np; e += nblk * blockDim.x) {
+    const int c = e / np, k = e % np;
     float v = 0.f;
     if (k < DP) v = k < d ? (float)(1.0 / l[k]) : 0.f;
     else if (k < 2 * DP) {
@@ -177,10 +177,12 @@ __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad
         const double iv = 1.0 / l[t];
         v = (float)(iv - (double)(float)iv);
       }
-    } else if (k == 2 * DP) v = (float)s2;
-    else if (COMP && k == 2 * DP + 1) v = (float)kp[0];
-    else if (COMP && k == 2 * DP + 2) v = (float)kp[1];
-    else if (COMP && k == 2 * DP + 3) v = (float)dtau;
+    } else if (k == 2 * DP + kParS2) v = (float)s2;
+    else if (COMP && k == 2 * DP + kParS2c) v = (float)kp[0];
+    else if (COMP && k == 2 * DP + kParS2x) v = (float)kp[1];
+    else if (COMP && k == 2 * DP + kParDtau) v = (float)dtau;
+    else if (k == 2 * DP + kParEW)  // the prior variance bounds K's diagonal from above
+      v = (float)w_scale_exp(noise, COMP ? s2 + kp[0] + kp[1] : s2);
     x[(size_t)c * cf + po + k] = v;
   }
 }
@@ -201,33 +203,50 @@ __global__ void __launch_bounds__(kSetupThreads) fit_setup_kernel(
                     Kl_all + (size_t)bt * n * n, il, kp, dtau);
   } else {
     float *x = xt + (size_t)bt * (npad / BOUTE_KCHUNK) * xt_chunk_floats(DP);
-    prep_part<COMP>(X, n, d, b, DP, npad, l, s2[bt], x, blockIdx.x - nkt, nprep, kp, dtau);
+    prep_part<COMP>(X, n, d, b, DP, npad, l, s2[bt], noise[bt], x, blockIdx.x - nkt, nprep, kp,
+                    dtau);
     // the prior variance's constant part (composite: s2 + s2_x; the
     // posterior adds s2_c w(x)^2)
     if (blockIdx.x == nkt && threadIdx.x == 0) s2f[bt] = (float)(COMP ? s2[bt] + kp[1] : s2[bt]);
   }
 }
 
-// fp32 tf32 hi/lo operand images of W = L^-1 (lower, row stride ld), swizzled
-// per column pass and 32-wide K chunk, written by the threads of one block (or
-// a grid of blocks: element e in [first, total) by stride).
-__device__ __forceinline__ void pack_elems(const float *W, int ld, const PostPlan &plan,
-                                           float *img, long long first, long long stride) {
+// The fp16 hi/lo operand images of W = L^-1 scaled by 2^e_W (see PostPlan):
+// the pair of elements (g, k), (g, k + 1) of W (row g = output column, k
+// even), zero above the diagonal and beyond n. Returns false if a scaled
+// element reaches the fp16 range (W beyond four times its bound 1/sigma_n:
+// the fp32 factor is numerically singular).
+__device__ __forceinline__ bool pack_pair(const float *wrow, int g, int k, const PostPlan &plan,
+                                          float scale, uint16_t *img) {
   const int n = plan.n;
-  const long long total = (long long)plan.ncols * plan.npad;
+  const float v0 = (k < n && g < n && k <= g) ? wrow[k] * scale : 0.f;
+  const float v1 = (k + 1 < n && g < n && k + 1 <= g) ? wrow[k + 1] * scale : 0.f;
+  uint32_t hi, lo;
+  split_f16x2(v0, v1, hi, lo);
+  const int q = g / BOUTE_BLKCOLS, c = k / BOUTE_ACHUNK, ncol = plan.ncol[q];
+  uint32_t *blk = (uint32_t *)(img + plan.off[q] + (long long)c * 2 * ncol * BOUTE_ACHUNK);
+  const int o = sw128_off16(g % BOUTE_BLKCOLS, k % BOUTE_ACHUNK) >> 1;
+  blk[o] = hi;
+  blk[(ncol * BOUTE_ACHUNK >> 1) + o] = lo;
+  return fabsf(v0) < 32768.f && fabsf(v1) < 32768.f;
+}
+
+// All of W's image elements, pairs [first, total) by stride (rows of the
+// blocks' padded widths, the chunks each block needs).
+__device__ __forceinline__ bool pack_elems(const float *W, int ld, const PostPlan &plan,
+                                           float scale, uint16_t *img, long long first,
+                                           long long stride) {
+  const int nblk = plan.nblk;
+  const long long rows = (long long)BOUTE_BLKCOLS * (nblk - 1) + plan.ncol[nblk - 1];
+  const int kmax = BOUTE_ACHUNK * plan.kc[nblk - 1];  // pairs per row: kmax / 2
+  const long long total = rows * (kmax / 2);
+  bool ok = true;
   for (long long e = first; e < total; e += stride) {
-    const int g = (int)(e / plan.npad), k = (int)(e % plan.npad);
-    const int p = g >> 8, c = k / BOUTE_KCHUNK;
-    if (c >= plan.kc[p]) continue;
-    const float v = (k < n && g < n && k <= g) ? W[(size_t)g * ld + k] : 0.f;
-    const float hi = tf32_rna(v);
-    const float lo = tf32_rna(v - hi);
-    const int ncol = plan.ncol[p];
-    float *blk = img + plan.off[p] + (long long)c * 2 * ncol * BOUTE_KCHUNK;
-    const int o = sw128_off(g - plan.col0[p], k % BOUTE_KCHUNK);
-    blk[o] = hi;
-    blk[ncol * BOUTE_KCHUNK + o] = lo;
+    const int g = (int)(e / (kmax / 2)), k = 2 * (int)(e % (kmax / 2));
+    if (k / BOUTE_ACHUNK >= plan.kc[g / BOUTE_BLKCOLS]) continue;
+    ok &= pack_pair(W + (size_t)(g < plan.npad ? g : 0) * ld, g, k, plan, scale, img);
   }
+  return ok;
 }
 
 // Error-free product and sum on fp32 pairs (Dekker / Knuth).
@@ -262,8 +281,8 @@ constexpr int fit_threads() { return SMEM ? 512 : 256; }
 template <bool SMEM>
 __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     const float *Kh_all, const float *Kl_all, const double *Ys, int standardize, int n, int m,
-    float *Aws, float *Wws, float *xt, int DP, int npad, PostPlan plan, float *bop, int kl_smem,
-    int early_trigger, int *status) {
+    float *Aws, float *Wws, float *xt, int DP, int npad, PostPlan plan, uint16_t *bop,
+    int kl_smem, int early_trigger, int comp, int *status) {
   extern __shared__ __align__(16) float sm[];
   __shared__ int bad;
   __shared__ uint64_t lbar, lbar_lo;  // K hi; K lo (needed only by the residual)
@@ -381,24 +400,22 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   if (tid == 0) bad = 0;
   for (int e = tid; e < 32 * 64; e += nthr) (&colL[0][0])[e] = 0.f;
   __syncthreads();
-  // Operand images of W for the posterior (one column pass, n <= 160): rows
-  // [g_lo, g_hi) of W, warps w0, w0 + nws, ... one row each, lane = k % 32.
-  // A block row of W is final once its panel's trailing update is done.
+  // Operand images of W for the posterior (n <= 160): rows [g_lo, g_hi) of W,
+  // warps w0, w0 + nws, ... one row each, lane = pair of columns 2 lane of
+  // each 64-wide chunk, scaled by 2^e_W. A block row of W is final once its
+  // panel's trailing update is done.
+  const float *xpar = xt + (size_t)bt * plan.nxt * xt_chunk_floats(DP) + xt_param_offset(DP) +
+                      2 * DP;
+  const float wscale = exp2i((int)xpar[kParEW]);
+  const int gmax = BOUTE_BLKCOLS * (plan.nblk - 1) + plan.ncol[plan.nblk - 1];
   auto pack_rows = [&](int g_lo, int g_hi, int w0, int nws) {
-    float *img = bop + (size_t)bt * plan.image_floats + plan.off[0];
-    const int ncol = plan.ncol[0], kc = plan.kc[0];
-    for (int g = g_lo + w0; g < g_hi && g < ncol; g += nws) {
+    uint16_t *img = bop + (size_t)bt * plan.image_halves;
+    for (int g = g_lo + w0; g < g_hi && g < gmax; g += nws) {
       const float *wr = W + (size_t)g * ld;
-      const int o = sw128_off(g, lane);
-#pragma unroll 4
-      for (int c = 0; c < kc; ++c) {
-        const int k = c * BOUTE_KCHUNK + lane;
-        const float v = (k < n && g < n && k <= g) ? wr[k] : 0.f;
-        const float hi = tf32_rna(v), lo = tf32_rna(v - hi);
-        float *blk = img + (size_t)c * 2 * ncol * BOUTE_KCHUNK;
-        blk[o] = hi;
-        blk[ncol * BOUTE_KCHUNK + o] = lo;
-      }
+      const int kc = plan.kc[g / BOUTE_BLKCOLS];
+      for (int c = 0; c < kc; ++c)
+        if (!pack_pair(wr, g, BOUTE_ACHUNK * c + 2 * lane, plan, wscale, img))
+          set_status(status, BOUTE_ERR_NOT_PD);
     }
   };
   // ---- blocked Cholesky and W = L^-1, 32-column panels -------------------------
@@ -820,18 +837,32 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   // side input
   if (SMEM) pack_rows(NP - 32, NP, warp, nw);  // the last block row (the others: above)
   const int cf = xt_chunk_floats(DP);
-  float *xa = xt + (size_t)bt * (npad / BOUTE_KCHUNK) * cf + 2 * BOUTE_KCHUNK * DP;
-  for (int k = tid; k < npad; k += nthr)
+  float *xa = xt + (size_t)bt * plan.nxt * cf + 2 * BOUTE_KCHUNK * DP;
+  for (int k = tid; k < BOUTE_KCHUNK * plan.nxt; k += nthr)
     xa[(size_t)(k / BOUTE_KCHUNK) * cf + k % BOUTE_KCHUNK] = k < n ? al[k] : 0.f;
+  if (comp && warp == nw - 1) {  // the largest preference weight w_j (composite kernel)
+    float *x0 = xt + (size_t)bt * plan.nxt * cf;
+    const float *xw = x0 + BOUTE_KCHUNK * DP;
+    float wm = 0.f;
+    for (int j = lane; j < n; j += 32) wm = fmaxf(wm, xw[(size_t)(j / BOUTE_KCHUNK) * cf + j % 32]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
+    if (lane == 0) x0[xt_param_offset(DP) + 2 * DP + kParWmax] = wm;
+  }
 }
 
-// ---- operand images of L^-1 as tf32 hi/lo, swizzled (global-workspace fit) ----
-__global__ void pack_kernel(const float *Wws, PostPlan plan, float *bop, const int *status) {
+// ---- operand images of L^-1 as fp16 hi/lo, swizzled (global-workspace fit) ----
+__global__ void pack_kernel(const float *Wws, PostPlan plan, uint16_t *bop, const float *xt,
+                            int DP, int *status) {
   if (*status == BOUTE_ERR_NOT_PD) return;
   const size_t bt = blockIdx.y;
   const int ld = plan.npad + 1;
-  pack_elems(Wws + bt * plan.npad * ld, ld, plan, bop + bt * plan.image_floats,
-             (long long)blockIdx.x * blockDim.x + threadIdx.x, (long long)gridDim.x * blockDim.x);
+  const float *xpar = xt + bt * plan.nxt * xt_chunk_floats(DP) + xt_param_offset(DP) + 2 * DP;
+  if (!pack_elems(Wws + bt * plan.npad * ld, ld, plan, exp2i((int)xpar[kParEW]),
+                  bop + bt * plan.image_halves,
+                  (long long)blockIdx.x * blockDim.x + threadIdx.x,
+                  (long long)gridDim.x * blockDim.x))
+    set_status(status, BOUTE_ERR_NOT_PD);
 }
 
 }  // namespace
@@ -875,7 +906,7 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
                            const double *ls, const double *s2, const double *noise,
                            cudaStream_t s, cudaEvent_t setup_done = nullptr) {
   const int n = gp->n, d = gp->d, m = gp->m, BM = gp->B * gp->m;
-  const int npad = gp->plan.npad;
+  const int npad = gp->plan.npad, xpad = BOUTE_KCHUNK * gp->plan.nxt;
   const int nkt = kmat_units(n);
   const int sms = num_sms();
   // side-input blocks: as many as leave one block per SM (K blocks first), 2 .. 16
@@ -888,7 +919,7 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
   const int fit_early = 2 * BM <= sms ? 1 : 0;
   auto setup = [&](auto kern) {
     prefer_shared(kern);
-    kern<<<dim3(nkt + nprep, BM), kSetupThreads, 0, s>>>(X, n, d, m, gp->DP, npad, ls, s2, noise,
+    kern<<<dim3(nkt + nprep, BM), kSetupThreads, 0, s>>>(X, n, d, m, gp->DP, xpad, ls, s2, noise,
                                                          gp->Kh, gp->Kl, gp->xt, gp->s2f, nkt,
                                                          nprep, setup_early, gp->status,
                                                          gp->kpar, gp->dtau);
@@ -903,15 +934,15 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
                          (int)smem);
     launch_pdl(fit32_kernel<true>, dim3(BM), dim3(fit_threads<true>()), smem, s, gp->Kh, gp->Kl,
                Ys, standardize, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop,
-               fit_kl_in_smem(n) ? 1 : 0, fit_early, gp->status);
+               fit_kl_in_smem(n) ? 1 : 0, fit_early, gp->kern, gp->status);
     count_launch(2);
   } else {
     launch_pdl(fit32_kernel<false>, dim3(BM), dim3(fit_threads<false>()),
                6 * npad * sizeof(float), s, gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws,
-               gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop, 0, 0, gp->status);
-    const long long tot = (long long)gp->plan.ncols * npad;
+               gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop, 0, 0, gp->kern, gp->status);
+    const long long tot = (long long)gp->plan.nblk * BOUTE_BLKCOLS * gp->plan.nchunk * 32;
     pack_kernel<<<dim3((unsigned)std::min<long long>((tot + 255) / 256, 4096), BM), 256, 0, s>>>(
-        gp->Wws, gp->plan, gp->bop, gp->status);
+        gp->Wws, gp->plan, gp->bop, gp->xt, gp->DP, gp->status);
     count_launch(3);
   }
   return last_launch_status();

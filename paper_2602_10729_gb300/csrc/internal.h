@@ -16,8 +16,8 @@ struct Gp {
   float *Kh, *Kl;  // B*m x n x n: kernel matrix (lower) as an fp32 pair hi + lo
   float *Aws;      // B*m x np x (np+1): factorisation workspace (large n; np = npad)
   float *Wws;      // B*m x np x (np+1): L^-1 (lower, row stride np+1)
-  float *bop;     // B*m x plan.image_floats: L^-1 as tf32 hi/lo operand images
-  float *xt;      // B*m x nchunk x xt_chunk_floats(DP): X/lengthscale hi/lo, alpha
+  uint16_t *bop;  // B*m x plan.image_halves: L^-1 as fp16 hi/lo operand images
+  float *xt;      // B*m x nxt x xt_chunk_floats(DP): X/lengthscale hi/lo, alpha
   float *s2f;     // B*m: outputscale
   int *status;    // device status word (first error wins)
   // the composite kernel (kern = 1): routing features [0, dtau) and per
@@ -82,8 +82,9 @@ int launch_fit(Gp *gp, const double *X, const double *Ys, const double *ls, cons
 // kst: K* precomputed by launch_kstar (the posterior then builds no K*), or null.
 int launch_posterior(const Gp *gp, const float *Xc, long long N, float *mean, float *var,
                      cudaStream_t s, const float *kst = nullptr);
-// K* of all candidates, per (128-candidate tile, objective) and 32-point chunk
-// as 128 x 32 fp32: kstar_floats(gp, N) floats. Reads the fit set-up's side
+// K* of all candidates, per (128-candidate tile, objective) and 64-point chunk
+// as the fp16 hi and lo images of an A stage (128 x 64 each, scaled by the
+// row's 2^e_r): kstar_floats(gp, N) 4-byte words. Reads the fit set-up's side
 // input (not the fit's results) and the candidates.
 size_t kstar_floats(const Gp *gp, long long N);
 int launch_kstar(const Gp *gp, const float *Xc, long long N, float *kst, cudaStream_t s);

@@ -1,34 +1,38 @@
 // Fused GP posterior on the 5th-generation tensor cores (sm_103a).
 //
 // For a tile of 128 candidates and each objective, the Matern-5/2
-// cross-covariance K* (128 x n) is built chunk by chunk (32 training points =
-// 128 B rows) straight into shared memory in the swizzled K-major operand
-// layout, split into tf32 hi/lo parts, and contracted against the prepacked
-// operand L^-1 (hi/lo, brought in by bulk TMA copies) with three
-// tcgen05.mma kind::tf32 per k-step (hi*hi + hi*lo + lo*hi, fp32 accumulate in
-// tensor memory). The variance is s2 - rowsum(V^2), V = K* L^-T, read back
-// from tensor memory with tcgen05.ld. The mean K* alpha is a matrix-vector
-// product: the threads building K* reduce it on the CUDA cores in fp32 with
+// cross-covariance K* (128 x n) is built chunk by chunk (64 training points =
+// one 128-byte row of fp16 per candidate) straight into shared memory in the
+// swizzled K-major operand layout, split into fp16 hi/lo parts, and
+// contracted against the prepacked operand W = L^-1 (fp16 hi/lo, brought in by
+// bulk TMA copies) with three tcgen05.mma kind::f16 per k-step (hi*hi + hi*lo
+// + lo*hi, fp32 accumulate in tensor memory): 22 significant bits per operand
+// at twice the tensor rate of tf32. Both operands are scaled by powers of two
+// into fp16's normal range (K* by 2^e_r from its bound, W by 2^e_W from
+// ||L^-1|| <= 1/sigma_n), which the epilogue divides out exactly. The
+// variance is s2 - rowsum(V^2), V = K* W^T, read back from tensor memory with
+// tcgen05.ld. The mean K* alpha is a matrix-vector product: the threads
+// building K* reduce it on the CUDA cores from the fp32 values, with
 // compensated (Kahan) accumulation across chunks, which is more accurate than
 // the tensor core's fp32 accumulation and takes no operand column. K* never
 // reaches HBM.
 //
+// Output columns come in blocks of 128, one per tensor-memory slot (4 slots
+// of 128 columns, assigned round-robin over the blocks a CTA processes, so the
+// epilogue of one block overlaps the MMAs of later ones). Up to four blocks
+// form a group that shares each K* chunk: the chunk is built once and feeds
+// every block of the group whose rows of W are not zero there (block q needs
+// chunks [0, kc[q])). With n <= 512 every chunk is built once per tile.
+//
 // Persistent and warp-specialised: each CTA loops over (tile, objective) units.
-//   warp 0      bulk-TMA producer of the operand images of L^-1 (B ring)
+//   warp 0      bulk-TMA producer of the operand images of W (B ring)
 //   warp 1      tcgen05.mma issuer; owns the 512-column TMEM allocation
 //   warps 2-5   epilogue: one TMEM lane quarter each, sum of squares, variance
 //   warp 6      bulk-TMA producer of the training-point chunks (side-input ring)
+//               and, with K* precomputed, of its fp32 images (staging ring)
 //   warps 7..   K* builders: packed f32x2 distance math, A ring
-// Three shared-memory rings with their own depths: A (K* hi/lo, builders ->
-// MMA), B (L^-1 hi/lo, TMA -> MMA) and the side input (scaled training points,
-// alpha and the objective's parameters, TMA -> builders), so that the builders
-// never wait on the operand copies of the MMA; the accumulator is
-// double-buffered in TMEM (2 x 256 columns; a pass with a reduction longer
-// than 256 takes both buffers, one per half of the reduction) so the
-// epilogue of one output pass overlaps the MMAs of the next. Output columns
-// beyond 256 are handled in passes; pass p skips the reduction chunks where
-// its rows of L^-1 are zero. All waits are bounded (BOUTE_WAIT_NS): a wait
-// that gives up records BOUTE_ERR_TIMEOUT and every role stops.
+// All waits are bounded (BOUTE_WAIT_NS): a wait that gives up records
+// BOUTE_ERR_TIMEOUT and every role stops.
 #include <math.h>
 
 #include <algorithm>
@@ -44,38 +48,44 @@ constexpr int kEpiWarp0 = 2;  // warps 2-5: epilogue, TMEM lane quarter = warp %
 constexpr int kEpiWarps = 4;
 constexpr int kXtWarp = 6;    // warp 6: side-input producer
 constexpr int kBldWarp0 = 7;  // warps 7..: K* builders
-constexpr int kMaxA = 4, kMaxB = 4, kMaxX = 8;  // ring depths
-constexpr uint32_t kABytes = 32768;             // one A stage: 128 x 32 fp32, hi and lo
+constexpr int kMaxA = 4, kMaxB = 6, kMaxX = 8;  // ring depths
+constexpr int kSlots = 4;                       // TMEM accumulator slots of 128 columns
+constexpr int kGroup = 4;                       // blocks sharing one K* chunk
+constexpr uint32_t kAPartBytes = BOUTE_TILE_M * BOUTE_ACHUNK * 2;   // one fp16 part: 16 KB
+constexpr uint32_t kABytes = 2 * kAPartBytes;                       // hi and lo
+constexpr uint32_t kStageBytes = BOUTE_TILE_M * BOUTE_ACHUNK * 4;   // fp32 K* image: 32 KB
 
-// The tensor core's fp32 accumulator truncates after each MMA, so its error
-// grows with the number of accumulations into one output. A pass whose
-// reduction is longer than 8 chunks (256 training points) accumulates its
-// first and second halves in the two TMEM buffers, which the epilogue adds in
-// round-to-nearest; returns the chunk count of the first half (kc: no split).
-__device__ __forceinline__ int split_chunks(int kc) { return kc > 8 ? (kc + 1) / 2 : kc; }
-// builder warps: 16 (8 elements per thread and chunk) when the candidate
-// coordinates are short enough to keep in registers, else 8 (16 elements)
+// builder warps: 16 (8 columns of each 32-point half per thread) when the
+// candidate coordinates are short enough to keep in registers, else 8 (16)
 template <int DP>
 struct Layout {
   static constexpr int kBld = DP <= 16 ? 16 : 8;
   static constexpr int kThreads = 32 * (kBldWarp0 + kBld);
-  static constexpr int kCols = 128 / kBld;  // chunk columns per builder thread (8 or 16)
+  static constexpr int kCols = 128 / kBld;  // columns of a 32-point half per builder thread
 };
 
 struct PostArgs {
   const float *Xc;
   const float *kst;  // precomputed K* (PRE variant), else unused
   float *mean, *var;
-  const float *bop, *xt, *s2f;
+  const uint16_t *bop;
+  const float *xt, *s2f;
   int *status;
   long long N;
   int B, m, d, n;
   int tiles_per_problem, tiles_total;
-  int sa, sb, sx;              // depths of the A, B and side-input rings
+  int sa, sb, sx;              // depths of the A (and staging), B and side-input rings
   uint32_t b_bytes, x_bytes;   // one B stage, one side-input entry
   int kern;                    // 1: the composite kernel (prior variance per candidate)
   PostPlan plan;
 };
+
+// Word offset, inside a [128 x 64] fp32 K* image (PRE), of element (row, kk):
+// 16-byte groups permuted by XOR with (row mod 16), so that a builder warp's
+// rows read distinct banks.
+__host__ __device__ __forceinline__ int st_off32(int row, int kk) {
+  return row * 64 + ((((kk >> 2) ^ (row & 15))) << 2) + (kk & 3);
+}
 
 constexpr float kSqrt5 = 2.2360679774997896964f;
 constexpr float kSqrt5Log2e = 3.2259641822295610f;  // sqrt(5) / ln(2)
@@ -254,6 +264,18 @@ __device__ __forceinline__ void scaled_candidate(const float (&xr)[DP], const fl
   for (int k = 0; k < DP; ++k) xs2[k] = f2_dup(fmaf(xr[k], il[k], xr[k] * il[DP + k]));
 }
 
+
+// The exponent e_r of a candidate row's K* scale (kstar_scale_exp of the
+// row's bound on K*): the outputscale for the Matern-5/2 kernel; for the
+// composite kernel s2 + s2_x + s2_c w* max_j w_j (each factor k52, k32 <= 1).
+// Builders, the epilogue and the K* kernel all derive it here.
+__device__ __forceinline__ int row_exp(int kern, const float *par, float ws) {
+  float bound = par[kParS2];
+  if (kern) bound = fmaf(par[kParS2c] * ws, par[kParWmax], par[kParS2] + par[kParS2x]);
+  if (!(bound > 0.f) || !(bound < 3.0e38f)) bound = 1.f;
+  return kstar_scale_exp(bound);
+}
+
 // Position in a ring of R stages: the stage index and the parity of the
 // stage's use count (the mbarrier phase a consumer waits for), advanced
 // without integer division.
@@ -287,14 +309,26 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity,
   }
 }
 
-// PRE: the K* values come precomputed (kstar_kernel) instead of being built
-// here; everything else is the same. KERN: the kernel the builders evaluate
-// (0 Matern-5/2, 1 composite; only when !PRE).
+// The work sequence every role follows: per unit (tile, objective), the
+// groups of up to kGroup blocks; per group the chunks [0, kc[last block]).
+struct Groups {
+  int n;  // groups per unit
+  __device__ __forceinline__ explicit Groups(const PostPlan &p) : n((p.nblk + kGroup - 1) / kGroup) {}
+  __device__ __forceinline__ static int first(int g) { return g * kGroup; }
+  __device__ __forceinline__ static int last(const PostPlan &p, int g) {
+    return min(p.nblk, (g + 1) * kGroup) - 1;
+  }
+};
+
+// PRE: the K* values come precomputed (kstar_kernel, scaled fp32 images)
+// instead of being built here; everything else is the same. KERN: the
+// handle's kernel (0 Matern-5/2, 1 composite), which the builders evaluate
+// (!PRE) and from which every role derives the rows' K* scale.
 template <int DP, bool PRE, int KERN = 0>
 __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
     posterior_kernel(const __grid_constant__ PostArgs a) {
   constexpr int kBldWarps = Layout<DP>::kBld;
-  constexpr int COLS = Layout<DP>::kCols;   // columns of a chunk per builder thread
+  constexpr int COLS = Layout<DP>::kCols;   // columns of a half per builder thread
   constexpr int GPR = 32 / COLS;            // column groups per row (threads per row)
   constexpr int RPW = 32 / GPR;             // rows per builder warp
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -305,27 +339,32 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   const PostPlan &pl = a.plan;
   const int n = a.n, m = a.m, d = a.d, SA = a.sa, SB = a.sb, SX = a.sx;
   const int cf = xt_chunk_floats(DP);
+  const Groups grp(pl);
 
   uint8_t *ring_b = sm + (size_t)SA * kABytes;
   uint8_t *ring_x = ring_b + (size_t)SB * a.b_bytes;
-  uint64_t *bars = (uint64_t *)(ring_x + (size_t)SX * a.x_bytes);
+  uint8_t *ring_s = ring_x + (size_t)SX * a.x_bytes;  // PRE staging (SA stages)
+  uint64_t *bars = (uint64_t *)(ring_s + (PRE ? (size_t)SA * kStageBytes : 0));
   uint64_t *a_full = bars, *a_empty = bars + kMaxA;
   uint64_t *b_full = bars + 2 * kMaxA, *b_empty = b_full + kMaxB;
   uint64_t *x_full = b_full + 2 * kMaxB, *x_empty = x_full + kMaxX;
-  uint64_t *acc_full = x_full + 2 * kMaxX, *acc_empty = acc_full + 2, *drain = acc_full + 4;
-  uint64_t *ahi_full = drain + 1;  // PRE: the K* image of an A stage has landed
-  uint32_t *tmem_holder = (uint32_t *)(ahi_full + kMaxA);
+  uint64_t *acc_full = x_full + 2 * kMaxX, *acc_empty = acc_full + kSlots;
+  uint64_t *drain = acc_empty + kSlots;
+  uint64_t *st_full = drain + 1, *st_empty = st_full + kMaxA;  // PRE staging
+  uint32_t *tmem_holder = (uint32_t *)(st_empty + kMaxA);
   volatile int *abort = (volatile int *)(tmem_holder + 1);
 
-  auto a_hi = [&](int s) { return (float *)(sm + (size_t)s * kABytes); };
-  auto a_lo = [&](int s) { return (float *)(sm + (size_t)s * kABytes + 16384); };
+  auto a_hi = [&](int s) { return sm + (size_t)s * kABytes; };
   auto b_reg = [&](int s) { return ring_b + (size_t)s * a.b_bytes; };
   auto xt_reg = [&](int j) { return (float *)(ring_x + (size_t)j * a.x_bytes); };
+  auto stage = [&](int s) { return (const float *)(ring_s + (size_t)s * kStageBytes); };
 
   if (tid == 0) {
     for (int s = 0; s < kMaxA; ++s) {
       mbar_init(&a_full[s], kBldWarps);
       mbar_init(&a_empty[s], 1);
+      mbar_init(&st_full[s], 1);
+      mbar_init(&st_empty[s], kBldWarps);
     }
     for (int s = 0; s < kMaxB; ++s) {
       mbar_init(&b_full[s], 1);
@@ -335,12 +374,11 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       mbar_init(&x_full[j], 1);
       mbar_init(&x_empty[j], kBldWarps);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < kSlots; ++i) {
       mbar_init(&acc_full[i], 1);
       mbar_init(&acc_empty[i], kEpiWarps);
     }
     mbar_init(drain, 1);
-    for (int s = 0; s < kMaxA; ++s) mbar_init(&ahi_full[s], 1);
     *abort = 0;
     fence_mbar_init();
   }
@@ -353,6 +391,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
   pdl_wait();  // the fit's outputs (operand images, side input) are complete
+  const int units = a.tiles_total * m;
 
   if (warp == 0 || warp == kXtWarp) {
     // ------------------------------------------------------ producers (B / side input)
@@ -360,43 +399,51 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       const bool is_b = warp == 0;
       const int R = is_b ? SB : SX;
       uint64_t *full = is_b ? b_full : x_full, *empty = is_b ? b_empty : x_empty;
-      // PRE: the side-input producer also brings each A stage's K* image (the
-      // stage is free once the MMAs that read it have completed)
-      const bool with_a = PRE && !is_b;
-      uint32_t q = 0;
+      const bool with_st = PRE && !is_b;  // the side-input producer also stages K*
+      uint32_t q = 0, qa = 0;
       RingPos rp, ra;
       int last_q = -1, last_qa = -1;  // last jobs issued
-      for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
+      for (int unit = blockIdx.x; unit < units && !*abort; unit += gridDim.x) {
         const int tile = unit / m, t = unit % m;
-        const int b = tile / a.tiles_per_problem;
-        {
-          const int bt = b * m + t;
-          for (int p = 0; p < pl.npass && !*abort; ++p) {
-            const uint32_t bbytes = (uint32_t)(2 * pl.ncol[p] * 128);
-            for (int c = 0; c < pl.kc[p]; ++c, ++q, rp.advance(R), ra.advance(SA)) {
-              if (with_a) {
-                const int sa = ra.idx;
-                if (q >= (uint32_t)SA && !wait_or_abort(&a_empty[sa], ra.phase ^ 1u, abort)) break;
-                mbar_arrive_expect_tx(&ahi_full[sa], kABytes / 2);
-                bulk_g2s(a_hi(sa),
-                         a.kst + ((size_t)unit * pl.nchunk + c) * BOUTE_TILE_M * BOUTE_KCHUNK,
-                         kABytes / 2, &ahi_full[sa]);
-                last_qa = (int)q;
-              }
+        const int bt = (tile / a.tiles_per_problem) * m + t;
+        for (int g = 0; g < grp.n && !*abort; ++g) {
+          const int q0 = Groups::first(g), q1 = Groups::last(pl, g), kcg = pl.kc[q1];
+          for (int c = 0; c < kcg && !*abort; ++c) {
+            if (with_st) {  // the chunk's fp32 K* image
+              const int s = ra.idx;
+              if (qa >= (uint32_t)SA && !wait_or_abort(&st_empty[s], ra.phase ^ 1u, abort)) break;
+              mbar_arrive_expect_tx(&st_full[s], kStageBytes);
+              bulk_g2s((void *)stage(s),
+                       a.kst + ((size_t)unit * pl.nchunk + c) * (kStageBytes / 4), kStageBytes,
+                       &st_full[s]);
+              last_qa = (int)qa;
+              ++qa;
+              ra.advance(SA);
+            }
+            // B: one stage per block of the group that needs chunk c; side
+            // input: the chunk's two 32-point halves
+            const int jobs = is_b ? q1 - q0 + 1 : 2;
+            for (int job = 0; job < jobs; ++job) {
+              const int qb = q0 + job;
+              if (is_b && pl.kc[qb] <= c) continue;
               const int s = rp.idx;
               if (q >= (uint32_t)R && !wait_or_abort(&empty[s], rp.phase ^ 1u, abort)) break;
               if (is_b) {
-                mbar_arrive_expect_tx(&full[s], bbytes);
+                const int ncol = pl.ncol[qb];
+                const uint32_t bytes = (uint32_t)(2 * ncol * 128);
+                mbar_arrive_expect_tx(&full[s], bytes);
                 bulk_g2s(b_reg(s),
-                         a.bop + (size_t)bt * pl.image_floats + pl.off[p] +
-                             (size_t)c * 2 * pl.ncol[p] * BOUTE_KCHUNK,
-                         bbytes, &full[s]);
+                         a.bop + (size_t)bt * pl.image_halves + pl.off[qb] +
+                             (size_t)c * 2 * ncol * BOUTE_ACHUNK,
+                         bytes, &full[s]);
               } else {
-                mbar_arrive_expect_tx(&full[s], (uint32_t)(cf * 4));
-                bulk_g2s(xt_reg(s), a.xt + ((size_t)bt * pl.nchunk + c) * cf, (uint32_t)(cf * 4),
+                mbar_arrive_expect_tx(&full[s], a.x_bytes);
+                bulk_g2s(xt_reg(s), a.xt + ((size_t)bt * pl.nxt + 2 * c + job) * cf, a.x_bytes,
                          &full[s]);
               }
               last_q = (int)q;
+              ++q;
+              rp.advance(R);
             }
           }
         }
@@ -405,57 +452,56 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
         for (int j = std::max(0, last_q - R + 1); j <= last_q; ++j)
           mbar_wait(&full[j % R], (j / R) & 1);
         for (int j = std::max(0, last_qa - SA + 1); j <= last_qa; ++j)
-          mbar_wait(&ahi_full[j % SA], (j / SA) & 1);
+          mbar_wait(&st_full[j % SA], (j / SA) & 1);
       }
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      uint32_t q = 0, nuse[2] = {0u, 0u};
-      int nxt = 0;
+      // the block at position P of this CTA's sequence uses slot P % 4 for
+      // the (P / 4)-th time: it waits for that slot's previous use to drain
+      uint32_t blkseq = 0;
       bool issued = false;
       RingPos pa, pb;
-      for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
-        {
-          for (int p = 0; p < pl.npass && !*abort; ++p) {
-            const int kc = pl.kc[p], h = split_chunks(kc);
-            const bool split = h < kc;  // second half of the reduction -> other buffer
-            const int A = nxt, Bf = nxt ^ 1;
-            if (nuse[A] >= 1 && !wait_or_abort(&acc_empty[A], (nuse[A] - 1) & 1, abort)) break;
-            if (split && nuse[Bf] >= 1 &&
-                !wait_or_abort(&acc_empty[Bf], (nuse[Bf] - 1) & 1, abort))
-              break;
-            tc_fence_after();
-            const int ncol = pl.ncol[p];
-            const uint32_t idesc = idesc_tf32(ncol);
-            for (int c = 0; c < kc; ++c, ++q, pa.advance(SA), pb.advance(SB)) {
-              const bool second = split && c >= h;
-              const uint32_t dtm = tmem + (uint32_t)((second ? Bf : A) * 256);
-              const int c0 = second ? h : 0;  // first chunk of this accumulator
-              const int sa = pa.idx, sb = pb.idx;
+      for (int unit = blockIdx.x; unit < units && !*abort; unit += gridDim.x) {
+        for (int g = 0; g < grp.n && !*abort; ++g) {
+          const int q0 = Groups::first(g), q1 = Groups::last(pl, g), kcg = pl.kc[q1];
+          for (int c = 0; c < kcg && !*abort; ++c) {
+            const int sa = pa.idx;
+            if (!wait_or_abort(&a_full[sa], pa.phase, abort)) break;
+            const uint32_t sah = smem_u32(a_hi(sa)), sal = sah + kAPartBytes;
+            for (int qb = q0; qb <= q1; ++qb) {
+              if (pl.kc[qb] <= c) continue;
+              const uint32_t P = blkseq + (uint32_t)(qb - q0);
+              const int sl = (int)(P % kSlots);
+              if (c == 0 && P >= kSlots &&
+                  !wait_or_abort(&acc_empty[sl], (P / kSlots - 1) & 1, abort))
+                break;
+              const int sb = pb.idx;
               if (!wait_or_abort(&b_full[sb], pb.phase, abort)) break;
-              if (!wait_or_abort(&a_full[sa], pa.phase, abort)) break;
               tc_fence_after();
-              const uint32_t sah = smem_u32(a_hi(sa)), sal = smem_u32(a_lo(sa));
+              const int ncol = pl.ncol[qb];
+              const uint32_t idesc = idesc_f16(ncol);
+              const uint32_t dtm = tmem + (uint32_t)(sl * BOUTE_BLKCOLS);
               const uint32_t sbh = smem_u32(b_reg(sb)), sbl = sbh + ncol * 128;
 #pragma unroll
               for (int ks = 0; ks < 4; ++ks) {
                 const uint64_t dah = sdesc_sw128(sah + ks * 32), dal = sdesc_sw128(sal + ks * 32);
                 const uint64_t dbh = sdesc_sw128(sbh + ks * 32), dbl = sdesc_sw128(sbl + ks * 32);
-                mma_tf32(dtm, dah, dbh, idesc, (c > c0 || ks > 0) ? 1u : 0u);
-                mma_tf32(dtm, dah, dbl, idesc, 1u);
-                mma_tf32(dtm, dal, dbh, idesc, 1u);
+                mma_f16(dtm, dah, dbh, idesc, (c > 0 || ks > 0) ? 1u : 0u);
+                mma_f16(dtm, dah, dbl, idesc, 1u);
+                mma_f16(dtm, dal, dbh, idesc, 1u);
               }
-              mma_commit(&a_empty[sa]);
               mma_commit(&b_empty[sb]);
-              if (split && c == h - 1) mma_commit(&acc_full[A]);
+              pb.advance(SB);
+              if (c == pl.kc[qb] - 1) mma_commit(&acc_full[sl]);  // the block is complete
               issued = true;
             }
-            mma_commit(&acc_full[split ? Bf : A]);
-            ++nuse[A];
-            if (split) ++nuse[Bf];
-            else nxt ^= 1;
+            if (*abort) break;
+            mma_commit(&a_empty[sa]);
+            pa.advance(SA);
           }
+          blkseq += (uint32_t)(q1 - q0 + 1);
         }
       }
       if (issued) {  // every MMA of ours has completed before TMEM is released
@@ -466,111 +512,110 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   } else if (warp >= kEpiWarp0 && warp < kEpiWarp0 + kEpiWarps) {
     // ---------------------------------------------------------------- epilogue
     const int eq = warp & 3;  // TMEM lane quarter this warp may access
-    uint32_t nuse[2] = {0u, 0u};
-    int nxt = 0;
-    for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
+    uint32_t blkseq = 0;
+    const uint32_t lanes = (uint32_t)(32 * eq) << 16;
+    for (int unit = blockIdx.x; unit < units && !*abort; unit += gridDim.x) {
       const int tile = unit / m, t = unit % m;
       const int b = tile / a.tiles_per_problem;
       const long long row =
           (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M + 32 * eq + lane;
-      {
-        float ss = 0.f;
-        for (int p = 0; p < pl.npass; ++p) {
-          const int kc = pl.kc[p];
-          const bool split = split_chunks(kc) < kc;
-          const int A = nxt, Bf = nxt ^ 1;
-          if (!wait_or_abort(&acc_full[A], nuse[A] & 1, abort)) break;
-          if (split && !wait_or_abort(&acc_full[Bf], nuse[Bf] & 1, abort)) break;
+      float ss = 0.f;
+      for (int g = 0; g < grp.n && !*abort; ++g) {
+        const int q0 = Groups::first(g), q1 = Groups::last(pl, g);
+        for (int qb = q0; qb <= q1; ++qb) {
+          const uint32_t P = blkseq + (uint32_t)(qb - q0);
+          const int sl = (int)(P % kSlots);
+          if (!wait_or_abort(&acc_full[sl], (P / kSlots) & 1, abort)) break;
           tc_fence_after();
-          const uint32_t lanes = (uint32_t)(32 * eq) << 16;
-          const uint32_t ta = tmem + (uint32_t)(A * 256) + lanes;
-          const uint32_t tbb = tmem + (uint32_t)(Bf * 256) + lanes;
-          for (int cc = 0; cc < pl.ncol[p]; cc += 16) {
+          const uint32_t ta = tmem + (uint32_t)(sl * BOUTE_BLKCOLS) + lanes;
+          for (int cc = 0; cc < pl.ncol[qb]; cc += 16) {
             float v[16];
             tmem_ld16(ta + cc, v);
-            if (split) {  // V = first half + second half of the reduction
-              float w[16];
-              tmem_ld16(tbb + cc, w);
-#pragma unroll
-              for (int e = 0; e < 16; ++e) v[e] += w[e];
-            }
 #pragma unroll
             for (int e = 0; e < 16; ++e) ss = fmaf(v[e], v[e], ss);  // zero beyond n
           }
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) {
-            mbar_arrive_count(&acc_empty[A]);
-            if (split) mbar_arrive_count(&acc_empty[Bf]);
-          }
-          ++nuse[A];
-          if (split) ++nuse[Bf];
-          else nxt ^= 1;
+          if (lane == 0) mbar_arrive_count(&acc_empty[sl]);
         }
-        if (*abort) break;
-        if (row < a.N) {
-          float prior = a.s2f[b * m + t];
-          if (a.kern) {  // composite kernel: k(x, x) = s2 + s2_x + s2_c w(x)^2
-            const float *c0 = a.xt + (size_t)(b * m + t) * pl.nchunk * cf;
-            const float *bp = chunk_pref(c0, DP), *xrow = a.Xc + ((size_t)b * a.N + row) * d;
-            float e = 0.f;
-            for (int k = 0; k < d; ++k) e = fmaf(bp[k], xrow[k], e);
-            const float w = expf(e);
-            prior = fmaf(chunk_comp(c0, DP).s2c * w, w, prior);
-          }
-          const float vv = prior - ss;
-          a.var[((size_t)b * m + t) * a.N + row] = vv > 0.f ? vv : 0.f;
+        blkseq += (uint32_t)(q1 - q0 + 1);
+      }
+      if (*abort) break;
+      if (row < a.N) {
+        const float *par = a.xt + (size_t)(b * m + t) * pl.nxt * cf + xt_param_offset(DP) + 2 * DP;
+        float prior = a.s2f[b * m + t], ws = 0.f;
+        if (a.kern) {  // composite kernel: k(x, x) = s2 + s2_x + s2_c w(x)^2
+          const float *c0 = a.xt + (size_t)(b * m + t) * pl.nxt * cf;
+          const float *bp = chunk_pref(c0, DP), *xrow = a.Xc + ((size_t)b * a.N + row) * d;
+          float e = 0.f;
+          for (int k = 0; k < d; ++k) e = fmaf(bp[k], xrow[k], e);
+          ws = expf(e);
+          prior = fmaf(par[kParS2c] * ws, ws, prior);
         }
+        // V carries the scales 2^e_r (K*) and 2^e_W (W)
+        const int ex = row_exp(a.kern, par, ws) + (int)par[kParEW];
+        const float vv = prior - ldexpf(ss, -2 * ex);
+        a.var[((size_t)b * m + t) * a.N + row] = vv > 0.f ? vv : 0.f;
       }
     }
   } else if (warp >= kBldWarp0) {
     // ---------------------------------------------------------------- K* builders
-    // thread -> (row r, column group g): COLS consecutive columns of each chunk
+    // thread -> (row r, column group g): COLS consecutive columns of each half
     const int bw = warp - kBldWarp0;
     const int r = bw * RPW + lane % RPW, g = lane / RPW;
-    uint32_t q = 0;
     RingPos pa, px;
-    for (int unit = blockIdx.x; unit < a.tiles_total * m && !*abort; unit += gridDim.x) {
+    uint32_t qa = 0;
+    for (int unit = blockIdx.x; unit < units && !*abort; unit += gridDim.x) {
       const int tile = unit / m, t = unit % m;
       const int b = tile / a.tiles_per_problem;
       const long long row = (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M + r;
       float xr[DP];
-      if (!PRE) {
+      if (!PRE || KERN == 1) {
         const float *xrow = a.Xc + ((long long)b * a.N + row) * d;
 #pragma unroll
         for (int k = 0; k < DP; ++k) xr[k] = (k < d && row < a.N) ? xrow[k] : 0.f;
       }
-      {
-        unsigned long long xs2[DP];
-        float s2 = 0.f;
-        CompIn ci{};
-        float mu = 0.f, comp = 0.f;
-        for (int p = 0; p < pl.npass && !*abort; ++p) {
-          const bool last_pass = p == pl.npass - 1;
-          for (int c = 0; c < pl.kc[p]; ++c, ++q, pa.advance(SA), px.advance(SX)) {
-            const int s = pa.idx, j = px.idx;
-            if (PRE) {
-              if (!wait_or_abort(&ahi_full[s], pa.phase, abort)) break;
-            } else if (q >= (uint32_t)SA && !wait_or_abort(&a_empty[s], pa.phase ^ 1u, abort)) {
-              break;
-            }
+      unsigned long long xs2[DP];
+      float s2 = 0.f;
+      CompIn ci{};
+      int er = 0;
+      float mu = 0.f, comp = 0.f;
+      for (int gi = 0; gi < grp.n && !*abort; ++gi) {
+        const bool last_grp = gi == grp.n - 1;
+        const int kcg = pl.kc[Groups::last(pl, gi)];
+        for (int c = 0; c < kcg && !*abort; ++c, ++qa, pa.advance(SA)) {
+          const int s = pa.idx;
+          if (qa >= (uint32_t)SA && !wait_or_abort(&a_empty[s], pa.phase ^ 1u, abort)) break;
+          if (PRE && !wait_or_abort(&st_full[s], pa.phase, abort)) break;
+          uint8_t *Ah = a_hi(s), *Al = Ah + kAPartBytes;
+          float mu_part = 0.f;
+          for (int h = 0; h < 2; ++h, px.advance(SX)) {
+            const int j = px.idx;
             if (!wait_or_abort(&x_full[j], px.phase, abort)) break;
-            const float *xth = xt_reg(j), *xtl = xth + BOUTE_KCHUNK * DP;  // x hi, x lo
-            const float *alp = xtl + BOUTE_KCHUNK * DP;
-            if (!PRE && p == 0 && c == 0) {  // new objective: its parameters came with the chunk
+            const float *xth = xt_reg(j);
+            const float *alp = xth + 2 * BOUTE_KCHUNK * DP;
+            if (gi == 0 && c == 0 && h == 0) {  // new objective: its parameters came with the chunk
               const float *il = xth + xt_param_offset(DP);
-              scaled_candidate<DP>(xr, il, xs2);
-              s2 = il[2 * DP];
-              if (KERN == 1) {
-                ci = chunk_comp(xth, DP);
-                ci.ws = cand_weight<DP>(xr, chunk_pref(xth, DP));
+              const float *par = il + 2 * DP;
+              if (KERN == 1) ci = chunk_comp(xth, DP);
+              const float ws = KERN == 1 ? cand_weight<DP>(xr, chunk_pref(xth, DP)) : 0.f;
+              er = row_exp(KERN, par, ws);
+              if (!PRE) {
+                scaled_candidate<DP>(xr, il, xs2);
+                s2 = ldexpf(par[kParS2], er);
+                if (KERN == 1) {
+                  ci.ws = ws;
+                  ci.s2c = ldexpf(ci.s2c, er);
+                  ci.s2x = ldexpf(ci.s2x, er);
+                }
               }
             }
             float kv[COLS];
-            if (PRE) {  // this thread's COLS values of chunk c, from the stage's image
+            const int col0 = BOUTE_KCHUNK * h + COLS * g;  // first column within the chunk
+            if (PRE) {  // this thread's COLS values, from the staged fp32 image
 #pragma unroll
               for (int e = 0; e < COLS / 4; ++e) {
-                const float4 v = *(const float4 *)(a_hi(s) + sw128_off(r, COLS * g + 4 * e));
+                const float4 v = *(const float4 *)(stage(s) + st_off32(r, col0 + 4 * e));
                 kv[4 * e] = v.x;
                 kv[4 * e + 1] = v.y;
                 kv[4 * e + 2] = v.z;
@@ -579,58 +624,56 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
             } else {
               kstar_cols<DP, COLS, KERN>(xs2, xth, g, s2, kv, ci);
             }
-            const bool full_chunk = (c + 1) * BOUTE_KCHUNK <= n;
-            const int jbase = c * BOUTE_KCHUNK + COLS * g;
+            const int jbase = BOUTE_ACHUNK * c + col0;
             const float *alg = alp + COLS * g;
-            float mu_part = 0.f;
-            float *Ah = a_hi(s), *Al = a_lo(s);
-            // kernel values of this thread's COLS columns into the A stage; the
-            // last chunk of a ragged n zeroes the columns beyond n
+            // kernel values of this thread's COLS columns into the A stage as
+            // fp16 hi/lo; a ragged last half zeroes the columns beyond n
             auto emit = [&](auto ragged) {
 #pragma unroll
-              for (int g4 = 0; g4 < COLS / 4; ++g4) {
-                float vh[4], vl[4];
+              for (int u = 0; u < COLS / 8; ++u) {
+                uint32_t hi[4], lo[4];
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
-                  const int kk = 4 * g4 + e;
-                  float v = kv[kk];
-                  if (decltype(ragged)::value) v = (jbase + kk < n) ? v : 0.f;
-                  mu_part = fmaf(v, alg[kk], mu_part);
-                  // hi keeps the 19 bits the tensor core reads (it truncates an
-                  // fp32 operand to tf32); lo = v - hi exactly
-                  const float hi = __uint_as_float(__float_as_uint(v) & 0xFFFFE000u);
-                  vh[e] = hi;
-                  vl[e] = v - hi;
+                  const int kk = 8 * u + 2 * e;
+                  float v0 = kv[kk], v1 = kv[kk + 1];
+                  if (decltype(ragged)::value) {
+                    v0 = (jbase + kk < n) ? v0 : 0.f;
+                    v1 = (jbase + kk + 1 < n) ? v1 : 0.f;
+                  }
+                  mu_part = fmaf(v0, alg[kk], mu_part);
+                  mu_part = fmaf(v1, alg[kk + 1], mu_part);
+                  split_f16x2(v0, v1, hi[e], lo[e]);
                 }
-                const int o = sw128_off(r, COLS * g + g4 * 4);
-                // (PRE: the stage already holds the full values, which the
-                // tensor core reads as their hi parts)
-                if (!PRE) *(float4 *)(Ah + o) = make_float4(vh[0], vh[1], vh[2], vh[3]);
-                *(float4 *)(Al + o) = make_float4(vl[0], vl[1], vl[2], vl[3]);
+                const int o = sw128_off16(r, col0 + 8 * u) * 2;  // bytes
+                *(uint4 *)(Ah + o) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                *(uint4 *)(Al + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
               }
             };
-            if (full_chunk) emit(std::false_type{});
+            if (jbase + COLS <= n) emit(std::false_type{});
             else emit(std::true_type{});
-            fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) {
-              mbar_arrive_count(&a_full[s]);
-              mbar_arrive_count(&x_empty[j]);
-            }
-            if (last_pass) {  // Kahan: mu += mu_part (the last pass builds every chunk)
-              const float yk = mu_part - comp;
-              const float tk = mu + yk;
-              comp = (tk - mu) - yk;
-              mu = tk;
-            }
+            if (lane == 0) mbar_arrive_count(&x_empty[j]);
+          }
+          if (*abort) break;
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            mbar_arrive_count(&a_full[s]);
+            if (PRE) mbar_arrive_count(&st_empty[s]);
+          }
+          if (last_grp) {  // Kahan: mu += mu_part (the last group builds every chunk)
+            const float yk = mu_part - comp;
+            const float tk = mu + yk;
+            comp = (tk - mu) - yk;
+            mu = tk;
           }
         }
-        if (*abort) break;
-        float mt = mu - comp;  // sum over the GPR column groups of the row
-#pragma unroll
-        for (int o = RPW; o < 32; o <<= 1) mt += __shfl_xor_sync(0xffffffffu, mt, o);
-        if (g == 0 && row < a.N) a.mean[((size_t)b * m + t) * a.N + row] = mt;
       }
+      if (*abort) break;
+      float mt = mu - comp;  // sum over the GPR column groups of the row
+#pragma unroll
+      for (int o = RPW; o < 32; o <<= 1) mt += __shfl_xor_sync(0xffffffffu, mt, o);
+      if (g == 0 && row < a.N) a.mean[((size_t)b * m + t) * a.N + row] = ldexpf(mt, -er);
     }
   }
 
@@ -667,33 +710,39 @@ int launch_dp(const Gp *gp, const float *Xc, const float *kst, long long N, floa
   a.kern = gp->kern;
   a.tiles_per_problem = (int)((N + BOUTE_TILE_M - 1) / BOUTE_TILE_M);
   a.tiles_total = a.tiles_per_problem * gp->B;
-  const int ncolmax = gp->plan.ncol[0];
-  a.b_bytes = (uint32_t)(2 * ncolmax * 128);  // a multiple of 1024 (ncol % 16 == 0)
+  a.b_bytes = (uint32_t)(2 * gp->plan.ncol[0] * 128);  // block 0 is the widest
   a.x_bytes = (uint32_t)round_up(xt_chunk_floats(DP) * 4, 16);
   const size_t fixed = 1024 + 512;  // alignment slack, barriers, TMEM address, flag
   const size_t budget = 227 * 1024 - fixed;
-  // deepest B ring first (it hides the operand copies), then A, then the side input
+  const size_t st = kst ? kStageBytes : 0;  // staging beside each A stage (PRE)
+  // deep B ring first (a chunk feeds up to four blocks), then A, then the side input
   a.sx = kMaxX;
   a.sa = 3;
-  a.sb = kMaxB;
-  while ((size_t)a.sa * kABytes + (size_t)a.sb * a.b_bytes + (size_t)a.sx * a.x_bytes > budget) {
+  a.sb = 4;
+  while ((size_t)a.sa * (kABytes + st) + (size_t)a.sb * a.b_bytes + (size_t)a.sx * a.x_bytes >
+         budget) {
     if (a.sx > 4) --a.sx;
-    else if (a.sb > a.sa) --a.sb;
     else if (a.sa > 2) --a.sa;
     else if (a.sb > 2) --a.sb;
+    else if (a.sx > 2) --a.sx;
     else return BOUTE_ERR_UNSUPPORTED;
   }
-  const size_t smem =
-      fixed + (size_t)a.sa * kABytes + (size_t)a.sb * a.b_bytes + (size_t)a.sx * a.x_bytes;
+  const size_t smem = fixed + (size_t)a.sa * (kABytes + st) + (size_t)a.sb * a.b_bytes +
+                      (size_t)a.sx * a.x_bytes;
   const int grid = std::max(1, std::min(a.tiles_total * a.m, num_sms()));  // (tile, objective) units
   auto go = [&](auto kern) {
     prefer_shared(kern);
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     launch_pdl(kern, dim3(grid), dim3(Layout<DP>::kThreads), smem, s, a);
   };
-  if (kst) go(posterior_kernel<DP, true>);
-  else if (gp->kern) go(posterior_kernel<DP, false, 1>);
-  else go(posterior_kernel<DP, false>);
+  if (kst) {
+    if (gp->kern) go(posterior_kernel<DP, true, 1>);
+    else go(posterior_kernel<DP, true, 0>);
+  } else if (gp->kern) {
+    go(posterior_kernel<DP, false, 1>);
+  } else {
+    go(posterior_kernel<DP, false, 0>);
+  }
   count_launch();
   return last_launch_status();
 }
@@ -701,49 +750,72 @@ int launch_dp(const Gp *gp, const float *Xc, const float *kst, long long N, floa
 // ---- K* ahead of the fit's results ------------------------------------------------
 // One block per (tile, objective) unit, threads laid out as the posterior's
 // builders: all n training points' K* values of the tile's 128 candidates, in
-// the builders' arithmetic, zero beyond n. Each 32-point chunk is stored as
-// the 16 KB image of an A stage (128 rows x 32 fp32, K-major, 128-byte
-// swizzle), so that the posterior brings it in with one bulk copy; the tensor
-// core reads an fp32 operand truncated to tf32, so the full value serves as
-// the hi part. The training points' side input is staged in shared memory.
-// It needs the set-up's side input (not the fit's results) and the candidates.
+// the builders' arithmetic and scale (2^e_r), zero beyond n. Each 64-point
+// chunk is stored as a 32 KB fp32 image ([128 x 64], st_off32), which the
+// posterior brings in with one bulk copy and splits into its fp16 operand
+// parts. The training points' side input is staged in shared memory. It needs
+// the set-up's side input (not the fit's results) and the candidates.
 template <int DP, int KERN>
 __global__ void __launch_bounds__(Layout<DP>::kBld * 32) kstar_kernel(
     const float *Xc, const float *xt, long long N, int d, int m, int n, int tiles_per_problem,
-    int nchunk, float *kst) {
+    int nxt, float *kst) {
   constexpr int COLS = Layout<DP>::kCols, GPR = 32 / COLS, RPW = 32 / GPR;
-  extern __shared__ __align__(16) float xs[];  // nchunk side-input chunks
+  extern __shared__ __align__(16) float xs[];  // nxt side-input chunks
+  __shared__ float wmax_s;
   const int unit = blockIdx.x, tile = unit / m, t = unit % m, b = tile / tiles_per_problem;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = warp * RPW + lane % RPW, g = lane / RPW;
   const long long row = (long long)(tile % tiles_per_problem) * BOUTE_TILE_M + r;
   const int cf = xt_chunk_floats(DP);  // a multiple of 4
-  const float4 *x4 = (const float4 *)(xt + (size_t)(b * m + t) * nchunk * cf);
-  for (int e = threadIdx.x; e < nchunk * cf / 4; e += blockDim.x) ((float4 *)xs)[e] = x4[e];
+  const float4 *x4 = (const float4 *)(xt + (size_t)(b * m + t) * nxt * cf);
+  for (int e = threadIdx.x; e < nxt * cf / 4; e += blockDim.x) ((float4 *)xs)[e] = x4[e];
   const float *xrow = Xc + ((long long)b * N + row) * d;
   float xr[DP];
 #pragma unroll
   for (int k = 0; k < DP; ++k) xr[k] = (k < d && row < N) ? xrow[k] : 0.f;
   __syncthreads();
   const float *il = xs + xt_param_offset(DP);
+  float par[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) par[k] = il[2 * DP + k];
+  if (KERN == 1) {  // the largest training-point preference weight (as the fit finds it)
+    if (warp == 0) {
+      float wm = 0.f;
+      for (int j = lane; j < n; j += 32)
+        wm = fmaxf(wm, xs[(size_t)(j / BOUTE_KCHUNK) * cf + BOUTE_KCHUNK * DP + j % 32]);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
+      if (lane == 0) wmax_s = wm;
+    }
+    __syncthreads();
+    par[kParWmax] = wmax_s;
+  }
   unsigned long long xs2[DP];
   scaled_candidate<DP>(xr, il, xs2);
-  const float s2 = il[2 * DP];
   CompIn ci{};
+  float ws = 0.f;
   if (KERN == 1) {
     ci = chunk_comp(xs, DP);
-    ci.ws = cand_weight<DP>(xr, chunk_pref(xs, DP));
+    ws = cand_weight<DP>(xr, chunk_pref(xs, DP));
   }
-  for (int c = 0; c < nchunk; ++c) {
+  const int er = row_exp(KERN, par, ws);
+  const float s2 = ldexpf(par[kParS2], er);
+  if (KERN == 1) {
+    ci.ws = ws;
+    ci.s2c = ldexpf(ci.s2c, er);
+    ci.s2x = ldexpf(ci.s2x, er);
+  }
+  for (int c = 0; c < nxt; ++c) {  // 32-point halves
     float kv[COLS];
     kstar_cols<DP, COLS, KERN>(xs2, xs + (size_t)c * cf, g, s2, kv, ci);
     const int jbase = c * BOUTE_KCHUNK + COLS * g;
 #pragma unroll
     for (int kk = 0; kk < COLS; ++kk) kv[kk] = (jbase + kk < n) ? kv[kk] : 0.f;
-    float *img = kst + ((size_t)unit * nchunk + c) * BOUTE_TILE_M * BOUTE_KCHUNK;
+    float *img = kst + ((size_t)unit * (nxt / 2) + c / 2) * (kStageBytes / 4);
+    const int col0 = BOUTE_KCHUNK * (c & 1) + COLS * g;
 #pragma unroll
     for (int g4 = 0; g4 < COLS / 4; ++g4)
-      *(float4 *)(img + sw128_off(r, COLS * g + 4 * g4)) =
+      *(float4 *)(img + st_off32(r, col0 + 4 * g4)) =
           make_float4(kv[4 * g4], kv[4 * g4 + 1], kv[4 * g4 + 2], kv[4 * g4 + 3]);
   }
 }
@@ -752,7 +824,7 @@ template <int DP>
 int launch_kstar_dp(const Gp *gp, const float *Xc, long long N, float *kst, cudaStream_t s) {
   const int tpp = (int)((N + BOUTE_TILE_M - 1) / BOUTE_TILE_M);
   const int units = tpp * gp->B * gp->m;
-  const size_t smem = (size_t)gp->plan.nchunk * xt_chunk_floats(DP) * sizeof(float);
+  const size_t smem = (size_t)gp->plan.nxt * xt_chunk_floats(DP) * sizeof(float);
   auto go = [&](auto kern) {
     prefer_shared(kern);
     if (smem > 48 * 1024 &&
@@ -760,7 +832,7 @@ int launch_kstar_dp(const Gp *gp, const float *Xc, long long N, float *kst, cuda
             cudaSuccess)
       return last_launch_status();
     kern<<<units, Layout<DP>::kBld * 32, smem, s>>>(Xc, gp->xt, N, gp->d, gp->m, gp->n, tpp,
-                                                    gp->plan.nchunk, kst);
+                                                    gp->plan.nxt, kst);
     return (int)BOUTE_OK;
   };
   if (int r = gp->kern ? go(kstar_kernel<DP, 1>) : go(kstar_kernel<DP, 0>)) return r;
@@ -785,7 +857,7 @@ int launch_posterior(const Gp *gp, const float *Xc, long long N, float *mean, fl
 
 size_t kstar_floats(const Gp *gp, long long N) {
   const size_t tpp = (size_t)((N + BOUTE_TILE_M - 1) / BOUTE_TILE_M);
-  return tpp * gp->B * gp->m * gp->plan.nchunk * BOUTE_TILE_M * BOUTE_KCHUNK;
+  return tpp * gp->B * gp->m * gp->plan.nchunk * (kStageBytes / 4);
 }
 
 int launch_kstar(const Gp *gp, const float *Xc, long long N, float *kst, cudaStream_t s) {
