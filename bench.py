@@ -51,10 +51,10 @@ DEFAULT_WORKLOAD = wl.WORKLOADS[3].name
 METRIC = "candidates scored/sec (GP posterior + EHVI) at 1 GB300; % of roofline"
 UNIT = "candidates/s"
 # The posterior contraction's operand type and products per algorithmic
-# product: tf32 hi/lo operands, three tcgen05.mma per product (hi*hi + hi*lo +
-# lo*hi). Its peak is the measured bf16 peak times the nominal dense ratio of
-# the operand type to bf16 (tf32 1.1 : 2.25 PFLOP/s).
-CONTRACTION = {"dtype": "tf32", "products": 3, "per_bf16": 1.1 / 2.25}
+# product: fp16 hi/lo operands, three tcgen05.mma kind::f16 per product
+# (hi*hi + hi*lo + lo*hi). Its peak is the measured bf16 peak times the
+# nominal dense ratio of the operand type to bf16 (fp16 1 : 1).
+CONTRACTION = {"dtype": "f16", "products": 3, "per_bf16": 1.0}
 NUM_SMS = 152
 FMA_LANES_PER_SM = 128
 

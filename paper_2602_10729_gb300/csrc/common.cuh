@@ -65,12 +65,16 @@ __device__ __forceinline__ double outcome_transform(double y, int code) {
 
 // Floats of one training-point chunk of the posterior's side input: X/ls as
 // fp32 hi [DP][32] and lo [DP][32] (dimension-major, so pairs of training
-// points load as packed f32x2), alpha [32], then the objective's parameters
-// 1/ls hi [DP], 1/ls lo [DP], and 8 scalars (kParS2 .. below).
+// points load as packed f32x2), alpha as an fp32 pair, hi [32] and lo [32],
+// then the objective's parameters 1/ls hi [DP], 1/ls lo [DP], and 8 scalars
+// (kParS2 .. below).
 inline __host__ __device__ int xt_chunk_floats(int DP) {
-  return 2 * BOUTE_KCHUNK * DP + BOUTE_KCHUNK + 2 * DP + 8;
+  return 2 * BOUTE_KCHUNK * DP + 2 * BOUTE_KCHUNK + 2 * DP + 8;
 }
-inline __host__ __device__ int xt_param_offset(int DP) { return 2 * BOUTE_KCHUNK * DP + BOUTE_KCHUNK; }
+inline __host__ __device__ int xt_alpha_offset(int DP) { return 2 * BOUTE_KCHUNK * DP; }
+inline __host__ __device__ int xt_param_offset(int DP) {
+  return 2 * BOUTE_KCHUNK * DP + 2 * BOUTE_KCHUNK;
+}
 // The scalars after 1/ls hi and lo: outputscale; the composite kernel's s2_c,
 // s2_x and d_tau; the power-of-two exponent e_W of W's operand scale; the
 // composite kernel's largest training-point preference weight (written by the

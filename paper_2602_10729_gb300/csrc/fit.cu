@@ -267,7 +267,7 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
 // product with that inverse, W_pJ = -W_pp sum_{K=J}^{p-1} L_pK W_KJ, and the
 // trailing update uses 4 x 4 register tiles. fp32 arithmetic on the FP32
 // pipes: the fp32 factor is as accurate as the posterior needs, while alpha,
-// which carries the condition number, gets one step of iterative refinement
+// which carries the condition number, gets two steps of iterative refinement
 // against the fp64-accurate K = hi + lo with double-float residuals. A pivot
 // at or below 16 * eps32 times its original diagonal entry counts as not
 // positive. Matrix and inverse live in shared memory (row stride NP+1, NP = n
@@ -621,7 +621,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     if (lo_copy) mbar_wait(&lbar_lo, 0);  // let it land before the block exits
     return;
   }
-  // ---- alpha0 = W^T (W y), refined once against K = hi + lo ----------------------
+  // ---- alpha0 = W^T (W y), refined twice against K = hi + lo ---------------------
   // out = W^T (W rhs). Shared-memory variant: the 32 x 32 blocks (I >= J) of
   // W, one warp per block (the diagonal blocks hold zeros above the diagonal,
   // the padding the identity), with the block partial sums in the space of
@@ -714,132 +714,153 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     mbar_wait(&lbar_lo, 0);
     return;
   }
-  // residual r = y - K alpha0 in double-float. Shared-memory variant: one
-  // warp per 32 x 32 block (I, J) of K, lane = row, two independent chains per
-  // lane; K lo through its symmetry (K lo[k][i], conflict-free across the
-  // lanes), from shared memory when it fits there; K hi from the upper
-  // triangle of A: at (k, i) below the diagonal blocks, at (i, k) above them,
-  // each with one fixed load form (a per-entry choice of address costs more
-  // than the arithmetic), and in the diagonal blocks both loaded and the
-  // value selected, the diagonal from dg. Indices past n are clamped and
-  // alpha is zero there (padding), so those terms add exact zeros. The block
-  // partial sums (hi, lo) go to the space of colL and are added per row in a
-  // fixed order.
-  if (SMEM) {
-    float *ph = &colL[0][0], *pl = ph + nb * NP;  // nb x NP each
-    const float *Klsm = vec + 6 * NP;  // = Kls when kl_smem (shared-space pointer)
-    for (int e = warp; e < nb * nb; e += nw) {
-      const int I = e / nb, J = e - I * nb, ci = min(32 * I + lane, n - 1);
-      const float *alJ = al + 32 * J;
-      float sh[2] = {0.f, 0.f}, sl[2] = {0.f, 0.f};
-      auto run = [&](auto form, auto lo_smem) {
-        constexpr int F = decltype(form)::value;  // 0: below, 1: above, 2: diagonal block
-        constexpr bool LS = decltype(lo_smem)::value;
-        const float di = dg[ci];
-#pragma unroll 8
-        for (int kk = 0; kk < 32; ++kk) {
-          const int kc = min(32 * J + kk, n - 1);
-          float h;
-          if (F == 0) {
-            h = A[kc * ld + ci];
-          } else if (F == 1) {
-            h = A[ci * ld + kc];
-          } else {
-            const float x = A[kc * ld + ci], y = A[ci * ld + kc];
-            h = kc < ci ? x : y;
-            h = kc == ci ? di : h;
+  auto residual = [&]() {
+    // residual r = y - K alpha in double-float. Shared-memory variant: one
+    // warp per 32 x 32 block (I, J) of K, lane = row, two independent chains per
+    // lane; K lo through its symmetry (K lo[k][i], conflict-free across the
+    // lanes), from shared memory when it fits there; K hi from the upper
+    // triangle of A: at (k, i) below the diagonal blocks, at (i, k) above them,
+    // each with one fixed load form (a per-entry choice of address costs more
+    // than the arithmetic), and in the diagonal blocks both loaded and the
+    // value selected, the diagonal from dg. Indices past n are clamped and
+    // alpha is zero there (padding), so those terms add exact zeros. The block
+    // partial sums (hi, lo) go to the space of colL and are added per row in a
+    // fixed order.
+    if (SMEM) {
+      float *ph = &colL[0][0], *pl = ph + nb * NP;  // nb x NP each
+      const float *Klsm = vec + 6 * NP;  // = Kls when kl_smem (shared-space pointer)
+      for (int e = warp; e < nb * nb; e += nw) {
+        const int I = e / nb, J = e - I * nb, ci = min(32 * I + lane, n - 1);
+        const float *alJ = al + 32 * J;
+        float sh[2] = {0.f, 0.f}, sl[2] = {0.f, 0.f};
+        auto run = [&](auto form, auto lo_smem) {
+          constexpr int F = decltype(form)::value;  // 0: below, 1: above, 2: diagonal block
+          constexpr bool LS = decltype(lo_smem)::value;
+          const float di = dg[ci];
+  #pragma unroll 8
+          for (int kk = 0; kk < 32; ++kk) {
+            const int kc = min(32 * J + kk, n - 1);
+            float h;
+            if (F == 0) {
+              h = A[kc * ld + ci];
+            } else if (F == 1) {
+              h = A[ci * ld + kc];
+            } else {
+              const float x = A[kc * ld + ci], y = A[ci * ld + kc];
+              h = kc < ci ? x : y;
+              h = kc == ci ? di : h;
+            }
+            const float l = LS ? Klsm[kc * n + ci] : Kl[(size_t)kc * n + ci];
+            const float a = alJ[kk];  // zero from n on
+            float pr, er, s_, e2;
+            two_prod(h, a, pr, er);
+            two_sum(sh[kk & 1], pr, s_, e2);
+            sh[kk & 1] = s_;
+            sl[kk & 1] += e2 + fmaf(l, a, er);
           }
-          const float l = LS ? Klsm[kc * n + ci] : Kl[(size_t)kc * n + ci];
-          const float a = alJ[kk];  // zero from n on
-          float pr, er, s_, e2;
-          two_prod(h, a, pr, er);
-          two_sum(sh[kk & 1], pr, s_, e2);
-          sh[kk & 1] = s_;
-          sl[kk & 1] += e2 + fmaf(l, a, er);
+        };
+        auto pick = [&](auto lo_smem) {
+          if (I > J) run(std::integral_constant<int, 0>{}, lo_smem);
+          else if (I < J) run(std::integral_constant<int, 1>{}, lo_smem);
+          else run(std::integral_constant<int, 2>{}, lo_smem);
+        };
+        if (kl_smem) pick(std::true_type{});
+        else pick(std::false_type{});
+        float s_, e2;
+        two_sum(sh[0], sh[1], s_, e2);
+        ph[J * NP + 32 * I + lane] = s_;
+        pl[J * NP + 32 * I + lane] = (sl[0] + sl[1]) + e2;
+      }
+      __syncthreads();
+      for (int i = tid; i < NP; i += nthr) {
+        float sh = 0.f, sl = 0.f;
+        for (int J = 0; J < nb; ++J) {
+          float s_, e2;
+          two_sum(sh, ph[J * NP + i], s_, e2);
+          sh = s_;
+          sl += pl[J * NP + i] + e2;
         }
-      };
-      auto pick = [&](auto lo_smem) {
-        if (I > J) run(std::integral_constant<int, 0>{}, lo_smem);
-        else if (I < J) run(std::integral_constant<int, 1>{}, lo_smem);
-        else run(std::integral_constant<int, 2>{}, lo_smem);
-      };
-      if (kl_smem) pick(std::true_type{});
-      else pick(std::false_type{});
-      float s_, e2;
-      two_sum(sh[0], sh[1], s_, e2);
-      ph[J * NP + 32 * I + lane] = s_;
-      pl[J * NP + 32 * I + lane] = (sl[0] + sl[1]) + e2;
+        if (i < n) rv[i] = (yv[i] - sh) + (ylo[i] - sl);
+      }
+    } else {
+      // global variant: two rows per half warp at a time, all their loads
+      // issued before the arithmetic
+      const int half = lane >> 4, hl = lane & 15;
+      for (int i0 = 2 * warp + half; i0 < NP; i0 += 4 * nw) {
+        const int rows[2] = {i0, i0 + 2 * nw};
+        float sh[2] = {0.f, 0.f}, sl[2] = {0.f, 0.f};
+        for (int k0 = 0; k0 < n; k0 += 128) {
+          float h8[2][8], l8[2][8], a8[8];
+  #pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int k = k0 + hl + 16 * u;
+            a8[u] = k < n ? al[k] : 0.f;
+  #pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              const bool ok = k < n && rows[q] < n;
+              h8[q][u] = ok ? Kh[(size_t)rows[q] * n + k] : 0.f;
+              l8[q][u] = ok ? Kl[(size_t)rows[q] * n + k] : 0.f;
+            }
+          }
+  #pragma unroll
+          for (int q = 0; q < 2; ++q)
+  #pragma unroll
+            for (int u = 0; u < 8; ++u) {
+              float pr, e, s_, e2;
+              two_prod(h8[q][u], a8[u], pr, e);
+              two_sum(sh[q], pr, s_, e2);
+              sh[q] = s_;
+              sl[q] += e2 + fmaf(l8[q][u], a8[u], e);
+            }
+        }
+  #pragma unroll
+        for (int q = 0; q < 2; ++q) {
+  #pragma unroll
+          for (int o = 8; o > 0; o >>= 1) {  // within the half warp
+            const float oh = __shfl_xor_sync(FULL, sh[q], o);
+            const float ol = __shfl_xor_sync(FULL, sl[q], o);
+            float s_, e;
+            two_sum(sh[q], oh, s_, e);
+            sh[q] = s_;
+            sl[q] += ol + e;
+          }
+          if (hl == 0 && rows[q] < n) rv[rows[q]] = (yv[rows[q]] - sh[q]) + (ylo[rows[q]] - sl[q]);
+        }
+      }
+    }
+  };
+  // two refinement steps: alpha carries the condition number of K, and the
+  // posterior mean amplifies its error by sum_j |K*_j alpha_j| / |mean|
+  // The second correction is kept exactly: alpha = hi + lo, hi = fl(alpha +
+  // delta), lo its rounding error (in rv), for the posterior's fp64 path.
+  for (int step = 0; step < 2; ++step) {
+    residual();
+    for (int i = n + tid; i < NP; i += nthr) rv[i] = 0.f;
+    __syncthreads();
+    solve(rv, rv);
+    for (int k = tid; k < NP; k += nthr) {
+      if (step == 0) {
+        al[k] += rv[k];
+      } else {
+        float s_, e;
+        two_sum(al[k], rv[k], s_, e);
+        al[k] = s_;
+        rv[k] = e;
+      }
     }
     __syncthreads();
-    for (int i = tid; i < NP; i += nthr) {
-      float sh = 0.f, sl = 0.f;
-      for (int J = 0; J < nb; ++J) {
-        float s_, e2;
-        two_sum(sh, ph[J * NP + i], s_, e2);
-        sh = s_;
-        sl += pl[J * NP + i] + e2;
-      }
-      if (i < n) rv[i] = (yv[i] - sh) + (ylo[i] - sl);
-    }
-  } else {
-    // global variant: two rows per half warp at a time, all their loads
-    // issued before the arithmetic
-    const int half = lane >> 4, hl = lane & 15;
-    for (int i0 = 2 * warp + half; i0 < NP; i0 += 4 * nw) {
-      const int rows[2] = {i0, i0 + 2 * nw};
-      float sh[2] = {0.f, 0.f}, sl[2] = {0.f, 0.f};
-      for (int k0 = 0; k0 < n; k0 += 128) {
-        float h8[2][8], l8[2][8], a8[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int k = k0 + hl + 16 * u;
-          a8[u] = k < n ? al[k] : 0.f;
-#pragma unroll
-          for (int q = 0; q < 2; ++q) {
-            const bool ok = k < n && rows[q] < n;
-            h8[q][u] = ok ? Kh[(size_t)rows[q] * n + k] : 0.f;
-            l8[q][u] = ok ? Kl[(size_t)rows[q] * n + k] : 0.f;
-          }
-        }
-#pragma unroll
-        for (int q = 0; q < 2; ++q)
-#pragma unroll
-          for (int u = 0; u < 8; ++u) {
-            float pr, e, s_, e2;
-            two_prod(h8[q][u], a8[u], pr, e);
-            two_sum(sh[q], pr, s_, e2);
-            sh[q] = s_;
-            sl[q] += e2 + fmaf(l8[q][u], a8[u], e);
-          }
-      }
-#pragma unroll
-      for (int q = 0; q < 2; ++q) {
-#pragma unroll
-        for (int o = 8; o > 0; o >>= 1) {  // within the half warp
-          const float oh = __shfl_xor_sync(FULL, sh[q], o);
-          const float ol = __shfl_xor_sync(FULL, sl[q], o);
-          float s_, e;
-          two_sum(sh[q], oh, s_, e);
-          sh[q] = s_;
-          sl[q] += ol + e;
-        }
-        if (hl == 0 && rows[q] < n) rv[rows[q]] = (yv[rows[q]] - sh[q]) + (ylo[rows[q]] - sl[q]);
-      }
-    }
   }
-  for (int i = n + tid; i < NP; i += nthr) rv[i] = 0.f;
-  __syncthreads();
-  solve(rv, rv);
-  for (int k = tid; k < NP; k += nthr) al[k] += rv[k];
-  __syncthreads();
   // outputs: the operand images of W (packed here from shared memory; the
   // global variant leaves W in the workspace for pack_kernel), alpha into the
   // side input
   if (SMEM) pack_rows(NP - 32, NP, warp, nw);  // the last block row (the others: above)
   const int cf = xt_chunk_floats(DP);
-  float *xa = xt + (size_t)bt * plan.nxt * cf + 2 * BOUTE_KCHUNK * DP;
-  for (int k = tid; k < BOUTE_KCHUNK * plan.nxt; k += nthr)
-    xa[(size_t)(k / BOUTE_KCHUNK) * cf + k % BOUTE_KCHUNK] = k < n ? al[k] : 0.f;
+  float *xa = xt + (size_t)bt * plan.nxt * cf + xt_alpha_offset(DP);
+  for (int k = tid; k < BOUTE_KCHUNK * plan.nxt; k += nthr) {
+    float *q = xa + (size_t)(k / BOUTE_KCHUNK) * cf + k % BOUTE_KCHUNK;
+    q[0] = k < n ? al[k] : 0.f;
+    q[BOUTE_KCHUNK] = k < n ? rv[k] : 0.f;
+  }
   if (comp && warp == nw - 1) {  // the largest preference weight w_j (composite kernel)
     float *x0 = xt + (size_t)bt * plan.nxt * cf;
     const float *xw = x0 + BOUTE_KCHUNK * DP;

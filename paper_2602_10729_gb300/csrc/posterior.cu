@@ -105,6 +105,8 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 constexpr float kFiveThirds = 1.6666666666666667f;
+constexpr float kSqrt5Log2eLo = 1.1286310597e-07f;  // sqrt(5) / ln(2) - kSqrt5Log2e
+constexpr float kLn2 = 0.6931471805599453f;
 
 // ---- packed fp32 pairs (sm_100+ f32x2 arithmetic) --------------------------------
 __device__ __forceinline__ unsigned long long f2_dup(float x) {
@@ -122,6 +124,38 @@ __device__ __forceinline__ unsigned long long f2_fma(unsigned long long a, unsig
   unsigned long long r;
   asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
   return r;
+}
+__device__ __forceinline__ unsigned long long f2_add(unsigned long long a, unsigned long long b) {
+  unsigned long long r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ unsigned long long f2_mul(unsigned long long a, unsigned long long b) {
+  unsigned long long r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ unsigned long long f2_pack(float x, float y) {
+  unsigned long long r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(x), "f"(y));
+  return r;
+}
+// Compensated (Kahan) accumulation of packed pairs: s + c carries the sum
+// of the terms with the rounding error of every addition.
+struct Kahan2 {
+  unsigned long long s = 0ull, c = 0ull;
+  __device__ __forceinline__ void add(unsigned long long x) {
+    const unsigned long long y = f2_sub(x, c);
+    const unsigned long long t = f2_add(s, y);
+    c = f2_sub(f2_sub(t, s), y);
+    s = t;
+  }
+};
+// Error-free sum of two floats (Knuth).
+__device__ __forceinline__ void two_sum_f(float a, float b, float &s, float &e) {
+  s = a + b;
+  const float bb = s - a;
+  e = (a - (s - bb)) + (b - bb);
 }
 __device__ __forceinline__ void f2_split(unsigned long long v, float &x, float &y) {
   asm("mov.b64 {%0, %1}, %2;" : "=f"(x), "=f"(y) : "l"(v));
@@ -242,16 +276,25 @@ __device__ __forceinline__ void kstar_cols(const unsigned long long (&xs2)[DP], 
     }
     return;
   }
+  // packed pairs: k = (s2 + s2 sqrt5 r + s2 5/3 r^2) 2^A (1 + (a - A) ln 2), where
+  // a = -sqrt5 r / ln 2 is the exact exponent and A its fp32 rounding, which ex2
+  // takes: fma(r, K, A) recovers the rounding exactly, so the exponential is
+  // as accurate as ex2 itself at any r (the rounding of A alone is 2^-24 |a|)
+  const unsigned long long nK = f2_dup(-kSqrt5Log2e), pK = f2_dup(kSqrt5Log2e),
+                           pKlo = f2_dup(kSqrt5Log2eLo), nLn2 = f2_dup(-kLn2), c0 = f2_dup(s2),
+                           c1 = f2_dup(s2 * kSqrt5), c2 = f2_dup(s2 * kFiveThirds);
 #pragma unroll
   for (int e = 0; e < COLS / 2; ++e) {
-    float r2[2];
-    f2_split(acc2[e], r2[0], r2[1]);
-#pragma unroll
-    for (int z = 0; z < 2; ++z) {
-      const float rr = sqrt_approx(r2[z]);
-      const float sr = kSqrt5 * rr;
-      kv[2 * e + z] = s2 * fmaf(kFiveThirds, r2[z], 1.0f + sr) * ex2_approx(-kSqrt5Log2e * rr);
-    }
+    float ra, rb;
+    f2_split(acc2[e], ra, rb);
+    const unsigned long long rr = f2_pack(sqrt_approx(ra), sqrt_approx(rb));
+    const unsigned long long A = f2_mul(rr, nK);
+    float A0, A1;
+    f2_split(A, A0, A1);
+    const unsigned long long ex = f2_pack(ex2_approx(A0), ex2_approx(A1));
+    const unsigned long long q = f2_mul(f2_fma(rr, pKlo, f2_fma(rr, pK, A)), nLn2);  // (a - A) ln 2
+    const unsigned long long t = f2_mul(f2_fma(acc2[e], c2, f2_fma(rr, c1, c0)), ex);
+    f2_split(f2_fma(t, q, t), kv[2 * e], kv[2 * e + 1]);
   }
 }
 
@@ -307,6 +350,49 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t *bar, uint32_t parity,
       }
     }
   }
+}
+
+// The mean of a candidate is recomputed in fp64 when its terms K*_j alpha_j
+// add up to more than kFixRatio times the mean's scale max(|mean|, s): the
+// fp32 cross-covariance's rounding (a few units in the last place per entry,
+// amplified by that ratio) would otherwise exceed the 1e-5 tolerance. Below
+// the ratio the fp32 mean's error stays under about 6e-6 of the scale.
+constexpr float kFixRatio = 256.f;
+
+// A row's mean in fp64 for the Matern-5/2 kernel, computed by a whole warp
+// (lane = column j mod 32) and returned to every lane: the candidate's
+// coordinates scaled by 1/l as hi + lo, the training points' x / l as hi + lo
+// and alpha as hi + lo, read from the side input in global memory (the rare,
+// exact path; the warp takes one flagged row at a time).
+template <int DP>
+__device__ double mean_fp64_warp(const float *xrow, int d, const float *x0, int cf, int n,
+                                 int lane) {
+  const float *il = x0 + xt_param_offset(DP);
+  const double s2 = il[2 * DP + kParS2];
+  // lane k holds the candidate's coordinate k scaled by 1/l
+  const double xs_l = lane < d ? (double)xrow[lane] * ((double)il[lane] + (double)il[DP + lane]) : 0.0;
+  double acc = 0.0;
+  for (int j0 = 0; j0 < n; j0 += 32) {
+    const int j = j0 + lane;
+    const float *ch = x0 + (size_t)(min(j, n - 1) / BOUTE_KCHUNK) * cf;
+    const int jj = j % BOUTE_KCHUNK;
+    double r2 = 0.0;
+    for (int k = 0; k < d; ++k) {
+      const double xs = __shfl_sync(0xffffffffu, xs_l, k);
+      const double df =
+          xs - ((double)ch[k * BOUTE_KCHUNK + jj] + (double)ch[(DP + k) * BOUTE_KCHUNK + jj]);
+      r2 = fma(df, df, r2);
+    }
+    if (j >= n) continue;
+    const double r = sqrt(r2);
+    const double kv = s2 * (1.0 + 2.2360679774997896964 * r + (5.0 / 3.0) * r2) *
+                      exp(-2.2360679774997896964 * r);
+    const float *al = ch + xt_alpha_offset(DP) + jj;  // alpha hi, lo
+    acc = fma(kv, (double)al[0] + (double)al[BOUTE_KCHUNK], acc);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  return acc;
 }
 
 // The work sequence every role follows: per unit (tile, objective), the
@@ -579,7 +665,12 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       float s2 = 0.f;
       CompIn ci{};
       int er = 0;
-      float mu = 0.f, comp = 0.f;
+      // the mean K* alpha: its terms reach hundreds of times the result when K
+      // is ill-conditioned, so they are summed with compensation, and their
+      // magnitudes sum_j K*_j |alpha_j| decide whether the row needs the fp64 path
+      Kahan2 mu2;
+      unsigned long long mag2 = 0ull;
+      float sc = 0.f;  // the mean's scale sqrt(s2), scaled like K*
       for (int gi = 0; gi < grp.n && !*abort; ++gi) {
         const bool last_grp = gi == grp.n - 1;
         const int kcg = pl.kc[Groups::last(pl, gi)];
@@ -588,18 +679,18 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
           if (qa >= (uint32_t)SA && !wait_or_abort(&a_empty[s], pa.phase ^ 1u, abort)) break;
           if (PRE && !wait_or_abort(&st_full[s], pa.phase, abort)) break;
           uint8_t *Ah = a_hi(s), *Al = Ah + kAPartBytes;
-          float mu_part = 0.f;
           for (int h = 0; h < 2; ++h, px.advance(SX)) {
             const int j = px.idx;
             if (!wait_or_abort(&x_full[j], px.phase, abort)) break;
             const float *xth = xt_reg(j);
-            const float *alp = xth + 2 * BOUTE_KCHUNK * DP;
+            const float *alp = xth + xt_alpha_offset(DP);
             if (gi == 0 && c == 0 && h == 0) {  // new objective: its parameters came with the chunk
               const float *il = xth + xt_param_offset(DP);
               const float *par = il + 2 * DP;
               if (KERN == 1) ci = chunk_comp(xth, DP);
               const float ws = KERN == 1 ? cand_weight<DP>(xr, chunk_pref(xth, DP)) : 0.f;
               er = row_exp(KERN, par, ws);
+              sc = ldexpf(sqrtf(par[kParS2]), er);
               if (!PRE) {
                 scaled_candidate<DP>(xr, il, xs2);
                 s2 = ldexpf(par[kParS2], er);
@@ -640,8 +731,12 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
                     v0 = (jbase + kk < n) ? v0 : 0.f;
                     v1 = (jbase + kk + 1 < n) ? v1 : 0.f;
                   }
-                  mu_part = fmaf(v0, alg[kk], mu_part);
-                  mu_part = fmaf(v1, alg[kk + 1], mu_part);
+                  if (last_grp) {  // (the last group builds every chunk)
+                    const unsigned long long v2 = f2_pack(v0, v1);
+                    const unsigned long long a2 = *(const unsigned long long *)(alg + kk);
+                    mu2.add(f2_mul(v2, a2));
+                    mag2 = f2_fma(v2, a2 & 0x7fffffff7fffffffull, mag2);  // (K* >= 0)
+                  }
                   split_f16x2(v0, v1, hi[e], lo[e]);
                 }
                 const int o = sw128_off16(r, col0 + 8 * u) * 2;  // bytes
@@ -661,19 +756,44 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
             mbar_arrive_count(&a_full[s]);
             if (PRE) mbar_arrive_count(&st_empty[s]);
           }
-          if (last_grp) {  // Kahan: mu += mu_part (the last group builds every chunk)
-            const float yk = mu_part - comp;
-            const float tk = mu + yk;
-            comp = (tk - mu) - yk;
-            mu = tk;
-          }
         }
       }
       if (*abort) break;
-      float mt = mu - comp;  // sum over the GPR column groups of the row
+      // the thread's sum as a float pair (hi, lo), then the GPR column groups
+      // of the row added with error-free sums
+      float se, so, ce, co, hi, lo;
+      f2_split(mu2.s, se, so);
+      f2_split(mu2.c, ce, co);
+      two_sum_f(se, so, hi, lo);
+      lo -= ce + co;
+      float me, mo;
+      f2_split(mag2, me, mo);
+      float mag = me + mo;
 #pragma unroll
-      for (int o = RPW; o < 32; o <<= 1) mt += __shfl_xor_sync(0xffffffffu, mt, o);
-      if (g == 0 && row < a.N) a.mean[((size_t)b * m + t) * a.N + row] = ldexpf(mt, -er);
+      for (int o = RPW; o < 32; o <<= 1) {
+        const float oh = __shfl_xor_sync(0xffffffffu, hi, o);
+        const float ol = __shfl_xor_sync(0xffffffffu, lo, o);
+        float e;
+        two_sum_f(hi, oh, hi, e);
+        lo += ol + e;
+        mag += __shfl_xor_sync(0xffffffffu, mag, o);
+      }
+      float mean = ldexpf(hi + lo, -er);
+      if (KERN == 0) {  // ill-conditioned rows: the mean in fp64, one row at a time
+        const bool fix = g == 0 && row < a.N && mag > kFixRatio * fmaxf(fabsf(hi), sc);
+        unsigned todo = __ballot_sync(0xffffffffu, fix);
+        while (todo) {
+          const int src = __ffs(todo) - 1;
+          todo &= todo - 1;
+          const long long rr = (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M +
+                               bw * RPW + src % RPW;
+          const float *x0 = a.xt + (size_t)(b * m + t) * pl.nxt * xt_chunk_floats(DP);
+          const double v = mean_fp64_warp<DP>(a.Xc + ((long long)b * a.N + rr) * d, d, x0,
+                                              xt_chunk_floats(DP), n, lane);
+          if (lane == src) mean = (float)v;
+        }
+      }
+      if (g == 0 && row < a.N) a.mean[((size_t)b * m + t) * a.N + row] = mean;
     }
   }
 

@@ -80,10 +80,9 @@ def test_dimensions(d):
 
 def test_ill_conditioned_problem_meets_fp32_error_bound():
     """40 points on a line with lengthscale 0.3: cond(K) ~ 2e5, |alpha| ~ 1e3.
-    The fp32-accurate path cannot give 1e-5 relative there; it must stay
-    within the error bound of fp32 dot products, a small multiple of
-    eps32 * sum_j |K*_j alpha_j| for the mean (and of eps32 * s2 * cond-scaled
-    terms for the variance)."""
+    The mean meets 1e-5 (its ill-conditioned rows take the fp64 path); the
+    variance s2 - ||L^-1 k*||^2 must stay within the error bound of an
+    fp32-accurate contraction, eps32 * s2 times cond-scaled terms."""
     hp = rand_problem(12, 40, 1, 2, 300)
     g = gpu_pipeline(hp)
     assert g["status"] == 0
@@ -93,8 +92,7 @@ def test_ill_conditioned_problem_meets_fp32_error_bound():
     for t in range(2):
         Ks = np.array([[oracle.matern52(c.astype(np.float64), x, hp.ls[0][t], hp.s2[0][t])
                         for x in hp.X[0]] for c in hp.Xc[0]])
-        bound_mu = 64 * eps32 * (np.abs(Ks) @ np.abs(fp.alpha[t])) + 1e-5
-        assert np.all(np.abs(g["mean"][0, t] - mean[:, t]) <= bound_mu)
+        check_mean(g["mean"][0, t], mean[:, t], fp.s2[t])
         W = np.linalg.inv(fp.L[t])
         v = Ks @ W.T
         bound_v = 64 * eps32 * 2 * (np.abs(v) * (np.abs(Ks) @ np.abs(W.T))).sum(1) + 1e-5
@@ -163,22 +161,24 @@ def test_candidates_on_training_points():
 
 
 def test_per_objective_hyperparameters():
+    """Per-objective lengthscales over an order of magnitude and noise down to
+    1e-5: sum_j |K*_j alpha_j| reaches about 220 times the mean's scale, and
+    the mean must still meet 1e-5 (the fp32 K* with its exponent-rounding
+    correction and compensated sums)."""
     rng = np.random.default_rng(8)
     hp = rand_problem(9, 70, 5, 2, 333)
-    hp.ls[0] = rng.uniform(0.2, 0.6, (2, 5))
+    hp.ls[0] = rng.uniform(0.1, 1.5, (2, 5))
     hp.s2[0] = [0.5, 2.5]
-    hp.noise[0] = [1e-3, 1e-4]
+    hp.noise[0] = [1e-3, 1e-5]
     compare(hp)
 
 
-@pytest.mark.parametrize("ls_range,noise", [((0.1, 1.5), (1e-3, 1e-5)), ((0.3, 1.5), (1e-3, 1e-4))])
-def test_ill_conditioned_mean_meets_fp32_error_bound(ls_range, noise):
-    """Long lengthscales (or tiny noise) over 70 points in 5-D: the mean K*
-    alpha cancels, sum_j |K*_j alpha_j| reaching 200-270 times its scale, so
-    fp32 K* entries (relative error a few eps32) cannot give 1e-5 relative.
-    The mean must stay within a small multiple of eps32 * sum_j |K*_j alpha_j|,
-    the forward error bound of an fp32-accurate cross-covariance; the variance
-    keeps the 1e-5 tolerance."""
+@pytest.mark.parametrize("ls_range,noise", [((0.3, 1.5), (1e-3, 1e-4)), ((0.5, 2.0), (1e-3, 1e-5)),
+                                            ((0.1, 1.5), (1e-5, 1e-6))])
+def test_ill_conditioned_means(ls_range, noise):
+    """Longer lengthscales or smaller noise: sum_j |K*_j alpha_j| reaches 270
+    to 590 times the mean's scale. Rows beyond 256 times take the fp64 path;
+    mean and variance meet 1e-5 everywhere."""
     rng = np.random.default_rng(8)
     hp = rand_problem(9, 70, 5, 2, 333)
     hp.ls[0] = rng.uniform(*ls_range, (2, 5))
@@ -188,12 +188,8 @@ def test_ill_conditioned_mean_meets_fp32_error_bound(ls_range, noise):
     assert g["status"] == 0
     fp = opl.fit_problem(hp.X[0], hp.Y[0], hp.ls[0], hp.s2[0], hp.noise[0], hp.ref[0])
     mean, var = opl.posterior(fp, hp.Xc[0])
-    eps32 = np.finfo(np.float32).eps
     for t in range(2):
-        Ks = np.array([[oracle.matern52(c.astype(np.float64), x, hp.ls[0][t], hp.s2[0][t])
-                        for x in hp.X[0]] for c in hp.Xc[0]])
-        bound_mu = 16 * eps32 * (np.abs(Ks) @ np.abs(fp.alpha[t])) + 1e-5 * np.sqrt(hp.s2[0][t])
-        assert np.all(np.abs(g["mean"][0, t] - mean[:, t]) <= bound_mu)
+        check_mean(g["mean"][0, t], mean[:, t], fp.s2[t])
         check_var(g["var"][0, t], var[:, t], fp.s2[t])
 
 
