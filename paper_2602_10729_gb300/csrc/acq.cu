@@ -112,6 +112,75 @@ __global__ void __launch_bounds__(256) ehvi2d_kernel(const float *mean, const fl
 // sum_k prod_t (u_kt - max(l_kt, y_t))_+.
 // CONS: a sample with some y_t above its threshold (cons: B x M) counts zero
 // (its first coordinate is moved beyond every box).
+//
+// With S a multiple of 128 up to 256 every lane holds its 4 S / 128 samples
+// of the candidate in registers, and each box is visited once per candidate:
+// its lower bounds are raised to the candidate's smallest sample per
+// objective (no sample lies below them), which makes every box finite,
+// w_t = u_t - l'_t, and a box with some w_t <= 0 (every sample at or above
+// its upper bound) is skipped by the whole warp; otherwise each sample adds
+// prod_t w_t * prod_t sat((u_t - y_t) / w_t), since (u - max(l', y))_+ =
+// w sat((u - y) / w) for y >= l': one saturating fma per objective.
+template <int M, bool CONS, int NV>
+__device__ __forceinline__ float mc_hvi_regs(const float *e, int S, const float (&mu)[M],
+                                             const float (&sg)[M], const float (&kc)[M],
+                                             const float *lo, const float *hi, int K, int lane) {
+  constexpr int NS = 4 * NV;
+  float y[NS][M];
+#pragma unroll
+  for (int v = 0; v < NV; ++v)
+#pragma unroll
+    for (int t = 0; t < M; ++t) {
+      const float4 z = __ldcs((const float4 *)(e + (size_t)t * S + 128 * v + 4 * lane));
+      y[4 * v][t] = fmaf(sg[t], z.x, mu[t]);
+      y[4 * v + 1][t] = fmaf(sg[t], z.y, mu[t]);
+      y[4 * v + 2][t] = fmaf(sg[t], z.z, mu[t]);
+      y[4 * v + 3][t] = fmaf(sg[t], z.w, mu[t]);
+    }
+  float ymin[M];
+#pragma unroll
+  for (int t = 0; t < M; ++t) {
+    float v = y[0][t];
+#pragma unroll
+    for (int j = 1; j < NS; ++j) v = fminf(v, y[j][t]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    ymin[t] = v;
+  }
+  if (CONS) {
+#pragma unroll
+    for (int j = 0; j < NS; ++j) {
+      bool ok = true;
+#pragma unroll
+      for (int t = 0; t < M; ++t) ok = ok && y[j][t] <= kc[t];
+      if (!ok) y[j][0] = kInfeasible;
+    }
+  }
+  float sum = 0.f;
+  for (int k = 0; k < K; ++k) {
+    float iw[M], hw[M], W = 1.f;
+    bool live = true;
+#pragma unroll
+    for (int t = 0; t < M; ++t) {
+      const float h = hi[k * M + t];
+      const float w = h - fmaxf(lo[k * M + t], ymin[t]);
+      live = live && w > 0.f;
+      iw[t] = __frcp_rn(w);
+      hw[t] = h * iw[t];
+      W *= w;
+    }
+    if (!live) continue;  // (uniform: the box and ymin are the warp's)
+#pragma unroll
+    for (int j = 0; j < NS; ++j) {
+      float p = fma_sat(-y[j][0], iw[0], hw[0]);
+#pragma unroll
+      for (int t = 1; t < M; ++t) p *= fma_sat(-y[j][t], iw[t], hw[t]);
+      sum = fmaf(W, p, sum);
+    }
+  }
+  return sum;
+}
+
 template <int M, bool CONS>
 __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const float *var, int B,
                                                     long long N, const float *lower,
@@ -145,7 +214,11 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
     const float *e = eps + ((size_t)b * N + c) * eps_stride +
                      (eps_stride == 0 ? (size_t)b * M * S : 0);
     float sum = 0.f;
-    if (vec) {
+    if (vec && S == 256) {
+      sum = mc_hvi_regs<M, CONS, 2>(e, S, mu, sg, kc, lo, hi, K, lane);
+    } else if (vec && S == 128) {
+      sum = mc_hvi_regs<M, CONS, 1>(e, S, mu, sg, kc, lo, hi, K, lane);
+    } else if (vec) {
       for (int s0 = 4 * lane; s0 < S; s0 += 128) {
         float4 z[M];
 #pragma unroll
