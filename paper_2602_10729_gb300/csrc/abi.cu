@@ -193,6 +193,10 @@ int boute_gp_create(int B, int n, int d, int m, boute_gp **out) {
   r |= dalloc(&g.Aws, BM * np * (np + 1));
   r |= dalloc(&g.Wws, BM * np * (np + 1));
   r |= dalloc(&g.bop, BM * (size_t)g.plan.image_halves);
+  g.kcache_chunks = kstar_cache_chunks(g.plan);
+  g.kcache_sms = num_sms();
+  if (g.kcache_chunks > 0)
+    r |= dalloc(&g.kcache, (size_t)g.kcache_sms * g.kcache_chunks * kKstarChunkHalves);
   r |= dalloc(&g.xt, BM * (size_t)g.plan.nxt * xt_chunk_floats(g.DP));
   r |= dalloc(&g.s2f, BM);
   r |= dalloc(&g.status, 1);
@@ -232,7 +236,7 @@ void boute_gp_free(boute_gp *gp) {
   if (!gp) return;
   Gp &g = gp->g;
   cudaFree(g.Kh); cudaFree(g.Kl); cudaFree(g.Aws); cudaFree(g.Wws); cudaFree(g.bop); cudaFree(g.xt);
-  cudaFree(g.s2f); cudaFree(g.status); cudaFree(g.kpar);
+  cudaFree(g.s2f); cudaFree(g.status); cudaFree(g.kpar); cudaFree(g.kcache);
   delete gp;
 }
 

@@ -23,18 +23,29 @@ constexpr float kInvSqrt2 = 0.7071067811865476f;
 // the difference itself cancels (gm ~ phi(t) / t^2), so for t >= 3 it is
 // taken from Laplace's continued fraction of the Mills ratio Phi(-t) / phi(t)
 // = 1 / x_0, x_k = t + (k + 1) / x_{k+1}: gm = phi(t) (1 - t / x_0) =
-// phi(t) / (x_0 x_1), without cancellation; twelve terms are within 1e-6 of
-// it for t >= 3 (and the rounding of t^2 in phi's exponent is recovered by an
-// fma). |z| is capped where gm is already zero, so that infinite z gives 0.
+// phi(t) / (x_0 x_1). Truncated at x_12 = t, the fraction is the rational
+// function P(t^2) / Q(t^2) below (positive coefficients, no cancellation),
+// within 1.2e-6 of gm / phi for t >= 3. The rounding of t^2 in phi's
+// exponent is recovered by an fma. |z| is capped where gm is already zero,
+// so that infinite z gives 0, not NaN.
 __device__ __forceinline__ float gm(float z) {
   const float t = fminf(fabsf(z), 1.0e4f);
   const float h = t * t, l = fmaf(t, t, -h);  // t^2 = h + l exactly
   const float phi = expf(-0.5f * h) * fmaf(-0.5f, l, 1.0f) * kInvSqrt2Pi;
   if (t < 3.0f) return phi - t * (0.5f * erfcf(t * kInvSqrt2));
-  float x = t;
-#pragma unroll
-  for (int k = 11; k >= 1; --k) x = t + (float)(k + 1) / x;  // x_1 after the loop
-  return phi / (fmaf(1.0f, t, 1.0f / x) * x);
+  if (t >= 14.0f) return 0.f;  // (phi(14) is below the fp32 range)
+  float p = h + 75.f;
+  p = fmaf(p, h, 1926.f);
+  p = fmaf(p, h, 20370.f);
+  p = fmaf(p, h, 82845.f);
+  p = fmaf(p, h, 89055.f);
+  float q = h + 78.f;
+  q = fmaf(q, h, 2145.f);
+  q = fmaf(q, h, 25740.f);
+  q = fmaf(q, h, 135135.f);
+  q = fmaf(q, h, 270270.f);
+  q = fmaf(q, h, 135135.f);
+  return phi * __fdividef(p, q);
 }
 
 __device__ __forceinline__ float std_cdf(float z) { return 0.5f * erfcf(-z * kInvSqrt2); }

@@ -17,6 +17,10 @@ struct Gp {
   float *Aws;      // B*m x np x (np+1): factorisation workspace (large n; np = npad)
   float *Wws;      // B*m x np x (np+1): L^-1 (lower, row stride np+1)
   uint16_t *bop;  // B*m x plan.image_halves: L^-1 as fp16 hi/lo operand images
+  // the posterior's cache of K* chunks that later groups of output blocks
+  // need again (n > 512): kcache_chunks fp16 A-stage images per SM
+  uint16_t *kcache;
+  int kcache_chunks, kcache_sms;
   float *xt;      // B*m x nxt x xt_chunk_floats(DP): X/lengthscale hi/lo, alpha
   float *s2f;     // B*m: outputscale
   int *status;    // device status word (first error wins)
@@ -82,6 +86,11 @@ int launch_fit(Gp *gp, const double *X, const double *Ys, const double *ls, cons
 // kst: K* precomputed by launch_kstar (the posterior then builds no K*), or null.
 int launch_posterior(const Gp *gp, const float *Xc, long long N, float *mean, float *var,
                      cudaStream_t s, const float *kst = nullptr);
+// Chunks of K* per CTA that the posterior caches across groups of output
+// blocks (0 when every chunk is needed by one group only).
+int kstar_cache_chunks(const PostPlan &plan);
+// fp16 halves of one cached chunk (an A stage: 128 x 64 hi and lo)
+constexpr size_t kKstarChunkHalves = 2 * BOUTE_TILE_M * BOUTE_ACHUNK;
 // K* of all candidates, per (128-candidate tile, objective) and 64-point chunk
 // as the fp16 hi and lo images of an A stage (128 x 64 each, scaled by the
 // row's 2^e_r): kstar_floats(gp, N) 4-byte words. Reads the fit set-up's side

@@ -77,6 +77,11 @@ struct PostArgs {
   int sa, sb, sx;              // depths of the A (and staging), B and side-input rings
   uint32_t b_bytes, x_bytes;   // one B stage, one side-input entry
   int kern;                    // 1: the composite kernel (prior variance per candidate)
+  // K* chunks built by one group and needed again by later groups: kept as
+  // their fp16 A-stage images in this CTA's slots of kcache (ncache chunks
+  // per CTA, 0 = rebuilt instead)
+  uint16_t *kcache;
+  int ncache;
   PostPlan plan;
 };
 
@@ -404,6 +409,20 @@ struct Groups {
   __device__ __forceinline__ static int last(const PostPlan &p, int g) {
     return min(p.nblk, (g + 1) * kGroup) - 1;
   }
+  // chunks [0, prev(g)) were built by an earlier group
+  __device__ __forceinline__ static int prev(const PostPlan &p, int g) {
+    return g > 0 ? p.kc[last(p, g - 1)] : 0;
+  }
+  // The chunk at position i of a group's sequence of kcg chunks. With cached
+  // chunks (mix) the new chunks [kcp, kcg) alternate with the cached ones
+  // [0, kcp), so that the builders always have a chunk to build while the
+  // tensor cores work through the cached ones; otherwise in order.
+  __device__ __forceinline__ static int chunk_at(int i, int kcp, int kcg, bool mix) {
+    if (!mix) return i;
+    const int nb = kcg - kcp, m = min(nb, kcp);
+    if (i < 2 * m) return (i & 1) ? (i >> 1) : kcp + (i >> 1);
+    return nb > kcp ? kcp + (i - m) : i - m;
+  }
 };
 
 // PRE: the K* values come precomputed (kstar_kernel, scaled fp32 images)
@@ -437,7 +456,8 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   uint64_t *acc_full = x_full + 2 * kMaxX, *acc_empty = acc_full + kSlots;
   uint64_t *drain = acc_empty + kSlots;
   uint64_t *st_full = drain + 1, *st_empty = st_full + kMaxA;  // PRE staging
-  uint32_t *tmem_holder = (uint32_t *)(st_empty + kMaxA);
+  uint64_t *cache_ready = st_empty + kMaxA;  // a group's K* chunks are stored
+  uint32_t *tmem_holder = (uint32_t *)(cache_ready + 1);
   volatile int *abort = (volatile int *)(tmem_holder + 1);
 
   auto a_hi = [&](int s) { return sm + (size_t)s * kABytes; };
@@ -465,6 +485,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       mbar_init(&acc_empty[i], kEpiWarps);
     }
     mbar_init(drain, 1);
+    mbar_init(cache_ready, 1);
     *abort = 0;
     fence_mbar_init();
   }
@@ -486,15 +507,42 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       const int R = is_b ? SB : SX;
       uint64_t *full = is_b ? b_full : x_full, *empty = is_b ? b_empty : x_empty;
       const bool with_st = PRE && !is_b;  // the side-input producer also stages K*
-      uint32_t q = 0, qa = 0;
+      // ... and brings cached K* chunks into their A stages
+      const bool with_cache = !is_b && a.ncache > 0;
+      uint32_t q = 0, qa = 0, nready = 0;
       RingPos rp, ra;
       int last_q = -1, last_qa = -1;  // last jobs issued
+      int last_ca = -1;               // last cached-chunk copy (A ring position)
       for (int unit = blockIdx.x; unit < units && !*abort; unit += gridDim.x) {
         const int tile = unit / m, t = unit % m;
         const int bt = (tile / a.tiles_per_problem) * m + t;
         for (int g = 0; g < grp.n && !*abort; ++g) {
           const int q0 = Groups::first(g), q1 = Groups::last(pl, g), kcg = pl.kc[q1];
-          for (int c = 0; c < kcg && !*abort; ++c) {
+          const int kcp = Groups::prev(pl, g);
+          if (with_cache && kcp > 0) {  // the earlier groups' stores have landed
+            if (!wait_or_abort(cache_ready, nready & 1u, abort)) break;
+            ++nready;
+            fence_proxy_async_global();
+          }
+          const bool mix = a.ncache > 0 && kcp > 0;
+          for (int i = 0; i < kcg && !*abort; ++i) {
+            const int c = Groups::chunk_at(i, kcp, kcg, mix);
+            if (with_cache) {
+              const int s = ra.idx;
+              const bool cached = c < kcp;
+              if (cached) {  // the A stage from this CTA's cache, no side input
+                if (qa >= (uint32_t)SA && !wait_or_abort(&a_empty[s], ra.phase ^ 1u, abort)) break;
+                mbar_expect_tx(&a_full[s], kABytes);
+                bulk_g2s(a_hi(s),
+                         a.kcache + ((size_t)blockIdx.x * a.ncache + c) * (kABytes / 2), kABytes,
+                         &a_full[s]);
+                mbar_arrive_n(&a_full[s], kBldWarps);
+                last_ca = (int)qa;
+              }
+              ++qa;
+              ra.advance(SA);
+              if (cached) continue;
+            }
             if (with_st) {  // the chunk's fp32 K* image
               const int s = ra.idx;
               if (qa >= (uint32_t)SA && !wait_or_abort(&st_empty[s], ra.phase ^ 1u, abort)) break;
@@ -539,6 +587,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
           mbar_wait(&full[j % R], (j / R) & 1);
         for (int j = std::max(0, last_qa - SA + 1); j <= last_qa; ++j)
           mbar_wait(&st_full[j % SA], (j / SA) & 1);
+        if (last_ca >= 0) mbar_wait(&a_full[last_ca % SA], (last_ca / SA) & 1);
       }
     }
   } else if (warp == 1) {
@@ -552,15 +601,29 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       for (int unit = blockIdx.x; unit < units && !*abort; unit += gridDim.x) {
         for (int g = 0; g < grp.n && !*abort; ++g) {
           const int q0 = Groups::first(g), q1 = Groups::last(pl, g), kcg = pl.kc[q1];
-          for (int c = 0; c < kcg && !*abort; ++c) {
+          const int kcp = Groups::prev(pl, g);
+          const bool storing = a.ncache > 0 && g < grp.n - 1;  // a later group needs them
+          const bool mix = a.ncache > 0 && kcp > 0;
+          uint32_t done = 0;  // chunks issued per block of the group, 5 bits each
+          for (int i = 0; i < kcg && !*abort; ++i) {
+            const int c = Groups::chunk_at(i, kcp, kcg, mix);
             const int sa = pa.idx;
             if (!wait_or_abort(&a_full[sa], pa.phase, abort)) break;
             const uint32_t sah = smem_u32(a_hi(sa)), sal = sah + kAPartBytes;
-            for (int qb = q0; qb <= q1; ++qb) {
+            const bool store = storing && c >= kcp;  // built here, needed later
+            if (store) {
+              bulk_s2g(a.kcache + ((size_t)blockIdx.x * a.ncache + c) * (kABytes / 2), a_hi(sa),
+                       kABytes);
+              bulk_commit();
+            }
+            for (int jb = 0; jb <= q1 - q0; ++jb) {
+              const int qb = q0 + jb;
               if (pl.kc[qb] <= c) continue;
-              const uint32_t P = blkseq + (uint32_t)(qb - q0);
+              const uint32_t P = blkseq + (uint32_t)jb;
               const int sl = (int)(P % kSlots);
-              if (c == 0 && P >= kSlots &&
+              const int nd = (int)((done >> (5 * jb)) & 31u);  // chunks of this block issued
+              done += 1u << (5 * jb);
+              if (nd == 0 && P >= kSlots &&
                   !wait_or_abort(&acc_empty[sl], (P / kSlots - 1) & 1, abort))
                 break;
               const int sb = pb.idx;
@@ -574,18 +637,23 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
               for (int ks = 0; ks < 4; ++ks) {
                 const uint64_t dah = sdesc_sw128(sah + ks * 32), dal = sdesc_sw128(sal + ks * 32);
                 const uint64_t dbh = sdesc_sw128(sbh + ks * 32), dbl = sdesc_sw128(sbl + ks * 32);
-                mma_f16(dtm, dah, dbh, idesc, (c > 0 || ks > 0) ? 1u : 0u);
+                mma_f16(dtm, dah, dbh, idesc, (nd > 0 || ks > 0) ? 1u : 0u);
                 mma_f16(dtm, dah, dbl, idesc, 1u);
                 mma_f16(dtm, dal, dbh, idesc, 1u);
               }
               mma_commit(&b_empty[sb]);
               pb.advance(SB);
-              if (c == pl.kc[qb] - 1) mma_commit(&acc_full[sl]);  // the block is complete
+              if (nd == pl.kc[qb] - 1) mma_commit(&acc_full[sl]);  // the block is complete
               issued = true;
             }
             if (*abort) break;
+            if (store) bulk_wait_read();  // the stage is read before it is reused
             mma_commit(&a_empty[sa]);
             pa.advance(SA);
+          }
+          if (storing && !*abort) {  // the group's chunks are in the cache
+            bulk_wait();
+            mbar_arrive_count(cache_ready);
           }
           blkseq += (uint32_t)(q1 - q0 + 1);
         }
@@ -594,6 +662,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
         mma_commit(drain);
         mbar_wait(drain, 0);
       }
+      bulk_wait();  // and every store of ours
     }
   } else if (warp >= kEpiWarp0 && warp < kEpiWarp0 + kEpiWarps) {
     // ---------------------------------------------------------------- epilogue
@@ -672,9 +741,14 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       unsigned long long mag2 = 0ull;
       float sc = 0.f;  // the mean's scale sqrt(s2), scaled like K*
       for (int gi = 0; gi < grp.n && !*abort; ++gi) {
-        const bool last_grp = gi == grp.n - 1;
-        const int kcg = pl.kc[Groups::last(pl, gi)];
-        for (int c = 0; c < kcg && !*abort; ++c, ++qa, pa.advance(SA)) {
+        const int kcg = pl.kc[Groups::last(pl, gi)], kcp = Groups::prev(pl, gi);
+        // with the cache every built chunk is new and adds to the mean;
+        // without it the last group builds every chunk and adds them all
+        const bool mix = a.ncache > 0 && kcp > 0;
+        const bool mean_grp = a.ncache > 0 || gi == grp.n - 1;
+        for (int i = 0; i < kcg && !*abort; ++i, ++qa, pa.advance(SA)) {
+          const int c = mix ? Groups::chunk_at(i, kcp, kcg, true) : i;
+          if (mix && c < kcp) continue;  // cached: the producer brings it
           const int s = pa.idx;
           if (qa >= (uint32_t)SA && !wait_or_abort(&a_empty[s], pa.phase ^ 1u, abort)) break;
           if (PRE && !wait_or_abort(&st_full[s], pa.phase, abort)) break;
@@ -731,7 +805,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
                     v0 = (jbase + kk < n) ? v0 : 0.f;
                     v1 = (jbase + kk + 1 < n) ? v1 : 0.f;
                   }
-                  if (last_grp) {  // (the last group builds every chunk)
+                  if (mean_grp) {  // (each chunk's terms once)
                     const unsigned long long v2 = f2_pack(v0, v1);
                     const unsigned long long a2 = *(const unsigned long long *)(alg + kk);
                     mu2.add(f2_mul(v2, a2));
@@ -828,6 +902,9 @@ int launch_dp(const Gp *gp, const float *Xc, const float *kst, long long N, floa
   a.n = gp->n;
   a.plan = gp->plan;
   a.kern = gp->kern;
+  // the chunk cache (not with K* precomputed, where no chunk is built)
+  a.kcache = gp->kcache;
+  a.ncache = (!kst && gp->kcache && gp->kcache_sms >= num_sms()) ? gp->kcache_chunks : 0;
   a.tiles_per_problem = (int)((N + BOUTE_TILE_M - 1) / BOUTE_TILE_M);
   a.tiles_total = a.tiles_per_problem * gp->B;
   a.b_bytes = (uint32_t)(2 * gp->plan.ncol[0] * 128);  // block 0 is the widest
@@ -973,6 +1050,13 @@ int launch_posterior(const Gp *gp, const float *Xc, long long N, float *mean, fl
     case 32: return launch_dp<32>(gp, Xc, kst, N, mean, var, s);
   }
   return BOUTE_ERR_UNSUPPORTED;
+}
+
+int kstar_cache_chunks(const PostPlan &plan) {
+  const int ngroup = (plan.nblk + kGroup - 1) / kGroup;
+  if (ngroup < 2) return 0;
+  const int last_of_prev = std::min(plan.nblk, (ngroup - 1) * kGroup) - 1;
+  return plan.kc[last_of_prev];  // every chunk the groups before the last build
 }
 
 size_t kstar_floats(const Gp *gp, long long N) {
