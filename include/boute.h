@@ -164,8 +164,11 @@ int boute_gp_learn_k(const double *X, const double *Ys, int B, int n, int d, int
  * (Sec. 5.2: the acquisition is taken over the GP posterior):
  *   mean = K* alpha,  var = max(0, s2 - rowsum((K* L^-T)^2)),
  * with the Matern-5/2 cross-covariance K* built tile by tile in shared memory
- * and contracted on the tensor cores in 3xTF32 (fp32-accurate) without ever
- * being written to HBM.
+ * and contracted on the tensor cores as fp16 hi/lo parts (three products per
+ * term, fp32 accumulate: fp32-accurate) without ever being written to HBM.
+ * The mean is reduced from the fp32 K* with compensated sums; a candidate
+ * whose terms K*_j alpha_j add up to more than 256 times the mean's scale
+ * (an ill-conditioned K) has its mean recomputed in fp64.
  *   Xc: B x N x d fp32 candidates (points of [0,1]^d or any real values);
  *   mean, var: B x m x N fp32 (objective-major per problem). */
 int boute_gp_posterior(const boute_gp *gp, const float *Xc, long long N, float *mean,

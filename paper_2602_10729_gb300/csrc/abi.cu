@@ -200,6 +200,7 @@ int boute_gp_create(int B, int n, int d, int m, boute_gp **out) {
   r |= dalloc(&g.xt, BM * (size_t)g.plan.nxt * xt_chunk_floats(g.DP));
   r |= dalloc(&g.s2f, BM);
   r |= dalloc(&g.status, 1);
+  r |= dalloc(&g.fbad, BM);
   if (r != BOUTE_OK) {
     boute_gp_free(h);
     return BOUTE_ERR_OOM;
@@ -236,7 +237,7 @@ void boute_gp_free(boute_gp *gp) {
   if (!gp) return;
   Gp &g = gp->g;
   cudaFree(g.Kh); cudaFree(g.Kl); cudaFree(g.Aws); cudaFree(g.Wws); cudaFree(g.bop); cudaFree(g.xt);
-  cudaFree(g.s2f); cudaFree(g.status); cudaFree(g.kpar); cudaFree(g.kcache);
+  cudaFree(g.s2f); cudaFree(g.status); cudaFree(g.kpar); cudaFree(g.kcache); cudaFree(g.fbad);
   delete gp;
 }
 

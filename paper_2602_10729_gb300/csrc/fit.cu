@@ -282,7 +282,7 @@ template <bool SMEM>
 __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     const float *Kh_all, const float *Kl_all, const double *Ys, int standardize, int n, int m,
     float *Aws, float *Wws, float *xt, int DP, int npad, PostPlan plan, uint16_t *bop,
-    int kl_smem, int early_trigger, int comp, int *status) {
+    int kl_smem, int early_trigger, int comp, int *status, const int *fbad) {
   extern __shared__ __align__(16) float sm[];
   __shared__ int bad;
   __shared__ uint64_t lbar, lbar_lo;  // K hi; K lo (needed only by the residual)
@@ -349,7 +349,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
         bulk_g2s(Kls, Kl, bytes, &lbar_lo);
       }
     }
-  } else {  // eight independent loads per thread in flight before their stores
+  } else if (!fbad) {  // eight independent loads per thread in flight before their stores
     const int nn = n * n;
     for (int base = 0; base < nn; base += 8 * nthr) {
       float v[8], w8[8];
@@ -370,7 +370,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
       }
     }
   }
-  for (int e = tid; e < (NP - n) * NP; e += nthr) {
+  for (int e = tid; e < (NP - n) * NP && !fbad; e += nthr) {
     const int i = n + e / NP, k = e % NP;
     if (k <= i) A[(size_t)i * ld + k] = (k == i) ? 1.f : 0.f;
   }
@@ -397,7 +397,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     ylo[i] = (float)(ys - (double)yv[i]);
     dg[i] = A[(size_t)i * ld + i];
   }
-  if (tid == 0) bad = 0;
+  if (tid == 0) bad = fbad ? fbad[bt] : 0;  // (factored by the blocked kernels)
   for (int e = tid; e < 32 * 64; e += nthr) (&colL[0][0])[e] = 0.f;
   __syncthreads();
   // Operand images of W for the posterior (n <= 160): rows [g_lo, g_hi) of W,
@@ -429,7 +429,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   // for T_pJ and W_pJ).
   const int nb = NP / 32;
   const unsigned FULL = 0xffffffffu;
-  for (int p = 0; p < nb; ++p) {
+  for (int p = 0; p < nb && !fbad; ++p) {
     const int p0 = 32 * p;
     if (warp == 0) {
       // Factor. Lane = row of the block. a[] is a window on the lane's row
@@ -872,6 +872,241 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   }
 }
 
+// ---- the global-workspace factorisation across many blocks -------------------------
+// For n > 160 the three phases of every 32-column panel of fit32_kernel's loop
+// run as three kernels, each over as many blocks as its tiles fill (a grid of
+// x blocks per problem-objective y), with programmatic dependent launch in
+// between: (a) fitb_diag_kernel factors and inverts the diagonal block, (b)
+// fitb_panel_kernel forms the panel below and the partial sums T_pJ, (c)
+// fitb_update_kernel applies the trailing update, forms W's block row and
+// copies the panel into A. The tiles' arithmetic is the same as in the
+// one-block loop; fit32_kernel then finishes alpha and the outputs from the
+// factored workspace. A non-positive pivot marks the problem-objective in fbad
+// and its later kernels return at once.
+constexpr int kFitbThreads = 256;
+
+// A = K hi below the diagonal, the identity on the padding; fbad cleared.
+__global__ void __launch_bounds__(kFitbThreads) fitb_load_kernel(const float *Kh_all, int n,
+                                                                 int NP, float *Aws, int *fbad) {
+  pdl_wait();
+  pdl_trigger();
+  const int bt = blockIdx.y, ld = NP + 1;
+  const float *Kh = Kh_all + (size_t)bt * n * n;
+  float *A = Aws + (size_t)bt * NP * ld;
+  const long long tot = (long long)NP * NP;
+  for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < tot;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int i = (int)(e / NP), k = (int)(e % NP);
+    if (k > i) continue;
+    A[(size_t)i * ld + k] = i < n ? Kh[(size_t)i * n + k] : (k == i ? 1.f : 0.f);
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) fbad[bt] = 0;
+}
+
+// (a) one block of two warps per problem-objective: warp 0 factors A_pp in
+// registers (the pivot test against K's own diagonal), warp 1 inverts it one
+// column behind into W_pp, as in fit32_kernel.
+__global__ void __launch_bounds__(64) fitb_diag_kernel(const float *Kh_all, int n, int NP,
+                                                       float *Aws, float *Wws, int p,
+                                                       int *fbad) {
+  __shared__ __align__(16) float colL[32][64];
+  __shared__ float invs[32];
+  pdl_wait();
+  pdl_trigger();
+  const int bt = blockIdx.x, ld = NP + 1, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (fbad[bt]) return;
+  const float *Kh = Kh_all + (size_t)bt * n * n;
+  float *A = Aws + (size_t)bt * NP * ld, *W = Wws + (size_t)bt * NP * ld;
+  const int p0 = 32 * p;
+  const unsigned FULL = 0xffffffffu;
+  for (int e = threadIdx.x; e < 32 * 64; e += 64) (&colL[0][0])[e] = 0.f;
+  __syncthreads();
+  if (warp == 0) {
+    float a[32];
+    float *Ar = A + (size_t)(p0 + lane) * ld + p0;
+#pragma unroll
+    for (int c = 0; c < 32; ++c) a[c] = (c <= lane) ? Ar[c] : 0.f;
+    const int gi = p0 + lane;
+    const float dgl = gi < n ? Kh[(size_t)gi * n + gi] : 1.f;
+    bool ok = true;
+    float piv = __shfl_sync(FULL, a[0], 0);
+    auto quarter = [&](auto nk, int c0) {
+      constexpr int NK = decltype(nk)::value;
+#pragma unroll 1
+      for (int c = c0; c < c0 + 8; ++c) {
+        if (!(piv > 16.f * 1.1920929e-7f * __shfl_sync(FULL, dgl, c))) ok = false;
+        float inv = rsqrtf(piv);
+        inv = inv * fmaf(-0.5f * piv * inv, inv, 1.5f);  // one Newton step; 1 / L_cc
+        const float l = lane > c ? a[0] * inv : (lane == c ? piv * inv : 0.f);
+        piv = __shfl_sync(FULL, fmaf(-l, l, a[1]), (c + 1) & 31);
+        if (lane >= c) Ar[c] = l;
+        colL[c][lane] = l;
+        if (lane == 0) invs[c] = inv;
+        __syncwarp();
+        named_barrier_sync(1, 64);  // column c is ready for warp 1
+#pragma unroll
+        for (int k = 0; k < NK; ++k) a[k] = fmaf(-l, colL[c][c + 1 + k], a[k + 1]);
+      }
+    };
+    quarter(std::integral_constant<int, 31>{}, 0);
+    quarter(std::integral_constant<int, 23>{}, 8);
+    quarter(std::integral_constant<int, 15>{}, 16);
+    quarter(std::integral_constant<int, 7>{}, 24);
+    if (__any_sync(FULL, !ok) && lane == 0) fbad[bt] = 1;
+  } else {
+    float w[32];
+#pragma unroll
+    for (int c = 0; c < 32; ++c) w[c] = (c == lane) ? 1.f : 0.f;
+    float myinv = 0.f;
+    auto quarter = [&](auto nk, int c0) {
+      constexpr int NK = decltype(nk)::value;
+#pragma unroll 1
+      for (int c = c0; c < c0 + 8; ++c) {
+        named_barrier_sync(1, 64);  // wait for column c
+        const float l = colL[c][lane], inv = invs[c];
+        if (lane == c) myinv = inv;
+        const float lw = lane > c ? l * inv : 0.f;
+#pragma unroll
+        for (int k = 0; k < NK; ++k) w[k] = fmaf(-lw, __shfl_sync(FULL, w[k], c), w[k]);
+      }
+    };
+    quarter(std::integral_constant<int, 8>{}, 0);
+    quarter(std::integral_constant<int, 16>{}, 8);
+    quarter(std::integral_constant<int, 24>{}, 16);
+    quarter(std::integral_constant<int, 32>{}, 24);
+    float *Wr = W + (size_t)(p0 + lane) * ld + p0;
+#pragma unroll
+    for (int c = 0; c < 32; ++c) Wr[c] = w[c] * myinv;
+  }
+}
+
+// (b) L_rp = A_rp W_pp^T for the rows below the panel (4 x 4 tiles) into block
+// column p of W, and T_pJ = sum_{K=J}^{p-1} L_pK W_KJ (J < p; 4 x 2 tiles)
+// parked, transposed, in W's upper triangle.
+__global__ void __launch_bounds__(kFitbThreads) fitb_panel_kernel(int NP, const float *Aws,
+                                                                  float *Wws, int p,
+                                                                  const int *fbad) {
+  pdl_wait();
+  pdl_trigger();
+  const int bt = blockIdx.y, ld = NP + 1;
+  if (fbad[bt]) return;
+  const float *A = Aws + (size_t)bt * NP * ld;
+  float *W = Wws + (size_t)bt * NP * ld;
+  const int p0 = 32 * p, r0 = p0 + 32, rows = NP - r0;
+  const int ntr = (rows / 4) * 8, ntt = p * 128;
+  for (int tix = blockIdx.x * blockDim.x + threadIdx.x; tix < ntr + ntt;
+       tix += gridDim.x * blockDim.x) {
+    float acc[4][4] = {};
+    if (tix < ntr) {
+      const int i0 = r0 + 4 * (tix >> 3), c0 = 4 * (tix & 7);
+#pragma unroll 4
+      for (int q = 0; q < 32; ++q) {
+        float x[4], y4[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          x[u] = A[(size_t)(i0 + u) * ld + p0 + q];
+          y4[u] = W[(size_t)(p0 + c0 + u) * ld + p0 + q];
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) W[(size_t)(i0 + u) * ld + p0 + c0 + v] = acc[u][v];
+    } else {
+      const int e = tix - ntr, J = e >> 7, rb = 4 * ((e >> 4) & 7), cb = 2 * (e & 15);
+#pragma unroll 4
+      for (int q = 32 * J; q < p0; ++q) {
+        float x[4], y2[2];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) x[u] = A[(size_t)(p0 + rb + u) * ld + q];
+#pragma unroll
+        for (int v = 0; v < 2; ++v) y2[v] = W[(size_t)q * ld + 32 * J + cb + v];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int v = 0; v < 2; ++v) acc[u][v] = fmaf(x[u], y2[v], acc[u][v]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 2; ++v) W[(size_t)(32 * J + cb + v) * ld + p0 + rb + u] = acc[u][v];
+    }
+  }
+}
+
+// (c) the trailing update A_ij -= sum_q L_iq L_jq below the panel (4 x 4
+// tiles of the lower triangle), W_pJ = -W_pp T_pJ (4 x 2 tiles), and the
+// panel (block column p of W, rows below it) copied into A.
+__global__ void __launch_bounds__(kFitbThreads) fitb_update_kernel(int NP, float *Aws,
+                                                                   float *Wws, int p,
+                                                                   const int *fbad) {
+  pdl_wait();
+  pdl_trigger();
+  const int bt = blockIdx.y, ld = NP + 1;
+  if (fbad[bt]) return;
+  float *A = Aws + (size_t)bt * NP * ld;
+  float *W = Wws + (size_t)bt * NP * ld;
+  const int p0 = 32 * p, r0 = p0 + 32, rows = NP - r0;
+  const int th = rows / 4, ntile = th * (th + 1) / 2, nwt = p * 128, ncp = rows * 32;
+  for (int tix = blockIdx.x * blockDim.x + threadIdx.x; tix < ntile + nwt + ncp;
+       tix += gridDim.x * blockDim.x) {
+    if (tix >= ntile + nwt) {  // the panel into A
+      const int e = tix - ntile - nwt;
+      const size_t o = (size_t)(r0 + (e >> 5)) * ld + p0 + (e & 31);
+      A[o] = W[o];
+      continue;
+    }
+    float acc[4][4] = {};
+    if (tix < ntile) {
+      int ti = (int)((sqrtf(8.f * tix + 1.f) - 1.f) * 0.5f);
+      while (ti * (ti + 1) / 2 > tix) --ti;
+      while ((ti + 1) * (ti + 2) / 2 <= tix) ++ti;
+      const int tj = tix - ti * (ti + 1) / 2;
+      const int i0 = r0 + 4 * ti, j0 = r0 + 4 * tj;
+#pragma unroll 4
+      for (int q = 0; q < 32; ++q) {
+        float x[4], y4[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          x[u] = W[(size_t)(i0 + u) * ld + p0 + q];
+          y4[u] = W[(size_t)(j0 + u) * ld + p0 + q];
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v)
+          if (ti != tj || v <= u) A[(size_t)(i0 + u) * ld + j0 + v] -= acc[u][v];
+    } else {
+      const int e = tix - ntile, J = e >> 7, rb = 4 * ((e >> 4) & 7), cb = 2 * (e & 15);
+#pragma unroll 4
+      for (int q = 0; q < 32; ++q) {
+        float x[4], y2[2];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) x[u] = W[(size_t)(p0 + rb + u) * ld + p0 + q];
+#pragma unroll
+        for (int v = 0; v < 2; ++v) y2[v] = W[(size_t)(32 * J + cb + v) * ld + p0 + q];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int v = 0; v < 2; ++v) acc[u][v] = fmaf(x[u], y2[v], acc[u][v]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 2; ++v) W[(size_t)(p0 + rb + u) * ld + 32 * J + cb + v] = -acc[u][v];
+    }
+  }
+}
+
 // ---- operand images of L^-1 as fp16 hi/lo, swizzled (global-workspace fit) ----
 __global__ void pack_kernel(const float *Wws, PostPlan plan, uint16_t *bop, const float *xt,
                             int DP, int *status) {
@@ -948,19 +1183,65 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
   if (gp->kern) setup(fit_setup_kernel<true>);
   else setup(fit_setup_kernel<false>);
   if (setup_done && cudaEventRecord(setup_done, s) != cudaSuccess) return last_launch_status();
-  if (fit_uses_smem(npad)) {
-    const size_t smem = fit_smem_bytes(npad, n);
-    prefer_shared(fit32_kernel<true>);
-    cudaFuncSetAttribute(fit32_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         (int)smem);
-    launch_pdl(fit32_kernel<true>, dim3(BM), dim3(fit_threads<true>()), smem, s, gp->Kh, gp->Kl,
-               Ys, standardize, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop,
-               fit_kl_in_smem(n) ? 1 : 0, fit_early, gp->kern, gp->status);
-    count_launch(2);
+  // the one-block fits already fill the GPU when there are many problem-
+  // objectives; with few, the blocked factorisation spreads each over blocks
+  const bool blocked = !fit_uses_smem(npad) && 4 * BM <= sms;
+  if (fit_uses_smem(npad) || !blocked) {
+    const bool sm_fit = fit_uses_smem(npad);
+    if (sm_fit) {
+      const size_t smem = fit_smem_bytes(npad, n);
+      prefer_shared(fit32_kernel<true>);
+      cudaFuncSetAttribute(fit32_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem);
+      launch_pdl(fit32_kernel<true>, dim3(BM), dim3(fit_threads<true>()), smem, s, gp->Kh,
+                 gp->Kl, Ys, standardize, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan,
+                 gp->bop, fit_kl_in_smem(n) ? 1 : 0, fit_early, gp->kern, gp->status,
+                 (const int *)nullptr);
+      count_launch(2);
+    } else {  // one block per problem-objective on the global workspace
+      launch_pdl(fit32_kernel<false>, dim3(BM), dim3(fit_threads<false>()),
+                 6 * npad * sizeof(float), s, gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws,
+                 gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop, 0, 0, gp->kern, gp->status,
+                 (const int *)nullptr);
+      const long long tot = (long long)gp->plan.nblk * BOUTE_BLKCOLS * gp->plan.nchunk * 32;
+      pack_kernel<<<dim3((unsigned)std::min<long long>((tot + 255) / 256, 4096), BM), 256, 0,
+                    s>>>(gp->Wws, gp->plan, gp->bop, gp->xt, gp->DP, gp->status);
+      count_launch(3);
+    }
   } else {
+    // the factorisation across many blocks, panel by panel, then alpha and the
+    // outputs by fit32_kernel on the factored workspace
+    const int cap = std::max(1, 2 * sms / BM);
+    auto ctas = [&](long long tiles) {
+      return (unsigned)std::max(1LL, std::min<long long>(cap, (tiles + kFitbThreads - 1) / kFitbThreads));
+    };
+    int nl = 0;
+    launch_pdl(fitb_load_kernel, dim3(ctas((long long)npad * npad / 2), BM), dim3(kFitbThreads), 0, s,
+               (const float *)gp->Kh, n, npad, gp->Aws, gp->fbad);
+    ++nl;
+    for (int p = 0; p < npad / 32; ++p) {
+      const int rows = npad - 32 * p - 32, th = rows / 4;
+      launch_pdl(fitb_diag_kernel, dim3(BM), dim3(64), 0, s, (const float *)gp->Kh, n, npad,
+                 gp->Aws, gp->Wws, p, gp->fbad);
+      const long long tb = (long long)th * 8 + 128LL * p;
+      if (tb > 0) {
+        launch_pdl(fitb_panel_kernel, dim3(ctas(tb), BM), dim3(kFitbThreads), 0, s, npad,
+                   (const float *)gp->Aws, gp->Wws, p, (const int *)gp->fbad);
+        ++nl;
+      }
+      const long long tc = (long long)th * (th + 1) / 2 + 128LL * p + 32LL * rows;
+      if (tc > 0) {
+        launch_pdl(fitb_update_kernel, dim3(ctas(tc), BM), dim3(kFitbThreads), 0, s, npad,
+                   gp->Aws, gp->Wws, p, (const int *)gp->fbad);
+        ++nl;
+      }
+      ++nl;
+    }
+    count_launch(nl);
     launch_pdl(fit32_kernel<false>, dim3(BM), dim3(fit_threads<false>()),
                6 * npad * sizeof(float), s, gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws,
-               gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop, 0, 0, gp->kern, gp->status);
+               gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop, 0, 0, gp->kern, gp->status,
+               (const int *)gp->fbad);
     const long long tot = (long long)gp->plan.nblk * BOUTE_BLKCOLS * gp->plan.nchunk * 32;
     pack_kernel<<<dim3((unsigned)std::min<long long>((tot + 255) / 256, 4096), BM), 256, 0, s>>>(
         gp->Wws, gp->plan, gp->bop, gp->xt, gp->DP, gp->status);

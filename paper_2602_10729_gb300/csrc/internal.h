@@ -24,6 +24,7 @@ struct Gp {
   float *xt;      // B*m x nxt x xt_chunk_floats(DP): X/lengthscale hi/lo, alpha
   float *s2f;     // B*m: outputscale
   int *status;    // device status word (first error wins)
+  int *fbad;      // B*m: a non-positive pivot in the blocked factorisation (n > 160)
   // the composite kernel (kern = 1): routing features [0, dtau) and per
   // problem-objective [s2_c, s2_x, beta, s_0 .. s_{d-1}] (B*m x (3 + d))
   int kern, dtau;

@@ -12,11 +12,13 @@ from oracle import pipeline as opl
 from paper_2602_10729_gb300 import workloads as wl
 
 # ---- tolerances ----------------------------------------------------------------
-# Posterior (3xTF32 contraction, fp32 accumulate): relative 1e-5 against the
-# quantity's natural scale: |g - o| <= 1e-5 * max(|o|, s) for the mean (s is
-# the prior standard deviation), |g - o| <= 1e-5 * s2 for the variance, whose
-# fp32 value s2 - ||v||^2 carries an absolute rounding error of order eps32 * s2
-# whatever its size.
+# Posterior (fp16 hi/lo contraction with fp32 accumulate, fp32-accurate):
+# relative 1e-5 against the quantity's natural scale: |g - o| <= 1e-5 *
+# max(|o|, s) for the mean (s is the prior standard deviation), |g - o| <=
+# 1e-5 * s2 for the variance, whose fp32 value s2 - ||v||^2 carries an
+# absolute rounding error of order eps32 * s2 whatever its size (near a
+# training point, where the variance is about the noise, a relative bound on
+# the variance itself would ask for digits an fp32 difference cannot keep).
 POST_REL = 1e-5
 # Acquisition: relative 1e-4 against max(|o|, 1e-3 * max_j |o_j|), the largest
 # value of the problem setting the scale below which fp32 rounding of the
