@@ -92,6 +92,27 @@ int boute_gp_fit(boute_gp *gp, const double *X, const double *Ys, const double *
                  const double *outputscale, const double *noise, void *stream);
 int boute_gp_status(boute_gp *gp, void *stream);
 void boute_gp_free(boute_gp *gp);
+/* ---- precision tiers ----------------------------------------------------------
+ * Sec. 6 and Appendix C: the paper's MOBO runs its GP kernels in double
+ * precision. BOUTE_PREC_FP32 (the default) is the fp32-accurate path of
+ * boute_gp_posterior (posterior mean and variance within 1e-5 of the fp64
+ * values). boute_gp_set_precision(gp, BOUTE_PREC_FP64) makes the handle's
+ * later fits also compute K, its Cholesky factor L, W = L^-1 and alpha in
+ * fp64 (on the CUDA cores; GB300's fp64 rate is a small fraction of its fp32
+ * rate, so this tier serves accuracy, not throughput), and
+ * boute_gp_posterior_fp64 then writes
+ *   mean = k*^T alpha,  var = max(0, s2 - ||W k*||^2)
+ * in fp64: Xc as for boute_gp_posterior; mean, var: B x m x N fp64 device
+ * arrays. The FP64 tier serves n <= 128 and the Matern-5/2 kernel: other
+ * handles return BOUTE_ERR_UNSUPPORTED from set_precision (and set_kernel
+ * with the composite kernel returns it for an FP64 handle); allocates its
+ * fp64 buffers on the first switch. boute_gp_posterior_fp64 on a handle not
+ * set to FP64 is INVALID_ARG; the fp32 path keeps working on an FP64 handle. */
+#define BOUTE_PREC_FP32 0
+#define BOUTE_PREC_FP64 1
+int boute_gp_set_precision(boute_gp *gp, int prec);
+int boute_gp_posterior_fp64(const boute_gp *gp, const float *Xc, long long N, double *mean,
+                            double *var, void *stream);
 /* The paper's composite kernel for the handle's later fits and posteriors
  * (Sec. 5.2 "Additive kernels" with the preference weighting of S5, as
  * Sec. 6 assembles it: k_tau + k~_c + k_x, each in its own ScaleKernel):

@@ -23,6 +23,7 @@ BOUTE_TF_IDENTITY, BOUTE_TF_LOG, BOUTE_TF_LOGIT, BOUTE_TF_NEGATE = 0, 1, 2, 4
 SYMBOLS = (
     "boute_status_string", "boute_launch_count", "boute_standardize", "boute_gp_create",
     "boute_gp_fit", "boute_gp_status", "boute_gp_free", "boute_gp_posterior",
+    "boute_gp_set_precision", "boute_gp_posterior_fp64",
     "boute_pareto_front", "boute_box_decompose", "boute_acq_ehvi", "boute_acq_mc_hvi",
     "boute_select_topk", "boute_select_topk_noalloc", "boute_engine_create", "boute_engine_step",
     "boute_engine_step_async",
@@ -83,6 +84,8 @@ def load(path: str | None = None):
         "boute_gp_status": ([_vp, _vp], _i),
         "boute_gp_free": ([_vp], None),
         "boute_gp_posterior": ([_vp, _vp, _ll, _vp, _vp, _vp], _i),
+        "boute_gp_set_precision": ([_vp, _i], _i),
+        "boute_gp_posterior_fp64": ([_vp, _vp, _ll, _vp, _vp, _vp], _i),
         "boute_pareto_front": ([_vp, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
         "boute_box_decompose": ([_vp, _vp, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
         "boute_acq_ehvi": ([_vp, _vp, _i, _ll, _vp, _vp, _i, _vp, _vp, _vp, _vp], _i),
@@ -329,6 +332,19 @@ def boute_gp_posterior(gp: Gp, Xc, N: int, mean, var, stream=None):
     f32 = torch.float32
     _check(load().boute_gp_posterior(gp.handle, _p(Xc, f32), N, _p(mean, f32), _p(var, f32),
                                      _s(stream)), "boute_gp_posterior")
+
+
+BOUTE_PREC_FP32, BOUTE_PREC_FP64 = 0, 1
+
+
+def boute_gp_set_precision(gp: Gp, prec: int):
+    _check(load().boute_gp_set_precision(gp.handle, int(prec)), "boute_gp_set_precision")
+
+
+def boute_gp_posterior_fp64(gp: Gp, Xc, N: int, mean, var, stream=None):
+    f64 = torch.float64
+    _check(load().boute_gp_posterior_fp64(gp.handle, _p(Xc, torch.float32), N, _p(mean, f64),
+                                          _p(var, f64), _s(stream)), "boute_gp_posterior_fp64")
 
 
 def boute_pareto_front(Ys, B, n, m, ref, mask, front, P, stream=None):

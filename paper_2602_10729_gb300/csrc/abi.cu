@@ -28,10 +28,14 @@ int last_launch_status() {
   return BOUTE_ERR_CUDA;
 }
 
-// The kernels are built for sm_103a only: refuse other devices up front.
-static int device_ok() {
+// The kernels are built for sm_103a only: refuse other devices up front (a
+// failed device query leaves no error behind for later calls to report).
+int device_ok() {
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return BOUTE_ERR_UNSUPPORTED;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return BOUTE_ERR_UNSUPPORTED;
+  }
   int major = 0, minor = 0;
   cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
   cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
@@ -218,7 +222,45 @@ int boute_gp_fit(boute_gp *gp, const double *X, const double *Ys, const double *
                  const double *outputscale, const double *noise, void *stream) {
   BOUTE_TRACE();
   if (!gp || !X || !Ys || !lengthscale || !outputscale || !noise) return BOUTE_ERR_INVALID_ARG;
-  return launch_fit(&gp->g, X, Ys, lengthscale, outputscale, noise, (cudaStream_t)stream);
+  Gp &g = gp->g;
+  const cudaStream_t s = (cudaStream_t)stream;
+  if (int r = launch_fit(&g, X, Ys, lengthscale, outputscale, noise, s)) return r;
+  if (g.prec != BOUTE_PREC_FP64) return BOUTE_OK;
+  const size_t BM = (size_t)g.B * g.m;
+  if (cudaMemcpyAsync(g.ls64, lengthscale, BM * g.d * sizeof(double), cudaMemcpyDeviceToDevice,
+                      s) != cudaSuccess ||
+      cudaMemcpyAsync(g.s2_64, outputscale, BM * sizeof(double), cudaMemcpyDeviceToDevice, s) !=
+          cudaSuccess)
+    return last_launch_status();
+  return launch_fit64(&g, X, Ys, lengthscale, outputscale, noise, s);
+}
+
+int boute_gp_set_precision(boute_gp *gp, int prec) {
+  BOUTE_TRACE();
+  if (!gp || (prec != BOUTE_PREC_FP32 && prec != BOUTE_PREC_FP64)) return BOUTE_ERR_INVALID_ARG;
+  Gp &g = gp->g;
+  if (prec == BOUTE_PREC_FP64) {
+    if (g.n > kFp64MaxN || g.kern) return BOUTE_ERR_UNSUPPORTED;
+    if (!g.W64) {
+      const size_t BM = (size_t)g.B * g.m;
+      int r = dalloc(&g.W64, BM * g.n * g.n);
+      r |= dalloc(&g.a64, BM * g.n);
+      r |= dalloc(&g.xs64, BM * g.n * g.d);
+      r |= dalloc(&g.ls64, BM * g.d);
+      r |= dalloc(&g.s2_64, BM);
+      if (r != BOUTE_OK) return BOUTE_ERR_OOM;
+    }
+  }
+  g.prec = prec;
+  return BOUTE_OK;
+}
+
+int boute_gp_posterior_fp64(const boute_gp *gp, const float *Xc, long long N, double *mean,
+                            double *var, void *stream) {
+  BOUTE_TRACE();
+  if (!gp || N < 0 || (N > 0 && (!Xc || !mean || !var))) return BOUTE_ERR_INVALID_ARG;
+  if (gp->g.prec != BOUTE_PREC_FP64) return BOUTE_ERR_INVALID_ARG;
+  return launch_posterior64(&gp->g, Xc, N, mean, var, (cudaStream_t)stream);
 }
 
 int boute_gp_status(boute_gp *gp, void *stream) {
@@ -238,6 +280,7 @@ void boute_gp_free(boute_gp *gp) {
   Gp &g = gp->g;
   cudaFree(g.Kh); cudaFree(g.Kl); cudaFree(g.Aws); cudaFree(g.Wws); cudaFree(g.bop); cudaFree(g.xt);
   cudaFree(g.s2f); cudaFree(g.status); cudaFree(g.kpar); cudaFree(g.kcache); cudaFree(g.fbad);
+  cudaFree(g.W64); cudaFree(g.a64); cudaFree(g.xs64); cudaFree(g.ls64); cudaFree(g.s2_64);
   delete gp;
 }
 
@@ -275,6 +318,7 @@ int boute_gp_set_kernel(boute_gp *gp, int d_tau, const double *params) {
     g.kern = 0;
     return BOUTE_OK;
   }
+  if (g.prec == BOUTE_PREC_FP64) return BOUTE_ERR_UNSUPPORTED;  // (Matern-5/2 only)
   if (d_tau < 0 || d_tau > g.d) return BOUTE_ERR_INVALID_ARG;
   const int BM = g.B * g.m, dc = g.d - d_tau, in = 3 + dc, out = 3 + g.d;
   std::vector<double> h((size_t)BM * out, 0.0);

@@ -25,6 +25,11 @@ struct Gp {
   float *s2f;     // B*m: outputscale
   int *status;    // device status word (first error wins)
   int *fbad;      // B*m: a non-positive pivot in the blocked factorisation (n > 160)
+  // the FP64 tier (prec = BOUTE_PREC_FP64): W = L^-1 (B*m x n x n), alpha
+  // (B*m x n), X / lengthscale (B*m x n x d), lengthscales (B*m x d) and
+  // outputscales (B*m) of the last fit, all fp64
+  int prec;
+  double *W64, *a64, *xs64, *ls64, *s2_64;
   // the composite kernel (kern = 1): routing features [0, dtau) and per
   // problem-objective [s2_c, s2_x, beta, s_0 .. s_{d-1}] (B*m x (3 + d))
   int kern, dtau;
@@ -79,6 +84,14 @@ void count_launch(int k = 1);
 unsigned long long launch_count();
 int last_launch_status();  // BOUTE_OK or BOUTE_ERR_CUDA after a launch
 
+// FP64 tier (n <= 128, Matern-5/2): the fit's fp64 factor and the posterior
+int launch_fit64(Gp *gp, const double *X, const double *Ys, const double *ls, const double *s2,
+                 const double *noise, cudaStream_t s);
+int launch_posterior64(const Gp *gp, const float *Xc, long long N, double *mean, double *var,
+                       cudaStream_t s);
+constexpr int kFp64MaxN = 128;
+// the library's device check (an sm_103a device is current)
+int device_ok();
 // codes: outcome transforms before standardising (objective_code)
 int launch_standardize(const double *Y, int B, int n, int m, int codes, double *Ys,
                        cudaStream_t s);

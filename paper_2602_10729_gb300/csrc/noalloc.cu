@@ -22,18 +22,6 @@ constexpr int kMaxDevices = 64;
 void *g_scratch_ptr[kMaxDevices] = {};
 std::mutex g_scratch_mu;
 
-// The kernels are built for sm_103a only.
-int device_is_sm103() {
-  int dev = 0, major = 0, minor = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) {
-    cudaGetLastError();
-    return 0;
-  }
-  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
-  cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
-  return major == 10 && minor == 3;
-}
-
 // Address of the current device's copy of the array, looked up once per device.
 int scratch_address(void **out) {
   int dev = -1;
@@ -71,7 +59,7 @@ extern "C" int boute_select_topk_noalloc(const float *acq, int B, long long N, i
       nseg <= 1 ? 0ull
                 : 2ull * (unsigned long long)B * nseg * (k < 32 ? 32 : k) * sizeof(unsigned long long);
   if (need > BOUTE_TOPK_NOALLOC_SCRATCH_BYTES) return BOUTE_ERR_UNSUPPORTED;
-  if (!device_is_sm103()) return BOUTE_ERR_UNSUPPORTED;
+  if (int r = device_ok()) return r;
   void *scratch = nullptr;
   if (int r = scratch_address(&scratch)) return r;
   return launch_topk(acq, B, N, k, idx, val, scratch, (cudaStream_t)stream);

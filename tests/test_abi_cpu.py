@@ -70,6 +70,9 @@ def test_invalid_arguments_are_rejected_before_any_device_call(lib):
     assert lib.boute_selftest_wait(0, 3_000_000_000, None) == bt.BOUTE_ERR_INVALID_ARG
     assert lib.boute_engine_set_kernel(None, 0, None) == bt.BOUTE_ERR_INVALID_ARG
     assert lib.boute_gp_set_kernel(None, 0, None) == bt.BOUTE_ERR_INVALID_ARG
+    # precision tiers
+    assert lib.boute_gp_set_precision(None, bt.BOUTE_PREC_FP64) == bt.BOUTE_ERR_INVALID_ARG
+    assert lib.boute_gp_posterior_fp64(None, p, 10, p, p, None) == bt.BOUTE_ERR_INVALID_ARG
     # hyperparameter learning: restarts, steps, step size, d_tau
     assert lib.boute_gp_learn(p, p, 1, 8, 2, 2, p, 0, 5, 0.1, p, p, None, None) == \
         bt.BOUTE_ERR_INVALID_ARG
