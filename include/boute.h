@@ -397,6 +397,17 @@ int boute_engine_set_kernel(boute_engine *e, int d_tau, const double *params);
  * (boute_base_normals) into a resident buffer; later steps whose eps is NULL
  * use them (and the host-input steps copy no normals). Synchronous. */
 int boute_engine_set_normals(boute_engine *e, unsigned long long seed);
+/* A growing data set (Sec. 3.1 loop: one observation is added per
+ * iteration): later steps use n observations, 1 <= n <= the n the engine was
+ * created with, which fixes every buffer's size; the steps' X and Y then hold
+ * n rows. The GP's posterior layout is re-planned for n and the cached step
+ * graphs are dropped (the next step on a stream captures a new one); no
+ * buffer is allocated, except the in-kernel selection's scratch of
+ * 2-objective Monte-Carlo engines when it must grow. Waits for all work on
+ * the device. Errors: BOUTE_ERR_INVALID_ARG for n out of range (the engine is
+ * unchanged), BOUTE_ERR_OOM / BOUTE_ERR_CUDA (the engine stays usable at
+ * n, selecting with the separate top-k kernel). */
+int boute_engine_set_n(boute_engine *e, int n);
 void boute_engine_free(boute_engine *e);
 
 /* ---- the optimisation loop ------------------------------------------------------

@@ -32,7 +32,7 @@ SYMBOLS = (
     "boute_engine_stage_times", "boute_engine_launches_per_step", "boute_engine_set_constraints",
     "boute_engine_set_outcome_transforms", "boute_engine_set_kernel", "boute_gp_set_kernel",
     "boute_gp_learn", "boute_gp_learn_k", "boute_mobo_run", "boute_base_normals",
-    "boute_engine_set_normals", "boute_selftest_wait",
+    "boute_engine_set_normals", "boute_engine_set_n", "boute_selftest_wait",
     "boute_engine_free",
 )
 #: stage names of boute_engine_stage_times, in order
@@ -113,6 +113,7 @@ def load(path: str | None = None):
                               _vp, _vp, _vp], _i),
         "boute_base_normals": ([ctypes.c_ulonglong, _i, _ll, _i, _i, _vp, _vp], _i),
         "boute_engine_set_normals": ([_vp, ctypes.c_ulonglong], _i),
+        "boute_engine_set_n": ([_vp, _i], _i),
         "boute_selftest_wait": ([_i, ctypes.c_ulonglong, _vp], _i),
         "boute_mobo_run": ([ctypes.POINTER(MoboConfig), _i, _i, _vp, _ll, _vp, _vp, _vp, _vp, _i,
                             _vp, _vp, _vp, _vp, _vp, _vp, _i, ObjectiveFn, _vp, _vp, _vp,
@@ -310,6 +311,12 @@ def boute_engine_set_normals(e: Engine, seed: int):
     _check(load().boute_engine_set_normals(e.handle, int(seed)), "boute_engine_set_normals")
 
 
+def boute_engine_set_n(e: Engine, n: int):
+    """Later steps use n <= the engine's creation n observations."""
+    _check(load().boute_engine_set_n(e.handle, int(n)), "boute_engine_set_n")
+    e.n = int(n)
+
+
 def boute_selftest_wait(complete: bool, limit_ns: int, stream=None) -> int:
     """Status of one bounded device-side wait (BOUTE_ERR_TIMEOUT if it ran out)."""
     return int(load().boute_selftest_wait(int(complete), int(limit_ns), _s(stream)))
@@ -400,6 +407,7 @@ class Engine:
     def __init__(self, B, n, d, m, N, mode, S, k):
         self.B, self.n, self.d, self.m, self.N, self.mode, self.S, self.k = (
             B, n, d, m, N, mode, S, k)
+        self.ncap = n
         h = _vp()
         _check(load().boute_engine_create(B, n, d, m, N, mode, S, k, ctypes.byref(h)),
                "boute_engine_create")

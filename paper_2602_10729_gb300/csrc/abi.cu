@@ -72,6 +72,7 @@ struct boute_gp {
 
 struct boute_engine {
   int B, n, d, m, mode, S, k;
+  int ncap;  // the buffers hold up to ncap observations (boute_engine_set_n)
   long long N;
   boute_gp *gp;
   double *X, *Y, *Ys, *ls, *s2, *noise, *ref, *front;
@@ -83,6 +84,7 @@ struct boute_engine {
   // 2-objective Monte-Carlo steps with k <= 32 select in the acquisition
   // kernel: its lists of keys and counters (zero between steps)
   unsigned char *sel;
+  size_t sel_bytes;
   bool fuse_sel;
   // K* of the candidates, computed on a second side stream while the fit
   // runs (it needs the fit's set-up, not its results); the posterior then
@@ -188,6 +190,7 @@ int boute_gp_create(int B, int n, int d, int m, boute_gp **out) {
   if (!h) return BOUTE_ERR_OOM;
   Gp &g = h->g;
   g.B = B; g.n = n; g.d = d; g.m = m; g.DP = pad_dims(d);
+  g.ncap = n;
   g.plan = make_post_plan(n);
   const size_t BM = (size_t)B * m;
   int r = BOUTE_OK;
@@ -197,7 +200,7 @@ int boute_gp_create(int B, int n, int d, int m, boute_gp **out) {
   r |= dalloc(&g.Aws, BM * np * (np + 1));
   r |= dalloc(&g.Wws, BM * np * (np + 1));
   r |= dalloc(&g.bop, BM * (size_t)g.plan.image_halves);
-  g.kcache_chunks = kstar_cache_chunks(g.plan);
+  g.kcache_chunks = g.kcache_cap = kstar_cache_chunks(g.plan);
   g.kcache_sms = num_sms();
   if (g.kcache_chunks > 0)
     r |= dalloc(&g.kcache, (size_t)g.kcache_sms * g.kcache_chunks * kKstarChunkHalves);
@@ -466,6 +469,7 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
   if (!e) return BOUTE_ERR_OOM;
   std::memset(e, 0, sizeof(*e));
   e->B = B; e->n = n; e->d = d; e->m = m; e->N = N; e->mode = mode; e->S = S; e->k = k;
+  e->ncap = n;
   int r = boute_gp_create(B, n, d, m, &e->gp);
   const size_t Bn = (size_t)B * n, BN = (size_t)B * N, cap = 2 * (size_t)n + 2;
   r |= dalloc(&e->X, Bn * d);
@@ -496,7 +500,7 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
   }
   e->fuse_sel = engine_fuses_selection(e);
   if (r == BOUTE_OK && e->fuse_sel) {
-    const size_t bytes = mchvi2_select_scratch_bytes(B, N, 2 * n + 2);
+    const size_t bytes = e->sel_bytes = mchvi2_select_scratch_bytes(B, N, 2 * n + 2);
     r |= dalloc(&e->sel, bytes);
     if (r == BOUTE_OK && cudaMemset(e->sel, 0, bytes) != cudaSuccess) {
       cudaGetLastError();
@@ -716,7 +720,7 @@ int boute_engine_step_async(boute_engine *e, const double *X, const double *Y,
 static void engine_reset_counters(boute_engine *e) {
   cudaDeviceSynchronize();
   cudaGetLastError();
-  if (e->sel) cudaMemset(e->sel, 0, mchvi2_select_scratch_bytes(e->B, e->N, 2 * e->n + 2));
+  if (e->sel) cudaMemset(e->sel, 0, e->sel_bytes);
   cudaMemset(e->scratch, 0, topk_scratch_bytes(e->B, e->N, e->k));
   cudaGetLastError();
 }
@@ -805,7 +809,7 @@ int boute_engine_step_host_async(boute_engine *e, const double *X, const double 
   if (!engine_args_ok(e, X, Y, lengthscale, outputscale, noise, ref, Xc, eps, idx, val))
     return BOUTE_ERR_INVALID_ARG;
   if (!e->X1) {  // the second input set, on first use
-    const size_t Bn = (size_t)e->B * e->n, BN = (size_t)e->B * e->N, Bm = (size_t)e->B * e->m;
+    const size_t Bn = (size_t)e->B * e->ncap, BN = (size_t)e->B * e->N, Bm = (size_t)e->B * e->m;
     int r = dalloc(&e->X1, Bn * e->d) | dalloc(&e->Y1, Bn * e->m) |
             dalloc(&e->ls1, Bm * e->d) | dalloc(&e->s21, Bm) | dalloc(&e->noise1, Bm) |
             dalloc(&e->ref1, Bm) | dalloc(&e->Xc1, BN * e->d);
@@ -892,6 +896,58 @@ static void engine_drop_graphs(boute_engine *e) {
     }
 }
 
+// Re-plan the handle for n <= ncap observations: the posterior's operand
+// layout (plan), its K* cache share, and zero padding in the operand images
+// and side inputs (their strides change with n).
+static int gp_set_n(Gp &g, int n) {
+  if (n < 1 || n > g.ncap) return BOUTE_ERR_INVALID_ARG;
+  if (n == g.n) return BOUTE_OK;
+  const size_t BM = (size_t)g.B * g.m;
+  const PostPlan cap = make_post_plan(g.ncap);
+  g.n = n;
+  g.plan = make_post_plan(n);
+  const int want = kstar_cache_chunks(g.plan);
+  g.kcache_chunks = want <= g.kcache_cap ? want : 0;  // else K* is rebuilt, not cached
+  if (cudaMemset(g.bop, 0, BM * (size_t)cap.image_halves * sizeof(uint16_t)) != cudaSuccess ||
+      cudaMemset(g.xt, 0, BM * (size_t)cap.nxt * xt_chunk_floats(g.DP) * sizeof(float)) !=
+          cudaSuccess) {
+    cudaGetLastError();
+    return BOUTE_ERR_CUDA;
+  }
+  return BOUTE_OK;
+}
+
+int boute_engine_set_n(boute_engine *e, int n) {
+  BOUTE_TRACE();
+  if (!e || n < 1 || n > e->ncap) return BOUTE_ERR_INVALID_ARG;
+  if (n == e->n) return BOUTE_OK;
+  if (cudaDeviceSynchronize() != cudaSuccess) return last_launch_status();
+  if (int r = gp_set_n(e->gp->g, n)) return r;
+  e->n = n;
+  engine_drop_graphs(e);  // the graphs hold n and the plan in their arguments
+  // the in-kernel selection's scratch grows as the boxes shrink (more
+  // resident blocks): keep it when it is large enough, else take a new one
+  e->fuse_sel = engine_fuses_selection(e);
+  if (e->fuse_sel) {
+    const size_t bytes = mchvi2_select_scratch_bytes(e->B, e->N, 2 * n + 2);
+    if (bytes > e->sel_bytes) {
+      cudaFree(e->sel);
+      e->sel = nullptr;
+      e->sel_bytes = 0;
+      if (dalloc(&e->sel, bytes) != BOUTE_OK) {
+        e->fuse_sel = false;
+        return BOUTE_ERR_OOM;
+      }
+      e->sel_bytes = bytes;
+      if (cudaMemset(e->sel, 0, bytes) != cudaSuccess) {
+        cudaGetLastError();
+        return BOUTE_ERR_CUDA;
+      }
+    }
+  }
+  return BOUTE_OK;
+}
+
 int boute_engine_set_kernel(boute_engine *e, int d_tau, const double *params) {
   BOUTE_TRACE();
   if (!e) return BOUTE_ERR_INVALID_ARG;
@@ -942,7 +998,7 @@ int boute_engine_set_outcome_transforms(boute_engine *e, const int *codes) {
   if (!e || !pack_codes(codes, e->m, &packed)) return BOUTE_ERR_INVALID_ARG;
   if (packed != e->tcodes) {
     if (cudaDeviceSynchronize() != cudaSuccess) return last_launch_status();
-    if (packed && !e->Yt && dalloc(&e->Yt, (size_t)e->B * e->n * e->m) != BOUTE_OK)
+    if (packed && !e->Yt && dalloc(&e->Yt, (size_t)e->B * e->ncap * e->m) != BOUTE_OK)
       return BOUTE_ERR_OOM;
     e->tcodes = packed;
     engine_drop_graphs(e);

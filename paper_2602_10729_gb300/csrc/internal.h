@@ -21,6 +21,9 @@ struct Gp {
   // need again (n > 512): kcache_chunks fp16 A-stage images per SM
   uint16_t *kcache;
   int kcache_chunks, kcache_sms;
+  // capacity: the buffers above are sized for ncap observations; n <= ncap
+  // (an engine re-plans its handle for each n of a growing data set)
+  int ncap, kcache_cap;
   float *xt;      // B*m x nxt x xt_chunk_floats(DP): X/lengthscale hi/lo, alpha
   float *s2f;     // B*m: outputscale
   int *status;    // device status word (first error wins)

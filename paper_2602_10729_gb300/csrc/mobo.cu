@@ -119,6 +119,13 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
       for (int k = 0; k < dc; ++k) pr[(size_t)t * dc + k] = kc[(size_t)t * KC + 3 + k];
     r = copy_in(dpref, pr.data(), sizeof(double) * m * dc);
   }
+  // one engine for the whole loop, sized for its largest data set (n grows
+  // by one per iteration up to nmax - 1 before the last selection)
+  boute_engine *e = nullptr;
+  if (!r && n0 < nmax) r = boute_engine_create(1, nmax - 1, d, m, N, cfg->mode, S, 1, &e);
+  if (!r && transforms) r = boute_engine_set_outcome_transforms(e, transforms);
+  if (!r && cons) r = boute_engine_set_constraints(e, cons);
+  if (!r && S && !eps) r = boute_engine_set_normals(e, cfg->seed);  // eps null: own normals
   std::vector<int> front = pareto_set(Y, n0, m, transforms);
   int n = n0, stable = 0, it = 0;
   std::vector<double> th((size_t)m * P);
@@ -169,14 +176,9 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
     if (!r) r = copy_in(ds2, s2, sizeof(double) * m);
     if (!r) r = copy_in(dnz, noise, sizeof(double) * m);
     // (ii) the acquisition over the pool and its best candidate
-    boute_engine *e = nullptr;
-    if (!r) r = boute_engine_create(1, n, d, m, N, cfg->mode, S, 1, &e);
-    if (!r && transforms) r = boute_engine_set_outcome_transforms(e, transforms);
-    if (!r && cons) r = boute_engine_set_constraints(e, cons);
+    if (!r) r = boute_engine_set_n(e, n);
     if (!r && kc) r = boute_engine_set_kernel(e, d_tau, kc);
-    if (!r && S && !eps) r = boute_engine_set_normals(e, cfg->seed);  // eps null: own normals
     if (!r) r = boute_engine_step(e, dX, dY, dls, ds2, dnz, dref, dXc, deps, didx, dval, nullptr);
-    boute_engine_free(e);
     long long pick = -1;
     if (!r && cudaMemcpy(&pick, didx, sizeof(pick), cudaMemcpyDeviceToHost) != cudaSuccess)
       r = BOUTE_ERR_CUDA;
@@ -200,6 +202,7 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
     }
   }
   *n_out = n;
+  boute_engine_free(e);
   void *bufs[] = {dX, dY, dYs, dls, ds2, dnz, dref, dth0, dth, dmll, dXc, deps, didx, dval, dpref};
   for (void *p : bufs) cudaFree(p);
   return r;

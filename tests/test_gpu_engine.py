@@ -218,3 +218,41 @@ def test_pipelined_host_steps_match_device_steps(wi, N, B):
     for (i, v), (wi_, wv) in zip(outs, want + want + want[:1]):
         assert np.array_equal(i.numpy(), wi_)
         assert np.array_equal(v.numpy(), wv)
+
+
+# (workload, cap, sizes): the engine is created for `cap` observations and
+# then stepped at each size in turn, on a stream (graphs re-captured per size),
+# from host buffers and eagerly; sizes above 512 use the posterior's K* cache, 2-objective
+# Monte-Carlo steps the in-kernel selection whose scratch depends on n
+SET_N_CASES = [(0, 300, [300, 37, 129, 200]), (1, 160, [64, 160, 95]),
+               (3, 1024, [1024, 700, 513, 600])]
+
+
+@pytest.mark.parametrize("case", SET_N_CASES, ids=lambda c: wl.WORKLOADS[c[0]].name)
+def test_engine_set_n_matches_fresh_engine(case):
+    """A capacity-sized engine re-planned to a smaller n gives the same
+    selection, bit for bit, as an engine created for that n."""
+    import torch
+
+    from paper_2602_10729_gb300 import boute as bt
+    wi, cap, sizes = case
+    base = wl.WORKLOADS[wi]
+    e = _engine(wl.scaled(base, N=2048 + 33, B=1, n=cap))
+    stream = torch.cuda.Stream()
+    for n in sizes:
+        w = wl.scaled(base, N=2048 + 33, B=1, n=n)
+        hp = host_problem(w)
+        bt.boute_engine_set_n(e, n)
+        fresh = _engine(w)
+        with torch.cuda.stream(stream):
+            ref_idx, ref_val = _run(fresh, w, _dev(hp), "device")
+            for how in ("device", "device", "host", "legacy"):  # capture, replay, ...
+                idx, val = _run(e, w, _host(hp) if how == "host" else _dev(hp), how)
+                assert np.array_equal(idx, ref_idx), (n, how)
+                assert np.array_equal(val, ref_val), (n, how)
+        fresh.free()
+    with pytest.raises(RuntimeError):
+        bt.boute_engine_set_n(e, cap + 1)
+    with pytest.raises(RuntimeError):
+        bt.boute_engine_set_n(e, 0)
+    e.free()
