@@ -7,8 +7,9 @@ wrapper. Only the test suite, ``__graft_entry__.smoke()`` and ``bench.py``'s
 CPU-baseline leg may import it; the CUDA library never does, and the two share
 no code.
 
-Parity pins live in ``tests/test_oracle_pins.py``. Functions without an
-independent pin: none.
+Parity pins live in ``tests/test_oracle_pins.py`` and, for the noisy
+acquisition (joint in-sample draws), ``tests/test_oracle_noisy.py``. Functions
+without an independent pin: none.
 """
 from __future__ import annotations
 
@@ -97,6 +98,14 @@ def lib():
                                 ctypes.c_longlong, _dp, ctypes.c_int, _dp, _dp, _dp,
                                 ctypes.c_int]
         L.bo_mc_hvi.restype = None
+        L.bo_joint_draws.argtypes = [_dp, _dp, ctypes.c_int, ctypes.c_int, _dp, ctypes.c_double,
+                                     ctypes.c_double, ctypes.c_int, _dp, ctypes.c_double, _fp,
+                                     ctypes.c_int, _fp, ctypes.c_longlong, _dp, _dp, _dp, _dp,
+                                     ctypes.c_int]
+        L.bo_nehvi_mc.argtypes = [_dp, ctypes.c_int, ctypes.c_int, ctypes.c_int, _dp, _dp, _dp,
+                                  _fp, ctypes.c_longlong, ctypes.c_longlong, _dp, _dp, _dp,
+                                  ctypes.c_int]
+        L.bo_nehvi_mc.restype = None
         L.bo_topk.argtypes = [_dp, ctypes.c_longlong, ctypes.c_int, _lp, _dp]
         L.bo_topk.restype = None
         L.bo_default_threads.restype = ctypes.c_int
@@ -361,6 +370,61 @@ def mc_hvi(mean, var, eps, F, ref, eps_stride: int | None = None, threads: int =
     acq = np.empty(N)
     lib().bo_mc_hvi(pm, pv, N, m, pe, S, stride, pF, F.shape[0], pr, pc,
                     acq.ctypes.data_as(_dp), threads)
+    return acq
+
+
+# The in-sample jitter of the noisy acquisition, relative to the outputscale:
+# the in-sample posterior covariance K_nn - K_nn K^-1 K_nn is singular up to
+# rounding wherever the data pin the function down (the paper's qNEHVI
+# samples it through a Cholesky factor and leaves the regularisation open).
+JOINT_JITTER = 1e-8
+
+
+def joint_draws(X, y, ls, s2, noise, z, Xc, jitter: float = JOINT_JITTER, threads: int = 0,
+                kernel=None):
+    """Joint posterior draws of one objective at the observed points and the
+    candidates (Sec. 5.2, constrained qNEHVI). z: (S, n) float32 in-sample
+    normals. Returns Yin (S, n), mean (N,), cvar (N,), shift (N, S); the
+    candidate's draw s is mean + shift[:, s] + sqrt(max(cvar, 0)) eps_s."""
+    X, pX = _d(X)
+    y, py = _d(y)
+    ls, pl = _d(ls)
+    z, pz = _f(z)
+    Xc, pc = _f(Xc)
+    n, d = X.shape
+    S = z.shape[0]
+    N = Xc.shape[0]
+    Yin = np.empty((S, n))
+    mean = np.empty(N)
+    cvar = np.empty(N)
+    shift = np.empty((N, S))
+    dtau, kc, pk = _kern(kernel)
+    rc = lib().bo_joint_draws(pX, py, n, d, pl, float(s2), float(noise), dtau, pk, float(jitter),
+                              pz, S, pc, N, Yin.ctypes.data_as(_dp), mean.ctypes.data_as(_dp),
+                              cvar.ctypes.data_as(_dp), shift.ctypes.data_as(_dp), threads)
+    if rc == 2:
+        raise NotPositiveDefinite("kernel matrix or in-sample covariance not positive definite")
+    if rc:
+        raise ValueError(rc)
+    return Yin, mean, cvar, shift
+
+
+def nehvi_mc(Yin, mean, cvar, shift, eps, ref, threads: int = 0, cons=None):
+    """Noisy MC hypervolume improvement (q = 1). Yin: (S, n, m) in-sample
+    draws; mean, cvar: (N, m); shift: (N, m, S); eps: float32 (N, m, S);
+    cons: m thresholds on the minimised objectives or None."""
+    Yin, pY = _d(Yin)
+    mean, pm = _d(mean)
+    cvar, pv = _d(cvar)
+    shift, ps = _d(shift)
+    eps, pe = _f(eps)
+    ref, pr = _d(ref)
+    c, pcn = _cons(cons)
+    S, n, m = Yin.shape
+    N = mean.shape[0]
+    acq = np.empty(N)
+    lib().bo_nehvi_mc(pY, n, m, S, pm, pv, ps, pe, m * S, N, pr, pcn, acq.ctypes.data_as(_dp),
+                      threads)
     return acq
 
 

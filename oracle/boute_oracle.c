@@ -676,6 +676,178 @@ void bo_mc_hvi(const double *mean, const double *var, long long N, int m,
   }
 }
 
+/* ---- noisy expected hypervolume improvement (in-sample joint draws) --------- */
+/* Lower Cholesky factor of the n x n matrix A in place (Cholesky-Banachiewicz);
+ * the upper triangle is set to 0. Returns 2 when a pivot is not positive. */
+static int chol_in_place(double *A, int n) {
+  for (int i = 0; i < n; ++i) {
+    for (int j = 0; j <= i; ++j) {
+      double s = A[(long)i * n + j];
+      for (int k = 0; k < j; ++k) s -= A[(long)i * n + k] * A[(long)j * n + k];
+      if (i == j) {
+        if (!(s > 0.0)) return 2;
+        A[(long)i * n + i] = sqrt(s);
+      } else {
+        A[(long)i * n + j] = s / A[(long)j * n + j];
+      }
+    }
+    for (int j = i + 1; j < n; ++j) A[(long)i * n + j] = 0.0;
+  }
+  return 0;
+}
+
+/* x = L^-1 b by forward substitution (L lower, n x n) */
+static void fwd_subst(const double *L, int n, const double *b, double *x) {
+  for (int i = 0; i < n; ++i) {
+    double s = b[i];
+    for (int k = 0; k < i; ++k) s -= L[(long)i * n + k] * x[k];
+    x[i] = s / L[(long)i * n + i];
+  }
+}
+
+int bo_joint_draws(const double *X, const double *y, int n, int d, const double *ls, double s2,
+                   double noise, int dtau, const double *kc, double jitter, const float *z, int S,
+                   const float *Xc, long long N, double *Yin, double *mean, double *cvar,
+                   double *shift, int nthreads) {
+  if (n < 1 || d < 1 || S < 1 || N < 0 || !X || !y || !ls || !z) return 1;
+  const long nn = (long)n * n;
+  double *L = (double *)malloc(sizeof(double) * nn), *alpha = (double *)malloc(sizeof(double) * n);
+  double *Knn = (double *)malloc(sizeof(double) * nn), *V = (double *)malloc(sizeof(double) * nn);
+  double *F = (double *)malloc(sizeof(double) * nn), *col = (double *)malloc(sizeof(double) * n);
+  double *mu = (double *)malloc(sizeof(double) * n);
+  int rc = bo_gp_fit_k(X, y, n, d, ls, s2, noise, dtau, kc, L, alpha);
+  if (rc) goto done;
+  /* the noise-free kernel matrix and V = L^-1 K_nn, column by column */
+  for (int i = 0; i < n; ++i)
+    for (int j = 0; j < n; ++j)
+      Knn[(long)i * n + j] = bo_kernel(X + (long)i * d, X + (long)j * d, d, ls, s2, dtau, kc);
+  for (int j = 0; j < n; ++j) {
+    for (int i = 0; i < n; ++i) col[i] = Knn[(long)i * n + j];
+    double *v = mu; /* scratch */
+    fwd_subst(L, n, col, v);
+    for (int i = 0; i < n; ++i) V[(long)i * n + j] = v[i];
+  }
+  /* in-sample posterior: mean K_nn alpha, covariance K_nn - K_nn K^-1 K_nn =
+   * K_nn - V^T V, plus jitter * s2 on the diagonal; F its Cholesky factor */
+  for (int i = 0; i < n; ++i) {
+    double m_i = 0.0;
+    for (int j = 0; j < n; ++j) m_i += Knn[(long)i * n + j] * alpha[j];
+    mu[i] = m_i;
+  }
+  for (int i = 0; i < n; ++i)
+    for (int j = 0; j < n; ++j) {
+      double c = Knn[(long)i * n + j];
+      for (int k = 0; k < n; ++k) c -= V[(long)k * n + i] * V[(long)k * n + j];
+      F[(long)i * n + j] = c + (i == j ? jitter * s2 : 0.0);
+    }
+  rc = chol_in_place(F, n);
+  if (rc) goto done;
+  /* the in-sample draws mu + F z_s */
+  for (int s = 0; s < S; ++s)
+    for (int i = 0; i < n; ++i) {
+      double v = mu[i];
+      for (int j = 0; j <= i; ++j) v += F[(long)i * n + j] * (double)z[(long)s * n + j];
+      Yin[(long)s * n + i] = v;
+    }
+  /* each candidate: marginal mean and variance, the cross-covariance with the
+   * observed points Sigma_nx = k* - K_nn K^-1 k* = k* - V^T (L^-1 k*), its
+   * coefficients l = F^-1 Sigma_nx on the in-sample normals, and the variance
+   * left once the in-sample values are fixed, var - l^T l */
+  {
+    const int nt = nthreads_or_default(nthreads);
+#pragma omp parallel num_threads(nt)
+    {
+      double *ks = (double *)malloc(sizeof(double) * (4 * (size_t)n + (size_t)d));
+      double *v = ks + n, *sx = v + n, *l = sx + n, *xd = l + n;
+#pragma omp for schedule(dynamic, 16)
+      for (long long c = 0; c < N; ++c) {
+        for (int k = 0; k < d; ++k) xd[k] = (double)Xc[c * d + k];
+        for (int j = 0; j < n; ++j) ks[j] = bo_kernel(X + (long)j * d, xd, d, ls, s2, dtau, kc);
+        const double kxx = bo_kernel(xd, xd, d, ls, s2, dtau, kc);
+        double mc = 0.0;
+        for (int j = 0; j < n; ++j) mc += ks[j] * alpha[j];
+        fwd_subst(L, n, ks, v);
+        double vv = 0.0;
+        for (int j = 0; j < n; ++j) vv += v[j] * v[j];
+        for (int i = 0; i < n; ++i) {
+          double t = ks[i];
+          for (int k = 0; k < n; ++k) t -= V[(long)k * n + i] * v[k];
+          sx[i] = t;
+        }
+        fwd_subst(F, n, sx, l);
+        double ll = 0.0;
+        for (int j = 0; j < n; ++j) ll += l[j] * l[j];
+        mean[c] = mc;
+        cvar[c] = kxx - vv - ll;
+        for (int s = 0; s < S; ++s) {
+          double t = 0.0;
+          for (int j = 0; j < n; ++j) t += l[j] * (double)z[(long)s * n + j];
+          shift[c * S + s] = t;
+        }
+      }
+      free(ks);
+    }
+  }
+done:
+  free(L); free(alpha); free(Knn); free(V); free(F); free(col); free(mu);
+  return rc;
+}
+
+void bo_nehvi_mc(const double *Yin, int n, int m, int S, const double *mean, const double *cvar,
+                 const double *shift, const float *eps, long long eps_stride, long long N,
+                 const double *ref, const double *cons, double *acq, int nthreads) {
+  /* per sample: the Pareto front of the feasible in-sample draws */
+  double *fr = (double *)malloc(sizeof(double) * (size_t)S * n * m + 1);
+  int *P = (int *)malloc(sizeof(int) * (size_t)S);
+  double *hvF = (double *)malloc(sizeof(double) * (size_t)S);
+  double *pts = (double *)malloc(sizeof(double) * (size_t)n * m + 1);
+  unsigned char *mask = (unsigned char *)malloc((size_t)n + 1);
+  int *order = (int *)malloc(sizeof(int) * (size_t)n + 1);
+  for (int s = 0; s < S; ++s) {
+    int q = 0;
+    for (int i = 0; i < n; ++i) {
+      const double *yi = Yin + ((long)s * n + i) * m;
+      int ok = 1;
+      for (int t = 0; t < m && cons; ++t)
+        if (!(yi[t] <= cons[t])) ok = 0;
+      if (ok) memcpy(pts + (long)(q++) * m, yi, sizeof(double) * m);
+    }
+    const int np = bo_pareto_front(pts, q, m, ref, mask, order);
+    for (int k = 0; k < np; ++k)
+      memcpy(fr + ((long)s * n + k) * m, pts + (long)order[k] * m, sizeof(double) * m);
+    P[s] = np;
+    hvF[s] = bo_hv(fr + (long)s * n * m, np, m, ref, NULL);
+  }
+  free(pts); free(mask); free(order);
+  const int nt = nthreads_or_default(nthreads);
+  long long scr = bo_hv_scratch_size(n + 1, m);
+#pragma omp parallel num_threads(nt)
+  {
+    double *all = (double *)malloc(sizeof(double) * (size_t)((n + 1) * m + m + scr));
+    double *sg = all + (long)(n + 1) * m, *scratch = sg + m;
+#pragma omp for schedule(dynamic, 64)
+    for (long long c = 0; c < N; ++c) {
+      for (int t = 0; t < m; ++t) sg[t] = sqrt(cvar[c * m + t] > 0.0 ? cvar[c * m + t] : 0.0);
+      double sum = 0.0;
+      for (int s = 0; s < S; ++s) {
+        const int np = P[s];
+        memcpy(all, fr + (long)s * n * m, sizeof(double) * (size_t)np * m);
+        int feasible = 1;
+        for (int t = 0; t < m; ++t) {
+          const double v = mean[c * m + t] + shift[(c * m + t) * S + s] +
+                           sg[t] * (double)eps[c * eps_stride + (long long)t * S + s];
+          all[(long)np * m + t] = v;
+          if (cons && !(v <= cons[t])) feasible = 0;
+        }
+        if (feasible) sum += bo_hv(all, np + 1, m, ref, scratch) - hvF[s]; /* else HVI x 0 */
+      }
+      acq[c] = sum / S;
+    }
+    free(all);
+  }
+  free(fr); free(P); free(hvF);
+}
+
 /* ---- top-k ----------------------------------------------------------------- */
 static _Thread_local const double *g_topv;
 static int cmp_top(const void *pa, const void *pb) {

@@ -176,6 +176,39 @@ void bo_mc_hvi(const double *mean, const double *var, long long N, int m,
                const float *eps, int S, long long eps_stride, const double *F,
                int P, const double *ref, const double *cons, double *acq, int nthreads);
 
+/* Joint posterior draws for the noisy acquisition (Sec. 5.2, constrained
+ * qNEHVI: the expectation runs over samples of the joint posterior, here of
+ * the objective at the n observed points and at each candidate, so that the
+ * front the candidate improves on is itself a posterior draw). One objective,
+ * the fit of bo_gp_fit_k. For S in-sample normals z (S x n float):
+ *   Yin[s] = mu_n + F z_s, mu_n = K_nn alpha, F = chol(K_nn - K_nn K^-1 K_nn
+ *   + jitter s2 I) (K_nn the noise-free kernel matrix, K = K_nn + noise I);
+ * and for each candidate x (Xc: N x d float) the marginal mean, the
+ * cross-covariance Sigma_nx = k* - K_nn K^-1 k*, l = F^-1 Sigma_nx, and
+ *   cvar = k(x, x) - k*^T K^-1 k* - l^T l,  shift[x][s] = l^T z_s,
+ * so that the joint draw at x is mean + shift_s + sqrt(cvar) eps_s: the
+ * Cholesky factor of the joint covariance of (f(X), f(x)) with the jitter on
+ * the in-sample block, applied to (z_s, eps_s). Yin: S x n; mean, cvar: N;
+ * shift: N x S. Returns 2 when K or the in-sample covariance is not positive
+ * definite. nthreads <= 0: library default. */
+int bo_joint_draws(const double *X, const double *y, int n, int d, const double *ls, double s2,
+                   double noise, int dtau, const double *kc, double jitter, const float *z, int S,
+                   const float *Xc, long long N, double *Yin, double *mean, double *cvar,
+                   double *shift, int nthreads);
+
+/* Monte-Carlo noisy expected hypervolume improvement (Sec. 5.2, constrained
+ * qNEHVI with q = 1): for each sample s the front is the Pareto front
+ * (bo_pareto_front against ref) of the in-sample draws Yin[s] (n x m) that
+ * satisfy the constraints (y_t <= cons[t] for every t; all of them when cons
+ * is NULL); the candidate's draw y_t = mean_t + shift_t,s + sqrt(max(cvar_t,
+ * 0)) eps_t,s counts its hypervolume improvement over that front when it is
+ * feasible itself; acq = the average over the S samples. Yin: S x n x m;
+ * mean, cvar: N x m; shift: N x m x S; eps: float, candidate c's block at
+ * c * eps_stride, (m, S) row-major. */
+void bo_nehvi_mc(const double *Yin, int n, int m, int S, const double *mean, const double *cvar,
+                 const double *shift, const float *eps, long long eps_stride, long long N,
+                 const double *ref, const double *cons, double *acq, int nthreads);
+
 /* Top-k selection (Sec. 5.2 step (ii): the next configuration is the best
  * scored candidate): the first k entries of the order (value descending, NaN
  * as -infinity, equal values by ascending index). idx, val: k. */

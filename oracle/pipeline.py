@@ -12,8 +12,8 @@ from dataclasses import dataclass
 
 import numpy as np
 
-from . import (ehvi2d, gp_fit, gp_posterior, mc_hvi, outcome_transform, pareto_front, standardize,
-               topk)
+from . import (JOINT_JITTER, ehvi2d, gp_fit, gp_posterior, joint_draws, mc_hvi, nehvi_mc,
+               outcome_transform, pareto_front, standardize, topk)
 
 
 @dataclass
@@ -78,3 +78,47 @@ def score(fp: FittedProblem, Xc, mode: str, k: int, eps=None, threads: int = 0, 
     acq = acquisition(fp, mean, var, mode, eps, threads, cons=cons)
     idx, val = topk(acq, k)
     return mean, var, acq, idx, val
+
+
+@dataclass
+class NoisyDraws:
+    Yin: np.ndarray  # S x n x m in-sample joint draws
+    mean: np.ndarray  # N x m
+    cvar: np.ndarray  # N x m, variance left once the in-sample values are drawn
+    shift: np.ndarray  # N x m x S
+
+
+def noisy_draws(fp: FittedProblem, Xc, z, jitter: float = JOINT_JITTER,
+                threads: int = 0) -> NoisyDraws:
+    """Joint posterior draws of every objective (independent GPs, Sec. 6) at
+    the observed points and the candidates. z: (m, S, n) float32 in-sample
+    normals."""
+    Xc = np.ascontiguousarray(Xc, np.float32)
+    m = fp.Ys.shape[1]
+    z = np.asarray(z, np.float32)
+    S, n = z.shape[1], z.shape[2]
+    N = Xc.shape[0]
+    Yin = np.empty((S, n, m))
+    mean = np.empty((N, m))
+    cvar = np.empty((N, m))
+    shift = np.empty((N, m, S))
+    for t in range(m):
+        Yin[:, :, t], mean[:, t], cvar[:, t], shift[:, t, :] = joint_draws(
+            fp.X, fp.Ys[:, t], fp.ls[t], fp.s2[t], fp.noise[t], z[t], Xc, jitter, threads,
+            None if fp.kernel is None else fp.kernel[t])
+    return NoisyDraws(Yin, mean, cvar, shift)
+
+
+def noisy_acquisition(fp: FittedProblem, dr: NoisyDraws, eps, threads: int = 0, cons=None):
+    """Noisy MC hypervolume improvement of every candidate (Sec. 5.2,
+    constrained qNEHVI, q = 1): the front of each sample is that of its
+    feasible in-sample draws."""
+    return nehvi_mc(dr.Yin, dr.mean, dr.cvar, dr.shift, eps, fp.ref, threads, cons=cons)
+
+
+def noisy_score(fp: FittedProblem, Xc, z, eps, k: int, threads: int = 0, cons=None,
+                jitter: float = JOINT_JITTER):
+    dr = noisy_draws(fp, Xc, z, jitter, threads)
+    acq = noisy_acquisition(fp, dr, eps, threads, cons)
+    idx, val = topk(acq, k)
+    return dr, acq, idx, val
