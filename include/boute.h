@@ -255,6 +255,61 @@ int boute_acq_mc_hvi(const float *mean, const float *var, int B, long long N, in
                      const float *eps, int S, long long eps_cand_stride, const double *cons,
                      float *acq, void *stream);
 
+/* ---- noisy acquisition: in-sample joint draws ------------------------------------
+ * Sec. 5.2, "Constrained qNEHVI" (q = 1): the expectation runs over samples of
+ * the JOINT posterior of each objective at the n observed points X and at the
+ * candidate, so that the front a candidate improves on is itself a posterior
+ * draw (the observations are noisy). Draw s of objective t uses the Cholesky
+ * factor of the joint covariance, with a jitter of 1e-8 * outputscale on the
+ * in-sample block, applied to the normals (z_s, eps_s):
+ *   Yin_s = mu_n + F z_s,  mu_n = K_nn alpha,
+ *   F = chol(K_nn - K_nn K^-1 K_nn + 1e-8 s2 I)   (K = K_nn + noise I)
+ *   y_s(x) = mean(x) + l(x)^T z_s + sqrt(cvar(x)) eps_s,  l = F^-1 Sigma_nx,
+ *   cvar = k(x, x) - k*^T K^-1 k* - l^T l,  Sigma_nx = k* - K_nn K^-1 k*.
+ * The per-candidate terms are contractions of k* (l^T z_s = k*^T G_s with
+ * G = noise K^-1 F^-T Z), computed by the posterior's tensor-core kernel as
+ * extra output columns.
+ *
+ * boute_gp_set_insample(gp, S): the handle's later fits prepare S in-sample
+ * draws (1 <= S <= 1024; 0 turns them off). It re-plans the operand images,
+ * which are then zero: fit again before the next insample or posterior call.
+ * Allocates; waits for all work on the device. n (the handle's capacity)
+ * <= 128 and the FP32 tier, else BOUTE_ERR_UNSUPPORTED.
+ * boute_gp_insample, after boute_gp_fit with the same Ys, outputscale and
+ * noise (B x n x m, B x m, B x m fp64): reads z (B x m x S x n fp32 standard
+ * normals) and writes Yin (B x m x S x n fp32), and prepares the handle's
+ * shift operands. A factor that is not positive definite records
+ * BOUTE_ERR_NOT_PD (boute_gp_status).
+ * boute_gp_posterior_joint: mean and cvar as boute_gp_posterior's mean and
+ * var (B x m x N fp32; cvar clamped at 0) and shift[b][t][s][c] = l(x_c)^T z_s
+ * (B x m x S x N fp32). boute_gp_posterior on such a handle still gives the
+ * plain posterior. */
+int boute_gp_set_insample(boute_gp *gp, int S);
+int boute_gp_insample(boute_gp *gp, const double *Ys, const double *outputscale,
+                      const double *noise, const float *z, float *Yin, void *stream);
+int boute_gp_posterior_joint(const boute_gp *gp, const float *Xc, long long N, float *mean,
+                             float *cvar, float *shift, void *stream);
+/* The front of each in-sample draw (two objectives): the Pareto front,
+ * against ref (B x 2 fp64), of the draw's points that meet the constraints
+ * (cons: NULL or B x 2 fp64 thresholds, y_t <= cons_t) as the vertical strips
+ * of the region it leaves undominated. Yin: B x 2 x S x n fp32 (n <= 128);
+ * strips: B x S x (n + 1) x 4 fp32, strip j of draw s = (l1, u1, u2, 0): the
+ * cells [l1, u1) x (-inf, u2), sorted by l1 (strip 0 has l1 = -inf);
+ * counts: B x S int, the strips of each draw (front size + 1). */
+int boute_insample_fronts(const float *Yin, int B, int n, int S, const double *ref,
+                          const double *cons, float *strips, int *counts, void *stream);
+/* Noisy MC hypervolume improvement (two objectives): draw s of candidate c
+ * is y_t = mean_t + shift_t,s + sqrt(cvar_t) eps_t,s (eps laid out as for
+ * boute_acq_mc_hvi); with cons, a draw counts only when y_t <= cons_t for
+ * both t (fp32 comparison); its improvement is the area of [y, ref] inside
+ * draw s's strips: sum_j (u1_j - max(l1_j, y_1))+ (u2_j - y_2)+; acq (B x N
+ * fp32) = the mean over the S draws. mean, cvar, shift: the layouts of
+ * boute_gp_posterior_joint; strips, counts, n: boute_insample_fronts's. */
+int boute_acq_nehvi2d(const float *mean, const float *cvar, const float *shift, int B,
+                      long long N, int S, const float *eps, long long eps_cand_stride,
+                      const float *strips, const int *counts, int n, const double *cons,
+                      float *acq, void *stream);
+
 /* Failure detection: every device-side wait of the library is bounded (about
  * 2 s) and a wait that runs out records BOUTE_ERR_TIMEOUT in the call's
  * status instead of hanging. This self-test runs one such bounded wait on

@@ -24,6 +24,8 @@ SYMBOLS = (
     "boute_status_string", "boute_launch_count", "boute_standardize", "boute_gp_create",
     "boute_gp_fit", "boute_gp_status", "boute_gp_free", "boute_gp_posterior",
     "boute_gp_set_precision", "boute_gp_posterior_fp64",
+    "boute_gp_set_insample", "boute_gp_insample", "boute_gp_posterior_joint",
+    "boute_insample_fronts", "boute_acq_nehvi2d",
     "boute_pareto_front", "boute_box_decompose", "boute_acq_ehvi", "boute_acq_mc_hvi",
     "boute_select_topk", "boute_select_topk_noalloc", "boute_engine_create", "boute_engine_step",
     "boute_engine_step_async",
@@ -84,6 +86,12 @@ def load(path: str | None = None):
         "boute_gp_status": ([_vp, _vp], _i),
         "boute_gp_free": ([_vp], None),
         "boute_gp_posterior": ([_vp, _vp, _ll, _vp, _vp, _vp], _i),
+        "boute_gp_set_insample": ([_vp, _i], _i),
+        "boute_gp_insample": ([_vp, _vp, _vp, _vp, _vp, _vp, _vp], _i),
+        "boute_gp_posterior_joint": ([_vp, _vp, _ll, _vp, _vp, _vp, _vp], _i),
+        "boute_insample_fronts": ([_vp, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
+        "boute_acq_nehvi2d": ([_vp, _vp, _vp, _i, _ll, _i, _vp, _ll, _vp, _vp, _i, _vp, _vp,
+                               _vp], _i),
         "boute_gp_set_precision": ([_vp, _i], _i),
         "boute_gp_posterior_fp64": ([_vp, _vp, _ll, _vp, _vp, _vp], _i),
         "boute_pareto_front": ([_vp, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
@@ -342,6 +350,44 @@ def boute_gp_posterior(gp: Gp, Xc, N: int, mean, var, stream=None):
 
 
 BOUTE_PREC_FP32, BOUTE_PREC_FP64 = 0, 1
+
+
+def boute_gp_set_insample(gp: Gp, S: int):
+    """S in-sample joint draws for the noisy acquisition (0: off); fit again after."""
+    _check(load().boute_gp_set_insample(gp.handle, int(S)), "boute_gp_set_insample")
+
+
+def boute_gp_insample(gp: Gp, Ys, outputscale, noise, z, Yin, stream=None):
+    """After boute_gp_fit: z (B x m x S x n fp32) in, Yin (same shape) out."""
+    f64, f32 = torch.float64, torch.float32
+    _check(load().boute_gp_insample(gp.handle, _p(Ys, f64), _p(outputscale, f64),
+                                    _p(noise, f64), _p(z, f32), _p(Yin, f32), _s(stream)),
+           "boute_gp_insample")
+
+
+def boute_gp_posterior_joint(gp: Gp, Xc, N: int, mean, cvar, shift, stream=None):
+    """mean, cvar: B x m x N; shift: B x m x S x N (fp32 CUDA tensors)."""
+    f32 = torch.float32
+    _check(load().boute_gp_posterior_joint(gp.handle, _p(Xc, f32), N, _p(mean, f32),
+                                           _p(cvar, f32), _p(shift, f32), _s(stream)),
+           "boute_gp_posterior_joint")
+
+
+def boute_insample_fronts(Yin, B, n, S, ref, strips, counts, stream=None, cons=None):
+    """Yin: B x 2 x S x n; strips: B x S x (n + 1) x 4 fp32; counts: B x S int32."""
+    _check(load().boute_insample_fronts(_p(Yin, torch.float32), B, n, S, _p(ref, torch.float64),
+                                        _p(cons, torch.float64), _p(strips, torch.float32),
+                                        _p(counts, torch.int32), _s(stream)),
+           "boute_insample_fronts")
+
+
+def boute_acq_nehvi2d(mean, cvar, shift, B, N, S, eps, eps_cand_stride, strips, counts, n, acq,
+                      stream=None, cons=None):
+    f32 = torch.float32
+    _check(load().boute_acq_nehvi2d(_p(mean, f32), _p(cvar, f32), _p(shift, f32), B, N, S,
+                                    _p(eps, f32), eps_cand_stride, _p(strips, f32),
+                                    _p(counts, torch.int32), n, _p(cons, torch.float64),
+                                    _p(acq, f32), _s(stream)), "boute_acq_nehvi2d")
 
 
 def boute_gp_set_precision(gp: Gp, prec: int):

@@ -243,7 +243,7 @@ int boute_gp_set_precision(boute_gp *gp, int prec) {
   if (!gp || (prec != BOUTE_PREC_FP32 && prec != BOUTE_PREC_FP64)) return BOUTE_ERR_INVALID_ARG;
   Gp &g = gp->g;
   if (prec == BOUTE_PREC_FP64) {
-    if (g.n > kFp64MaxN || g.kern) return BOUTE_ERR_UNSUPPORTED;
+    if (g.n > kFp64MaxN || g.kern || g.plan.S_in > 0) return BOUTE_ERR_UNSUPPORTED;
     if (!g.W64) {
       const size_t BM = (size_t)g.B * g.m;
       int r = dalloc(&g.W64, BM * g.n * g.n);
@@ -266,6 +266,97 @@ int boute_gp_posterior_fp64(const boute_gp *gp, const float *Xc, long long N, do
   return launch_posterior64(&gp->g, Xc, N, mean, var, (cudaStream_t)stream);
 }
 
+// ---- noisy acquisition: in-sample draws -----------------------------------------
+int boute_gp_set_insample(boute_gp *gp, int S) {
+  BOUTE_TRACE();
+  if (!gp || S < 0 || S > kInsMaxS) return BOUTE_ERR_INVALID_ARG;
+  Gp &g = gp->g;
+  if (S == g.plan.S_in) return BOUTE_OK;
+  if (S > 0 && (g.ncap > kInsMaxN || g.prec != BOUTE_PREC_FP32)) return BOUTE_ERR_UNSUPPORTED;
+  if (cudaDeviceSynchronize() != cudaSuccess) return last_launch_status();
+  const size_t BM = (size_t)g.B * g.m;
+  const PostPlan cap = make_post_plan(g.ncap, S);
+  // new operand images (W's blocks then H^T's and G^T's), zero: fit again
+  uint16_t *bop = nullptr;
+  if (dalloc(&bop, BM * (size_t)cap.image_halves) != BOUTE_OK) return BOUTE_ERR_OOM;
+  float *gws = nullptr;
+  if (S > 0 && dalloc(&gws, BM * (size_t)S * g.ncap) != BOUTE_OK) {
+    cudaFree(bop);
+    return BOUTE_ERR_OOM;
+  }
+  const int want = kstar_cache_chunks(cap);
+  uint16_t *kc = nullptr;
+  if (want > g.kcache_cap &&
+      dalloc(&kc, (size_t)g.kcache_sms * want * kKstarChunkHalves) != BOUTE_OK) {
+    cudaFree(bop);
+    cudaFree(gws);
+    return BOUTE_ERR_OOM;
+  }
+  if (cudaMemset(bop, 0, BM * (size_t)cap.image_halves * sizeof(uint16_t)) != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(bop);
+    cudaFree(gws);
+    cudaFree(kc);
+    return BOUTE_ERR_CUDA;
+  }
+  cudaFree(g.bop);
+  g.bop = bop;
+  cudaFree(g.gws);
+  g.gws = gws;
+  if (kc) {
+    cudaFree(g.kcache);
+    g.kcache = kc;
+    g.kcache_cap = want;
+  }
+  g.plan = make_post_plan(g.n, S);
+  const int now = kstar_cache_chunks(g.plan);
+  g.kcache_chunks = now <= g.kcache_cap ? now : 0;
+  return BOUTE_OK;
+}
+
+int boute_gp_insample(boute_gp *gp, const double *Ys, const double *outputscale,
+                      const double *noise, const float *z, float *Yin, void *stream) {
+  BOUTE_TRACE();
+  if (!gp || !Ys || !outputscale || !noise || !z || !Yin) return BOUTE_ERR_INVALID_ARG;
+  if (gp->g.plan.S_in < 1) return BOUTE_ERR_INVALID_ARG;
+  return launch_insample(&gp->g, Ys, outputscale, noise, z, Yin, (cudaStream_t)stream);
+}
+
+int boute_gp_posterior_joint(const boute_gp *gp, const float *Xc, long long N, float *mean,
+                             float *cvar, float *shift, void *stream) {
+  BOUTE_TRACE();
+  if (!gp || N < 0 || (N > 0 && (!Xc || !mean || !cvar || !shift))) return BOUTE_ERR_INVALID_ARG;
+  if (gp->g.plan.S_in < 1) return BOUTE_ERR_INVALID_ARG;
+  if ((long long)gp->g.B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;
+  return launch_posterior_joint(&gp->g, Xc, N, mean, cvar, shift, (cudaStream_t)stream);
+}
+
+int boute_insample_fronts(const float *Yin, int B, int n, int S, const double *ref,
+                          const double *cons, float *strips, int *counts, void *stream) {
+  BOUTE_TRACE();
+  if (!Yin || !ref || !strips || !counts || B < 1 || n < 1 || S < 1 || S > kInsMaxS)
+    return BOUTE_ERR_INVALID_ARG;
+  if (n > kInsMaxN) return BOUTE_ERR_UNSUPPORTED;
+  if (int r = device_ok()) return r;
+  return launch_insample_fronts(Yin, B, n, S, ref, cons, strips, counts, (cudaStream_t)stream);
+}
+
+int boute_acq_nehvi2d(const float *mean, const float *cvar, const float *shift, int B,
+                      long long N, int S, const float *eps, long long eps_cand_stride,
+                      const float *strips, const int *counts, int n, const double *cons,
+                      float *acq, void *stream) {
+  BOUTE_TRACE();
+  if (B < 1 || N < 0 || S < 1 || S > kInsMaxS || n < 1 || eps_cand_stride < 0 || !strips ||
+      !counts || (N > 0 && (!mean || !cvar || !shift || !eps || !acq)))
+    return BOUTE_ERR_INVALID_ARG;
+  if (n > kInsMaxN) return BOUTE_ERR_UNSUPPORTED;
+  if ((long long)B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;
+  if (int r = device_ok()) return r;
+  if (N == 0) return BOUTE_OK;
+  return launch_nehvi2(mean, cvar, shift, B, N, S, eps, eps_cand_stride, strips, counts, n, cons,
+                       acq, (cudaStream_t)stream);
+}
+
 int boute_gp_status(boute_gp *gp, void *stream) {
   BOUTE_TRACE();
   if (!gp) return BOUTE_ERR_INVALID_ARG;
@@ -284,6 +375,7 @@ void boute_gp_free(boute_gp *gp) {
   cudaFree(g.Kh); cudaFree(g.Kl); cudaFree(g.Aws); cudaFree(g.Wws); cudaFree(g.bop); cudaFree(g.xt);
   cudaFree(g.s2f); cudaFree(g.status); cudaFree(g.kpar); cudaFree(g.kcache); cudaFree(g.fbad);
   cudaFree(g.W64); cudaFree(g.a64); cudaFree(g.xs64); cudaFree(g.ls64); cudaFree(g.s2_64);
+  cudaFree(g.gws);
   delete gp;
 }
 
@@ -903,9 +995,10 @@ static int gp_set_n(Gp &g, int n) {
   if (n < 1 || n > g.ncap) return BOUTE_ERR_INVALID_ARG;
   if (n == g.n) return BOUTE_OK;
   const size_t BM = (size_t)g.B * g.m;
-  const PostPlan cap = make_post_plan(g.ncap);
+  const int S_in = g.plan.S_in;
+  const PostPlan cap = make_post_plan(g.ncap, S_in);
   g.n = n;
-  g.plan = make_post_plan(n);
+  g.plan = make_post_plan(n, S_in);
   const int want = kstar_cache_chunks(g.plan);
   g.kcache_chunks = want <= g.kcache_cap ? want : 0;  // else K* is rebuilt, not cached
   if (cudaMemset(g.bop, 0, BM * (size_t)cap.image_halves * sizeof(uint16_t)) != cudaSuccess ||

@@ -37,6 +37,10 @@ namespace boute {
 // CUDA cores while K* is built, in compensated fp32.)
 struct PostPlan {
   int n, npad, nxt, nchunk, nblk;
+  // blocks [0, nwblk) hold W = L^-1 (lower triangular); with in-sample draws
+  // (S_in > 0) the dense blocks of H^T (nhblk, summed squares) and of G^T
+  // (the rest, one output column per in-sample draw) follow
+  int nwblk, nhblk, S_in;
   int ncol[BOUTE_MAX_BLK], kc[BOUTE_MAX_BLK];
   long long off[BOUTE_MAX_BLK];  // half offset of block q's first chunk image
   long long image_halves;        // per (problem, objective)
@@ -79,7 +83,10 @@ inline __host__ __device__ int xt_param_offset(int DP) {
 // s2_x and d_tau; the power-of-two exponent e_W of W's operand scale; the
 // composite kernel's largest training-point preference weight (written by the
 // fit, in chunk 0 only).
-enum { kParS2 = 0, kParS2c = 1, kParS2x = 2, kParDtau = 3, kParEW = 4, kParWmax = 5 };
+// With in-sample draws, chunk 0 also holds the exponents of H's and G's
+// operand scales (written by the in-sample preparation).
+enum { kParS2 = 0, kParS2c = 1, kParS2x = 2, kParDtau = 3, kParEW = 4, kParWmax = 5, kParEH = 6,
+       kParEG = 7 };
 
 // Operand scales. The contraction runs on fp16 hi/lo parts, whose normal
 // range is [2^-14, 65504]: K* is scaled by 2^e_r so that its bound lies in
@@ -95,19 +102,29 @@ inline __host__ __device__ int w_scale_exp(double noise, double s2) {
   return 13 - ilogb(1.0 / sqrt(v));
 }
 
-inline PostPlan make_post_plan(int n) {
+// S_in > 0: the in-sample draws' blocks after W's (a noisy acquisition's
+// posterior, Sec. 5.2): H^T (n rows) and G^T (S_in rows), dense, every chunk.
+inline PostPlan make_post_plan(int n, int S_in = 0) {
   PostPlan p{};
   p.n = n;
   p.npad = round_up(n, BOUTE_KCHUNK);
   p.nxt = round_up(n, BOUTE_ACHUNK) / BOUTE_KCHUNK;
   p.nchunk = p.nxt / 2;
-  p.nblk = (n + BOUTE_BLKCOLS - 1) / BOUTE_BLKCOLS;
+  p.nwblk = (n + BOUTE_BLKCOLS - 1) / BOUTE_BLKCOLS;
+  p.nhblk = S_in > 0 ? p.nwblk : 0;
+  p.S_in = S_in > 0 ? S_in : 0;
+  p.nblk = p.nwblk + p.nhblk + (p.S_in + BOUTE_BLKCOLS - 1) / BOUTE_BLKCOLS;
   long long off = 0;
   for (int q = 0; q < p.nblk; ++q) {
-    const int c0 = BOUTE_BLKCOLS * q;
-    const int w = n - c0 < BOUTE_BLKCOLS ? n - c0 : BOUTE_BLKCOLS;
+    const bool wq = q < p.nwblk;
+    // rows of this block: W and H^T have n, G^T has S_in
+    const int c0 = BOUTE_BLKCOLS * (wq ? q : q < p.nwblk + p.nhblk ? q - p.nwblk
+                                                                      : q - p.nwblk - p.nhblk);
+    const int rows = q < p.nwblk + p.nhblk ? n : p.S_in;
+    const int w = rows - c0 < BOUTE_BLKCOLS ? rows - c0 : BOUTE_BLKCOLS;
     p.ncol[q] = round_up(w, 16);
-    p.kc[q] = (c0 + w + BOUTE_ACHUNK - 1) / BOUTE_ACHUNK;  // rows < c0 + w need columns < c0 + w
+    // W's rows < c0 + w need columns < c0 + w; the dense blocks need them all
+    p.kc[q] = wq ? (c0 + w + BOUTE_ACHUNK - 1) / BOUTE_ACHUNK : p.nchunk;
     p.off[q] = off;
     off += (long long)p.kc[q] * 2 * p.ncol[q] * BOUTE_ACHUNK;
   }

@@ -236,7 +236,7 @@ __device__ __forceinline__ bool pack_pair(const float *wrow, int g, int k, const
 __device__ __forceinline__ bool pack_elems(const float *W, int ld, const PostPlan &plan,
                                            float scale, uint16_t *img, long long first,
                                            long long stride) {
-  const int nblk = plan.nblk;
+  const int nblk = plan.nwblk;
   const long long rows = (long long)BOUTE_BLKCOLS * (nblk - 1) + plan.ncol[nblk - 1];
   const int kmax = BOUTE_ACHUNK * plan.kc[nblk - 1];  // pairs per row: kmax / 2
   const long long total = rows * (kmax / 2);
@@ -282,7 +282,7 @@ template <bool SMEM>
 __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     const float *Kh_all, const float *Kl_all, const double *Ys, int standardize, int n, int m,
     float *Aws, float *Wws, float *xt, int DP, int npad, PostPlan plan, uint16_t *bop,
-    int kl_smem, int early_trigger, int comp, int *status, const int *fbad) {
+    int kl_smem, int early_trigger, int comp, int *status, const int *fbad, float *Wkeep) {
   extern __shared__ __align__(16) float sm[];
   __shared__ int bad;
   __shared__ uint64_t lbar, lbar_lo;  // K hi; K lo (needed only by the residual)
@@ -407,7 +407,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   const float *xpar = xt + (size_t)bt * plan.nxt * xt_chunk_floats(DP) + xt_param_offset(DP) +
                       2 * DP;
   const float wscale = exp2i((int)xpar[kParEW]);
-  const int gmax = BOUTE_BLKCOLS * (plan.nblk - 1) + plan.ncol[plan.nblk - 1];
+  const int gmax = BOUTE_BLKCOLS * (plan.nwblk - 1) + plan.ncol[plan.nwblk - 1];
   auto pack_rows = [&](int g_lo, int g_hi, int w0, int nws) {
     uint16_t *img = bop + (size_t)bt * plan.image_halves;
     for (int g = g_lo + w0; g < g_hi && g < gmax; g += nws) {
@@ -854,6 +854,11 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   // global variant leaves W in the workspace for pack_kernel), alpha into the
   // side input
   if (SMEM) pack_rows(NP - 32, NP, warp, nw);  // the last block row (the others: above)
+  if (SMEM && Wkeep) {  // W for the in-sample preparation (its lower triangle)
+    float *dst = Wkeep + (size_t)bt * NP * ld;
+    for (int i = warp; i < n; i += nw)
+      for (int k = lane; k <= i; k += 32) dst[(size_t)i * ld + k] = W[(size_t)i * ld + k];
+  }
   const int cf = xt_chunk_floats(DP);
   float *xa = xt + (size_t)bt * plan.nxt * cf + xt_alpha_offset(DP);
   for (int k = tid; k < BOUTE_KCHUNK * plan.nxt; k += nthr) {
@@ -1196,14 +1201,14 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
       launch_pdl(fit32_kernel<true>, dim3(BM), dim3(fit_threads<true>()), smem, s, gp->Kh,
                  gp->Kl, Ys, standardize, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan,
                  gp->bop, fit_kl_in_smem(n) ? 1 : 0, fit_early, gp->kern, gp->status,
-                 (const int *)nullptr);
+                 (const int *)nullptr, gp->plan.S_in > 0 ? gp->Wws : nullptr);
       count_launch(2);
     } else {  // one block per problem-objective on the global workspace
       launch_pdl(fit32_kernel<false>, dim3(BM), dim3(fit_threads<false>()),
                  6 * npad * sizeof(float), s, gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws,
                  gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop, 0, 0, gp->kern, gp->status,
-                 (const int *)nullptr);
-      const long long tot = (long long)gp->plan.nblk * BOUTE_BLKCOLS * gp->plan.nchunk * 32;
+                 (const int *)nullptr, (float *)nullptr);
+      const long long tot = (long long)gp->plan.nwblk * BOUTE_BLKCOLS * gp->plan.nchunk * 32;
       pack_kernel<<<dim3((unsigned)std::min<long long>((tot + 255) / 256, 4096), BM), 256, 0,
                     s>>>(gp->Wws, gp->plan, gp->bop, gp->xt, gp->DP, gp->status);
       count_launch(3);
@@ -1241,8 +1246,8 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
     launch_pdl(fit32_kernel<false>, dim3(BM), dim3(fit_threads<false>()),
                6 * npad * sizeof(float), s, gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws,
                gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop, 0, 0, gp->kern, gp->status,
-               (const int *)gp->fbad);
-    const long long tot = (long long)gp->plan.nblk * BOUTE_BLKCOLS * gp->plan.nchunk * 32;
+               (const int *)gp->fbad, (float *)nullptr);
+    const long long tot = (long long)gp->plan.nwblk * BOUTE_BLKCOLS * gp->plan.nchunk * 32;
     pack_kernel<<<dim3((unsigned)std::min<long long>((tot + 255) / 256, 4096), BM), 256, 0, s>>>(
         gp->Wws, gp->plan, gp->bop, gp->xt, gp->DP, gp->status);
     count_launch(3);

@@ -37,6 +37,9 @@ struct Gp {
   // problem-objective [s2_c, s2_x, beta, s_0 .. s_{d-1}] (B*m x (3 + d))
   int kern, dtau;
   double *kpar;
+  // in-sample draws of the noisy acquisition (plan.S_in > 0, n <= kInsMaxN):
+  // G^T = (H Z)^T, S_in x n per problem-objective, before it is packed
+  float *gws;
 };
 
 // An NVTX range over one call of the C-ABI (visible in a profiler's timeline;
@@ -93,6 +96,24 @@ int launch_fit64(Gp *gp, const double *X, const double *Ys, const double *ls, co
 int launch_posterior64(const Gp *gp, const float *Xc, long long N, double *mean, double *var,
                        cudaStream_t s);
 constexpr int kFp64MaxN = 128;
+// Noisy acquisition (Sec. 5.2): the in-sample preparation after a fit (the
+// in-sample draws Yin, and H, G into the operand images; n <= kInsMaxN), the
+// fronts of the draws and the acquisition over them (two objectives).
+constexpr int kInsMaxN = 128, kInsMaxS = 1024;
+constexpr double kInsJitter = 1e-8;  // times the outputscale
+int launch_insample(Gp *gp, const double *Ys, const double *s2, const double *noise,
+                    const float *z, float *Yin, cudaStream_t s);
+size_t insample_smem_bytes(int n);
+int launch_insample_fronts(const float *Yin, int B, int n, int S, const double *ref,
+                           const double *cons, float *strips, int *counts, cudaStream_t s);
+int launch_nehvi2(const float *mean, const float *cvar, const float *shift, int B, long long N,
+                  int S, const float *eps, long long eps_stride, const float *strips,
+                  const int *counts, int n, const double *cons, float *acq, cudaStream_t s);
+// The posterior with the in-sample blocks: mean, the conditional variance
+// (cvar) and the shifts (B x m x S_in x N); shift null: the plain posterior
+// (W's blocks only) on a handle with in-sample draws.
+int launch_posterior_joint(const Gp *gp, const float *Xc, long long N, float *mean, float *cvar,
+                           float *shift, cudaStream_t s, const float *kst = nullptr);
 // the library's device check (an sm_103a device is current)
 int device_ok();
 // codes: outcome transforms before standardising (objective_code)

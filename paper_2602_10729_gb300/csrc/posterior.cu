@@ -68,6 +68,9 @@ struct PostArgs {
   const float *Xc;
   const float *kst;  // precomputed K* (PRE variant), else unused
   float *mean, *var;
+  // in-sample draws (plan.S_in > 0): the shifts l^T z_s, B x m x S_in x N;
+  // var then receives the conditional variance
+  float *shift;
   const uint16_t *bop;
   const float *xt, *s2f;
   int *status;
@@ -674,7 +677,23 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       const int b = tile / a.tiles_per_problem;
       const long long row =
           (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M + 32 * eq + lane;
-      float ss = 0.f;
+      const bool live = row < a.N;
+      const float *par = a.xt + (size_t)(b * m + t) * pl.nxt * cf + xt_param_offset(DP) + 2 * DP;
+      float prior = a.s2f[b * m + t], ws = 0.f;
+      if (a.kern && live) {  // composite kernel: k(x, x) = s2 + s2_x + s2_c w(x)^2
+        const float *c0 = a.xt + (size_t)(b * m + t) * pl.nxt * cf;
+        const float *bp = chunk_pref(c0, DP), *xrow = a.Xc + ((size_t)b * a.N + row) * d;
+        float e = 0.f;
+        for (int k = 0; k < d; ++k) e = fmaf(bp[k], xrow[k], e);
+        ws = expf(e);
+        prior = fmaf(par[kParS2c] * ws, ws, prior);
+      }
+      // the row's K* scale 2^e_r; the in-sample shifts (G blocks) leave with
+      // 2^-(e_r + e_G) applied
+      const int er = row_exp(a.kern, par, ws);
+      const float gscale = pl.S_in > 0 ? exp2i(-(er + (int)par[kParEG])) : 0.f;
+      float* shrow = pl.S_in > 0 ? a.shift + (size_t)(b * m + t) * pl.S_in * a.N + row : nullptr;
+      float ss = 0.f, ssh = 0.f;  // W's and H^T's sums of squares
       for (int g = 0; g < grp.n && !*abort; ++g) {
         const int q0 = Groups::first(g), q1 = Groups::last(pl, g);
         for (int qb = q0; qb <= q1; ++qb) {
@@ -683,11 +702,26 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
           if (!wait_or_abort(&acc_full[sl], (P / kSlots) & 1, abort)) break;
           tc_fence_after();
           const uint32_t ta = tmem + (uint32_t)(sl * BOUTE_BLKCOLS) + lanes;
-          for (int cc = 0; cc < pl.ncol[qb]; cc += 16) {
-            float v[16];
-            tmem_ld16(ta + cc, v);
+          if (qb < pl.nwblk + pl.nhblk) {
+            float sq = 0.f;
+            for (int cc = 0; cc < pl.ncol[qb]; cc += 16) {
+              float v[16];
+              tmem_ld16(ta + cc, v);
 #pragma unroll
-            for (int e = 0; e < 16; ++e) ss = fmaf(v[e], v[e], ss);  // zero beyond n
+              for (int e = 0; e < 16; ++e) sq = fmaf(v[e], v[e], sq);  // zero beyond n
+            }
+            if (qb < pl.nwblk) ss += sq;
+            else ssh += sq;
+          } else {  // G block: the shifts of draws s0 .. s0 + ncol
+            const int s0 = BOUTE_BLKCOLS * (qb - pl.nwblk - pl.nhblk);
+            for (int cc = 0; cc < pl.ncol[qb]; cc += 16) {
+              float v[16];
+              tmem_ld16(ta + cc, v);
+              if (live)
+#pragma unroll
+                for (int e = 0; e < 16; ++e)
+                  if (s0 + cc + e < pl.S_in) shrow[(size_t)(s0 + cc + e) * a.N] = v[e] * gscale;
+            }
           }
           tc_fence_before();
           __syncwarp();
@@ -696,20 +730,10 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
         blkseq += (uint32_t)(q1 - q0 + 1);
       }
       if (*abort) break;
-      if (row < a.N) {
-        const float *par = a.xt + (size_t)(b * m + t) * pl.nxt * cf + xt_param_offset(DP) + 2 * DP;
-        float prior = a.s2f[b * m + t], ws = 0.f;
-        if (a.kern) {  // composite kernel: k(x, x) = s2 + s2_x + s2_c w(x)^2
-          const float *c0 = a.xt + (size_t)(b * m + t) * pl.nxt * cf;
-          const float *bp = chunk_pref(c0, DP), *xrow = a.Xc + ((size_t)b * a.N + row) * d;
-          float e = 0.f;
-          for (int k = 0; k < d; ++k) e = fmaf(bp[k], xrow[k], e);
-          ws = expf(e);
-          prior = fmaf(par[kParS2c] * ws, ws, prior);
-        }
-        // V carries the scales 2^e_r (K*) and 2^e_W (W)
-        const int ex = row_exp(a.kern, par, ws) + (int)par[kParEW];
-        const float vv = prior - ldexpf(ss, -2 * ex);
+      if (live) {
+        // V carries the scales 2^e_r (K*) and 2^e_W (W); H^T k* 2^e_r and 2^e_H
+        float vv = prior - ldexpf(ss, -2 * (er + (int)par[kParEW]));
+        if (pl.nhblk > 0) vv -= ldexpf(ssh, -2 * (er + (int)par[kParEH]));
         a.var[((size_t)b * m + t) * a.N + row] = vv > 0.f ? vv : 0.f;
       }
     }
@@ -885,7 +909,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
 
 template <int DP>
 int launch_dp(const Gp *gp, const float *Xc, const float *kst, long long N, float *mean,
-              float *var, cudaStream_t s) {
+              float *var, cudaStream_t s, float *shift) {
   PostArgs a;
   a.Xc = Xc;
   a.kst = kst;
@@ -901,13 +925,23 @@ int launch_dp(const Gp *gp, const float *Xc, const float *kst, long long N, floa
   a.d = gp->d;
   a.n = gp->n;
   a.plan = gp->plan;
+  a.shift = shift;
+  if (!shift && a.plan.S_in > 0) {  // the plain posterior: W's blocks only
+    a.plan.nblk = a.plan.nwblk;
+    a.plan.nhblk = 0;
+    a.plan.S_in = 0;
+  }
   a.kern = gp->kern;
   // the chunk cache (not with K* precomputed, where no chunk is built)
   a.kcache = gp->kcache;
-  a.ncache = (!kst && gp->kcache && gp->kcache_sms >= num_sms()) ? gp->kcache_chunks : 0;
+  const int want = kstar_cache_chunks(a.plan);
+  a.ncache =
+      (!kst && gp->kcache && gp->kcache_sms >= num_sms() && want <= gp->kcache_cap) ? want : 0;
   a.tiles_per_problem = (int)((N + BOUTE_TILE_M - 1) / BOUTE_TILE_M);
   a.tiles_total = a.tiles_per_problem * gp->B;
-  a.b_bytes = (uint32_t)(2 * gp->plan.ncol[0] * 128);  // block 0 is the widest
+  int wmax = 0;  // the widest block sizes a B stage
+  for (int q = 0; q < a.plan.nblk; ++q) wmax = std::max(wmax, a.plan.ncol[q]);
+  a.b_bytes = (uint32_t)(2 * wmax * 128);
   a.x_bytes = (uint32_t)round_up(xt_chunk_floats(DP) * 4, 16);
   const size_t fixed = 1024 + 512;  // alignment slack, barriers, TMEM address, flag
   const size_t budget = 227 * 1024 - fixed;
@@ -1039,17 +1073,22 @@ int launch_kstar_dp(const Gp *gp, const float *Xc, long long N, float *kst, cuda
 
 }  // namespace
 
-int launch_posterior(const Gp *gp, const float *Xc, long long N, float *mean, float *var,
-                     cudaStream_t s, const float *kst) {
+int launch_posterior_joint(const Gp *gp, const float *Xc, long long N, float *mean, float *cvar,
+                           float *shift, cudaStream_t s, const float *kst) {
   if (N <= 0) return BOUTE_OK;
   switch (gp->DP) {
-    case 8: return launch_dp<8>(gp, Xc, kst, N, mean, var, s);
-    case 12: return launch_dp<12>(gp, Xc, kst, N, mean, var, s);
-    case 16: return launch_dp<16>(gp, Xc, kst, N, mean, var, s);
-    case 24: return launch_dp<24>(gp, Xc, kst, N, mean, var, s);
-    case 32: return launch_dp<32>(gp, Xc, kst, N, mean, var, s);
+    case 8: return launch_dp<8>(gp, Xc, kst, N, mean, cvar, s, shift);
+    case 12: return launch_dp<12>(gp, Xc, kst, N, mean, cvar, s, shift);
+    case 16: return launch_dp<16>(gp, Xc, kst, N, mean, cvar, s, shift);
+    case 24: return launch_dp<24>(gp, Xc, kst, N, mean, cvar, s, shift);
+    case 32: return launch_dp<32>(gp, Xc, kst, N, mean, cvar, s, shift);
   }
   return BOUTE_ERR_UNSUPPORTED;
+}
+
+int launch_posterior(const Gp *gp, const float *Xc, long long N, float *mean, float *var,
+                     cudaStream_t s, const float *kst) {
+  return launch_posterior_joint(gp, Xc, N, mean, var, nullptr, s, kst);
 }
 
 int kstar_cache_chunks(const PostPlan &plan) {

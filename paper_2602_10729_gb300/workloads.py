@@ -47,7 +47,7 @@ import numpy as np
 CHUNK = 8192  # candidates per independently seeded block
 
 # stream ids within one seed
-_S_TRAIN_X, _S_NOISE, _S_CAND, _S_EPS, _S_SHIFT, _S_PREF = 0, 1, 2, 3, 4, 5
+_S_TRAIN_X, _S_NOISE, _S_CAND, _S_EPS, _S_SHIFT, _S_PREF, _S_INSAMPLE = 0, 1, 2, 3, 4, 5, 6
 MAX_COUNT = 4  # deployment features of composite variants: GPU counts 0 .. MAX_COUNT
 
 
@@ -228,6 +228,14 @@ def candidates(w: Workload, b: int, start: int = 0, count: int | None = None,
     return _fill(out, start, count,
                  lambda j: _counts(_rng(w.seeds[b], _S_CAND, j).random((CHUNK, w.d)),
                                    w).astype(np.float32), threads)
+
+
+def insample_normals(w: Workload, b: int, S: int | None = None) -> np.ndarray:
+    """Standard-normal base samples of the in-sample draws of problem b (the
+    noisy acquisition), fp32, layout (m, S, n)."""
+    S = w.S if S is None else S
+    return _rng(w.seeds[b], _S_INSAMPLE, w.eps_seed).standard_normal(
+        (w.m, S, w.n)).astype(np.float32)
 
 
 def base_normals(w: Workload, b: int, start: int = 0, count: int | None = None,
