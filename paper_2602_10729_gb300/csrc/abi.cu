@@ -279,9 +279,11 @@ int boute_gp_set_insample(boute_gp *gp, int S) {
   // new operand images (W's blocks then H^T's and G^T's), zero: fit again
   uint16_t *bop = nullptr;
   if (dalloc(&bop, BM * (size_t)cap.image_halves) != BOUTE_OK) return BOUTE_ERR_OOM;
-  float *gws = nullptr;
-  if (S > 0 && dalloc(&gws, BM * (size_t)S * g.ncap) != BOUTE_OK) {
+  float *gws = nullptr, *iws = nullptr;
+  if (S > 0 && (dalloc(&gws, BM * (size_t)S * g.ncap) != BOUTE_OK ||
+                dalloc(&iws, BM * insample_ws_floats(g.ncap)) != BOUTE_OK)) {
     cudaFree(bop);
+    cudaFree(gws);
     return BOUTE_ERR_OOM;
   }
   const int want = kstar_cache_chunks(cap);
@@ -290,12 +292,14 @@ int boute_gp_set_insample(boute_gp *gp, int S) {
       dalloc(&kc, (size_t)g.kcache_sms * want * kKstarChunkHalves) != BOUTE_OK) {
     cudaFree(bop);
     cudaFree(gws);
+    cudaFree(iws);
     return BOUTE_ERR_OOM;
   }
   if (cudaMemset(bop, 0, BM * (size_t)cap.image_halves * sizeof(uint16_t)) != cudaSuccess) {
     cudaGetLastError();
     cudaFree(bop);
     cudaFree(gws);
+    cudaFree(iws);
     cudaFree(kc);
     return BOUTE_ERR_CUDA;
   }
@@ -303,6 +307,8 @@ int boute_gp_set_insample(boute_gp *gp, int S) {
   g.bop = bop;
   cudaFree(g.gws);
   g.gws = gws;
+  cudaFree(g.iws);
+  g.iws = iws;
   if (kc) {
     cudaFree(g.kcache);
     g.kcache = kc;
@@ -376,6 +382,7 @@ void boute_gp_free(boute_gp *gp) {
   cudaFree(g.s2f); cudaFree(g.status); cudaFree(g.kpar); cudaFree(g.kcache); cudaFree(g.fbad);
   cudaFree(g.W64); cudaFree(g.a64); cudaFree(g.xs64); cudaFree(g.ls64); cudaFree(g.s2_64);
   cudaFree(g.gws);
+  cudaFree(g.iws);
   delete gp;
 }
 

@@ -38,8 +38,9 @@ struct Gp {
   int kern, dtau;
   double *kpar;
   // in-sample draws of the noisy acquisition (plan.S_in > 0, n <= kInsMaxN):
-  // G^T = (H Z)^T, S_in x n per problem-objective, before it is packed
-  float *gws;
+  // G^T = (H Z)^T, S_in x n per problem-objective, before it is packed, and
+  // the preparation's workspace (F, H^T, mu_n, max |G|: insample_ws_floats)
+  float *gws, *iws;
 };
 
 // An NVTX range over one call of the C-ABI (visible in a profiler's timeline;
@@ -104,6 +105,7 @@ constexpr double kInsJitter = 1e-8;  // times the outputscale
 int launch_insample(Gp *gp, const double *Ys, const double *s2, const double *noise,
                     const float *z, float *Yin, cudaStream_t s);
 size_t insample_smem_bytes(int n);
+size_t insample_ws_floats(int n);  // per problem-objective
 int launch_insample_fronts(const float *Yin, int B, int n, int S, const double *ref,
                            const double *cons, float *strips, int *counts, cudaStream_t s);
 int launch_nehvi2(const float *mean, const float *cvar, const float *shift, int B, long long N,
