@@ -320,11 +320,16 @@ def main():
     ap.add_argument("--no-serial-stages", action="store_true",
                     help="skip the serialised per-stage breakdown")
     ap.add_argument("--e2e-steps", type=int, default=0, help="0: same as --steps (max 200)")
+    ap.add_argument("--candidates", type=int, default=0,
+                    help="candidates per problem (0: the workload's N); a smaller N keeps "
+                         "profiler captures small")
     ap.add_argument("--constraints", default="",
                     help="comma-separated thresholds on the standardised, minimised objectives "
                          "(constrained acquisition; 'inf' leaves an objective unconstrained)")
     args = ap.parse_args()
     w = wl.by_name(args.workload)
+    if args.candidates:
+        w = wl.scaled(w, N=args.candidates)
     args.cons = [float(c) for c in args.constraints.split(",")] if args.constraints else None
     if args.cons is not None and len(args.cons) != w.m:
         ap.error(f"--constraints needs {w.m} values")
