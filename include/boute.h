@@ -43,7 +43,7 @@ typedef enum {
   BOUTE_ERR_TIMEOUT = 6      /* a device-side wait gave up (nothing hung) */
 } boute_status;
 
-typedef enum { BOUTE_ACQ_EHVI2D = 0, BOUTE_ACQ_MC_HVI = 1 } boute_acq_mode;
+typedef enum { BOUTE_ACQ_EHVI2D = 0, BOUTE_ACQ_MC_HVI = 1, BOUTE_ACQ_NEHVI = 2 } boute_acq_mode;
 
 /* Human-readable name of a status code (static string). */
 const char *boute_status_string(int status);
@@ -376,7 +376,8 @@ int boute_select_topk_noalloc(const float *acq, int B, long long N, int k, long 
  * and return the fit status or the first device error.
  *   X: B x n x d fp64; Y: B x n x m fp64 raw outcomes (standardised inside);
  *   lengthscale: B x m x d; outputscale, noise: B x m; ref: B x m (fp64);
- *   Xc: B x N x d fp32; eps: B x N x m x S fp32 (mode MC_HVI; NULL otherwise);
+ *   Xc: B x N x d fp32; eps: B x N x m x S fp32 (modes MC_HVI and NEHVI; NULL
+ *   otherwise);
  *   idx: B x k int64, val: B x k fp32.
  * boute_engine_step_async: as boute_engine_step without the final
  * synchronisation (device errors surface at the next synchronising call).
@@ -391,7 +392,17 @@ int boute_select_topk_noalloc(const float *acq, int B, long long N, int k, long 
  * fit status or the first device error.
  * On a non-default stream the step is captured once per argument set (device
  * or host buffers) into a CUDA graph and replayed afterwards; a first call
- * with new pointers therefore must not itself run inside a stream capture. */
+ * with new pointers therefore must not itself run inside a stream capture.
+ * Mode BOUTE_ACQ_NEHVI (m = 2, n <= 128, 1 <= S <= 1024): the noisy
+ * acquisition of Sec. 5.2 (see boute_gp_set_insample): after the fit the
+ * in-sample draws, then the joint posterior, each draw's front and the
+ * draws' hypervolume improvements; eps as for MC_HVI. The engine's S x n
+ * in-sample normals per objective come from the generator of
+ * boute_base_normals: for seed s (0 at creation, then that of
+ * boute_engine_set_normals) they are boute_base_normals(s ^
+ * 0x6a09e667f3bcc909, B, m*S, 1, n) read as B x m x S x n. In stage timing
+ * the in-sample preparation counts in the fit stage (live) or the front
+ * stage (serial), the draws' fronts in the acquisition stage. */
 typedef struct boute_engine boute_engine;
 int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S, int k,
                         boute_engine **out);

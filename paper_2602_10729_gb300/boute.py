@@ -16,7 +16,7 @@ from . import build as _build
 
 BOUTE_OK, BOUTE_ERR_INVALID_ARG, BOUTE_ERR_NOT_PD, BOUTE_ERR_CUDA = 0, 1, 2, 3
 BOUTE_ERR_OOM, BOUTE_ERR_UNSUPPORTED, BOUTE_ERR_TIMEOUT = 4, 5, 6
-BOUTE_ACQ_EHVI2D, BOUTE_ACQ_MC_HVI = 0, 1
+BOUTE_ACQ_EHVI2D, BOUTE_ACQ_MC_HVI, BOUTE_ACQ_NEHVI = 0, 1, 2
 BOUTE_TF_IDENTITY, BOUTE_TF_LOG, BOUTE_TF_LOGIT, BOUTE_TF_NEGATE = 0, 1, 2, 4
 
 #: exported symbols declared in include/boute.h

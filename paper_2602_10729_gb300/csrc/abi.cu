@@ -134,7 +134,24 @@ struct boute_engine {
   // the engine's own base normals (boute_engine_set_normals), used by steps
   // whose eps is null; null until set
   float *gen_eps;
+  // noisy acquisition (BOUTE_ACQ_NEHVI): in-sample normals (B x m x S x n,
+  // drawn from zseed), in-sample draws, the posterior's shifts (B x m x S x N),
+  // and the draws' fronts as strips (B x S x (n + 1) x 4) with their counts
+  float *zin, *Yin, *shift, *strips;
+  int *counts;
+  unsigned long long zseed;
 };
+
+namespace boute {
+// Key of the in-sample normals of seed s: s ^ kInsampleKey (the first 64
+// bits of the fractional part of sqrt(2)), so that they are drawn
+// independently of the candidates' normals of the same seed.
+constexpr unsigned long long kInsampleKey = 0x6a09e667f3bcc909ull;
+static int draw_insample_normals(boute_engine *e, cudaStream_t s) {
+  return launch_base_normals(e->zseed ^ kInsampleKey, e->B, (long long)e->m * e->S, 1, e->n,
+                             e->zin, s);
+}
+}  // namespace boute
 
 // Stage order of one step as timed (with timing on, the front stage runs
 // after the fit on the step's stream, so the stage times add up).
@@ -536,7 +553,8 @@ void boute_engine_free(boute_engine *e) {
   void *ptrs[] = {e->X, e->Y, e->Ys, e->ls, e->s2, e->noise, e->ref, e->front, e->mask, e->P,
                   e->K, e->lower, e->upper, e->Xc, e->eps, e->mean, e->var, e->acq, e->val,
                   e->idx, e->scratch, e->sel, e->kst, e->X1, e->Y1, e->ls1, e->s21,
-                  e->noise1, e->ref1, e->Xc1, e->eps1, e->cons, e->Yt, e->gen_eps};
+                  e->noise1, e->ref1, e->Xc1, e->eps1, e->cons, e->Yt, e->gen_eps,
+                  e->zin,    e->Yin,  e->shift, e->strips, e->counts};
   for (void *p : ptrs) cudaFree(p);
   delete e;
 }
@@ -562,7 +580,10 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
   if ((long long)B * N >= (1ll << 31)) return BOUTE_ERR_INVALID_ARG;
   if (mode == BOUTE_ACQ_EHVI2D && m != 2) return BOUTE_ERR_INVALID_ARG;
   if (mode == BOUTE_ACQ_MC_HVI && (m < 2 || m > 3 || S < 1)) return BOUTE_ERR_INVALID_ARG;
-  if (mode != BOUTE_ACQ_EHVI2D && mode != BOUTE_ACQ_MC_HVI) return BOUTE_ERR_INVALID_ARG;
+  if (mode == BOUTE_ACQ_NEHVI && (m != 2 || S < 1 || S > kInsMaxS)) return BOUTE_ERR_INVALID_ARG;
+  if (mode != BOUTE_ACQ_EHVI2D && mode != BOUTE_ACQ_MC_HVI && mode != BOUTE_ACQ_NEHVI)
+    return BOUTE_ERR_INVALID_ARG;
+  if (mode == BOUTE_ACQ_NEHVI && n > kInsMaxN) return BOUTE_ERR_UNSUPPORTED;
   if (int r = device_ok()) return r;
   boute_engine *e = new (std::nothrow) boute_engine();
   if (!e) return BOUTE_ERR_OOM;
@@ -585,7 +606,17 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
   r |= dalloc(&e->lower, (size_t)B * cap * m);
   r |= dalloc(&e->upper, (size_t)B * cap * m);
   r |= dalloc(&e->Xc, BN * d);
-  if (mode == BOUTE_ACQ_MC_HVI) r |= dalloc(&e->eps, BN * m * S);
+  if (mode != BOUTE_ACQ_EHVI2D) r |= dalloc(&e->eps, BN * m * S);
+  if (mode == BOUTE_ACQ_NEHVI) {
+    const size_t zc = (size_t)B * m * S * n;
+    r |= dalloc(&e->zin, zc);
+    r |= dalloc(&e->Yin, zc);
+    r |= dalloc(&e->shift, BN * m * S);
+    r |= dalloc(&e->strips, (size_t)B * S * (n + 1) * 4);
+    r |= dalloc(&e->counts, (size_t)B * S);
+    if (r == BOUTE_OK) r = boute_gp_set_insample(e->gp, S);
+    if (r == BOUTE_OK) r = draw_insample_normals(e, nullptr);  // seed 0 until set_normals
+  }
   r |= dalloc(&e->mean, BN * m);
   r |= dalloc(&e->var, BN * m);
   r |= dalloc(&e->acq, BN);
@@ -645,7 +676,7 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
   const unsigned long long l0 = launch_count();
   int r;
   const int B = e->B, n = e->n, m = e->m;
-  const int mc = e->mode == BOUTE_ACQ_MC_HVI;
+  const int mc = e->mode != BOUTE_ACQ_EHVI2D, nehvi = e->mode == BOUTE_ACQ_NEHVI;
   // stage boundaries: event-record nodes when captured, plain records when eager
   cudaStreamCaptureStatus run_cap = cudaStreamCaptureStatusNone;
   if (e->timing && s && cudaStreamIsCapturing(s, &run_cap) != cudaSuccess)
@@ -704,11 +735,17 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
     if ((r = front(s))) return r;
     mark(ST_POSTERIOR);
   }
+  if (nehvi) {  // the in-sample draws need the front stage's standardised outcomes
+    if (!serial && cudaStreamWaitEvent(s, e->join, 0) != cudaSuccess) return last_launch_status();
+    if ((r = launch_insample(&e->gp->g, e->Ys, s2, noise, e->zin, e->Yin, s))) return r;
+  }
   if (host && cudaStreamWaitEvent(s, ev_xc, wait_flags) != cudaSuccess)
     return last_launch_status();
   if (kst && cudaStreamWaitEvent(s, e->join2, 0) != cudaSuccess) return last_launch_status();
   if (live) mark(ST_POSTERIOR);  // the posterior starts here (the front ran beside the fit)
-  if ((r = launch_posterior(&e->gp->g, Xc, e->N, e->mean, e->var, s, kst))) return r;
+  if ((r = nehvi ? launch_posterior_joint(&e->gp->g, Xc, e->N, e->mean, e->var, e->shift, s, kst)
+                 : launch_posterior(&e->gp->g, Xc, e->N, e->mean, e->var, s, kst)))
+    return r;
   if (live) mark(ST_ACQ);
   if (!serial && cudaStreamWaitEvent(s, e->join, 0) != cudaSuccess)  // join
     return last_launch_status();
@@ -725,6 +762,11 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
       return r;
   } else if (!mc) {
     if ((r = launch_ehvi(e->mean, e->var, B, e->N, e->front, e->P, n, ref, cons, e->acq, s)))
+      return r;
+  } else if (nehvi) {  // each draw's front, then the draws' improvements over them
+    if ((r = launch_insample_fronts(e->Yin, B, n, e->S, ref, cons, e->strips, e->counts, s)) ||
+        (r = launch_nehvi2(e->mean, e->var, e->shift, B, e->N, e->S, eps, 2ll * e->S, e->strips,
+                           e->counts, n, cons, e->acq, s)))
       return r;
   } else {
     if ((r = launch_mchvi(e->mean, e->var, B, e->N, m, e->lower, e->upper, e->K, 2 * n + 2, eps,
@@ -744,7 +786,7 @@ static int engine_args_ok(const boute_engine *e, const void *X, const void *Y, c
                           const void *s2, const void *noise, const void *ref, const void *Xc,
                           const void *eps, const void *idx, const void *val) {
   if (!e || !X || !Y || !ls || !s2 || !noise || !ref || !Xc || !idx || !val) return 0;
-  if (e->mode == BOUTE_ACQ_MC_HVI && !eps && !e->gen_eps) return 0;
+  if (e->mode != BOUTE_ACQ_EHVI2D && !eps && !e->gen_eps) return 0;
   return 1;
 }
 
@@ -867,7 +909,7 @@ static int engine_host_step(boute_engine *e, int set, const double *X, const dou
   cudaEventRecord(e->ev_small[set], c0);
   cudaMemcpyAsync(dXc, Xc, B * N * d * sizeof(float), cudaMemcpyHostToDevice, c0);
   cudaEventRecord(ev_xc, e->cpy[0]);
-  const size_t eps_n = e->mode == BOUTE_ACQ_MC_HVI && eps ? B * N * m * S : 0,
+  const size_t eps_n = e->mode != BOUTE_ACQ_EHVI2D && eps ? B * N * m * S : 0,
                half = eps_n / 2;
   for (int i = 0; eps && i < 2; ++i) {  // the normals in two halves, one per copy stream
     const size_t off = i ? half : 0, cnt = i ? eps_n - half : half;
@@ -912,7 +954,7 @@ int boute_engine_step_host_async(boute_engine *e, const double *X, const double 
     int r = dalloc(&e->X1, Bn * e->d) | dalloc(&e->Y1, Bn * e->m) |
             dalloc(&e->ls1, Bm * e->d) | dalloc(&e->s21, Bm) | dalloc(&e->noise1, Bm) |
             dalloc(&e->ref1, Bm) | dalloc(&e->Xc1, BN * e->d);
-    if (e->mode == BOUTE_ACQ_MC_HVI) r |= dalloc(&e->eps1, BN * e->m * e->S);
+    if (e->mode != BOUTE_ACQ_EHVI2D) r |= dalloc(&e->eps1, BN * e->m * e->S);
     if (r) return BOUTE_ERR_OOM;
   }
   const int set = e->host_set;
@@ -1025,6 +1067,10 @@ int boute_engine_set_n(boute_engine *e, int n) {
   if (int r = gp_set_n(e->gp->g, n)) return r;
   e->n = n;
   engine_drop_graphs(e);  // the graphs hold n and the plan in their arguments
+  if (e->mode == BOUTE_ACQ_NEHVI) {  // the in-sample normals in the layout of n
+    if (int r = draw_insample_normals(e, nullptr)) return r;
+    if (cudaDeviceSynchronize() != cudaSuccess) return last_launch_status();
+  }
   // the in-kernel selection's scratch grows as the boxes shrink (more
   // resident blocks): keep it when it is large enough, else take a new one
   e->fuse_sel = engine_fuses_selection(e);
@@ -1083,11 +1129,15 @@ int boute_base_normals(unsigned long long seed, int B, long long N, int m, int S
 
 int boute_engine_set_normals(boute_engine *e, unsigned long long seed) {
   BOUTE_TRACE();
-  if (!e || e->mode != BOUTE_ACQ_MC_HVI) return BOUTE_ERR_INVALID_ARG;
+  if (!e || e->mode == BOUTE_ACQ_EHVI2D) return BOUTE_ERR_INVALID_ARG;
   if (cudaDeviceSynchronize() != cudaSuccess) return last_launch_status();
   const size_t count = (size_t)e->B * e->N * e->m * e->S;
   if (!e->gen_eps && dalloc(&e->gen_eps, count) != BOUTE_OK) return BOUTE_ERR_OOM;
   int r = launch_base_normals(seed, e->B, e->N, e->m, e->S, e->gen_eps, nullptr);
+  if (!r && e->mode == BOUTE_ACQ_NEHVI) {
+    e->zseed = seed;
+    r = draw_insample_normals(e, nullptr);
+  }
   if (!r && cudaDeviceSynchronize() != cudaSuccess) r = last_launch_status();
   return r;
 }

@@ -80,13 +80,13 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
       !converged || d < 1 || m < 2 || N < 1 || n0 < 1 || cfg->max_evals < n0 ||
       cfg->patience < 1 || cfg->learn_iters < 0)
     return BOUTE_ERR_INVALID_ARG;
-  if (cfg->mode == BOUTE_ACQ_MC_HVI && cfg->S < 1) return BOUTE_ERR_INVALID_ARG;
+  if (cfg->mode != BOUTE_ACQ_EHVI2D && cfg->S < 1) return BOUTE_ERR_INVALID_ARG;
   if (kc && (d_tau < 0 || d_tau > d)) return BOUTE_ERR_INVALID_ARG;
   // the composite kernel (kc: m x (3 + dc) [s2_c, s2_x, beta, s...]) adds
   // (log s2_c, log s2_x, beta) to the learned parameters
   const int dc = d - d_tau, KC = 3 + dc;
   const int nmax = cfg->max_evals, P = d + (kc ? 5 : 2),
-            S = cfg->mode == BOUTE_ACQ_MC_HVI ? cfg->S : 0;
+            S = cfg->mode != BOUTE_ACQ_EHVI2D ? cfg->S : 0;
   *n_out = n0;
   *converged = 0;
   double *dX = nullptr, *dY = nullptr, *dYs = nullptr, *dls = nullptr, *ds2 = nullptr,

@@ -221,3 +221,97 @@ def test_insample_limits():
     assert ei.value.code == bt.BOUTE_ERR_UNSUPPORTED
     bt.boute_gp_set_insample(gp, 0)
     gp.free()
+
+
+INSAMPLE_KEY = 0x6a09e667f3bcc909  # the engine's in-sample normals: seed ^ this key
+
+
+def _engine_inputs(hp):
+    import torch
+    t = lambda a, dt: torch.as_tensor(np.ascontiguousarray(a), device="cuda", dtype=dt)
+    f64, f32 = torch.float64, torch.float32
+    return (t(hp.X, f64), t(hp.Y, f64), t(hp.ls, f64), t(hp.s2, f64), t(hp.noise, f64),
+            t(hp.ref, f64), t(hp.Xc, f32), t(hp.eps, f32))
+
+
+def _engine_step(e, w, inputs, how="device"):
+    import torch
+
+    from paper_2602_10729_gb300 import boute as bt
+    if how == "host":
+        hin = tuple(a.cpu().pin_memory() for a in inputs)
+        idx = torch.empty((w.B, w.k), dtype=torch.int64).pin_memory()
+        val = torch.empty((w.B, w.k), dtype=torch.float32).pin_memory()
+        bt.boute_engine_step_host(e, *hin, idx, val)
+        return idx.numpy().copy(), val.numpy().copy()
+    idx = torch.empty((w.B, w.k), dtype=torch.int64, device="cuda")
+    val = torch.empty((w.B, w.k), dtype=torch.float32, device="cuda")
+    if how == "legacy":
+        torch.cuda.synchronize()
+        bt.boute_engine_step(e, *inputs, idx, val, stream=0)
+    else:
+        bt.boute_engine_step(e, *inputs, idx, val)
+    return idx.cpu().numpy(), val.cpu().numpy()
+
+
+@pytest.mark.parametrize("case", [(1, 3000 + 77, 128, 128, 1, False, 7),
+                                  (4, 999, 64, 64, 2, True, 0)],
+                         ids=["medium-n128-S128", "batched-n64-S64-cons"])
+def test_engine_noisy_step_matches_oracle(case):
+    """The whole noisy step through the engine: graph replay, host inputs and
+    eager launches agree value for value, and the selection is the oracle's
+    (in-sample normals regenerated from the documented key)."""
+    import torch
+
+    from paper_2602_10729_gb300 import boute as bt
+    wi, N, n, S, B, constrained, seed = case
+    w = _workload(wi, N, n, S, B)
+    hp = host_problem(w)
+    cons = _cons(hp) if constrained else None
+    e = bt.Engine(B, n, w.d, w.m, N, bt.BOUTE_ACQ_NEHVI, S, w.k)
+    if seed:
+        bt.boute_engine_set_normals(e, seed)
+    if cons is not None:
+        bt.boute_engine_set_constraints(e, torch.as_tensor(cons, dtype=torch.float64))
+    inputs = _engine_inputs(hp)
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        ref_idx, ref_val = _engine_step(e, w, inputs)
+        for how in ("device", "host", "legacy"):
+            idx, val = _engine_step(e, w, inputs, how)
+            assert np.array_equal(idx, ref_idx), how
+            assert np.array_equal(val, ref_val), how
+    e.free()
+    z = oracle.base_normals(seed ^ INSAMPLE_KEY, B, w.m * S, 1, n).reshape(B, w.m, S, n)
+    for b in range(B):
+        fp = oracle_fit(hp, b)
+        dr = opl.noisy_draws(fp, hp.Xc[b], z[b])
+        cb = None if cons is None else cons[b]
+        o, sens = _sensitivity(fp, dr, hp.eps[b], cb, hp.s2[b])
+        tol = ACQ_REL * np.maximum(np.abs(o), ACQ_FLOOR * np.abs(o).max()) + 2 * sens
+        check_topk_consistent_tol(ref_idx[b], o, w.k, tol)
+        np.testing.assert_allclose(ref_val[b], o[ref_idx[b]], rtol=0, atol=float(tol.max()))
+
+
+def test_engine_noisy_set_n_matches_fresh_engine():
+    import torch
+
+    from paper_2602_10729_gb300 import boute as bt
+    base = _workload(1, 1024 + 3, 128, 64, 1)
+    e = bt.Engine(1, 128, base.d, 2, base.N, bt.BOUTE_ACQ_NEHVI, 64, base.k)
+    bt.boute_engine_set_normals(e, 5)
+    stream = torch.cuda.Stream()
+    for n in (128, 57, 100):
+        w = _workload(1, 1024 + 3, n, 64, 1)
+        hp = host_problem(w)
+        inputs = _engine_inputs(hp)
+        bt.boute_engine_set_n(e, n)
+        fresh = bt.Engine(1, n, w.d, 2, w.N, bt.BOUTE_ACQ_NEHVI, 64, w.k)
+        bt.boute_engine_set_normals(fresh, 5)
+        with torch.cuda.stream(stream):
+            ri, rv = _engine_step(fresh, w, inputs)
+            for how in ("device", "device", "legacy"):
+                idx, val = _engine_step(e, w, inputs, how)
+                assert np.array_equal(idx, ri) and np.array_equal(val, rv), (n, how)
+        fresh.free()
+    e.free()
