@@ -59,6 +59,10 @@ NUM_SMS = 152
 FMA_LANES_PER_SM = 128
 
 
+# The engine's in-sample normals of seed s are drawn under the key s ^ this.
+INSAMPLE_KEY = 0x6a09e667f3bcc909
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -80,7 +84,7 @@ def host_inputs(w: wl.Workload, threads: int = 16, count: int | None = None):
         X.append(x); Y.append(y); L.append(ls); S2.append(s2); NZ.append(nz)
     Xc = np.stack([wl.candidates(w, b, 0, count, threads) for b in range(w.B)])
     eps = (np.stack([wl.base_normals(w, b, 0, count, threads) for b in range(w.B)])
-           if w.mode == "mc" else None)
+           if w.mode in ("mc", "nehvi") else None)
     ref = np.tile(wl.ref_point(w), (w.B, 1))
     kc = np.stack([wl.kernel_params(w, b)[1] for b in range(w.B)]) if w.d_tau else None
     return dict(X=np.stack(X), Y=np.stack(Y), ls=np.stack(L), s2=np.stack(S2),
@@ -143,14 +147,20 @@ def tensor_peak(bf16_tflops: float) -> float:
 def contraction_flops(w: wl.Workload) -> float:
     """Algorithmic flops of the posterior: V = K* (L^-1)^T over the lower
     triangle (n(n+1)/2 multiply-adds per candidate and objective) and the mean
-    K* alpha (n multiply-adds)."""
-    return float(w.B) * w.N * w.m * (w.n * (w.n + 1) + 2 * w.n)
+    K* alpha (n multiply-adds); the noisy acquisition's joint posterior adds
+    the dense H^T k* (n^2) and G^T k* (n S) multiply-adds."""
+    per = w.n * (w.n + 1) + 2 * w.n
+    if w.mode == "nehvi":
+        per += 2 * w.n * w.n + 2 * w.n * w.S
+    return float(w.B) * w.N * w.m * per
 
 
 def pass_bytes(w: wl.Workload) -> float:
     """HBM bytes the scoring pass must move per step: each candidate's
     coordinates (4d), its base normals (4mS, Monte-Carlo) and its score (4)."""
-    per = 4 * w.d + (4 * w.m * w.S if w.mode == "mc" else 0) + 4
+    per = 4 * w.d + (4 * w.m * w.S if w.mode in ("mc", "nehvi") else 0) + 4
+    if w.mode == "nehvi":  # the shifts l^T z_s: written by the posterior, read back
+        per += 2 * 4 * w.m * w.S
     return float(w.B) * w.N * per
 
 
@@ -163,10 +173,11 @@ def stage_roofline(w: wl.Workload, stage: str, ms: float, hbm, tens, sm_mhz):
         return dict(bound="tensor", achieved=flops / (ms * 1e-3) / 1e12, peak=tens,
                     unit="TFLOP/s", per_launch=flops, kernel="posterior_kernel")
     if stage == "acquisition":
-        per = (m * S * 4 if w.mode == "mc" else 0) + 2 * m * 4 + 4
+        per = (m * S * 4 * (2 if w.mode == "nehvi" else 1) if w.mode != "ehvi" else 0) + \
+            2 * m * 4 + 4
         byts = float(B) * N * per
-        kern = ("ehvi2d_kernel" if w.mode != "mc" else
-                "mchvi2_kernel" if m == 2 else "mchvi_kernel")
+        kern = ("ehvi2d_kernel" if w.mode == "ehvi" else "nehvi2_kernel" if w.mode == "nehvi"
+                else "mchvi2_kernel" if m == 2 else "mchvi_kernel")
         return dict(bound="hbm", achieved=byts / (ms * 1e-3) / 1e9, peak=hbm, unit="GB/s",
                     per_launch=byts, kernel=kern)
     if stage == "topk":
@@ -253,6 +264,9 @@ def oracle_rate(w: wl.Workload, inp, budget_s: float, threads: int = 0, cons=Non
     import oracle
     from oracle import pipeline as opl
     threads = threads or oracle.default_threads()
+    if w.mode == "nehvi" and "z" not in inp:  # the engine's in-sample normals (seed 0)
+        inp["z"] = oracle.base_normals(INSAMPLE_KEY, 1, w.m * w.S, 1, w.n)[0].reshape(
+            w.m, w.S, w.n)
     kern = None if inp["kc"] is None else (w.d_tau, inp["kc"][0])
     tfs = list(w.transforms) or None
     avail = inp["Xc"].shape[1]
@@ -264,7 +278,8 @@ def oracle_rate(w: wl.Workload, inp, budget_s: float, threads: int = 0, cons=Non
         n_try = min(avail, 2048)
         t0 = time.perf_counter()
         opl.score(fp, inp["Xc"][0, :n_try], w.mode, min(w.k, n_try),
-                  None if inp["eps"] is None else inp["eps"][0, :n_try], threads, cons=cons)
+                  None if inp["eps"] is None else inp["eps"][0, :n_try], threads, cons=cons,
+                  z=inp.get("z"))
         per = (time.perf_counter() - t0) / n_try
         sample = int(max(n_try, min(avail, (budget_s - fit_s) / max(per, 1e-9))))
     sample = min(sample, avail)
@@ -272,7 +287,8 @@ def oracle_rate(w: wl.Workload, inp, budget_s: float, threads: int = 0, cons=Non
     fp = opl.fit_problem(inp["X"][0], inp["Y"][0], inp["ls"][0], inp["s2"][0], inp["noise"][0],
                          inp["ref"][0], kernel=kern, transforms=tfs)
     opl.score(fp, inp["Xc"][0, :sample], w.mode, min(w.k, sample),
-              None if inp["eps"] is None else inp["eps"][0, :sample], threads, cons=cons)
+              None if inp["eps"] is None else inp["eps"][0, :sample], threads, cons=cons,
+              z=inp.get("z"))
     dt = time.perf_counter() - t0
     return sample / dt, threads, sample, dt
 
@@ -320,6 +336,9 @@ def main():
     ap.add_argument("--no-serial-stages", action="store_true",
                     help="skip the serialised per-stage breakdown")
     ap.add_argument("--e2e-steps", type=int, default=0, help="0: same as --steps (max 200)")
+    ap.add_argument("--noisy", action="store_true",
+                    help="score with the noisy acquisition (joint in-sample draws; two "
+                         "objectives, n <= 128)")
     ap.add_argument("--candidates", type=int, default=0,
                     help="candidates per problem (0: the workload's N); a smaller N keeps "
                          "profiler captures small")
@@ -328,6 +347,8 @@ def main():
                          "(constrained acquisition; 'inf' leaves an objective unconstrained)")
     args = ap.parse_args()
     w = wl.by_name(args.workload)
+    if args.noisy:
+        w = wl.noisy(w)
     if args.candidates:
         w = wl.scaled(w, N=args.candidates)
     args.cons = [float(c) for c in args.constraints.split(",")] if args.constraints else None
@@ -360,7 +381,7 @@ def main():
     f64, f32 = torch.float64, torch.float32
     dX, dY, dls, ds2, dnz, dref = (t(inp[k], f64) for k in ("X", "Y", "ls", "s2", "noise", "ref"))
     dXc, deps = t(inp["Xc"], f32), t(inp["eps"], f32)
-    mode = bt.BOUTE_ACQ_MC_HVI if w.mode == "mc" else bt.BOUTE_ACQ_EHVI2D
+    mode = {"mc": bt.BOUTE_ACQ_MC_HVI, "nehvi": bt.BOUTE_ACQ_NEHVI}.get(w.mode, bt.BOUTE_ACQ_EHVI2D)
     e = bt.Engine(w.B, w.n, w.d, w.m, w.N, mode, w.S, w.k)
     if args.cons is not None:
         bt.boute_engine_set_constraints(e, torch.tensor([args.cons] * w.B, dtype=f64))
@@ -474,8 +495,8 @@ def main():
     e2e = {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
            "d2h_bytes_per_step": d2h, "call": "boute_engine_step_host_async",
            "pipelined": True, "steps": n_e2e,
-           "normals": "host (copied every step)" if w.mode == "mc" else None}
-    if w.mode == "mc":
+           "normals": "host (copied every step)" if w.mode != "ehvi" else None}
+    if w.mode != "ehvi":
         # the engine's own base normals, drawn once on the device from a seed
         bt.boute_engine_set_normals(e, 1234)
         dn_value, dn_h2d = e2e_stream(None)

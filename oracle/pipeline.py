@@ -73,7 +73,13 @@ def acquisition(fp: FittedProblem, mean, var, mode: str, eps=None, threads: int 
     raise ValueError(mode)
 
 
-def score(fp: FittedProblem, Xc, mode: str, k: int, eps=None, threads: int = 0, cons=None):
+def score(fp: FittedProblem, Xc, mode: str, k: int, eps=None, threads: int = 0, cons=None,
+          z=None):
+    """mode "nehvi": the noisy acquisition with in-sample normals z (m, S, n);
+    mean and var are then the marginal mean and the conditional variance."""
+    if mode == "nehvi":
+        dr, acq, idx, val = noisy_score(fp, Xc, z, eps, k, threads, cons)
+        return dr.mean, dr.cvar, acq, idx, val
     mean, var = posterior(fp, Xc, threads)
     acq = acquisition(fp, mean, var, mode, eps, threads, cons=cons)
     idx, val = topk(acq, k)

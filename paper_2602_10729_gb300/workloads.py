@@ -101,12 +101,23 @@ def composite(w: Workload) -> Workload:
     return dataclasses.replace(w, name=w.name + "-composite", d_tau=w.d // 2, transforms=codes)
 
 
+def noisy(w: Workload) -> Workload:
+    """The same shapes scored by the noisy acquisition (joint in-sample draws,
+    S per objective; two objectives, n <= 128): mode "nehvi", normals as for
+    the Monte-Carlo workloads."""
+    if w.m != 2 or w.S < 1:
+        raise ValueError("the noisy acquisition needs two objectives and S >= 1")
+    return dataclasses.replace(w, name=w.name + "-noisy", mode="nehvi")
+
+
 def by_name(name: str) -> Workload:
     for w in WORKLOADS:
         if w.name == name:
             return w
         if w.name + "-composite" == name:
             return composite(w)
+        if w.name + "-noisy" == name:
+            return noisy(w)
     raise KeyError(name)
 
 

@@ -147,7 +147,7 @@ def host_problem(w: wl.Workload, N: int | None = None, threads: int = 8) -> Host
         Xs.append(X); Ys.append(Y); L.append(ls); S2.append(s2); NZ.append(nz)
     Xc = np.stack([wl.candidates(w, b, 0, N, threads) for b in range(w.B)])
     eps = None
-    if w.mode == "mc":
+    if w.mode in ("mc", "nehvi"):
         eps = np.stack([wl.base_normals(w, b, 0, N, threads) for b in range(w.B)])
     ref = np.tile(wl.ref_point(w), (w.B, 1))
     kc = None
