@@ -120,3 +120,26 @@ def test_topk_bit_exact_on_oracle_values(case):
         oi, ov = oracle.topk(vals[b].astype(np.float64), k)
         assert idx[b].cpu().numpy().tolist() == oi.tolist()
         assert np.array_equal(val[b].cpu().numpy(), ov.astype(np.float32))
+
+
+def test_acquisition_isolated_absolute_floor(case):
+    """The acquisition kernel alone at an absolute floor of 1e-9 instead of
+    1e-3 of the largest value: every candidate, including those far below
+    the best, within 1e-4 relative + 1e-9."""
+    w, hp, g, fits = case
+    N = hp.Xc.shape[1]
+    mi = np.empty((w.B, w.m, N), np.float32)
+    vi = np.empty_like(mi)
+    posts = []
+    for b, fp in enumerate(fits):
+        mean, var = opl.posterior(fp, hp.Xc[b])
+        mi[b], vi[b] = mean.T, var.T
+        posts.append((mi[b].T.astype(np.float64), vi[b].T.astype(np.float64)))
+    g2 = gpu_pipeline(hp, mean_var_in=(mi, vi))
+    for b, fp in enumerate(fits):
+        o = opl.acquisition(fp, *posts[b], w.mode, None if hp.eps is None else hp.eps[b])
+        gv = g2["acq"][b].astype(np.float64)
+        err = np.abs(gv - o) - (1e-4 * np.abs(o) + 1e-9)
+        i = int(np.argmax(err))
+        assert err.max() <= 0, f"candidate {i}: gpu {gv[i]:.6g} oracle {o[i]:.6g}"
+        assert (o < 1e-3 * o.max()).any()  # the case reaches values the relative floor skips
