@@ -991,18 +991,25 @@ __global__ void __launch_bounds__(64) fitb_diag_kernel(const float *Kh_all, int 
 __global__ void __launch_bounds__(kFitbThreads) fitb_panel_kernel(int NP, const float *Aws,
                                                                   float *Wws, int p,
                                                                   const int *fbad) {
+  // T_pJ's tiles of the panel's block row and of W: L_pK (32 x 32) and
+  // W_KJ for the block's two J (row stride 33)
+  __shared__ float Ls[32][33], Ws[2][32][33];
   pdl_wait();
   pdl_trigger();
-  const int bt = blockIdx.y, ld = NP + 1;
+  const int bt = blockIdx.y, ld = NP + 1, tid = threadIdx.x;
   if (fbad[bt]) return;
   const float *A = Aws + (size_t)bt * NP * ld;
   float *W = Wws + (size_t)bt * NP * ld;
   const int p0 = 32 * p, r0 = p0 + 32, rows = NP - r0;
-  const int ntr = (rows / 4) * 8, ntt = p * 128;
-  for (int tix = blockIdx.x * blockDim.x + threadIdx.x; tix < ntr + ntt;
-       tix += gridDim.x * blockDim.x) {
-    float acc[4][4] = {};
-    if (tix < ntr) {
+  // work items: blocks of the panel below (4 x 4 tiles, 256 threads each),
+  // then one item per pair of W's block columns J of T_pJ
+  const int ntr = (rows / 4) * 8, nbr = (ntr + kFitbThreads - 1) / kFitbThreads;
+  const int items = nbr + (p + 1) / 2;
+  for (int item = blockIdx.x; item < items; item += gridDim.x) {
+    if (item < nbr) {
+      const int tix = item * kFitbThreads + tid;
+      if (tix >= ntr) continue;
+      float acc[4][4] = {};
       const int i0 = r0 + 4 * (tix >> 3), c0 = 4 * (tix & 7);
 #pragma unroll 4
       for (int q = 0; q < 32; ++q) {
@@ -1021,25 +1028,45 @@ __global__ void __launch_bounds__(kFitbThreads) fitb_panel_kernel(int NP, const 
       for (int u = 0; u < 4; ++u)
 #pragma unroll
         for (int v = 0; v < 4; ++v) W[(size_t)(i0 + u) * ld + p0 + c0 + v] = acc[u][v];
-    } else {
-      const int e = tix - ntr, J = e >> 7, rb = 4 * ((e >> 4) & 7), cb = 2 * (e & 15);
-#pragma unroll 4
-      for (int q = 32 * J; q < p0; ++q) {
-        float x[4], y2[2];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) x[u] = A[(size_t)(p0 + rb + u) * ld + q];
-#pragma unroll
-        for (int v = 0; v < 2; ++v) y2[v] = W[(size_t)q * ld + 32 * J + cb + v];
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-#pragma unroll
-          for (int v = 0; v < 2; ++v) acc[u][v] = fmaf(x[u], y2[v], acc[u][v]);
+      continue;
+    }
+    // T_pJ = sum_{K=J}^{p-1} L_pK W_KJ for J = J0 (threads 0..127) and J0 + 1
+    // (128..255), 4 x 2 outputs per thread, K block by K block (W_KJ = 0 for
+    // K < J, and W's upper triangle holds other data, so each J starts at K = J)
+    const int J0 = 2 * (item - nbr), half = tid >> 7, e = tid & 127;
+    const int J = J0 + half, rb = 4 * (e >> 4), cb = 2 * (e & 15);
+    float acc[4][2] = {};
+    for (int K = J0; K < p; ++K) {
+      __syncthreads();  // the previous K's tiles are consumed
+      for (int x = tid; x < 32 * 32; x += kFitbThreads) {
+        const int r = x >> 5, c = x & 31;
+        Ls[r][c] = A[(size_t)(p0 + r) * ld + 32 * K + c];
+        Ws[0][r][c] = W[(size_t)(32 * K + r) * ld + 32 * J0 + c];
+        Ws[1][r][c] = J0 + 1 < p ? W[(size_t)(32 * K + r) * ld + 32 * (J0 + 1) + c] : 0.f;
       }
+      __syncthreads();
+      if (K >= J && J < p) {
+#pragma unroll 8
+        for (int q = 0; q < 32; ++q) {
+          float xv[4], yv[2];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) xv[u] = Ls[rb + u][q];
+#pragma unroll
+          for (int v = 0; v < 2; ++v) yv[v] = Ws[half][q][cb + v];
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+#pragma unroll
+            for (int v = 0; v < 2; ++v) acc[u][v] = fmaf(xv[u], yv[v], acc[u][v]);
+        }
+      }
+    }
+    if (J < p) {
 #pragma unroll
       for (int u = 0; u < 4; ++u)
 #pragma unroll
         for (int v = 0; v < 2; ++v) W[(size_t)(32 * J + cb + v) * ld + p0 + rb + u] = acc[u][v];
     }
+    __syncthreads();  // before the next item reuses the tiles
   }
 }
 
@@ -1228,10 +1255,13 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
       const int rows = npad - 32 * p - 32, th = rows / 4;
       launch_pdl(fitb_diag_kernel, dim3(BM), dim3(64), 0, s, (const float *)gp->Kh, n, npad,
                  gp->Aws, gp->Wws, p, gp->fbad);
-      const long long tb = (long long)th * 8 + 128LL * p;
-      if (tb > 0) {
-        launch_pdl(fitb_panel_kernel, dim3(ctas(tb), BM), dim3(kFitbThreads), 0, s, npad,
-                   (const float *)gp->Aws, gp->Wws, p, (const int *)gp->fbad);
+      // items: the panel below's blocks, then one per pair of W's block columns
+      const long long items = ((long long)th * 8 + kFitbThreads - 1) / kFitbThreads + (p + 1) / 2;
+      if (items > 0) {
+        launch_pdl(fitb_panel_kernel,
+                   dim3((unsigned)std::max(1LL, std::min<long long>(cap, items)), BM),
+                   dim3(kFitbThreads), 0, s, npad, (const float *)gp->Aws, gp->Wws, p,
+                   (const int *)gp->fbad);
         ++nl;
       }
       const long long tc = (long long)th * (th + 1) / 2 + 128LL * p + 32LL * rows;
