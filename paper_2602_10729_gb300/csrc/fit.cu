@@ -674,23 +674,25 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     }
     __syncthreads();
   };
-  // global variant: thread per row, then thread per column (4 accumulators)
+  // global variant: a warp per row of W (coalesced loads, lanes combined by
+  // shuffles in a fixed order), then a thread per column (4 accumulators)
   auto solve = [&](const float *rhs, float *out) {
     if constexpr (SMEM) {
       solve_blocks(rhs, out);
     } else {
-    for (int i = tid; i < NP; i += nthr) {
+    for (int i = warp; i < NP; i += nw) {
       const float *wr = W + (size_t)i * ld;
-      float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-      int k = 0;
-      for (; k + 3 <= i; k += 4) {
+      float s0 = 0.f, s1 = 0.f;
+      int k = lane;
+      for (; k + 32 <= i; k += 64) {
         s0 = fmaf(wr[k], rhs[k], s0);
-        s1 = fmaf(wr[k + 1], rhs[k + 1], s1);
-        s2 = fmaf(wr[k + 2], rhs[k + 2], s2);
-        s3 = fmaf(wr[k + 3], rhs[k + 3], s3);
+        s1 = fmaf(wr[k + 32], rhs[k + 32], s1);
       }
-      for (; k <= i; ++k) s0 = fmaf(wr[k], rhs[k], s0);
-      tv[i] = (s0 + s1) + (s2 + s3);
+      if (k <= i) s0 = fmaf(wr[k], rhs[k], s0);
+      float v = s0 + s1;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL, v, o);
+      if (lane == 0) tv[i] = v;
     }
     __syncthreads();
     for (int k = tid; k < NP; k += nthr) {
