@@ -319,6 +319,18 @@ int boute_acq_nehvi2d(const float *mean, const float *cvar, const float *shift, 
  * the device stays usable either way. */
 int boute_selftest_wait(int complete, unsigned long long limit_ns, void *stream);
 
+/* Debug build (the library compiled with BOUTE_DEBUG_BOUNDS, see the
+ * package's build_debug): the kernels check their index arithmetic — every
+ * guarded access tests 0 <= index < extent, records the first index out of
+ * its extent per source unit and skips the access (the bulk copies, the
+ * operand images, the outputs, the strips and boxes, the selection). This
+ * call waits for the device, returns 1 and fills rec (4 words: the source
+ * unit 1 posterior, 2 in-sample, 3 acquisition, 4 front, 5 fit, 6 top-k;
+ * the source line; the index; the extent) when some unit recorded one since
+ * the last call, else 0; it clears the records. The product library returns
+ * BOUTE_ERR_UNSUPPORTED (its checks compile to nothing). */
+int boute_bounds_report(long long *rec);
+
 /* Monte-Carlo base normals from a counter-based generator, for callers that
  * do not draw their own: Philox4x64-10 (Salmon et al., SC'11, counter-based:
  * any sample can be regenerated alone) and the Box-Muller transform in fp64,

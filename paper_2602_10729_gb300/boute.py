@@ -25,7 +25,7 @@ SYMBOLS = (
     "boute_gp_fit", "boute_gp_status", "boute_gp_free", "boute_gp_posterior",
     "boute_gp_set_precision", "boute_gp_posterior_fp64",
     "boute_gp_set_insample", "boute_gp_insample", "boute_gp_posterior_joint",
-    "boute_insample_fronts", "boute_acq_nehvi2d",
+    "boute_insample_fronts", "boute_acq_nehvi2d", "boute_bounds_report",
     "boute_pareto_front", "boute_box_decompose", "boute_acq_ehvi", "boute_acq_mc_hvi",
     "boute_select_topk", "boute_select_topk_noalloc", "boute_engine_create", "boute_engine_step",
     "boute_engine_step_async",
@@ -87,6 +87,7 @@ def load(path: str | None = None):
         "boute_gp_free": ([_vp], None),
         "boute_gp_posterior": ([_vp, _vp, _ll, _vp, _vp, _vp], _i),
         "boute_gp_set_insample": ([_vp, _i], _i),
+        "boute_bounds_report": ([_vp], _i),
         "boute_gp_insample": ([_vp, _vp, _vp, _vp, _vp, _vp, _vp], _i),
         "boute_gp_posterior_joint": ([_vp, _vp, _ll, _vp, _vp, _vp, _vp], _i),
         "boute_insample_fronts": ([_vp, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
@@ -323,6 +324,16 @@ def boute_engine_set_n(e: Engine, n: int):
     """Later steps use n <= the engine's creation n observations."""
     _check(load().boute_engine_set_n(e.handle, int(n)), "boute_engine_set_n")
     e.n = int(n)
+
+
+def boute_bounds_report():
+    """Debug build: (unit, line, index, extent) of the first index found outside
+    its extent since the last call, or None; raises on the product library."""
+    rec = (ctypes.c_longlong * 4)()
+    rc = load().boute_bounds_report(rec)
+    if rc not in (0, 1):
+        raise BouteError(rc, "boute_bounds_report")
+    return tuple(rec) if rc == 1 else None
 
 
 def boute_selftest_wait(complete: bool, limit_ns: int, stream=None) -> int:

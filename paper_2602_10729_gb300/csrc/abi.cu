@@ -1102,6 +1102,33 @@ int boute_engine_set_kernel(boute_engine *e, int d_tau, const double *params) {
   return r;
 }
 
+int boute_bounds_report(long long *rec) {
+  BOUTE_TRACE();
+  if (!rec) return BOUTE_ERR_INVALID_ARG;
+#ifndef BOUTE_DEBUG_BOUNDS
+  rec[0] = rec[1] = rec[2] = rec[3] = 0;
+  return BOUTE_ERR_UNSUPPORTED;
+#else
+  if (cudaDeviceSynchronize() != cudaSuccess) return last_launch_status();
+  int (*readers[])(long long *) = {bounds_read_posterior, bounds_read_insample, bounds_read_acq,
+                                   bounds_read_front,     bounds_read_fit,      bounds_read_topk};
+  int found = 0;
+  rec[0] = rec[1] = rec[2] = rec[3] = 0;
+  for (int u = 0; u < (int)(sizeof(readers) / sizeof(readers[0])); ++u) {
+    long long r[4];
+    if (readers[u](r) != 0) return BOUTE_ERR_CUDA;
+    if (r[0] && !found) {  // the first unit with a record; every record is cleared
+      rec[0] = u + 1;
+      rec[1] = r[1];
+      rec[2] = r[2];
+      rec[3] = r[3];
+      found = 1;
+    }
+  }
+  return found;
+#endif
+}
+
 int boute_selftest_wait(int complete, unsigned long long limit_ns, void *stream) {
   BOUTE_TRACE();
   if (limit_ns > BOUTE_WAIT_NS) return BOUTE_ERR_INVALID_ARG;

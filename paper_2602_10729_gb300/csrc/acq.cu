@@ -114,7 +114,7 @@ __global__ void __launch_bounds__(256) ehvi2d_kernel(const float *mean, const fl
       ga = gb;
       a = bb;
     }
-    acq[(size_t)b * N + c] = e;
+    if (BOUTE_INB((long long)b * N + c, (long long)gridDim.y * N)) acq[(size_t)b * N + c] = e;
   }
 }
 
@@ -203,7 +203,7 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
   pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
   const int b = blockIdx.y;
-  const int K = Kc[b];
+  const int K = BOUTE_INB(Kc[b], box_cap + 1) ? Kc[b] : 0;
   float *lo = boxes, *hi = boxes + (size_t)box_cap * M;
   for (int i = threadIdx.x; i < K * M; i += blockDim.x) {
     lo[i] = lower[(size_t)b * box_cap * M + i];
@@ -224,6 +224,10 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
     }
     const float *e = eps + ((size_t)b * N + c) * eps_stride +
                      (eps_stride == 0 ? (size_t)b * M * S : 0);
+    if (!BOUTE_INB((eps_stride ? ((long long)b * N + c) * eps_stride : (long long)b * M * S) +
+                       M * S - 1,
+                   eps_stride ? (long long)B * N * eps_stride : (long long)B * M * S))
+      continue;  // (warp-uniform)
     float sum = 0.f;
     if (vec && S == 256) {
       sum = mc_hvi_regs<M, CONS, 2>(e, S, mu, sg, kc, lo, hi, K, lane);
@@ -288,7 +292,8 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    if (lane == 0) acq[(size_t)b * N + c] = sum / (float)S;
+    if (lane == 0 && BOUTE_INB((long long)b * N + c, (long long)B * N))
+      acq[(size_t)b * N + c] = sum / (float)S;
   }
 }
 
@@ -373,7 +378,8 @@ __global__ void __launch_bounds__(512, 2) mchvi2_kernel(const float *mean, const
       pm1 = m1[cn]; pm2 = m2[cn]; pv1 = v1[cn]; pv2 = v2[cn];
       const float sum =
           mc2_warp_total(mc2_lane_sum<CONS>(strips4, K, Kp, t0, c1, c2, mu1, mu2, qv1, qv2, k1, k2));
-      if (lane == 0) acq[(size_t)b * N + c] = sum * inv_s;
+      if (lane == 0 && BOUTE_INB((long long)b * N + c, (long long)gridDim.y * N))
+        acq[(size_t)b * N + c] = sum * inv_s;
       if (SEL) sel.add(make_key(sum * inv_s, (unsigned)c), lane);
     }
   } else {
@@ -390,7 +396,8 @@ __global__ void __launch_bounds__(512, 2) mchvi2_kernel(const float *mean, const
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    if (lane == 0) acq[(size_t)b * N + c] = sum * inv_s;
+    if (lane == 0 && BOUTE_INB((long long)b * N + c, (long long)gridDim.y * N))
+        acq[(size_t)b * N + c] = sum * inv_s;
     if (SEL) sel.add(make_key(sum * inv_s, (unsigned)c), lane);
   }
   }
@@ -668,6 +675,8 @@ __global__ void normals_kernel(unsigned long long seed, int B, long long N, int 
 }
 
 }  // namespace
+
+BOUTE_BOUNDS_READER(acq)
 
 int launch_base_normals(unsigned long long seed, int B, long long N, int m, int S, float *eps,
                         cudaStream_t s) {

@@ -226,8 +226,13 @@ __device__ __forceinline__ bool pack_pair(const float *wrow, int g, int k, const
   const int q = g / BOUTE_BLKCOLS, c = k / BOUTE_ACHUNK, ncol = plan.ncol[q];
   uint32_t *blk = (uint32_t *)(img + plan.off[q] + (long long)c * 2 * ncol * BOUTE_ACHUNK);
   const int o = sw128_off16(g % BOUTE_BLKCOLS, k % BOUTE_ACHUNK) >> 1;
-  blk[o] = hi;
-  blk[(ncol * BOUTE_ACHUNK >> 1) + o] = lo;
+  const long long base = plan.off[q] + (long long)c * 2 * ncol * BOUTE_ACHUNK;
+  (void)base;  // (used by the debug build's checks)
+  if (BOUTE_INB(base + 2 * ((ncol * BOUTE_ACHUNK >> 1) + o) + 1, plan.image_halves) &&
+      BOUTE_INB(q, plan.nwblk)) {
+    blk[o] = hi;
+    blk[(ncol * BOUTE_ACHUNK >> 1) + o] = lo;
+  }
   return fabsf(v0) < 32768.f && fabsf(v1) < 32768.f;
 }
 
@@ -1296,5 +1301,7 @@ int launch_fit_raw(Gp *gp, const double *X, const double *Y, const double *ls, c
                    const double *noise, cudaStream_t s, cudaEvent_t setup_done) {
   return launch_fit_impl(gp, X, Y, 1, ls, s2, noise, s, setup_done);
 }
+
+BOUTE_BOUNDS_READER(fit)
 
 }  // namespace boute

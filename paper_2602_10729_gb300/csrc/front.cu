@@ -119,8 +119,10 @@ __device__ void boxes_block(const double *F, int Pb, int n, int m, const double 
                             float *hi, int *Kout, void *smem) {
   double *ws = (double *)smem;
   const int cap = 2 * n + 2;
+  (void)cap;  // (the debug build checks the box count against it)
   if (m == 2) {
     for (int i = threadIdx.x; i <= Pb; i += blockDim.x) {
+      if (!BOUTE_INB(i, cap)) break;
       lo[2 * i] = i == 0 ? -INFINITY : (float)F[2 * (i - 1)];
       lo[2 * i + 1] = -INFINITY;
       hi[2 * i] = i == Pb ? (float)r[0] : (float)F[2 * i];
@@ -149,7 +151,8 @@ __device__ void boxes_block(const double *F, int Pb, int n, int m, const double 
   int ns = 0, nc = 1, K = 0;
   ca[0] = -INFINITY; cb[0] = r[0]; cu[0] = r[1]; cz[0] = -INFINITY;
   auto emit = [&](double a, double bb, double u, double z0, double z1) {
-    if (z1 > z0 && bb > a && K < cap) {
+    // (a decomposition with more than cap boxes is reported by the debug build)
+    if (z1 > z0 && bb > a && BOUTE_INB(K, cap)) {
       lo[K * 3 + 0] = (float)a; lo[K * 3 + 1] = -INFINITY; lo[K * 3 + 2] = (float)z0;
       hi[K * 3 + 0] = (float)bb; hi[K * 3 + 1] = (float)u; hi[K * 3 + 2] = (float)z1;
       ++K;
@@ -291,5 +294,7 @@ int launch_front_fused(const double *Y, int B, int n, int m, const double *ref, 
   count_launch();
   return last_launch_status();
 }
+
+BOUTE_BOUNDS_READER(front)
 
 }  // namespace boute

@@ -61,8 +61,13 @@ __device__ __forceinline__ void pack_dense_pair(const float *src, int n, int k, 
   const int ncol = plan.ncol[q], cidx = k / BOUTE_ACHUNK;
   uint32_t *blk = (uint32_t *)(img + plan.off[q] + (long long)cidx * 2 * ncol * BOUTE_ACHUNK);
   const int o = sw128_off16(row % BOUTE_BLKCOLS, k % BOUTE_ACHUNK) >> 1;
-  blk[o] = hi;
-  blk[(ncol * BOUTE_ACHUNK >> 1) + o] = lo;
+  const long long base = plan.off[q] + (long long)cidx * 2 * ncol * BOUTE_ACHUNK;
+  (void)base;  // (used by the debug build's checks)
+  if (BOUTE_INB(base + 2 * ((ncol * BOUTE_ACHUNK >> 1) + o) + 1, plan.image_halves) &&
+      BOUTE_INB(k, plan.nchunk * BOUTE_ACHUNK)) {
+    blk[o] = hi;
+    blk[(ncol * BOUTE_ACHUNK >> 1) + o] = lo;
+  }
 }
 
 // (1) one CTA per problem-objective: the sequential part. K^-1 = W^T W, the
@@ -352,7 +357,7 @@ __global__ void __launch_bounds__(kDrawThreads)
 #pragma unroll
   for (int r = 0; r < R; ++r) {
     const int i = lane + 32 * r;
-    if (i < n) {
+    if (i < n && BOUTE_INB(zoff + (long long)s * n + i, (long long)gridDim.y * S * n)) {
       Yin[zoff + (size_t)s * n + i] = y[r];
       gws[zoff + (size_t)s * n + i] = g[r];
       gm = fmaxf(gm, fabsf(g[r]));
@@ -507,7 +512,7 @@ __global__ void __launch_bounds__(32 * kFrontWarps)
   __syncwarp();
 #pragma unroll
   for (int r = 0; r < kFrontPts; ++r)
-    if (keep[r]) {
+    if (keep[r] && BOUTE_INB(rank[r] + 1, n + 1)) {
       const float u1 = rank[r] + 1 < P ? f1s[w][rank[r] + 1] : r1;
       st[rank[r] + 1] = make_float4(p1[r], u1, p2[r], 0.f);
     }
@@ -571,7 +576,7 @@ __global__ void __launch_bounds__(kAcqThreads)
         if (off_s[mid] <= q) lo = mid;
         else hi = mid;
       }
-      st_s[q] = stb[(size_t)lo * (n + 1) + (q - off_s[lo])];
+      if (BOUTE_INB(q - off_s[lo], n + 1)) st_s[q] = stb[(size_t)lo * (n + 1) + (q - off_s[lo])];
     }
   __syncthreads();
   if (c >= N) return;
@@ -583,12 +588,17 @@ __global__ void __launch_bounds__(kAcqThreads)
   const float c1 = hc ? (float)cons[(size_t)b * 2 + 1] : INFINITY;
   const float *e = eps + ((size_t)b * N + c) * eps_stride + (eps_stride == 0 ? (size_t)b * 2 * S : 0);
   const float *sh0 = shift + ((size_t)b * 2) * S * N + c, *sh1 = sh0 + (size_t)S * N;
+  // the candidate's normals and its last shift lie inside their arrays
+  if (!BOUTE_INB((eps_stride ? ((long long)b * N + c) * eps_stride : (long long)b * 2 * S) + 2 * S - 1,
+                 eps_stride ? (long long)gridDim.y * N * eps_stride : (long long)gridDim.y * 2 * S) ||
+      !BOUTE_INB((((long long)b * 2 + 1) * S + S - 1) * N + c, (long long)gridDim.y * 2 * S * N))
+    return;
   float acc = 0.f;
   auto draw = [&](int s, float e0, float e1, float h0, float h1) {
     const float ya = fmaf(sd0, e0, m0 + h0);
     const float yb = fmaf(sd1, e1, m1 + h1);
     if (!(ya <= c0 && yb <= c1)) return;  // infeasible (or no improvement possible)
-    const int k = off_s[s + 1] - off_s[s];
+    const int k = BOUTE_INB(off_s[s + 1] - off_s[s] - 1, n + 1) ? off_s[s + 1] - off_s[s] : 0;
     const float4 *st = staged ? st_s + off_s[s] : stb + (size_t)s * (n + 1);
     float h = 0.f;
     for (int j = 0; j < k; ++j) {
@@ -622,10 +632,12 @@ __global__ void __launch_bounds__(kAcqThreads)
     }
   }
   for (; s < S; ++s) draw(s, e[s], e[S + s], sh0[(size_t)s * N], sh1[(size_t)s * N]);
-  acq[(size_t)b * N + c] = acc / (float)S;
+  if (BOUTE_INB((long long)b * N + c, (long long)gridDim.y * N)) acq[(size_t)b * N + c] = acc / (float)S;
 }
 
 }  // namespace
+
+BOUTE_BOUNDS_READER(insample)
 
 int launch_insample_fronts(const float *Yin, int B, int n, int S, const double *ref,
                            const double *cons, float *strips, int *counts, cudaStream_t s) {

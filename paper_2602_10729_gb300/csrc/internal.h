@@ -3,6 +3,7 @@
 
 #include <cuda_runtime.h>
 
+#include "bounds.cuh"
 #include "common.cuh"
 
 #include <nvtx3/nvToolsExt.h>
@@ -118,6 +119,13 @@ int launch_posterior_joint(const Gp *gp, const float *Xc, long long N, float *me
                            float *shift, cudaStream_t s, const float *kst = nullptr);
 // the library's device check (an sm_103a device is current)
 int device_ok();
+// bounds records of the debug build, per translation unit (bounds.cuh)
+int bounds_read_posterior(long long *out);
+int bounds_read_insample(long long *out);
+int bounds_read_acq(long long *out);
+int bounds_read_front(long long *out);
+int bounds_read_fit(long long *out);
+int bounds_read_topk(long long *out);
 // codes: outcome transforms before standardising (objective_code)
 int launch_standardize(const double *Y, int B, int n, int m, int codes, double *Ys,
                        cudaStream_t s);

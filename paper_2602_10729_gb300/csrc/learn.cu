@@ -88,7 +88,7 @@ __global__ void __launch_bounds__(kLearnThreads) learn_kernel(
   __shared__ double logdet, mll_s;
   __shared__ int bad;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int blk = blockIdx.x, r = blk % R, bt = blk / R, b = bt / m, t = bt % m;
+  const int blk = blockIdx.x, bt = blk / R, b = bt / m, t = bt % m;
   const int P = d + (COMP ? 5 : 2), ld = learn_ld(n), dc = d - dtau;
   double *A = use_smem ? lsm : ws + (size_t)blk * learn_ws_doubles(n, d);
   double *xs = A + (size_t)n * ld, *yv = xs + (size_t)n * d, *av = yv + n, *tmp = av + n, *dinv = tmp + n,

@@ -41,7 +41,7 @@ __device__ __forceinline__ float rcp_fast(float x) {
 __device__ __forceinline__ int mc2_load_strips(float4 *strips4, const float *lower,
                                                const float *upper, const int *Kc, int b,
                                                int box_cap, int t, int nthr) {
-  const int K = Kc[b];
+  const int K = BOUTE_INB(Kc[b], box_cap + 1) ? Kc[b] : 0;
   const int Kp = K > 0 ? 1 + (K & ~1) : 0;
   for (int i = t; i < Kp; i += nthr) {
     if (i >= K) {

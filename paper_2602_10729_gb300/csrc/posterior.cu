@@ -536,9 +536,10 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
               if (cached) {  // the A stage from this CTA's cache, no side input
                 if (qa >= (uint32_t)SA && !wait_or_abort(&a_empty[s], ra.phase ^ 1u, abort)) break;
                 mbar_expect_tx(&a_full[s], kABytes);
-                bulk_g2s(a_hi(s),
-                         a.kcache + ((size_t)blockIdx.x * a.ncache + c) * (kABytes / 2), kABytes,
-                         &a_full[s]);
+                if (BOUTE_INB(blockIdx.x * a.ncache + c, (long long)gridDim.x * a.ncache))
+                  bulk_g2s(a_hi(s),
+                           a.kcache + ((size_t)blockIdx.x * a.ncache + c) * (kABytes / 2),
+                           kABytes, &a_full[s]);
                 mbar_arrive_n(&a_full[s], kBldWarps);
                 last_ca = (int)qa;
               }
@@ -550,9 +551,10 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
               const int s = ra.idx;
               if (qa >= (uint32_t)SA && !wait_or_abort(&st_empty[s], ra.phase ^ 1u, abort)) break;
               mbar_arrive_expect_tx(&st_full[s], kStageBytes);
-              bulk_g2s((void *)stage(s),
-                       a.kst + ((size_t)unit * pl.nchunk + c) * (kStageBytes / 4), kStageBytes,
-                       &st_full[s]);
+              if (BOUTE_INB((long long)unit * pl.nchunk + c, (long long)units * pl.nchunk))
+                bulk_g2s((void *)stage(s),
+                         a.kst + ((size_t)unit * pl.nchunk + c) * (kStageBytes / 4), kStageBytes,
+                         &st_full[s]);
               last_qa = (int)qa;
               ++qa;
               ra.advance(SA);
@@ -569,14 +571,16 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
                 const int ncol = pl.ncol[qb];
                 const uint32_t bytes = (uint32_t)(2 * ncol * 128);
                 mbar_arrive_expect_tx(&full[s], bytes);
-                bulk_g2s(b_reg(s),
-                         a.bop + (size_t)bt * pl.image_halves + pl.off[qb] +
-                             (size_t)c * 2 * ncol * BOUTE_ACHUNK,
-                         bytes, &full[s]);
+                const long long bo = (long long)bt * pl.image_halves + pl.off[qb] +
+                                     (long long)c * 2 * ncol * BOUTE_ACHUNK;
+                if (BOUTE_INB(bo + bytes / 2 - 1, (long long)a.B * m * pl.image_halves) &&
+                    BOUTE_INB(bytes, (long long)a.b_bytes + 1))
+                  bulk_g2s(b_reg(s), a.bop + bo, bytes, &full[s]);
               } else {
                 mbar_arrive_expect_tx(&full[s], a.x_bytes);
-                bulk_g2s(xt_reg(s), a.xt + ((size_t)bt * pl.nxt + 2 * c + job) * cf, a.x_bytes,
-                         &full[s]);
+                const long long xo = ((long long)bt * pl.nxt + 2 * c + job) * cf;
+                if (BOUTE_INB(xo + a.x_bytes / 4 - 1, (long long)a.B * m * pl.nxt * cf))
+                  bulk_g2s(xt_reg(s), a.xt + xo, a.x_bytes, &full[s]);
               }
               last_q = (int)q;
               ++q;
@@ -615,8 +619,9 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
             const uint32_t sah = smem_u32(a_hi(sa)), sal = sah + kAPartBytes;
             const bool store = storing && c >= kcp;  // built here, needed later
             if (store) {
-              bulk_s2g(a.kcache + ((size_t)blockIdx.x * a.ncache + c) * (kABytes / 2), a_hi(sa),
-                       kABytes);
+              if (BOUTE_INB(blockIdx.x * a.ncache + c, (long long)gridDim.x * a.ncache))
+                bulk_s2g(a.kcache + ((size_t)blockIdx.x * a.ncache + c) * (kABytes / 2),
+                         a_hi(sa), kABytes);
               bulk_commit();
             }
             for (int jb = 0; jb <= q1 - q0; ++jb) {
@@ -720,7 +725,10 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
               if (live)
 #pragma unroll
                 for (int e = 0; e < 16; ++e)
-                  if (s0 + cc + e < pl.S_in) shrow[(size_t)(s0 + cc + e) * a.N] = v[e] * gscale;
+                  if (s0 + cc + e < pl.S_in &&
+                      BOUTE_INB((((long long)b * m + t) * pl.S_in + s0 + cc + e) * a.N + row,
+                                (long long)a.B * m * pl.S_in * a.N))
+                    shrow[(size_t)(s0 + cc + e) * a.N] = v[e] * gscale;
             }
           }
           tc_fence_before();
@@ -734,7 +742,8 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
         // V carries the scales 2^e_r (K*) and 2^e_W (W); H^T k* 2^e_r and 2^e_H
         float vv = prior - ldexpf(ss, -2 * (er + (int)par[kParEW]));
         if (pl.nhblk > 0) vv -= ldexpf(ssh, -2 * (er + (int)par[kParEH]));
-        a.var[((size_t)b * m + t) * a.N + row] = vv > 0.f ? vv : 0.f;
+        if (BOUTE_INB(((long long)b * m + t) * a.N + row, (long long)a.B * m * a.N))
+          a.var[((size_t)b * m + t) * a.N + row] = vv > 0.f ? vv : 0.f;
       }
     }
   } else if (warp >= kBldWarp0) {
@@ -838,8 +847,10 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
                   split_f16x2(v0, v1, hi[e], lo[e]);
                 }
                 const int o = sw128_off16(r, col0 + 8 * u) * 2;  // bytes
-                *(uint4 *)(Ah + o) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-                *(uint4 *)(Al + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+                if (BOUTE_INB(o + 15, (long long)kAPartBytes)) {
+                  *(uint4 *)(Ah + o) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                  *(uint4 *)(Al + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+                }
               }
             };
             if (jbase + COLS <= n) emit(std::false_type{});
@@ -891,7 +902,9 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
           if (lane == src) mean = (float)v;
         }
       }
-      if (g == 0 && row < a.N) a.mean[((size_t)b * m + t) * a.N + row] = mean;
+      if (g == 0 && row < a.N &&
+          BOUTE_INB(((long long)b * m + t) * a.N + row, (long long)a.B * m * a.N))
+        a.mean[((size_t)b * m + t) * a.N + row] = mean;
     }
   }
 
@@ -1072,6 +1085,8 @@ int launch_kstar_dp(const Gp *gp, const float *Xc, long long N, float *kst, cuda
 }
 
 }  // namespace
+
+BOUTE_BOUNDS_READER(posterior)
 
 int launch_posterior_joint(const Gp *gp, const float *Xc, long long N, float *mean, float *cvar,
                            float *shift, cudaStream_t s, const float *kst) {

@@ -66,8 +66,10 @@ __global__ void __launch_bounds__(kThreads) segment_topk_kernel(
   if (idx) {  // final level: one segment per problem
     for (int i = threadIdx.x; i < k; i += blockDim.x) {
       const unsigned j = key_index(buf[i]);
-      idx[(size_t)b * k + i] = (long long)j;
-      val[(size_t)b * k + i] = acq[(size_t)b * N + j];
+      if (BOUTE_INB(i, k) && BOUTE_INB(j, N)) {
+        idx[(size_t)b * k + i] = (long long)j;
+        val[(size_t)b * k + i] = acq[(size_t)b * N + j];
+      }
     }
   } else {
     unsigned long long *out = keys_out + ((size_t)b * nseg + seg) * k;
@@ -149,8 +151,10 @@ __global__ void __launch_bounds__(kWarpBlock) warp_topk_kernel(
   }
   if (lane < k) {
     const unsigned j = key_index(top);
-    idx[(size_t)b * k + lane] = (long long)j;
-    val[(size_t)b * k + lane] = vals[row + j];
+    if (BOUTE_INB(lane, k)) {
+      idx[(size_t)b * k + lane] = (long long)j;
+      val[(size_t)b * k + lane] = vals[row + j];
+    }
   }
 }
 
@@ -223,5 +227,7 @@ int launch_topk(const float *acq, int B, long long N, int k, long long *idx, flo
   count_launch(launches);
   return last_launch_status();
 }
+
+BOUTE_BOUNDS_READER(topk)
 
 }  // namespace boute
