@@ -128,3 +128,121 @@ def noisy_score(fp: FittedProblem, Xc, z, eps, k: int, threads: int = 0, cons=No
     acq = noisy_acquisition(fp, dr, eps, threads, cons)
     idx, val = topk(acq, k)
     return dr, acq, idx, val
+
+
+# ---- optimising the acquisition over the decision space (Sec. 5.2 step (ii)) -----
+# The Monte-Carlo hypervolume improvement with fixed base normals (a sample
+# average, so that the acquisition is a deterministic, piecewise smooth
+# function of the point x), its gradient through the GP posterior, and
+# projected Adam ascent from given starting points. Two objectives, the
+# Matern-5/2 kernel, the observed front.
+_SQRT5 = 5.0 ** 0.5
+
+
+def _kstar_grad(X, ls, s2, x):
+    """k*_j = s2 (1 + sqrt5 r + 5/3 r^2) exp(-sqrt5 r) at the scaled distance r
+    of x to X_j, and its gradient in x: dk*_j/dx = -5/3 s2 (1 + sqrt5 r)
+    exp(-sqrt5 r) (x - X_j) / ls^2 (n x d)."""
+    diff = (x[None, :] - X) / ls
+    r = np.sqrt((diff * diff).sum(1))
+    ex = np.exp(-_SQRT5 * r)
+    k = s2 * (1.0 + _SQRT5 * r + 5.0 / 3.0 * r * r) * ex
+    dk = (-5.0 / 3.0 * s2 * (1.0 + _SQRT5 * r) * ex)[:, None] * diff / ls[None, :]
+    return k, dk
+
+
+def _forward(L, b):
+    x = np.empty_like(b)
+    for i in range(len(b)):
+        x[i] = (b[i] - L[i, :i] @ x[:i]) / L[i, i]
+    return x
+
+
+def _backward(L, b):  # solves L^T x = b
+    n = len(b)
+    x = np.empty_like(b)
+    for i in range(n - 1, -1, -1):
+        x[i] = (b[i] - L[i + 1:, i] @ x[i + 1:]) / L[i, i]
+    return x
+
+
+def posterior_grad(fp: FittedProblem, t: int, x):
+    """Posterior mean and variance of objective t at x and their gradients:
+    mean = k*^T alpha, var = s2 - v^T v with v = L^-1 k*, d var/dx = -2
+    (K^-1 k*)^T dk*/dx."""
+    k, dk = _kstar_grad(fp.X, fp.ls[t], fp.s2[t], np.asarray(x, np.float64))
+    mean = k @ fp.alpha[t]
+    dmean = dk.T @ fp.alpha[t]
+    v = _forward(fp.L[t], k)
+    var = fp.s2[t] - v @ v
+    kinv_k = _backward(fp.L[t], v)
+    dvar = -2.0 * dk.T @ kinv_k
+    return mean, var, dmean, dvar
+
+
+def _strips(front, ref):
+    """The undominated region of a 2-D front (f1 ascending) as strips
+    (a_k, b_k, u_k): x in [a_k, b_k), y below u_k."""
+    P = len(front)
+    a = np.concatenate([[-np.inf], front[:, 0]])
+    b = np.concatenate([front[:, 0], [ref[0]]]) if P else np.array([ref[0]])
+    u = np.concatenate([[ref[1]], front[:, 1]])
+    return a, b, u
+
+
+def hvi2_grad(front, ref, y):
+    """Hypervolume improvement of y over a 2-D front and its gradient in y:
+    HVI = sum_k (b_k - max(a_k, y1))+ (u_k - y2)+."""
+    a, b, u = _strips(front, ref)
+    w = np.maximum(b - np.maximum(a, y[0]), 0.0)
+    h = np.maximum(u - y[1], 0.0)
+    val = float((w * h).sum())
+    inside = (a < y[0]) & (y[0] < b)
+    g1 = -float((inside * h).sum())
+    g2 = -float((w * (y[1] < u)).sum())
+    return val, np.array([g1, g2])
+
+
+def mc_hvi_value_grad(fp: FittedProblem, x, eps):
+    """The sample-average acquisition (1/S) sum_s HVI(mean + sd eps_s) at x,
+    eps: (2, S) base normals, and its gradient in x (the chain through the
+    posterior mean and standard deviation of both objectives)."""
+    x = np.asarray(x, np.float64)
+    eps = np.asarray(eps, np.float64)
+    S = eps.shape[1]
+    mu, sd, dmu, dsd = [], [], [], []
+    for t in range(2):
+        m_, v_, dm_, dv_ = posterior_grad(fp, t, x)
+        s_ = np.sqrt(max(v_, 0.0))
+        mu.append(m_)
+        sd.append(s_)
+        dmu.append(dm_)
+        dsd.append(dv_ / (2.0 * s_) if s_ > 0 else np.zeros_like(dv_))
+    val, grad = 0.0, np.zeros_like(x)
+    for s in range(S):
+        y = np.array([mu[0] + sd[0] * eps[0, s], mu[1] + sd[1] * eps[1, s]])
+        h, g = hvi2_grad(fp.front, fp.ref, y)
+        val += h
+        grad += g[0] * (dmu[0] + eps[0, s] * dsd[0]) + g[1] * (dmu[1] + eps[1, s] * dsd[1])
+    return val / S, grad / S
+
+
+def optimize_acq(fp: FittedProblem, X0, eps, lower, upper, steps: int, lr: float):
+    """Projected Adam ascent (beta1 0.9, beta2 0.999, eps 1e-8) on
+    mc_hvi_value_grad from each row of X0, every iterate clamped to
+    [lower, upper]. Returns the final points and their acquisition values."""
+    X = np.array(X0, np.float64, copy=True)
+    out = np.empty(len(X))
+    for p in range(len(X)):
+        x = X[p]
+        m1 = np.zeros_like(x)
+        m2 = np.zeros_like(x)
+        for it in range(1, steps + 1):
+            _, g = mc_hvi_value_grad(fp, x, eps)
+            m1 = 0.9 * m1 + 0.1 * g
+            m2 = 0.999 * m2 + 0.001 * g * g
+            step = lr * (m1 / (1 - 0.9 ** it)) / (np.sqrt(m2 / (1 - 0.999 ** it)) + 1e-8)
+            x = np.clip(x + step, lower, upper)
+        X[p] = x
+        out[p] = mc_hvi_value_grad(fp, x, eps)[0]
+    return X, out
