@@ -310,6 +310,28 @@ int boute_acq_nehvi2d(const float *mean, const float *cvar, const float *shift, 
                       const float *strips, const int *counts, int n, const double *cons,
                       float *acq, void *stream);
 
+/* Optimising the acquisition over the decision space (Sec. 5.2 step (ii):
+ * the acquisition is optimised to pick the next configuration; BoTorch does
+ * it by gradient ascent from the best of many raw samples). Two objectives,
+ * the Matern-5/2 kernel, the fitted handle `gp` (B problems); the
+ * acquisition is the sample-average Monte-Carlo hypervolume improvement over
+ * the observed front with base normals eps shared by every point,
+ *   A(x) = (1/S) sum_s HVI(mean(x) + sd(x) eps_s),
+ * differentiated through the posterior (k*, W = L^-1 and alpha of the fit).
+ * From each starting point, `steps` steps of projected Adam ascent (beta1
+ * 0.9, beta2 0.999, eps 1e-8, step size lr), every iterate clamped to
+ * [xlo, xhi]; then the value and gradient at the final point.
+ *   lower, upper, K, box_cap: boute_box_decompose's output for the front;
+ *   eps: 2 x S fp32 (objective-major); X0: B x P x d fp32 starting points;
+ *   xlo, xhi: d fp32 bounds; X: B x P x d fp32 final points; acq: B x P fp32
+ *   their acquisition values; grad: B x P x d fp32 gradients there, or NULL.
+ * steps = 0 evaluates the acquisition and its gradient at X0. Other kernels
+ * or m != 2: BOUTE_ERR_UNSUPPORTED. */
+int boute_acq_optimize(const boute_gp *gp, const float *lower, const float *upper, const int *K,
+                       int box_cap, const float *eps, int S, const float *X0, int P,
+                       const float *xlo, const float *xhi, int steps, float lr, float *X,
+                       float *acq, float *grad, void *stream);
+
 /* Failure detection: every device-side wait of the library is bounded (about
  * 2 s) and a wait that runs out records BOUTE_ERR_TIMEOUT in the call's
  * status instead of hanging. This self-test runs one such bounded wait on

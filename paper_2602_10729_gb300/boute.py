@@ -25,7 +25,7 @@ SYMBOLS = (
     "boute_gp_fit", "boute_gp_status", "boute_gp_free", "boute_gp_posterior",
     "boute_gp_set_precision", "boute_gp_posterior_fp64",
     "boute_gp_set_insample", "boute_gp_insample", "boute_gp_posterior_joint",
-    "boute_insample_fronts", "boute_acq_nehvi2d", "boute_bounds_report",
+    "boute_insample_fronts", "boute_acq_nehvi2d", "boute_bounds_report", "boute_acq_optimize",
     "boute_pareto_front", "boute_box_decompose", "boute_acq_ehvi", "boute_acq_mc_hvi",
     "boute_select_topk", "boute_select_topk_noalloc", "boute_engine_create", "boute_engine_step",
     "boute_engine_step_async",
@@ -88,6 +88,8 @@ def load(path: str | None = None):
         "boute_gp_posterior": ([_vp, _vp, _ll, _vp, _vp, _vp], _i),
         "boute_gp_set_insample": ([_vp, _i], _i),
         "boute_bounds_report": ([_vp], _i),
+        "boute_acq_optimize": ([_vp, _vp, _vp, _vp, _i, _vp, _i, _vp, _i, _vp, _vp, _i,
+                                ctypes.c_float, _vp, _vp, _vp, _vp], _i),
         "boute_gp_insample": ([_vp, _vp, _vp, _vp, _vp, _vp, _vp], _i),
         "boute_gp_posterior_joint": ([_vp, _vp, _ll, _vp, _vp, _vp, _vp], _i),
         "boute_insample_fronts": ([_vp, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
@@ -324,6 +326,18 @@ def boute_engine_set_n(e: Engine, n: int):
     """Later steps use n <= the engine's creation n observations."""
     _check(load().boute_engine_set_n(e.handle, int(n)), "boute_engine_set_n")
     e.n = int(n)
+
+
+def boute_acq_optimize(gp: Gp, lower, upper, K, box_cap, eps, S, X0, P, xlo, xhi, steps, lr, X,
+                       acq, grad=None, stream=None):
+    """Projected Adam ascent on the 2-objective sample-average MC acquisition
+    (CUDA tensors: X0, X B x P x d; acq B x P; grad B x P x d or None)."""
+    f32 = torch.float32
+    _check(load().boute_acq_optimize(gp.handle, _p(lower, f32), _p(upper, f32),
+                                     _p(K, torch.int32), int(box_cap), _p(eps, f32), int(S),
+                                     _p(X0, f32), int(P), _p(xlo, f32), _p(xhi, f32), int(steps),
+                                     float(lr), _p(X, f32), _p(acq, f32), _p(grad, f32),
+                                     _s(stream)), "boute_acq_optimize")
 
 
 def boute_bounds_report():

@@ -1102,6 +1102,18 @@ int boute_engine_set_kernel(boute_engine *e, int d_tau, const double *params) {
   return r;
 }
 
+int boute_acq_optimize(const boute_gp *gp, const float *lower, const float *upper, const int *K,
+                       int box_cap, const float *eps, int S, const float *X0, int P,
+                       const float *xlo, const float *xhi, int steps, float lr, float *X,
+                       float *acq, float *grad, void *stream) {
+  BOUTE_TRACE();
+  if (!gp || !lower || !upper || !K || !eps || !X0 || !xlo || !xhi || !X || !acq || box_cap < 1 ||
+      S < 1 || P < 1 || steps < 0 || !(lr > 0.f) || P > 65535)
+    return BOUTE_ERR_INVALID_ARG;
+  return launch_acq_optimize(&gp->g, lower, upper, K, box_cap, eps, S, X0, P, xlo, xhi, steps, lr,
+                             X, acq, grad, (cudaStream_t)stream);
+}
+
 int boute_bounds_report(long long *rec) {
   BOUTE_TRACE();
   if (!rec) return BOUTE_ERR_INVALID_ARG;

@@ -861,7 +861,8 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   // global variant leaves W in the workspace for pack_kernel), alpha into the
   // side input
   if (SMEM) pack_rows(NP - 32, NP, warp, nw);  // the last block row (the others: above)
-  if (SMEM && Wkeep) {  // W for the in-sample preparation (its lower triangle)
+  if (SMEM && Wkeep) {  // W in global memory too (the in-sample preparation, the
+                        // acquisition's gradient), its lower triangle
     float *dst = Wkeep + (size_t)bt * NP * ld;
     for (int i = warp; i < n; i += nw)
       for (int k = lane; k <= i; k += 32) dst[(size_t)i * ld + k] = W[(size_t)i * ld + k];
@@ -1235,7 +1236,7 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
       launch_pdl(fit32_kernel<true>, dim3(BM), dim3(fit_threads<true>()), smem, s, gp->Kh,
                  gp->Kl, Ys, standardize, n, m, gp->Aws, gp->Wws, gp->xt, gp->DP, npad, gp->plan,
                  gp->bop, fit_kl_in_smem(n) ? 1 : 0, fit_early, gp->kern, gp->status,
-                 (const int *)nullptr, gp->plan.S_in > 0 ? gp->Wws : nullptr);
+                 (const int *)nullptr, gp->Wws);  // W kept in global memory as well
       count_launch(2);
     } else {  // one block per problem-objective on the global workspace
       launch_pdl(fit32_kernel<false>, dim3(BM), dim3(fit_threads<false>()),

@@ -112,6 +112,12 @@ int launch_insample_fronts(const float *Yin, int B, int n, int S, const double *
 int launch_nehvi2(const float *mean, const float *cvar, const float *shift, int B, long long N,
                   int S, const float *eps, long long eps_stride, const float *strips,
                   const int *counts, int n, const double *cons, float *acq, cudaStream_t s);
+// Projected Adam ascent on the 2-objective sample-average MC acquisition
+// from P starting points per problem (acqopt.cu).
+int launch_acq_optimize(const Gp *gp, const float *lower, const float *upper, const int *K,
+                        int box_cap, const float *eps, int S, const float *X0, int P,
+                        const float *xlo, const float *xhi, int steps, float lr, float *X,
+                        float *acq, float *grad, cudaStream_t s);
 // The posterior with the in-sample blocks: mean, the conditional variance
 // (cvar) and the shifts (B x m x S_in x N); shift null: the plain posterior
 // (W's blocks only) on a handle with in-sample draws.
