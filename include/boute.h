@@ -508,6 +508,14 @@ int boute_engine_set_normals(boute_engine *e, unsigned long long seed);
  * unchanged), BOUTE_ERR_OOM / BOUTE_ERR_CUDA (the engine stays usable at
  * n, selecting with the separate top-k kernel). */
 int boute_engine_set_n(boute_engine *e, int n);
+/* The acquisition optimised over the decision space from the engine's last
+ * step (Sec. 5.2 step (ii)): boute_acq_optimize on the engine's fit and the
+ * observed front of that step (mode BOUTE_ACQ_MC_HVI, m = 2, the Matern-5/2
+ * kernel; otherwise BOUTE_ERR_UNSUPPORTED). Arguments as for
+ * boute_acq_optimize (device pointers; X0, X B x P x d). */
+int boute_engine_optimize(boute_engine *e, const float *eps, int S, const float *X0, int P,
+                          const float *xlo, const float *xhi, int steps, float lr, float *X,
+                          float *acq, float *grad, void *stream);
 void boute_engine_free(boute_engine *e);
 
 /* ---- the optimisation loop ------------------------------------------------------
@@ -536,13 +544,15 @@ void boute_engine_free(boute_engine *e);
  *   ls (m x d), s2 (m), noise (m): HOST hyperparameters, updated in place
  *      when learning;
  *   X (max_evals x d), Y (max_evals x m): HOST, the first n0 rows given;
- *   sel (out, max_evals - n0): the candidate index chosen per iteration;
+ *   sel (out, max_evals - n0): the candidate index chosen per iteration
+ *      (with refinement: the start whose end point was evaluated);
  *   theta_hist (out, optional, (max_evals - n0) x m x P): the parameters
  *      each iteration scored with (P = d + 2, or d + 5 with the composite
  *      kernel, as for boute_gp_learn / boute_gp_learn_k);
  *   n_out: observations at the end; converged: 1 if the stability test
  *      stopped the loop.
- * Synchronous; allocates its device buffers and one engine per iteration. */
+ * Synchronous; allocates its device buffers and one engine for the whole run
+ * (created for the largest data set, boute_engine_set_n every iteration). */
 typedef int (*boute_objective_fn)(const double *x, int d, double *y, int m, void *user);
 typedef struct {
   int mode;         /* BOUTE_ACQ_EHVI2D or BOUTE_ACQ_MC_HVI */
@@ -552,6 +562,14 @@ typedef struct {
   int learn_iters;  /* Adam steps per iteration; 0 keeps the hyperparameters */
   double learn_lr;  /* Adam step size */
   unsigned long long seed;  /* base normals when eps is NULL (boute_engine_set_normals) */
+  /* optional: the acquisition optimised over the decision space (Sec. 5.2
+   * step (ii)): from the pool's best refine_starts candidates, refine_steps
+   * steps of boute_engine_optimize (step size refine_lr, bounds [0, 1]^d,
+   * shared normals boute_base_normals(seed ^ 0xbb67ae8584caa73b, 1, 1, 2, S));
+   * the loop then evaluates the best end point (mode BOUTE_ACQ_MC_HVI, m = 2,
+   * the Matern-5/2 kernel). refine_steps = 0: the pool's best, as above. */
+  int refine_starts, refine_steps;
+  double refine_lr;
 } boute_mobo_config;
 int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const float *cand, long long N,
                    const float *eps, const double *ref, const int *transforms,

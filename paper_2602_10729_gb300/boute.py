@@ -26,6 +26,7 @@ SYMBOLS = (
     "boute_gp_set_precision", "boute_gp_posterior_fp64",
     "boute_gp_set_insample", "boute_gp_insample", "boute_gp_posterior_joint",
     "boute_insample_fronts", "boute_acq_nehvi2d", "boute_bounds_report", "boute_acq_optimize",
+    "boute_engine_optimize",
     "boute_pareto_front", "boute_box_decompose", "boute_acq_ehvi", "boute_acq_mc_hvi",
     "boute_select_topk", "boute_select_topk_noalloc", "boute_engine_create", "boute_engine_step",
     "boute_engine_step_async",
@@ -50,7 +51,9 @@ class MoboConfig(ctypes.Structure):
     """boute_mobo_config."""
     _fields_ = [("mode", ctypes.c_int), ("S", ctypes.c_int), ("max_evals", ctypes.c_int),
                 ("patience", ctypes.c_int), ("learn_iters", ctypes.c_int),
-                ("learn_lr", ctypes.c_double), ("seed", ctypes.c_ulonglong)]
+                ("learn_lr", ctypes.c_double), ("seed", ctypes.c_ulonglong),
+                ("refine_starts", ctypes.c_int), ("refine_steps", ctypes.c_int),
+                ("refine_lr", ctypes.c_double)]
 
 
 #: boute_objective_fn
@@ -88,6 +91,8 @@ def load(path: str | None = None):
         "boute_gp_posterior": ([_vp, _vp, _ll, _vp, _vp, _vp], _i),
         "boute_gp_set_insample": ([_vp, _i], _i),
         "boute_bounds_report": ([_vp], _i),
+        "boute_engine_optimize": ([_vp, _vp, _i, _vp, _i, _vp, _vp, _i, ctypes.c_float, _vp, _vp,
+                                   _vp, _vp], _i),
         "boute_acq_optimize": ([_vp, _vp, _vp, _vp, _i, _vp, _i, _vp, _i, _vp, _vp, _i,
                                 ctypes.c_float, _vp, _vp, _vp, _vp], _i),
         "boute_gp_insample": ([_vp, _vp, _vp, _vp, _vp, _vp, _vp], _i),
@@ -242,7 +247,8 @@ def boute_gp_learn(X, Ys, theta0, iters: int, lr: float, theta, mll, grad=None, 
 
 def boute_mobo_run(objective, cand, ref, ls, s2, noise, X0, Y0, *, mode=BOUTE_ACQ_EHVI2D, S=0,
                    eps=None, max_evals=50, patience=20, learn_iters=0, learn_lr=0.05,
-                   transforms=None, cons=None, d_tau=0, kc=None, seed=0):
+                   transforms=None, cons=None, d_tau=0, kc=None, seed=0, refine_starts=0,
+                   refine_steps=0, refine_lr=0.01):
     """The optimisation loop. objective(x: (d,) float64 array) -> m outcomes.
     cand: N x d; eps: N x m x S (mode MC); ls: m x d, s2, noise: m (initial
     hyperparameters); X0 / Y0: the first observations. Returns a dict with X,
@@ -283,7 +289,8 @@ def boute_mobo_run(objective, cand, ref, ls, s2, noise, X0, Y0, *, mode=BOUTE_AC
             return 1
 
     fn = ObjectiveFn(cb)
-    cfg = MoboConfig(mode, S, max_evals, patience, learn_iters, learn_lr, int(seed))
+    cfg = MoboConfig(mode, S, max_evals, patience, learn_iters, learn_lr, int(seed),
+                     int(refine_starts), int(refine_steps), float(refine_lr))
     n_out, conv = ctypes.c_int(0), ctypes.c_int(0)
     a = lambda v: None if v is None else v.ctypes.data
     rc = load().boute_mobo_run(ctypes.byref(cfg), d, m, a(cand), N, a(eps), a(ref), a(tf), a(cs),
@@ -338,6 +345,16 @@ def boute_acq_optimize(gp: Gp, lower, upper, K, box_cap, eps, S, X0, P, xlo, xhi
                                      _p(X0, f32), int(P), _p(xlo, f32), _p(xhi, f32), int(steps),
                                      float(lr), _p(X, f32), _p(acq, f32), _p(grad, f32),
                                      _s(stream)), "boute_acq_optimize")
+
+
+def boute_engine_optimize(e: Engine, eps, S, X0, P, xlo, xhi, steps, lr, X, acq, grad=None,
+                          stream=None):
+    """boute_acq_optimize on the engine's last step (fit and observed front)."""
+    f32 = torch.float32
+    _check(load().boute_engine_optimize(e.handle, _p(eps, f32), int(S), _p(X0, f32), int(P),
+                                        _p(xlo, f32), _p(xhi, f32), int(steps), float(lr),
+                                        _p(X, f32), _p(acq, f32), _p(grad, f32), _s(stream)),
+           "boute_engine_optimize")
 
 
 def boute_bounds_report():

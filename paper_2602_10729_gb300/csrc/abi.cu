@@ -1059,6 +1059,16 @@ static int gp_set_n(Gp &g, int n) {
   return BOUTE_OK;
 }
 
+int boute_engine_optimize(boute_engine *e, const float *eps, int S, const float *X0, int P,
+                          const float *xlo, const float *xhi, int steps, float lr, float *X,
+                          float *acq, float *grad, void *stream) {
+  BOUTE_TRACE();
+  if (!e) return BOUTE_ERR_INVALID_ARG;
+  if (e->mode != BOUTE_ACQ_MC_HVI || e->m != 2) return BOUTE_ERR_UNSUPPORTED;
+  return boute_acq_optimize(e->gp, e->lower, e->upper, e->K, 2 * e->n + 2, eps, S, X0, P, xlo,
+                            xhi, steps, lr, X, acq, grad, stream);
+}
+
 int boute_engine_set_n(boute_engine *e, int n) {
   BOUTE_TRACE();
   if (!e || n < 1 || n > e->ncap) return BOUTE_ERR_INVALID_ARG;

@@ -82,6 +82,13 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
     return BOUTE_ERR_INVALID_ARG;
   if (cfg->mode != BOUTE_ACQ_EHVI2D && cfg->S < 1) return BOUTE_ERR_INVALID_ARG;
   if (kc && (d_tau < 0 || d_tau > d)) return BOUTE_ERR_INVALID_ARG;
+  // refinement of the pool's best by gradient ascent (optional)
+  const bool refine = cfg->refine_steps > 0;
+  if (refine && (cfg->refine_starts < 1 || cfg->refine_starts > 1024 ||
+                 (long long)cfg->refine_starts > N || !(cfg->refine_lr > 0.0)))
+    return BOUTE_ERR_INVALID_ARG;
+  if (refine && (cfg->mode != BOUTE_ACQ_MC_HVI || m != 2 || kc)) return BOUTE_ERR_UNSUPPORTED;
+  const int KS = refine ? cfg->refine_starts : 1;  // candidates selected per iteration
   // the composite kernel (kc: m x (3 + dc) [s2_c, s2_x, beta, s...]) adds
   // (log s2_c, log s2_x, beta) to the learned parameters
   const int dc = d - d_tau, KC = 3 + dc;
@@ -108,8 +115,23 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
   if (kc) r |= dmalloc(&dpref, (size_t)m * dc);
   r |= dmalloc(&dXc, (size_t)N * d);
   if (S && eps) r |= dmalloc(&deps, (size_t)N * m * S);
-  r |= dmalloc(&didx, 1);
-  r |= dmalloc(&dval, 1);
+  r |= dmalloc(&didx, (size_t)KS);
+  r |= dmalloc(&dval, (size_t)KS);
+  // refinement: start and end points, their values, shared normals, bounds
+  float *dX0 = nullptr, *dXo = nullptr, *dacq = nullptr, *deps_r = nullptr, *dlo = nullptr,
+        *dhi = nullptr;
+  if (refine) {
+    r |= dmalloc(&dX0, (size_t)KS * d);
+    r |= dmalloc(&dXo, (size_t)KS * d);
+    r |= dmalloc(&dacq, (size_t)KS);
+    r |= dmalloc(&deps_r, (size_t)2 * S);
+    r |= dmalloc(&dlo, (size_t)d);
+    r |= dmalloc(&dhi, (size_t)d);
+    if (!r) r = boute_base_normals(cfg->seed ^ 0xbb67ae8584caa73bull, 1, 1, 2, S, deps_r, nullptr);
+    std::vector<float> zo((size_t)d, 0.f), on((size_t)d, 1.f);
+    if (!r) r = copy_in(dlo, zo.data(), sizeof(float) * d);
+    if (!r) r = copy_in(dhi, on.data(), sizeof(float) * d);
+  }
   if (!r) r = copy_in(dXc, cand, sizeof(float) * N * d);
   if (!r && S && eps) r = copy_in(deps, eps, sizeof(float) * N * m * S);
   if (!r) r = copy_in(dref, ref, sizeof(double) * m);
@@ -122,7 +144,7 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
   // one engine for the whole loop, sized for its largest data set (n grows
   // by one per iteration up to nmax - 1 before the last selection)
   boute_engine *e = nullptr;
-  if (!r && n0 < nmax) r = boute_engine_create(1, nmax - 1, d, m, N, cfg->mode, S, 1, &e);
+  if (!r && n0 < nmax) r = boute_engine_create(1, nmax - 1, d, m, N, cfg->mode, S, KS, &e);
   if (!r && transforms) r = boute_engine_set_outcome_transforms(e, transforms);
   if (!r && cons) r = boute_engine_set_constraints(e, cons);
   if (!r && S && !eps) r = boute_engine_set_normals(e, cfg->seed);  // eps null: own normals
@@ -179,13 +201,35 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
     if (!r) r = boute_engine_set_n(e, n);
     if (!r && kc) r = boute_engine_set_kernel(e, d_tau, kc);
     if (!r) r = boute_engine_step(e, dX, dY, dls, ds2, dnz, dref, dXc, deps, didx, dval, nullptr);
-    long long pick = -1;
-    if (!r && cudaMemcpy(&pick, didx, sizeof(pick), cudaMemcpyDeviceToHost) != cudaSuccess)
+    std::vector<long long> picks((size_t)KS, -1);
+    if (!r && cudaMemcpy(picks.data(), didx, sizeof(long long) * KS, cudaMemcpyDeviceToHost) !=
+                  cudaSuccess)
       r = BOUTE_ERR_CUDA;
     if (r) break;
-    // (iii) evaluate it and add the observation
+    long long pick = picks[0];
     double *xn = X + (size_t)n * d, *yn = Y + (size_t)n * m;
     for (int q = 0; q < d; ++q) xn[q] = (double)cand[(size_t)pick * d + q];
+    if (refine) {  // gradient ascent from the pool's best KS; the best end point
+      std::vector<float> x0((size_t)KS * d), xo((size_t)KS * d), ao((size_t)KS);
+      for (int p = 0; p < KS; ++p)
+        for (int q = 0; q < d; ++q) x0[(size_t)p * d + q] = cand[(size_t)picks[p] * d + q];
+      r = copy_in(dX0, x0.data(), sizeof(float) * KS * d);
+      if (!r)
+        r = boute_engine_optimize(e, deps_r, S, dX0, KS, dlo, dhi, cfg->refine_steps,
+                                  (float)cfg->refine_lr, dXo, dacq, nullptr, nullptr);
+      if (!r && (cudaMemcpy(xo.data(), dXo, sizeof(float) * KS * d, cudaMemcpyDeviceToHost) !=
+                     cudaSuccess ||
+                 cudaMemcpy(ao.data(), dacq, sizeof(float) * KS, cudaMemcpyDeviceToHost) !=
+                     cudaSuccess))
+        r = BOUTE_ERR_CUDA;
+      if (r) break;
+      int best = 0;
+      for (int p = 1; p < KS; ++p)
+        if (ao[p] > ao[best]) best = p;
+      pick = picks[best];
+      for (int q = 0; q < d; ++q) xn[q] = (double)xo[(size_t)best * d + q];
+    }
+    // (iii) evaluate it and add the observation
     if (f(xn, d, yn, m, user) != 0) {
       r = BOUTE_ERR_INVALID_ARG;
       break;
@@ -203,7 +247,8 @@ extern "C" int boute_mobo_run(const boute_mobo_config *cfg, int d, int m, const 
   }
   *n_out = n;
   boute_engine_free(e);
-  void *bufs[] = {dX, dY, dYs, dls, ds2, dnz, dref, dth0, dth, dmll, dXc, deps, didx, dval, dpref};
+  void *bufs[] = {dX,   dY,  dYs,  dls, ds2,  dnz,  dref,   dth0, dth, dmll,
+                  dXc,  deps, didx, dval, dpref, dX0, dXo, dacq, deps_r, dlo, dhi};
   for (void *p : bufs) cudaFree(p);
   return r;
 }

@@ -148,3 +148,41 @@ def test_objective_errors_stop_the_loop():
     with pytest.raises(ValueError):
         bt.boute_mobo_run(bad, cand, [1.1, 1.1], np.full((2, 3), 0.4), np.ones(2),
                           np.full(2, 1e-4), X0, Y0, max_evals=8, patience=3)
+
+
+def test_loop_with_gradient_refinement():
+    """Sec. 5.2 step (ii) with the acquisition optimised over the decision
+    space: each iteration ascends from the pool's best candidates and
+    evaluates the best end point. Against the oracle on the same
+    observations: the end point's sample-average acquisition (the loop's
+    shared normals, regenerated here) is at least its start's and matches the
+    oracle's own ascent from that start."""
+    from paper_2602_10729_gb300 import boute as bt
+    rng = np.random.default_rng(13)
+    d, N, n0, S = 3, 1024, 6, 32
+    cand = rng.random((N, d)).astype(np.float32)
+    X0 = cand[:n0].astype(np.float64)
+    Y0 = np.stack([_objective(x) for x in X0])
+    ls0 = np.full((2, d), 0.4)
+    s2, noise = np.ones(2), np.full(2, 1e-4)
+    seed, starts, steps, lr = 17, 4, 25, 0.02
+    max_evals = n0 + 6
+    res = bt.boute_mobo_run(_objective, cand, [1.1, 1.1], ls0, s2, noise, X0, Y0,
+                            mode=bt.BOUTE_ACQ_MC_HVI, S=S, seed=seed, max_evals=max_evals,
+                            patience=100, refine_starts=starts, refine_steps=steps, refine_lr=lr)
+    X, Y, sel = res["X"], res["Y"], res["sel"]
+    assert len(sel) == max_evals - n0
+    er = oracle.base_normals(seed ^ 0xbb67ae8584caa73b, 1, 1, 2, S)[0, 0].astype(np.float64)
+    for t, p in enumerate(sel):
+        nt = n0 + t
+        x = X[nt]
+        assert (x >= 0).all() and (x <= 1).all()
+        np.testing.assert_array_equal(Y[nt], _objective(x))
+        fp = opl.fit_problem(X[:nt], Y[:nt], ls0, s2, noise, np.array([1.1, 1.1]))
+        a_end = opl.mc_hvi_value_grad(fp, x, er)[0]
+        a_start = opl.mc_hvi_value_grad(fp, cand[p].astype(np.float64), er)[0]
+        _, ao = opl.optimize_acq(fp, cand[p][None].astype(np.float64), er, np.zeros(d),
+                                 np.ones(d), steps, lr)
+        scale = max(abs(ao[0]), abs(a_start), 1e-12)
+        assert a_end >= a_start - 1e-5 * scale, (t, a_end, a_start)
+        assert abs(a_end - ao[0]) <= 1e-3 * scale, (t, a_end, ao[0])
