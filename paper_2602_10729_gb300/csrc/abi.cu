@@ -225,6 +225,8 @@ int boute_gp_create(int B, int n, int d, int m, boute_gp **out) {
   r |= dalloc(&g.s2f, BM);
   r |= dalloc(&g.status, 1);
   r |= dalloc(&g.fbad, BM);
+  if (const size_t tp = fit_tpart_floats((int)np, (int)BM)) r |= dalloc(&g.tpart, tp);
+  if (const size_t fv = fit_fvec_floats((int)np, (int)BM)) r |= dalloc(&g.fvec, fv);
   if (r != BOUTE_OK) {
     boute_gp_free(h);
     return BOUTE_ERR_OOM;
@@ -397,6 +399,7 @@ void boute_gp_free(boute_gp *gp) {
   Gp &g = gp->g;
   cudaFree(g.Kh); cudaFree(g.Kl); cudaFree(g.Aws); cudaFree(g.Wws); cudaFree(g.bop); cudaFree(g.xt);
   cudaFree(g.s2f); cudaFree(g.status); cudaFree(g.kpar); cudaFree(g.kcache); cudaFree(g.fbad);
+  cudaFree(g.tpart); cudaFree(g.fvec);
   cudaFree(g.W64); cudaFree(g.a64); cudaFree(g.xs64); cudaFree(g.ls64); cudaFree(g.s2_64);
   cudaFree(g.gws);
   cudaFree(g.iws);

@@ -265,6 +265,50 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
   e = (a - (s - bb)) + (b - bb);
 }
 
+// The standardisation of one outcome column (stride m) by one warp: with
+// standardize != 0 the column's mean and 1 / (sample standard deviation) (1
+// when that is below 1e-8 or n = 1), as standardize_kernel computes them,
+// else 0 and 1; lane 0 stores them.
+__device__ __forceinline__ void standardize_stats(const double *y, int n, int m, int standardize,
+                                                  int lane, double &mu, double &isd) {
+  if (!standardize) {
+    if (lane == 0) {
+      mu = 0.0;
+      isd = 1.0;
+    }
+    return;
+  }
+  double sum = 0.0;
+  for (int i = lane; i < n; i += 32) sum += y[(size_t)i * m];
+  const double mean = warp_sum(sum) / n;
+  double ss = 0.0;
+  for (int i = lane; i < n; i += 32) {
+    const double z = y[(size_t)i * m] - mean;
+    ss += z * z;
+  }
+  ss = warp_sum(ss);
+  double sd = n > 1 ? sqrt(ss / (n - 1)) : 1.0;
+  if (!(sd >= 1e-8)) sd = 1.0;
+  if (lane == 0) {
+    mu = mean;
+    isd = 1.0 / sd;
+  }
+}
+
+// The largest preference weight w_j of problem-objective bt (composite
+// kernel), by one warp, into its parameter slot.
+__device__ __forceinline__ void composite_wmax(float *xt, int bt, const PostPlan &plan, int DP,
+                                               int n, int lane) {
+  const int cf = xt_chunk_floats(DP);
+  float *x0 = xt + (size_t)bt * plan.nxt * cf;
+  const float *xw = x0 + BOUTE_KCHUNK * DP;
+  float wm = 0.f;
+  for (int j = lane; j < n; j += 32) wm = fmaxf(wm, xw[(size_t)(j / BOUTE_KCHUNK) * cf + j % BOUTE_KCHUNK]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
+  if (lane == 0) x0[xt_param_offset(DP) + 2 * DP + kParWmax] = wm;
+}
+
 // ---- factorisation: one block per (problem, objective) -------------------------
 // Blocked right-looking Cholesky of K (its fp32 rounding) in 32-column panels,
 // with W = L^-1 formed block row by block row inside the same loop: one warp
@@ -308,28 +352,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
   if (early_trigger) pdl_trigger();  // every block is resident: the posterior may launch
   // standardize != 0: Ys holds raw outcomes; this column is standardised here
   // (zero mean, unit sample standard deviation, as standardize_kernel does)
-  if (standardize) {  // warp 0 alone: few fp64 instructions
-    if (warp == 0) {
-      double sum = 0.0;
-      for (int i = lane; i < n; i += 32) sum += y[(size_t)i * m];
-      const double mean = warp_sum(sum) / n;
-      double ss = 0.0;
-      for (int i = lane; i < n; i += 32) {
-        const double z = y[(size_t)i * m] - mean;
-        ss += z * z;
-      }
-      ss = warp_sum(ss);
-      double sd = n > 1 ? sqrt(ss / (n - 1)) : 1.0;
-      if (!(sd >= 1e-8)) sd = 1.0;
-      if (lane == 0) {
-        ymu = mean;
-        yisd = 1.0 / sd;
-      }
-    }
-  } else if (tid == 0) {
-    ymu = 0.0;
-    yisd = 1.0;
-  }
+  if (warp == 0) standardize_stats(y, n, m, standardize, lane, ymu, yisd);  // few fp64 ops
   // everything below reads what the set-up kernel wrote
   pdl_wait();
   // A = K (hi; the lower triangle becomes L, the upper triangle keeps K for the
@@ -874,15 +897,7 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
     q[0] = k < n ? al[k] : 0.f;
     q[BOUTE_KCHUNK] = k < n ? rv[k] : 0.f;
   }
-  if (comp && warp == nw - 1) {  // the largest preference weight w_j (composite kernel)
-    float *x0 = xt + (size_t)bt * plan.nxt * cf;
-    const float *xw = x0 + BOUTE_KCHUNK * DP;
-    float wm = 0.f;
-    for (int j = lane; j < n; j += 32) wm = fmaxf(wm, xw[(size_t)(j / BOUTE_KCHUNK) * cf + j % 32]);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
-    if (lane == 0) x0[xt_param_offset(DP) + 2 * DP + kParWmax] = wm;
-  }
+  if (comp && warp == nw - 1) composite_wmax(xt, bt, plan, DP, n, lane);
 }
 
 // ---- the global-workspace factorisation across many blocks -------------------------
@@ -890,11 +905,12 @@ __global__ void __launch_bounds__(fit_threads<SMEM>(), 1) fit32_kernel(
 // run as three kernels, each over as many blocks as its tiles fill (a grid of
 // x blocks per problem-objective y), with programmatic dependent launch in
 // between: (a) fitb_diag_kernel factors and inverts the diagonal block, (b)
-// fitb_panel_kernel forms the panel below and the partial sums T_pJ, (c)
-// fitb_update_kernel applies the trailing update, forms W's block row and
+// fitb_panel_kernel forms the panel below and the partial sums of T_pJ, (c)
+// fitb_update_kernel applies the trailing update, adds the partials in a fixed
+// order (the result does not depend on the grid), forms W's block row and
 // copies the panel into A. The tiles' arithmetic is the same as in the
-// one-block loop; fit32_kernel then finishes alpha and the outputs from the
-// factored workspace. A non-positive pivot marks the problem-objective in fbad
+// one-block loop; the fitr_* kernels then form alpha from the factored
+// workspace. A non-positive pivot marks the problem-objective in fbad
 // and its later kernels return at once.
 constexpr int kFitbThreads = 256;
 
@@ -994,14 +1010,25 @@ __global__ void __launch_bounds__(64) fitb_diag_kernel(const float *Kh_all, int 
 }
 
 // (b) L_rp = A_rp W_pp^T for the rows below the panel (4 x 4 tiles) into block
-// column p of W, and T_pJ = sum_{K=J}^{p-1} L_pK W_KJ (J < p; 4 x 2 tiles)
-// parked, transposed, in W's upper triangle.
+// column p of W, and the partial sums of T_pJ = sum_{K=J}^{p-1} L_pK W_KJ
+// (J < p) into the workspace tpart: T_pJ's K range is split into chunks of
+// kFitbChunk blocks, one work item each, so that no item runs more than
+// kFitbChunk tile steps and the panel's critical path stays short for every p.
+// tpart holds, per problem-objective, nbw x ncw tiles of 32 x 32 floats (J,
+// chunk), nbw = NP / 32 and ncw = ceil(nbw / kFitbChunk).
+constexpr int kFitbChunk = 4;
+__host__ __device__ __forceinline__ int fitb_t_items(int p) {
+  int t = 0;
+  for (int J = 0; J < p; ++J) t += (p - J + kFitbChunk - 1) / kFitbChunk;
+  return t;
+}
+
 __global__ void __launch_bounds__(kFitbThreads) fitb_panel_kernel(int NP, const float *Aws,
                                                                   float *Wws, int p,
-                                                                  const int *fbad) {
-  // T_pJ's tiles of the panel's block row and of W: L_pK (32 x 32) and
-  // W_KJ for the block's two J (row stride 33)
-  __shared__ float Ls[32][33], Ws[2][32][33];
+                                                                  const int *fbad, float *tpart) {
+  // T_pJ's tiles of the panel's block row and of W: L_pK and W_KJ (32 x 32,
+  // row stride 33)
+  __shared__ float Ls[32][33], Ws[32][33];
   pdl_wait();
   pdl_trigger();
   const int bt = blockIdx.y, ld = NP + 1, tid = threadIdx.x;
@@ -1010,9 +1037,10 @@ __global__ void __launch_bounds__(kFitbThreads) fitb_panel_kernel(int NP, const 
   float *W = Wws + (size_t)bt * NP * ld;
   const int p0 = 32 * p, r0 = p0 + 32, rows = NP - r0;
   // work items: blocks of the panel below (4 x 4 tiles, 256 threads each),
-  // then one item per pair of W's block columns J of T_pJ
+  // then one item per (J, chunk) of T_pJ
   const int ntr = (rows / 4) * 8, nbr = (ntr + kFitbThreads - 1) / kFitbThreads;
-  const int items = nbr + (p + 1) / 2;
+  const int nbw = NP / 32, ncw = (nbw + kFitbChunk - 1) / kFitbChunk;  // the partials' layout
+  const int items = nbr + fitb_t_items(p);
   for (int item = blockIdx.x; item < items; item += gridDim.x) {
     if (item < nbr) {
       const int tix = item * kFitbThreads + tid;
@@ -1038,42 +1066,41 @@ __global__ void __launch_bounds__(kFitbThreads) fitb_panel_kernel(int NP, const 
         for (int v = 0; v < 4; ++v) W[(size_t)(i0 + u) * ld + p0 + c0 + v] = acc[u][v];
       continue;
     }
-    // T_pJ = sum_{K=J}^{p-1} L_pK W_KJ for J = J0 (threads 0..127) and J0 + 1
-    // (128..255), 4 x 2 outputs per thread, K block by K block (W_KJ = 0 for
-    // K < J, and W's upper triangle holds other data, so each J starts at K = J)
-    const int J0 = 2 * (item - nbr), half = tid >> 7, e = tid & 127;
-    const int J = J0 + half, rb = 4 * (e >> 4), cb = 2 * (e & 15);
-    float acc[4][2] = {};
-    for (int K = J0; K < p; ++K) {
+    // a partial sum of T_pJ = sum_{K=J}^{p-1} L_pK W_KJ over the chunk
+    // [J + c kFitbChunk, min(J + (c + 1) kFitbChunk, p)) of K blocks, for the
+    // item's (J, c); 2 x 2 outputs per thread; the update kernel adds a J's
+    // partials in chunk order
+    int J = 0, rest = item - nbr;
+    while (rest >= (p - J + kFitbChunk - 1) / kFitbChunk) {
+      rest -= (p - J + kFitbChunk - 1) / kFitbChunk;
+      ++J;
+    }
+    const int c = rest, Kb = J + c * kFitbChunk, Ke = min(Kb + kFitbChunk, p);
+    const int rb = 2 * (tid >> 4), cb = 2 * (tid & 15);
+    float acc[2][2] = {};
+    for (int K = Kb; K < Ke; ++K) {
       __syncthreads();  // the previous K's tiles are consumed
       for (int x = tid; x < 32 * 32; x += kFitbThreads) {
-        const int r = x >> 5, c = x & 31;
-        Ls[r][c] = A[(size_t)(p0 + r) * ld + 32 * K + c];
-        Ws[0][r][c] = W[(size_t)(32 * K + r) * ld + 32 * J0 + c];
-        Ws[1][r][c] = J0 + 1 < p ? W[(size_t)(32 * K + r) * ld + 32 * (J0 + 1) + c] : 0.f;
+        const int r = x >> 5, cc = x & 31;
+        Ls[r][cc] = A[(size_t)(p0 + r) * ld + 32 * K + cc];
+        Ws[r][cc] = W[(size_t)(32 * K + r) * ld + 32 * J + cc];
       }
       __syncthreads();
-      if (K >= J && J < p) {
 #pragma unroll 8
-        for (int q = 0; q < 32; ++q) {
-          float xv[4], yv[2];
-#pragma unroll
-          for (int u = 0; u < 4; ++u) xv[u] = Ls[rb + u][q];
-#pragma unroll
-          for (int v = 0; v < 2; ++v) yv[v] = Ws[half][q][cb + v];
-#pragma unroll
-          for (int u = 0; u < 4; ++u)
-#pragma unroll
-            for (int v = 0; v < 2; ++v) acc[u][v] = fmaf(xv[u], yv[v], acc[u][v]);
-        }
+      for (int q = 0; q < 32; ++q) {
+        const float x0 = Ls[rb][q], x1 = Ls[rb + 1][q];
+        const float y0 = Ws[q][cb], y1 = Ws[q][cb + 1];
+        acc[0][0] = fmaf(x0, y0, acc[0][0]);
+        acc[0][1] = fmaf(x0, y1, acc[0][1]);
+        acc[1][0] = fmaf(x1, y0, acc[1][0]);
+        acc[1][1] = fmaf(x1, y1, acc[1][1]);
       }
     }
-    if (J < p) {
+    float *tp = tpart + (((size_t)bt * nbw + J) * ncw + c) * 1024;
 #pragma unroll
-      for (int u = 0; u < 4; ++u)
+    for (int u = 0; u < 2; ++u)
 #pragma unroll
-        for (int v = 0; v < 2; ++v) W[(size_t)(32 * J + cb + v) * ld + p0 + rb + u] = acc[u][v];
-    }
+      for (int v = 0; v < 2; ++v) tp[(rb + u) * 32 + cb + v] = acc[u][v];
     __syncthreads();  // before the next item reuses the tiles
   }
 }
@@ -1083,7 +1110,8 @@ __global__ void __launch_bounds__(kFitbThreads) fitb_panel_kernel(int NP, const 
 // panel (block column p of W, rows below it) copied into A.
 __global__ void __launch_bounds__(kFitbThreads) fitb_update_kernel(int NP, float *Aws,
                                                                    float *Wws, int p,
-                                                                   const int *fbad) {
+                                                                   const int *fbad,
+                                                                   const float *tpart) {
   pdl_wait();
   pdl_trigger();
   const int bt = blockIdx.y, ld = NP + 1;
@@ -1127,13 +1155,20 @@ __global__ void __launch_bounds__(kFitbThreads) fitb_update_kernel(int NP, float
           if (ti != tj || v <= u) A[(size_t)(i0 + u) * ld + j0 + v] -= acc[u][v];
     } else {
       const int e = tix - ntile, J = e >> 7, rb = 4 * ((e >> 4) & 7), cb = 2 * (e & 15);
+      const int nbw = NP / 32, ncw = (nbw + kFitbChunk - 1) / kFitbChunk;
+      const int nc = (p - J + kFitbChunk - 1) / kFitbChunk;  // this J's partials
+      const float *tp = tpart + ((size_t)bt * nbw + J) * ncw * 1024;
 #pragma unroll 4
       for (int q = 0; q < 32; ++q) {
         float x[4], y2[2];
 #pragma unroll
         for (int u = 0; u < 4; ++u) x[u] = W[(size_t)(p0 + rb + u) * ld + p0 + q];
 #pragma unroll
-        for (int v = 0; v < 2; ++v) y2[v] = W[(size_t)(32 * J + cb + v) * ld + p0 + q];
+        for (int v = 0; v < 2; ++v) {  // T_pJ(q, cb + v): the partials in chunk order
+          float t = 0.f;
+          for (int c = 0; c < nc; ++c) t += tp[(size_t)c * 1024 + q * 32 + cb + v];
+          y2[v] = t;
+        }
 #pragma unroll
         for (int u = 0; u < 4; ++u)
 #pragma unroll
@@ -1145,6 +1180,182 @@ __global__ void __launch_bounds__(kFitbThreads) fitb_update_kernel(int NP, float
         for (int v = 0; v < 2; ++v) W[(size_t)(p0 + rb + u) * ld + 32 * J + cb + v] = -acc[u][v];
     }
   }
+}
+
+// ---- alpha on the blocked path, across many blocks -----------------------------
+// After the blocked factorisation, fit32_kernel's alpha (alpha0 = W^T (W y),
+// then two refinement steps against K = hi + lo with double-float residuals,
+// the second correction kept as alpha's lo part) runs as a chain of kernels,
+// each spread over many blocks per problem-objective (a grid of x blocks per
+// problem-objective y): fitr_init_kernel (the standardised y, the output
+// padding), then per solve fitr_wx_kernel (t = W rhs, a warp per row) and
+// fitr_wtx_kernel (W^T t, 32 columns per block, the rows split over its warps
+// and added in a fixed order), and fitr_resid_kernel (r = y - K alpha, a half
+// warp per row) between the solves. The vectors live in the workspace fvec,
+// kFitrVecs x NP floats per problem-objective.
+enum { kVy = 0, kVylo = 1, kVal = 2, kVlo = 3, kVt = 4, kVr = 5, kFitrVecs = 6 };
+
+__global__ void __launch_bounds__(256) fitr_init_kernel(const double *Ys, int standardize, int n,
+                                                        int m, int NP, float *fvec, float *xt,
+                                                        int DP, PostPlan plan, int comp,
+                                                        int *status, const int *fbad) {
+  __shared__ double ymu, yisd;
+  pdl_wait();
+  pdl_trigger();
+  const int bt = blockIdx.x, b = bt / m, t = bt % m, tid = threadIdx.x, lane = tid & 31;
+  if (fbad[bt]) {
+    if (tid == 0) set_status(status, BOUTE_ERR_NOT_PD);
+    return;
+  }
+  const double *y = Ys + (size_t)b * n * m + t;
+  if (tid < 32) standardize_stats(y, n, m, standardize, lane, ymu, yisd);
+  __syncthreads();
+  float *v = fvec + (size_t)bt * kFitrVecs * NP;
+  for (int i = tid; i < NP; i += blockDim.x) {  // standardised y as an fp32 pair
+    const double ys = i < n ? (y[(size_t)i * m] - ymu) * yisd : 0.0;
+    const float hi = (float)ys;
+    BOUTE_INB(i, NP);
+    v[kVy * NP + i] = hi;
+    v[kVylo * NP + i] = (float)(ys - (double)hi);
+  }
+  const int cf = xt_chunk_floats(DP);
+  float *xa = xt + (size_t)bt * plan.nxt * cf + xt_alpha_offset(DP);
+  for (int k = n + tid; k < BOUTE_KCHUNK * plan.nxt; k += blockDim.x) {  // alpha's padding
+    float *q = xa + (size_t)(k / BOUTE_KCHUNK) * cf + k % BOUTE_KCHUNK;
+    q[0] = 0.f;
+    q[BOUTE_KCHUNK] = 0.f;
+  }
+  if (comp && tid < 32) composite_wmax(xt, bt, plan, DP, n, lane);
+}
+
+// t = W rhs (W lower triangular): a warp per row, two accumulators per lane,
+// the lanes combined by shuffles in a fixed order.
+__global__ void __launch_bounds__(256) fitr_wx_kernel(int NP, const float *Wws, float *fvec,
+                                                      int src, const int *fbad) {
+  pdl_wait();
+  pdl_trigger();
+  const int bt = blockIdx.y, ld = NP + 1, lane = threadIdx.x & 31;
+  if (fbad[bt]) return;
+  const float *W = Wws + (size_t)bt * NP * ld;
+  float *v = fvec + (size_t)bt * kFitrVecs * NP;
+  const float *rhs = v + src * NP;
+  const int i = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (i >= NP) return;
+  const float *wr = W + (size_t)i * ld;
+  float s0 = 0.f, s1 = 0.f;
+  int k = lane;
+  for (; k + 32 <= i; k += 64) {
+    s0 = fmaf(wr[k], rhs[k], s0);
+    s1 = fmaf(wr[k + 32], rhs[k + 32], s1);
+  }
+  if (k <= i) s0 = fmaf(wr[k], rhs[k], s0);
+  float r = s0 + s1;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) r += __shfl_xor_sync(0xffffffffu, r, o);
+  if (lane == 0 && BOUTE_INB(i, NP)) v[kVt * NP + i] = r;
+}
+
+// W^T t for columns [32 x, 32 x + 32): lane = column, warp w takes the rows
+// i = k0 + w, k0 + w + 8, ... (those at or below the column's diagonal), the
+// eight partial sums added in a fixed order. mode 0: alpha = the result;
+// mode 1: alpha += the result; mode 2: alpha + the result kept exactly as a
+// pair (hi, lo), written with alpha's padding into the side input.
+__global__ void __launch_bounds__(256) fitr_wtx_kernel(int NP, int n, const float *Wws,
+                                                       float *fvec, int mode, float *xt, int DP,
+                                                       PostPlan plan, const int *fbad) {
+  __shared__ float part[8][33];
+  pdl_wait();
+  pdl_trigger();
+  const int bt = blockIdx.y, ld = NP + 1, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (fbad[bt]) return;
+  const float *W = Wws + (size_t)bt * NP * ld;
+  float *v = fvec + (size_t)bt * kFitrVecs * NP;
+  const float *tv = v + kVt * NP;
+  const int k0 = 32 * blockIdx.x, k = k0 + lane;
+  float s0 = 0.f, s1 = 0.f;  // entries above the diagonal are never loaded
+  int i = k0 + warp;
+  for (; i + 8 < NP; i += 16) {
+    const float w0 = i >= k ? W[(size_t)i * ld + k] : 0.f;
+    const float w1 = i + 8 >= k ? W[(size_t)(i + 8) * ld + k] : 0.f;
+    s0 = fmaf(w0, tv[i], s0);
+    s1 = fmaf(w1, tv[i + 8], s1);
+  }
+  if (i < NP && i >= k) s0 = fmaf(W[(size_t)i * ld + k], tv[i], s0);
+  part[warp][lane] = s0 + s1;
+  __syncthreads();
+  if (warp == 0 && BOUTE_INB(k, NP)) {
+    const float out = ((part[0][lane] + part[1][lane]) + (part[2][lane] + part[3][lane])) +
+                      ((part[4][lane] + part[5][lane]) + (part[6][lane] + part[7][lane]));
+    float *al = v + kVal * NP;
+    if (mode == 0) {
+      al[k] = out;
+    } else if (mode == 1) {
+      al[k] += out;
+    } else {
+      float hi, lo;
+      two_sum(al[k], out, hi, lo);
+      al[k] = hi;
+      v[kVlo * NP + k] = lo;
+      if (k < n) {
+        const int cf = xt_chunk_floats(DP);
+        float *q = xt + (size_t)bt * plan.nxt * cf + xt_alpha_offset(DP) +
+                   (size_t)(k / BOUTE_KCHUNK) * cf + k % BOUTE_KCHUNK;
+        q[0] = hi;
+        q[BOUTE_KCHUNK] = lo;
+      }
+    }
+  }
+}
+
+// r = y - K alpha in double-float (K = hi + lo, alpha zero from n on): a half
+// warp per row, eight loads of each of K hi and K lo per lane in flight, the
+// lanes combined by shuffles in a fixed order; zero from n on.
+__global__ void __launch_bounds__(256) fitr_resid_kernel(const float *Kh_all, const float *Kl_all,
+                                                         int n, int NP, float *fvec,
+                                                         const int *fbad) {
+  pdl_wait();
+  pdl_trigger();
+  const int bt = blockIdx.y, lane = threadIdx.x & 31, hl = lane & 15;
+  if (fbad[bt]) return;
+  const float *Kh = Kh_all + (size_t)bt * n * n, *Kl = Kl_all + (size_t)bt * n * n;
+  float *v = fvec + (size_t)bt * kFitrVecs * NP;
+  const float *al = v + kVal * NP;
+  const int i = blockIdx.x * 16 + (threadIdx.x >> 4);
+  if (i >= NP) return;  // a whole half warp
+  float sh = 0.f, sl = 0.f;
+  if (i < n) {
+    for (int k0 = 0; k0 < n; k0 += 128) {
+      float h8[8], l8[8], a8[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int k = k0 + hl + 16 * u;
+        const bool ok = k < n;
+        a8[u] = ok ? al[k] : 0.f;
+        h8[u] = ok ? Kh[(size_t)i * n + k] : 0.f;
+        l8[u] = ok ? Kl[(size_t)i * n + k] : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        float pr, e, s_, e2;
+        two_prod(h8[u], a8[u], pr, e);
+        two_sum(sh, pr, s_, e2);
+        sh = s_;
+        sl += e2 + fmaf(l8[u], a8[u], e);
+      }
+    }
+  }
+  const unsigned half = 0xffffu << (lane & 16);
+#pragma unroll
+  for (int o = 8; o > 0; o >>= 1) {  // within the half warp
+    const float oh = __shfl_xor_sync(half, sh, o);
+    const float ol = __shfl_xor_sync(half, sl, o);
+    float s_, e;
+    two_sum(sh, oh, s_, e);
+    sh = s_;
+    sl += ol + e;
+  }
+  if (hl == 0 && BOUTE_INB(i, NP))
+    v[kVr * NP + i] = i < n ? (v[kVy * NP + i] - sh) + (v[kVylo * NP + i] - sl) : 0.f;
 }
 
 // ---- operand images of L^-1 as fp16 hi/lo, swizzled (global-workspace fit) ----
@@ -1189,6 +1400,16 @@ int launch_standardize(const double *Y, int B, int n, int m, int codes, double *
 // The shared-memory variant holds n up to 160 (n rounded up to 32).
 bool fit_uses_smem(int npad) { return npad <= 160; }
 
+size_t fit_tpart_floats(int npad, int BM) {
+  if (fit_uses_smem(npad) || 4 * BM > num_sms()) return 0;  // no blocked factorisation
+  const int nbw = npad / 32, ncw = (nbw + kFitbChunk - 1) / kFitbChunk;
+  return (size_t)BM * nbw * ncw * 1024;
+}
+
+size_t fit_fvec_floats(int npad, int BM) {
+  return fit_tpart_floats(npad, BM) ? (size_t)BM * kFitrVecs * npad : 0;
+}
+
 // Dynamic shared memory of the shared-memory fit: A and W (np x (np+1)), six
 // vectors, and K lo (n x n) when n <= 128.
 static bool fit_kl_in_smem(int n) { return n <= 128; }
@@ -1225,7 +1446,7 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
   if (setup_done && cudaEventRecord(setup_done, s) != cudaSuccess) return last_launch_status();
   // the one-block fits already fill the GPU when there are many problem-
   // objectives; with few, the blocked factorisation spreads each over blocks
-  const bool blocked = !fit_uses_smem(npad) && 4 * BM <= sms;
+  const bool blocked = !fit_uses_smem(npad) && 4 * BM <= sms && gp->tpart && gp->fvec;
   if (fit_uses_smem(npad) || !blocked) {
     const bool sm_fit = fit_uses_smem(npad);
     if (sm_fit) {
@@ -1249,8 +1470,8 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
       count_launch(3);
     }
   } else {
-    // the factorisation across many blocks, panel by panel, then alpha and the
-    // outputs by fit32_kernel on the factored workspace
+    // the factorisation across many blocks, panel by panel, then alpha across
+    // many blocks and the operand images
     const int cap = std::max(1, 2 * sms / BM);
     auto ctas = [&](long long tiles) {
       return (unsigned)std::max(1LL, std::min<long long>(cap, (tiles + kFitbThreads - 1) / kFitbThreads));
@@ -1263,32 +1484,42 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
       const int rows = npad - 32 * p - 32, th = rows / 4;
       launch_pdl(fitb_diag_kernel, dim3(BM), dim3(64), 0, s, (const float *)gp->Kh, n, npad,
                  gp->Aws, gp->Wws, p, gp->fbad);
-      // items: the panel below's blocks, then one per pair of W's block columns
-      const long long items = ((long long)th * 8 + kFitbThreads - 1) / kFitbThreads + (p + 1) / 2;
+      // items: the panel below's blocks, then one per (J, chunk) of T_pJ
+      const long long items = ((long long)th * 8 + kFitbThreads - 1) / kFitbThreads + fitb_t_items(p);
       if (items > 0) {
         launch_pdl(fitb_panel_kernel,
                    dim3((unsigned)std::max(1LL, std::min<long long>(cap, items)), BM),
                    dim3(kFitbThreads), 0, s, npad, (const float *)gp->Aws, gp->Wws, p,
-                   (const int *)gp->fbad);
+                   (const int *)gp->fbad, gp->tpart);
         ++nl;
       }
       const long long tc = (long long)th * (th + 1) / 2 + 128LL * p + 32LL * rows;
       if (tc > 0) {
         launch_pdl(fitb_update_kernel, dim3(ctas(tc), BM), dim3(kFitbThreads), 0, s, npad,
-                   gp->Aws, gp->Wws, p, (const int *)gp->fbad);
+                   gp->Aws, gp->Wws, p, (const int *)gp->fbad, (const float *)gp->tpart);
         ++nl;
       }
       ++nl;
     }
-    count_launch(nl);
-    launch_pdl(fit32_kernel<false>, dim3(BM), dim3(fit_threads<false>()),
-               6 * npad * sizeof(float), s, gp->Kh, gp->Kl, Ys, standardize, n, m, gp->Aws,
-               gp->Wws, gp->xt, gp->DP, npad, gp->plan, gp->bop, 0, 0, gp->kern, gp->status,
-               (const int *)gp->fbad, (float *)nullptr);
+    // alpha: W^T (W y) and two refinement steps, each matvec over many blocks
+    const int *fb = gp->fbad;
+    launch_pdl(fitr_init_kernel, dim3(BM), dim3(256), 0, s, Ys, standardize, n, m, npad,
+               gp->fvec, gp->xt, gp->DP, gp->plan, gp->kern, gp->status, fb);
+    for (int step = 0; step < 3; ++step) {
+      if (step > 0)
+        launch_pdl(fitr_resid_kernel, dim3((npad + 15) / 16, BM), dim3(256), 0, s,
+                   (const float *)gp->Kh, (const float *)gp->Kl, n, npad, gp->fvec, fb);
+      launch_pdl(fitr_wx_kernel, dim3((npad + 7) / 8, BM), dim3(256), 0, s, npad,
+                 (const float *)gp->Wws, gp->fvec, step == 0 ? (int)kVy : (int)kVr, fb);
+      launch_pdl(fitr_wtx_kernel, dim3(npad / 32, BM), dim3(256), 0, s, npad, n,
+                 (const float *)gp->Wws, gp->fvec, step, gp->xt, gp->DP, gp->plan, fb);
+      nl += step > 0 ? 3 : 2;
+    }
+    count_launch(nl + 1);
     const long long tot = (long long)gp->plan.nwblk * BOUTE_BLKCOLS * gp->plan.nchunk * 32;
     pack_kernel<<<dim3((unsigned)std::min<long long>((tot + 255) / 256, 4096), BM), 256, 0, s>>>(
         gp->Wws, gp->plan, gp->bop, gp->xt, gp->DP, gp->status);
-    count_launch(3);
+    count_launch(1);
   }
   return last_launch_status();
 }

@@ -29,6 +29,8 @@ struct Gp {
   float *s2f;     // B*m: outputscale
   int *status;    // device status word (first error wins)
   int *fbad;      // B*m: a non-positive pivot in the blocked factorisation (n > 160)
+  float *tpart;   // the blocked factorisation's partial sums of T_pJ (fit_tpart_floats)
+  float *fvec;    // the blocked path's alpha vectors (fit_fvec_floats)
   // the FP64 tier (prec = BOUTE_PREC_FP64): W = L^-1 (B*m x n x n), alpha
   // (B*m x n), X / lengthscale (B*m x n x d), lengthscales (B*m x d) and
   // outputscales (B*m) of the last fit, all fp64
@@ -87,6 +89,12 @@ inline int num_sms() {
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   return sms;
 }
+
+// floats of the blocked factorisation's partial-sum workspace for B*m = BM
+// problem-objectives at padded size npad (0 when that size never takes it)
+size_t fit_tpart_floats(int npad, int BM);
+// floats of the blocked path's alpha vectors (0 likewise)
+size_t fit_fvec_floats(int npad, int BM);
 
 void count_launch(int k = 1);
 unsigned long long launch_count();
