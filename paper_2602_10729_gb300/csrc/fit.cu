@@ -1009,10 +1009,50 @@ __global__ void __launch_bounds__(64) fitb_diag_kernel(const float *Kh_all, int 
   }
 }
 
-// (b) L_rp = A_rp W_pp^T for the rows below the panel (4 x 4 tiles) into block
-// column p of W, and the partial sums of T_pJ = sum_{K=J}^{p-1} L_pK W_KJ
-// (J < p) into the workspace tpart: T_pJ's K range is split into chunks of
-// kFitbChunk blocks, one work item each, so that no item runs more than
+// The 32 x 32 tiles of (b) and (c): a block of kFitbThreads threads stages
+// its two operand tiles in shared memory (row stride 33) with coalesced loads
+// and forms a 2 x 2 output tile per thread (rows rb, rb + 1, columns cb,
+// cb + 1), each output an fmaf chain over q = 0..31 in order.
+using Tile = float[32][33];
+
+__device__ __forceinline__ void fitb_tile_load(Tile &dst, const float *src, int ld, int tid) {
+#pragma unroll
+  for (int j = 0; j < 1024 / kFitbThreads; ++j) {
+    const int x = tid + kFitbThreads * j, r = x >> 5, c = x & 31;
+    dst[r][c] = src[(size_t)r * ld + c];
+  }
+}
+
+// acc[u][v] += sum_q X[rb + u][q] Y[cb + v][q]  (X Y^T)
+__device__ __forceinline__ void fitb_mma_abt(const Tile &X, const Tile &Y, int rb, int cb,
+                                             float (&acc)[2][2]) {
+#pragma unroll 8
+  for (int q = 0; q < 32; ++q) {
+    const float x0 = X[rb][q], x1 = X[rb + 1][q], y0 = Y[cb][q], y1 = Y[cb + 1][q];
+    acc[0][0] = fmaf(x0, y0, acc[0][0]);
+    acc[0][1] = fmaf(x0, y1, acc[0][1]);
+    acc[1][0] = fmaf(x1, y0, acc[1][0]);
+    acc[1][1] = fmaf(x1, y1, acc[1][1]);
+  }
+}
+
+// acc[u][v] += sum_q X[rb + u][q] Y[q][cb + v]  (X Y)
+__device__ __forceinline__ void fitb_mma_ab(const Tile &X, const Tile &Y, int rb, int cb,
+                                            float (&acc)[2][2]) {
+#pragma unroll 8
+  for (int q = 0; q < 32; ++q) {
+    const float x0 = X[rb][q], x1 = X[rb + 1][q], y0 = Y[q][cb], y1 = Y[q][cb + 1];
+    acc[0][0] = fmaf(x0, y0, acc[0][0]);
+    acc[0][1] = fmaf(x0, y1, acc[0][1]);
+    acc[1][0] = fmaf(x1, y0, acc[1][0]);
+    acc[1][1] = fmaf(x1, y1, acc[1][1]);
+  }
+}
+
+// (b) the panel, L_Rp = A_Rp W_pp^T, in place in A for every block row R > p
+// (one work item each), and the partial sums of T_pJ = sum_{K=J}^{p-1} L_pK
+// W_KJ (J < p) into the workspace tpart: T_pJ's K range is split into chunks
+// of kFitbChunk blocks, one work item each, so that no item runs more than
 // kFitbChunk tile steps and the panel's critical path stays short for every p.
 // tpart holds, per problem-objective, nbw x ncw tiles of 32 x 32 floats (J,
 // chunk), nbw = NP / 32 and ncw = ceil(nbw / kFitbChunk).
@@ -1023,162 +1063,121 @@ __host__ __device__ __forceinline__ int fitb_t_items(int p) {
   return t;
 }
 
-__global__ void __launch_bounds__(kFitbThreads) fitb_panel_kernel(int NP, const float *Aws,
-                                                                  float *Wws, int p,
+__global__ void __launch_bounds__(kFitbThreads) fitb_panel_kernel(int NP, float *Aws,
+                                                                  const float *Wws, int p,
                                                                   const int *fbad, float *tpart) {
-  // T_pJ's tiles of the panel's block row and of W: L_pK and W_KJ (32 x 32,
-  // row stride 33)
-  __shared__ float Ls[32][33], Ws[32][33];
+  __shared__ Tile Xs, Ys;
   pdl_wait();
   pdl_trigger();
   const int bt = blockIdx.y, ld = NP + 1, tid = threadIdx.x;
   if (fbad[bt]) return;
-  const float *A = Aws + (size_t)bt * NP * ld;
-  float *W = Wws + (size_t)bt * NP * ld;
-  const int p0 = 32 * p, r0 = p0 + 32, rows = NP - r0;
-  // work items: blocks of the panel below (4 x 4 tiles, 256 threads each),
-  // then one item per (J, chunk) of T_pJ
-  const int ntr = (rows / 4) * 8, nbr = (ntr + kFitbThreads - 1) / kFitbThreads;
-  const int nbw = NP / 32, ncw = (nbw + kFitbChunk - 1) / kFitbChunk;  // the partials' layout
-  const int items = nbr + fitb_t_items(p);
+  float *A = Aws + (size_t)bt * NP * ld;
+  const float *W = Wws + (size_t)bt * NP * ld;
+  const int nbw = NP / 32, ncw = (nbw + kFitbChunk - 1) / kFitbChunk, p0 = 32 * p;
+  const int nr = nbw - 1 - p, items = nr + fitb_t_items(p);
+  const int rb = 2 * (tid >> 4), cb = 2 * (tid & 15);
+  bool wpp = false;  // W_pp staged in Ys
   for (int item = blockIdx.x; item < items; item += gridDim.x) {
-    if (item < nbr) {
-      const int tix = item * kFitbThreads + tid;
-      if (tix >= ntr) continue;
-      float acc[4][4] = {};
-      const int i0 = r0 + 4 * (tix >> 3), c0 = 4 * (tix & 7);
-#pragma unroll 4
-      for (int q = 0; q < 32; ++q) {
-        float x[4], y4[4];
+    float acc[2][2] = {};
+    if (item < nr) {  // L_Rp = A_Rp W_pp^T
+      float *ar = A + (size_t)(p0 + 32 + 32 * item) * ld + p0;
+      __syncthreads();  // the previous item's tiles are consumed
+      fitb_tile_load(Xs, ar, ld, tid);
+      if (!wpp) fitb_tile_load(Ys, W + (size_t)p0 * ld + p0, ld, tid);
+      wpp = true;
+      __syncthreads();
+      fitb_mma_abt(Xs, Ys, rb, cb, acc);
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          x[u] = A[(size_t)(i0 + u) * ld + p0 + q];
-          y4[u] = W[(size_t)(p0 + c0 + u) * ld + p0 + q];
-        }
+      for (int u = 0; u < 2; ++u)
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
-#pragma unroll
-          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-#pragma unroll
-        for (int v = 0; v < 4; ++v) W[(size_t)(i0 + u) * ld + p0 + c0 + v] = acc[u][v];
+        for (int v = 0; v < 2; ++v) ar[(size_t)(rb + u) * ld + cb + v] = acc[u][v];
       continue;
     }
-    // a partial sum of T_pJ = sum_{K=J}^{p-1} L_pK W_KJ over the chunk
-    // [J + c kFitbChunk, min(J + (c + 1) kFitbChunk, p)) of K blocks, for the
-    // item's (J, c); 2 x 2 outputs per thread; the update kernel adds a J's
-    // partials in chunk order
-    int J = 0, rest = item - nbr;
+    // the item's (J, c): K in [J + c kFitbChunk, min(J + (c + 1) kFitbChunk, p))
+    int J = 0, rest = item - nr;
     while (rest >= (p - J + kFitbChunk - 1) / kFitbChunk) {
       rest -= (p - J + kFitbChunk - 1) / kFitbChunk;
       ++J;
     }
     const int c = rest, Kb = J + c * kFitbChunk, Ke = min(Kb + kFitbChunk, p);
-    const int rb = 2 * (tid >> 4), cb = 2 * (tid & 15);
-    float acc[2][2] = {};
+    wpp = false;
     for (int K = Kb; K < Ke; ++K) {
-      __syncthreads();  // the previous K's tiles are consumed
-      for (int x = tid; x < 32 * 32; x += kFitbThreads) {
-        const int r = x >> 5, cc = x & 31;
-        Ls[r][cc] = A[(size_t)(p0 + r) * ld + 32 * K + cc];
-        Ws[r][cc] = W[(size_t)(32 * K + r) * ld + 32 * J + cc];
-      }
       __syncthreads();
-#pragma unroll 8
-      for (int q = 0; q < 32; ++q) {
-        const float x0 = Ls[rb][q], x1 = Ls[rb + 1][q];
-        const float y0 = Ws[q][cb], y1 = Ws[q][cb + 1];
-        acc[0][0] = fmaf(x0, y0, acc[0][0]);
-        acc[0][1] = fmaf(x0, y1, acc[0][1]);
-        acc[1][0] = fmaf(x1, y0, acc[1][0]);
-        acc[1][1] = fmaf(x1, y1, acc[1][1]);
-      }
+      fitb_tile_load(Xs, A + (size_t)p0 * ld + 32 * K, ld, tid);
+      fitb_tile_load(Ys, W + (size_t)(32 * K) * ld + 32 * J, ld, tid);
+      __syncthreads();
+      fitb_mma_ab(Xs, Ys, rb, cb, acc);
     }
-    float *tp = tpart + (((size_t)bt * nbw + J) * ncw + c) * 1024;
+    const size_t tile = ((size_t)bt * nbw + J) * ncw + c;
+    if (!BOUTE_INB(tile, (size_t)gridDim.y * nbw * ncw)) continue;
+    float *tp = tpart + tile * 1024;
 #pragma unroll
     for (int u = 0; u < 2; ++u)
 #pragma unroll
       for (int v = 0; v < 2; ++v) tp[(rb + u) * 32 + cb + v] = acc[u][v];
-    __syncthreads();  // before the next item reuses the tiles
   }
 }
 
-// (c) the trailing update A_ij -= sum_q L_iq L_jq below the panel (4 x 4
-// tiles of the lower triangle), W_pJ = -W_pp T_pJ (4 x 2 tiles), and the
-// panel (block column p of W, rows below it) copied into A.
+// (c) W_pJ = -W_pp T_pJ for J < p (one work item each; T_pJ the partials
+// added in chunk order, so the result does not depend on the grid), then the
+// trailing update A_IJ -= L_Ip L_Jp^T for p < J <= I (one item per 32 x 32
+// tile; the lower triangle of the diagonal tiles).
 __global__ void __launch_bounds__(kFitbThreads) fitb_update_kernel(int NP, float *Aws,
                                                                    float *Wws, int p,
                                                                    const int *fbad,
                                                                    const float *tpart) {
+  __shared__ Tile Xs, Ys;
   pdl_wait();
   pdl_trigger();
-  const int bt = blockIdx.y, ld = NP + 1;
+  const int bt = blockIdx.y, ld = NP + 1, tid = threadIdx.x;
   if (fbad[bt]) return;
   float *A = Aws + (size_t)bt * NP * ld;
   float *W = Wws + (size_t)bt * NP * ld;
-  const int p0 = 32 * p, r0 = p0 + 32, rows = NP - r0;
-  const int th = rows / 4, ntile = th * (th + 1) / 2, nwt = p * 128, ncp = rows * 32;
-  for (int tix = blockIdx.x * blockDim.x + threadIdx.x; tix < ntile + nwt + ncp;
-       tix += gridDim.x * blockDim.x) {
-    if (tix >= ntile + nwt) {  // the panel into A
-      const int e = tix - ntile - nwt;
-      const size_t o = (size_t)(r0 + (e >> 5)) * ld + p0 + (e & 31);
-      A[o] = W[o];
+  const int nbw = NP / 32, ncw = (nbw + kFitbChunk - 1) / kFitbChunk, p0 = 32 * p;
+  const int T = nbw - 1 - p, items = p + T * (T + 1) / 2;
+  const int rb = 2 * (tid >> 4), cb = 2 * (tid & 15);
+  bool wpp = false;  // W_pp staged in Xs
+  for (int item = blockIdx.x; item < items; item += gridDim.x) {
+    float acc[2][2] = {};
+    if (item < p) {  // W_pJ, J = item
+      const int J = item, nc = (p - J + kFitbChunk - 1) / kFitbChunk;
+      const float *tp = tpart + ((size_t)bt * nbw + J) * ncw * 1024;
+      __syncthreads();
+      if (!wpp) fitb_tile_load(Xs, W + (size_t)p0 * ld + p0, ld, tid);
+      wpp = true;
+#pragma unroll
+      for (int j = 0; j < 1024 / kFitbThreads; ++j) {
+        const int x = tid + kFitbThreads * j;
+        float t = 0.f;
+        for (int c = 0; c < nc; ++c) t += tp[(size_t)c * 1024 + x];
+        Ys[x >> 5][x & 31] = t;
+      }
+      __syncthreads();
+      fitb_mma_ab(Xs, Ys, rb, cb, acc);
+      float *wr = W + (size_t)p0 * ld + 32 * J;
+#pragma unroll
+      for (int u = 0; u < 2; ++u)
+#pragma unroll
+        for (int v = 0; v < 2; ++v) wr[(size_t)(rb + u) * ld + cb + v] = -acc[u][v];
       continue;
     }
-    float acc[4][4] = {};
-    if (tix < ntile) {
-      int ti = (int)((sqrtf(8.f * tix + 1.f) - 1.f) * 0.5f);
-      while (ti * (ti + 1) / 2 > tix) --ti;
-      while ((ti + 1) * (ti + 2) / 2 <= tix) ++ti;
-      const int tj = tix - ti * (ti + 1) / 2;
-      const int i0 = r0 + 4 * ti, j0 = r0 + 4 * tj;
-#pragma unroll 4
-      for (int q = 0; q < 32; ++q) {
-        float x[4], y4[4];
+    const int e = item - p;
+    int ti = (int)((sqrtf(8.f * e + 1.f) - 1.f) * 0.5f);
+    while (ti * (ti + 1) / 2 > e) --ti;
+    while ((ti + 1) * (ti + 2) / 2 <= e) ++ti;
+    const int tj = e - ti * (ti + 1) / 2, I = p + 1 + ti, J = p + 1 + tj;
+    wpp = false;
+    __syncthreads();
+    fitb_tile_load(Xs, A + (size_t)(32 * I) * ld + p0, ld, tid);
+    fitb_tile_load(Ys, A + (size_t)(32 * J) * ld + p0, ld, tid);
+    __syncthreads();
+    fitb_mma_abt(Xs, Ys, rb, cb, acc);
+    float *ar = A + (size_t)(32 * I) * ld + 32 * J;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          x[u] = W[(size_t)(i0 + u) * ld + p0 + q];
-          y4[u] = W[(size_t)(j0 + u) * ld + p0 + q];
-        }
+    for (int u = 0; u < 2; ++u)
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
-#pragma unroll
-          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(x[u], y4[v], acc[u][v]);
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-#pragma unroll
-        for (int v = 0; v < 4; ++v)
-          if (ti != tj || v <= u) A[(size_t)(i0 + u) * ld + j0 + v] -= acc[u][v];
-    } else {
-      const int e = tix - ntile, J = e >> 7, rb = 4 * ((e >> 4) & 7), cb = 2 * (e & 15);
-      const int nbw = NP / 32, ncw = (nbw + kFitbChunk - 1) / kFitbChunk;
-      const int nc = (p - J + kFitbChunk - 1) / kFitbChunk;  // this J's partials
-      const float *tp = tpart + ((size_t)bt * nbw + J) * ncw * 1024;
-#pragma unroll 4
-      for (int q = 0; q < 32; ++q) {
-        float x[4], y2[2];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) x[u] = W[(size_t)(p0 + rb + u) * ld + p0 + q];
-#pragma unroll
-        for (int v = 0; v < 2; ++v) {  // T_pJ(q, cb + v): the partials in chunk order
-          float t = 0.f;
-          for (int c = 0; c < nc; ++c) t += tp[(size_t)c * 1024 + q * 32 + cb + v];
-          y2[v] = t;
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-#pragma unroll
-          for (int v = 0; v < 2; ++v) acc[u][v] = fmaf(x[u], y2[v], acc[u][v]);
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-#pragma unroll
-        for (int v = 0; v < 2; ++v) W[(size_t)(p0 + rb + u) * ld + 32 * J + cb + v] = -acc[u][v];
-    }
+      for (int v = 0; v < 2; ++v)
+        if (I != J || cb + v <= rb + u) ar[(size_t)(rb + u) * ld + cb + v] -= acc[u][v];
   }
 }
 
@@ -1476,30 +1475,33 @@ static int launch_fit_impl(Gp *gp, const double *X, const double *Ys, int standa
     auto ctas = [&](long long tiles) {
       return (unsigned)std::max(1LL, std::min<long long>(cap, (tiles + kFitbThreads - 1) / kFitbThreads));
     };
+    auto grid = [&](long long items) {  // one block per item up to 4 blocks per SM
+      return (unsigned)std::max(1LL, std::min<long long>(std::max(1, 4 * sms / BM), items));
+    };
     int nl = 0;
     launch_pdl(fitb_load_kernel, dim3(ctas((long long)npad * npad / 2), BM), dim3(kFitbThreads), 0, s,
                (const float *)gp->Kh, n, npad, gp->Aws, gp->fbad);
     ++nl;
-    for (int p = 0; p < npad / 32; ++p) {
-      const int rows = npad - 32 * p - 32, th = rows / 4;
+    const int nbw = npad / 32;
+    for (int p = 0; p < nbw; ++p) {
+      const int T = nbw - 1 - p;
       launch_pdl(fitb_diag_kernel, dim3(BM), dim3(64), 0, s, (const float *)gp->Kh, n, npad,
                  gp->Aws, gp->Wws, p, gp->fbad);
-      // items: the panel below's blocks, then one per (J, chunk) of T_pJ
-      const long long items = ((long long)th * 8 + kFitbThreads - 1) / kFitbThreads + fitb_t_items(p);
+      ++nl;
+      // items: the panel's block rows below p, then one per (J, chunk) of T_pJ
+      const long long items = (long long)T + fitb_t_items(p);
       if (items > 0) {
-        launch_pdl(fitb_panel_kernel,
-                   dim3((unsigned)std::max(1LL, std::min<long long>(cap, items)), BM),
-                   dim3(kFitbThreads), 0, s, npad, (const float *)gp->Aws, gp->Wws, p,
-                   (const int *)gp->fbad, gp->tpart);
+        launch_pdl(fitb_panel_kernel, dim3(grid(items), BM), dim3(kFitbThreads), 0, s, npad,
+                   gp->Aws, (const float *)gp->Wws, p, (const int *)gp->fbad, gp->tpart);
         ++nl;
       }
-      const long long tc = (long long)th * (th + 1) / 2 + 128LL * p + 32LL * rows;
-      if (tc > 0) {
-        launch_pdl(fitb_update_kernel, dim3(ctas(tc), BM), dim3(kFitbThreads), 0, s, npad,
+      // items: W_pJ for J < p, then the trailing tiles
+      const long long uitems = (long long)p + (long long)T * (T + 1) / 2;
+      if (uitems > 0) {
+        launch_pdl(fitb_update_kernel, dim3(grid(uitems), BM), dim3(kFitbThreads), 0, s, npad,
                    gp->Aws, gp->Wws, p, (const int *)gp->fbad, (const float *)gp->tpart);
         ++nl;
       }
-      ++nl;
     }
     // alpha: W^T (W y) and two refinement steps, each matvec over many blocks
     const int *fb = gp->fbad;
