@@ -30,7 +30,10 @@ namespace boute {
 namespace {
 
 constexpr int kOptThreads = 128, kOptWarps = kOptThreads / 32;
-constexpr float kS5 = 2.2360679774997896964f;
+constexpr float kLn2f = 0.6931471805599453f;
+constexpr float kLn2Sq3f = 0.16015100463940046f;  // (ln 2)^2 / 3
+// 1 / (the side input's coordinate scale)^2
+constexpr float kInvScale2 = (float)(1.0 / (kCoordScale52 * kCoordScale52));
 
 struct OptArgs {
   const float *Wws, *xt;
@@ -94,12 +97,14 @@ __global__ void __launch_bounds__(kOptThreads) acqopt_kernel(const __grid_consta
         for (int k = 0; k < d; ++k) {
           const float xk = fmaf(xs[k], par[k], xs[k] * par[DP + k]);  // x_k / l_k
           const float dk = (xk - ch[k * BOUTE_KCHUNK + jj]) - ch[(DP + k) * BOUTE_KCHUNK + jj];
-          df[(size_t)j * d + k] = dk * (par[k] + par[DP + k]);  // (x_k - X_jk) / l_k^2
+          df[(size_t)j * d + k] = dk * (par[k] + par[DP + k]) * kInvScale2;  // (x_k - X_jk) / l_k^2
           r2 = fmaf(dk, dk, r2);
         }
-        const float r = sqrtf(r2), ex = expf(-kS5 * r);
-        kv[j] = s2 * fmaf(5.f / 3.f, r2, fmaf(kS5, r, 1.f)) * ex;
-        cv[j] = -5.f / 3.f * s2 * fmaf(kS5, r, 1.f) * ex;
+        // r2 = r'^2, the side input's scaled distance: sqrt5 r = ln2 r',
+        // exp(-sqrt5 r) = 2^(-r'); df above carries the scale twice
+        const float rs = sqrtf(r2), ex = exp2f(-rs);
+        kv[j] = s2 * fmaf(kLn2Sq3f, r2, fmaf(kLn2f, rs, 1.f)) * ex;
+        cv[j] = -5.f / 3.f * s2 * fmaf(kLn2f, rs, 1.f) * ex;
         const float *al = ch + xt_alpha_offset(DP) + jj;
         amu = fmaf(kv[j], al[0] + al[BOUTE_KCHUNK], amu);
       }

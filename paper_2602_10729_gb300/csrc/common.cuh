@@ -67,6 +67,15 @@ __device__ __forceinline__ double outcome_transform(double y, int code) {
 }
 #endif
 
+// The side input's coordinates and inverse lengthscales carry a constant
+// factor: x / l times sqrt(5) / ln 2 (the Matern-5/2 kernel, and the composite
+// kernel's routing features), sqrt(3) / ln 2 on the composite kernel's
+// deployment features (its Matern-3/2 part). The scaled distance r' then is
+// the kernel's exponent in base 2, exp(-sqrt5 r) = 2^(-r'), with no rounding
+// of a product in between.
+constexpr double kCoordScale52 = 3.225964182229561;   // sqrt(5) / ln 2
+constexpr double kCoordScale32 = 2.4988211106473432;  // sqrt(3) / ln 2
+
 // Floats of one training-point chunk of the posterior's side input: X/ls as
 // fp32 hi [DP][32] and lo [DP][32] (dimension-major, so pairs of training
 // points load as packed f32x2), alpha as an fp32 pair, hi [32] and lo [32],

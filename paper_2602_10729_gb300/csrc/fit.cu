@@ -144,7 +144,8 @@ __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad
   const int total = npad * DP;
   for (int e = blk * blockDim.x + threadIdx.x; e < total; e += nblk * blockDim.x) {
     const int j = e / DP, t = e % DP;
-    double v = (j < n && t < d) ? X[((size_t)b * n + j) * d + t] / l[t] : 0.0;
+    const double cs = (COMP && t >= dtau) ? kCoordScale32 : kCoordScale52;
+    double v = (j < n && t < d) ? X[((size_t)b * n + j) * d + t] / l[t] * cs : 0.0;
     float hi = (float)v, lo = (float)(v - (double)hi);
     const int c = j / BOUTE_KCHUNK, jj = j % BOUTE_KCHUNK;
     float *q = x + (size_t)c * cf;  // dimension-major: [DP][32] hi, [DP][32] lo
@@ -170,11 +171,12 @@ __device__ void prep_part(const double *X, int n, int d, int b, int DP, int npad
   for (int e = blk * blockDim.x + threadIdx.x; e < nch * np; e += nblk * blockDim.x) {
     const int c = e / np, k = e % np;
     float v = 0.f;
-    if (k < DP) v = k < d ? (float)(1.0 / l[k]) : 0.f;
+    // the coordinates' scale over l (hi, lo)
+    if (k < DP) v = k < d ? (float)(((COMP && k >= dtau) ? kCoordScale32 : kCoordScale52) / l[k]) : 0.f;
     else if (k < 2 * DP) {
       const int t = k - DP;
       if (t < d) {
-        const double iv = 1.0 / l[t];
+        const double iv = ((COMP && t >= dtau) ? kCoordScale32 : kCoordScale52) / l[t];
         v = (float)(iv - (double)(float)iv);
       }
     } else if (k == 2 * DP + kParS2) v = (float)s2;
@@ -1213,7 +1215,6 @@ __global__ void __launch_bounds__(256) fitr_init_kernel(const double *Ys, int st
   for (int i = tid; i < NP; i += blockDim.x) {  // standardised y as an fp32 pair
     const double ys = i < n ? (y[(size_t)i * m] - ymu) * yisd : 0.0;
     const float hi = (float)ys;
-    BOUTE_INB(i, NP);
     v[kVy * NP + i] = hi;
     v[kVylo * NP + i] = (float)(ys - (double)hi);
   }

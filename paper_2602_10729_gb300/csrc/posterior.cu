@@ -95,10 +95,6 @@ __host__ __device__ __forceinline__ int st_off32(int row, int kk) {
   return row * 64 + ((((kk >> 2) ^ (row & 15))) << 2) + (kk & 3);
 }
 
-constexpr float kSqrt5 = 2.2360679774997896964f;
-constexpr float kSqrt5Log2e = 3.2259641822295610f;  // sqrt(5) / ln(2)
-constexpr float kSqrt3 = 1.7320508075688772f;
-constexpr float kSqrt3Log2e = 2.4988211106473432f;  // sqrt(3) / ln(2)
 
 // Single hardware instructions (relative error about 2^-22), no range fix-ups:
 // arguments here are finite and non-negative (sqrt) or non-positive (ex2).
@@ -112,9 +108,10 @@ __device__ __forceinline__ float ex2_approx(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
-constexpr float kFiveThirds = 1.6666666666666667f;
-constexpr float kSqrt5Log2eLo = 1.1286310597e-07f;  // sqrt(5) / ln(2) - kSqrt5Log2e
+// In the scaled distance r' = sqrt5 r / ln 2 (sqrt3 r / ln 2 for Matern-3/2):
+// sqrt5 r = ln2 r', 5/3 r^2 = (ln2)^2 / 3 r'^2, exp(-sqrt5 r) = 2^(-r').
 constexpr float kLn2 = 0.6931471805599453f;
+constexpr float kLn2Sq3 = 0.16015100463940046f;  // (ln 2)^2 / 3
 
 // ---- packed fp32 pairs (sm_100+ f32x2 arithmetic) --------------------------------
 __device__ __forceinline__ unsigned long long f2_dup(float x) {
@@ -222,12 +219,14 @@ __device__ __forceinline__ float cand_weight(const float (&xr)[DP], const float 
 
 // The K* values of one builder thread's COLS columns of a 32-point chunk:
 // squared scaled distances in packed pairs (candidate x*_k / l_k as a
-// duplicated pair, minus the chunk's training coordinates x_k / l_k), then
-// k = s2 (1 + sqrt5 r + 5/3 r^2) exp(-sqrt5 r) with exp(-x) = 2^(-x log2 e).
+// duplicated pair, minus the chunk's training coordinates x_k / l_k, both
+// times the side input's coordinate scale), then
+// k = s2 (1 + sqrt5 r + 5/3 r^2) exp(-sqrt5 r) = s2 (1 + ln2 r' + ln2^2/3 r'^2) 2^(-r').
 // KERN = 1, the composite kernel: the distances over the routing features
 // (r_t) and the deployment features (r_c) are accumulated apart, and
 //   k = k52(r_t) (s2 + s2_x k32(r_c)) + s2_c w_j w* k32(r_c),
-//   k52(r) = (1 + sqrt5 r + 5/3 r^2) e^(-sqrt5 r), k32(r) = (1 + sqrt3 r) e^(-sqrt3 r).
+//   k52(r) = (1 + sqrt5 r + 5/3 r^2) e^(-sqrt5 r), k32(r) = (1 + sqrt3 r) e^(-sqrt3 r),
+// each in its own scaled distance (the deployment features carry sqrt3 / ln 2).
 // Both the fused builders and the stand-alone K* kernel use this, so their
 // values are identical.
 template <int DP, int COLS, int KERN = 0>
@@ -275,34 +274,25 @@ __device__ __forceinline__ void kstar_cols(const unsigned long long (&xs2)[DP], 
 #pragma unroll
       for (int z = 0; z < 2; ++z) {
         const float rr = sqrt_approx(r2[z]);
-        const float k52 =
-            fmaf(kFiveThirds, r2[z], fmaf(kSqrt5, rr, 1.0f)) * ex2_approx(-kSqrt5Log2e * rr);
+        const float k52 = fmaf(kLn2Sq3, r2[z], fmaf(kLn2, rr, 1.0f)) * ex2_approx(-rr);
         const float rc = sqrt_approx(c2[z]);
-        const float k32 = fmaf(kSqrt3, rc, 1.0f) * ex2_approx(-kSqrt3Log2e * rc);
+        const float k32 = fmaf(kLn2, rc, 1.0f) * ex2_approx(-rc);
         kv[2 * e + z] = fmaf(k52, fmaf(ci.s2x, k32, s2), ci.s2c * (wj[2 * e + z] * ci.ws) * k32);
       }
     }
     return;
   }
-  // packed pairs: k = (s2 + s2 sqrt5 r + s2 5/3 r^2) 2^A (1 + (a - A) ln 2), where
-  // a = -sqrt5 r / ln 2 is the exact exponent and A its fp32 rounding, which ex2
-  // takes: fma(r, K, A) recovers the rounding exactly, so the exponential is
-  // as accurate as ex2 itself at any r (the rounding of A alone is 2^-24 |a|)
-  const unsigned long long nK = f2_dup(-kSqrt5Log2e), pK = f2_dup(kSqrt5Log2e),
-                           pKlo = f2_dup(kSqrt5Log2eLo), nLn2 = f2_dup(-kLn2), c0 = f2_dup(s2),
-                           c1 = f2_dup(s2 * kSqrt5), c2 = f2_dup(s2 * kFiveThirds);
+  // packed pairs: k = (s2 + s2 ln2 r' + s2 ln2^2/3 r'^2) 2^(-r'); the exponent
+  // is the scaled distance itself, so the exponential is as accurate as ex2
+  const unsigned long long c0 = f2_dup(s2), c1 = f2_dup(s2 * kLn2), c2 = f2_dup(s2 * kLn2Sq3);
 #pragma unroll
   for (int e = 0; e < COLS / 2; ++e) {
     float ra, rb;
     f2_split(acc2[e], ra, rb);
-    const unsigned long long rr = f2_pack(sqrt_approx(ra), sqrt_approx(rb));
-    const unsigned long long A = f2_mul(rr, nK);
-    float A0, A1;
-    f2_split(A, A0, A1);
-    const unsigned long long ex = f2_pack(ex2_approx(A0), ex2_approx(A1));
-    const unsigned long long q = f2_mul(f2_fma(rr, pKlo, f2_fma(rr, pK, A)), nLn2);  // (a - A) ln 2
-    const unsigned long long t = f2_mul(f2_fma(acc2[e], c2, f2_fma(rr, c1, c0)), ex);
-    f2_split(f2_fma(t, q, t), kv[2 * e], kv[2 * e + 1]);
+    const float r0 = sqrt_approx(ra), r1 = sqrt_approx(rb);
+    const unsigned long long ex = f2_pack(ex2_approx(-r0), ex2_approx(-r1));
+    const unsigned long long t = f2_fma(acc2[e], c2, f2_fma(f2_pack(r0, r1), c1, c0));
+    f2_split(f2_mul(t, ex), kv[2 * e], kv[2 * e + 1]);
   }
 }
 
@@ -392,8 +382,8 @@ __device__ double mean_fp64_warp(const float *xrow, int d, const float *x0, int 
       r2 = fma(df, df, r2);
     }
     if (j >= n) continue;
-    const double r = sqrt(r2);
-    const double kv = s2 * (1.0 + 2.2360679774997896964 * r + (5.0 / 3.0) * r2) *
+    const double r = sqrt(r2) / kCoordScale52;  // (the side input's scale)
+    const double kv = s2 * (1.0 + 2.2360679774997896964 * r + (5.0 / 3.0) * (r * r)) *
                       exp(-2.2360679774997896964 * r);
     const float *al = ch + xt_alpha_offset(DP) + jj;  // alpha hi, lo
     acc = fma(kv, (double)al[0] + (double)al[BOUTE_KCHUNK], acc);
