@@ -167,7 +167,9 @@ __device__ __forceinline__ float mc_hvi_regs(const float *e, int S, const float 
       if (!ok) y[j][0] = kInfeasible;
     }
   }
-  float sum = 0.f;
+  // the products and the sum over pairs of samples in packed f32x2 (the
+  // saturating fmas have no packed form): two partial sums per lane
+  unsigned long long sum2 = 0ull;
   for (int k = 0; k < K; ++k) {
     float iw[M], hw[M], W = 1.f;
     bool live = true;
@@ -181,15 +183,21 @@ __device__ __forceinline__ float mc_hvi_regs(const float *e, int S, const float 
       W *= w;
     }
     if (!live) continue;  // (uniform: the box and ymin are the warp's)
+    const unsigned long long W2 = f2_dup(W);
 #pragma unroll
-    for (int j = 0; j < NS; ++j) {
-      float p = fma_sat(-y[j][0], iw[0], hw[0]);
+    for (int j = 0; j < NS; j += 2) {
+      unsigned long long p = f2_pack(fma_sat(-y[j][0], iw[0], hw[0]),
+                                     fma_sat(-y[j + 1][0], iw[0], hw[0]));
 #pragma unroll
-      for (int t = 1; t < M; ++t) p *= fma_sat(-y[j][t], iw[t], hw[t]);
-      sum = fmaf(W, p, sum);
+      for (int t = 1; t < M; ++t)
+        p = f2_mul(p, f2_pack(fma_sat(-y[j][t], iw[t], hw[t]),
+                              fma_sat(-y[j + 1][t], iw[t], hw[t])));
+      sum2 = f2_fma(W2, p, sum2);
     }
   }
-  return sum;
+  float s0, s1;
+  f2_split(sum2, s0, s1);
+  return s0 + s1;
 }
 
 template <int M, bool CONS>

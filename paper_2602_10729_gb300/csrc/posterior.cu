@@ -113,38 +113,6 @@ __device__ __forceinline__ float ex2_approx(float x) {
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kLn2Sq3 = 0.16015100463940046f;  // (ln 2)^2 / 3
 
-// ---- packed fp32 pairs (sm_100+ f32x2 arithmetic) --------------------------------
-__device__ __forceinline__ unsigned long long f2_dup(float x) {
-  unsigned long long r;
-  asm("mov.b64 %0, {%1, %1};" : "=l"(r) : "f"(x));
-  return r;
-}
-__device__ __forceinline__ unsigned long long f2_sub(unsigned long long a, unsigned long long b) {
-  unsigned long long r;
-  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
-  return r;
-}
-__device__ __forceinline__ unsigned long long f2_fma(unsigned long long a, unsigned long long b,
-                                                     unsigned long long c) {
-  unsigned long long r;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
-  return r;
-}
-__device__ __forceinline__ unsigned long long f2_add(unsigned long long a, unsigned long long b) {
-  unsigned long long r;
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
-  return r;
-}
-__device__ __forceinline__ unsigned long long f2_mul(unsigned long long a, unsigned long long b) {
-  unsigned long long r;
-  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
-  return r;
-}
-__device__ __forceinline__ unsigned long long f2_pack(float x, float y) {
-  unsigned long long r;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(x), "f"(y));
-  return r;
-}
 // Compensated (Kahan) accumulation of packed pairs: s + c carries the sum
 // of the terms with the rounding error of every addition.
 struct Kahan2 {
@@ -161,9 +129,6 @@ __device__ __forceinline__ void two_sum_f(float a, float b, float &s, float &e) 
   s = a + b;
   const float bb = s - a;
   e = (a - (s - bb)) + (b - bb);
-}
-__device__ __forceinline__ void f2_split(unsigned long long v, float &x, float &y) {
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(x), "=f"(y) : "l"(v));
 }
 
 // 32 lanes x 32 bit, 16 consecutive columns per thread, wait fused.
