@@ -178,7 +178,7 @@ __device__ __forceinline__ float mc_hvi_regs(const float *e, int S, const float 
       const float h = hi[k * M + t];
       const float w = h - fmaxf(lo[k * M + t], ymin[t]);
       live = live && w > 0.f;
-      iw[t] = __frcp_rn(w);
+      iw[t] = rcp_fast(w);  // (relative error ~2^-23; the clamp absorbs it at the edges)
       hw[t] = h * iw[t];
       W *= w;
     }
