@@ -135,7 +135,9 @@ __global__ void __launch_bounds__(256) ehvi2d_kernel(const float *mean, const fl
 template <int M, bool CONS, int NV>
 __device__ __forceinline__ float mc_hvi_regs(const float *e, int S, const float (&mu)[M],
                                              const float (&sg)[M], const float (&kc)[M],
-                                             const float *lo, const float *hi, int K, int lane) {
+                                             const float *lo, const float *hi, int K, int lane,
+                                             float4 *stage) {
+  static_assert(M <= 3, "a box's constants fit two float4");
   constexpr int NS = 4 * NV;
   float y[NS][M];
 #pragma unroll
@@ -168,31 +170,50 @@ __device__ __forceinline__ float mc_hvi_regs(const float *e, int S, const float 
     }
   }
   // the products and the sum over pairs of samples in packed f32x2 (the
-  // saturating fmas have no packed form): two partial sums per lane
+  // saturating fmas have no packed form): two partial sums per lane. The
+  // boxes' constants (1/w_t, u_t/w_t, prod w_t) are formed 32 boxes at a time,
+  // one box per lane, and staged in this warp's 64 float4 of shared memory;
+  // the live boxes are then visited in order, their constants read back by
+  // broadcast
   unsigned long long sum2 = 0ull;
-  for (int k = 0; k < K; ++k) {
-    float iw[M], hw[M], W = 1.f;
-    bool live = true;
+  for (int k0 = 0; k0 < K; k0 += 32) {
+    const int kb = k0 + lane;
+    float cw[3] = {0.f, 0.f, 0.f}, ch[3] = {0.f, 0.f, 0.f}, Wb = 0.f;
+    bool lv = false;
+    if (kb < K) {
+      lv = true;
+      Wb = 1.f;
 #pragma unroll
-    for (int t = 0; t < M; ++t) {
-      const float h = hi[k * M + t];
-      const float w = h - fmaxf(lo[k * M + t], ymin[t]);
-      live = live && w > 0.f;
-      iw[t] = rcp_fast(w);  // (relative error ~2^-23; the clamp absorbs it at the edges)
-      hw[t] = h * iw[t];
-      W *= w;
+      for (int t = 0; t < M; ++t) {
+        const float h = hi[kb * M + t];
+        const float w = h - fmaxf(lo[kb * M + t], ymin[t]);
+        lv = lv && w > 0.f;
+        cw[t] = rcp_fast(w);  // (relative error ~2^-23; the clamp absorbs it at the edges)
+        ch[t] = h * cw[t];
+        Wb *= w;
+      }
     }
-    if (!live) continue;  // (uniform: the box and ymin are the warp's)
-    const unsigned long long W2 = f2_dup(W);
+    __syncwarp();  // the previous group's constants are read
+    stage[lane] = make_float4(cw[0], cw[1], cw[2], Wb);
+    stage[32 + lane] = make_float4(ch[0], ch[1], ch[2], 0.f);
+    __syncwarp();
+    unsigned todo = __ballot_sync(0xffffffffu, lv);
+    while (todo) {
+      const int jb = __ffs(todo) - 1;
+      todo &= todo - 1;
+      const float4 ca = stage[jb], cb = stage[32 + jb];
+      const float iw[3] = {ca.x, ca.y, ca.z}, hw[3] = {cb.x, cb.y, cb.z};
+      const unsigned long long W2 = f2_dup(ca.w);
 #pragma unroll
-    for (int j = 0; j < NS; j += 2) {
-      unsigned long long p = f2_pack(fma_sat(-y[j][0], iw[0], hw[0]),
-                                     fma_sat(-y[j + 1][0], iw[0], hw[0]));
+      for (int j = 0; j < NS; j += 2) {
+        unsigned long long p = f2_pack(fma_sat(-y[j][0], iw[0], hw[0]),
+                                       fma_sat(-y[j + 1][0], iw[0], hw[0]));
 #pragma unroll
-      for (int t = 1; t < M; ++t)
-        p = f2_mul(p, f2_pack(fma_sat(-y[j][t], iw[t], hw[t]),
-                              fma_sat(-y[j + 1][t], iw[t], hw[t])));
-      sum2 = f2_fma(W2, p, sum2);
+        for (int t = 1; t < M; ++t)
+          p = f2_mul(p, f2_pack(fma_sat(-y[j][t], iw[t], hw[t]),
+                                fma_sat(-y[j + 1][t], iw[t], hw[t])));
+        sum2 = f2_fma(W2, p, sum2);
+      }
     }
   }
   float s0, s1;
@@ -208,6 +229,7 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
                                                     long long eps_stride, const double *cons,
                                                     float *acq) {
   extern __shared__ float boxes[];  // per problem in this block: lo[K][M], hi[K][M]
+  __shared__ float4 stage[16][64];  // per warp: 32 boxes' constants (mc_hvi_regs)
   pdl_wait();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
   const int b = blockIdx.y;
@@ -238,9 +260,9 @@ __global__ void __launch_bounds__(512) mchvi_kernel(const float *mean, const flo
       continue;  // (warp-uniform)
     float sum = 0.f;
     if (vec && S == 256) {
-      sum = mc_hvi_regs<M, CONS, 2>(e, S, mu, sg, kc, lo, hi, K, lane);
+      sum = mc_hvi_regs<M, CONS, 2>(e, S, mu, sg, kc, lo, hi, K, lane, stage[warp]);
     } else if (vec && S == 128) {
-      sum = mc_hvi_regs<M, CONS, 1>(e, S, mu, sg, kc, lo, hi, K, lane);
+      sum = mc_hvi_regs<M, CONS, 1>(e, S, mu, sg, kc, lo, hi, K, lane, stage[warp]);
     } else if (vec) {
       for (int s0 = 4 * lane; s0 < S; s0 += 128) {
         float4 z[M];
