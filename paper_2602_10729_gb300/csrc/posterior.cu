@@ -914,10 +914,13 @@ int launch_dp(const Gp *gp, const float *Xc, const float *kst, long long N, floa
   const size_t fixed = 1024 + 512;  // alignment slack, barriers, TMEM address, flag
   const size_t budget = 227 * 1024 - fixed;
   const size_t st = kst ? kStageBytes : 0;  // staging beside each A stage (PRE)
-  // deep B ring first (a chunk feeds up to four blocks), then A, then the side input
+  // K* stages before B stages: a deeper A ring lets the builders run ahead of
+  // the tensor cores through the groups where the MMAs outweigh the building
+  // (measured best: 4 A + 2 B stages with 8 builder warps, 3 + 3 with 16),
+  // then the side input's ring as deep as what is left allows
   a.sx = kMaxX;
-  a.sa = 3;
-  a.sb = 4;
+  a.sa = Layout<DP>::kBld == 8 ? 4 : 3;
+  a.sb = Layout<DP>::kBld == 8 ? 2 : 3;
   while ((size_t)a.sa * (kABytes + st) + (size_t)a.sb * a.b_bytes + (size_t)a.sx * a.x_bytes >
          budget) {
     if (a.sx > 4) --a.sx;
