@@ -44,7 +44,7 @@ namespace boute {
 
 namespace {
 
-constexpr int kEpiWarp0 = 2;  // warps 2-5: epilogue, TMEM lane quarter = warp % 4
+constexpr int kEpiWarp0 = 2;  // warps 2-5: epilogue (variance, mean), TMEM lane quarter = warp % 4
 constexpr int kEpiWarps = 4;
 constexpr int kXtWarp = 6;    // warp 6: side-input producer
 constexpr int kBldWarp0 = 7;  // warps 7..: K* builders
@@ -392,8 +392,8 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
     posterior_kernel(const __grid_constant__ PostArgs a) {
   constexpr int kBldWarps = Layout<DP>::kBld;
   constexpr int COLS = Layout<DP>::kCols;   // columns of a half per builder thread
-  constexpr int GPR = 32 / COLS;            // column groups per row (threads per row)
-  constexpr int RPW = 32 / GPR;             // rows per builder warp
+  constexpr int GPR = 32 / COLS;            // column groups per row
+  constexpr int RPW = 32 / GPR;             // rows per builder warp (16 builder warps)
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-byte alignment (the 128-byte swizzle atom) as an offset from the
   // shared array, so that every access below stays a shared-memory access
@@ -415,8 +415,13 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   uint64_t *drain = acc_empty + kSlots;
   uint64_t *st_full = drain + 1, *st_empty = st_full + kMaxA;  // PRE staging
   uint64_t *cache_ready = st_empty + kMaxA;  // a group's K* chunks are stored
-  uint32_t *tmem_holder = (uint32_t *)(cache_ready + 1);
+  // the builders' partial means of a unit are written / read by the epilogue
+  uint64_t *mean_ready = cache_ready + 1, *mean_empty = mean_ready + 1;
+  uint32_t *tmem_holder = (uint32_t *)(mean_empty + 1);
   volatile int *abort = (volatile int *)(tmem_holder + 1);
+  // after the 512-byte barrier area: per column group and row of the tile,
+  // a builder thread's partial mean (hi, lo) and magnitude sum
+  float *red = (float *)(bars + 64);
 
   auto a_hi = [&](int s) { return sm + (size_t)s * kABytes; };
   auto b_reg = [&](int s) { return ring_b + (size_t)s * a.b_bytes; };
@@ -444,6 +449,8 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
     }
     mbar_init(drain, 1);
     mbar_init(cache_ready, 1);
+    mbar_init(mean_ready, kBldWarps);
+    mbar_init(mean_empty, kEpiWarps);
     *abort = 0;
     fence_mbar_init();
   }
@@ -630,7 +637,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   } else if (warp >= kEpiWarp0 && warp < kEpiWarp0 + kEpiWarps) {
     // ---------------------------------------------------------------- epilogue
     const int eq = warp & 3;  // TMEM lane quarter this warp may access
-    uint32_t blkseq = 0;
+    uint32_t blkseq = 0, nmean = 0;
     const uint32_t lanes = (uint32_t)(32 * eq) << 16;
     for (int unit = blockIdx.x; unit < units && !*abort; unit += gridDim.x) {
       const int tile = unit / m, t = unit % m;
@@ -693,6 +700,40 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
         blkseq += (uint32_t)(q1 - q0 + 1);
       }
       if (*abort) break;
+      // the mean: the builders' partials of this row, one per column group,
+      // added in order with error-free sums; its terms reach hundreds of times
+      // the result when K is ill-conditioned, and their magnitudes
+      // sum_j K*_j |alpha_j| decide whether the row is recomputed in fp64
+      if (!wait_or_abort(mean_ready, nmean & 1u, abort)) break;
+      ++nmean;
+      float mhi = 0.f, mlo = 0.f, mag = 0.f;
+#pragma unroll
+      for (int q = 0; q < GPR; ++q) {
+        const float *rp = red + ((size_t)q * BOUTE_TILE_M + 32 * eq + lane) * 3;
+        float e;
+        two_sum_f(mhi, rp[0], mhi, e);
+        mlo += rp[1] + e;
+        mag += rp[2];
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive_count(mean_empty);
+      float mean = ldexpf(mhi + mlo, -er);
+      if (KERN == 0) {  // ill-conditioned rows: the mean in fp64, one row at a time
+        const float sc = ldexpf(sqrtf(par[kParS2]), er);  // the mean's scale, scaled like K*
+        const bool fix = live && mag > kFixRatio * fmaxf(fabsf(mhi), sc);
+        unsigned todo = __ballot_sync(0xffffffffu, fix);
+        while (todo) {
+          const int src = __ffs(todo) - 1;
+          todo &= todo - 1;
+          const long long rr = (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M + 32 * eq + src;
+          const float *x0 = a.xt + (size_t)(b * m + t) * pl.nxt * cf;
+          const double v = mean_fp64_warp<DP>(a.Xc + ((long long)b * a.N + rr) * d, d, x0, cf, n,
+                                              lane);
+          if (lane == src) mean = (float)v;
+        }
+      }
+      if (live && BOUTE_INB(((long long)b * m + t) * a.N + row, (long long)a.B * m * a.N))
+        a.mean[((size_t)b * m + t) * a.N + row] = mean;
       if (live) {
         // V carries the scales 2^e_r (K*) and 2^e_W (W); H^T k* 2^e_r and 2^e_H
         float vv = prior - ldexpf(ss, -2 * (er + (int)par[kParEW]));
@@ -704,12 +745,18 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   } else if (warp >= kBldWarp0) {
     // ---------------------------------------------------------------- K* builders
     // thread -> (row r, column group g): COLS consecutive columns of each half
+    // 8 builder warps: lane = row within the warp's 32-row quarter of the tile,
+    // warp = (quarter, column group), so that the whole warp reads the same
+    // training points (broadcast); 16: RPW rows x GPR column groups per warp
+    // (measured faster there)
     const int bw = warp - kBldWarp0;
-    const int r = bw * RPW + lane % RPW, g = lane / RPW;
+    const int r = kBldWarps == 8 ? 32 * (bw & 3) + lane : bw * RPW + lane % RPW;
+    const int g = kBldWarps == 8 ? bw >> 2 : lane / RPW;
+    uint32_t nmean = 0;
     RingPos pa, px;
     uint32_t qa = 0;
     for (int unit = blockIdx.x; unit < units && !*abort; unit += gridDim.x) {
-      const int tile = unit / m, t = unit % m;
+      const int tile = unit / m;
       const int b = tile / a.tiles_per_problem;
       const long long row = (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M + r;
       float xr[DP];
@@ -727,7 +774,6 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       // magnitudes sum_j K*_j |alpha_j| decide whether the row needs the fp64 path
       Kahan2 mu2;
       unsigned long long mag2 = 0ull;
-      float sc = 0.f;  // the mean's scale sqrt(s2), scaled like K*
       for (int gi = 0; gi < grp.n && !*abort; ++gi) {
         const int kcg = pl.kc[Groups::last(pl, gi)], kcp = Groups::prev(pl, gi);
         // with the cache every built chunk is new and adds to the mean;
@@ -752,7 +798,6 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
               if (KERN == 1) ci = chunk_comp(xth, DP);
               const float ws = KERN == 1 ? cand_weight<DP>(xr, chunk_pref(xth, DP)) : 0.f;
               er = row_exp(KERN, par, ws);
-              sc = ldexpf(sqrtf(par[kParS2]), er);
               if (!PRE) {
                 scaled_candidate<DP>(xr, il, xs2);
                 s2 = ldexpf(par[kParS2], er);
@@ -823,8 +868,8 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
         }
       }
       if (*abort) break;
-      // the thread's sum as a float pair (hi, lo), then the GPR column groups
-      // of the row added with error-free sums
+      // the thread's sum as a float pair (hi, lo) and its magnitude sum, for
+      // the epilogue (the buffer is free once it has read the previous unit's)
       float se, so, ce, co, hi, lo;
       f2_split(mu2.s, se, so);
       f2_split(mu2.c, ce, co);
@@ -832,34 +877,14 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       lo -= ce + co;
       float me, mo;
       f2_split(mag2, me, mo);
-      float mag = me + mo;
-#pragma unroll
-      for (int o = RPW; o < 32; o <<= 1) {
-        const float oh = __shfl_xor_sync(0xffffffffu, hi, o);
-        const float ol = __shfl_xor_sync(0xffffffffu, lo, o);
-        float e;
-        two_sum_f(hi, oh, hi, e);
-        lo += ol + e;
-        mag += __shfl_xor_sync(0xffffffffu, mag, o);
-      }
-      float mean = ldexpf(hi + lo, -er);
-      if (KERN == 0) {  // ill-conditioned rows: the mean in fp64, one row at a time
-        const bool fix = g == 0 && row < a.N && mag > kFixRatio * fmaxf(fabsf(hi), sc);
-        unsigned todo = __ballot_sync(0xffffffffu, fix);
-        while (todo) {
-          const int src = __ffs(todo) - 1;
-          todo &= todo - 1;
-          const long long rr = (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M +
-                               bw * RPW + src % RPW;
-          const float *x0 = a.xt + (size_t)(b * m + t) * pl.nxt * xt_chunk_floats(DP);
-          const double v = mean_fp64_warp<DP>(a.Xc + ((long long)b * a.N + rr) * d, d, x0,
-                                              xt_chunk_floats(DP), n, lane);
-          if (lane == src) mean = (float)v;
-        }
-      }
-      if (g == 0 && row < a.N &&
-          BOUTE_INB(((long long)b * m + t) * a.N + row, (long long)a.B * m * a.N))
-        a.mean[((size_t)b * m + t) * a.N + row] = mean;
+      if (nmean > 0 && !wait_or_abort(mean_empty, (nmean - 1) & 1u, abort)) break;
+      ++nmean;
+      float *rp = red + ((size_t)g * BOUTE_TILE_M + r) * 3;
+      rp[0] = hi;
+      rp[1] = lo;
+      rp[2] = me + mo;
+      __syncwarp();
+      if (lane == 0) mbar_arrive_count(mean_ready);
     }
   }
 
@@ -911,7 +936,8 @@ int launch_dp(const Gp *gp, const float *Xc, const float *kst, long long N, floa
   for (int q = 0; q < a.plan.nblk; ++q) wmax = std::max(wmax, a.plan.ncol[q]);
   a.b_bytes = (uint32_t)(2 * wmax * 128);
   a.x_bytes = (uint32_t)round_up(xt_chunk_floats(DP) * 4, 16);
-  const size_t fixed = 1024 + 512;  // alignment slack, barriers, TMEM address, flag
+  // alignment slack, barriers, TMEM address, flag; the partial means
+  const size_t fixed = 1024 + 512 + (size_t)(32 / Layout<DP>::kCols) * BOUTE_TILE_M * 3 * 4;
   const size_t budget = 227 * 1024 - fixed;
   const size_t st = kst ? kStageBytes : 0;  // staging beside each A stage (PRE)
   // K* stages before B stages: a deeper A ring lets the builders run ahead of
