@@ -46,8 +46,8 @@ namespace {
 
 constexpr int kEpiWarp0 = 2;  // warps 2-5: epilogue (variance, mean), TMEM lane quarter = warp % 4
 constexpr int kEpiWarps = 4;
-constexpr int kXtWarp = 6;    // warp 6: side-input producer
-constexpr int kBldWarp0 = 7;  // warps 7..: K* builders
+constexpr int kXtWarp = 6;     // warp 6: side-input producer
+constexpr int kCacheWarp = 7;  // warp 7 (8 builder warps): cached K* chunks into their A stages
 constexpr int kMaxA = 4, kMaxB = 6, kMaxX = 8;  // ring depths
 constexpr int kSlots = 4;                       // TMEM accumulator slots of 128 columns
 constexpr int kGroup = 4;                       // blocks sharing one K* chunk
@@ -60,6 +60,11 @@ constexpr uint32_t kStageBytes = BOUTE_TILE_M * BOUTE_ACHUNK * 4;   // fp32 K* i
 template <int DP>
 struct Layout {
   static constexpr int kBld = DP <= 16 ? 16 : 8;
+  // with 8 builder warps the cached K* chunks have a warp of their own (warp
+  // 7); with 16 the side-input producer brings them (a 25th warp would cost
+  // the builders registers), and the builders start at warp 7
+  static constexpr bool kSepCache = kBld == 8;
+  static constexpr int kBldWarp0 = kSepCache ? 8 : 7;
   static constexpr int kThreads = 32 * (kBldWarp0 + kBld);
   static constexpr int kCols = 128 / kBld;  // columns of a 32-point half per builder thread
 };
@@ -465,15 +470,18 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   pdl_wait();  // the fit's outputs (operand images, side input) are complete
   const int units = a.tiles_total * m;
 
-  if (warp == 0 || warp == kXtWarp) {
-    // ------------------------------------------------------ producers (B / side input)
-    if (lane == 0) {
+  constexpr bool kSep = Layout<DP>::kSepCache;
+  constexpr int kBldWarp0 = Layout<DP>::kBldWarp0;
+  if (warp == 0 || warp == kXtWarp || (kSep && warp == kCacheWarp)) {
+    // ------------------------------------ producers (B / side input / cached K* chunks)
+    // With a warp of their own for the cached chunks, waiting for the A stage
+    // of a cached chunk never holds up the side input of the new ones.
+    if (lane == 0 && (warp != kCacheWarp || a.ncache > 0)) {
       const bool is_b = warp == 0;
       const int R = is_b ? SB : SX;
       uint64_t *full = is_b ? b_full : x_full, *empty = is_b ? b_empty : x_empty;
-      const bool with_st = PRE && !is_b;  // the side-input producer also stages K*
-      // ... and brings cached K* chunks into their A stages
-      const bool with_cache = !is_b && a.ncache > 0;
+      const bool with_st = PRE && warp == kXtWarp;  // the side-input producer also stages K*
+      const bool with_cache = a.ncache > 0 && warp == (kSep ? kCacheWarp : kXtWarp);
       uint32_t q = 0, qa = 0, nready = 0;
       RingPos rp, ra;
       int last_q = -1, last_qa = -1;  // last jobs issued
@@ -492,10 +500,10 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
           const bool mix = a.ncache > 0 && kcp > 0;
           for (int i = 0; i < kcg && !*abort; ++i) {
             const int c = Groups::chunk_at(i, kcp, kcg, mix);
-            if (with_cache) {
+            if (with_cache) {  // the A ring's positions; the cached chunks' A stages
               const int s = ra.idx;
               const bool cached = c < kcp;
-              if (cached) {  // the A stage from this CTA's cache, no side input
+              if (cached) {  // the A stage from this CTA's cache
                 if (qa >= (uint32_t)SA && !wait_or_abort(&a_empty[s], ra.phase ^ 1u, abort)) break;
                 mbar_expect_tx(&a_full[s], kABytes);
                 if (BOUTE_INB(blockIdx.x * a.ncache + c, (long long)gridDim.x * a.ncache))
@@ -507,8 +515,9 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
               }
               ++qa;
               ra.advance(SA);
-              if (cached) continue;
+              if (cached || kSep) continue;  // (the cache warp does nothing else)
             }
+            if (!is_b && mix && c < kcp) continue;  // a cached chunk needs no side input
             if (with_st) {  // the chunk's fp32 K* image
               const int s = ra.idx;
               if (qa >= (uint32_t)SA && !wait_or_abort(&st_empty[s], ra.phase ^ 1u, abort)) break;
