@@ -70,6 +70,9 @@ struct boute_gp {
   Gp g;
 };
 
+// copy streams of a host-input step (the normals are split over all of them)
+constexpr int kCopyStreams = 2;
+
 struct boute_engine {
   int B, n, d, m, mode, S, k;
   int ncap;  // the buffers hold up to ncap observations (boute_engine_set_n)
@@ -109,18 +112,19 @@ struct boute_engine {
   // (ev_setup) and joined back into the step's stream, beside the GP fit
   cudaStream_t side;
   cudaEvent_t join;
-  // host-input steps: candidates and base normals are copied on two copy
-  // streams while the fit runs; the step waits for them only where it needs
-  // them (posterior, acquisition)
-  cudaStream_t cpy[2];
-  cudaEvent_t ev_in, ev_xc, ev_eps[2];
+  // host-input steps: candidates and base normals are copied on kCopyStreams
+  // copy streams while the fit runs (the normals split evenly over them, so
+  // that several copy engines carry them); the step waits for them only where
+  // it needs them (posterior, acquisition)
+  cudaStream_t cpy[kCopyStreams];
+  cudaEvent_t ev_in, ev_xc, ev_eps[kCopyStreams];
   // pipelined host-input steps: a second set of device input buffers (the
   // first is X .. eps above, allocated on first use) so that one step's copies
   // overlap the previous step's computation; in_free[s] marks the end of the
   // last step that read set s
   double *X1, *Y1, *ls1, *s21, *noise1, *ref1;
   float *Xc1, *eps1;
-  cudaEvent_t ev_xc1, ev_eps1[2], in_free[2];
+  cudaEvent_t ev_xc1, ev_eps1[kCopyStreams], in_free[2];
   cudaEvent_t ev_small[2];  // the small inputs of set 0 / 1 are in place
   int host_set;
   // constrained acquisition (boute_engine_set_constraints): B x m thresholds,
@@ -546,10 +550,13 @@ void boute_engine_free(boute_engine *e) {
     if (g.exec) cudaGraphExecDestroy(g.exec);
   if (e->join) cudaEventDestroy(e->join);
   if (e->side) cudaStreamDestroy(e->side);
-  for (cudaEvent_t ev : {e->ev_in, e->ev_xc, e->ev_eps[0], e->ev_eps[1], e->ev_setup, e->join2,
-                         e->ev_xc1, e->ev_eps1[0], e->ev_eps1[1], e->in_free[0], e->in_free[1],
-                         e->ev_small[0], e->ev_small[1]})
+  for (cudaEvent_t ev : {e->ev_in, e->ev_xc, e->ev_setup, e->join2, e->ev_xc1, e->in_free[0],
+                         e->in_free[1], e->ev_small[0], e->ev_small[1]})
     if (ev) cudaEventDestroy(ev);
+  for (int i = 0; i < kCopyStreams; ++i) {
+    if (e->ev_eps[i]) cudaEventDestroy(e->ev_eps[i]);
+    if (e->ev_eps1[i]) cudaEventDestroy(e->ev_eps1[i]);
+  }
   if (e->side2) cudaStreamDestroy(e->side2);
   for (cudaStream_t c : e->cpy)
     if (c) cudaStreamDestroy(c);
@@ -648,15 +655,9 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
        cudaEventCreateWithFlags(&e->ev_setup, cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->join2, cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->join, cudaEventDisableTiming) != cudaSuccess ||
-       cudaStreamCreateWithFlags(&e->cpy[0], cudaStreamNonBlocking) != cudaSuccess ||
-       cudaStreamCreateWithFlags(&e->cpy[1], cudaStreamNonBlocking) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->ev_in, cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->ev_xc, cudaEventDisableTiming) != cudaSuccess ||
-       cudaEventCreateWithFlags(&e->ev_eps[0], cudaEventDisableTiming) != cudaSuccess ||
-       cudaEventCreateWithFlags(&e->ev_eps[1], cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->ev_xc1, cudaEventDisableTiming) != cudaSuccess ||
-       cudaEventCreateWithFlags(&e->ev_eps1[0], cudaEventDisableTiming) != cudaSuccess ||
-       cudaEventCreateWithFlags(&e->ev_eps1[1], cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->in_free[0], cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->in_free[1], cudaEventDisableTiming) != cudaSuccess ||
        cudaEventCreateWithFlags(&e->ev_small[0], cudaEventDisableTiming) != cudaSuccess ||
@@ -664,6 +665,13 @@ int boute_engine_create(int B, int n, int d, int m, long long N, int mode, int S
     cudaGetLastError();
     r = BOUTE_ERR_CUDA;
   }
+  for (int i = 0; r == BOUTE_OK && i < kCopyStreams; ++i)
+    if (cudaStreamCreateWithFlags(&e->cpy[i], cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&e->ev_eps[i], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&e->ev_eps1[i], cudaEventDisableTiming) != cudaSuccess) {
+      cudaGetLastError();
+      r = BOUTE_ERR_CUDA;
+    }
   if (r != BOUTE_OK) {
     boute_engine_free(e);
     return BOUTE_ERR_OOM;
@@ -753,7 +761,7 @@ static int engine_run(boute_engine *e, const double *X, const double *Y, const d
   if (!serial && cudaStreamWaitEvent(s, e->join, 0) != cudaSuccess)  // join
     return last_launch_status();
   if (host && mc && eps != e->gen_eps)  // (the engine's own normals are resident)
-    for (int i = 0; i < 2; ++i)
+    for (int i = 0; i < kCopyStreams; ++i)
       if (cudaStreamWaitEvent(s, ev_eps[i], wait_flags) != cudaSuccess)
         return last_launch_status();
   if (!live) mark(ST_ACQ);
@@ -912,10 +920,9 @@ static int engine_host_step(boute_engine *e, int set, const double *X, const dou
   cudaEventRecord(e->ev_small[set], c0);
   cudaMemcpyAsync(dXc, Xc, B * N * d * sizeof(float), cudaMemcpyHostToDevice, c0);
   cudaEventRecord(ev_xc, e->cpy[0]);
-  const size_t eps_n = e->mode != BOUTE_ACQ_EHVI2D && eps ? B * N * m * S : 0,
-               half = eps_n / 2;
-  for (int i = 0; eps && i < 2; ++i) {  // the normals in two halves, one per copy stream
-    const size_t off = i ? half : 0, cnt = i ? eps_n - half : half;
+  const size_t eps_n = e->mode != BOUTE_ACQ_EHVI2D && eps ? B * N * m * S : 0;
+  for (int i = 0; eps && i < kCopyStreams; ++i) {  // the normals in equal parts, one per stream
+    const size_t off = eps_n * i / kCopyStreams, cnt = eps_n * (i + 1) / kCopyStreams - off;
     if (cnt)
       cudaMemcpyAsync(deps + off, eps + off, cnt * sizeof(float), cudaMemcpyHostToDevice,
                       e->cpy[i]);
