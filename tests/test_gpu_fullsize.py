@@ -58,16 +58,20 @@ def test_full_size_workload(wi):
     assert torch.all((acq >= kth).sum(1) >= w.k)
     problems = [0] if w.B == 1 else [0, w.B // 2, w.B - 1]
     A, M, V, I = acq.cpu().numpy(), mean.cpu().numpy(), var.cpu().numpy(), idx.cpu().numpy()
+    errs = {"mean": 0.0, "var": 0.0, "acq": 0.0}
     for b in problems:
         fp = oracle_fit(hp, b)
         sel = sample_indices(w.N, I[b], seed=b)
         mo, vo = opl.posterior(fp, hp.Xc[b][sel])
         for tt in range(w.m):
-            check_mean(M[b, tt, sel], mo[:, tt], fp.s2[tt])
-            check_var(V[b, tt, sel], vo[:, tt], fp.s2[tt])
+            errs["mean"] = max(errs["mean"], check_mean(M[b, tt, sel], mo[:, tt], fp.s2[tt]))
+            errs["var"] = max(errs["var"], check_var(V[b, tt, sel], vo[:, tt], fp.s2[tt]))
         ao = opl.acquisition(fp, mo, vo, w.mode, None if hp.eps is None else hp.eps[b][sel])
-        check_acq(A[b, sel], ao)
+        errs["acq"] = max(errs["acq"], check_acq(A[b, sel], ao))
         check_topk_against_oracle(hp, fp, w, b, A[b], I[b])
+    # the measured errors (pytest -s shows them): mean relative to max(|mu|, s),
+    # variance relative to s2, acquisition relative to max(|a|, 1e-3 max|a|)
+    print(f"\n{w.name}: max err mean {errs['mean']:.2e} var {errs['var']:.2e} acq {errs['acq']:.2e}")
 
 
 BAND = 4      # candidates within BAND tolerances below the GPU's k-th compete
