@@ -398,7 +398,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   constexpr int kBldWarps = Layout<DP>::kBld;
   constexpr int COLS = Layout<DP>::kCols;   // columns of a half per builder thread
   constexpr int GPR = 32 / COLS;            // column groups per row
-  constexpr int RPW = 32 / GPR;             // rows per builder warp (16 builder warps)
+  constexpr int RPW = 32 / GPR;             // rows per builder warp
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-byte alignment (the 128-byte swizzle atom) as an offset from the
   // shared array, so that every access below stays a shared-memory access
@@ -754,13 +754,11 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
   } else if (warp >= kBldWarp0) {
     // ---------------------------------------------------------------- K* builders
     // thread -> (row r, column group g): COLS consecutive columns of each half
-    // 8 builder warps: lane = row within the warp's 32-row quarter of the tile,
-    // warp = (quarter, column group), so that the whole warp reads the same
-    // training points (broadcast); 16: RPW rows x GPR column groups per warp
-    // (measured faster there)
+    // RPW rows x GPR column groups per warp (a layout with 32 rows of one
+    // column group per warp, whose coordinate loads are broadcasts, measured
+    // slower: those loads cost more shared-memory wavefronts, not fewer)
     const int bw = warp - kBldWarp0;
-    const int r = kBldWarps == 8 ? 32 * (bw & 3) + lane : bw * RPW + lane % RPW;
-    const int g = kBldWarps == 8 ? bw >> 2 : lane / RPW;
+    const int r = bw * RPW + lane % RPW, g = lane / RPW;
     uint32_t nmean = 0;
     RingPos pa, px;
     uint32_t qa = 0;
