@@ -275,6 +275,55 @@ __device__ __forceinline__ void scaled_candidate(const float (&xr)[DP], const fl
   for (int k = 0; k < DP; ++k) xs2[k] = f2_dup(fmaf(xr[k], il[k], xr[k] * il[DP + k]));
 }
 
+// Two candidates' scaled coordinates as (row 0, row 1) pairs.
+template <int DP>
+__device__ __forceinline__ void scaled_pair(const float (&x0)[DP], const float (&x1)[DP],
+                                            const float *il, unsigned long long (&xs2)[DP]) {
+#pragma unroll
+  for (int k = 0; k < DP; ++k)
+    xs2[k] = f2_pack(fmaf(x0[k], il[k], x0[k] * il[DP + k]), fmaf(x1[k], il[k], x1[k] * il[DP + k]));
+}
+
+// kstar_cols for a pair of candidate rows (Matern-5/2): C columns of a 32-point
+// chunk, each value a (row 0, row 1) pair; every training coordinate is loaded
+// once for the two rows and duplicated in registers. Per entry the same
+// operations in the same order as kstar_cols, so the values are identical.
+template <int DP, int C>
+__device__ __forceinline__ void kstar_pair(const unsigned long long (&xs2)[DP], const float *xth,
+                                           int g, float s2, unsigned long long (&kv)[C]) {
+  unsigned long long acc[C];
+#pragma unroll
+  for (int e = 0; e < C; ++e) acc[e] = 0ull;
+#pragma unroll
+  for (int k = 0; k < DP; ++k) {
+    const float4 *h4 = (const float4 *)(xth + k * BOUTE_KCHUNK + C * g);
+    float h[C];
+#pragma unroll
+    for (int e = 0; e < C / 4; ++e) {
+      const float4 v = h4[e];
+      h[4 * e] = v.x;
+      h[4 * e + 1] = v.y;
+      h[4 * e + 2] = v.z;
+      h[4 * e + 3] = v.w;
+    }
+#pragma unroll
+    for (int e = 0; e < C; ++e) {
+      const unsigned long long df = f2_sub(xs2[k], f2_dup(h[e]));
+      acc[e] = f2_fma(df, df, acc[e]);
+    }
+  }
+  const unsigned long long c0 = f2_dup(s2), c1 = f2_dup(s2 * kLn2), c2 = f2_dup(s2 * kLn2Sq3);
+#pragma unroll
+  for (int e = 0; e < C; ++e) {
+    float ra, rb;
+    f2_split(acc[e], ra, rb);
+    const float r0 = sqrt_approx(ra), r1 = sqrt_approx(rb);
+    const unsigned long long ex = f2_pack(ex2_approx(-r0), ex2_approx(-r1));
+    const unsigned long long t = f2_fma(acc[e], c2, f2_fma(f2_pack(r0, r1), c1, c0));
+    kv[e] = f2_mul(t, ex);
+  }
+}
+
 
 // The exponent e_r of a candidate row's K* scale (kstar_scale_exp of the
 // row's bound on K*): the outputscale for the Matern-5/2 kernel; for the
@@ -397,8 +446,14 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
     posterior_kernel(const __grid_constant__ PostArgs a) {
   constexpr int kBldWarps = Layout<DP>::kBld;
   constexpr int COLS = Layout<DP>::kCols;   // columns of a half per builder thread
-  constexpr int GPR = 32 / COLS;            // column groups per row
-  constexpr int RPW = 32 / GPR;             // rows per builder warp
+  // 8 builder warps building the Matern kernel here: each builder thread
+  // covers two candidate rows (kstar_pair), so that every training coordinate
+  // it loads serves two K* entries (half the shared-memory loads per entry)
+  constexpr bool kPair = !PRE && KERN == 0 && kBldWarps == 8;
+  constexpr int RP = kPair ? 2 : 1;  // candidate rows per builder thread
+  constexpr int CT = COLS / RP;      // its columns of a 32-point half
+  constexpr int GPT = 32 / CT;       // column groups (partial means per row)
+  constexpr int RPT = 32 / GPT;      // builder threads of a warp along the rows
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-byte alignment (the 128-byte swizzle atom) as an offset from the
   // shared array, so that every access below stays a shared-memory access
@@ -717,7 +772,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       ++nmean;
       float mhi = 0.f, mlo = 0.f, mag = 0.f;
 #pragma unroll
-      for (int q = 0; q < GPR; ++q) {
+      for (int q = 0; q < GPT; ++q) {
         const float *rp = red + ((size_t)q * BOUTE_TILE_M + 32 * eq + lane) * 3;
         float e;
         two_sum_f(mhi, rp[0], mhi, e);
@@ -758,7 +813,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
     // column group per warp, whose coordinate loads are broadcasts, measured
     // slower: those loads cost more shared-memory wavefronts, not fewer)
     const int bw = warp - kBldWarp0;
-    const int r = bw * RPW + lane % RPW, g = lane / RPW;
+    const int r = bw * (RPT * RP) + lane % RPT, g = lane / RPT;  // rows r (and r + RPT)
     uint32_t nmean = 0;
     RingPos pa, px;
     uint32_t qa = 0;
@@ -766,16 +821,33 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       const int tile = unit / m;
       const int b = tile / a.tiles_per_problem;
       const long long row = (long long)(tile % a.tiles_per_problem) * BOUTE_TILE_M + r;
-      float xr[DP];
-      if (!PRE || KERN == 1) {
-        const float *xrow = a.Xc + ((long long)b * a.N + row) * d;
-#pragma unroll
-        for (int k = 0; k < DP; ++k) xr[k] = (k < d && row < a.N) ? xrow[k] : 0.f;
-      }
+      float xr[DP];  // (unused with rows in pairs)
       unsigned long long xs2[DP];
       float s2 = 0.f;
       CompIn ci{};
       int er = 0;
+      if constexpr (kPair) {
+        // both rows' scaled coordinates now, with the objective's scales read
+        // from the side input in global memory, so that the raw coordinates
+        // die here instead of living through the chunk loop
+        const float *il = a.xt + (size_t)(b * m + unit % m) * pl.nxt * cf + xt_param_offset(DP);
+        er = row_exp(0, il + 2 * DP, 0.f);
+        s2 = ldexpf(il[2 * DP + kParS2], er);
+        float x0[DP], x1[DP];
+        const long long row1 = row + RPT;
+        const float *xrow = a.Xc + ((long long)b * a.N + row) * d;
+        const float *xrow1 = a.Xc + ((long long)b * a.N + row1) * d;
+#pragma unroll
+        for (int k = 0; k < DP; ++k) {
+          x0[k] = (k < d && row < a.N) ? xrow[k] : 0.f;
+          x1[k] = (k < d && row1 < a.N) ? xrow1[k] : 0.f;
+        }
+        scaled_pair<DP>(x0, x1, il, xs2);
+      } else if (!PRE || KERN == 1) {
+        const float *xrow = a.Xc + ((long long)b * a.N + row) * d;
+#pragma unroll
+        for (int k = 0; k < DP; ++k) xr[k] = (k < d && row < a.N) ? xrow[k] : 0.f;
+      }
       // the mean K* alpha: its terms reach hundreds of times the result when K
       // is ill-conditioned, so they are summed with compensation, and their
       // magnitudes sum_j K*_j |alpha_j| decide whether the row needs the fp64 path
@@ -799,7 +871,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
             if (!wait_or_abort(&x_full[j], px.phase, abort)) break;
             const float *xth = xt_reg(j);
             const float *alp = xth + xt_alpha_offset(DP);
-            if (gi == 0 && c == 0 && h == 0) {  // new objective: its parameters came with the chunk
+            if (!kPair && gi == 0 && c == 0 && h == 0) {  // new objective: its parameters came with the chunk
               const float *il = xth + xt_param_offset(DP);
               const float *par = il + 2 * DP;
               if (KERN == 1) ci = chunk_comp(xth, DP);
@@ -815,6 +887,51 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
                 }
               }
             }
+            if constexpr (kPair) {
+              const int col0 = BOUTE_KCHUNK * h + CT * g;  // first column within the chunk
+              unsigned long long kvp[CT];  // (row r, row r + RPT) per column
+              kstar_pair<DP, CT>(xs2, xth, g, s2, kvp);
+              const int jbase = BOUTE_ACHUNK * c + col0;
+              const float *alg = alp + CT * g;
+              // both rows' CT = 8 columns into the A stage as fp16 hi/lo, the
+              // mean's terms summed per row; a ragged last half zeroes the
+              // columns beyond n
+              auto emit2 = [&](auto ragged) {
+                static_assert(CT == 8, "one 16-byte store per row and part");
+                uint32_t hi[2][4], lo[2][4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                  const int kk = 2 * e;
+                  unsigned long long va = kvp[kk], vb = kvp[kk + 1];
+                  if (decltype(ragged)::value) {
+                    va = (jbase + kk < n) ? va : 0ull;
+                    vb = (jbase + kk + 1 < n) ? vb : 0ull;
+                  }
+                  if (mean_grp) {  // (each chunk's terms once)
+                    const float a0 = alg[kk], a1 = alg[kk + 1];
+                    mu2.add(f2_mul(va, f2_dup(a0)));
+                    mu2.add(f2_mul(vb, f2_dup(a1)));
+                    mag2 = f2_fma(va, f2_dup(fabsf(a0)), mag2);  // (K* >= 0)
+                    mag2 = f2_fma(vb, f2_dup(fabsf(a1)), mag2);
+                  }
+                  float a_0, a_1, b_0, b_1;
+                  f2_split(va, a_0, a_1);
+                  f2_split(vb, b_0, b_1);
+                  split_f16x2(a_0, b_0, hi[0][e], lo[0][e]);
+                  split_f16x2(a_1, b_1, hi[1][e], lo[1][e]);
+                }
+#pragma unroll
+                for (int q = 0; q < 2; ++q) {
+                  const int o = sw128_off16(r + q * RPT, col0) * 2;  // bytes
+                  if (BOUTE_INB(o + 15, (long long)kAPartBytes)) {
+                    *(uint4 *)(Ah + o) = make_uint4(hi[q][0], hi[q][1], hi[q][2], hi[q][3]);
+                    *(uint4 *)(Al + o) = make_uint4(lo[q][0], lo[q][1], lo[q][2], lo[q][3]);
+                  }
+                }
+              };
+              if (jbase + CT <= n) emit2(std::false_type{});
+              else emit2(std::true_type{});
+            } else {
             float kv[COLS];
             const int col0 = BOUTE_KCHUNK * h + COLS * g;  // first column within the chunk
             if (PRE) {  // this thread's COLS values, from the staged fp32 image
@@ -862,6 +979,7 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
             };
             if (jbase + COLS <= n) emit(std::false_type{});
             else emit(std::true_type{});
+            }
             __syncwarp();
             if (lane == 0) mbar_arrive_count(&x_empty[j]);
           }
@@ -877,19 +995,29 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
       if (*abort) break;
       // the thread's sum as a float pair (hi, lo) and its magnitude sum, for
       // the epilogue (the buffer is free once it has read the previous unit's)
-      float se, so, ce, co, hi, lo;
+      float se, so, ce, co, me, mo;
       f2_split(mu2.s, se, so);
       f2_split(mu2.c, ce, co);
-      two_sum_f(se, so, hi, lo);
-      lo -= ce + co;
-      float me, mo;
       f2_split(mag2, me, mo);
       if (nmean > 0 && !wait_or_abort(mean_empty, (nmean - 1) & 1u, abort)) break;
       ++nmean;
       float *rp = red + ((size_t)g * BOUTE_TILE_M + r) * 3;
-      rp[0] = hi;
-      rp[1] = lo;
-      rp[2] = me + mo;
+      if constexpr (kPair) {  // the pair's lanes are the two rows, each a Kahan sum s - c
+        float *rq = red + ((size_t)g * BOUTE_TILE_M + r + RPT) * 3;
+        rp[0] = se;
+        rp[1] = -ce;
+        rp[2] = me;
+        rq[0] = so;
+        rq[1] = -co;
+        rq[2] = mo;
+      } else {  // the pair's lanes are two sets of the row's columns
+        float hi, lo;
+        two_sum_f(se, so, hi, lo);
+        lo -= ce + co;
+        rp[0] = hi;
+        rp[1] = lo;
+        rp[2] = me + mo;
+      }
       __syncwarp();
       if (lane == 0) mbar_arrive_count(mean_ready);
     }
@@ -943,8 +1071,11 @@ int launch_dp(const Gp *gp, const float *Xc, const float *kst, long long N, floa
   for (int q = 0; q < a.plan.nblk; ++q) wmax = std::max(wmax, a.plan.ncol[q]);
   a.b_bytes = (uint32_t)(2 * wmax * 128);
   a.x_bytes = (uint32_t)round_up(xt_chunk_floats(DP) * 4, 16);
-  // alignment slack, barriers, TMEM address, flag; the partial means
-  const size_t fixed = 1024 + 512 + (size_t)(32 / Layout<DP>::kCols) * BOUTE_TILE_M * 3 * 4;
+  // alignment slack, barriers, TMEM address, flag; the partial means (twice
+  // the column groups where the builders take rows in pairs)
+  const bool pair = !kst && !gp->kern && Layout<DP>::kBld == 8;
+  const size_t fixed =
+      1024 + 512 + (size_t)(32 / Layout<DP>::kCols) * (pair ? 2 : 1) * BOUTE_TILE_M * 3 * 4;
   const size_t budget = 227 * 1024 - fixed;
   const size_t st = kst ? kStageBytes : 0;  // staging beside each A stage (PRE)
   // K* stages before B stages: a deeper A ring lets the builders run ahead of
