@@ -56,7 +56,8 @@ constexpr uint32_t kABytes = 2 * kAPartBytes;                       // hi and lo
 constexpr uint32_t kStageBytes = BOUTE_TILE_M * BOUTE_ACHUNK * 4;   // fp32 K* image: 32 KB
 
 // builder warps: 16 (8 columns of each 32-point half per thread) when the
-// candidate coordinates are short enough to keep in registers, else 8 (16)
+// candidate coordinates are short enough to keep in registers, else 8 (16
+// columns of one row, or 8 columns of two rows: kstar_pair)
 template <int DP>
 struct Layout {
   static constexpr int kBld = DP <= 16 ? 16 : 8;
@@ -808,10 +809,11 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
     }
   } else if (warp >= kBldWarp0) {
     // ---------------------------------------------------------------- K* builders
-    // thread -> (row r, column group g): COLS consecutive columns of each half
-    // RPW rows x GPR column groups per warp (a layout with 32 rows of one
-    // column group per warp, whose coordinate loads are broadcasts, measured
-    // slower: those loads cost more shared-memory wavefronts, not fewer)
+    // thread -> (row r, and r + RPT with rows in pairs; column group g): CT
+    // consecutive columns of each half, RPT threads x GPT column groups per
+    // warp (a layout with 32 rows of one column group per warp, whose
+    // coordinate loads are broadcasts, measured slower: those loads cost more
+    // shared-memory wavefronts, not fewer)
     const int bw = warp - kBldWarp0;
     const int r = bw * (RPT * RP) + lane % RPT, g = lane / RPT;  // rows r (and r + RPT)
     uint32_t nmean = 0;
@@ -932,53 +934,53 @@ __global__ void __launch_bounds__(Layout<DP>::kThreads, 1)
               if (jbase + CT <= n) emit2(std::false_type{});
               else emit2(std::true_type{});
             } else {
-            float kv[COLS];
-            const int col0 = BOUTE_KCHUNK * h + COLS * g;  // first column within the chunk
-            if (PRE) {  // this thread's COLS values, from the staged fp32 image
+              float kv[COLS];
+              const int col0 = BOUTE_KCHUNK * h + COLS * g;  // first column within the chunk
+              if (PRE) {  // this thread's COLS values, from the staged fp32 image
 #pragma unroll
-              for (int e = 0; e < COLS / 4; ++e) {
-                const float4 v = *(const float4 *)(stage(s) + st_off32(r, col0 + 4 * e));
-                kv[4 * e] = v.x;
-                kv[4 * e + 1] = v.y;
-                kv[4 * e + 2] = v.z;
-                kv[4 * e + 3] = v.w;
-              }
-            } else {
-              kstar_cols<DP, COLS, KERN>(xs2, xth, g, s2, kv, ci);
-            }
-            const int jbase = BOUTE_ACHUNK * c + col0;
-            const float *alg = alp + COLS * g;
-            // kernel values of this thread's COLS columns into the A stage as
-            // fp16 hi/lo; a ragged last half zeroes the columns beyond n
-            auto emit = [&](auto ragged) {
-#pragma unroll
-              for (int u = 0; u < COLS / 8; ++u) {
-                uint32_t hi[4], lo[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                  const int kk = 8 * u + 2 * e;
-                  float v0 = kv[kk], v1 = kv[kk + 1];
-                  if (decltype(ragged)::value) {
-                    v0 = (jbase + kk < n) ? v0 : 0.f;
-                    v1 = (jbase + kk + 1 < n) ? v1 : 0.f;
-                  }
-                  if (mean_grp) {  // (each chunk's terms once)
-                    const unsigned long long v2 = f2_pack(v0, v1);
-                    const unsigned long long a2 = *(const unsigned long long *)(alg + kk);
-                    mu2.add(f2_mul(v2, a2));
-                    mag2 = f2_fma(v2, a2 & 0x7fffffff7fffffffull, mag2);  // (K* >= 0)
-                  }
-                  split_f16x2(v0, v1, hi[e], lo[e]);
+                for (int e = 0; e < COLS / 4; ++e) {
+                  const float4 v = *(const float4 *)(stage(s) + st_off32(r, col0 + 4 * e));
+                  kv[4 * e] = v.x;
+                  kv[4 * e + 1] = v.y;
+                  kv[4 * e + 2] = v.z;
+                  kv[4 * e + 3] = v.w;
                 }
-                const int o = sw128_off16(r, col0 + 8 * u) * 2;  // bytes
-                if (BOUTE_INB(o + 15, (long long)kAPartBytes)) {
-                  *(uint4 *)(Ah + o) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-                  *(uint4 *)(Al + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
-                }
+              } else {
+                kstar_cols<DP, COLS, KERN>(xs2, xth, g, s2, kv, ci);
               }
-            };
-            if (jbase + COLS <= n) emit(std::false_type{});
-            else emit(std::true_type{});
+              const int jbase = BOUTE_ACHUNK * c + col0;
+              const float *alg = alp + COLS * g;
+              // kernel values of this thread's COLS columns into the A stage as
+              // fp16 hi/lo; a ragged last half zeroes the columns beyond n
+              auto emit = [&](auto ragged) {
+#pragma unroll
+                for (int u = 0; u < COLS / 8; ++u) {
+                  uint32_t hi[4], lo[4];
+#pragma unroll
+                  for (int e = 0; e < 4; ++e) {
+                    const int kk = 8 * u + 2 * e;
+                    float v0 = kv[kk], v1 = kv[kk + 1];
+                    if (decltype(ragged)::value) {
+                      v0 = (jbase + kk < n) ? v0 : 0.f;
+                      v1 = (jbase + kk + 1 < n) ? v1 : 0.f;
+                    }
+                    if (mean_grp) {  // (each chunk's terms once)
+                      const unsigned long long v2 = f2_pack(v0, v1);
+                      const unsigned long long a2 = *(const unsigned long long *)(alg + kk);
+                      mu2.add(f2_mul(v2, a2));
+                      mag2 = f2_fma(v2, a2 & 0x7fffffff7fffffffull, mag2);  // (K* >= 0)
+                    }
+                    split_f16x2(v0, v1, hi[e], lo[e]);
+                  }
+                  const int o = sw128_off16(r, col0 + 8 * u) * 2;  // bytes
+                  if (BOUTE_INB(o + 15, (long long)kAPartBytes)) {
+                    *(uint4 *)(Ah + o) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                    *(uint4 *)(Al + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+                  }
+                }
+              };
+              if (jbase + COLS <= n) emit(std::false_type{});
+              else emit(std::true_type{});
             }
             __syncwarp();
             if (lane == 0) mbar_arrive_count(&x_empty[j]);
