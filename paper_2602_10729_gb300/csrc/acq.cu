@@ -533,11 +533,12 @@ namespace {
 
 size_t mchvi2_smem(int box_cap) { return ((size_t)box_cap + 4) * sizeof(float4); }
 
+// The dynamic shared-memory limit is set on every launch: the kernels' static
+// arrays count against the same 48 KB default as the dynamic part.
 template <class Kern>
 void configure_smem(Kern kernel, size_t smem) {
   prefer_shared(kernel);
-  if (smem > 48 * 1024)
-    cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
 }
 
 void mchvi2_configure(int box_cap) {
@@ -612,9 +613,10 @@ void launch_mchvi3(const float *mean, const float *var, int B, long long N, cons
                    const float *upper, const int *K, int box_cap, const float *eps, int S,
                    long long eps_stride, const double *cons, float *acq, cudaStream_t s) {
   const size_t smem = 2 * (size_t)box_cap * 3 * sizeof(float);
-  if (smem > 48 * 1024)
-    cudaFuncSetAttribute(mchvi_kernel<3, CONS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         (int)smem);
+  // (the kernel's 16 KB of static staging counts against the same 48 KB
+  // default, so the dynamic limit is always set)
+  cudaFuncSetAttribute(mchvi_kernel<3, CONS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)smem);
   const unsigned gx = resident_grid_x(mchvi_kernel<3, CONS>, 512, smem, B, N, 16);
   launch_pdl(mchvi_kernel<3, CONS>, dim3(gx, B), dim3(16 * 32), smem, s, mean, var, B, N, lower,
              upper, K, box_cap, eps, S, eps_stride, cons, acq);

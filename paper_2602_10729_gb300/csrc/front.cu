@@ -256,8 +256,7 @@ __global__ void front_fused_kernel(const double *Y, int n, int m, const double *
 int launch_pareto(const double *Ys, int B, int n, int m, const double *ref, unsigned char *mask,
                   double *front, int *P, cudaStream_t s) {
   const size_t smem = (size_t)n * m * sizeof(long long) + 2 * (size_t)n * sizeof(int) + 16;
-  if (smem > 48 * 1024)
-    cudaFuncSetAttribute(pareto_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaFuncSetAttribute(pareto_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   pareto_kernel<<<B, 512, smem, s>>>(Ys, n, m, ref, mask, front, P);
   count_launch();
   return last_launch_status();
@@ -268,8 +267,7 @@ int launch_boxes(const double *front, const int *P, int B, int n, int m, const d
   size_t smem = 0;
   if (m == 3) smem = (size_t)10 * (n + 2) * sizeof(double) + (size_t)(n + 2) * sizeof(int);
   else if (m != 2) return BOUTE_ERR_UNSUPPORTED;
-  if (smem > 48 * 1024)
-    cudaFuncSetAttribute(boxes_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaFuncSetAttribute(boxes_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   boxes_kernel<<<B, 256, smem, s>>>(front, P, n, m, ref, lower, upper, K);
   count_launch();
   return last_launch_status();
@@ -286,9 +284,9 @@ int launch_front_fused(const double *Y, int B, int n, int m, const double *ref, 
                        int *K, int want_boxes, cudaStream_t s) {
   const size_t smem = front_smem_bytes(n, m);
   prefer_shared(front_fused_kernel);
-  if (smem > 48 * 1024)
-    cudaFuncSetAttribute(front_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         (int)smem);
+  // (static arrays count against the same 48 KB default: always set)
+  cudaFuncSetAttribute(front_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)smem);
   front_fused_kernel<<<B, 512, smem, s>>>(Y, n, m, ref, Ys, mask, front, P, lower, upper, K,
                                           want_boxes);
   count_launch();

@@ -1195,9 +1195,10 @@ int launch_kstar_dp(const Gp *gp, const float *Xc, long long N, float *kst, cuda
   const size_t smem = (size_t)gp->plan.nxt * xt_chunk_floats(DP) * sizeof(float);
   auto go = [&](auto kern) {
     prefer_shared(kern);
-    if (smem > 48 * 1024 &&
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-            cudaSuccess)
+    // (set on every launch: the kernel's static array counts against the same
+    // 48 KB default as the dynamic part)
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+        cudaSuccess)
       return last_launch_status();
     kern<<<units, Layout<DP>::kBld * 32, smem, s>>>(Xc, gp->xt, N, gp->d, gp->m, gp->n, tpp,
                                                     gp->plan.nxt, kst);

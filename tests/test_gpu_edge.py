@@ -8,7 +8,7 @@ import pytest
 
 import oracle
 from _pipeline import (HostProblem, check_acq, check_acq_end_to_end, check_mean, check_var,
-                       gpu_pipeline)
+                       gpu_pipeline, host_problem, oracle_fit)
 from oracle import pipeline as opl
 from paper_2602_10729_gb300 import workloads as wl
 
@@ -76,6 +76,49 @@ def test_dimensions(d):
     # the kernel matrix well conditioned (see the ill-conditioned test below)
     n, ls = (6, 0.1) if d == 1 else (40, 0.2 * np.sqrt(d))
     compare(rand_problem(3, n, d, 2, 300, ls=ls))
+
+
+@pytest.mark.parametrize("n,d,m,N,mode,S", [(600, 20, 2, 700, "ehvi", 0),
+                                            (777, 24, 3, 385, "mc", 64),
+                                            (97, 32, 3, 257, "mc", 64)])
+def test_wide_candidates_large_and_ragged(n, d, m, N, mode, S):
+    # d > 16: the builders take candidate rows in pairs; n > 512 adds the
+    # cached K* chunks of a second group; n, N not multiples of the chunk and
+    # the tile; n = 777 with three objectives puts the MC kernel's boxes
+    # (2n + 2) just under 48 KB of dynamic shared memory, beside its static
+    # staging
+    compare(rand_problem(13, n, d, m, N, mode=mode, S=S, ls=0.2 * np.sqrt(d)))
+
+
+@pytest.mark.parametrize("n", [420, 440])
+def test_kstar_side_input_near_48kb(n):
+    # K* beside the fit (the engine, few candidates): the side input of
+    # n = 420 .. 448 points at d = 12 needs just under 48 KB of dynamic shared
+    # memory next to the K* kernel's static array
+    import torch
+
+    from paper_2602_10729_gb300 import boute as bt
+    w = wl.scaled(wl.WORKLOADS[1], N=2048 + 5, B=1, n=n)
+    hp = host_problem(w)
+    dev = torch.device("cuda")
+    t = lambda a, dt: torch.as_tensor(a, dtype=dt, device=dev)
+    e = bt.Engine(1, w.n, w.d, w.m, w.N, bt.BOUTE_ACQ_MC_HVI, w.S, w.k)
+    idx = torch.empty((1, w.k), dtype=torch.int64, device=dev)
+    val = torch.empty((1, w.k), dtype=torch.float32, device=dev)
+    bt.boute_engine_step(e, t(hp.X, torch.float64), t(hp.Y, torch.float64),
+                         t(hp.ls, torch.float64), t(hp.s2, torch.float64),
+                         t(hp.noise, torch.float64), t(hp.ref, torch.float64),
+                         t(hp.Xc, torch.float32), t(hp.eps, torch.float32), idx, val)
+    mean = torch.empty((1, w.m, w.N), dtype=torch.float32, device=dev)
+    var = torch.empty_like(mean)
+    bt.boute_engine_scores(e, None, mean, var)
+    torch.cuda.synchronize()
+    e.free()
+    fp = oracle_fit(hp, 0)
+    mo, vo = opl.posterior(fp, hp.Xc[0])
+    for tt in range(w.m):
+        check_mean(mean[0, tt].cpu().numpy(), mo[:, tt], fp.s2[tt])
+        check_var(var[0, tt].cpu().numpy(), vo[:, tt], fp.s2[tt])
 
 
 def test_ill_conditioned_problem_meets_fp32_error_bound():
